@@ -1,0 +1,130 @@
+"""Plain fp64 CPU oracle for DMS decode (arXiv 2506.05345, Sec. 3.1-3.2).
+
+TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference leg of ``bench.py`` are the only callers.  The product
+library never imports this package, and this package never imports the product.
+
+The arithmetic lives in ``dms_oracle.c`` (plain C, fp64, sequential sums); this
+module compiles it with gcc on first use and wraps it with ctypes.
+
+Functions (all take bf16 data as ``numpy.uint16`` bit patterns):
+  alpha(logit_bits)                      Sec. 3.2 decision, [logit > 0]
+  retained(logits, j, w)                 Sec. 3.1 / Fig. 1b retained positions
+  decode(q, k, v, logits, j, w, scale)   softmax attention over the retained set
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "dms_oracle.c")
+_LIB = os.path.join(_HERE, "libdms_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (no fast-math: sums stay in source order)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(
+            ["gcc", "-O2", "-fno-fast-math", "-ffp-contract=off", "-std=c11",
+             "-shared", "-fPIC", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            u16p = ctypes.POINTER(ctypes.c_uint16)
+            i32p = ctypes.POINTER(ctypes.c_int32)
+            f64p = ctypes.POINTER(ctypes.c_double)
+            lib.dms_oracle_bf16_to_double.argtypes = [ctypes.c_uint16]
+            lib.dms_oracle_bf16_to_double.restype = ctypes.c_double
+            lib.dms_oracle_alpha.argtypes = [ctypes.c_uint16]
+            lib.dms_oracle_alpha.restype = ctypes.c_int
+            lib.dms_oracle_retained.argtypes = [u16p, ctypes.c_int64, ctypes.c_int64,
+                                                ctypes.c_int64, i32p]
+            lib.dms_oracle_retained.restype = ctypes.c_int64
+            lib.dms_oracle_decode.argtypes = [u16p, ctypes.c_int32, ctypes.c_int32, u16p, u16p,
+                                              ctypes.c_int64, u16p, ctypes.c_int64,
+                                              ctypes.c_int64, ctypes.c_int64, ctypes.c_double,
+                                              f64p]
+            lib.dms_oracle_decode.restype = None
+            _lib = lib
+    return _lib
+
+
+def _u16(a) -> np.ndarray:
+    a = np.asarray(a)
+    if a.dtype != np.uint16:
+        raise TypeError("bf16 data must be passed as uint16 bit patterns")
+    return a
+
+
+def _ptr(a: np.ndarray, ctype):
+    return a.ctypes.data_as(ctypes.POINTER(ctype))
+
+
+def bf16_to_double(bits: int) -> float:
+    return _load().dms_oracle_bf16_to_double(int(bits) & 0xFFFF)
+
+
+def alpha(logit_bits: int) -> int:
+    """Sec. 3.2: alpha_bin = round(sigmoid(logit)) read as [logit > 0]."""
+    return int(_load().dms_oracle_alpha(int(logit_bits) & 0xFFFF))
+
+
+def retained(logits, j: int, w: int) -> np.ndarray:
+    """Sorted positions retained by one KV head after appending position j.
+
+    ``logits`` is a 1-D uint16 array (any stride) holding positions 0..j.
+    """
+    lg = _u16(logits)
+    if lg.ndim != 1:
+        raise ValueError("logits must be 1-D")
+    if j >= lg.shape[0]:
+        raise ValueError("j beyond the logits given")
+    stride = lg.strides[0] // 2
+    out = np.empty(max(j + 1, 1), dtype=np.int32)
+    n = _load().dms_oracle_retained(_ptr(lg, ctypes.c_uint16), stride, j, w,
+                                    _ptr(out, ctypes.c_int32))
+    return out[:n].copy()
+
+
+def decode(q, k, v, logits, j: int, w: int, scale: float = 0.0) -> np.ndarray:
+    """Attention of G query heads over the retained set of their KV head at step j.
+
+    q: [G, D] uint16; k, v: [T, D] uint16 (row-strided views allowed, rows 0..j);
+    logits: [T] uint16.  Returns [G, D] float64.
+    """
+    q = np.ascontiguousarray(_u16(q))
+    k = _u16(k)
+    v = _u16(v)
+    lg = _u16(logits)
+    if q.ndim != 2 or k.ndim != 2 or v.ndim != 2 or lg.ndim != 1:
+        raise ValueError("q, k, v must be 2-D and logits 1-D")
+    G, D = q.shape
+    if k.shape[1] != D or v.shape[1] != D:
+        raise ValueError("head_dim mismatch")
+    if k.strides[1] != 2 or v.strides[1] != 2:
+        raise ValueError("k and v rows must be contiguous")
+    if k.strides[0] != v.strides[0]:
+        v = np.ascontiguousarray(v)
+        k = np.ascontiguousarray(k)
+    if j >= k.shape[0] or j >= lg.shape[0]:
+        raise ValueError("j beyond the data given")
+    out = np.zeros((G, D), dtype=np.float64)
+    _load().dms_oracle_decode(_ptr(q, ctypes.c_uint16), G, D, _ptr(k, ctypes.c_uint16),
+                              _ptr(v, ctypes.c_uint16), k.strides[0] // 2,
+                              _ptr(lg, ctypes.c_uint16), lg.strides[0] // 2, j, w,
+                              float(scale), _ptr(out, ctypes.c_double))
+    return out

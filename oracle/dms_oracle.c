@@ -1,0 +1,124 @@
+/*
+ * Plain fp64 CPU oracle for Dynamic Memory Sparsification (DMS) decode.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path may include, link or
+ * call this file: only the test suite, the smoke check and the CPU-baseline /
+ * reference leg of the benchmark use it.  It shares no code, header, table or
+ * helper with the CUDA library; the only thing both sides share is the seeded
+ * input generator (which holds none of the method's arithmetic).
+ *
+ * What it computes (arXiv 2506.05345):
+ *   - Sec. 3.2 (Inference): the binary decision alpha_t = round(sigmoid(logit_t)).
+ *     sigmoid is strictly increasing with sigmoid(0) = 1/2, so alpha_t = 1 exactly
+ *     when logit_t > 0.  The tie logit = 0 (sigmoid = 1/2) is read as "keep";
+ *     NaN compares false and therefore keeps.
+ *   - Sec. 3.1 "Delayed Eviction via Sliding Window" and Fig. 1b: a token flagged
+ *     at step i stays visible while it is inside the window and disappears once it
+ *     leaves it.  Reading used here: key i is visible to the query at step j iff
+ *     i <= j and (alpha_i == 0 or j - i <= w).  With w = 3 this reproduces the
+ *     pattern printed in Fig. 1b (q_4 loses k_0, q_5 loses k_0 and k_1 but still
+ *     sees k_2).
+ *   - Sec. 3.2 / Sec. 4 (GQA): plain softmax attention of each query head over
+ *     the retained set of its KV head, scale 1/sqrt(D) unless given.
+ *
+ * The retained set R_j is built by scanning the decisions directly from the
+ * definition above; there is no ring, slot or page logic here.  All arithmetic
+ * is fp64 with plain sequential sums in index order.  bf16 inputs are widened
+ * exactly (a bf16 value is the upper half of an IEEE binary32).
+ *
+ * Parity pins (tests, no GPU): Fig. 1b pattern, brute-force dense masked
+ * softmax with the training mask M_alpha of Sec. 3.1, dense causal attention
+ * when nothing is evicted, w = 0 with all-evict, the closed-form retained count.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* Exact widening of a bf16 bit pattern to double. */
+double dms_oracle_bf16_to_double(uint16_t bits) {
+  uint32_t u = ((uint32_t)bits) << 16;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return (double)f;
+}
+
+/* Sec. 3.2: alpha_bin = round(sigmoid(logit)) == [logit > 0] (tie keeps). */
+int dms_oracle_alpha(uint16_t logit_bits) {
+  double x = dms_oracle_bf16_to_double(logit_bits);
+  return x > 0.0 ? 1 : 0;
+}
+
+/* Sec. 3.1 delayed eviction: is key i visible to the query at step j? */
+static int visible(const uint16_t* logits, int64_t logit_stride, int64_t i,
+                   int64_t j, int64_t w) {
+  if (i > j) return 0;                 /* causal */
+  if (j - i <= w) return 1;            /* still inside the sliding window */
+  return dms_oracle_alpha(logits[i * logit_stride]) ? 0 : 1;
+}
+
+/*
+ * Retained set R_j of one (layer, sequence, KV head) after the token at
+ * position j has been appended.  logits[i * logit_stride] is the bf16 decision
+ * logit of position i.  Writes the sorted positions to pos_out (may be NULL)
+ * and returns |R_j|.  Returns 0 for j < 0.
+ */
+int64_t dms_oracle_retained(const uint16_t* logits, int64_t logit_stride,
+                            int64_t j, int64_t w, int32_t* pos_out) {
+  int64_t n = 0;
+  for (int64_t i = 0; i <= j; ++i) {
+    if (visible(logits, logit_stride, i, j, w)) {
+      if (pos_out) pos_out[n] = (int32_t)i;
+      ++n;
+    }
+  }
+  return n;
+}
+
+/*
+ * Decode attention for the G query heads sharing one KV head, at step j.
+ *   q:      [G][D] bf16 bits, row stride D
+ *   k, v:   row i at k + i * kv_stride (bf16 bits, D contiguous), i = 0..j
+ *   logits: logits[i * logit_stride], i = 0..j
+ *   scale:  softmax scale (<= 0 means 1/sqrt(D))
+ *   out:    [G][D] fp64
+ * Softmax over R_j of s_i = scale * <q, k_i>; out = sum_i p_i v_i.
+ * An empty retained set (j < 0) yields zeros.
+ */
+void dms_oracle_decode(const uint16_t* q, int32_t G, int32_t D,
+                       const uint16_t* k, const uint16_t* v, int64_t kv_stride,
+                       const uint16_t* logits, int64_t logit_stride, int64_t j,
+                       int64_t w, double scale, double* out) {
+  if (scale <= 0.0) scale = 1.0 / sqrt((double)D);
+  int64_t cap = j + 1 > 0 ? j + 1 : 0;
+  int32_t* pos = (int32_t*)malloc(sizeof(int32_t) * (size_t)(cap > 0 ? cap : 1));
+  double* s = (double*)malloc(sizeof(double) * (size_t)(cap > 0 ? cap : 1));
+  int64_t n = dms_oracle_retained(logits, logit_stride, j, w, pos);
+  for (int32_t g = 0; g < G; ++g) {
+    double* o = out + (int64_t)g * D;
+    for (int32_t d = 0; d < D; ++d) o[d] = 0.0;
+    if (n == 0) continue;
+    const uint16_t* qg = q + (int64_t)g * D;
+    double m = -INFINITY;
+    for (int64_t r = 0; r < n; ++r) {
+      const uint16_t* kr = k + (int64_t)pos[r] * kv_stride;
+      double dot = 0.0;
+      for (int32_t d = 0; d < D; ++d)
+        dot += dms_oracle_bf16_to_double(qg[d]) * dms_oracle_bf16_to_double(kr[d]);
+      s[r] = scale * dot;
+      if (s[r] > m) m = s[r];
+    }
+    double den = 0.0;
+    for (int64_t r = 0; r < n; ++r) {
+      s[r] = exp(s[r] - m);
+      den += s[r];
+    }
+    for (int64_t r = 0; r < n; ++r) {
+      const uint16_t* vr = v + (int64_t)pos[r] * kv_stride;
+      double p = s[r] / den;
+      for (int32_t d = 0; d < D; ++d) o[d] += p * dms_oracle_bf16_to_double(vr[d]);
+    }
+  }
+  free(pos);
+  free(s);
+}

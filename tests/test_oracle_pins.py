@@ -1,0 +1,322 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix (no GPU).
+
+Each test ties the oracle to something other than itself:
+  * Fig. 1b's printed mask pattern (golden fixture),
+  * the training-mask formulation of Sec. 3.1 evaluated as a dense masked softmax
+    by a library routine (torch SDPA, float64) -- a different computation from
+    the oracle's gather over the retained set,
+  * dense causal attention when nothing is evicted (library routine),
+  * the degenerate w = 0 / all-evict case (out = v_j exactly),
+  * the closed-form retained count and its monotonicity,
+  * the sign rule that round(sigmoid(x)) reduces to (Sec. 3.2),
+  * App. H's KV-read coefficient for the byte model.
+A few tests also show that a plausible mistake (an off-by-one window, a wrong
+scale, a transposed operand) is caught by these pins.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _bf16(x) -> np.ndarray:
+    t = torch.as_tensor(np.asarray(x, dtype=np.float32)).to(torch.bfloat16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def _f64(bits: np.ndarray) -> np.ndarray:
+    return torch.from_numpy(bits.view(np.int16).copy()).view(torch.bfloat16).double().numpy()
+
+
+def _rand_case(rng, T, G, D, p):
+    q = _bf16(rng.standard_normal((T, G, D)))
+    k = _bf16(rng.standard_normal((T, D)))
+    v = _bf16(rng.standard_normal((T, D)))
+    lg = _bf16(rng.standard_normal(T) + (math.inf if p >= 1 else (-math.inf if p <= 0 else
+                                                                    _probit(p))))
+    return q, k, v, lg
+
+
+def _probit(p):
+    import statistics
+    return statistics.NormalDist().inv_cdf(p)
+
+
+def _read_fig1b():
+    rows = []
+    with open(os.path.join(GOLDEN, "fig1b_mask.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            rows.append(line.split()[1:])
+    return rows
+
+
+# --------------------------------------------------------------------------- Fig. 1b
+
+
+def test_fig1b_pattern_all_evict():
+    """With every alpha = 1, the retained sets reproduce the printed mask (w = 3)."""
+    rows = _read_fig1b()
+    T = len(rows)
+    lg = _bf16(np.ones(T))  # logit 1 > 0 -> alpha = 1 for every key
+    for j, row in enumerate(rows):
+        R = set(oracle.retained(lg, j, 3).tolist())
+        for i, e in enumerate(row):
+            if e == "-":
+                assert i not in R, (j, i)
+            elif e == "0":
+                assert i in R, (j, i)
+            else:  # "L": log(1 - alpha) with alpha = 1 -> -inf -> masked
+                assert i not in R, (j, i)
+        assert j in R  # diagonal is always 0
+
+
+def test_fig1b_pattern_no_evict():
+    """With every alpha = 0, log(1 - alpha) = 0: nothing outside the causal mask is hidden."""
+    rows = _read_fig1b()
+    lg = _bf16(-np.ones(len(rows)))
+    for j, row in enumerate(rows):
+        R = set(oracle.retained(lg, j, 3).tolist())
+        for i, e in enumerate(row):
+            assert (i in R) == (e != "-"), (j, i)
+
+
+def test_fig1b_rejects_off_by_one_window():
+    """A window one shorter or longer than the figure's does not reproduce it."""
+    rows = _read_fig1b()
+    lg = _bf16(np.ones(len(rows)))
+    for w_bad in (2, 4):
+        mismatch = False
+        for j, row in enumerate(rows):
+            R = set(oracle.retained(lg, j, w_bad).tolist())
+            for i, e in enumerate(row):
+                if (i in R) != (e == "0"):
+                    mismatch = True
+        assert mismatch, w_bad
+
+
+# --------------------------------------------------------------------------- decision rule
+
+
+@pytest.mark.parametrize("bits,expect", [
+    (0x0000, 0),   # +0: sigmoid = 1/2 exactly, the tie keeps
+    (0x8000, 0),   # -0
+    (0x0001, 1),   # smallest positive subnormal
+    (0x8001, 0),   # smallest negative subnormal
+    (0x3F80, 1),   # 1.0
+    (0xBF80, 0),   # -1.0
+    (0x7F80, 1),   # +inf: sigmoid = 1
+    (0xFF80, 0),   # -inf: sigmoid = 0
+    (0x7FC0, 0),   # NaN: compares false, keeps
+    (0xFFC1, 0),   # negative NaN
+    (0x7F7F, 1),   # largest finite
+])
+def test_alpha_sign_rule_edges(bits, expect):
+    assert oracle.alpha(bits) == expect
+
+
+def test_alpha_matches_rounded_sigmoid():
+    """round(sigmoid(x)) computed in float64 agrees wherever float64 resolves sigmoid - 1/2."""
+    rng = np.random.default_rng(0)
+    xs = np.concatenate([rng.standard_normal(4000) * 3, rng.standard_normal(1000) * 1e-6,
+                         np.array([2.0 ** -30, -2.0 ** -30, 40.0, -40.0])])
+    bits = _bf16(xs)
+    for b, x in zip(bits, _f64(bits)):
+        if abs(x) < 2.0 ** -40:
+            continue
+        s = 1.0 / (1.0 + math.exp(-x))
+        assert s != 0.5
+        assert oracle.alpha(int(b)) == (1 if s > 0.5 else 0), x
+
+
+# --------------------------------------------------------------------------- retained counts
+
+
+@pytest.mark.parametrize("w", [0, 1, 3, 16, 255, 256])
+def test_closed_form_count_and_monotone(w):
+    rng = np.random.default_rng(w + 7)
+    T = 700
+    lg = _bf16(rng.standard_normal(T) + 0.7)
+    a = _f64(lg) > 0
+    prev = 0
+    for j in range(T):
+        n = len(oracle.retained(lg, j, w))
+        evicted_left = int(np.sum(a[: max(0, j - w)]))  # positions i <= j - w - 1
+        assert n == (j + 1) - evicted_left
+        assert n >= prev
+        prev = n
+
+
+def test_retained_sorted_and_contains_window():
+    rng = np.random.default_rng(3)
+    T, w = 300, 17
+    lg = _bf16(rng.standard_normal(T) + 1.0)
+    for j in (0, 5, 17, 18, 150, T - 1):
+        R = oracle.retained(lg, j, w)
+        assert np.all(np.diff(R) > 0)
+        assert set(range(max(0, j - w), j + 1)) <= set(R.tolist())
+
+
+def test_expected_count_statistics():
+    """Mean retained count over many heads is within a few sigma of T - p (T - w - 1)."""
+    rng = np.random.default_rng(11)
+    T, w, p, H = 2000, 256, 0.875, 64
+    mu = _probit(p)
+    counts = []
+    for _ in range(H):
+        lg = _bf16(rng.standard_normal(T) + mu)
+        counts.append(len(oracle.retained(lg, T - 1, w)))
+    expect = T - p * (T - w - 1)
+    sigma = math.sqrt((T - w - 1) * p * (1 - p) / H)
+    assert abs(np.mean(counts) - expect) < 5 * sigma
+
+
+# --------------------------------------------------------------------------- attention values
+
+
+def _sdpa_masked(q, k, v, mask_add, scale):
+    """Dense masked softmax via the library routine, float64.
+
+    q: [Tq, D] queries, k, v: [T, D], mask_add: [Tq, T] additive mask -> [Tq, D].
+    """
+    return torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(np.ascontiguousarray(q))[None], torch.from_numpy(k)[None],
+        torch.from_numpy(v)[None], attn_mask=torch.from_numpy(np.ascontiguousarray(mask_add))[None],
+        scale=scale).numpy()[0]
+
+
+def _training_mask(alpha, w):
+    """M_alpha of Sec. 3.1 / Fig. 1b for binary alpha: -inf above the diagonal,
+    0 inside the window, log(1 - alpha_i) outside it."""
+    T = len(alpha)
+    M = np.full((T, T), -np.inf)
+    with np.errstate(divide="ignore"):
+        la = np.log(1.0 - alpha.astype(np.float64))
+    for j in range(T):
+        for i in range(j + 1):
+            M[j, i] = 0.0 if j - i <= w else la[i]
+    return M
+
+
+@pytest.mark.parametrize("T,G,D,w,p,seed", [
+    (40, 4, 16, 3, 0.6, 0), (64, 1, 32, 0, 0.5, 1), (50, 7, 8, 9, 0.875, 2),
+    (33, 5, 128, 4, 0.9, 3), (20, 2, 16, 30, 0.7, 4)])
+def test_brute_force_training_mask(T, G, D, w, p, seed):
+    """Every step's decode equals the dense softmax with the training mask M_alpha."""
+    rng = np.random.default_rng(seed)
+    q, k, v, lg = _rand_case(rng, T, G, D, p)
+    alpha = (_f64(lg) > 0).astype(np.float64)
+    M = _training_mask(alpha, w)
+    scale = 1.0 / math.sqrt(D)
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    # the query at step j is row j of M for each of the G heads
+    ref = np.stack([_sdpa_masked(qd[:, g], kd, vd, M, scale) for g in range(G)],
+                   axis=1)  # [T, G, D]
+    for j in range(T):
+        got = oracle.decode(q[j], k, v, lg, j, w)
+        np.testing.assert_allclose(got, ref[j], rtol=0, atol=1e-12)
+
+
+def test_no_eviction_equals_dense_causal():
+    rng = np.random.default_rng(5)
+    T, G, D, w = 96, 4, 64, 8
+    q, k, v, _ = _rand_case(rng, T, G, D, 0.5)
+    lg = _bf16(-np.abs(rng.standard_normal(T)) - 0.01)  # all logits < 0: nothing evicted
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    for g in range(G):
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(qd[:, g])[None], torch.from_numpy(kd)[None],
+            torch.from_numpy(vd)[None], is_causal=True).numpy()[0]
+        for j in range(T):
+            got = oracle.decode(q[j], k, v, lg, j, w)[g]
+            np.testing.assert_allclose(got, ref[j], rtol=0, atol=1e-12)
+
+
+def test_window_covering_everything_is_dense():
+    rng = np.random.default_rng(6)
+    T, G, D = 70, 2, 32
+    q, k, v, _ = _rand_case(rng, T, G, D, 0.5)
+    lg = _bf16(np.ones(T))  # all evict, but the window covers the whole history
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(qd.transpose(1, 0, 2)), torch.from_numpy(kd)[None].expand(G, T, D),
+        torch.from_numpy(vd)[None].expand(G, T, D), is_causal=True).numpy()
+    for j in range(T):
+        np.testing.assert_allclose(oracle.decode(q[j], k, v, lg, j, T), ref[:, j], rtol=0,
+                                   atol=1e-12)
+
+
+def test_w0_all_evict_keeps_only_current_token():
+    rng = np.random.default_rng(7)
+    T, G, D = 50, 3, 128
+    q, k, v, _ = _rand_case(rng, T, G, D, 0.5)
+    lg = _bf16(np.ones(T))
+    vd = _f64(v)
+    for j in range(T):
+        assert oracle.retained(lg, j, 0).tolist() == [j]
+        out = oracle.decode(q[j], k, v, lg, j, 0)
+        assert np.array_equal(out, np.broadcast_to(vd[j], out.shape))
+
+
+def test_scale_and_gqa_rows():
+    """Explicit scale equals the default 1/sqrt(D); G heads equal G single-head calls."""
+    rng = np.random.default_rng(8)
+    T, G, D, w = 60, 5, 128, 10
+    q, k, v, lg = _rand_case(rng, T, G, D, 0.8)
+    j = T - 1
+    full = oracle.decode(q[j], k, v, lg, j, w)
+    np.testing.assert_array_equal(full, oracle.decode(q[j], k, v, lg, j, w, 1 / math.sqrt(D)))
+    for g in range(G):
+        np.testing.assert_array_equal(full[g], oracle.decode(q[j][g:g + 1], k, v, lg, j, w)[0])
+
+
+def test_empty_history_gives_zeros():
+    q = _bf16(np.ones((2, 8)))
+    k = _bf16(np.ones((1, 8)))
+    out = oracle.decode(q, k, k, _bf16(np.ones(1)), -1, 4)
+    assert np.all(out == 0)
+
+
+def test_pins_catch_planted_mistakes():
+    """A wrong scale or swapped K/V in the oracle's call would fail the brute-force pin."""
+    rng = np.random.default_rng(9)
+    T, G, D, w = 30, 2, 16, 4
+    q, k, v, lg = _rand_case(rng, T, G, D, 0.7)
+    j = T - 1
+    lg[j - w] = _bf16([1.0])[0]  # the token at distance w is flagged: an off-by-one drops it
+    alpha = (_f64(lg) > 0).astype(np.float64)
+    M = _training_mask(alpha, w)
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    ref = np.stack([_sdpa_masked(qd[j:j + 1, g], kd, vd, M[j:j + 1], 1 / math.sqrt(D))[0]
+                    for g in range(G)])
+    good = oracle.decode(q[j], k, v, lg, j, w)
+    np.testing.assert_allclose(good, ref, atol=1e-12, rtol=0)
+    assert not np.allclose(oracle.decode(q[j], k, v, lg, j, w, 2 / math.sqrt(D)), ref, atol=1e-6)
+    assert not np.allclose(oracle.decode(q[j], v, k, lg, j, w), ref, atol=1e-6)
+    assert not np.allclose(oracle.decode(q[j], k, v, lg, j, w - 1), ref, atol=1e-6)
+
+
+# --------------------------------------------------------------------------- App. H byte model
+
+
+def test_appH_kv_read_coefficient():
+    vals = {}
+    with open(os.path.join(GOLDEN, "appH_llama31_8b_reads.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                key, val = line.split()
+                vals[key] = float(val)
+    n, d_kv = int(vals["layers"]), int(vals["d_kv"])
+    kv_heads = d_kv // workloads.HEAD_DIM
+    coef = workloads.kv_bytes_per_token_head() * kv_heads * n  # bytes per (B*L) per step
+    digits = int(vals["printed_digits"])
+    assert float(f"{coef:.{digits - 1}e}") == vals["kv_read_coefficient"]
