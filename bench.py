@@ -1,0 +1,528 @@
+"""DMS decode benchmark on GB300: retained KV tokens read per second.
+
+One step = one decode step of the whole model: for every layer, the fused
+append + delayed eviction of the new token (all sequences, all KV heads) and the
+split-K decode attention over the retained sets (GQA).  The default workload is
+the Qwen-R1-7B shape: 28 layers, 28 query / 4 KV heads, head_dim 128, batch 64,
+context 8192 (prefill 7936, then decode), window 256, P(evict) = 0.75.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Prints one JSON line.  `value` = retained KV tokens read per second over the
+whole step (device-resident inputs, CUDA events, barrier + synchronize around K
+steps, max over ranks).  `e2e` repeats it through the C ABI with the step inputs
+copied from pinned host memory and the outputs copied back inside the timed
+region.  `roofline` reports the decode kernel against the measured HBM copy
+bandwidth.  `cpu_baseline` times the fp64 CPU oracle on a bounded sample.
+Multi-GPU (torchrun): every rank runs an independent replica (weak scaling, no
+collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = "retained KV tokens read/s and decode-attn µs/layer-step; % of GB300 HBM peak"
+UNIT = "tokens/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+DECODE_SRC = os.path.join(ROOT, "paper_2506_05345_gb300", "csrc", "dms_decode.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default=workloads.QWEN7B_B64_8K.name)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--dense", action="store_true", help="no evictions (CR 1) with the same shape")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--ctas-per-sm", type=int, default=0)
+    ap.add_argument("--min-pages", type=int, default=0)
+    return ap.parse_args()
+
+
+def get_workload(args):
+    wl = workloads.WORKLOADS.get(args.workload)
+    if wl is None:
+        for s in workloads.sweep_workloads():
+            if s.name == args.workload:
+                wl = s
+    if wl is None:
+        raise SystemExit(f"unknown workload {args.workload}")
+    if args.dense:
+        import dataclasses
+        wl = dataclasses.replace(wl, p_evict=0.0, ragged_beta=False, name=wl.name + "-dense")
+    return wl
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def decode_source_sha():
+    with open(DECODE_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def traffic_per_launch(units_per_launch):
+    """DRAM bytes per decode launch from the committed ncu summary, scaled to this
+    launch's units; None if there is none or the kernel changed since."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            t = json.load(f)
+    except Exception:
+        return None
+    if t.get("kernel_source_sha") != decode_source_sha():
+        return None
+    per_unit = t["dram_bytes_per_launch"] / t["units_per_launch"]
+    return per_unit * units_per_launch
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "20"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+            return
+        t0 = time.time()
+        while time.time() - t0 < 5.0 and os.path.getsize(self.path) == 0:
+            time.sleep(0.01)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 7:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[3 + i].lower() == "active"})
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() and args.impl == "ours" else "gloo"
+        dist.init_process_group(backend=backend)
+        pg = dist
+    return world, rank, local, pg
+
+
+def barrier(pg, dev=None):
+    if pg is not None:
+        pg.barrier()
+
+
+def max_over_ranks(pg, x, dev):
+    if pg is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(pg, x, dev):
+    if pg is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    pg.all_reduce(t, op=pg.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ============================================================================ ours
+
+
+def run_ours(args, wl, world, rank, local, pg):
+    import torch
+
+    import paper_2506_05345_gb300 as dms
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    B, L, H, G, D = wl.batch, wl.layers, wl.kv_heads, wl.gqa_group, wl.head_dim
+    Hq = H * G
+    K_, W_ = args.steps, args.warmup
+    E_K, E_W = (0, 0) if args.no_e2e else (min(K_, 50), 2)
+    decode_needed = max(wl.decode_steps, W_ + K_ + E_W + E_K)
+    capacity = wl.prefill_tokens + decode_needed
+    seed_tag = f"rank{rank}"
+    cache = dms.DmsCache(layers=L, kv_heads=H, window=wl.window, capacity=capacity, batch=B,
+                         ctas_per_sm=args.ctas_per_sm, min_pages_per_cta=args.min_pages)
+    stream = torch.cuda.current_stream()
+
+    # ---- sampled heads for the parity check and the CPU baseline (layer 0)
+    rng = np.random.default_rng(workloads.stable_seed(wl.name, "sample", rank))
+    n_sample = min(8, B * H)
+    flat = rng.choice(B * H, size=n_sample, replace=False)
+    sample = [(int(x) // H, int(x) % H) for x in flat]
+    hist = {s: {"k": [], "v": [], "l": []} for s in sample}
+
+    # ---- prefill (untimed)
+    t_setup = time.time()
+    for layer in range(L):
+        for i, (n, shared) in enumerate(wl.prefill):
+            if shared:
+                k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}prefill{i}", n, dev, batch=1)
+                k = k.expand(B, -1, -1, -1).contiguous()
+                v = v.expand(B, -1, -1, -1).contiguous()
+                lg = lg.expand(B, -1, -1).contiguous()
+            else:
+                k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}prefill{i}", n, dev)
+            cache.append_and_evict(layer, k, v, lg)
+            if layer == 0 and rank == 0:
+                for (b, h) in sample:
+                    hist[(b, h)]["k"].append(workloads.bf16_bits(k[b, :, h]))
+                    hist[(b, h)]["v"].append(workloads.bf16_bits(v[b, :, h]))
+                    hist[(b, h)]["l"].append(workloads.bf16_bits(lg[b, :, h]))
+            del k, v, lg
+    torch.cuda.synchronize()
+    st0 = cache.stats()
+    if st0["device_error"]:
+        raise RuntimeError(f"device error after prefill: {st0}")
+
+    # ---- step inputs, resident in HBM before the timed region
+    n_dev_steps = W_ + K_
+    ins = []
+    for s in range(n_dev_steps):
+        per = []
+        for layer in range(L):
+            k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}decode{s}", 1, dev)
+            q = workloads.gen_q(wl, layer, f"{seed_tag}decode{s}", dev)
+            per.append((k, v, lg, q))
+        ins.append(per)
+    outs = [torch.empty((B, Hq, D), dtype=torch.bfloat16, device=dev) for _ in range(L)]
+
+    ev_dec = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(L)] for _ in range(K_)]
+    ev_app = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(L)] for _ in range(K_)]
+
+    def do_step(s, timed_idx=None):
+        for layer in range(L):
+            k, v, lg, q = ins[s][layer]
+            if timed_idx is not None:
+                ev_app[timed_idx][layer][0].record(stream)
+            cache.append_and_evict(layer, k, v, lg)
+            if timed_idx is not None:
+                ev_app[timed_idx][layer][1].record(stream)
+                ev_dec[timed_idx][layer][0].record(stream)
+            cache.decode_attention(layer, q, outs[layer], gqa_group=G)
+            if timed_idx is not None:
+                ev_dec[timed_idx][layer][1].record(stream)
+
+    for s in range(W_):
+        do_step(s)
+    torch.cuda.synchronize()
+    st_before = cache.stats()
+    clocks = Clocks(local)
+    if rank == 0:
+        clocks.start()
+    barrier(pg)
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(K_):
+        do_step(W_ + i, timed_idx=i)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier(pg)
+    clk = clocks.stop() if rank == 0 else None
+    elapsed_ms = t_start.elapsed_time(t_end)
+    st_after = cache.stats()
+    if st_after["device_error"]:
+        raise RuntimeError(f"device error during timed steps: {st_after}")
+    # tokens read per step: every head reads n_h after its append; n_h grows by 0 or 1
+    # per step, so the per-step total is interpolated between the two snapshots
+    # (the error is below the growth over the run, < 0.2 % here).
+    tok_first = st_before["total_retained"]
+    tok_last = st_after["total_retained"]
+    tokens_read = K_ * 0.5 * (tok_first + tok_last)
+    dec_ms = [ev_dec[i][layer][0].elapsed_time(ev_dec[i][layer][1])
+              for i in range(K_) for layer in range(L)]
+    app_ms = [ev_app[i][layer][0].elapsed_time(ev_app[i][layer][1])
+              for i in range(K_) for layer in range(L)]
+    units_per_launch = 0.5 * (tok_first + tok_last) / L
+    bytes_per_unit = workloads.kv_bytes_per_token_head(D)
+    dec_avg_s = float(np.mean(dec_ms)) * 1e-3
+
+    elapsed_max_ms = max_over_ranks(pg, elapsed_ms, dev)
+    tokens_all = sum_over_ranks(pg, tokens_read, dev)
+    value = tokens_all / (elapsed_max_ms * 1e-3)
+
+    # ---- parity sample (layer 0, last timed step) and CPU baseline
+    parity = None
+    cpu_baseline = None
+    if rank == 0:
+        import oracle
+        Gs = G
+        last = W_ + K_ - 1
+        for s in range(W_ + K_):
+            k, v, lg, q = ins[s][0]
+            for (b, h) in sample:
+                hist[(b, h)]["k"].append(workloads.bf16_bits(k[b, :, h]))
+                hist[(b, h)]["v"].append(workloads.bf16_bits(v[b, :, h]))
+                hist[(b, h)]["l"].append(workloads.bf16_bits(lg[b, :, h]))
+        q_last = workloads.bf16_bits(ins[last][0][3])
+        got = outs[0].float().cpu().numpy()
+        j = wl.prefill_tokens + W_ + K_ - 1
+        errs = []
+        cases = []
+        for (b, h) in sample:
+            kk = np.concatenate(hist[(b, h)]["k"])
+            vv = np.concatenate(hist[(b, h)]["v"])
+            ll = np.concatenate(hist[(b, h)]["l"])
+            qq = q_last[b, h * Gs:(h + 1) * Gs]
+            ref = oracle.decode(qq, kk, vv, ll, j, wl.window)
+            errs.append(np.abs(got[b, h * Gs:(h + 1) * Gs] - ref).ravel())
+            cases.append((qq, kk, vv, ll, len(oracle.retained(ll, j, wl.window))))
+        e = np.concatenate(errs)
+        parity = {"sampled_kv_heads": len(sample), "max_abs": float(e.max()),
+                  "mean_abs": float(e.mean()), "ok": bool(e.max() <= 2e-2 and e.mean() <= 2e-3)}
+        # CPU oracle: repeat the sampled heads' decode until the budget is spent
+        tok = 0
+        calls = 0
+        t0 = time.perf_counter()
+        while True:
+            for (qq, kk, vv, ll, n) in cases:
+                oracle.decode(qq, kk, vv, ll, j, wl.window)
+                tok += n
+                calls += 1
+            if time.perf_counter() - t0 >= args.cpu_seconds:
+                break
+        cpu_s = time.perf_counter() - t0
+        cpu_baseline = {"value": tok / cpu_s, "unit": UNIT, "cores": 1, "kind": "oracle",
+                        "sample": f"{calls} fp64 oracle decodes of sampled (layer 0, seq, KV head) "
+                                  f"groups ({G} query heads each) at position {j}, "
+                                  f"{cpu_s:.1f} s single-threaded"}
+
+    # ---- end to end through the C ABI with host buffers
+    e2e = None
+    if E_K > 0:
+        pin = []
+        for s in range(E_W + E_K):
+            per = []
+            for layer in range(L):
+                k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}e2e{s}", 1, dev)
+                q = workloads.gen_q(wl, layer, f"{seed_tag}e2e{s}", dev)
+                per.append(tuple(t.cpu().pin_memory() for t in (k, v, lg, q)))
+            pin.append(per)
+        dk = [torch.empty_like(ins[0][layer][0]) for layer in range(L)]
+        dv = [torch.empty_like(ins[0][layer][1]) for layer in range(L)]
+        dl = [torch.empty_like(ins[0][layer][2]) for layer in range(L)]
+        dq = [torch.empty_like(ins[0][layer][3]) for layer in range(L)]
+        host_out = [torch.empty((B, Hq, D), dtype=torch.bfloat16).pin_memory() for _ in range(L)]
+        h2d = sum(t.numel() * t.element_size() for t in pin[0][0]) * L
+        d2h = sum(t.numel() * t.element_size() for t in host_out)
+
+        def e2e_step(s):
+            for layer in range(L):
+                k, v, lg, q = pin[s][layer]
+                dk[layer].copy_(k, non_blocking=True)
+                dv[layer].copy_(v, non_blocking=True)
+                dl[layer].copy_(lg, non_blocking=True)
+                dq[layer].copy_(q, non_blocking=True)
+                cache.append_and_evict(layer, dk[layer], dv[layer], dl[layer])
+                cache.decode_attention(layer, dq[layer], outs[layer], gqa_group=G)
+                host_out[layer].copy_(outs[layer], non_blocking=True)
+
+        for s in range(E_W):
+            e2e_step(s)
+        torch.cuda.synchronize()
+        sb = cache.stats()
+        barrier(pg)
+        a = torch.cuda.Event(enable_timing=True)
+        z = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for s in range(E_K):
+            e2e_step(E_W + s)
+        z.record(stream)
+        torch.cuda.synchronize()
+        barrier(pg)
+        sa = cache.stats()
+        e_ms = max_over_ranks(pg, a.elapsed_time(z), dev)
+        e_tok = sum_over_ranks(pg, E_K * 0.5 * (sb["total_retained"] + sa["total_retained"]), dev)
+        e2e = {"value": e_tok / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms / E_K, "steps": E_K}
+
+    if rank != 0:
+        cache.close()
+        return None
+
+    peak, peak_kind = measured_peak()
+    achieved_gbs = units_per_launch * bytes_per_unit / dec_avg_s / 1e9
+    traffic = traffic_per_launch(units_per_launch)
+    res = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K_,
+        "warmup": W_, "ms_per_step": elapsed_max_ms / K_, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "impl": "ours",
+        "config": {"workload": wl.name, "batch_per_gpu": B, "layers": L, "q_heads": Hq,
+                   "kv_heads": H, "head_dim": D, "window": wl.window, "prefill": wl.prefill_tokens,
+                   "timed_positions": [wl.prefill_tokens + W_, wl.prefill_tokens + W_ + K_ - 1],
+                   "p_evict": (None if wl.ragged_beta else wl.p_evict),
+                   "ragged_beta": wl.ragged_beta,
+                   "l2": "no flush: per-layer retained KV "
+                         f"{units_per_launch * bytes_per_unit / 1e6:.0f} MB x {L} layers rotate, "
+                         "larger than the 129 MB L2",
+                   "parallelism": f"replicas x{world}"},
+        "decode_us_per_layer_step": float(np.mean(dec_ms)) * 1e3,
+        "append_us_per_layer_step": float(np.mean(app_ms)) * 1e3,
+        "retained_tokens_per_layer_step": units_per_launch,
+        "compression": (wl.prefill_tokens + W_ + K_) * B * H / (units_per_launch),
+        "hbm_frac_of_nominal_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
+        "roofline": {"kernel": "decode_tiled_kernel", "bound": "hbm", "achieved": achieved_gbs,
+                     "peak": peak, "unit": "GB/s", "frac": achieved_gbs / peak,
+                     "peak_kind": f"{peak_kind} copy bandwidth",
+                     "traffic": traffic,
+                     "algorithmic_bytes_per_launch": units_per_launch * bytes_per_unit},
+        "cpu_baseline": cpu_baseline,
+        "e2e": e2e,
+        "gpu_launches": 2 * L * K_,
+        "clocks": clk,
+        "parity_sample": parity,
+        "setup_s": time.time() - t_setup,
+    }
+    cache.close()
+    return res
+
+
+# ============================================================================ reference (oracle)
+
+
+def run_reference(args, wl, world, rank):
+    """The fp64 CPU oracle on the host cores, same workload and metric, bounded sample."""
+    import oracle
+    import torch
+    if rank != 0:
+        return None
+    B, H, G, D = wl.batch, wl.kv_heads, wl.gqa_group, wl.head_dim
+    rng = np.random.default_rng(workloads.stable_seed(wl.name, "refsample"))
+    n_sample = 4
+    flat = rng.choice(B * H, size=n_sample, replace=False)
+    sample = [(int(x) // H, int(x) % H) for x in flat]
+    # history of the sampled heads (layer 0), generated on the CPU with the same recipe
+    sub = workloads.Workload(**{**wl.__dict__, "batch": 1, "name": wl.name})
+    hist = {}
+    for (b, h) in sample:
+        ks, vs, ls = [], [], []
+        for i, (n, _shared) in enumerate(wl.prefill):
+            k, v, lg = workloads.gen_kv(sub, 0, f"ref{b}prefill{i}", n, "cpu")
+            ks.append(workloads.bf16_bits(k[0, :, h]))
+            vs.append(workloads.bf16_bits(v[0, :, h]))
+            ls.append(workloads.bf16_bits(lg[0, :, h]))
+        hist[(b, h)] = [ks, vs, ls]
+    steps = args.warmup + args.steps
+    per_step_s = []
+    per_step_tok = []
+    for s in range(steps):
+        tok = 0
+        t0 = time.perf_counter()
+        for (b, h) in sample:
+            k, v, lg = workloads.gen_kv(sub, 0, f"ref{b}decode{s}", 1, "cpu")
+            q = workloads.gen_q(sub, 0, f"ref{b}decode{s}", "cpu")
+            ks, vs, ls = hist[(b, h)]
+            ks.append(workloads.bf16_bits(k[0, :, h]))
+            vs.append(workloads.bf16_bits(v[0, :, h]))
+            ls.append(workloads.bf16_bits(lg[0, :, h]))
+            kk, vv, ll = np.concatenate(ks), np.concatenate(vs), np.concatenate(ls)
+            j = len(ll) - 1
+            qq = workloads.bf16_bits(q[0, h * G:(h + 1) * G])
+            t1 = time.perf_counter()
+            oracle.decode(qq, kk, vv, ll, j, wl.window)
+            per_step_s.append(time.perf_counter() - t1)
+            tok += len(oracle.retained(ll, j, wl.window))
+        per_step_tok.append(tok)
+    timed_s = sum(per_step_s[args.warmup * n_sample:])
+    timed_tok = sum(per_step_tok[args.warmup:])
+    value = timed_tok / timed_s
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * timed_s / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name, "batch_per_gpu": B, "layers": wl.layers,
+                       "q_heads": wl.q_heads, "kv_heads": H, "head_dim": D, "window": wl.window},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{n_sample} sampled (layer 0, seq, KV head) groups per step, "
+                                       f"{G} query heads each, fp64 single-threaded"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+
+
+def main():
+    args = parse()
+    wl = get_workload(args)
+    world, rank, local, pg = dist_setup(args)
+    if args.impl == "reference":
+        res = run_reference(args, wl, world, rank)
+    else:
+        res = run_ours(args, wl, world, rank, local, pg)
+    if rank == 0 and res is not None:
+        print(json.dumps(res), flush=True)
+    if pg is not None:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

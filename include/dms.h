@@ -1,0 +1,170 @@
+/*
+ * dms.h -- C ABI of libdms: Dynamic Memory Sparsification (DMS) decode on one
+ * NVIDIA GB300 (sm_103a).  arXiv 2506.05345, "Inference-Time Hyper-Scaling with
+ * KV Cache Compression".
+ *
+ * What the library does.  Every (layer, sequence, KV head) keeps its own KV
+ * cache.  Each appended token carries a binary eviction decision alpha, taken
+ * from a bf16 logit as round(sigmoid(logit)) == [logit > 0] (Sec. 3.2; the tie
+ * logit = 0 keeps, NaN keeps).  The eviction is delayed (Sec. 3.1, "Delayed
+ * Eviction via Sliding Window"): a flagged token stays visible while it is within
+ * the window and is dropped when it leaves it.  Precisely, after the token at
+ * position j has been appended, the retained set of a head is
+ *     R_j = { i <= j : alpha_i == 0  or  j - i <= window },
+ * which reproduces the mask of Fig. 1b with window = 3.  The slot of a dropped
+ * token is overwritten by the incoming one (Sec. 3.2: evicted tokens are simply
+ * overwritten; pages belong to individual heads), so each head's retained tokens
+ * occupy slots [0, n_h) of its own page list.  Decode attention is plain softmax
+ * attention of the query heads of a GQA group (Sec. 4) over R_j of their KV head.
+ *
+ * Conventions for every entry point:
+ *   - Data pointers (k, v, decision_logit, q, out) are DEVICE pointers to
+ *     caller-owned, contiguous memory, 16-byte aligned.  bf16 means IEEE
+ *     bfloat16 (the upper half of a binary32).  The caller keeps them alive
+ *     until the work queued on `stream` has completed.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Calls
+ *     are asynchronous unless stated; only dms_cache_stats and
+ *     dms_cache_export_positions wait for the stream.
+ *   - One cache is driven from one stream at a time (calls are not
+ *     thread-safe on the same cache).  All sequences of the batch advance in
+ *     lockstep: every call appends the same number of tokens to every sequence,
+ *     and each layer keeps its own length.
+ *   - Argument errors are detected on the host and return
+ *     DMS_ERR_INVALID_ARGUMENT without queuing any work.  Errors found on the
+ *     device (page pool exhausted, a bounded wait that ran out) set a sticky
+ *     flag in the cache; the call that queued the work still returns DMS_OK and
+ *     dms_cache_stats reports the flag.  No entry point traps or throws.
+ */
+#ifndef DMS_H_
+#define DMS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct dms_cache dms_cache; /* opaque; the library owns all cache memory */
+
+typedef enum dms_status {
+  DMS_OK = 0,
+  DMS_ERR_INVALID_ARGUMENT = 1, /* bad pointer, shape, layer or option        */
+  DMS_ERR_OUT_OF_MEMORY = 2,    /* device allocation failed                   */
+  DMS_ERR_CAPACITY = 3,         /* sequence longer than `capacity`, or the
+                                   page pool ran out (sticky device flag)      */
+  DMS_ERR_CUDA = 4,             /* a CUDA runtime call failed                 */
+  DMS_ERR_TIMEOUT = 5,          /* a bounded in-kernel wait gave up (sticky)  */
+  DMS_ERR_STATE = 6             /* call not valid in the cache's current state */
+} dms_status;
+
+/* Decode kernels selectable through dms_options.decode_kernel. */
+enum {
+  DMS_DECODE_TILED = 0,  /* default: TMA-staged, tensor-core, page-balanced split-K */
+  DMS_DECODE_SIMPLE = 1  /* one CTA per KV head, CUDA cores; a cross-check path     */
+};
+
+typedef struct dms_options {
+  int32_t batch;         /* sequences per layer (required, >= 1)                    */
+  int32_t page_tokens;   /* tokens per page; 0 = 64 (only 64 is accepted)           */
+  int64_t pool_tokens;   /* page pool size in tokens, shared by all layers and
+                            heads; 0 = layers * batch * kv_heads * capacity (the
+                            dense worst case), rounded up to whole pages           */
+  int32_t decode_kernel; /* DMS_DECODE_TILED (0) or DMS_DECODE_SIMPLE (1)           */
+  int32_t ctas_per_sm;   /* split-K CTAs per SM for the tiled kernel; 0 = 1         */
+  int32_t min_pages_per_cta; /* lower bound on pages per split-K CTA; 0 = 2         */
+  int32_t reserved[5];   /* must be zero                                            */
+} dms_options;
+
+typedef struct dms_stats {
+  int64_t total_retained; /* sum over layers, sequences, KV heads of n_h            */
+  int64_t total_appended; /* tokens appended, summed the same way                  */
+  int64_t total_evicted;  /* total_appended - total_retained                       */
+  int64_t pages_in_use;   /* pages handed out from the pool                        */
+  int64_t pool_pages;     /* pages in the pool                                     */
+  int64_t peak_pages;     /* largest pages_in_use seen since creation              */
+  int32_t max_retained;   /* largest n_h over all heads                            */
+  int32_t min_retained;   /* smallest n_h over all heads                           */
+  int32_t device_error;   /* sticky device-side dms_status (DMS_OK if none)        */
+  int32_t reserved;
+} dms_stats;
+
+/*
+ * Create a cache for `layers` layers of `kv_heads` KV heads (head_dim must be
+ * 128), sliding window `window` >= 0 (Sec. 3.1; the paper's default is 256), and
+ * at most `capacity` >= 1 appended tokens per sequence.  `opt` must be non-NULL
+ * with opt->batch >= 1; zeroed fields take their defaults.  Allocates the page
+ * pool, page tables, per-head counts, decision rings and decode scratch, and
+ * zeroes the counts.  On success *out receives the cache; on failure *out is
+ * NULL and nothing stays allocated.  Limits: batch * kv_heads <= 4096,
+ * capacity < 2^31.
+ */
+dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim,
+                            int32_t window, int64_t capacity, const dms_options* opt,
+                            dms_cache** out);
+
+/* Free everything the cache owns (synchronises the device first).  NULL is a no-op. */
+dms_status dms_cache_destroy(dms_cache* cache);
+
+/*
+ * Empty every head of every layer (all n_h = 0, all layer lengths 0, pool
+ * returned, sticky device error cleared).  Queued on `stream`.
+ */
+dms_status dms_cache_reset(dms_cache* cache, void* stream);
+
+/*
+ * Append n_tokens >= 1 tokens to every sequence of `layer` and apply delayed
+ * eviction (Sec. 3.1-3.2).  Positions t0 .. t0 + n_tokens - 1 are appended,
+ * t0 being the layer's current length.
+ *   k, v            [batch, n_tokens, kv_heads, 128] bf16 (keys already carry
+ *                   their positional encoding, Sec. 3.2)
+ *   decision_logit  [batch, n_tokens, kv_heads] bf16; alpha = [logit > 0]
+ * After the call each head holds exactly R_{t0+n_tokens-1}.  A bulk call
+ * (prefill) gives the same retained sets as n_tokens single-token calls.
+ * Returns DMS_ERR_CAPACITY (nothing queued) if the layer would exceed
+ * `capacity`.  Page-pool exhaustion is reported through the sticky flag.
+ */
+dms_status dms_append_and_evict(dms_cache* cache, int32_t layer, const void* k,
+                                const void* v, const void* decision_logit,
+                                int32_t n_tokens, void* stream);
+
+/*
+ * Decode attention for `layer` over the current retained sets (GQA, Sec. 4):
+ *   q    [batch, kv_heads * gqa_group, 128] bf16; query head hq reads KV head
+ *        hq / gqa_group
+ *   out  [batch, kv_heads * gqa_group, 128] bf16 (round to nearest even)
+ * out[b][hq] = sum_{i in R} softmax_i(sm_scale * <q, k_i>) v_i, with fp32
+ * accumulation.  sm_scale <= 0 means 1/sqrt(128).  1 <= gqa_group <= 16.  A
+ * head with no tokens yet (nothing appended) yields zeros.
+ */
+dms_status dms_decode_attention(dms_cache* cache, int32_t layer, const void* q, void* out,
+                                int32_t gqa_group, float sm_scale, void* stream);
+
+/*
+ * Synchronise `stream`, then report totals into *out (non-NULL) and, if
+ * `counts` is non-NULL, copy the per-head retained counts n_h into the HOST
+ * array counts[layers * batch * kv_heads] (layer-major, then sequence, then KV
+ * head).  Returns the sticky device error, if any, as its own status as well.
+ */
+dms_status dms_cache_stats(dms_cache* cache, dms_stats* out, int32_t* counts, void* stream);
+
+/*
+ * Test/inspection helper.  Synchronise `stream` and write, for every
+ * (sequence b, KV head h) of `layer`, the positions held in slots [0, n_h) into
+ * the HOST array host_pos[(b * kv_heads + h) * capacity + slot], in slot order
+ * (not sorted); unused entries are set to -1.
+ */
+dms_status dms_cache_export_positions(dms_cache* cache, int32_t layer, int32_t* host_pos,
+                                      void* stream);
+
+/* Current length (tokens appended per sequence) of `layer`, into *out. */
+dms_status dms_cache_layer_length(const dms_cache* cache, int32_t layer, int64_t* out);
+
+/* Static description of a status code. */
+const char* dms_status_string(dms_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DMS_H_ */

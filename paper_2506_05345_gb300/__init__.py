@@ -1,0 +1,203 @@
+"""DMS decode on one GB300: Python face of libdms (include/dms.h).
+
+Dynamic Memory Sparsification (arXiv 2506.05345) keeps, per (layer, sequence,
+KV head), only the tokens whose eviction decision is 0 plus the last `window`
+ones (delayed eviction, Sec. 3.1); decode attention reads only those.
+
+Two layers of API, both thin:
+  * the C names (``dms_cache_create``, ``dms_append_and_evict``,
+    ``dms_decode_attention``, ``dms_cache_stats``, ...) re-exported from the
+    ctypes binding, taking raw pointers exactly like the C ABI;
+  * ``DmsCache``, which takes torch CUDA tensors, checks their shapes, and
+    passes ``data_ptr()`` and the current stream.
+PyTorch provides device memory and streams only; all computation is in the
+library's CUDA kernels.  Nothing here falls back to a CPU implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+
+from . import _native
+from ._native import (DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
+                      DMS_ERR_INVALID_ARGUMENT, DMS_ERR_TIMEOUT, DMS_OK, DmsLibraryError,
+                      dms_options, dms_stats)
+
+HEAD_DIM = 128
+
+
+class DmsError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        self.code = int(code)
+        try:
+            msg = _native.status_string(code)
+        except DmsLibraryError:
+            msg = f"status {code}"
+        super().__init__(f"{what}: {msg} (status {code})")
+
+
+def _check(code: int, what: str):
+    if code != DMS_OK:
+        raise DmsError(code, what)
+
+
+def library():
+    """The loaded libdms (raises DmsLibraryError if it is not built)."""
+    return _native.load()
+
+
+# ---- C names, same arguments as the header (raw pointers / ints) -------------
+
+def dms_cache_create(layers, kv_heads, head_dim, window, capacity, opt: dms_options):
+    out = ctypes.c_void_p()
+    code = library().dms_cache_create(layers, kv_heads, head_dim, window, capacity,
+                                      ctypes.byref(opt), ctypes.byref(out))
+    return code, out.value
+
+
+def dms_cache_destroy(cache):
+    return library().dms_cache_destroy(cache)
+
+
+def dms_cache_reset(cache, stream):
+    return library().dms_cache_reset(cache, stream)
+
+
+def dms_append_and_evict(cache, layer, k_ptr, v_ptr, logit_ptr, n_tokens, stream):
+    return library().dms_append_and_evict(cache, layer, k_ptr, v_ptr, logit_ptr, n_tokens, stream)
+
+
+def dms_decode_attention(cache, layer, q_ptr, out_ptr, gqa_group, sm_scale, stream):
+    return library().dms_decode_attention(cache, layer, q_ptr, out_ptr, gqa_group,
+                                          float(sm_scale), stream)
+
+
+def dms_cache_stats(cache, stats: dms_stats, counts_ptr, stream):
+    return library().dms_cache_stats(cache, ctypes.byref(stats), counts_ptr, stream)
+
+
+def dms_cache_export_positions(cache, layer, host_pos_ptr, stream):
+    return library().dms_cache_export_positions(cache, layer, host_pos_ptr, stream)
+
+
+def dms_cache_layer_length(cache, layer):
+    out = ctypes.c_int64()
+    code = library().dms_cache_layer_length(cache, layer, ctypes.byref(out))
+    return code, out.value
+
+
+# ---- torch-facing wrapper ---------------------------------------------------
+
+def _stream_ptr(stream=None):
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _bf16_cuda(t, shape, name):
+    import torch
+    if not isinstance(t, torch.Tensor) or not t.is_cuda or t.dtype != torch.bfloat16:
+        raise TypeError(f"{name} must be a CUDA bfloat16 tensor")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class DmsCache:
+    """Per-head sparsified KV cache for `layers` layers of `batch` x `kv_heads` heads."""
+
+    def __init__(self, layers: int, kv_heads: int, window: int, capacity: int, batch: int,
+                 head_dim: int = HEAD_DIM, pool_tokens: int = 0,
+                 decode_kernel: int = DMS_DECODE_TILED, ctas_per_sm: int = 0,
+                 min_pages_per_cta: int = 0):
+        self._h = None
+        opt = dms_options()
+        opt.batch = batch
+        opt.pool_tokens = pool_tokens
+        opt.decode_kernel = decode_kernel
+        opt.ctas_per_sm = ctas_per_sm
+        opt.min_pages_per_cta = min_pages_per_cta
+        code, h = dms_cache_create(layers, kv_heads, head_dim, window, capacity, opt)
+        _check(code, "dms_cache_create")
+        self._h = h
+        self.layers, self.kv_heads, self.window = layers, kv_heads, window
+        self.capacity, self.batch, self.head_dim = capacity, batch, head_dim
+
+    def close(self):
+        if self._h is not None:
+            dms_cache_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    @property
+    def handle(self):
+        return self._h
+
+    def reset(self, stream=None):
+        _check(dms_cache_reset(self._h, _stream_ptr(stream)), "dms_cache_reset")
+
+    def append_and_evict(self, layer: int, k, v, decision_logit, stream=None):
+        """k, v: [batch, n, kv_heads, 128] bf16; decision_logit: [batch, n, kv_heads] bf16."""
+        n = k.shape[1]
+        B, H, D = self.batch, self.kv_heads, self.head_dim
+        kp = _bf16_cuda(k, (B, n, H, D), "k")
+        vp = _bf16_cuda(v, (B, n, H, D), "v")
+        lp = _bf16_cuda(decision_logit, (B, n, H), "decision_logit")
+        _check(dms_append_and_evict(self._h, layer, kp, vp, lp, n, _stream_ptr(stream)),
+               "dms_append_and_evict")
+
+    def decode_attention(self, layer: int, q, out=None, gqa_group: int | None = None,
+                         sm_scale: float = 0.0, stream=None):
+        """q, out: [batch, kv_heads * gqa_group, 128] bf16.  Returns out."""
+        import torch
+        B, H, D = self.batch, self.kv_heads, self.head_dim
+        if gqa_group is None:
+            gqa_group = q.shape[1] // H
+        if out is None:
+            out = torch.empty_like(q)
+        qp = _bf16_cuda(q, (B, H * gqa_group, D), "q")
+        op = _bf16_cuda(out, (B, H * gqa_group, D), "out")
+        _check(dms_decode_attention(self._h, layer, qp, op, gqa_group, sm_scale,
+                                    _stream_ptr(stream)), "dms_decode_attention")
+        return out
+
+    def stats(self, stream=None, with_counts: bool = False):
+        st = dms_stats()
+        counts = None
+        cptr = None
+        if with_counts:
+            counts = np.zeros((self.layers, self.batch, self.kv_heads), dtype=np.int32)
+            cptr = ctypes.c_void_p(counts.ctypes.data)
+        code = dms_cache_stats(self._h, st, cptr, _stream_ptr(stream))
+        d = {f: getattr(st, f) for f, _ in dms_stats._fields_ if f != "reserved"}
+        if code not in (DMS_OK, st.device_error):
+            _check(code, "dms_cache_stats")
+        if with_counts:
+            d["counts"] = counts
+        return d
+
+    def export_positions(self, layer: int, stream=None) -> np.ndarray:
+        """[batch, kv_heads, capacity] int32 positions in slot order, -1 past n_h."""
+        out = np.empty((self.batch, self.kv_heads, self.capacity), dtype=np.int32)
+        _check(dms_cache_export_positions(self._h, layer, ctypes.c_void_p(out.ctypes.data),
+                                          _stream_ptr(stream)), "dms_cache_export_positions")
+        return out
+
+    def layer_length(self, layer: int) -> int:
+        code, n = dms_cache_layer_length(self._h, layer)
+        _check(code, "dms_cache_layer_length")
+        return n

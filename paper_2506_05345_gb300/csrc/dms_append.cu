@@ -1,0 +1,303 @@
+// Fused append + delayed eviction (arXiv 2506.05345, Sec. 3.1 "Delayed Eviction via
+// Sliding Window" and Sec. 3.2 "Inference").
+//
+// State per (layer, sequence, KV head): n_h retained tokens in slots [0, n_h), a
+// page list, and a ring holding (slot, alpha) of the last window+1 positions.
+// Appending position j: the token j - window - 1 leaves the window now; if its
+// decision was alpha = 1 it is dropped and the new token takes over its slot,
+// otherwise the new token gets the fresh slot n_h (Sec. 3.2: evicted tokens are
+// overwritten by incoming ones).  One token enters and at most one leaves, so the
+// slots stay dense and n_h never decreases; pages are only ever added.
+#include "dms_internal.cuh"
+
+namespace dms {
+namespace {
+
+struct AppendParams {
+  uint8_t* pool;
+  int32_t* pos;
+  int32_t* page_table;  // this layer: [heads][max_pages]
+  int32_t* counts;      // this layer: [heads]
+  uint32_t* ring;       // this layer: [heads][ring_len]
+  int32_t* ctrl;
+  int32_t* freed;       // [heads][ring_len]
+  const uint16_t* k;
+  const uint16_t* v;
+  const uint16_t* logit;
+  int64_t t0;           // position of the first appended token
+  int64_t window;
+  int64_t pool_pages;
+  int32_t n;            // tokens appended by this call
+  int32_t heads, kv_heads, max_pages, ring_len;
+};
+
+// Copy one 256-byte K row and one V row into `row` of `page`, applying the chunk
+// permutation of the pool layout.  Lanes 0-15 move K, lanes 16-31 move V.
+__device__ __forceinline__ void store_row(uint8_t* pool, int32_t page, uint32_t row, int lane,
+                                          uint4 val) {
+  const uint32_t chunk = lane & 15;
+  uint8_t* dst = pool + (int64_t)page * kPageBytes + (lane >= 16 ? kHalfPageBytes : 0) +
+                 swizzled_offset(row, chunk);
+  *reinterpret_cast<uint4*>(dst) = val;
+}
+
+__device__ __forceinline__ uint4 load_row_chunk(const uint16_t* k, const uint16_t* v,
+                                                int64_t row_elem, int lane) {
+  const uint16_t* src = (lane >= 16 ? v : k) + row_elem + (lane & 15) * 8;
+  return __ldg(reinterpret_cast<const uint4*>(src));
+}
+
+// n = 1: one warp per head.  Lane 0 runs the ring/slot logic, the warp moves the
+// 512 bytes of K and V.
+__global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int bh = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (bh >= p.heads) return;
+  const int b = bh / p.kv_heads, hk = bh - b * p.kv_heads;
+  const int64_t row_elem = ((int64_t)b * p.kv_heads + hk) * kHeadDim;  // [B,1,Hkv,D]
+  const uint4 val = load_row_chunk(p.k, p.v, row_elem, lane);
+
+  int32_t slot = 0, page = 0, ok = 1;
+  if (lane == 0) {
+    const int64_t j = p.t0;
+    const int64_t R = p.window + 1;
+    const uint32_t alpha = decision_from_bf16(p.logit[(int64_t)b * p.kv_heads + hk]);
+    uint32_t* ring = p.ring + (int64_t)bh * p.ring_len;
+    int32_t* pt = p.page_table + (int64_t)bh * p.max_pages;
+    int32_t n = p.counts[bh];
+    slot = -1;
+    const int32_t ridx = (int32_t)(j % R);
+    if (j >= R) {  // token j - window - 1 leaves the window now
+      const uint32_t e = ring[ridx];
+      if (e & kAlphaBit) slot = (int32_t)(e & kSlotMask);  // evicted: reuse its slot
+    }
+    if (slot < 0) {
+      slot = n;
+      if ((slot & (kPageTokens - 1)) == 0) {
+        const int32_t np = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
+        if ((int64_t)np >= p.pool_pages) {
+          set_device_error(p.ctrl, DMS_ERR_CAPACITY);
+          ok = 0;
+        } else {
+          pt[slot / kPageTokens] = np;
+        }
+      }
+      n += ok;
+    }
+    if (ok) {
+      ring[ridx] = (uint32_t)slot | (alpha << 31);
+      p.counts[bh] = n;
+      page = pt[slot / kPageTokens];
+      p.pos[(int64_t)page * kPageTokens + (slot & (kPageTokens - 1))] = (int32_t)j;
+    }
+  }
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (!ok) return;
+  slot = __shfl_sync(0xffffffffu, slot, 0);
+  page = __shfl_sync(0xffffffffu, page, 0);
+  store_row(p.pool, page, (uint32_t)(slot & (kPageTokens - 1)), lane, val);
+}
+
+constexpr int kBulkThreads = 512;
+constexpr int kBulkWarps = kBulkThreads / 32;
+
+// Block-wide exclusive scan of 0/1 flags; returns the prefix, writes the total.
+__device__ __forceinline__ int block_scan_flags(int flag, int* s_warp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned ballot = __ballot_sync(0xffffffffu, flag);
+  const int in_warp = __popc(ballot & ((1u << lane) - 1u));
+  if (lane == 0) s_warp[warp] = __popc(ballot);
+  __syncthreads();
+  int before = 0, sum = 0;
+  for (int w = 0; w < kBulkWarps; ++w) {
+    const int c = s_warp[w];
+    before += (w < warp) ? c : 0;
+    sum += c;
+  }
+  __syncthreads();
+  *total = sum;
+  return before + in_warp;
+}
+
+// n >= 1 tokens per call (prefill): one CTA per head.  Produces the same retained
+// set as n single-token appends; slots freed by tokens that leave during the call
+// are refilled first (in order), further kept tokens extend [0, n_h).
+__global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendParams p) {
+  __shared__ int s_warp[kBulkWarps];
+  __shared__ int32_t s_slot[kBulkThreads];
+  __shared__ int32_t s_misc[4];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int bh = blockIdx.x;
+  const int b = bh / p.kv_heads, hk = bh - b * p.kv_heads;
+  const int64_t R = p.window + 1, t0 = p.t0, n = p.n;
+  uint32_t* ring = p.ring + (int64_t)bh * p.ring_len;
+  int32_t* F = p.freed + (int64_t)bh * p.ring_len;
+  int32_t* pt = p.page_table + (int64_t)bh * p.max_pages;
+  const int32_t nh = p.counts[bh];
+
+  // 1. Old tokens leaving the window during this call: positions [lo, hi], all < t0.
+  const int64_t lo = t0 - R > 0 ? t0 - R : 0;
+  const int64_t hi = (t0 - 1) < (t0 + n - R - 1) ? (t0 - 1) : (t0 + n - R - 1);
+  const int64_t len_old = hi >= lo ? hi - lo + 1 : 0;
+  int nf = 0;
+  for (int64_t base = 0; base < len_old; base += kBulkThreads) {
+    int flag = 0;
+    uint32_t e = 0;
+    if (base + tid < len_old) {
+      e = ring[(lo + base + tid) % R];
+      flag = (e & kAlphaBit) ? 1 : 0;
+    }
+    int total;
+    const int r = block_scan_flags(flag, s_warp, &total);
+    if (flag) F[nf + r] = (int32_t)(e & kSlotMask);
+    nf += total;
+  }
+
+  // 2. New tokens that also leave within this call (local index < n - R) and are
+  //    flagged are never stored.
+  const int64_t n_leave_new = n - R > 0 ? n - R : 0;
+  int evicted_new = 0;
+  for (int64_t base = 0; base < n_leave_new; base += kBulkThreads) {
+    int flag = 0;
+    if (base + tid < n_leave_new)
+      flag = (int)decision_from_bf16(p.logit[((int64_t)b * n + base + tid) * p.kv_heads + hk]);
+    int total;
+    block_scan_flags(flag, s_warp, &total);
+    evicted_new += total;
+  }
+  const int64_t kept_total = n - evicted_new;
+  const int64_t new_n = nh + kept_total - nf;
+
+  // 3. Pages for the slots [nh, new_n).
+  const int32_t old_pages = (nh + kPageTokens - 1) / kPageTokens;
+  const int32_t new_pages = (int32_t)((new_n + kPageTokens - 1) / kPageTokens);
+  const int32_t add = new_pages - old_pages;
+  if (tid == 0) {
+    int32_t base = 0, ok = 1;
+    if (add > 0) {
+      base = atomicAdd(p.ctrl + kCtrlPoolNext, add);
+      if ((int64_t)base + add > p.pool_pages) {
+        set_device_error(p.ctrl, DMS_ERR_CAPACITY);
+        ok = 0;
+      }
+    }
+    s_misc[0] = base;
+    s_misc[1] = ok;
+  }
+  __syncthreads();
+  if (!s_misc[1]) return;
+  for (int i = tid; i < add; i += kBulkThreads) pt[old_pages + i] = s_misc[0] + i;
+  __syncthreads();
+
+  // 4. Slot assignment, ring update for the final window, row copies.
+  int64_t kept_before = 0;
+  for (int64_t base = 0; base < n; base += kBulkThreads) {
+    const int64_t li = base + tid;
+    const bool valid = li < n;
+    uint32_t alpha = 0;
+    if (valid) alpha = decision_from_bf16(p.logit[((int64_t)b * n + li) * p.kv_heads + hk]);
+    const int kept = (valid && !(alpha && li < n_leave_new)) ? 1 : 0;
+    int total;
+    const int r = block_scan_flags(kept, s_warp, &total);
+    int32_t slot = -1;
+    if (kept) {
+      const int64_t rank = kept_before + r;
+      slot = rank < nf ? F[rank] : (int32_t)(nh + (rank - nf));
+    }
+    s_slot[tid] = slot;
+    if (valid && li >= n - R) ring[(t0 + li) % R] = (uint32_t)slot | (alpha << 31);
+    kept_before += total;
+    __syncthreads();
+    // Each warp moves 4 rows at a time (loads first, then stores).
+    const int64_t chunk_n = (n - base) < kBulkThreads ? (n - base) : kBulkThreads;
+    for (int t = warp * 4; t < chunk_n; t += kBulkWarps * 4) {
+      uint4 val[4];
+      int32_t sl[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        sl[u] = (t + u < chunk_n) ? s_slot[t + u] : -1;
+        if (sl[u] >= 0) {
+          const int64_t row_elem = (((int64_t)b * n + base + t + u) * p.kv_heads + hk) * kHeadDim;
+          val[u] = load_row_chunk(p.k, p.v, row_elem, lane);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (sl[u] >= 0) {
+          const int32_t page = pt[sl[u] / kPageTokens];
+          const uint32_t row = (uint32_t)(sl[u] & (kPageTokens - 1));
+          store_row(p.pool, page, row, lane, val[u]);
+          if (lane == 0) p.pos[(int64_t)page * kPageTokens + row] = (int32_t)(t0 + base + t + u);
+        }
+      }
+    }
+    __syncthreads();
+  }
+  if (tid == 0) p.counts[bh] = (int32_t)new_n;
+}
+
+__global__ void export_positions_kernel(const int32_t* counts, const int32_t* page_table,
+                                        const int32_t* pos, int32_t max_pages, int64_t capacity,
+                                        int32_t* out) {
+  const int bh = blockIdx.x;
+  const int32_t n = counts[bh];
+  const int32_t* pt = page_table + (int64_t)bh * max_pages;
+  int32_t* o = out + (int64_t)bh * capacity;
+  for (int64_t s = threadIdx.x; s < capacity; s += blockDim.x) {
+    int32_t val = -1;
+    if (s < n) val = pos[(int64_t)pt[s / kPageTokens] * kPageTokens + (s & (kPageTokens - 1))];
+    o[s] = val;
+  }
+}
+
+AppendParams make_params(const Cache& c, int32_t layer, const void* k, const void* v,
+                         const void* logit, int64_t t0, int32_t n) {
+  AppendParams p;
+  p.pool = c.pool;
+  p.pos = c.pos;
+  p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
+  p.counts = c.counts + (int64_t)layer * c.heads;
+  p.ring = c.rings + (int64_t)layer * c.heads * c.ring_len;
+  p.ctrl = c.ctrl;
+  p.freed = c.freed;
+  p.k = static_cast<const uint16_t*>(k);
+  p.v = static_cast<const uint16_t*>(v);
+  p.logit = static_cast<const uint16_t*>(logit);
+  p.t0 = t0;
+  p.window = c.window;
+  p.pool_pages = c.pool_pages;
+  p.n = n;
+  p.heads = c.heads;
+  p.kv_heads = c.kv_heads;
+  p.max_pages = c.max_pages;
+  p.ring_len = c.ring_len;
+  return p;
+}
+
+}  // namespace
+
+cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, const void* v,
+                              const void* logit, int64_t t0, cudaStream_t stream) {
+  const AppendParams p = make_params(c, layer, k, v, logit, t0, 1);
+  const int threads = 256, per_block = threads / 32;
+  const int blocks = (c.heads + per_block - 1) / per_block;
+  append_one_kernel<<<blocks, threads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, const void* v,
+                               const void* logit, int64_t t0, int32_t n, cudaStream_t stream) {
+  const AppendParams p = make_params(c, layer, k, v, logit, t0, n);
+  append_bulk_kernel<<<c.heads, kBulkThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_export_positions(const Cache& c, int32_t layer, int32_t* dev_out,
+                                    cudaStream_t stream) {
+  export_positions_kernel<<<c.heads, 256, 0, stream>>>(
+      c.counts + (int64_t)layer * c.heads, c.page_table + (int64_t)layer * c.heads * c.max_pages,
+      c.pos, c.max_pages, c.capacity, dev_out);
+  return cudaGetLastError();
+}
+
+}  // namespace dms

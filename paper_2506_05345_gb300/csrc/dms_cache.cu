@@ -1,0 +1,265 @@
+// Host side of the C ABI declared in include/dms.h: argument checks, cache
+// memory, dispatch to the append and decode kernels, statistics.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+#include <new>
+#include <vector>
+
+#include "dms_internal.cuh"
+
+struct dms_cache {
+  dms::Cache c;
+};
+
+namespace {
+
+using dms::Cache;
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+void free_device(Cache& c) {
+  cudaFree(c.pool);
+  cudaFree(c.pos);
+  cudaFree(c.page_table);
+  cudaFree(c.counts);
+  cudaFree(c.rings);
+  cudaFree(c.ctrl);
+  cudaFree(c.freed);
+  cudaFree(c.pieces);
+  cudaFree(c.piece_counters);
+  c.pool = nullptr;
+  c.pos = c.page_table = c.counts = c.ctrl = c.freed = c.piece_counters = nullptr;
+  c.rings = nullptr;
+  c.pieces = nullptr;
+}
+
+template <typename T>
+cudaError_t alloc(T** p, size_t count) {
+  return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* dms_status_string(dms_status s) {
+  switch (s) {
+    case DMS_OK: return "ok";
+    case DMS_ERR_INVALID_ARGUMENT: return "invalid argument";
+    case DMS_ERR_OUT_OF_MEMORY: return "out of device memory";
+    case DMS_ERR_CAPACITY: return "capacity exceeded (sequence length or page pool)";
+    case DMS_ERR_CUDA: return "CUDA runtime error";
+    case DMS_ERR_TIMEOUT: return "bounded device wait timed out";
+    case DMS_ERR_STATE: return "invalid cache state";
+  }
+  return "unknown status";
+}
+
+dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, int32_t window,
+                            int64_t capacity, const dms_options* opt, dms_cache** out) {
+  if (out == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  *out = nullptr;
+  if (opt == nullptr || layers < 1 || kv_heads < 1 || head_dim != dms::kHeadDim || window < 0 ||
+      capacity < 1 || capacity > 0x7fffffffLL || opt->batch < 1)
+    return DMS_ERR_INVALID_ARGUMENT;
+  if (opt->page_tokens != 0 && opt->page_tokens != dms::kPageTokens) return DMS_ERR_INVALID_ARGUMENT;
+  if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SIMPLE ||
+      opt->ctas_per_sm < 0 || opt->ctas_per_sm > dms::kMaxCtasPerSm || opt->min_pages_per_cta < 0)
+    return DMS_ERR_INVALID_ARGUMENT;
+  for (int i = 0; i < 5; ++i)
+    if (opt->reserved[i] != 0) return DMS_ERR_INVALID_ARGUMENT;
+  const int64_t heads = (int64_t)opt->batch * kv_heads;
+  if (heads > dms::kMaxHeads) return DMS_ERR_INVALID_ARGUMENT;
+
+  dms_cache* h = new (std::nothrow) dms_cache();
+  if (h == nullptr) return DMS_ERR_OUT_OF_MEMORY;
+  Cache& c = h->c;
+  c.layers = layers;
+  c.kv_heads = kv_heads;
+  c.head_dim = head_dim;
+  c.window = window;
+  c.batch = opt->batch;
+  c.capacity = capacity;
+  c.heads = (int32_t)heads;
+  c.ring_len = (int32_t)std::min<int64_t>((int64_t)window + 1, capacity);
+  c.max_pages = (int32_t)((capacity + dms::kPageTokens - 1) / dms::kPageTokens);
+  int64_t pool_tokens = opt->pool_tokens;
+  if (pool_tokens == 0) pool_tokens = (int64_t)layers * heads * capacity;
+  c.pool_pages = (pool_tokens + dms::kPageTokens - 1) / dms::kPageTokens;
+  c.decode_kernel = opt->decode_kernel;
+  c.ctas_per_sm = opt->ctas_per_sm > 0 ? opt->ctas_per_sm : 1;
+  c.min_pages_per_cta = opt->min_pages_per_cta > 0 ? opt->min_pages_per_cta : 2;
+  if (c.pool_pages < 1 || c.pool_pages > 0x7fffffffLL) {
+    delete h;
+    return DMS_ERR_INVALID_ARGUMENT;
+  }
+
+  if (cudaGetDevice(&c.device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, c.device) != cudaSuccess) {
+    delete h;
+    return DMS_ERR_CUDA;
+  }
+  c.piece_capacity = (int64_t)c.num_sms * dms::kMaxCtasPerSm + heads;
+  c.lengths = static_cast<int64_t*>(calloc((size_t)layers, sizeof(int64_t)));
+  if (c.lengths == nullptr) {
+    delete h;
+    return DMS_ERR_OUT_OF_MEMORY;
+  }
+
+  cudaError_t e = cudaSuccess;
+  if (e == cudaSuccess) e = alloc(&c.pool, (size_t)c.pool_pages * dms::kPageBytes);
+  if (e == cudaSuccess) e = alloc(&c.pos, (size_t)c.pool_pages * dms::kPageTokens);
+  if (e == cudaSuccess) e = alloc(&c.page_table, (size_t)layers * heads * c.max_pages);
+  if (e == cudaSuccess) e = alloc(&c.counts, (size_t)layers * heads);
+  if (e == cudaSuccess) e = alloc(&c.rings, (size_t)layers * heads * c.ring_len);
+  if (e == cudaSuccess) e = alloc(&c.ctrl, (size_t)dms::kCtrlWords);
+  if (e == cudaSuccess) e = alloc(&c.freed, (size_t)heads * c.ring_len);
+  if (e == cudaSuccess) e = alloc(&c.pieces, (size_t)c.piece_capacity * dms::kPieceFloats);
+  if (e == cudaSuccess) e = alloc(&c.piece_counters, (size_t)heads);
+  if (e == cudaSuccess) e = cudaMemset(c.counts, 0, sizeof(int32_t) * (size_t)layers * heads);
+  if (e == cudaSuccess) e = cudaMemset(c.ctrl, 0, sizeof(int32_t) * dms::kCtrlWords);
+  if (e == cudaSuccess) e = cudaMemset(c.piece_counters, 0, sizeof(int32_t) * (size_t)heads);
+  if (e == cudaSuccess) e = dms::prepare_decode(c);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    const bool oom = (e == cudaErrorMemoryAllocation);
+    cudaGetLastError();
+    free_device(c);
+    free(c.lengths);
+    delete h;
+    return oom ? DMS_ERR_OUT_OF_MEMORY : DMS_ERR_CUDA;
+  }
+  *out = h;
+  return DMS_OK;
+}
+
+dms_status dms_cache_destroy(dms_cache* h) {
+  if (h == nullptr) return DMS_OK;
+  cudaDeviceSynchronize();
+  free_device(h->c);
+  free(h->c.lengths);
+  delete h;
+  return DMS_OK;
+}
+
+dms_status dms_cache_reset(dms_cache* h, void* stream) {
+  if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // Remember the high-water mark before the pool is handed back.
+  int32_t next = 0;
+  if (cudaMemcpyAsync(&next, c.ctrl + dms::kCtrlPoolNext, sizeof(int32_t), cudaMemcpyDeviceToHost,
+                      st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return DMS_ERR_CUDA;
+  c.peak_pages = std::max<int64_t>(c.peak_pages, std::min<int64_t>(next, c.pool_pages));
+  if (cudaMemsetAsync(c.counts, 0, sizeof(int32_t) * (size_t)c.layers * c.heads, st) != cudaSuccess ||
+      cudaMemsetAsync(c.ctrl, 0, sizeof(int32_t) * dms::kCtrlWords, st) != cudaSuccess ||
+      cudaMemsetAsync(c.piece_counters, 0, sizeof(int32_t) * (size_t)c.heads, st) != cudaSuccess)
+    return DMS_ERR_CUDA;
+  for (int l = 0; l < c.layers; ++l) c.lengths[l] = 0;
+  return DMS_OK;
+}
+
+dms_status dms_append_and_evict(dms_cache* h, int32_t layer, const void* k, const void* v,
+                                const void* decision_logit, int32_t n_tokens, void* stream) {
+  if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  if (layer < 0 || layer >= c.layers || n_tokens < 1 || k == nullptr || v == nullptr ||
+      decision_logit == nullptr || !aligned16(k) || !aligned16(v))
+    return DMS_ERR_INVALID_ARGUMENT;
+  if ((reinterpret_cast<uintptr_t>(decision_logit) & 1u) != 0) return DMS_ERR_INVALID_ARGUMENT;
+  const int64_t t0 = c.lengths[layer];
+  if (t0 + n_tokens > c.capacity) return DMS_ERR_CAPACITY;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const cudaError_t e = (n_tokens == 1)
+                            ? dms::launch_append_one(c, layer, k, v, decision_logit, t0, st)
+                            : dms::launch_append_bulk(c, layer, k, v, decision_logit, t0, n_tokens, st);
+  if (e != cudaSuccess) return DMS_ERR_CUDA;
+  c.lengths[layer] = t0 + n_tokens;
+  return DMS_OK;
+}
+
+dms_status dms_decode_attention(dms_cache* h, int32_t layer, const void* q, void* out,
+                                int32_t gqa_group, float sm_scale, void* stream) {
+  if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  if (layer < 0 || layer >= c.layers || q == nullptr || out == nullptr || !aligned16(q) ||
+      !aligned16(out) || gqa_group < 1 || gqa_group > dms::kMaxGroup || !(sm_scale == sm_scale))
+    return DMS_ERR_INVALID_ARGUMENT;
+  const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (c.decode_kernel == DMS_DECODE_SIMPLE)
+    e = dms::launch_decode_simple(c, layer, q, out, gqa_group, scale, st);
+  else
+    e = dms::launch_decode_tiled(c, layer, q, out, gqa_group, scale * 1.4426950408889634f, st);
+  return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+}
+
+dms_status dms_cache_stats(dms_cache* h, dms_stats* out, int32_t* counts, void* stream) {
+  if (h == nullptr || out == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t n = (size_t)c.layers * c.heads;
+  std::vector<int32_t> host(n);
+  int32_t ctrl[dms::kCtrlWords];
+  if (cudaMemcpyAsync(host.data(), c.counts, n * sizeof(int32_t), cudaMemcpyDeviceToHost, st) !=
+          cudaSuccess ||
+      cudaMemcpyAsync(ctrl, c.ctrl, sizeof(ctrl), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return DMS_ERR_CUDA;
+  memset(out, 0, sizeof(*out));
+  int64_t total = 0;
+  int32_t mx = 0, mn = n ? host[0] : 0;
+  for (size_t i = 0; i < n; ++i) {
+    total += host[i];
+    mx = std::max(mx, host[i]);
+    mn = std::min(mn, host[i]);
+  }
+  int64_t appended = 0;
+  for (int l = 0; l < c.layers; ++l) appended += c.lengths[l] * c.heads;
+  out->total_retained = total;
+  out->total_appended = appended;
+  out->total_evicted = appended - total;
+  out->pages_in_use = std::min<int64_t>(ctrl[dms::kCtrlPoolNext], c.pool_pages);
+  out->pool_pages = c.pool_pages;
+  c.peak_pages = std::max(c.peak_pages, out->pages_in_use);
+  out->peak_pages = c.peak_pages;
+  out->max_retained = mx;
+  out->min_retained = mn;
+  out->device_error = ctrl[dms::kCtrlError];
+  if (counts != nullptr) memcpy(counts, host.data(), n * sizeof(int32_t));
+  return ctrl[dms::kCtrlError] != 0 ? static_cast<dms_status>(ctrl[dms::kCtrlError]) : DMS_OK;
+}
+
+dms_status dms_cache_export_positions(dms_cache* h, int32_t layer, int32_t* host_pos,
+                                      void* stream) {
+  if (h == nullptr || host_pos == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  if (layer < 0 || layer >= c.layers) return DMS_ERR_INVALID_ARGUMENT;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t n = (size_t)c.heads * (size_t)c.capacity;
+  int32_t* dev = nullptr;
+  if (cudaMalloc(&dev, n * sizeof(int32_t)) != cudaSuccess) {
+    cudaGetLastError();
+    return DMS_ERR_OUT_OF_MEMORY;
+  }
+  cudaError_t e = dms::launch_export_positions(c, layer, dev, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(host_pos, dev, n * sizeof(int32_t), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(dev);
+  return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+}
+
+dms_status dms_cache_layer_length(const dms_cache* h, int32_t layer, int64_t* out) {
+  if (h == nullptr || out == nullptr || layer < 0 || layer >= h->c.layers)
+    return DMS_ERR_INVALID_ARGUMENT;
+  *out = h->c.lengths[layer];
+  return DMS_OK;
+}
+
+}  // extern "C"

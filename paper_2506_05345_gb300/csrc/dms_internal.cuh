@@ -1,0 +1,102 @@
+// Internal declarations of libdms (not part of the C ABI).
+//
+// HBM layout of one cache (all device memory owned by the cache):
+//   pool        [pool_pages][2][64][128] bf16   page = 64 K rows then 64 V rows (32 KiB).
+//               Each 256-byte row is stored with its sixteen 16-byte chunks permuted:
+//               logical chunk c of row r sits at physical chunk c ^ (r & 7).  A 1-D bulk
+//               copy of whole rows therefore lands in shared memory already in a
+//               bank-conflict-free order for ldmatrix (8 consecutive rows hit 8 distinct
+//               16-byte bank groups).
+//   pos         [pool_pages][64] int32          position held by each slot (inspection only;
+//                                               decode never reads it).
+//   page_table  [layers][heads][max_pages] int32 page of slot s is page_table[.][s / 64].
+//   counts      [layers][heads] int32            n_h: slots [0, n_h) hold the retained set.
+//   rings       [layers][heads][ring_len] u32    decision ring of the last window+1 tokens:
+//               entry for position j at j % (window + 1) = slot | alpha << 31.
+//   ctrl        [kCtrlWords] int32               [0] next free page, [1] sticky error.
+//   freed       [heads][ring_len] int32          bulk-append scratch (slots freed this call).
+//   pieces      [piece_capacity][kPieceFloats]   split-K partial records of the decode.
+//   piece_counters [heads] int32                 arrivals per head for the last-CTA combine.
+// heads = batch * kv_heads, indexed b * kv_heads + h.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dms.h"
+
+namespace dms {
+
+constexpr int kHeadDim = 128;
+constexpr int kPageTokens = 64;
+constexpr int kRowBytes = kHeadDim * 2;                       // 256
+constexpr int kHalfPageBytes = kPageTokens * kRowBytes;       // 16384
+constexpr int kPageBytes = 2 * kHalfPageBytes;                // 32768
+constexpr int kMaxGroup = 16;                                 // query heads per KV head
+constexpr int kMaxHeads = 4096;                               // batch * kv_heads
+constexpr int kMaxCtasPerSm = 4;
+constexpr uint32_t kAlphaBit = 0x80000000u;
+constexpr uint32_t kSlotMask = 0x7fffffffu;
+constexpr int kPieceFloats = 2 * kMaxGroup + kMaxGroup * kHeadDim;  // m[16] l[16] o[16][128]
+constexpr int kCtrlWords = 16;
+constexpr int kCtrlPoolNext = 0;
+constexpr int kCtrlError = 1;
+// A bounded wait gives up after this many nanoseconds of %globaltimer.
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+struct Cache {
+  int32_t layers = 0, kv_heads = 0, head_dim = 0, window = 0, batch = 0;
+  int64_t capacity = 0;
+  int32_t heads = 0;        // batch * kv_heads
+  int32_t ring_len = 0;     // min(window + 1, capacity)
+  int32_t max_pages = 0;    // ceil(capacity / 64)
+  int64_t pool_pages = 0;
+  int32_t decode_kernel = 0, ctas_per_sm = 1, min_pages_per_cta = 2;
+  int32_t device = 0, num_sms = 0;
+  int64_t piece_capacity = 0;
+
+  uint8_t* pool = nullptr;
+  int32_t* pos = nullptr;
+  int32_t* page_table = nullptr;
+  int32_t* counts = nullptr;
+  uint32_t* rings = nullptr;
+  int32_t* ctrl = nullptr;
+  int32_t* freed = nullptr;
+  float* pieces = nullptr;
+  int32_t* piece_counters = nullptr;
+
+  int64_t* lengths = nullptr;  // host: tokens appended per layer
+  int64_t peak_pages = 0;      // host: largest pages_in_use observed
+};
+
+// Sticky device error: the first code written wins.
+__device__ __forceinline__ void set_device_error(int32_t* ctrl, int32_t code) {
+  atomicCAS(ctrl + kCtrlError, 0, code);
+}
+
+// Sec. 3.2: alpha = round(sigmoid(x)) = [x > 0] on the bf16 bit pattern:
+// sign bit clear, not +0, and not a NaN (+inf, 0x7f80, counts as > 0).
+__device__ __forceinline__ uint32_t decision_from_bf16(uint16_t bits) {
+  return (bits != 0u && bits <= 0x7f80u) ? 1u : 0u;
+}
+
+// Byte offset of logical 16-byte chunk `chunk` of row `row` inside a half page.
+__host__ __device__ __forceinline__ uint32_t swizzled_offset(uint32_t row, uint32_t chunk) {
+  return row * kRowBytes + ((chunk ^ (row & 7u)) << 4);
+}
+
+// Launchers (defined in the .cu files).
+cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, const void* v,
+                              const void* logit, int64_t t0, cudaStream_t stream);
+cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, const void* v,
+                               const void* logit, int64_t t0, int32_t n, cudaStream_t stream);
+cudaError_t launch_export_positions(const Cache& c, int32_t layer, int32_t* dev_out,
+                                    cudaStream_t stream);
+cudaError_t prepare_decode(const Cache& c);
+cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, void* out,
+                                int32_t group, float scale_log2, cudaStream_t stream);
+cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
+                                 int32_t group, float scale, cudaStream_t stream);
+
+}  // namespace dms

@@ -1,0 +1,111 @@
+"""Drives the CUDA path through the C ABI and checks it against the fp64 oracle.
+
+The full appended history (K, V, logits) of the layer under test is kept on the
+device so that any (sequence, KV head) can be handed to the oracle at any step.
+Tolerances: retained sets bit-exact; attention outputs max-abs <= 2e-2 and
+mean-abs <= 2e-3 against the fp64 oracle on the same bf16 inputs.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+import paper_2506_05345_gb300 as dms
+import workloads
+
+MAX_ABS = 2e-2
+MEAN_ABS = 2e-3
+
+
+class Run:
+    def __init__(self, wl: workloads.Workload, device="cuda", layer: int = 0,
+                 capacity: int | None = None, **cache_kw):
+        self.wl, self.layer, self.dev = wl, layer, torch.device(device)
+        self.T = capacity or wl.context
+        B, H, D = wl.batch, wl.kv_heads, wl.head_dim
+        self.cache = dms.DmsCache(layers=1, kv_heads=H, window=wl.window, capacity=self.T,
+                                  batch=B, **cache_kw)
+        self.K = torch.zeros((B, self.T, H, D), dtype=torch.bfloat16, device=self.dev)
+        self.V = torch.zeros_like(self.K)
+        self.L = torch.zeros((B, self.T, H), dtype=torch.bfloat16, device=self.dev)
+        self.t = 0
+        self.errs = []
+
+    def close(self):
+        self.cache.close()
+
+    def append(self, k, v, lg):
+        n = k.shape[1]
+        self.cache.append_and_evict(0, k, v, lg)
+        self.K[:, self.t:self.t + n] = k
+        self.V[:, self.t:self.t + n] = v
+        self.L[:, self.t:self.t + n] = lg
+        self.t += n
+
+    def prefill(self):
+        for i, (n, shared) in enumerate(self.wl.prefill):
+            if shared:
+                k, v, lg = workloads.gen_kv(self.wl, self.layer, f"prefill{i}", n, self.dev, batch=1)
+                B = self.wl.batch
+                k, v = k.expand(B, -1, -1, -1).contiguous(), v.expand(B, -1, -1, -1).contiguous()
+                lg = lg.expand(B, -1, -1).contiguous()
+            else:
+                k, v, lg = workloads.gen_kv(self.wl, self.layer, f"prefill{i}", n, self.dev)
+            self.append(k, v, lg)
+
+    def step(self, s: int):
+        k, v, lg = workloads.gen_kv(self.wl, self.layer, f"decode{s}", 1, self.dev)
+        self.append(k, v, lg)
+        q = workloads.gen_q(self.wl, self.layer, f"decode{s}", self.dev)
+        out = self.cache.decode_attention(0, q, gqa_group=self.wl.gqa_group)
+        return q, out
+
+    # ---- checks
+
+    def logits_host(self) -> np.ndarray:
+        return workloads.bf16_bits(self.L[:, :self.t])
+
+    def check_retained(self, heads=None):
+        """Retained positions of every (b, h) equal the oracle's R_j, bit for bit."""
+        j = self.t - 1
+        pos = self.cache.export_positions(0)
+        L = self.logits_host()
+        B, H = self.wl.batch, self.wl.kv_heads
+        heads = heads if heads is not None else [(b, h) for b in range(B) for h in range(H)]
+        st = self.cache.stats(with_counts=True)
+        assert st["device_error"] == 0, st
+        for b, h in heads:
+            row = pos[b, h]
+            n = int(st["counts"][0, b, h])
+            assert np.all(row[:n] >= 0) and np.all(row[n:] == -1), (b, h)
+            have = np.sort(row[:n])
+            want = oracle.retained(L[b, :, h], j, self.wl.window)
+            assert np.array_equal(have, want), (b, h, len(have), len(want))
+        return st
+
+    def check_outputs(self, q, out, pairs=None, record=True):
+        """Outputs of the given (b, h) KV heads (all G query heads each) vs the oracle."""
+        j = self.t - 1
+        G, B, H = self.wl.gqa_group, self.wl.batch, self.wl.kv_heads
+        pairs = pairs if pairs is not None else [(b, h) for b in range(B) for h in range(H)]
+        Q = workloads.bf16_bits(q)
+        got = out.float().cpu().numpy()
+        errs = []
+        for b, h in pairs:
+            k = workloads.bf16_bits(self.K[b, :j + 1, h])
+            v = workloads.bf16_bits(self.V[b, :j + 1, h])
+            lg = workloads.bf16_bits(self.L[b, :j + 1, h])
+            ref = oracle.decode(Q[b, h * G:(h + 1) * G], k, v, lg, j, self.wl.window)
+            errs.append(np.abs(got[b, h * G:(h + 1) * G].astype(np.float64) - ref).ravel())
+        e = np.concatenate(errs)
+        assert np.all(np.isfinite(got)), "non-finite output"
+        if record:
+            self.errs.append(e)
+        assert e.max() <= MAX_ABS, e.max()
+        return e
+
+    def summary(self):
+        e = np.concatenate(self.errs) if self.errs else np.zeros(1)
+        assert e.mean() <= MEAN_ABS, e.mean()
+        return float(e.max()), float(e.mean())

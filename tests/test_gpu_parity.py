@@ -1,0 +1,268 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Retained sets bit-exact; outputs within max-abs 2e-2 / mean-abs 2e-3.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2506_05345_gb300 as dms
+import workloads
+from _harness import MAX_ABS, MEAN_ABS, Run
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    dms.library()
+
+
+def small(**kw):
+    base = dict(name="t", batch=2, layers=1, q_heads=8, kv_heads=2, window=32,
+                prefill=((300, False),), decode_steps=8, p_evict=0.75)
+    base.update(kw)
+    return workloads.Workload(**base)
+
+
+def _run_all_steps(wl, check_every=1, retained_every=4, **cache_kw):
+    r = Run(wl, **cache_kw)
+    try:
+        r.prefill()
+        r.check_retained()
+        for s in range(wl.decode_steps):
+            q, out = r.step(s)
+            if s % check_every == 0 or s == wl.decode_steps - 1:
+                r.check_outputs(q, out)
+            if s % retained_every == 0 or s == wl.decode_steps - 1:
+                r.check_retained()
+        return r.summary()
+    finally:
+        r.close()
+
+
+# ---------------------------------------------------------------- the small config, in full
+
+
+@pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_SIMPLE])
+def test_llama_b1_ctx4352_every_step(kernel):
+    """Batch 1, 32 q / 8 kv heads, prefill 4096 + 256 decode steps, w = 256, P(evict) 0.875:
+    every step, every query head; retained sets every 16 steps."""
+    wl = workloads.LLAMA_B1_4K
+    mx, mean = _run_all_steps(wl, check_every=1, retained_every=16, decode_kernel=kernel)
+    assert mx <= MAX_ABS and mean <= MEAN_ABS
+
+
+# ---------------------------------------------------------------- edge cases
+
+
+@pytest.mark.parametrize("w", [0, 1, 15, 63, 64, 255, 256])
+def test_windows(w):
+    _run_all_steps(small(window=w, prefill=((333, False),), decode_steps=6))
+
+
+@pytest.mark.parametrize("G", [1, 3, 4, 5, 7, 8, 16])
+def test_gqa_groups(G):
+    _run_all_steps(small(q_heads=2 * G, kv_heads=2, decode_steps=4))
+
+
+@pytest.mark.parametrize("prefill", [1, 2, 63, 64, 65, 127, 128, 129, 1000])
+def test_page_boundaries(prefill):
+    _run_all_steps(small(prefill=((prefill, False),), decode_steps=5, window=20, p_evict=0.5))
+
+
+@pytest.mark.parametrize("p", [0.0, 1.0])
+def test_no_and_total_eviction(p):
+    """p = 0: dense (CR 1).  p = 1: every token is flagged, only the window survives."""
+    wl = small(p_evict=p, prefill=((400, False),), window=40, decode_steps=5)
+    r = Run(wl)
+    try:
+        r.prefill()
+        st = r.check_retained()
+        expect = 400 if p == 0.0 else 41
+        assert np.all(st["counts"] == expect)
+        for s in range(wl.decode_steps):
+            q, out = r.step(s)
+            r.check_outputs(q, out)
+        r.check_retained()
+        r.summary()
+    finally:
+        r.close()
+
+
+def test_w0_all_evict_single_token():
+    """w = 0 and every decision 1: one token remains and the output is v_j (bf16)."""
+    wl = small(window=0, p_evict=1.0, prefill=((70, False),), decode_steps=3)
+    r = Run(wl)
+    try:
+        r.prefill()
+        for s in range(3):
+            q, out = r.step(s)
+            st = r.check_retained()
+            assert np.all(st["counts"] == 1)
+            G = wl.gqa_group
+            want = r.V[:, r.t - 1].repeat_interleave(G, dim=1)
+            assert torch.equal(out, want)
+    finally:
+        r.close()
+
+
+def test_ragged_heads_mixed_probabilities():
+    """Heads with P(evict) from 0 to 1 in one layer: very different n_h per head."""
+    wl = small(batch=3, kv_heads=4, q_heads=20, window=24, prefill=((900, False),), decode_steps=6)
+    r = Run(wl)
+    try:
+        B, H = wl.batch, wl.kv_heads
+        p = [0.0, 0.5, 0.95, 1.0]
+        k, v, lg = workloads.gen_kv(wl, 0, "prefill0", 900, r.dev, p_override=p)
+        r.append(k, v, lg)
+        r.check_retained()
+        for s in range(wl.decode_steps):
+            k, v, lg = workloads.gen_kv(wl, 0, f"decode{s}", 1, r.dev, p_override=p)
+            r.append(k, v, lg)
+            q = workloads.gen_q(wl, 0, f"decode{s}", r.dev)
+            out = r.cache.decode_attention(0, q, gqa_group=wl.gqa_group)
+            r.check_outputs(q, out)
+        st = r.check_retained()
+        assert st["counts"].max() > 5 * st["counts"].min()
+        r.summary()
+    finally:
+        r.close()
+
+
+def test_special_logits():
+    """NaN, +-0, -inf keep; +inf and tiny positives evict (Sec. 3.2 sign rule)."""
+    wl = small(window=4, prefill=((64, False),), decode_steps=0)
+    r = Run(wl)
+    try:
+        vals = torch.tensor([float("nan"), 0.0, -0.0, float("-inf"), float("inf"), 1e-38,
+                             -1e-38, 3.0], dtype=torch.float32)
+        B, H = wl.batch, wl.kv_heads
+        lg = vals.repeat(8)[None, :, None].expand(B, 64, H).contiguous().to(torch.bfloat16).to(r.dev)
+        k, v, _ = workloads.gen_kv(wl, 0, "p", 64, r.dev)
+        r.append(k, v, lg)
+        st = r.check_retained()
+        # kept outside the window: NaN, +0, -0, -inf, -1e-38 (5 of every 8)
+        assert int(st["counts"][0, 0, 0]) == len(np.arange(0, 59)[np.isin(np.arange(59) % 8,
+                                                                           [0, 1, 2, 3, 6])]) + 5
+    finally:
+        r.close()
+
+
+def test_bulk_then_decode_equals_sequential():
+    """Bulk prefill of P tokens gives the same retained sets as P single-token appends."""
+    wl = small(batch=2, kv_heads=2, window=16, prefill=((150, False),), decode_steps=0)
+    a, b = Run(wl), Run(wl)
+    try:
+        k, v, lg = workloads.gen_kv(wl, 0, "prefill0", 150, a.dev)
+        a.append(k, v, lg)
+        for t in range(150):
+            b.append(k[:, t:t + 1].contiguous(), v[:, t:t + 1].contiguous(), lg[:, t:t + 1].contiguous())
+        a.check_retained()
+        b.check_retained()
+        pa, pb = a.cache.export_positions(0), b.cache.export_positions(0)
+        for bb in range(2):
+            for h in range(2):
+                assert np.array_equal(np.sort(pa[bb, h][pa[bb, h] >= 0]), np.sort(pb[bb, h][pb[bb, h] >= 0]))
+        # mixed: bulk chunks of uneven size then singles, still the oracle's sets
+        c = Run(wl)
+        try:
+            for lo, hi in ((0, 7), (7, 100), (100, 101), (101, 150)):
+                c.append(k[:, lo:hi].contiguous(), v[:, lo:hi].contiguous(), lg[:, lo:hi].contiguous())
+            c.check_retained()
+        finally:
+            c.close()
+    finally:
+        a.close()
+        b.close()
+
+
+@pytest.mark.parametrize("min_pages,ctas", [(1, 4), (1, 1), (1000000, 1), (3, 2)])
+def test_split_shapes(min_pages, ctas):
+    """Heads split over many CTAs (multi-piece combine) and one CTA walking all heads."""
+    wl = small(batch=2, kv_heads=3, q_heads=15, window=40, prefill=((2500, False),), decode_steps=3,
+               p_evict=0.3)
+    _run_all_steps(wl, min_pages_per_cta=min_pages, ctas_per_sm=ctas)
+
+
+def test_empty_cache_gives_zeros():
+    wl = small()
+    r = Run(wl)
+    try:
+        q = workloads.gen_q(wl, 0, "q", r.dev)
+        out = r.cache.decode_attention(0, q, gqa_group=wl.gqa_group)
+        torch.cuda.synchronize()
+        assert torch.count_nonzero(out) == 0
+    finally:
+        r.close()
+
+
+def test_deterministic_outputs():
+    wl = small(prefill=((3000, False),), decode_steps=1, window=64)
+    r = Run(wl, min_pages_per_cta=1)
+    try:
+        r.prefill()
+        q, out = r.step(0)
+        again = [r.cache.decode_attention(0, q, gqa_group=wl.gqa_group) for _ in range(3)]
+        for o in again:
+            assert torch.equal(o, out)
+    finally:
+        r.close()
+
+
+def test_stats_and_capacity_errors():
+    wl = small(prefill=((200, False),), decode_steps=2, window=16)
+    r = Run(wl, capacity=203)
+    try:
+        r.prefill()
+        r.step(0)
+        r.step(1)
+        st = r.cache.stats(with_counts=True)
+        assert st["total_appended"] == 202 * wl.batch * wl.kv_heads
+        assert st["total_retained"] == int(st["counts"].sum())
+        assert st["total_evicted"] == st["total_appended"] - st["total_retained"]
+        pages = int(np.sum((st["counts"] + 63) // 64))
+        assert st["pages_in_use"] == pages
+        assert st["max_retained"] == st["counts"].max()
+        k, v, lg = workloads.gen_kv(wl, 0, "over", 2, r.dev)
+        with pytest.raises(dms.DmsError) as ei:
+            r.cache.append_and_evict(0, k, v, lg)  # 202 + 2 > capacity 203
+        assert ei.value.code == dms.DMS_ERR_CAPACITY
+    finally:
+        r.close()
+
+
+def test_pool_exhaustion_is_sticky():
+    """A page pool too small for the batch sets the sticky capacity error."""
+    wl = small(batch=2, kv_heads=2, prefill=((200, False),), decode_steps=0, p_evict=0.0)
+    r = Run(wl, pool_tokens=64 * 6)  # 4 heads need 4 pages each
+    try:
+        r.prefill()
+        st = r.cache.stats()
+        assert st["device_error"] == dms.DMS_ERR_CAPACITY
+        r.cache.reset()
+        assert r.cache.stats()["device_error"] == 0
+    finally:
+        r.close()
+
+
+def test_reset_and_reuse():
+    wl = small(prefill=((500, False),), decode_steps=2)
+    r = Run(wl)
+    try:
+        r.prefill()
+        r.cache.reset()
+        r.t = 0
+        r.K.zero_()
+        r.prefill()
+        for s in range(2):
+            q, out = r.step(s)
+            r.check_outputs(q, out)
+        r.check_retained()
+        assert r.cache.stats()["peak_pages"] > 0
+    finally:
+        r.close()
