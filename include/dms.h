@@ -67,9 +67,10 @@ enum {
 typedef struct dms_options {
   int32_t batch;         /* sequences per layer (required, >= 1)                    */
   int32_t page_tokens;   /* tokens per page; 0 = 64 (only 64 is accepted)           */
-  int64_t pool_tokens;   /* page pool size in tokens, shared by all layers and
-                            heads; 0 = layers * batch * kv_heads * capacity (the
-                            dense worst case), rounded up to whole pages           */
+  int64_t pool_tokens;   /* page pool size in tokens (rounded up to whole pages),
+                            shared by all layers and heads; 0 = the dense worst
+                            case, layers * batch * kv_heads * ceil(capacity / 64)
+                            pages                                                  */
   int32_t decode_kernel; /* DMS_DECODE_TILED (0) or DMS_DECODE_SIMPLE (1)           */
   int32_t ctas_per_sm;   /* split-K CTAs per SM for the tiled kernel; 0 = 1         */
   int32_t min_pages_per_cta; /* lower bound on pages per split-K CTA; 0 = 2         */

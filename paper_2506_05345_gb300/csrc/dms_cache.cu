@@ -86,9 +86,10 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   c.heads = (int32_t)heads;
   c.ring_len = (int32_t)std::min<int64_t>((int64_t)window + 1, capacity);
   c.max_pages = (int32_t)((capacity + dms::kPageTokens - 1) / dms::kPageTokens);
-  int64_t pool_tokens = opt->pool_tokens;
-  if (pool_tokens == 0) pool_tokens = (int64_t)layers * heads * capacity;
-  c.pool_pages = (pool_tokens + dms::kPageTokens - 1) / dms::kPageTokens;
+  // Default: the dense worst case, every head of every layer at full capacity.
+  c.pool_pages = opt->pool_tokens > 0
+                     ? (opt->pool_tokens + dms::kPageTokens - 1) / dms::kPageTokens
+                     : (int64_t)layers * heads * c.max_pages;
   c.decode_kernel = opt->decode_kernel;
   c.ctas_per_sm = opt->ctas_per_sm > 0 ? opt->ctas_per_sm : 1;
   c.min_pages_per_cta = opt->min_pages_per_cta > 0 ? opt->min_pages_per_cta : 2;
