@@ -161,6 +161,48 @@ dms_status dms_cache_export_positions(dms_cache* cache, int32_t layer, int32_t* 
 /* Current length (tokens appended per sequence) of `layer`, into *out. */
 dms_status dms_cache_layer_length(const dms_cache* cache, int32_t layer, int64_t* out);
 
+/*
+ * Decode attention over CALLER-OWNED pages, allocating nothing.
+ *
+ * The paper has no counterpart to this entry point: it exists for callers that
+ * cannot call cudaMalloc at all -- for example code running inside a host
+ * application whose device memory is wholly owned by that application's own
+ * allocator (a framework caching allocator or an arena reserved at start-up),
+ * where a direct device allocation would bypass its budget or fail.  Such a
+ * caller owns every input and output; the library neither creates a cache nor
+ * allocates scratch.  The split-K scratch of the tiled decode kernel lives in a
+ * file-scope device array of about 8.5 MB that every GPU loading the library
+ * holds until the process exits.
+ *
+ * Inputs (device pointers, 16-byte aligned where they hold bf16 rows):
+ *   pool        pages of 32 KiB: page p holds 64 K rows then 64 V rows, each row
+ *               128 bf16 (256 bytes) whose sixteen 16-byte chunks are stored
+ *               permuted -- logical chunk c of row r at physical chunk
+ *               c ^ (r & 7) -- the layout dms_append_and_evict writes.
+ *   page_table  [batch * kv_heads][max_pages] int32: slot s of head (b, h) is
+ *               row s % 64 of page page_table[(b * kv_heads + h) * max_pages + s / 64].
+ *   counts      [batch * kv_heads] int32: head (b, h) attends to its slots
+ *               [0, counts[.]); the caller guarantees counts <= 64 * max_pages
+ *               and valid page ids for every slot below the count.
+ *   q, out      as for dms_decode_attention.
+ * Limits: batch * kv_heads + (number of SMs) <= 1024 (872 heads on a 152-SM
+ * GB300), else DMS_ERR_CAPACITY; 1 <= gqa_group <= 16.
+ *
+ * The first call on each device does a one-time set-up on the calling thread
+ * with that device current (looks up the scratch array's device address and sets
+ * the kernel's shared-memory limit); make that first call before any stream
+ * capture.  Every call clears the scratch counters it needs with an asynchronous
+ * memset on `stream` and then launches; all calls share the one array, so calls
+ * whose work overlaps on the GPU (other streams, other host threads) race and
+ * must be serialised by the caller.  A bounded in-kernel wait that gives up is
+ * recorded only in the scratch array, not reported.
+ */
+dms_status dms_decode_attention_paged_noalloc(const void* pool, const int32_t* page_table,
+                                              const int32_t* counts, int32_t batch,
+                                              int32_t kv_heads, int32_t max_pages,
+                                              const void* q, void* out, int32_t gqa_group,
+                                              float sm_scale, void* stream);
+
 /* Static description of a status code. */
 const char* dms_status_string(dms_status status);
 

@@ -87,6 +87,14 @@ def dms_cache_layer_length(cache, layer):
     return code, out.value
 
 
+def dms_decode_attention_paged_noalloc(pool_ptr, page_table_ptr, counts_ptr, batch, kv_heads,
+                                       max_pages, q_ptr, out_ptr, gqa_group, sm_scale, stream):
+    """Decode over caller-owned pages with the library's static scratch (no allocation)."""
+    return library().dms_decode_attention_paged_noalloc(
+        pool_ptr, page_table_ptr, counts_ptr, batch, kv_heads, max_pages, q_ptr, out_ptr,
+        gqa_group, float(sm_scale), stream)
+
+
 # ---- torch-facing wrapper ---------------------------------------------------
 
 def _stream_ptr(stream=None):

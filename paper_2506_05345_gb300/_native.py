@@ -26,7 +26,7 @@ DMS_DECODE_SIMPLE = 1
 EXPORTS = (
     "dms_cache_create", "dms_cache_destroy", "dms_cache_reset", "dms_append_and_evict",
     "dms_decode_attention", "dms_cache_stats", "dms_cache_export_positions",
-    "dms_cache_layer_length", "dms_status_string",
+    "dms_cache_layer_length", "dms_status_string", "dms_decode_attention_paged_noalloc",
 )
 
 
@@ -77,6 +77,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_cache_export_positions": (st, [vp, i32, vp, vp]),
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),
         "dms_status_string": (ctypes.c_char_p, [st]),
+        "dms_decode_attention_paged_noalloc": (st, [vp, vp, vp, i32, i32, i32, vp, vp, i32, f32,
+                                                    vp]),
     }
     for name, (res, args) in proto.items():
         fn = getattr(lib, name)

@@ -602,3 +602,115 @@ cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, v
 }
 
 }  // namespace dms
+
+// ============================================================================
+// Allocation-free decode over caller-owned pages.
+//
+// Some callers cannot call cudaMalloc at all: for example a plugin living inside
+// a host application whose device memory is entirely owned by that application's
+// own allocator (a framework caching allocator or a fixed-budget arena reserved
+// at start-up), where a direct cudaMalloc would bypass the budget or fail.  Such a
+// caller owns the paged KV arrays and the query/output buffers itself.  The only
+// extra memory the tiled decode kernel needs is its split-K scratch (partial
+// records and per-head arrival counters); here it lives in one file-scope device
+// array that every GPU loading the library holds until the process exits.
+// ============================================================================
+
+#include <mutex>
+
+namespace {
+
+// Partial records the static scratch can hold; a launch needs (CTAs + heads).
+constexpr int kStaticRecords = 1024;
+constexpr int kStaticCounters = kStaticRecords;  // per-head arrival counters (int32)
+constexpr int kStaticCtrl = dms::kCtrlWords;     // error word of the kernel (int32)
+constexpr size_t kStaticScratchWords =
+    (size_t)kStaticRecords * dms::kPieceFloats + kStaticCounters + kStaticCtrl;
+constexpr int kMaxDevices = 64;
+
+struct StaticDeviceState {
+  bool ready = false;
+  float* scratch = nullptr;  // device address of g_decode_scratch on this device
+  int num_sms = 0;
+};
+std::mutex g_static_mu;
+StaticDeviceState g_static_state[kMaxDevices];
+
+}  // namespace
+
+// 32-bit words: [records][kPieceFloats] floats, then counters, then the error word.
+static __device__ __align__(256) float g_decode_scratch[kStaticScratchWords];
+
+extern "C" dms_status dms_decode_attention_paged_noalloc(
+    const void* pool, const int32_t* page_table, const int32_t* counts, int32_t batch,
+    int32_t kv_heads, int32_t max_pages, const void* q, void* out, int32_t gqa_group,
+    float sm_scale, void* stream) {
+  using namespace dms;
+  auto misaligned = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; };
+  if (pool == nullptr || page_table == nullptr || counts == nullptr || q == nullptr ||
+      out == nullptr || misaligned(pool) || misaligned(q) || misaligned(out) || batch < 1 ||
+      kv_heads < 1 || max_pages < 1 || gqa_group < 1 || gqa_group > kMaxGroup ||
+      !(sm_scale == sm_scale))
+    return DMS_ERR_INVALID_ARGUMENT;
+  const int64_t heads = (int64_t)batch * kv_heads;
+  if (heads > kMaxHeads) return DMS_ERR_INVALID_ARGUMENT;
+
+  // One-time set-up per device, with that device current: the device address of
+  // the scratch array (the host-side name is only a stand-in), the kernel's
+  // shared-memory limit and the SM count.
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return DMS_ERR_CUDA;
+  StaticDeviceState st;
+  {
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    StaticDeviceState& s = g_static_state[dev];
+    if (!s.ready) {
+      void* ptr = nullptr;
+      if (cudaGetSymbolAddress(&ptr, g_decode_scratch) != cudaSuccess) {
+        cudaGetLastError();
+        return DMS_ERR_CUDA;
+      }
+      int sms = 0;
+      if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+          cudaFuncSetAttribute(decode_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)tiled_smem_bytes(kMaxHeads)) != cudaSuccess) {
+        cudaGetLastError();
+        return DMS_ERR_CUDA;
+      }
+      s.scratch = static_cast<float*>(ptr);
+      s.num_sms = sms;
+      s.ready = true;
+    }
+    st = s;
+  }
+  const int grid = st.num_sms;
+  if (grid + heads > kStaticRecords) return DMS_ERR_CAPACITY;  // scratch too small for this batch
+
+  int32_t* counters = reinterpret_cast<int32_t*>(st.scratch + (size_t)kStaticRecords * kPieceFloats);
+  int32_t* ctrl = counters + kStaticCounters;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // The array keeps whatever the previous call left: the arrival counters and the
+  // error word must start at zero.
+  if (cudaMemsetAsync(counters, 0, sizeof(int32_t) * (size_t)(kStaticCounters + kStaticCtrl), s) !=
+      cudaSuccess)
+    return DMS_ERR_CUDA;
+
+  DecodeParams p;
+  p.pool = static_cast<const uint8_t*>(pool);
+  p.page_table = page_table;
+  p.counts = counts;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.pieces = st.scratch;
+  p.piece_counters = counters;
+  p.ctrl = ctrl;
+  p.heads = (int32_t)heads;
+  p.kv_heads = kv_heads;
+  p.group = gqa_group;
+  p.max_pages = max_pages;
+  p.min_pages = 2;
+  const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)kHeadDim);
+  p.scale_log2 = scale * 1.4426950408889634f;
+  decode_tiled_kernel<<<grid, kThreads, tiled_smem_bytes((int)heads), s>>>(p);
+  return cudaGetLastError() == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+}
