@@ -55,6 +55,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--ctas-per-sm", type=int, default=0)
     ap.add_argument("--min-pages", type=int, default=0)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="override the layer count (small cases for profiling)")
     return ap.parse_args()
 
 
@@ -66,8 +68,10 @@ def get_workload(args):
                 wl = s
     if wl is None:
         raise SystemExit(f"unknown workload {args.workload}")
+    import dataclasses
+    if args.layers > 0:
+        wl = dataclasses.replace(wl, layers=args.layers)
     if args.dense:
-        import dataclasses
         wl = dataclasses.replace(wl, p_evict=0.0, ragged_beta=False, name=wl.name + "-dense")
     return wl
 
