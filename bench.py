@@ -206,8 +206,9 @@ def run_ours(args, wl, world, rank, local, pg):
     B, L, H, G, D = wl.batch, wl.layers, wl.kv_heads, wl.gqa_group, wl.head_dim
     Hq = H * G
     K_, W_ = args.steps, args.warmup
+    K2 = max(1, min(K_, 20))  # extra steps with per-kernel events (roofline durations)
     E_K, E_W = (0, 0) if args.no_e2e else (min(K_, 50), 2)
-    decode_needed = max(wl.decode_steps, W_ + K_ + E_W + E_K)
+    decode_needed = max(wl.decode_steps, W_ + K_ + K2 + E_W + E_K)
     capacity = wl.prefill_tokens + decode_needed
     seed_tag = f"rank{rank}"
     cache = dms.DmsCache(layers=L, kv_heads=H, window=wl.window, capacity=capacity, batch=B,
@@ -245,7 +246,7 @@ def run_ours(args, wl, world, rank, local, pg):
         raise RuntimeError(f"device error after prefill: {st0}")
 
     # ---- step inputs, resident in HBM before the timed region
-    n_dev_steps = W_ + K_
+    n_dev_steps = W_ + K_ + K2
     ins = []
     for s in range(n_dev_steps):
         per = []
@@ -257,9 +258,9 @@ def run_ours(args, wl, world, rank, local, pg):
     outs = [torch.empty((B, Hq, D), dtype=torch.bfloat16, device=dev) for _ in range(L)]
 
     ev_dec = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(L)] for _ in range(K_)]
+               for _ in range(L)] for _ in range(K2)]
     ev_app = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(L)] for _ in range(K_)]
+               for _ in range(L)] for _ in range(K2)]
 
     def do_step(s, timed_idx=None):
         for layer in range(L):
@@ -285,9 +286,11 @@ def run_ours(args, wl, world, rank, local, pg):
     torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
+    # Timed region: K whole steps back to back, no events between kernels (an event
+    # between two kernels would serialise their programmatic overlap).
     t_start.record(stream)
     for i in range(K_):
-        do_step(W_ + i, timed_idx=i)
+        do_step(W_ + i)
     t_end.record(stream)
     torch.cuda.synchronize()
     barrier(pg)
@@ -296,6 +299,13 @@ def run_ours(args, wl, world, rank, local, pg):
     st_after = cache.stats()
     if st_after["device_error"]:
         raise RuntimeError(f"device error during timed steps: {st_after}")
+    # Second timed region: K2 further steps with CUDA events around every append
+    # and decode launch, for the per-kernel durations of the roofline.
+    torch.cuda.synchronize()
+    for i in range(K2):
+        do_step(W_ + K_ + i, timed_idx=i)
+    torch.cuda.synchronize()
+    st_k2 = cache.stats()
     # tokens read per step: every head reads n_h after its append; n_h grows by 0 or 1
     # per step, so the per-step total is interpolated between the two snapshots
     # (the error is below the growth over the run, < 0.2 % here).
@@ -303,10 +313,10 @@ def run_ours(args, wl, world, rank, local, pg):
     tok_last = st_after["total_retained"]
     tokens_read = K_ * 0.5 * (tok_first + tok_last)
     dec_ms = [ev_dec[i][layer][0].elapsed_time(ev_dec[i][layer][1])
-              for i in range(K_) for layer in range(L)]
+              for i in range(K2) for layer in range(L)]
     app_ms = [ev_app[i][layer][0].elapsed_time(ev_app[i][layer][1])
-              for i in range(K_) for layer in range(L)]
-    units_per_launch = 0.5 * (tok_first + tok_last) / L
+              for i in range(K2) for layer in range(L)]
+    units_per_launch = 0.5 * (tok_last + st_k2["total_retained"]) / L
     bytes_per_unit = workloads.kv_bytes_per_token_head(D)
     dec_avg_s = float(np.mean(dec_ms)) * 1e-3
 
@@ -320,8 +330,8 @@ def run_ours(args, wl, world, rank, local, pg):
     if rank == 0:
         import oracle
         Gs = G
-        last = W_ + K_ - 1
-        for s in range(W_ + K_):
+        last = n_dev_steps - 1
+        for s in range(n_dev_steps):
             k, v, lg, q = ins[s][0]
             for (b, h) in sample:
                 hist[(b, h)]["k"].append(workloads.bf16_bits(k[b, :, h]))
@@ -329,7 +339,7 @@ def run_ours(args, wl, world, rank, local, pg):
                 hist[(b, h)]["l"].append(workloads.bf16_bits(lg[b, :, h]))
         q_last = workloads.bf16_bits(ins[last][0][3])
         got = outs[0].float().cpu().numpy()
-        j = wl.prefill_tokens + W_ + K_ - 1
+        j = wl.prefill_tokens + n_dev_steps - 1
         errs = []
         cases = []
         for (b, h) in sample:
@@ -433,7 +443,7 @@ def run_ours(args, wl, world, rank, local, pg):
         "decode_us_per_layer_step": float(np.mean(dec_ms)) * 1e3,
         "append_us_per_layer_step": float(np.mean(app_ms)) * 1e3,
         "retained_tokens_per_layer_step": units_per_launch,
-        "compression": (wl.prefill_tokens + W_ + K_) * B * H / (units_per_launch),
+        "compression": (wl.prefill_tokens + n_dev_steps) * B * H / units_per_launch,
         "hbm_frac_of_nominal_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
         "roofline": {"kernel": "decode_tiled_kernel", "bound": "hbm", "achieved": achieved_gbs,
                      "peak": peak, "unit": "GB/s", "frac": achieved_gbs / peak,

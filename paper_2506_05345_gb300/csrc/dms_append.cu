@@ -13,6 +13,14 @@
 namespace dms {
 namespace {
 
+// Programmatic dependent launch (see the decode kernel): no-ops without it.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait_prerequisites() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 struct AppendParams {
   uint8_t* pool;
   int32_t* pos;
@@ -50,6 +58,8 @@ __device__ __forceinline__ uint4 load_row_chunk(const uint16_t* k, const uint16_
 // n = 1: one warp per head.  Lane 0 runs the ring/slot logic, the warp moves the
 // 512 bytes of K and V.
 __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
+  pdl_launch_dependents();
+  pdl_wait_prerequisites();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.x * (blockDim.x >> 5) + warp;
   if (bh >= p.heads) return;
@@ -123,6 +133,8 @@ __device__ __forceinline__ int block_scan_flags(int flag, int* s_warp, int* tota
 // set as n single-token appends; slots freed by tokens that leave during the call
 // are refilled first (in order), further kept tokens extend [0, n_h).
 __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendParams p) {
+  pdl_launch_dependents();
+  pdl_wait_prerequisites();
   __shared__ int s_warp[kBulkWarps];
   __shared__ int32_t s_slot[kBulkThreads];
   __shared__ int32_t s_misc[4];
@@ -280,9 +292,16 @@ cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, cons
                               const void* logit, int64_t t0, cudaStream_t stream) {
   const AppendParams p = make_params(c, layer, k, v, logit, t0, 1);
   const int threads = 256, per_block = threads / 32;
-  const int blocks = (c.heads + per_block - 1) / per_block;
-  append_one_kernel<<<blocks, threads, 0, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3((c.heads + per_block - 1) / per_block);
+  cfg.blockDim = dim3(threads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, append_one_kernel, p);
 }
 
 cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, const void* v,

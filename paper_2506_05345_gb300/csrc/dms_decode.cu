@@ -5,19 +5,26 @@
 // Tiled kernel (default).  The work is the flat list of all pages of all heads of
 // the layer, split into equal contiguous ranges, one per CTA (page-balanced
 // split-K: ragged heads cost nothing extra and every SM streams the same number
-// of bytes).  Per CTA:
-//   * one producer warp walks its page range and stages each page's valid K rows,
+// of bytes).  Per CTA, three warp roles:
+//   * a producer warp walks the CTA's pages and stages each page's valid K rows,
 //     V rows (and, at the first page of a head, the group's queries) into a
-//     shared-memory ring of NST stages with 1-D bulk async copies (TMA engine)
+//     shared-memory ring of kStages stages with 1-D bulk async copies (TMA engine)
 //     completing on mbarriers;
-//   * four consumer warps each own 16 tokens of every page: S = Q K^T and O += P V
-//     on the tensor cores (mma.sync m16n8k16 bf16 -> fp32, G query heads padded to
-//     16 rows), fp32 online softmax in the exp2 domain, quad shuffles for the row
-//     reductions;
-//   * at the end of each head segment the four warp states are merged in shared
-//     memory; a head covered by one CTA is written directly, otherwise the CTA
-//     writes a partial record (m, l, O) and the last CTA to arrive on the head's
-//     counter merges all records (log-sum-exp combine) and writes the output.
+//   * four consumer warps each own 16 tokens of every page.  With the tokens and
+//     head_dim in the M dimension of the tensor-core tiles and the group's <= 8
+//     query heads in N (16 with two n-tiles), one page costs each warp
+//     S^T = K Q^T (8 mma.sync m16n8k16, two independent accumulation chains) and
+//     O^T += V^T P^T (8 mma.sync); P^T is formed from S^T in registers with
+//     movmatrix.  fp32 online softmax in the exp2 domain; S^T and O^T share their
+//     column (head) layout, so the running rescale needs no shuffles;
+//   * an epilogue warp finishes each head segment while the consumers move on:
+//     it merges the four warp partials from a double-buffered shared-memory slot,
+//     writes the output of a head the CTA covers alone, or writes a partial record
+//     (m, l, O); the last CTA to arrive on a split head's counter merges all
+//     records (log-sum-exp combine) and writes the output.
+// A CTA takes its pages in the order: its first head's part, its last head's part
+// (the two it may share with neighbours), then the heads in between, so the
+// cross-CTA combines happen early and the CTA ends on directly written heads.
 // Arithmetic intensity is G flop per byte of K/V, far below the tensor-core ridge:
 // the kernel is HBM-bound and the tensor cores only keep the issue slots free.
 //
@@ -31,13 +38,26 @@ namespace dms {
 namespace {
 
 constexpr int kConsumerWarps = 4;
-constexpr int kThreads = (kConsumerWarps + 1) * 32;
-constexpr int kConsumerThreads = kConsumerWarps * 32;
+constexpr int kProducerWarp = 4;
+constexpr int kEpilogueWarp = 5;
+constexpr int kThreads = 6 * 32;
 constexpr int kQBytes = kMaxGroup * kRowBytes;                 // 4096
 constexpr int kStageBytes = 2 * kHalfPageBytes + kQBytes;      // 36864
-constexpr int kMergeOBytes = kConsumerWarps * kMaxGroup * kHeadDim * 4;  // 32768
-constexpr int kMergeMLBytes = kConsumerWarps * kMaxGroup * 2 * 4;         // 512
-constexpr int kStages = 4;
+// Merge rows (one per query head, 128 floats of head_dim) are padded to 132
+// floats: the stores of an O^T accumulator fragment then hit 32 distinct banks.
+constexpr int kMergeRow = kHeadDim + 4;
+// Pipeline depth per CTA: 4 stages with one CTA per SM, 2 stages with two.
+constexpr int kStagesOneCta = 4;
+constexpr int kStagesTwoCta = 2;
+
+// Shared-memory plan that depends on the number of 8-head n-tiles (NT).
+template <int NT>
+struct Plan {
+  static constexpr int kHeadsPad = 8 * NT;
+  static constexpr int kSlots = NT == 1 ? 2 : 1;  // merge slots (double-buffered if they fit)
+  static constexpr int kSlotOFloats = kConsumerWarps * kHeadsPad * kMergeRow;
+  static constexpr int kSlotMLFloats = kConsumerWarps * kHeadsPad * 2;
+};
 
 struct DecodeParams {
   const uint8_t* pool;
@@ -95,9 +115,8 @@ __device__ __forceinline__ unsigned long long global_timer_ns() {
 // kWaitLimitNs, or at once when another thread of the CTA has already given up
 // (*abort != 0); then records DMS_ERR_TIMEOUT and returns false.  Callers keep
 // their control flow unchanged on failure, so no barrier is ever left waiting.
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                       int32_t* ctrl) {
-  if (mbar_try_wait(bar, parity)) return true;
+__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                            int32_t* ctrl) {
   const unsigned long long t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -110,6 +129,12 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
       }
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          int32_t* ctrl) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, abort, ctrl);
 }
 
 __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes,
@@ -147,14 +172,28 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// Transpose of an 8x8 b16 matrix held one 32-bit fragment per thread.
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-__device__ __forceinline__ void named_barrier_consumers() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kConsumerThreads) : "memory");
+// Programmatic dependent launch: let the next kernel of the stream start its
+// prologue now; wait until the previous kernel's results are visible.  Both are
+// no-ops when the launches carry no programmatic dependency.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
+__device__ __forceinline__ void pdl_wait_prerequisites() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 
 // ---------------------------------------------------------------- partition helpers
 
@@ -174,39 +213,86 @@ __device__ __forceinline__ int head_of_page(const int32_t* pstart, int heads, in
   return lo - 1;
 }
 
-size_t tiled_smem_bytes(int heads) {
-  return (size_t)kStages * kStageBytes + kMergeOBytes + kMergeMLBytes +
-         2 * kStages * sizeof(uint64_t) + 64 + (size_t)(2 * heads + 1) * sizeof(int32_t);
+template <int NT>
+size_t tiled_smem_bytes(int heads, int stages) {
+  using PL = Plan<NT>;
+  return (size_t)stages * kStageBytes + (size_t)PL::kSlots * (PL::kSlotOFloats + PL::kSlotMLFloats) * 4 +
+         (size_t)(2 * stages + 2 * PL::kSlots) * sizeof(uint64_t) + 64 +
+         (size_t)(2 * heads + 1) * sizeof(int32_t);
 }
 
-// ---------------------------------------------------------------- tiled kernel
+// Iteration order over a CTA's pages (parts A, C, B; see the file comment) and the
+// per-iteration position (head h, page pg within the head).  Every warp role walks
+// it identically from shared-memory tables only.
+struct PageWalk {
+  const int32_t* pstart;  // [heads + 1] page prefix
+  int heads;
+  int64_t pbeg, a_end, c_beg;
+  int nA, nC;
+  int h, pg;
 
-__global__ void __launch_bounds__(kThreads, 1) decode_tiled_kernel(const DecodeParams p) {
+  __device__ __forceinline__ int64_t flat(int it) const {
+    return it < nA ? pbeg + it : (it < nA + nC ? c_beg + (it - nA) : a_end + (it - nA - nC));
+  }
+  // Position for iteration `it` (call with it = 0, 1, 2, ... in order).
+  __device__ __forceinline__ void enter(int it) {
+    if (it == 0 || it == nA || it == nA + nC) {
+      const int64_t x = flat(it);
+      h = head_of_page(pstart, heads, x);
+      pg = (int)(x - pstart[h]);
+    }
+  }
+  __device__ __forceinline__ int pages_of_head() const { return pstart[h + 1] - pstart[h]; }
+  __device__ __forceinline__ bool seg_start(int it) const { return it == 0 || pg == 0; }
+  __device__ __forceinline__ bool seg_end(int it, int niters) const {
+    return it == nA - 1 || it == nA + nC - 1 || it == niters - 1 || pg == pages_of_head() - 1;
+  }
+  __device__ __forceinline__ void advance() {
+    if (++pg == pages_of_head()) {
+      pg = 0;
+      do { ++h; } while (h < heads && pstart[h + 1] == pstart[h]);
+      if (h >= heads) h = heads - 1;  // only past the end of a part
+    }
+  }
+};
+
+template <int kStages, int NT>
+__global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
+    decode_tiled_kernel(const DecodeParams p) {
+  using PL = Plan<NT>;
+  constexpr int HP = PL::kHeadsPad;
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
-  float* merge_o = reinterpret_cast<float*>(smem + kStages * kStageBytes);  // [4][16][128]
-  float* merge_m = merge_o + kConsumerWarps * kMaxGroup * kHeadDim;           // [4][16]
-  float* merge_l = merge_m + kConsumerWarps * kMaxGroup;                      // [4][16]
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(merge_l + kConsumerWarps * kMaxGroup);
+  float* merge_o = reinterpret_cast<float*>(smem + kStages * kStageBytes);  // [slots][4][HP][132]
+  float* merge_ml = merge_o + PL::kSlots * PL::kSlotOFloats;                  // [slots][4][HP][2]
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(merge_ml + PL::kSlots * PL::kSlotMLFloats);
   uint64_t* empty_bar = full_bar + kStages;
-  int* s_misc = reinterpret_cast<int*>(empty_bar + kStages);  // [0] abort [1] last flag [2..7] warp sums
-  int32_t* s_cnt = s_misc + 16;                                // [heads]
-  int32_t* s_pstart = s_cnt + p.heads;                         // [heads + 1]
+  uint64_t* mfull_bar = empty_bar + kStages;
+  uint64_t* mempty_bar = mfull_bar + PL::kSlots;
+  int* s_misc = reinterpret_cast<int*>(mempty_bar + PL::kSlots);  // [0] abort [2..7] warp sums
+  int32_t* s_cnt = s_misc + 16;                                   // [heads]
+  int32_t* s_pstart = s_cnt + p.heads;                            // [heads + 1]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int heads = p.heads, G = p.group, Hq = p.kv_heads * p.group;
   volatile int* abort_flag = s_misc;
 
-  // ---- prologue: per-head counts, page prefix, CTA range
-  for (int h = tid; h < heads; h += kThreads) s_cnt[h] = p.counts[h];
+  // ---- prologue: barriers (before the dependency), per-head counts, page prefix
+  pdl_launch_dependents();
   if (tid == 0) {
     s_misc[0] = 0;
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kConsumerWarps);
     }
+    for (int s = 0; s < PL::kSlots; ++s) {
+      mbar_init(&mfull_bar[s], kConsumerWarps);
+      mbar_init(&mempty_bar[s], 1);
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  pdl_wait_prerequisites();
+  for (int h = tid; h < heads; h += kThreads) s_cnt[h] = p.counts[h];
   __syncthreads();
   {
     const int per = (heads + kThreads - 1) / kThreads;
@@ -247,16 +333,29 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tiled_kernel(const DecodeP
   if (k >= P) return;
   const int64_t pbeg = (int64_t)k * N / P, pend = (int64_t)(k + 1) * N / P;
   const int niters = (int)(pend - pbeg);
-  const int h_first = head_of_page(s_pstart, heads, pbeg);
+  PageWalk walk;
+  walk.pstart = s_pstart;
+  walk.heads = heads;
+  walk.pbeg = pbeg;
+  {
+    const int h_first = head_of_page(s_pstart, heads, pbeg);
+    const int h_last = head_of_page(s_pstart, heads, pend - 1);
+    walk.a_end = (h_first == h_last) ? pend : (int64_t)s_pstart[h_first + 1];
+    walk.c_beg = (h_first == h_last) ? pend : (int64_t)s_pstart[h_last];
+    walk.nA = (int)(walk.a_end - pbeg);
+    walk.nC = (int)(pend - walk.c_beg);
+    walk.h = h_first;
+    walk.pg = 0;
+  }
 
-  if (warp == kConsumerWarps) {
+  if (warp == kProducerWarp) {
     // ================================================================ producer warp
     int issued = 0;
     for (int it0 = 0; it0 < niters; it0 += 32) {
       const int it = it0 + lane;
       int hh = 0, pg = 0, nv = 0, page = 0;
       if (it < niters) {
-        const int64_t x = pbeg + it;
+        const int64_t x = walk.flat(it);
         hh = head_of_page(s_pstart, heads, x);
         pg = (int)(x - s_pstart[hh]);
         nv = min(kPageTokens, s_cnt[hh] - pg * kPageTokens);
@@ -300,123 +399,238 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tiled_kernel(const DecodeP
     return;
   }
 
+  if (warp == kEpilogueWarp) {
+    // ================================================================ epilogue warp
+    int q = 0;  // segment counter
+    for (int it = 0; it < niters; ++it) {
+      walk.enter(it);
+      if (walk.seg_end(it, niters)) {
+        const int h = walk.h;
+        const int slot = q % PL::kSlots;
+        mbar_wait(&mfull_bar[slot], (q / PL::kSlots) & 1, abort_flag, p.ctrl);
+        const float* so = merge_o + slot * PL::kSlotOFloats;
+        const float* sml = merge_ml + slot * PL::kSlotMLFloats;
+        const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
+        const int64_t first = s_pstart[h], last = s_pstart[h + 1] - 1;
+        const int k_lo = cta_of_page(first, P, N), k_hi = cta_of_page(last, P, N);
+        const bool single = (k_lo == k_hi);
+        __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+        float* rec = p.pieces + (int64_t)(k + h) * kPieceFloats;  // m[16] l[16] o[16][128]
+        for (int r = 0; r < G; ++r) {
+          float M = sml[(0 * HP + r) * 2];
+#pragma unroll
+          for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, sml[(w * HP + r) * 2]);
+          float wt[kConsumerWarps];
+          float L = 0.f;
+#pragma unroll
+          for (int w = 0; w < kConsumerWarps; ++w) {
+            wt[w] = exp2f(sml[(w * HP + r) * 2] - M);
+            L += wt[w] * sml[(w * HP + r) * 2 + 1];
+          }
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int d = lane + 32 * i;
+            float O = 0.f;
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) O += wt[w] * so[(w * HP + r) * kMergeRow + d];
+            if (single) out_h[r * kHeadDim + d] = __float2bfloat16_rn(O / L);
+            else rec[2 * kMaxGroup + r * kHeadDim + d] = O;
+          }
+          if (!single && lane == 0) {
+            rec[r] = M;
+            rec[kMaxGroup + r] = L;
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&mempty_bar[slot]);  // the slot may be refilled
+        if (!single) {
+          __threadfence();
+          __syncwarp();
+          int is_last = 0;
+          if (lane == 0) is_last = (atomicAdd(p.piece_counters + h, 1) == k_hi - k_lo) ? 1 : 0;
+          is_last = __shfl_sync(0xffffffffu, is_last, 0);
+          if (is_last) {
+            // Last CTA of this head: online log-sum-exp merge of all records, in
+            // CTA order, eight rows at a time; every load of one record for eight
+            // rows is issued together.
+            __threadfence();
+            for (int r0 = 0; r0 < G; r0 += 8) {
+              float Mr[8], Lr[8], Or[8][4];
+#pragma unroll
+              for (int r = 0; r < 8; ++r) {
+                Mr[r] = -INFINITY;
+                Lr[r] = 0.f;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) Or[r][i] = 0.f;
+              }
+              for (int kk = k_lo; kk <= k_hi; ++kk) {
+                const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
+                float mk[8], lk[8], ok[8][4];
+#pragma unroll
+                for (int r = 0; r < 8; ++r) {
+                  if (r0 + r < G) {
+                    mk[r] = __ldcg(rk + r0 + r);
+                    lk[r] = __ldcg(rk + kMaxGroup + r0 + r);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                      ok[r][i] = __ldcg(rk + 2 * kMaxGroup + (r0 + r) * kHeadDim + lane + 32 * i);
+                  }
+                }
+#pragma unroll
+                for (int r = 0; r < 8; ++r) {
+                  if (r0 + r < G) {
+                    const float Mn = fmaxf(Mr[r], mk[r]);
+                    const float a = exp2f(Mr[r] - Mn), bw = exp2f(mk[r] - Mn);
+                    Lr[r] = Lr[r] * a + lk[r] * bw;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) Or[r][i] = Or[r][i] * a + ok[r][i] * bw;
+                    Mr[r] = Mn;
+                  }
+                }
+              }
+#pragma unroll
+              for (int r = 0; r < 8; ++r)
+                if (r0 + r < G)
+#pragma unroll
+                  for (int i = 0; i < 4; ++i)
+                    out_h[(r0 + r) * kHeadDim + lane + 32 * i] = __float2bfloat16_rn(Or[r][i] / Lr[r]);
+            }
+            if (lane == 0) p.piece_counters[h] = 0;
+          }
+        }
+        ++q;
+      }
+      walk.advance();
+    }
+    return;
+  }
+
   // ================================================================ consumer warps
   const int g = lane >> 2, c4 = lane & 3;
   const int tb = warp * 16;  // this warp's first token within a page
-  uint32_t qa[8][4];
-  float o[16][4];
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-  int h = h_first;
-  int pg = (int)(pbeg - s_pstart[h]);
+  const int mi = lane >> 3;  // ldmatrix: which of the four 8x8 matrices this lane addresses
+  uint32_t qb[8][NT][2];     // Q^T B-fragments: (d = 16 kk + 2c.., head 8 nt + g)
+  float o[8][NT][4];         // O^T accumulators: (d = 16 mt + g (+8), heads 8 nt + 2c, +1)
+  float me[NT], mo[NT], le[NT], lo[NT];  // running max / sum of heads 8 nt + 2c and + 1
+  int q = 0;
 
   for (int it = 0; it < niters; ++it) {
+    walk.enter(it);
     const int s = it % kStages;
     const int use = it / kStages;
-    const int pc = s_pstart[h + 1] - s_pstart[h];
-    const int nvalid = min(kPageTokens, s_cnt[h] - pg * kPageTokens);
-    const bool seg_start = (it == 0) || (pg == 0);
-    const bool seg_end = (it == niters - 1) || (pg == pc - 1);
+    const int nvalid = min(kPageTokens, s_cnt[walk.h] - walk.pg * kPageTokens);
+    const bool seg_start = walk.seg_start(it);
+    const bool seg_end = walk.seg_end(it, niters);
     uint8_t* st = stages + s * kStageBytes;
     mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
 
     if (seg_start) {
       const uint32_t qbase = smem_addr(st + 2 * kHalfPageBytes);
-      const int mi = lane >> 3;
-      const int row = (mi & 1) * 8 + (lane & 7);
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const int chunk = 2 * kk + (mi >> 1);
-        ldsm_x4(qbase + row * kRowBytes + chunk * 16, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
-        if (g >= G) { qa[kk][0] = 0u; qa[kk][2] = 0u; }
-        if (g + 8 >= G) { qa[kk][1] = 0u; qa[kk][3] = 0u; }
+      for (int nt = 0; nt < NT; ++nt) {
+        const int row = 8 * nt + (lane & 7);
+#pragma unroll
+        for (int k2 = 0; k2 < 4; ++k2) {
+          const int kk = 2 * k2 + (mi >> 1);
+          uint32_t r0, r1, r2, r3;
+          ldsm_x4(qbase + row * kRowBytes + (2 * kk + (mi & 1)) * 16, r0, r1, r2, r3);
+          const bool live = 8 * nt + g < G;
+          qb[2 * k2][nt][0] = live ? r0 : 0u;
+          qb[2 * k2][nt][1] = live ? r1 : 0u;
+          qb[2 * k2 + 1][nt][0] = live ? r2 : 0u;
+          qb[2 * k2 + 1][nt][1] = live ? r3 : 0u;
+        }
+        me[nt] = mo[nt] = -INFINITY;
+        le[nt] = lo[nt] = 0.f;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
       }
-#pragma unroll
-      for (int j = 0; j < 16; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
-      m0 = m1 = -INFINITY;
-      l0 = l1 = 0.f;
     }
 
     if (tb < nvalid) {
-      // ---- S = Q K^T for tokens tb .. tb+15 (two n8 tiles)
-      float sc[2][4];
+      // ---- S^T = K Q^T for tokens tb .. tb+15: two independent chains over k
+      float sa[NT][4], sb[NT][4];
 #pragma unroll
-      for (int nt = 0; nt < 2; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sa[nt][e] = sb[nt][e] = 0.f;
       const uint32_t kbase = smem_addr(st);
       {
-        const int mi = lane >> 3;
-        const uint32_t row = (uint32_t)(tb + (mi >> 1) * 8 + (lane & 7));
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          uint32_t b00, b01, b10, b11;
-          ldsm_x4(kbase + swizzled_offset(row, (uint32_t)(2 * kk + (mi & 1))), b00, b01, b10, b11);
-          mma_bf16_16816(sc[0], qa[kk], b00, b01);
-          mma_bf16_16816(sc[1], qa[kk], b10, b11);
-        }
-      }
-      // ---- mask tokens past n_valid, online softmax (exp2 domain)
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int t = tb + nt * 8 + 2 * c4 + (e & 1);
-          sc[nt][e] = (t < nvalid) ? sc[nt][e] * p.scale_log2 : -INFINITY;
-        }
-      float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][1]), fmaxf(sc[1][0], sc[1][1]));
-      float mx1 = fmaxf(fmaxf(sc[0][2], sc[0][3]), fmaxf(sc[1][2], sc[1][3]));
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-      const float corr0 = exp2f(m0 - mn0), corr1 = exp2f(m1 - mn1);
-      m0 = mn0;
-      m1 = mn1;
-      float pr[2][4];
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-        pr[nt][0] = exp2f(sc[nt][0] - mn0);
-        pr[nt][1] = exp2f(sc[nt][1] - mn0);
-        pr[nt][2] = exp2f(sc[nt][2] - mn1);
-        pr[nt][3] = exp2f(sc[nt][3] - mn1);
-      }
-      l0 = l0 * corr0 + (pr[0][0] + pr[0][1]) + (pr[1][0] + pr[1][1]);
-      l1 = l1 * corr1 + (pr[0][2] + pr[0][3]) + (pr[1][2] + pr[1][3]);
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        o[j][0] *= corr0;
-        o[j][1] *= corr0;
-        o[j][2] *= corr1;
-        o[j][3] *= corr1;
-      }
-      uint32_t pa[4];
-      pa[0] = pack_bf16x2(pr[0][0], pr[0][1]);
-      pa[1] = pack_bf16x2(pr[0][2], pr[0][3]);
-      pa[2] = pack_bf16x2(pr[1][0], pr[1][1]);
-      pa[3] = pack_bf16x2(pr[1][2], pr[1][3]);
-
-      // ---- O += P V (16 n8 tiles over head_dim)
-      const uint32_t vbase = smem_addr(st + kHalfPageBytes);
-      const bool partial = tb + 16 > nvalid;
-      uint32_t mk0 = 0xffffffffu, mk1 = 0xffffffffu;
-      if (partial) {
-        const int t = tb + 2 * c4;
-        mk0 = (t < nvalid ? 0x0000ffffu : 0u) | (t + 1 < nvalid ? 0xffff0000u : 0u);
-        mk1 = (t + 8 < nvalid ? 0x0000ffffu : 0u) | (t + 9 < nvalid ? 0xffff0000u : 0u);
-      }
-      {
-        const int mi = lane >> 3;
         const uint32_t row = (uint32_t)(tb + (mi & 1) * 8 + (lane & 7));
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
-          uint32_t v0, v1, v2, v3;
-          ldsm_x4_trans(vbase + swizzled_offset(row, (uint32_t)(2 * jj + (mi >> 1))), v0, v1, v2,
-                        v3);
-          v0 &= mk0;
-          v1 &= mk1;
-          v2 &= mk0;
-          v3 &= mk1;
-          mma_bf16_16816(o[2 * jj], pa, v0, v1);
-          mma_bf16_16816(o[2 * jj + 1], pa, v2, v3);
+        for (int kk = 0; kk < 8; ++kk) {
+          uint32_t a[4];
+          ldsm_x4(kbase + swizzled_offset(row, (uint32_t)(2 * kk + (mi >> 1))), a[0], a[1], a[2], a[3]);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            if (kk & 1) mma_bf16_16816(sb[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
+            else mma_bf16_16816(sa[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
+          }
+        }
+      }
+      // ---- mask tokens past n_valid, online softmax per head (column), P^T fragments
+      const bool v0 = tb + g < nvalid, v1 = tb + g + 8 < nvalid;
+      bool rescale = false;
+      float ce[NT], co[NT];
+      uint32_t pb[NT][2];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        const float s0 = v0 ? (sa[nt][0] + sb[nt][0]) * p.scale_log2 : -INFINITY;
+        const float s1 = v0 ? (sa[nt][1] + sb[nt][1]) * p.scale_log2 : -INFINITY;
+        const float s2 = v1 ? (sa[nt][2] + sb[nt][2]) * p.scale_log2 : -INFINITY;
+        const float s3 = v1 ? (sa[nt][3] + sb[nt][3]) * p.scale_log2 : -INFINITY;
+        float xe = fmaxf(s0, s2), xo = fmaxf(s1, s3);
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+          xe = fmaxf(xe, __shfl_xor_sync(0xffffffffu, xe, off));
+          xo = fmaxf(xo, __shfl_xor_sync(0xffffffffu, xo, off));
+        }
+        const float ne = fmaxf(me[nt], xe), no = fmaxf(mo[nt], xo);
+        ce[nt] = exp2f(me[nt] - ne);
+        co[nt] = exp2f(mo[nt] - no);
+        me[nt] = ne;
+        mo[nt] = no;
+        const float p0 = exp2f(s0 - ne), p1 = exp2f(s1 - no);
+        const float p2 = exp2f(s2 - ne), p3 = exp2f(s3 - no);
+        le[nt] = le[nt] * ce[nt] + (p0 + p2);
+        lo[nt] = lo[nt] * co[nt] + (p1 + p3);
+        rescale |= (ce[nt] != 1.f) || (co[nt] != 1.f);
+        // (token g, heads 2c..) -> transpose -> (head g, tokens 2c..): the B operand
+        pb[nt][0] = movmatrix_trans(pack_bf16x2(p0, p1));
+        pb[nt][1] = movmatrix_trans(pack_bf16x2(p2, p3));
+      }
+      if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            o[mt][nt][0] *= ce[nt];
+            o[mt][nt][1] *= co[nt];
+            o[mt][nt][2] *= ce[nt];
+            o[mt][nt][3] *= co[nt];
+          }
+      }
+      // ---- O^T += V^T P^T over head_dim (8 m-tiles of 16)
+      const uint32_t vbase = smem_addr(st + kHalfPageBytes);
+      uint32_t mk_lo = 0xffffffffu, mk_hi = 0xffffffffu;
+      if (tb + 16 > nvalid) {  // stale rows past n_valid must not reach the tensor cores
+        const int t = tb + 2 * c4;
+        mk_lo = (t < nvalid ? 0x0000ffffu : 0u) | (t + 1 < nvalid ? 0xffff0000u : 0u);
+        mk_hi = (t + 8 < nvalid ? 0x0000ffffu : 0u) | (t + 9 < nvalid ? 0xffff0000u : 0u);
+      }
+      {
+        const uint32_t row = (uint32_t)(tb + (mi >> 1) * 8 + (lane & 7));
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          uint32_t a[4];
+          ldsm_x4_trans(vbase + swizzled_offset(row, (uint32_t)(2 * mt + (mi & 1))), a[0], a[1], a[2],
+                        a[3]);
+          a[0] &= mk_lo;
+          a[1] &= mk_lo;
+          a[2] &= mk_hi;
+          a[3] &= mk_hi;
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(o[mt][nt], a, pb[nt][0], pb[nt][1]);
         }
       }
     }
@@ -424,92 +638,43 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tiled_kernel(const DecodeP
     if (lane == 0) mbar_arrive(&empty_bar[s]);
 
     if (seg_end) {
-      // ---- merge the four warp states of this head segment
-      float lt0 = l0 + __shfl_xor_sync(0xffffffffu, l0, 1);
-      lt0 += __shfl_xor_sync(0xffffffffu, lt0, 2);
-      float lt1 = l1 + __shfl_xor_sync(0xffffffffu, l1, 1);
-      lt1 += __shfl_xor_sync(0xffffffffu, lt1, 2);
-      if (c4 == 0) {
-        merge_m[warp * kMaxGroup + g] = m0;
-        merge_m[warp * kMaxGroup + g + 8] = m1;
-        merge_l[warp * kMaxGroup + g] = lt0;
-        merge_l[warp * kMaxGroup + g + 8] = lt1;
-      }
-      float* mo = merge_o + warp * kMaxGroup * kHeadDim;
+      // ---- hand this warp's partial (m, l, O^T) of the segment to the epilogue warp
+      const int slot = q % PL::kSlots;
+      if (q >= PL::kSlots) mbar_wait(&mempty_bar[slot], ((q / PL::kSlots) - 1) & 1, abort_flag, p.ctrl);
+      float* so = merge_o + slot * PL::kSlotOFloats + warp * HP * kMergeRow;
+      float* sml = merge_ml + slot * PL::kSlotMLFloats + warp * HP * 2;
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        *reinterpret_cast<float2*>(mo + g * kHeadDim + 8 * j + 2 * c4) = make_float2(o[j][0], o[j][1]);
-        *reinterpret_cast<float2*>(mo + (g + 8) * kHeadDim + 8 * j + 2 * c4) =
-            make_float2(o[j][2], o[j][3]);
-      }
-      named_barrier_consumers();
-
-      const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
-      const int64_t first = s_pstart[h], last = s_pstart[h] + pc - 1;
-      const int k_lo = cta_of_page(first, P, N), k_hi = cta_of_page(last, P, N);
-      const bool single = (k_lo == k_hi);
-      __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
-      float* rec = p.pieces + (int64_t)(k + h) * kPieceFloats;  // m[16] l[16] o[16][128]
-      const int d = tid;  // 0..127
-      for (int r = 0; r < G; ++r) {
-        float M = merge_m[r];
+      for (int nt = 0; nt < NT; ++nt) {
+        float te = le[nt], to = lo[nt];
 #pragma unroll
-        for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, merge_m[w * kMaxGroup + r]);
-        float L = 0.f, O = 0.f;
+        for (int off = 4; off < 32; off <<= 1) {
+          te += __shfl_xor_sync(0xffffffffu, te, off);
+          to += __shfl_xor_sync(0xffffffffu, to, off);
+        }
+        const int he = 8 * nt + 2 * c4, ho = he + 1;
+        if (g == 0) {
+          sml[he * 2] = me[nt];
+          sml[he * 2 + 1] = te;
+          sml[ho * 2] = mo[nt];
+          sml[ho * 2 + 1] = to;
+        }
 #pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) {
-          const float wt = exp2f(merge_m[w * kMaxGroup + r] - M);
-          L += wt * merge_l[w * kMaxGroup + r];
-          O += wt * merge_o[(w * kMaxGroup + r) * kHeadDim + d];
-        }
-        if (single) {
-          out_h[r * kHeadDim + d] = __float2bfloat16_rn(O / L);
-        } else {
-          rec[2 * kMaxGroup + r * kHeadDim + d] = O;
-          if (d == 0) {
-            rec[r] = M;
-            rec[kMaxGroup + r] = L;
-          }
+        for (int mt = 0; mt < 8; ++mt) {
+          so[he * kMergeRow + 16 * mt + g] = o[mt][nt][0];
+          so[ho * kMergeRow + 16 * mt + g] = o[mt][nt][1];
+          so[he * kMergeRow + 16 * mt + g + 8] = o[mt][nt][2];
+          so[ho * kMergeRow + 16 * mt + g + 8] = o[mt][nt][3];
         }
       }
-      if (!single) {
-        __threadfence();
-        named_barrier_consumers();
-        if (tid == 0) {
-          const int prev = atomicAdd(p.piece_counters + h, 1);
-          s_misc[1] = (prev == k_hi - k_lo) ? 1 : 0;
-        }
-        named_barrier_consumers();
-        if (s_misc[1]) {
-          // Last CTA of this head: log-sum-exp merge of all records, in CTA order.
-          __threadfence();
-          for (int r = 0; r < G; ++r) {
-            float M = -INFINITY;
-            for (int kk = k_lo; kk <= k_hi; ++kk)
-              M = fmaxf(M, __ldcg(p.pieces + (int64_t)(kk + h) * kPieceFloats + r));
-            float L = 0.f, O = 0.f;
-            for (int kk = k_lo; kk <= k_hi; ++kk) {
-              const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
-              const float wt = exp2f(__ldcg(rk + r) - M);
-              L += wt * __ldcg(rk + kMaxGroup + r);
-              O += wt * __ldcg(rk + 2 * kMaxGroup + r * kHeadDim + d);
-            }
-            out_h[r * kHeadDim + d] = __float2bfloat16_rn(O / L);
-          }
-          if (tid == 0) p.piece_counters[h] = 0;
-        }
-      }
-      named_barrier_consumers();  // merge buffers are reused by the next segment
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&mfull_bar[slot]);
+      ++q;
     }
-
-    // ---- advance to the next page of the flat list
-    if (++pg == pc) {
-      pg = 0;
-      do { ++h; } while (h < heads && s_pstart[h + 1] == s_pstart[h]);
-      if (h >= heads) h = heads - 1;  // only reached after the last iteration
-    }
+    walk.advance();
   }
 }
+
+// ---------------------------------------------------------------- simple kernel
 
 // ---------------------------------------------------------------- simple kernel
 
@@ -566,9 +731,46 @@ cudaError_t prepare_decode(const Cache& c) {
   (void)c;
   // Sized for the largest head count any cache may have, so that caches of
   // different sizes never lower the limit under one another.
-  return cudaFuncSetAttribute(decode_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)tiled_smem_bytes(kMaxHeads));
+  cudaError_t e = cudaSuccess;
+  auto set = [&](auto kernel, size_t bytes) {
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  };
+  set(decode_tiled_kernel<kStagesOneCta, 1>, tiled_smem_bytes<1>(kMaxHeads, kStagesOneCta));
+  set(decode_tiled_kernel<kStagesOneCta, 2>, tiled_smem_bytes<2>(kMaxHeads, kStagesOneCta));
+  set(decode_tiled_kernel<kStagesTwoCta, 1>, tiled_smem_bytes<1>(kMaxHeads, kStagesTwoCta));
+  set(decode_tiled_kernel<kStagesTwoCta, 2>, tiled_smem_bytes<2>(kMaxHeads, kStagesTwoCta));
+  return e;
 }
+
+namespace {
+
+// Launch with programmatic stream serialisation (the kernel waits for its
+// prerequisites itself); the variant is picked by CTAs per SM and group size.
+cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cudaStream_t stream,
+                         bool programmatic) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.blockDim = dim3(kThreads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = programmatic ? 1 : 0;
+  const bool two = ctas_per_sm >= 2;
+  const int stages = two ? kStagesTwoCta : kStagesOneCta;
+  cfg.gridDim = dim3(num_sms * (two ? ctas_per_sm : 1));
+  if (p.group <= 8) {
+    cfg.dynamicSmemBytes = tiled_smem_bytes<1>(p.heads, stages);
+    return two ? cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesTwoCta, 1>, p)
+               : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 1>, p);
+  }
+  cfg.dynamicSmemBytes = tiled_smem_bytes<2>(p.heads, stages);
+  return two ? cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesTwoCta, 2>, p)
+             : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 2>, p);
+}
+
+}  // namespace
 
 cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, void* out,
                                 int32_t group, float scale_log2, cudaStream_t stream) {
@@ -587,9 +789,7 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
   p.max_pages = c.max_pages;
   p.min_pages = c.min_pages_per_cta;
   p.scale_log2 = scale_log2;
-  const int grid = c.num_sms * c.ctas_per_sm;
-  decode_tiled_kernel<<<grid, kThreads, tiled_smem_bytes(c.heads), stream>>>(p);
-  return cudaGetLastError();
+  return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true);
 }
 
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
@@ -672,8 +872,7 @@ extern "C" dms_status dms_decode_attention_paged_noalloc(
       }
       int sms = 0;
       if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-          cudaFuncSetAttribute(decode_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)tiled_smem_bytes(kMaxHeads)) != cudaSuccess) {
+          prepare_decode(Cache()) != cudaSuccess) {
         cudaGetLastError();
         return DMS_ERR_CUDA;
       }
@@ -711,6 +910,5 @@ extern "C" dms_status dms_decode_attention_paged_noalloc(
   p.min_pages = 2;
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)kHeadDim);
   p.scale_log2 = scale * 1.4426950408889634f;
-  decode_tiled_kernel<<<grid, kThreads, tiled_smem_bytes((int)heads), s>>>(p);
-  return cudaGetLastError() == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+  return launch_tiled(p, grid, 1, s, false) == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
 }
