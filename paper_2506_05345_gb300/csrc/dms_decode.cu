@@ -184,6 +184,11 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
+// Four consecutive bf16 outputs (round to nearest even) with one 8-byte store.
+__device__ __forceinline__ void store_bf16x4(__nv_bfloat16* dst, float a, float b, float c, float d) {
+  *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(a, b), pack_bf16x2(c, d));
+}
+
 // Programmatic dependent launch: let the next kernel of the stream start its
 // prologue now; wait until the previous kernel's results are visible.  Both are
 // no-ops when the launches carry no programmatic dependency.
@@ -416,29 +421,33 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
         const bool single = (k_lo == k_hi);
         __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
         float* rec = p.pieces + (int64_t)(k + h) * kPieceFloats;  // m[16] l[16] o[16][128]
+        // Lane owns head_dim columns 4 lane .. 4 lane + 3 (128-bit loads / stores).
+        const int d4 = 4 * lane;
         for (int r = 0; r < G; ++r) {
           float M = sml[(0 * HP + r) * 2];
 #pragma unroll
           for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, sml[(w * HP + r) * 2]);
-          float wt[kConsumerWarps];
           float L = 0.f;
+          float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
           for (int w = 0; w < kConsumerWarps; ++w) {
-            wt[w] = exp2f(sml[(w * HP + r) * 2] - M);
-            L += wt[w] * sml[(w * HP + r) * 2 + 1];
+            const float wt = exp2f(sml[(w * HP + r) * 2] - M);
+            L += wt * sml[(w * HP + r) * 2 + 1];
+            const float4 x = *reinterpret_cast<const float4*>(so + (w * HP + r) * kMergeRow + d4);
+            O.x += wt * x.x;
+            O.y += wt * x.y;
+            O.z += wt * x.z;
+            O.w += wt * x.w;
           }
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int d = lane + 32 * i;
-            float O = 0.f;
-#pragma unroll
-            for (int w = 0; w < kConsumerWarps; ++w) O += wt[w] * so[(w * HP + r) * kMergeRow + d];
-            if (single) out_h[r * kHeadDim + d] = __float2bfloat16_rn(O / L);
-            else rec[2 * kMaxGroup + r * kHeadDim + d] = O;
-          }
-          if (!single && lane == 0) {
-            rec[r] = M;
-            rec[kMaxGroup + r] = L;
+          if (single) {
+            const float inv = 1.f / L;
+            store_bf16x4(out_h + r * kHeadDim + d4, O.x * inv, O.y * inv, O.z * inv, O.w * inv);
+          } else {
+            *reinterpret_cast<float4*>(rec + 2 * kMaxGroup + r * kHeadDim + d4) = O;
+            if (lane == 0) {
+              rec[r] = M;
+              rec[kMaxGroup + r] = L;
+            }
           }
         }
         __syncwarp();
@@ -455,25 +464,25 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
             // rows is issued together.
             __threadfence();
             for (int r0 = 0; r0 < G; r0 += 8) {
-              float Mr[8], Lr[8], Or[8][4];
+              float Mr[8], Lr[8];
+              float4 Or[8];
 #pragma unroll
               for (int r = 0; r < 8; ++r) {
                 Mr[r] = -INFINITY;
                 Lr[r] = 0.f;
-#pragma unroll
-                for (int i = 0; i < 4; ++i) Or[r][i] = 0.f;
+                Or[r] = make_float4(0.f, 0.f, 0.f, 0.f);
               }
               for (int kk = k_lo; kk <= k_hi; ++kk) {
                 const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
-                float mk[8], lk[8], ok[8][4];
+                float mk[8], lk[8];
+                float4 ok[8];
 #pragma unroll
                 for (int r = 0; r < 8; ++r) {
                   if (r0 + r < G) {
                     mk[r] = __ldcg(rk + r0 + r);
                     lk[r] = __ldcg(rk + kMaxGroup + r0 + r);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                      ok[r][i] = __ldcg(rk + 2 * kMaxGroup + (r0 + r) * kHeadDim + lane + 32 * i);
+                    ok[r] = __ldcg(reinterpret_cast<const float4*>(rk + 2 * kMaxGroup +
+                                                                   (r0 + r) * kHeadDim + d4));
                   }
                 }
 #pragma unroll
@@ -482,18 +491,22 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
                     const float Mn = fmaxf(Mr[r], mk[r]);
                     const float a = exp2f(Mr[r] - Mn), bw = exp2f(mk[r] - Mn);
                     Lr[r] = Lr[r] * a + lk[r] * bw;
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) Or[r][i] = Or[r][i] * a + ok[r][i] * bw;
+                    Or[r].x = Or[r].x * a + ok[r].x * bw;
+                    Or[r].y = Or[r].y * a + ok[r].y * bw;
+                    Or[r].z = Or[r].z * a + ok[r].z * bw;
+                    Or[r].w = Or[r].w * a + ok[r].w * bw;
                     Mr[r] = Mn;
                   }
                 }
               }
 #pragma unroll
-              for (int r = 0; r < 8; ++r)
-                if (r0 + r < G)
-#pragma unroll
-                  for (int i = 0; i < 4; ++i)
-                    out_h[(r0 + r) * kHeadDim + lane + 32 * i] = __float2bfloat16_rn(Or[r][i] / Lr[r]);
+              for (int r = 0; r < 8; ++r) {
+                if (r0 + r < G) {
+                  const float inv = 1.f / Lr[r];
+                  store_bf16x4(out_h + (r0 + r) * kHeadDim + d4, Or[r].x * inv, Or[r].y * inv,
+                               Or[r].z * inv, Or[r].w * inv);
+                }
+              }
             }
             if (lane == 0) p.piece_counters[h] = 0;
           }
