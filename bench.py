@@ -55,6 +55,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--ctas-per-sm", type=int, default=0)
     ap.add_argument("--min-pages", type=int, default=0)
+    ap.add_argument("--separate", action="store_true",
+                    help="append and decode as two launches instead of the fused step")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (small cases for profiling)")
     return ap.parse_args()
@@ -265,6 +267,13 @@ def run_ours(args, wl, world, rank, local, pg):
     def do_step(s, timed_idx=None):
         for layer in range(L):
             k, v, lg, q = ins[s][layer]
+            if not args.separate:  # one launch: single-token append fused into the decode
+                if timed_idx is not None:
+                    ev_dec[timed_idx][layer][0].record(stream)
+                cache.append_and_decode(layer, k, v, lg, q, outs[layer], gqa_group=G)
+                if timed_idx is not None:
+                    ev_dec[timed_idx][layer][1].record(stream)
+                continue
             if timed_idx is not None:
                 ev_app[timed_idx][layer][0].record(stream)
             cache.append_and_evict(layer, k, v, lg)
@@ -314,8 +323,8 @@ def run_ours(args, wl, world, rank, local, pg):
     tokens_read = K_ * 0.5 * (tok_first + tok_last)
     dec_ms = [ev_dec[i][layer][0].elapsed_time(ev_dec[i][layer][1])
               for i in range(K2) for layer in range(L)]
-    app_ms = [ev_app[i][layer][0].elapsed_time(ev_app[i][layer][1])
-              for i in range(K2) for layer in range(L)]
+    app_ms = ([ev_app[i][layer][0].elapsed_time(ev_app[i][layer][1])
+               for i in range(K2) for layer in range(L)] if args.separate else [0.0])
     units_per_launch = 0.5 * (tok_last + st_k2["total_retained"]) / L
     bytes_per_unit = workloads.kv_bytes_per_token_head(D)
     dec_avg_s = float(np.mean(dec_ms)) * 1e-3
@@ -396,8 +405,12 @@ def run_ours(args, wl, world, rank, local, pg):
                 dv[layer].copy_(v, non_blocking=True)
                 dl[layer].copy_(lg, non_blocking=True)
                 dq[layer].copy_(q, non_blocking=True)
-                cache.append_and_evict(layer, dk[layer], dv[layer], dl[layer])
-                cache.decode_attention(layer, dq[layer], outs[layer], gqa_group=G)
+                if args.separate:
+                    cache.append_and_evict(layer, dk[layer], dv[layer], dl[layer])
+                    cache.decode_attention(layer, dq[layer], outs[layer], gqa_group=G)
+                else:
+                    cache.append_and_decode(layer, dk[layer], dv[layer], dl[layer], dq[layer],
+                                            outs[layer], gqa_group=G)
                 host_out[layer].copy_(outs[layer], non_blocking=True)
 
         for s in range(E_W):
@@ -440,19 +453,22 @@ def run_ours(args, wl, world, rank, local, pg):
                          f"{units_per_launch * bytes_per_unit / 1e6:.0f} MB x {L} layers rotate, "
                          "larger than the 129 MB L2",
                    "parallelism": f"replicas x{world}"},
+        "step_mode": "separate append + decode launches" if args.separate else
+                     "fused single-token append + decode, one launch per layer",
         "decode_us_per_layer_step": float(np.mean(dec_ms)) * 1e3,
-        "append_us_per_layer_step": float(np.mean(app_ms)) * 1e3,
+        "append_us_per_layer_step": (float(np.mean(app_ms)) * 1e3 if args.separate else None),
         "retained_tokens_per_layer_step": units_per_launch,
         "compression": (wl.prefill_tokens + n_dev_steps) * B * H / units_per_launch,
         "hbm_frac_of_nominal_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
-        "roofline": {"kernel": "decode_tiled_kernel", "bound": "hbm", "achieved": achieved_gbs,
+        "roofline": {"kernel": "decode_tiled_kernel" + ("" if args.separate else " (append fused)"),
+                     "bound": "hbm", "achieved": achieved_gbs,
                      "peak": peak, "unit": "GB/s", "frac": achieved_gbs / peak,
                      "peak_kind": f"{peak_kind} copy bandwidth",
                      "traffic": traffic,
                      "algorithmic_bytes_per_launch": units_per_launch * bytes_per_unit},
         "cpu_baseline": cpu_baseline,
         "e2e": e2e,
-        "gpu_launches": 2 * L * K_,
+        "gpu_launches": (2 if args.separate else 1) * L * K_,
         "clocks": clk,
         "parity_sample": parity,
         "setup_s": time.time() - t_setup,

@@ -98,7 +98,7 @@ typedef struct dms_stats {
  * pool, page tables, per-head counts, decision rings and decode scratch, and
  * zeroes the counts.  On success *out receives the cache; on failure *out is
  * NULL and nothing stays allocated.  Limits: batch * kv_heads <= 4096,
- * capacity < 2^31.
+ * capacity < 2^30.
  */
 dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim,
                             int32_t window, int64_t capacity, const dms_options* opt,
@@ -140,6 +140,20 @@ dms_status dms_append_and_evict(dms_cache* cache, int32_t layer, const void* k,
  */
 dms_status dms_decode_attention(dms_cache* cache, int32_t layer, const void* q, void* out,
                                 int32_t gqa_group, float sm_scale, void* stream);
+
+/*
+ * One decode step of one layer in a single launch: exactly
+ * dms_append_and_evict(cache, layer, k, v, decision_logit, 1, stream) followed by
+ * dms_decode_attention(cache, layer, q, out, gqa_group, sm_scale, stream), with
+ * the same arguments, layouts and results (n_tokens = 1: k, v are
+ * [batch, 1, kv_heads, 128] bf16, decision_logit [batch, 1, kv_heads] bf16).
+ * The single-token append is fused into the tiled decode kernel; when the fused
+ * kernel does not apply (decode_kernel = DMS_DECODE_SIMPLE, ctas_per_sm >= 2, or
+ * batch * kv_heads > 4000) the two separate kernels run instead.
+ */
+dms_status dms_append_and_decode(dms_cache* cache, int32_t layer, const void* k, const void* v,
+                                 const void* decision_logit, const void* q, void* out,
+                                 int32_t gqa_group, float sm_scale, void* stream);
 
 /*
  * Synchronise `stream`, then report totals into *out (non-NULL) and, if

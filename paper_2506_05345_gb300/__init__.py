@@ -73,6 +73,12 @@ def dms_decode_attention(cache, layer, q_ptr, out_ptr, gqa_group, sm_scale, stre
                                           float(sm_scale), stream)
 
 
+def dms_append_and_decode(cache, layer, k_ptr, v_ptr, logit_ptr, q_ptr, out_ptr, gqa_group,
+                          sm_scale, stream):
+    return library().dms_append_and_decode(cache, layer, k_ptr, v_ptr, logit_ptr, q_ptr, out_ptr,
+                                           gqa_group, float(sm_scale), stream)
+
+
 def dms_cache_stats(cache, stats: dms_stats, counts_ptr, stream):
     return library().dms_cache_stats(cache, ctypes.byref(stats), counts_ptr, stream)
 
@@ -181,6 +187,24 @@ class DmsCache:
         op = _bf16_cuda(out, (B, H * gqa_group, D), "out")
         _check(dms_decode_attention(self._h, layer, qp, op, gqa_group, sm_scale,
                                     _stream_ptr(stream)), "dms_decode_attention")
+        return out
+
+    def append_and_decode(self, layer: int, k, v, decision_logit, q, out=None,
+                          gqa_group: int | None = None, sm_scale: float = 0.0, stream=None):
+        """One decode step of one layer (single-token append + decode in one launch)."""
+        import torch
+        B, H, D = self.batch, self.kv_heads, self.head_dim
+        if gqa_group is None:
+            gqa_group = q.shape[1] // H
+        if out is None:
+            out = torch.empty_like(q)
+        kp = _bf16_cuda(k, (B, 1, H, D), "k")
+        vp = _bf16_cuda(v, (B, 1, H, D), "v")
+        lp = _bf16_cuda(decision_logit, (B, 1, H), "decision_logit")
+        qp = _bf16_cuda(q, (B, H * gqa_group, D), "q")
+        op = _bf16_cuda(out, (B, H * gqa_group, D), "out")
+        _check(dms_append_and_decode(self._h, layer, kp, vp, lp, qp, op, gqa_group, sm_scale,
+                                     _stream_ptr(stream)), "dms_append_and_decode")
         return out
 
     def stats(self, stream=None, with_counts: bool = False):

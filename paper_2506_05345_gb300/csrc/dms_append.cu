@@ -25,7 +25,8 @@ struct AppendParams {
   uint8_t* pool;
   int32_t* pos;
   int32_t* page_table;  // this layer: [heads][max_pages]
-  int32_t* counts;      // this layer: [heads]
+  const int32_t* counts_cur;  // this layer, current buffer: [heads]
+  int32_t* counts_next;       // this layer, buffer after the append: [heads]
   uint32_t* ring;       // this layer: [heads][ring_len]
   int32_t* ctrl;
   int32_t* freed;       // [heads][ring_len]
@@ -70,15 +71,14 @@ __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
   int32_t slot = 0, page = 0, ok = 1;
   if (lane == 0) {
     const int64_t j = p.t0;
-    const int64_t R = p.window + 1;
+    const int64_t R = p.window + 1, RP = ring_period(p.window);
     const uint32_t alpha = decision_from_bf16(p.logit[(int64_t)b * p.kv_heads + hk]);
     uint32_t* ring = p.ring + (int64_t)bh * p.ring_len;
     int32_t* pt = p.page_table + (int64_t)bh * p.max_pages;
-    int32_t n = p.counts[bh];
+    int32_t n = p.counts_cur[bh];
     slot = -1;
-    const int32_t ridx = (int32_t)(j % R);
     if (j >= R) {  // token j - window - 1 leaves the window now
-      const uint32_t e = ring[ridx];
+      const uint32_t e = ring[(j - R) % RP];
       if (e & kAlphaBit) slot = (int32_t)(e & kSlotMask);  // evicted: reuse its slot
     }
     if (slot < 0) {
@@ -94,9 +94,9 @@ __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
       }
       n += ok;
     }
+    p.counts_next[bh] = n;  // unchanged if the page pool ran out
     if (ok) {
-      ring[ridx] = (uint32_t)slot | (alpha << 31);
-      p.counts[bh] = n;
+      ring[j % RP] = (uint32_t)slot | (alpha << 31);
       page = pt[slot / kPageTokens];
       p.pos[(int64_t)page * kPageTokens + (slot & (kPageTokens - 1))] = (int32_t)j;
     }
@@ -141,11 +141,11 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int bh = blockIdx.x;
   const int b = bh / p.kv_heads, hk = bh - b * p.kv_heads;
-  const int64_t R = p.window + 1, t0 = p.t0, n = p.n;
+  const int64_t R = p.window + 1, RP = ring_period(p.window), t0 = p.t0, n = p.n;
   uint32_t* ring = p.ring + (int64_t)bh * p.ring_len;
   int32_t* F = p.freed + (int64_t)bh * p.ring_len;
   int32_t* pt = p.page_table + (int64_t)bh * p.max_pages;
-  const int32_t nh = p.counts[bh];
+  const int32_t nh = p.counts_cur[bh];
 
   // 1. Old tokens leaving the window during this call: positions [lo, hi], all < t0.
   const int64_t lo = t0 - R > 0 ? t0 - R : 0;
@@ -156,7 +156,7 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
     int flag = 0;
     uint32_t e = 0;
     if (base + tid < len_old) {
-      e = ring[(lo + base + tid) % R];
+      e = ring[(lo + base + tid) % RP];
       flag = (e & kAlphaBit) ? 1 : 0;
     }
     int total;
@@ -197,7 +197,10 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
     s_misc[1] = ok;
   }
   __syncthreads();
-  if (!s_misc[1]) return;
+  if (!s_misc[1]) {  // page pool ran out: the head keeps its state
+    if (tid == 0) p.counts_next[bh] = nh;
+    return;
+  }
   for (int i = tid; i < add; i += kBulkThreads) pt[old_pages + i] = s_misc[0] + i;
   __syncthreads();
 
@@ -217,7 +220,7 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
       slot = rank < nf ? F[rank] : (int32_t)(nh + (rank - nf));
     }
     s_slot[tid] = slot;
-    if (valid && li >= n - R) ring[(t0 + li) % R] = (uint32_t)slot | (alpha << 31);
+    if (valid && li >= n - R) ring[(t0 + li) % RP] = (uint32_t)slot | (alpha << 31);
     kept_before += total;
     __syncthreads();
     // Each warp moves 4 rows at a time (loads first, then stores).
@@ -245,7 +248,7 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
     }
     __syncthreads();
   }
-  if (tid == 0) p.counts[bh] = (int32_t)new_n;
+  if (tid == 0) p.counts_next[bh] = (int32_t)new_n;
 }
 
 __global__ void export_positions_kernel(const int32_t* counts, const int32_t* page_table,
@@ -268,7 +271,8 @@ AppendParams make_params(const Cache& c, int32_t layer, const void* k, const voi
   p.pool = c.pool;
   p.pos = c.pos;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
-  p.counts = c.counts + (int64_t)layer * c.heads;
+  p.counts_cur = c.counts_at(layer, t0);
+  p.counts_next = c.counts_at(layer, t0 + n);
   p.ring = c.rings + (int64_t)layer * c.heads * c.ring_len;
   p.ctrl = c.ctrl;
   p.freed = c.freed;
@@ -314,7 +318,7 @@ cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, con
 cudaError_t launch_export_positions(const Cache& c, int32_t layer, int32_t* dev_out,
                                     cudaStream_t stream) {
   export_positions_kernel<<<c.heads, 256, 0, stream>>>(
-      c.counts + (int64_t)layer * c.heads, c.page_table + (int64_t)layer * c.heads * c.max_pages,
+      c.counts_at(layer, c.lengths[layer]), c.page_table + (int64_t)layer * c.heads * c.max_pages,
       c.pos, c.max_pages, c.capacity, dev_out);
   return cudaGetLastError();
 }

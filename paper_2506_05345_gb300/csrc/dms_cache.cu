@@ -63,7 +63,7 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   if (out == nullptr) return DMS_ERR_INVALID_ARGUMENT;
   *out = nullptr;
   if (opt == nullptr || layers < 1 || kv_heads < 1 || head_dim != dms::kHeadDim || window < 0 ||
-      capacity < 1 || capacity > 0x7fffffffLL || opt->batch < 1)
+      capacity < 1 || capacity > dms::kMaxCapacity || opt->batch < 1)
     return DMS_ERR_INVALID_ARGUMENT;
   if (opt->page_tokens != 0 && opt->page_tokens != dms::kPageTokens) return DMS_ERR_INVALID_ARGUMENT;
   if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SIMPLE ||
@@ -84,7 +84,7 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   c.batch = opt->batch;
   c.capacity = capacity;
   c.heads = (int32_t)heads;
-  c.ring_len = (int32_t)std::min<int64_t>((int64_t)window + 1, capacity);
+  c.ring_len = (int32_t)std::min<int64_t>(dms::ring_period(window), capacity);
   c.max_pages = (int32_t)((capacity + dms::kPageTokens - 1) / dms::kPageTokens);
   // Default: the dense worst case, every head of every layer at full capacity.
   c.pool_pages = opt->pool_tokens > 0
@@ -114,13 +114,13 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   if (e == cudaSuccess) e = alloc(&c.pool, (size_t)c.pool_pages * dms::kPageBytes);
   if (e == cudaSuccess) e = alloc(&c.pos, (size_t)c.pool_pages * dms::kPageTokens);
   if (e == cudaSuccess) e = alloc(&c.page_table, (size_t)layers * heads * c.max_pages);
-  if (e == cudaSuccess) e = alloc(&c.counts, (size_t)layers * heads);
+  if (e == cudaSuccess) e = alloc(&c.counts, (size_t)layers * 2 * heads);
   if (e == cudaSuccess) e = alloc(&c.rings, (size_t)layers * heads * c.ring_len);
   if (e == cudaSuccess) e = alloc(&c.ctrl, (size_t)dms::kCtrlWords);
   if (e == cudaSuccess) e = alloc(&c.freed, (size_t)heads * c.ring_len);
   if (e == cudaSuccess) e = alloc(&c.pieces, (size_t)c.piece_capacity * dms::kPieceFloats);
   if (e == cudaSuccess) e = alloc(&c.piece_counters, (size_t)heads);
-  if (e == cudaSuccess) e = cudaMemset(c.counts, 0, sizeof(int32_t) * (size_t)layers * heads);
+  if (e == cudaSuccess) e = cudaMemset(c.counts, 0, sizeof(int32_t) * (size_t)layers * 2 * heads);
   if (e == cudaSuccess) e = cudaMemset(c.ctrl, 0, sizeof(int32_t) * dms::kCtrlWords);
   if (e == cudaSuccess) e = cudaMemset(c.piece_counters, 0, sizeof(int32_t) * (size_t)heads);
   if (e == cudaSuccess) e = dms::prepare_decode(c);
@@ -157,7 +157,8 @@ dms_status dms_cache_reset(dms_cache* h, void* stream) {
       cudaStreamSynchronize(st) != cudaSuccess)
     return DMS_ERR_CUDA;
   c.peak_pages = std::max<int64_t>(c.peak_pages, std::min<int64_t>(next, c.pool_pages));
-  if (cudaMemsetAsync(c.counts, 0, sizeof(int32_t) * (size_t)c.layers * c.heads, st) != cudaSuccess ||
+  if (cudaMemsetAsync(c.counts, 0, sizeof(int32_t) * (size_t)c.layers * 2 * c.heads, st) !=
+          cudaSuccess ||
       cudaMemsetAsync(c.ctrl, 0, sizeof(int32_t) * dms::kCtrlWords, st) != cudaSuccess ||
       cudaMemsetAsync(c.piece_counters, 0, sizeof(int32_t) * (size_t)c.heads, st) != cudaSuccess)
     return DMS_ERR_CUDA;
@@ -201,18 +202,48 @@ dms_status dms_decode_attention(dms_cache* h, int32_t layer, const void* q, void
   return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
 }
 
+dms_status dms_append_and_decode(dms_cache* h, int32_t layer, const void* k, const void* v,
+                                 const void* decision_logit, const void* q, void* out,
+                                 int32_t gqa_group, float sm_scale, void* stream) {
+  if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  if (layer < 0 || layer >= c.layers || k == nullptr || v == nullptr || decision_logit == nullptr ||
+      q == nullptr || out == nullptr || !aligned16(k) || !aligned16(v) || !aligned16(q) ||
+      !aligned16(out) || (reinterpret_cast<uintptr_t>(decision_logit) & 1u) != 0 ||
+      gqa_group < 1 || gqa_group > dms::kMaxGroup || !(sm_scale == sm_scale))
+    return DMS_ERR_INVALID_ARGUMENT;
+  const int64_t t0 = c.lengths[layer];
+  if (t0 + 1 > c.capacity) return DMS_ERR_CAPACITY;
+  if (!dms::append_decode_fusable(c)) {
+    const dms_status st = dms_append_and_evict(h, layer, k, v, decision_logit, 1, stream);
+    if (st != DMS_OK) return st;
+    return dms_decode_attention(h, layer, q, out, gqa_group, sm_scale, stream);
+  }
+  const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
+  const cudaError_t e =
+      dms::launch_append_decode(c, layer, k, v, decision_logit, q, out, gqa_group,
+                                scale * 1.4426950408889634f, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return DMS_ERR_CUDA;
+  c.lengths[layer] = t0 + 1;
+  return DMS_OK;
+}
+
 dms_status dms_cache_stats(dms_cache* h, dms_stats* out, int32_t* counts, void* stream) {
   if (h == nullptr || out == nullptr) return DMS_ERR_INVALID_ARGUMENT;
   Cache& c = h->c;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t n = (size_t)c.layers * c.heads;
-  std::vector<int32_t> host(n);
+  std::vector<int32_t> both(2 * n), host(n);
   int32_t ctrl[dms::kCtrlWords];
-  if (cudaMemcpyAsync(host.data(), c.counts, n * sizeof(int32_t), cudaMemcpyDeviceToHost, st) !=
+  if (cudaMemcpyAsync(both.data(), c.counts, 2 * n * sizeof(int32_t), cudaMemcpyDeviceToHost, st) !=
           cudaSuccess ||
       cudaMemcpyAsync(ctrl, c.ctrl, sizeof(ctrl), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
       cudaStreamSynchronize(st) != cudaSuccess)
     return DMS_ERR_CUDA;
+  for (int l = 0; l < c.layers; ++l) {
+    const int32_t* src = both.data() + ((size_t)l * 2 + (c.lengths[l] & 1)) * c.heads;
+    memcpy(host.data() + (size_t)l * c.heads, src, sizeof(int32_t) * c.heads);
+  }
   memset(out, 0, sizeof(*out));
   int64_t total = 0;
   int32_t mx = 0, mn = n ? host[0] : 0;

@@ -42,7 +42,15 @@ constexpr int kProducerWarp = 4;
 constexpr int kEpilogueWarp = 5;
 constexpr int kThreads = 6 * 32;
 constexpr int kQBytes = kMaxGroup * kRowBytes;                 // 4096
-constexpr int kStageBytes = 2 * kHalfPageBytes + kQBytes;      // 36864
+constexpr int kPatchBytes = 2 * kRowBytes;                     // new K and V row (fused append)
+constexpr int kStageBytesPlain = 2 * kHalfPageBytes + kQBytes;  // 36864
+constexpr int kStageBytesFused = kStageBytesPlain + kPatchBytes;  // 37376
+__host__ __device__ constexpr int stage_bytes(bool fused) {
+  return fused ? kStageBytesFused : kStageBytesPlain;
+}
+// Largest batch * kv_heads the fused append + decode kernel takes (its per-head
+// slot table must fit next to the stages); larger caches use the two kernels.
+constexpr int kMaxHeadsFused = 4000;
 // Merge rows (one per query head, 128 floats of head_dim) are padded to 132
 // floats: the stores of an O^T accumulator fragment then hit 32 distinct banks.
 constexpr int kMergeRow = kHeadDim + 4;
@@ -60,9 +68,9 @@ struct Plan {
 };
 
 struct DecodeParams {
-  const uint8_t* pool;
-  const int32_t* page_table;  // this layer
-  const int32_t* counts;      // this layer
+  uint8_t* pool;
+  int32_t* page_table;        // this layer
+  const int32_t* counts;      // this layer, current buffer
   const __nv_bfloat16* q;
   __nv_bfloat16* out;
   float* pieces;
@@ -70,6 +78,15 @@ struct DecodeParams {
   int32_t* ctrl;
   int32_t heads, kv_heads, group, max_pages, min_pages;
   float scale_log2;  // sm_scale * log2(e)
+  // Fused single-token append (position j) in front of the decode.
+  const uint16_t* k_new;      // [batch, 1, kv_heads, 128]
+  const uint16_t* v_new;
+  const uint16_t* logit_new;  // [batch, 1, kv_heads]
+  int32_t* counts_next;       // this layer, buffer after the append
+  uint32_t* ring;             // this layer: [heads][ring_len]
+  int32_t* pos;
+  int64_t j, window, pool_pages;
+  int32_t ring_len;
 };
 
 // ---------------------------------------------------------------- PTX wrappers
@@ -218,12 +235,13 @@ __device__ __forceinline__ int head_of_page(const int32_t* pstart, int heads, in
   return lo - 1;
 }
 
-template <int NT>
+template <int NT, bool kFused>
 size_t tiled_smem_bytes(int heads, int stages) {
   using PL = Plan<NT>;
-  return (size_t)stages * kStageBytes + (size_t)PL::kSlots * (PL::kSlotOFloats + PL::kSlotMLFloats) * 4 +
+  return (size_t)stages * stage_bytes(kFused) +
+         (size_t)PL::kSlots * (PL::kSlotOFloats + PL::kSlotMLFloats) * 4 +
          (size_t)(2 * stages + 2 * PL::kSlots) * sizeof(uint64_t) + 64 +
-         (size_t)(2 * heads + 1) * sizeof(int32_t);
+         (size_t)((kFused ? 3 : 2) * heads + 1) * sizeof(int32_t);
 }
 
 // Iteration order over a CTA's pages (parts A, C, B; see the file comment) and the
@@ -261,11 +279,12 @@ struct PageWalk {
   }
 };
 
-template <int kStages, int NT>
+template <int kStages, int NT, bool kFused>
 __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     decode_tiled_kernel(const DecodeParams p) {
   using PL = Plan<NT>;
   constexpr int HP = PL::kHeadsPad;
+  constexpr int kStageBytes = stage_bytes(kFused);
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
   float* merge_o = reinterpret_cast<float*>(smem + kStages * kStageBytes);  // [slots][4][HP][132]
@@ -274,9 +293,12 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   uint64_t* empty_bar = full_bar + kStages;
   uint64_t* mfull_bar = empty_bar + kStages;
   uint64_t* mempty_bar = mfull_bar + PL::kSlots;
-  int* s_misc = reinterpret_cast<int*>(mempty_bar + PL::kSlots);  // [0] abort [2..7] warp sums
-  int32_t* s_cnt = s_misc + 16;                                   // [heads]
+  // s_misc: [0] abort, [2..7] warp sums, [8..8+kStages) page id staged in each stage
+  int* s_misc = reinterpret_cast<int*>(mempty_bar + PL::kSlots);
+  int32_t* s_cnt = s_misc + 16;                                   // [heads] n_h (after the append)
   int32_t* s_pstart = s_cnt + p.heads;                            // [heads + 1]
+  // fused: new token's slot | fresh << 30 | alpha << 31 per head
+  uint32_t* s_slot = reinterpret_cast<uint32_t*>(s_pstart + p.heads + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int heads = p.heads, G = p.group, Hq = p.kv_heads * p.group;
@@ -297,7 +319,29 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   pdl_wait_prerequisites();
-  for (int h = tid; h < heads; h += kThreads) s_cnt[h] = p.counts[h];
+  if constexpr (kFused) {
+    // Delayed eviction for position j (Sec. 3.1-3.2): the token j - window - 1 leaves
+    // the window; if it was flagged, the new token takes its slot, otherwise the
+    // fresh slot n_h.  Every CTA derives this for every head from the ring; only
+    // the CTA owning a head's last page stores the new count and ring entry.
+    const int64_t R = p.window + 1, RP = ring_period(p.window);
+    for (int h = tid; h < heads; h += kThreads) {
+      const int32_t n = p.counts[h];
+      uint32_t slot = (uint32_t)n, fresh = 1u;
+      if (p.j >= R) {
+        const uint32_t e = p.ring[(int64_t)h * p.ring_len + (p.j - R) % RP];
+        if (e & kAlphaBit) {
+          slot = e & kSlotMask;
+          fresh = 0u;
+        }
+      }
+      const uint32_t alpha = decision_from_bf16(p.logit_new[h]);
+      s_cnt[h] = n + (int32_t)fresh;
+      s_slot[h] = slot | (fresh << 30) | (alpha << 31);
+    }
+  } else {
+    for (int h = tid; h < heads; h += kThreads) s_cnt[h] = p.counts[h];
+  }
   __syncthreads();
   {
     const int per = (heads + kThreads - 1) / kThreads;
@@ -364,7 +408,23 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
         hh = head_of_page(s_pstart, heads, x);
         pg = (int)(x - s_pstart[hh]);
         nv = min(kPageTokens, s_cnt[hh] - pg * kPageTokens);
-        page = __ldg(p.page_table + (int64_t)hh * p.max_pages + pg);
+        bool new_page = false;
+        if constexpr (kFused) {
+          const uint32_t sl = s_slot[hh];
+          const int32_t slot = (int32_t)(sl & 0x3fffffffu);
+          new_page = ((sl >> 30) & 1u) && (slot % kPageTokens == 0) && (pg == slot / kPageTokens);
+        }
+        if (new_page) {  // fused: the new token opens a page
+          page = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
+          if ((int64_t)page >= p.pool_pages) {
+            set_device_error(p.ctrl, DMS_ERR_CAPACITY);
+            page = -1;
+          } else {
+            p.page_table[(int64_t)hh * p.max_pages + pg] = page;
+          }
+        } else {
+          page = __ldg(p.page_table + (int64_t)hh * p.max_pages + pg);
+        }
       }
       const int nb = min(32, niters - it0);
       for (int i = 0; i < nb; ++i) {
@@ -381,14 +441,30 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
           const uint32_t kv_bytes = (uint32_t)nv_i * kRowBytes;
           const uint32_t q_bytes = seg_start ? (uint32_t)G * kRowBytes : 0u;
           uint8_t* st = stages + s * kStageBytes;
-          mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + q_bytes);
-          const uint8_t* src = p.pool + (int64_t)page_i * kPageBytes;
+          bool patch = false;
+          if constexpr (kFused) {
+            const uint32_t sl = s_slot[h_i];
+            patch = (int32_t)(sl & 0x3fffffffu) / kPageTokens == pg_i;
+            s_misc[8 + s] = page_i;
+            if (pg_i == s_pstart[h_i + 1] - s_pstart[h_i] - 1) {  // owner of the head's last page
+              p.counts_next[h_i] = s_cnt[h_i];
+              p.ring[(int64_t)h_i * p.ring_len + p.j % ring_period(p.window)] = sl & ~(1u << 30);
+            }
+          }
+          mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + q_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
+          const uint8_t* src = p.pool + (int64_t)(page_i < 0 ? 0 : page_i) * kPageBytes;
           bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
           bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
           if (seg_start) {
             const int b = h_i / p.kv_heads, hk = h_i - b * p.kv_heads;
             const __nv_bfloat16* qsrc = p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
             bulk_copy_g2s(st + 2 * kHalfPageBytes, qsrc, q_bytes, &full_bar[s]);
+          }
+          if (patch) {  // fused: the new token's K and V rows, as given (unpermuted)
+            bulk_copy_g2s(st + kStageBytesPlain, p.k_new + (int64_t)h_i * kHeadDim, kRowBytes,
+                          &full_bar[s]);
+            bulk_copy_g2s(st + kStageBytesPlain + kRowBytes, p.v_new + (int64_t)h_i * kHeadDim,
+                          kRowBytes, &full_bar[s]);
           }
           ++issued;
         }
@@ -536,6 +612,29 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     const bool seg_end = walk.seg_end(it, niters);
     uint8_t* st = stages + s * kStageBytes;
     mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
+
+    if constexpr (kFused) {
+      const uint32_t sl = s_slot[walk.h];
+      const int32_t slot = (int32_t)(sl & 0x3fffffffu);
+      const uint32_t r = (uint32_t)(slot % kPageTokens);
+      if (slot / kPageTokens == walk.pg && (int)(r >> 4) == warp) {
+        // The warp whose 16 rows hold the new token moves its K and V row from the
+        // patch buffer into the staged page (permuted layout) and into the pool.
+        const int half = lane >> 4, chunk = lane & 15;
+        const uint4 val =
+            *reinterpret_cast<const uint4*>(st + kStageBytesPlain + half * kRowBytes + chunk * 16);
+        const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
+        *reinterpret_cast<uint4*>(st + off) = val;
+        const int page = s_misc[8 + s];
+        if (page >= 0) {
+          *reinterpret_cast<uint4*>(p.pool + (int64_t)page * kPageBytes + off) = val;
+          if (lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
+        }
+        // These generic writes precede the next bulk copy into this stage.
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+      }
+    }
 
     if (seg_start) {
       const uint32_t qbase = smem_addr(st + 2 * kHalfPageBytes);
@@ -749,19 +848,28 @@ cudaError_t prepare_decode(const Cache& c) {
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   };
-  set(decode_tiled_kernel<kStagesOneCta, 1>, tiled_smem_bytes<1>(kMaxHeads, kStagesOneCta));
-  set(decode_tiled_kernel<kStagesOneCta, 2>, tiled_smem_bytes<2>(kMaxHeads, kStagesOneCta));
-  set(decode_tiled_kernel<kStagesTwoCta, 1>, tiled_smem_bytes<1>(kMaxHeads, kStagesTwoCta));
-  set(decode_tiled_kernel<kStagesTwoCta, 2>, tiled_smem_bytes<2>(kMaxHeads, kStagesTwoCta));
+  set(decode_tiled_kernel<kStagesOneCta, 1, false>,
+      tiled_smem_bytes<1, false>(kMaxHeads, kStagesOneCta));
+  set(decode_tiled_kernel<kStagesOneCta, 2, false>,
+      tiled_smem_bytes<2, false>(kMaxHeads, kStagesOneCta));
+  set(decode_tiled_kernel<kStagesTwoCta, 1, false>,
+      tiled_smem_bytes<1, false>(kMaxHeads, kStagesTwoCta));
+  set(decode_tiled_kernel<kStagesTwoCta, 2, false>,
+      tiled_smem_bytes<2, false>(kMaxHeads, kStagesTwoCta));
+  set(decode_tiled_kernel<kStagesOneCta, 1, true>,
+      tiled_smem_bytes<1, true>(kMaxHeadsFused, kStagesOneCta));
+  set(decode_tiled_kernel<kStagesOneCta, 2, true>,
+      tiled_smem_bytes<2, true>(kMaxHeadsFused, kStagesOneCta));
   return e;
 }
 
 namespace {
 
 // Launch with programmatic stream serialisation (the kernel waits for its
-// prerequisites itself); the variant is picked by CTAs per SM and group size.
+// prerequisites itself); the variant is picked by CTAs per SM, group size and
+// whether the single-token append is fused in.
 cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cudaStream_t stream,
-                         bool programmatic) {
+                         bool programmatic, bool fused) {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -770,27 +878,33 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = programmatic ? 1 : 0;
-  const bool two = ctas_per_sm >= 2;
+  const bool two = !fused && ctas_per_sm >= 2;
   const int stages = two ? kStagesTwoCta : kStagesOneCta;
   cfg.gridDim = dim3(num_sms * (two ? ctas_per_sm : 1));
-  if (p.group <= 8) {
-    cfg.dynamicSmemBytes = tiled_smem_bytes<1>(p.heads, stages);
-    return two ? cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesTwoCta, 1>, p)
-               : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 1>, p);
+  if (fused) {
+    if (p.group <= 8) {
+      cfg.dynamicSmemBytes = tiled_smem_bytes<1, true>(p.heads, stages);
+      return cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 1, true>, p);
+    }
+    cfg.dynamicSmemBytes = tiled_smem_bytes<2, true>(p.heads, stages);
+    return cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 2, true>, p);
   }
-  cfg.dynamicSmemBytes = tiled_smem_bytes<2>(p.heads, stages);
-  return two ? cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesTwoCta, 2>, p)
-             : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 2>, p);
+  if (p.group <= 8) {
+    cfg.dynamicSmemBytes = tiled_smem_bytes<1, false>(p.heads, stages);
+    return two ? cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesTwoCta, 1, false>, p)
+               : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 1, false>, p);
+  }
+  cfg.dynamicSmemBytes = tiled_smem_bytes<2, false>(p.heads, stages);
+  return two ? cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesTwoCta, 2, false>, p)
+             : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 2, false>, p);
 }
 
-}  // namespace
-
-cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, void* out,
-                                int32_t group, float scale_log2, cudaStream_t stream) {
-  DecodeParams p;
+DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* out, int32_t group,
+                          float scale_log2) {
+  DecodeParams p = {};
   p.pool = c.pool;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
-  p.counts = c.counts + (int64_t)layer * c.heads;
+  p.counts = c.counts_at(layer, c.lengths[layer]);
   p.q = static_cast<const __nv_bfloat16*>(q);
   p.out = static_cast<__nv_bfloat16*>(out);
   p.pieces = c.pieces;
@@ -802,14 +916,46 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
   p.max_pages = c.max_pages;
   p.min_pages = c.min_pages_per_cta;
   p.scale_log2 = scale_log2;
-  return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true);
+  return p;
+}
+
+}  // namespace
+
+cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, void* out,
+                                int32_t group, float scale_log2, cudaStream_t stream) {
+  const DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
+  return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false);
+}
+
+bool append_decode_fusable(const Cache& c) {
+  return c.decode_kernel == DMS_DECODE_TILED && c.heads <= kMaxHeadsFused && c.ctas_per_sm < 2;
+}
+
+// Single-token append of position lengths[layer] fused with the decode (requires
+// append_decode_fusable).
+cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,
+                                 const void* logit, const void* q, void* out, int32_t group,
+                                 float scale_log2, cudaStream_t stream) {
+  const int64_t t0 = c.lengths[layer];
+  DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
+  p.k_new = static_cast<const uint16_t*>(k);
+  p.v_new = static_cast<const uint16_t*>(v);
+  p.logit_new = static_cast<const uint16_t*>(logit);
+  p.counts_next = c.counts_at(layer, t0 + 1);
+  p.ring = c.rings + (int64_t)layer * c.heads * c.ring_len;
+  p.pos = c.pos;
+  p.j = t0;
+  p.window = c.window;
+  p.pool_pages = c.pool_pages;
+  p.ring_len = c.ring_len;
+  return launch_tiled(p, c.num_sms, 1, stream, true, true);
 }
 
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
                                  int32_t group, float scale, cudaStream_t stream) {
   decode_simple_kernel<<<c.heads, 128, 0, stream>>>(
       c.pool, c.page_table + (int64_t)layer * c.heads * c.max_pages,
-      c.counts + (int64_t)layer * c.heads, static_cast<const __nv_bfloat16*>(q),
+      c.counts_at(layer, c.lengths[layer]), static_cast<const __nv_bfloat16*>(q),
       static_cast<__nv_bfloat16*>(out), c.kv_heads, group, c.max_pages, scale);
   return cudaGetLastError();
 }
@@ -907,9 +1053,9 @@ extern "C" dms_status dms_decode_attention_paged_noalloc(
       cudaSuccess)
     return DMS_ERR_CUDA;
 
-  DecodeParams p;
-  p.pool = static_cast<const uint8_t*>(pool);
-  p.page_table = page_table;
+  DecodeParams p = {};
+  p.pool = static_cast<uint8_t*>(const_cast<void*>(pool));
+  p.page_table = const_cast<int32_t*>(page_table);
   p.counts = counts;
   p.q = static_cast<const __nv_bfloat16*>(q);
   p.out = static_cast<__nv_bfloat16*>(out);
@@ -923,5 +1069,5 @@ extern "C" dms_status dms_decode_attention_paged_noalloc(
   p.min_pages = 2;
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)kHeadDim);
   p.scale_log2 = scale * 1.4426950408889634f;
-  return launch_tiled(p, grid, 1, s, false) == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+  return launch_tiled(p, grid, 1, s, false, false) == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
 }

@@ -10,9 +10,17 @@
 //   pos         [pool_pages][64] int32          position held by each slot (inspection only;
 //                                               decode never reads it).
 //   page_table  [layers][heads][max_pages] int32 page of slot s is page_table[.][s / 64].
-//   counts      [layers][heads] int32            n_h: slots [0, n_h) hold the retained set.
-//   rings       [layers][heads][ring_len] u32    decision ring of the last window+1 tokens:
-//               entry for position j at j % (window + 1) = slot | alpha << 31.
+//   counts      [layers][2][heads] int32         n_h: slots [0, n_h) hold the retained set.
+//               Double-buffered: a layer of length T keeps its counts in buffer T & 1,
+//               and an append of n tokens reads buffer T & 1 and writes (T + n) & 1, so
+//               a kernel whose CTAs all read every head's count never sees a count
+//               that another CTA of the same launch has already advanced.
+//   rings       [layers][heads][ring_len] u32    decisions of recent tokens: the entry of
+//               position j sits at j % (window + 2) and holds slot | alpha << 31.  The
+//               period is one longer than the window + 1 tokens that must be kept, so
+//               the entry read for the token leaving at step j ((j - window - 1) %
+//               (window + 2)) and the entry written for the new token (j % (window + 2))
+//               are always different words.
 //   ctrl        [kCtrlWords] int32               [0] next free page, [1] sticky error.
 //   freed       [heads][ring_len] int32          bulk-append scratch (slots freed this call).
 //   pieces      [piece_capacity][kPieceFloats]   split-K partial records of the decode.
@@ -38,6 +46,7 @@ constexpr int kMaxHeads = 4096;                               // batch * kv_head
 constexpr int kMaxCtasPerSm = 4;
 constexpr uint32_t kAlphaBit = 0x80000000u;
 constexpr uint32_t kSlotMask = 0x7fffffffu;
+constexpr int64_t kMaxCapacity = (1ll << 30) - 1;  // slots stay below 2^30
 constexpr int kPieceFloats = 2 * kMaxGroup + kMaxGroup * kHeadDim;  // m[16] l[16] o[16][128]
 constexpr int kCtrlWords = 16;
 constexpr int kCtrlPoolNext = 0;
@@ -49,7 +58,7 @@ struct Cache {
   int32_t layers = 0, kv_heads = 0, head_dim = 0, window = 0, batch = 0;
   int64_t capacity = 0;
   int32_t heads = 0;        // batch * kv_heads
-  int32_t ring_len = 0;     // min(window + 1, capacity)
+  int32_t ring_len = 0;     // min(window + 2, capacity)
   int32_t max_pages = 0;    // ceil(capacity / 64)
   int64_t pool_pages = 0;
   int32_t decode_kernel = 0, ctas_per_sm = 1, min_pages_per_cta = 2;
@@ -68,7 +77,15 @@ struct Cache {
 
   int64_t* lengths = nullptr;  // host: tokens appended per layer
   int64_t peak_pages = 0;      // host: largest pages_in_use observed
+
+  // Count buffer of `layer` for a layer length of parity `parity`.
+  int32_t* counts_at(int32_t layer, int64_t parity) const {
+    return counts + ((int64_t)layer * 2 + (parity & 1)) * heads;
+  }
 };
+
+// Ring period (entries per head cycle) for a sliding window w.
+__host__ __device__ __forceinline__ int64_t ring_period(int64_t window) { return window + 2; }
 
 // Sticky device error: the first code written wins.
 __device__ __forceinline__ void set_device_error(int32_t* ctrl, int32_t code) {
@@ -98,5 +115,9 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
                                 int32_t group, float scale_log2, cudaStream_t stream);
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
                                  int32_t group, float scale, cudaStream_t stream);
+bool append_decode_fusable(const Cache& c);
+cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,
+                                 const void* logit, const void* q, void* out, int32_t group,
+                                 float scale_log2, cudaStream_t stream);
 
 }  // namespace dms

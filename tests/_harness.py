@@ -20,8 +20,9 @@ MEAN_ABS = 2e-3
 
 class Run:
     def __init__(self, wl: workloads.Workload, device="cuda", layer: int = 0,
-                 capacity: int | None = None, **cache_kw):
+                 capacity: int | None = None, fused: bool = False, **cache_kw):
         self.wl, self.layer, self.dev = wl, layer, torch.device(device)
+        self.fused = fused  # decode steps through dms_append_and_decode
         self.T = capacity or wl.context
         B, H, D = wl.batch, wl.kv_heads, wl.head_dim
         self.cache = dms.DmsCache(layers=1, kv_heads=H, window=wl.window, capacity=self.T,
@@ -54,11 +55,23 @@ class Run:
                 k, v, lg = workloads.gen_kv(self.wl, self.layer, f"prefill{i}", n, self.dev)
             self.append(k, v, lg)
 
-    def step(self, s: int):
-        k, v, lg = workloads.gen_kv(self.wl, self.layer, f"decode{s}", 1, self.dev)
-        self.append(k, v, lg)
+    def record(self, k, v, lg):
+        n = k.shape[1]
+        self.K[:, self.t:self.t + n] = k
+        self.V[:, self.t:self.t + n] = v
+        self.L[:, self.t:self.t + n] = lg
+        self.t += n
+
+    def step(self, s: int, p_override=None):
+        k, v, lg = workloads.gen_kv(self.wl, self.layer, f"decode{s}", 1, self.dev,
+                                    p_override=p_override)
         q = workloads.gen_q(self.wl, self.layer, f"decode{s}", self.dev)
-        out = self.cache.decode_attention(0, q, gqa_group=self.wl.gqa_group)
+        if self.fused:
+            out = self.cache.append_and_decode(0, k, v, lg, q, gqa_group=self.wl.gqa_group)
+            self.record(k, v, lg)
+        else:
+            self.append(k, v, lg)
+            out = self.cache.decode_attention(0, q, gqa_group=self.wl.gqa_group)
         return q, out
 
     # ---- checks

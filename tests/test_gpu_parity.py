@@ -48,31 +48,67 @@ def _run_all_steps(wl, check_every=1, retained_every=4, **cache_kw):
 # ---------------------------------------------------------------- the small config, in full
 
 
-@pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_SIMPLE])
-def test_llama_b1_ctx4352_every_step(kernel):
+@pytest.mark.parametrize("kernel,fused", [(dms.DMS_DECODE_TILED, False), (dms.DMS_DECODE_TILED, True),
+                                          (dms.DMS_DECODE_SIMPLE, False)])
+def test_llama_b1_ctx4352_every_step(kernel, fused):
     """Batch 1, 32 q / 8 kv heads, prefill 4096 + 256 decode steps, w = 256, P(evict) 0.875:
     every step, every query head; retained sets every 16 steps."""
     wl = workloads.LLAMA_B1_4K
-    mx, mean = _run_all_steps(wl, check_every=1, retained_every=16, decode_kernel=kernel)
+    mx, mean = _run_all_steps(wl, check_every=1, retained_every=16, decode_kernel=kernel,
+                              fused=fused)
     assert mx <= MAX_ABS and mean <= MEAN_ABS
 
 
 # ---------------------------------------------------------------- edge cases
 
 
+@pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("w", [0, 1, 15, 63, 64, 255, 256])
-def test_windows(w):
-    _run_all_steps(small(window=w, prefill=((333, False),), decode_steps=6))
+def test_windows(w, fused):
+    _run_all_steps(small(window=w, prefill=((333, False),), decode_steps=6), fused=fused)
 
 
-@pytest.mark.parametrize("G", [1, 3, 4, 5, 7, 8, 16])
-def test_gqa_groups(G):
-    _run_all_steps(small(q_heads=2 * G, kv_heads=2, decode_steps=4))
+@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("G", [1, 3, 4, 5, 7, 8, 9, 16])
+def test_gqa_groups(G, fused):
+    _run_all_steps(small(q_heads=2 * G, kv_heads=2, decode_steps=4), fused=fused)
 
 
+@pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("prefill", [1, 2, 63, 64, 65, 127, 128, 129, 1000])
-def test_page_boundaries(prefill):
-    _run_all_steps(small(prefill=((prefill, False),), decode_steps=5, window=20, p_evict=0.5))
+def test_page_boundaries(prefill, fused):
+    _run_all_steps(small(prefill=((prefill, False),), decode_steps=5, window=20, p_evict=0.5),
+                   fused=fused)
+
+
+@pytest.mark.parametrize("w", [0, 3, 40])
+def test_fused_decode_from_empty_cache(w):
+    """The fused step appends and attends from the very first token (pages opened in-kernel)."""
+    wl = small(window=w, prefill=(), decode_steps=150, p_evict=0.6)
+    _run_all_steps(wl, check_every=7, retained_every=10, fused=True)
+
+
+def test_fused_matches_separate_bitwise():
+    """dms_append_and_decode gives the same retained sets and the same bits as the two calls."""
+    wl = small(batch=3, kv_heads=4, q_heads=28, window=30, prefill=((700, False),), decode_steps=40,
+               p_evict=0.7)
+    a, b = Run(wl, fused=False), Run(wl, fused=True)
+    try:
+        a.prefill()
+        b.prefill()
+        for s_ in range(wl.decode_steps):
+            _, oa = a.step(s_)
+            _, ob = b.step(s_)
+            assert torch.equal(oa, ob), s_
+        pa, pb = a.cache.export_positions(0), b.cache.export_positions(0)
+        for bb in range(wl.batch):
+            for h in range(wl.kv_heads):
+                assert np.array_equal(np.sort(pa[bb, h][pa[bb, h] >= 0]), np.sort(pb[bb, h][pb[bb, h] >= 0]))
+        a.check_retained()
+        b.check_retained()
+    finally:
+        a.close()
+        b.close()
 
 
 @pytest.mark.parametrize("p", [0.0, 1.0])
@@ -111,10 +147,11 @@ def test_w0_all_evict_single_token():
         r.close()
 
 
-def test_ragged_heads_mixed_probabilities():
+@pytest.mark.parametrize("fused", [False, True])
+def test_ragged_heads_mixed_probabilities(fused):
     """Heads with P(evict) from 0 to 1 in one layer: very different n_h per head."""
     wl = small(batch=3, kv_heads=4, q_heads=20, window=24, prefill=((900, False),), decode_steps=6)
-    r = Run(wl)
+    r = Run(wl, fused=fused)
     try:
         B, H = wl.batch, wl.kv_heads
         p = [0.0, 0.5, 0.95, 1.0]
@@ -122,10 +159,7 @@ def test_ragged_heads_mixed_probabilities():
         r.append(k, v, lg)
         r.check_retained()
         for s in range(wl.decode_steps):
-            k, v, lg = workloads.gen_kv(wl, 0, f"decode{s}", 1, r.dev, p_override=p)
-            r.append(k, v, lg)
-            q = workloads.gen_q(wl, 0, f"decode{s}", r.dev)
-            out = r.cache.decode_attention(0, q, gqa_group=wl.gqa_group)
+            q, out = r.step(s, p_override=p)
             r.check_outputs(q, out)
         st = r.check_retained()
         assert st["counts"].max() > 5 * st["counts"].min()
@@ -181,12 +215,13 @@ def test_bulk_then_decode_equals_sequential():
         b.close()
 
 
+@pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("min_pages,ctas", [(1, 4), (1, 1), (1000000, 1), (3, 2)])
-def test_split_shapes(min_pages, ctas):
+def test_split_shapes(min_pages, ctas, fused):
     """Heads split over many CTAs (multi-piece combine) and one CTA walking all heads."""
     wl = small(batch=2, kv_heads=3, q_heads=15, window=40, prefill=((2500, False),), decode_steps=3,
                p_evict=0.3)
-    _run_all_steps(wl, min_pages_per_cta=min_pages, ctas_per_sm=ctas)
+    _run_all_steps(wl, min_pages_per_cta=min_pages, ctas_per_sm=ctas, fused=fused)
 
 
 def test_empty_cache_gives_zeros():
