@@ -217,6 +217,18 @@ dms_status dms_decode_attention_paged_noalloc(const void* pool, const int32_t* p
                                               const void* q, void* out, int32_t gqa_group,
                                               float sm_scale, void* stream);
 
+/*
+ * Self-test of the bounded wait every kernel of this library uses on its
+ * shared-memory barriers (the paper has no counterpart: this is failure
+ * detection of the implementation).  Launches one small kernel in which a thread
+ * waits on a barrier that a second thread completes only if `arrive` is non-zero.
+ * Returns DMS_OK when the wait completed, DMS_ERR_TIMEOUT when it gave up after
+ * `limit_ns` nanoseconds (1 us .. 10 s; the kernels use 2 s) -- in both cases the
+ * kernel exits normally and the CUDA context stays usable.  Synchronises `stream`;
+ * allocates and frees a few bytes of device memory.
+ */
+dms_status dms_selftest_bounded_wait(int32_t arrive, int64_t limit_ns, void* stream);
+
 /* Static description of a status code. */
 const char* dms_status_string(dms_status status);
 

@@ -101,6 +101,10 @@ def dms_decode_attention_paged_noalloc(pool_ptr, page_table_ptr, counts_ptr, bat
         gqa_group, float(sm_scale), stream)
 
 
+def dms_selftest_bounded_wait(arrive, limit_ns, stream):
+    return library().dms_selftest_bounded_wait(int(arrive), int(limit_ns), stream)
+
+
 # ---- torch-facing wrapper ---------------------------------------------------
 
 def _stream_ptr(stream=None):

@@ -287,6 +287,25 @@ dms_status dms_cache_export_positions(dms_cache* h, int32_t layer, int32_t* host
   return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
 }
 
+dms_status dms_selftest_bounded_wait(int32_t arrive, int64_t limit_ns, void* stream) {
+  if (limit_ns < 1000 || limit_ns > 10000000000LL) return DMS_ERR_INVALID_ARGUMENT;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int32_t* dev = nullptr;
+  int32_t host[dms::kCtrlWords] = {0};
+  if (cudaMalloc(&dev, sizeof(host)) != cudaSuccess) {
+    cudaGetLastError();
+    return DMS_ERR_OUT_OF_MEMORY;
+  }
+  cudaError_t e = cudaMemsetAsync(dev, 0, sizeof(host), st);
+  if (e == cudaSuccess) e = dms::launch_bounded_wait_probe(arrive != 0, limit_ns, dev, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(host, dev, sizeof(host), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(dev);
+  if (e != cudaSuccess) return DMS_ERR_CUDA;
+  if (host[dms::kCtrlError] != 0) return static_cast<dms_status>(host[dms::kCtrlError]);
+  return host[dms::kCtrlError + 1] == 1 ? DMS_OK : DMS_ERR_STATE;
+}
+
 dms_status dms_cache_layer_length(const dms_cache* h, int32_t layer, int64_t* out) {
   if (h == nullptr || out == nullptr || layer < 0 || layer >= h->c.layers)
     return DMS_ERR_INVALID_ARGUMENT;

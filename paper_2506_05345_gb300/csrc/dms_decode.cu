@@ -133,13 +133,14 @@ __device__ __forceinline__ unsigned long long global_timer_ns() {
 // (*abort != 0); then records DMS_ERR_TIMEOUT and returns false.  Callers keep
 // their control flow unchanged on failure, so no barrier is ever left waiting.
 __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                            int32_t* ctrl) {
+                                            int32_t* ctrl,
+                                            unsigned long long limit_ns = kWaitLimitNs) {
   const unsigned long long t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 31u) == 0u) {
       if (*abort) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
+      if (global_timer_ns() - t0 > limit_ns) {
         *abort = 1;
         set_device_error(ctrl, DMS_ERR_TIMEOUT);
         return false;
@@ -837,7 +838,32 @@ __global__ void __launch_bounds__(128) decode_simple_kernel(const uint8_t* pool,
   }
 }
 
+// Self-test of the bounded wait used by every kernel: thread 0 waits on an
+// mbarrier of count 1; thread 32 arrives on it only when `arrive` is set.
+__global__ void bounded_wait_probe_kernel(int arrive, unsigned long long limit_ns, int32_t* status) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 32 && arrive) mbar_arrive(&bar);
+  if (threadIdx.x == 0) {
+    const bool ok = mbar_try_wait(&bar, 0) ||
+                    mbar_wait_slow(&bar, 0, &abort_flag, status, limit_ns);
+    if (ok) status[kCtrlError + 1] = 1;  // completion seen
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_bounded_wait_probe(int arrive, int64_t limit_ns, int32_t* dev_status,
+                                      cudaStream_t stream) {
+  bounded_wait_probe_kernel<<<1, 64, 0, stream>>>(arrive, (unsigned long long)limit_ns, dev_status);
+  return cudaGetLastError();
+}
 
 cudaError_t prepare_decode(const Cache& c) {
   (void)c;

@@ -116,6 +116,8 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
                                  int32_t group, float scale, cudaStream_t stream);
 bool append_decode_fusable(const Cache& c);
+cudaError_t launch_bounded_wait_probe(int arrive, int64_t limit_ns, int32_t* dev_status,
+                                      cudaStream_t stream);
 cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,
                                  const void* logit, const void* q, void* out, int32_t group,
                                  float scale_log2, cudaStream_t stream);
