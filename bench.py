@@ -195,6 +195,22 @@ def sum_over_ranks(pg, x, dev):
     return float(t.item())
 
 
+def aggregate_throughput(pg, units, elapsed_ms, dev):
+    """Whole-job throughput: units processed by all ranks / the slowest rank's time.
+
+    Returns (units per second, max elapsed ms).  Each rank runs an independent replica
+    (weak scaling); this reduction is the only cross-rank traffic.
+    """
+    t_max = max_over_ranks(pg, elapsed_ms, dev)
+    total = sum_over_ranks(pg, units, dev)
+    return total / (t_max * 1e-3), t_max
+
+
+def replica_tag(rank):
+    """Seed tag of a rank's replica: every rank draws its own batch of sequences."""
+    return f"rank{rank}"
+
+
 # ============================================================================ ours
 
 
@@ -212,7 +228,7 @@ def run_ours(args, wl, world, rank, local, pg):
     E_K, E_W = (0, 0) if args.no_e2e else (min(K_, 50), 2)
     decode_needed = max(wl.decode_steps, W_ + K_ + K2 + E_W + E_K)
     capacity = wl.prefill_tokens + decode_needed
-    seed_tag = f"rank{rank}"
+    seed_tag = replica_tag(rank)
     cache = dms.DmsCache(layers=L, kv_heads=H, window=wl.window, capacity=capacity, batch=B,
                          ctas_per_sm=args.ctas_per_sm, min_pages_per_cta=args.min_pages)
     stream = torch.cuda.current_stream()
@@ -329,9 +345,7 @@ def run_ours(args, wl, world, rank, local, pg):
     bytes_per_unit = workloads.kv_bytes_per_token_head(D)
     dec_avg_s = float(np.mean(dec_ms)) * 1e-3
 
-    elapsed_max_ms = max_over_ranks(pg, elapsed_ms, dev)
-    tokens_all = sum_over_ranks(pg, tokens_read, dev)
-    value = tokens_all / (elapsed_max_ms * 1e-3)
+    value, elapsed_max_ms = aggregate_throughput(pg, tokens_read, elapsed_ms, dev)
 
     # ---- parity sample (layer 0, last timed step) and CPU baseline
     parity = None
@@ -427,9 +441,9 @@ def run_ours(args, wl, world, rank, local, pg):
         torch.cuda.synchronize()
         barrier(pg)
         sa = cache.stats()
-        e_ms = max_over_ranks(pg, a.elapsed_time(z), dev)
-        e_tok = sum_over_ranks(pg, E_K * 0.5 * (sb["total_retained"] + sa["total_retained"]), dev)
-        e2e = {"value": e_tok / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        e_val, e_ms = aggregate_throughput(
+            pg, E_K * 0.5 * (sb["total_retained"] + sa["total_retained"]), a.elapsed_time(z), dev)
+        e2e = {"value": e_val, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms / E_K, "steps": E_K}
 
     if rank != 0:
