@@ -155,6 +155,13 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   return mbar_wait_slow(bar, parity, abort, ctrl);
 }
 
+// atomicAdd with acquire-release semantics at GPU scope; returns the old value.
+__device__ __forceinline__ int atomic_add_acq_rel(int32_t* addr, int v) {
+  int old;
+  asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(addr), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes,
                                               uint64_t* bar) {
   asm volatile(
@@ -220,14 +227,20 @@ __device__ __forceinline__ void pdl_wait_prerequisites() {
 
 // ---------------------------------------------------------------- partition helpers
 
-// Flat page x belongs to CTA ceil((x + 1) * P / N) - 1 when CTA k owns pages
-// [floor(k N / P), floor((k + 1) N / P)).
-__device__ __forceinline__ int cta_of_page(int64_t x, int64_t P, int64_t N) {
-  return (int)(((x + 1) * P + N - 1) / N - 1);
-}
+// Balanced split of N pages over P CTAs in 32-bit arithmetic (N < 2^31): with
+// N = q P + r, CTA k owns pages [k q + min(k, r), (k + 1) q + min(k + 1, r)).
+struct Split {
+  int q, r;
+  __device__ __forceinline__ int begin(int k) const { return k * q + min(k, r); }
+  // CTA owning flat page x.
+  __device__ __forceinline__ int cta_of(int x) const {
+    const int big = r * (q + 1);  // pages of the CTAs that hold q + 1 pages
+    return x < big ? x / (q + 1) : r + (x - big) / q;
+  }
+};
 
 // Last head h with pstart[h] <= x (x < pstart[heads]).
-__device__ __forceinline__ int head_of_page(const int32_t* pstart, int heads, int64_t x) {
+__device__ __forceinline__ int head_of_page(const int32_t* pstart, int heads, int x) {
   int lo = 0, hi = heads;
   while (lo < hi) {
     const int mid = (lo + hi) >> 1;
@@ -251,19 +264,19 @@ size_t tiled_smem_bytes(int heads, int stages) {
 struct PageWalk {
   const int32_t* pstart;  // [heads + 1] page prefix
   int heads;
-  int64_t pbeg, a_end, c_beg;
+  int pbeg, a_end, c_beg;
   int nA, nC;
   int h, pg;
 
-  __device__ __forceinline__ int64_t flat(int it) const {
+  __device__ __forceinline__ int flat(int it) const {
     return it < nA ? pbeg + it : (it < nA + nC ? c_beg + (it - nA) : a_end + (it - nA - nC));
   }
   // Position for iteration `it` (call with it = 0, 1, 2, ... in order).
   __device__ __forceinline__ void enter(int it) {
     if (it == 0 || it == nA || it == nA + nC) {
-      const int64_t x = flat(it);
+      const int x = flat(it);
       h = head_of_page(pstart, heads, x);
-      pg = (int)(x - pstart[h]);
+      pg = x - pstart[h];
     }
   }
   __device__ __forceinline__ int pages_of_head() const { return pstart[h + 1] - pstart[h]; }
@@ -319,29 +332,74 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  // While the previous kernel finishes, warm L2 with the small tables the prologue
+  // reads next (this CTA's slice of the layer's page table; the counts, leaving ring
+  // entries and decision logits).  L2 is coherent with the previous kernel's
+  // writes, so a prefetch can never make a later load stale.
+  {
+    const size_t pt_bytes = (size_t)heads * p.max_pages * sizeof(int32_t);
+    const size_t slice = ((pt_bytes + gridDim.x - 1) / gridDim.x + 15) & ~(size_t)15;
+    const size_t beg = slice * blockIdx.x;
+    if (tid == 0 && beg < pt_bytes) {
+      const size_t len = (beg + slice <= pt_bytes ? slice : pt_bytes - beg) & ~(size_t)15;
+      if (len > 0)
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(
+                         reinterpret_cast<const uint8_t*>(p.page_table) + beg),
+                     "r"((uint32_t)len)
+                     : "memory");
+    }
+    for (int h = blockIdx.x * kThreads + tid; h < heads; h += gridDim.x * kThreads) {
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(p.counts + h));
+      if constexpr (kFused) {
+        const int64_t R = p.window + 1;
+        if (p.j >= R)
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(
+              p.ring + (int64_t)h * p.ring_len + (p.j - R) % ring_period(p.window)));
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(p.logit_new + h));
+      }
+    }
+  }
   pdl_wait_prerequisites();
-  if constexpr (kFused) {
-    // Delayed eviction for position j (Sec. 3.1-3.2): the token j - window - 1 leaves
-    // the window; if it was flagged, the new token takes its slot, otherwise the
-    // fresh slot n_h.  Every CTA derives this for every head from the ring; only
-    // the CTA owning a head's last page stores the new count and ring entry.
+  {
+    // Per-head state, with every load of a batch issued before any is used.  In the
+    // fused variant: delayed eviction for position j (Sec. 3.1-3.2) -- the token
+    // j - window - 1 leaves the window; if it was flagged, the new token takes its
+    // slot, otherwise the fresh slot n_h.  Every CTA derives this for every head
+    // from the ring; only the CTA owning a head's last page stores the new count
+    // and ring entry.
+    constexpr int kPer = 8;
     const int64_t R = p.window + 1, RP = ring_period(p.window);
-    for (int h = tid; h < heads; h += kThreads) {
-      const int32_t n = p.counts[h];
-      uint32_t slot = (uint32_t)n, fresh = 1u;
-      if (p.j >= R) {
-        const uint32_t e = p.ring[(int64_t)h * p.ring_len + (p.j - R) % RP];
-        if (e & kAlphaBit) {
-          slot = e & kSlotMask;
-          fresh = 0u;
+    for (int base = 0; base < heads; base += kThreads * kPer) {
+      int32_t nn[kPer];
+      uint32_t ee[kPer];
+      uint16_t ll[kPer];
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const int h = base + tid + i * kThreads;
+        if (h < heads) {
+          nn[i] = p.counts[h];
+          if constexpr (kFused) {
+            ee[i] = p.j >= R ? p.ring[(int64_t)h * p.ring_len + (p.j - R) % RP] : 0u;
+            ll[i] = p.logit_new[h];
+          }
         }
       }
-      const uint32_t alpha = decision_from_bf16(p.logit_new[h]);
-      s_cnt[h] = n + (int32_t)fresh;
-      s_slot[h] = slot | (fresh << 30) | (alpha << 31);
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const int h = base + tid + i * kThreads;
+        if (h < heads) {
+          if constexpr (kFused) {
+            const bool reuse = (ee[i] & kAlphaBit) != 0u;
+            const uint32_t slot = reuse ? (ee[i] & kSlotMask) : (uint32_t)nn[i];
+            const uint32_t fresh = reuse ? 0u : 1u;
+            s_cnt[h] = nn[i] + (int32_t)fresh;
+            s_slot[h] = slot | (fresh << 30) | (decision_from_bf16(ll[i]) << 31);
+          } else {
+            s_cnt[h] = nn[i];
+          }
+        }
+      }
     }
-  } else {
-    for (int h = tid; h < heads; h += kThreads) s_cnt[h] = p.counts[h];
   }
   __syncthreads();
   {
@@ -366,7 +424,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     if (tid == kThreads - 1) s_pstart[heads] = run;
   }
   __syncthreads();
-  const int64_t N = s_pstart[heads];
+  const int N = s_pstart[heads];
 
   // Heads with no tokens yet produce zeros (spread over the CTAs).
   for (int h = blockIdx.x; h < heads; h += gridDim.x) {
@@ -376,13 +434,14 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     for (int i = tid; i < G * kHeadDim; i += kThreads) o[i] = __float2bfloat16_rn(0.f);
   }
   if (N == 0) return;
-  int64_t P = N / (p.min_pages > 0 ? p.min_pages : 1);
+  int P = N / (p.min_pages > 0 ? p.min_pages : 1);
   if (P < 1) P = 1;
-  if (P > gridDim.x) P = gridDim.x;
+  if (P > (int)gridDim.x) P = (int)gridDim.x;
   const int k = blockIdx.x;
   if (k >= P) return;
-  const int64_t pbeg = (int64_t)k * N / P, pend = (int64_t)(k + 1) * N / P;
-  const int niters = (int)(pend - pbeg);
+  const Split split{N / P, N % P};
+  const int pbeg = split.begin(k), pend = split.begin(k + 1);
+  const int niters = pend - pbeg;
   PageWalk walk;
   walk.pstart = s_pstart;
   walk.heads = heads;
@@ -390,10 +449,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   {
     const int h_first = head_of_page(s_pstart, heads, pbeg);
     const int h_last = head_of_page(s_pstart, heads, pend - 1);
-    walk.a_end = (h_first == h_last) ? pend : (int64_t)s_pstart[h_first + 1];
-    walk.c_beg = (h_first == h_last) ? pend : (int64_t)s_pstart[h_last];
-    walk.nA = (int)(walk.a_end - pbeg);
-    walk.nC = (int)(pend - walk.c_beg);
+    walk.a_end = (h_first == h_last) ? pend : s_pstart[h_first + 1];
+    walk.c_beg = (h_first == h_last) ? pend : s_pstart[h_last];
+    walk.nA = walk.a_end - pbeg;
+    walk.nC = pend - walk.c_beg;
     walk.h = h_first;
     walk.pg = 0;
   }
@@ -405,9 +464,9 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
       const int it = it0 + lane;
       int hh = 0, pg = 0, nv = 0, page = 0;
       if (it < niters) {
-        const int64_t x = walk.flat(it);
+        const int x = walk.flat(it);
         hh = head_of_page(s_pstart, heads, x);
-        pg = (int)(x - s_pstart[hh]);
+        pg = x - s_pstart[hh];
         nv = min(kPageTokens, s_cnt[hh] - pg * kPageTokens);
         bool new_page = false;
         if constexpr (kFused) {
@@ -493,53 +552,79 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
         const float* so = merge_o + slot * PL::kSlotOFloats;
         const float* sml = merge_ml + slot * PL::kSlotMLFloats;
         const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
-        const int64_t first = s_pstart[h], last = s_pstart[h + 1] - 1;
-        const int k_lo = cta_of_page(first, P, N), k_hi = cta_of_page(last, P, N);
+        const int k_lo = split.cta_of(s_pstart[h]), k_hi = split.cta_of(s_pstart[h + 1] - 1);
         const bool single = (k_lo == k_hi);
         __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
         float* rec = p.pieces + (int64_t)(k + h) * kPieceFloats;  // m[16] l[16] o[16][128]
-        // Lane owns head_dim columns 4 lane .. 4 lane + 3 (128-bit loads / stores).
+        // Row statistics in parallel (lane r < G owns row r: the four warps' maxima,
+        // their weights and the merged sum), then the outputs: lane owns head_dim
+        // columns 4 lane .. 4 lane + 3, four rows' shared-memory loads in flight.
         const int d4 = 4 * lane;
-        for (int r = 0; r < G; ++r) {
-          float M = sml[(0 * HP + r) * 2];
+        float rM = -INFINITY, rL = 0.f, rw[kConsumerWarps];
+        if (lane < G) {
 #pragma unroll
-          for (int w = 1; w < kConsumerWarps; ++w) M = fmaxf(M, sml[(w * HP + r) * 2]);
-          float L = 0.f;
-          float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int w = 0; w < kConsumerWarps; ++w) rM = fmaxf(rM, sml[(w * HP + lane) * 2]);
 #pragma unroll
           for (int w = 0; w < kConsumerWarps; ++w) {
-            const float wt = exp2f(sml[(w * HP + r) * 2] - M);
-            L += wt * sml[(w * HP + r) * 2 + 1];
-            const float4 x = *reinterpret_cast<const float4*>(so + (w * HP + r) * kMergeRow + d4);
-            O.x += wt * x.x;
-            O.y += wt * x.y;
-            O.z += wt * x.z;
-            O.w += wt * x.w;
+            rw[w] = exp2f(sml[(w * HP + lane) * 2] - rM);
+            rL += rw[w] * sml[(w * HP + lane) * 2 + 1];
           }
-          if (single) {
-            const float inv = 1.f / L;
-            store_bf16x4(out_h + r * kHeadDim + d4, O.x * inv, O.y * inv, O.z * inv, O.w * inv);
-          } else {
-            *reinterpret_cast<float4*>(rec + 2 * kMaxGroup + r * kHeadDim + d4) = O;
-            if (lane == 0) {
-              rec[r] = M;
-              rec[kMaxGroup + r] = L;
+          if (!single) {
+            rec[lane] = rM;
+            rec[kMaxGroup + lane] = rL;
+          }
+        } else {
+#pragma unroll
+          for (int w = 0; w < kConsumerWarps; ++w) rw[w] = 0.f;
+        }
+        for (int r0 = 0; r0 < G; r0 += 4) {
+          float4 x[4][kConsumerWarps];
+#pragma unroll
+          for (int rr = 0; rr < 4; ++rr)
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w)
+              x[rr][w] = (r0 + rr < G) ? *reinterpret_cast<const float4*>(
+                                             so + (w * HP + r0 + rr) * kMergeRow + d4)
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int rr = 0; rr < 4; ++rr) {
+            const int r = r0 + rr;
+            float wt[kConsumerWarps];
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) wt[w] = __shfl_sync(0xffffffffu, rw[w], r & 31);
+            const float L = __shfl_sync(0xffffffffu, rL, r & 31);
+            if (r < G) {
+              float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+              for (int w = 0; w < kConsumerWarps; ++w) {
+                O.x += wt[w] * x[rr][w].x;
+                O.y += wt[w] * x[rr][w].y;
+                O.z += wt[w] * x[rr][w].z;
+                O.w += wt[w] * x[rr][w].w;
+              }
+              if (single) {
+                const float inv = 1.f / L;
+                store_bf16x4(out_h + r * kHeadDim + d4, O.x * inv, O.y * inv, O.z * inv, O.w * inv);
+              } else {
+                *reinterpret_cast<float4*>(rec + 2 * kMaxGroup + r * kHeadDim + d4) = O;
+              }
             }
           }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&mempty_bar[slot]);  // the slot may be refilled
         if (!single) {
-          __threadfence();
+          // Publish this record and count the arrival in one acquire-release atomic
+          // (the warp barrier orders every lane's record stores before it).
           __syncwarp();
           int is_last = 0;
-          if (lane == 0) is_last = (atomicAdd(p.piece_counters + h, 1) == k_hi - k_lo) ? 1 : 0;
+          if (lane == 0) is_last = (atomic_add_acq_rel(p.piece_counters + h, 1) == k_hi - k_lo) ? 1 : 0;
           is_last = __shfl_sync(0xffffffffu, is_last, 0);
+          __syncwarp();
           if (is_last) {
-            // Last CTA of this head: online log-sum-exp merge of all records, in
-            // CTA order, eight rows at a time; every load of one record for eight
-            // rows is issued together.
-            __threadfence();
+            // Last CTA of this head: online log-sum-exp merge of all records in CTA
+            // order, eight rows at a time; the loads of the next record are in
+            // flight while the current one is merged.
             for (int r0 = 0; r0 < G; r0 += 8) {
               float Mr[8], Lr[8];
               float4 Or[8];
@@ -549,31 +634,42 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
                 Lr[r] = 0.f;
                 Or[r] = make_float4(0.f, 0.f, 0.f, 0.f);
               }
-              for (int kk = k_lo; kk <= k_hi; ++kk) {
+              float mA[8], lA[8], mB[8], lB[8];
+              float4 oA[8], oB[8];
+              auto load = [&](float (&m)[8], float (&l)[8], float4 (&o)[8], int kk) {
                 const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
-                float mk[8], lk[8];
-                float4 ok[8];
 #pragma unroll
                 for (int r = 0; r < 8; ++r) {
                   if (r0 + r < G) {
-                    mk[r] = __ldcg(rk + r0 + r);
-                    lk[r] = __ldcg(rk + kMaxGroup + r0 + r);
-                    ok[r] = __ldcg(reinterpret_cast<const float4*>(rk + 2 * kMaxGroup +
-                                                                   (r0 + r) * kHeadDim + d4));
+                    m[r] = __ldcg(rk + r0 + r);
+                    l[r] = __ldcg(rk + kMaxGroup + r0 + r);
+                    o[r] = __ldcg(reinterpret_cast<const float4*>(rk + 2 * kMaxGroup +
+                                                                  (r0 + r) * kHeadDim + d4));
                   }
                 }
+              };
+              auto merge = [&](const float (&m)[8], const float (&l)[8], const float4 (&o)[8]) {
 #pragma unroll
                 for (int r = 0; r < 8; ++r) {
                   if (r0 + r < G) {
-                    const float Mn = fmaxf(Mr[r], mk[r]);
-                    const float a = exp2f(Mr[r] - Mn), bw = exp2f(mk[r] - Mn);
-                    Lr[r] = Lr[r] * a + lk[r] * bw;
-                    Or[r].x = Or[r].x * a + ok[r].x * bw;
-                    Or[r].y = Or[r].y * a + ok[r].y * bw;
-                    Or[r].z = Or[r].z * a + ok[r].z * bw;
-                    Or[r].w = Or[r].w * a + ok[r].w * bw;
+                    const float Mn = fmaxf(Mr[r], m[r]);
+                    const float a = exp2f(Mr[r] - Mn), bw = exp2f(m[r] - Mn);
+                    Lr[r] = Lr[r] * a + l[r] * bw;
+                    Or[r].x = Or[r].x * a + o[r].x * bw;
+                    Or[r].y = Or[r].y * a + o[r].y * bw;
+                    Or[r].z = Or[r].z * a + o[r].z * bw;
+                    Or[r].w = Or[r].w * a + o[r].w * bw;
                     Mr[r] = Mn;
                   }
+                }
+              };
+              load(mA, lA, oA, k_lo);
+              for (int kk = k_lo; kk <= k_hi; kk += 2) {
+                if (kk + 1 <= k_hi) load(mB, lB, oB, kk + 1);
+                merge(mA, lA, oA);
+                if (kk + 1 <= k_hi) {
+                  if (kk + 2 <= k_hi) load(mA, lA, oA, kk + 2);
+                  merge(mB, lB, oB);
                 }
               }
 #pragma unroll
