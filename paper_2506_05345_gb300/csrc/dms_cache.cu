@@ -163,6 +163,7 @@ dms_status dms_cache_reset(dms_cache* h, void* stream) {
       cudaMemsetAsync(c.piece_counters, 0, sizeof(int32_t) * (size_t)c.heads, st) != cudaSuccess)
     return DMS_ERR_CUDA;
   for (int l = 0; l < c.layers; ++l) c.lengths[l] = 0;
+  c.last_layer = -1;
   return DMS_OK;
 }
 
@@ -182,6 +183,7 @@ dms_status dms_append_and_evict(dms_cache* h, int32_t layer, const void* k, cons
                             : dms::launch_append_bulk(c, layer, k, v, decision_logit, t0, n_tokens, st);
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = t0 + n_tokens;
+  c.last_layer = layer;
   return DMS_OK;
 }
 
@@ -199,7 +201,9 @@ dms_status dms_decode_attention(dms_cache* h, int32_t layer, const void* q, void
     e = dms::launch_decode_simple(c, layer, q, out, gqa_group, scale, st);
   else
     e = dms::launch_decode_tiled(c, layer, q, out, gqa_group, scale * 1.4426950408889634f, st);
-  return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+  if (e != cudaSuccess) return DMS_ERR_CUDA;
+  c.last_layer = layer;
+  return DMS_OK;
 }
 
 dms_status dms_append_and_decode(dms_cache* h, int32_t layer, const void* k, const void* v,
@@ -225,6 +229,7 @@ dms_status dms_append_and_decode(dms_cache* h, int32_t layer, const void* k, con
                                 scale * 1.4426950408889634f, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = t0 + 1;
+  c.last_layer = layer;
   return DMS_OK;
 }
 

@@ -87,6 +87,11 @@ struct DecodeParams {
   int32_t* pos;
   int64_t j, window, pool_pages;
   int32_t ring_len;
+  // Nonzero when the kernel launched just before on the stream cannot have written
+  // this layer's cache state (it served another layer): the state is read, and the
+  // first pages are staged, before waiting for that kernel; only the inputs (q, the
+  // new K/V rows, the logits), the outputs and the shared split-K scratch wait.
+  int32_t state_ready;
 };
 
 // ---------------------------------------------------------------- PTX wrappers
@@ -311,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   int* s_misc = reinterpret_cast<int*>(mempty_bar + PL::kSlots);
   int32_t* s_cnt = s_misc + 16;                                   // [heads] n_h (after the append)
   int32_t* s_pstart = s_cnt + p.heads;                            // [heads + 1]
-  // fused: new token's slot | fresh << 30 | alpha << 31 per head
+  // fused: new token's slot | fresh << 30 per head
   uint32_t* s_slot = reinterpret_cast<uint32_t*>(s_pstart + p.heads + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -359,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
       }
     }
   }
-  pdl_wait_prerequisites();
+  if (!p.state_ready) pdl_wait_prerequisites();
   {
     // Per-head state, with every load of a batch issued before any is used.  In the
     // fused variant: delayed eviction for position j (Sec. 3.1-3.2) -- the token
@@ -372,16 +377,12 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     for (int base = 0; base < heads; base += kThreads * kPer) {
       int32_t nn[kPer];
       uint32_t ee[kPer];
-      uint16_t ll[kPer];
 #pragma unroll
       for (int i = 0; i < kPer; ++i) {
         const int h = base + tid + i * kThreads;
         if (h < heads) {
           nn[i] = p.counts[h];
-          if constexpr (kFused) {
-            ee[i] = p.j >= R ? p.ring[(int64_t)h * p.ring_len + (p.j - R) % RP] : 0u;
-            ll[i] = p.logit_new[h];
-          }
+          if constexpr (kFused) ee[i] = p.j >= R ? p.ring[(int64_t)h * p.ring_len + (p.j - R) % RP] : 0u;
         }
       }
 #pragma unroll
@@ -393,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
             const uint32_t slot = reuse ? (ee[i] & kSlotMask) : (uint32_t)nn[i];
             const uint32_t fresh = reuse ? 0u : 1u;
             s_cnt[h] = nn[i] + (int32_t)fresh;
-            s_slot[h] = slot | (fresh << 30) | (decision_from_bf16(ll[i]) << 31);
+            s_slot[h] = slot | (fresh << 30);
           } else {
             s_cnt[h] = nn[i];
           }
@@ -426,14 +427,15 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   __syncthreads();
   const int N = s_pstart[heads];
 
-  // Heads with no tokens yet produce zeros (spread over the CTAs).
-  for (int h = blockIdx.x; h < heads; h += gridDim.x) {
-    if (s_cnt[h] != 0) continue;
-    const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
-    __nv_bfloat16* o = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
-    for (int i = tid; i < G * kHeadDim; i += kThreads) o[i] = __float2bfloat16_rn(0.f);
+  if (N == 0) {  // nothing appended yet: every output is zero
+    if (p.state_ready) pdl_wait_prerequisites();
+    for (int h = blockIdx.x; h < heads; h += gridDim.x) {
+      const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
+      __nv_bfloat16* o = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+      for (int i = tid; i < G * kHeadDim; i += kThreads) o[i] = __float2bfloat16_rn(0.f);
+    }
+    return;
   }
-  if (N == 0) return;
   int P = N / (p.min_pages > 0 ? p.min_pages : 1);
   if (P < 1) P = 1;
   if (P > (int)gridDim.x) P = (int)gridDim.x;
@@ -460,6 +462,42 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   if (warp == kProducerWarp) {
     // ================================================================ producer warp
     int issued = 0;
+    // With ready state, the first kStages pages are staged before the dependency
+    // wait; their input copies (queries, new K/V rows) and the ring entries, which
+    // read inputs, are issued once the previous kernel has completed.
+    bool waited = !p.state_ready;
+    int d_s[kStages], d_h[kStages], d_pg[kStages], d_flags[kStages];
+    int nd = 0;
+    auto issue_inputs = [&](int s, int h_i, int pg_i, bool seg_start, bool patch) {
+      uint8_t* st = stages + s * kStageBytes;
+      if (seg_start) {
+        const int b = h_i / p.kv_heads, hk = h_i - b * p.kv_heads;
+        const __nv_bfloat16* qsrc = p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+        bulk_copy_g2s(st + 2 * kHalfPageBytes, qsrc, (uint32_t)G * kRowBytes, &full_bar[s]);
+      }
+      if constexpr (kFused) {
+        if (patch) {  // the new token's K and V rows, as given (unpermuted)
+          bulk_copy_g2s(st + kStageBytesPlain, p.k_new + (int64_t)h_i * kHeadDim, kRowBytes,
+                        &full_bar[s]);
+          bulk_copy_g2s(st + kStageBytesPlain + kRowBytes, p.v_new + (int64_t)h_i * kHeadDim,
+                        kRowBytes, &full_bar[s]);
+        }
+        if (pg_i == s_pstart[h_i + 1] - s_pstart[h_i] - 1) {  // owner of the head's last page
+          const uint32_t sl = s_slot[h_i] & 0x3fffffffu;
+          const uint32_t alpha = decision_from_bf16(p.logit_new[h_i]);
+          p.counts_next[h_i] = s_cnt[h_i];
+          p.ring[(int64_t)h_i * p.ring_len + p.j % ring_period(p.window)] = sl | (alpha << 31);
+        }
+      }
+    };
+    auto finish_wait = [&]() {
+      if (waited) return;
+      pdl_wait_prerequisites();
+      waited = true;
+      for (int d = 0; d < nd; ++d)
+        issue_inputs(d_s[d], d_h[d], d_pg[d], (d_flags[d] & 1) != 0, (d_flags[d] & 2) != 0);
+      nd = 0;
+    };
     for (int it0 = 0; it0 < niters; it0 += 32) {
       const int it = it0 + lane;
       int hh = 0, pg = 0, nv = 0, page = 0;
@@ -496,40 +534,37 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
           const int itg = it0 + i;
           const int s = itg % kStages;
           const int use = itg / kStages;
-          if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.ctrl);
+          if (use > 0) {
+            finish_wait();
+            mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.ctrl);
+          }
           const bool seg_start = (itg == 0) || (pg_i == 0);
           const uint32_t kv_bytes = (uint32_t)nv_i * kRowBytes;
           const uint32_t q_bytes = seg_start ? (uint32_t)G * kRowBytes : 0u;
           uint8_t* st = stages + s * kStageBytes;
           bool patch = false;
           if constexpr (kFused) {
-            const uint32_t sl = s_slot[h_i];
-            patch = (int32_t)(sl & 0x3fffffffu) / kPageTokens == pg_i;
+            patch = (int32_t)(s_slot[h_i] & 0x3fffffffu) / kPageTokens == pg_i;
             s_misc[8 + s] = page_i;
-            if (pg_i == s_pstart[h_i + 1] - s_pstart[h_i] - 1) {  // owner of the head's last page
-              p.counts_next[h_i] = s_cnt[h_i];
-              p.ring[(int64_t)h_i * p.ring_len + p.j % ring_period(p.window)] = sl & ~(1u << 30);
-            }
           }
           mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + q_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
           const uint8_t* src = p.pool + (int64_t)(page_i < 0 ? 0 : page_i) * kPageBytes;
           bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
           bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
-          if (seg_start) {
-            const int b = h_i / p.kv_heads, hk = h_i - b * p.kv_heads;
-            const __nv_bfloat16* qsrc = p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
-            bulk_copy_g2s(st + 2 * kHalfPageBytes, qsrc, q_bytes, &full_bar[s]);
-          }
-          if (patch) {  // fused: the new token's K and V rows, as given (unpermuted)
-            bulk_copy_g2s(st + kStageBytesPlain, p.k_new + (int64_t)h_i * kHeadDim, kRowBytes,
-                          &full_bar[s]);
-            bulk_copy_g2s(st + kStageBytesPlain + kRowBytes, p.v_new + (int64_t)h_i * kHeadDim,
-                          kRowBytes, &full_bar[s]);
+          if (waited) {
+            issue_inputs(s, h_i, pg_i, seg_start, patch);
+          } else {
+            d_s[nd] = s;
+            d_h[nd] = h_i;
+            d_pg[nd] = pg_i;
+            d_flags[nd] = (seg_start ? 1 : 0) | (patch ? 2 : 0);
+            ++nd;
           }
           ++issued;
         }
       }
     }
+    if (lane == 0) finish_wait();  // fewer pages than stages
     // Drain: do not leave while a bulk copy may still be writing shared memory.
     if (lane == 0) {
       for (int s = 0; s < kStages && s < issued; ++s) {
@@ -542,6 +577,15 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
 
   if (warp == kEpilogueWarp) {
     // ================================================================ epilogue warp
+    // Everything it writes (outputs, records, counters) may be read by the previous
+    // kernel until that completes.
+    if (p.state_ready) pdl_wait_prerequisites();
+    for (int h = k; h < heads; h += P) {  // heads with no tokens yet produce zeros
+      if (s_cnt[h] != 0) continue;
+      const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
+      __nv_bfloat16* o = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+      for (int i = lane; i < G * kHeadDim; i += 32) o[i] = __float2bfloat16_rn(0.f);
+    }
     int q = 0;  // segment counter
     for (int it = 0; it < niters; ++it) {
       walk.enter(it);
@@ -1024,6 +1068,7 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
 DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* out, int32_t group,
                           float scale_log2) {
   DecodeParams p = {};
+  p.state_ready = (c.last_layer != layer) ? 1 : 0;
   p.pool = c.pool;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
   p.counts = c.counts_at(layer, c.lengths[layer]);

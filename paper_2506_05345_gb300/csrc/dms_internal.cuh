@@ -77,6 +77,9 @@ struct Cache {
 
   int64_t* lengths = nullptr;  // host: tokens appended per layer
   int64_t peak_pages = 0;      // host: largest pages_in_use observed
+  // host: layer of the last kernel launched on this cache (-1: none since creation or
+  // reset).  A launch for another layer cannot depend on that kernel's cache writes.
+  int32_t last_layer = -1;
 
   // Count buffer of `layer` for a layer length of parity `parity`.
   int32_t* counts_at(int32_t layer, int64_t parity) const {

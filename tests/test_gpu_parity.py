@@ -301,3 +301,57 @@ def test_reset_and_reuse():
         assert r.cache.stats()["peak_pages"] > 0
     finally:
         r.close()
+
+
+@pytest.mark.parametrize("fused", [True, False])
+def test_multilayer_interleaved_steps(fused):
+    """Three layers advanced together, as a model decodes: each step visits layer 0, 1, 2.
+    Consecutive launches serve different layers, so the fused kernel reads the layer's state
+    and stages its first pages before waiting for the previous launch."""
+    import oracle
+    from _harness import MAX_ABS, MEAN_ABS
+    L, B, Hkv, G, w, P, steps = 3, 2, 2, 4, 24, 500, 12
+    wl = small(batch=B, kv_heads=Hkv, q_heads=Hkv * G, window=w)
+    dev = torch.device("cuda")
+    cache = dms.DmsCache(layers=L, kv_heads=Hkv, window=w, capacity=P + steps, batch=B)
+    hist = []
+    try:
+        for l in range(L):
+            k, v, lg = workloads.gen_kv(wl, l, "prefill", P, dev, p_override=[0.6 + 0.1 * l] * Hkv)
+            cache.append_and_evict(l, k, v, lg)
+            hist.append([k, v, lg])
+        errs = []
+        for s_ in range(steps):
+            outs = []
+            for l in range(L):
+                k, v, lg = workloads.gen_kv(wl, l, f"d{s_}", 1, dev)
+                q = workloads.gen_q(wl, l, f"d{s_}", dev)  # written right before the call
+                if fused:
+                    out = cache.append_and_decode(l, k, v, lg, q, gqa_group=G)
+                else:
+                    cache.append_and_evict(l, k, v, lg)
+                    out = cache.decode_attention(l, q, gqa_group=G)
+                for i, t in enumerate((k, v, lg)):
+                    hist[l][i] = torch.cat([hist[l][i], t], 1)
+                outs.append((q, out))
+            if s_ % 3 == 2 or s_ == steps - 1:
+                j = P + s_
+                for l, (q, out) in enumerate(outs):
+                    K, V, LG = (workloads.bf16_bits(t) for t in hist[l])
+                    Q = workloads.bf16_bits(q)
+                    got = out.float().cpu().numpy()
+                    for b in range(B):
+                        for h in range(Hkv):
+                            ref = oracle.decode(Q[b, h * G:(h + 1) * G], K[b, :, h], V[b, :, h],
+                                                LG[b, :, h], j, w)
+                            errs.append(np.abs(got[b, h * G:(h + 1) * G] - ref).ravel())
+                    pos = cache.export_positions(l)
+                    for b in range(B):
+                        for h in range(Hkv):
+                            have = np.sort(pos[b, h][pos[b, h] >= 0])
+                            assert np.array_equal(have, oracle.retained(LG[b, :, h], j, w)), (l, b, h)
+        e = np.concatenate(errs)
+        assert e.max() <= MAX_ABS and e.mean() <= MEAN_ABS, (e.max(), e.mean())
+        assert cache.stats()["device_error"] == 0
+    finally:
+        cache.close()
