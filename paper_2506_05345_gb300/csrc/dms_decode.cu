@@ -17,11 +17,16 @@
 //     O^T += V^T P^T (8 mma.sync); P^T is formed from S^T in registers with
 //     movmatrix.  fp32 online softmax in the exp2 domain; S^T and O^T share their
 //     column (head) layout, so the running rescale needs no shuffles;
-//   * an epilogue warp finishes each head segment while the consumers move on:
-//     it merges the four warp partials from a double-buffered shared-memory slot,
-//     writes the output of a head the CTA covers alone, or writes a partial record
-//     (m, l, O); the last CTA to arrive on a split head's counter merges all
-//     records (log-sum-exp combine) and writes the output.
+//   * an epilogue warp finishes each head segment but the CTA's last while the
+//     consumers move on: it merges the four warp partials from a double-buffered
+//     shared-memory slot, writes the output of a head the CTA covers alone, or
+//     writes a partial record (m, l, O); the last CTA to arrive on a split head's
+//     counter merges all records (log-sum-exp combine) and writes the output.
+//     The CTA's last segment has nothing left to overlap with, so the four
+//     consumer warps finish it themselves, each merging a quarter of the query
+//     heads; when every other CTA of a split last head has already counted its
+//     record (read while the last page is in flight), they merge those records
+//     straight away instead of publishing their own.
 // A CTA takes its pages in the order: its first head's part, its last head's part
 // (the two it may share with neighbours), then the heads in between, so the
 // cross-CTA combines happen early and the CTA ends on directly written heads.
@@ -217,6 +222,20 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // Four consecutive bf16 outputs (round to nearest even) with one 8-byte store.
 __device__ __forceinline__ void store_bf16x4(__nv_bfloat16* dst, float a, float b, float c, float d) {
   *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(a, b), pack_bf16x2(c, d));
+}
+
+// Relaxed GPU-scope load (no ordering); paired with fence.acq_rel.gpu once its
+// value is acted on, it forms an acquire.
+__device__ __forceinline__ int ld_relaxed_gpu(const int32_t* addr) {
+  int v;
+  asm volatile("ld.relaxed.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(addr) : "memory");
+  return v;
+}
+
+// Barrier of the four consumer warps only (named barrier 1; barrier 0 is the
+// CTA-wide __syncthreads).
+__device__ __forceinline__ void consumer_bar_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kConsumerWarps * 32) : "memory");
 }
 
 // Programmatic dependent launch: let the next kernel of the stream start its
@@ -587,7 +606,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
       for (int i = lane; i < G * kHeadDim; i += 32) o[i] = __float2bfloat16_rn(0.f);
     }
     int q = 0;  // segment counter
-    for (int it = 0; it < niters; ++it) {
+    // The CTA's last segment is finished by the consumer warps themselves.
+    for (int it = 0; it < niters - 1; ++it) {
       walk.enter(it);
       if (walk.seg_end(it, niters)) {
         const int h = walk.h;
@@ -743,6 +763,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   float o[8][NT][4];         // O^T accumulators: (d = 16 mt + g (+8), heads 8 nt + 2c, +1)
   float me[NT], mo[NT], le[NT], lo[NT];  // running max / sum of heads 8 nt + 2c and + 1
   int q = 0;
+  // Arrivals on the last segment's head, read while its last page is in flight: if
+  // every other CTA of a split head has already arrived, this CTA merges their
+  // records directly, without publishing its own.
+  int arrivals_seen = -1;
 
   for (int it = 0; it < niters; ++it) {
     walk.enter(it);
@@ -752,6 +776,9 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     const bool seg_start = walk.seg_start(it);
     const bool seg_end = walk.seg_end(it, niters);
     uint8_t* st = stages + s * kStageBytes;
+    if (it == niters - 1 && tid == 0 &&
+        split.cta_of(s_pstart[walk.h]) != split.cta_of(s_pstart[walk.h + 1] - 1))
+      arrivals_seen = ld_relaxed_gpu(p.piece_counters + walk.h);
     mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
 
     if constexpr (kFused) {
@@ -919,9 +946,158 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
           so[ho * kMergeRow + 16 * mt + g + 8] = o[mt][nt][3];
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&mfull_bar[slot]);
-      ++q;
+      if (it != niters - 1) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&mfull_bar[slot]);
+        ++q;
+      } else {
+        // ---- the CTA's last segment: nothing is left to stream, so the four warps
+        // finish it together: warp w merges query-head rows w, w + 4, ..., lane l
+        // head_dim columns 4 l .. 4 l + 3.
+        const int h = walk.h;
+        const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
+        const int k_lo = split.cta_of(s_pstart[h]), k_hi = split.cta_of(s_pstart[h + 1] - 1);
+        const bool single = (k_lo == k_hi);
+        if (tid == 0) {
+          int early = 0;
+          if (!single && arrivals_seen == k_hi - k_lo) {
+            asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
+            early = 1;
+          }
+          s_misc[1] = early;
+        }
+        consumer_bar_sync();
+        const bool early_last = s_misc[1] != 0;
+        constexpr int RPW = HP / kConsumerWarps;  // rows per warp
+        const int d4 = 4 * lane;
+        __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+        const float* mo_all = merge_o + slot * PL::kSlotOFloats;
+        const float* ml_all = merge_ml + slot * PL::kSlotMLFloats;
+        float Mo[RPW], Lo[RPW];
+        float4 Oo[RPW];
+#pragma unroll
+        for (int i = 0; i < RPW; ++i) {
+          const int r = warp + kConsumerWarps * i;
+          Mo[i] = -INFINITY;
+          Lo[i] = 0.f;
+          Oo[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (r < G) {
+            float mw[kConsumerWarps];
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) {
+              mw[w] = ml_all[(w * HP + r) * 2];
+              Mo[i] = fmaxf(Mo[i], mw[w]);
+            }
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) {
+              const float a = exp2f(mw[w] - Mo[i]);
+              const float4 x = *reinterpret_cast<const float4*>(mo_all + (w * HP + r) * kMergeRow + d4);
+              Lo[i] += a * ml_all[(w * HP + r) * 2 + 1];
+              Oo[i].x += a * x.x;
+              Oo[i].y += a * x.y;
+              Oo[i].z += a * x.z;
+              Oo[i].w += a * x.w;
+            }
+          }
+        }
+        if (single) {
+#pragma unroll
+          for (int i = 0; i < RPW; ++i) {
+            const int r = warp + kConsumerWarps * i;
+            if (r < G) {
+              const float inv = 1.f / Lo[i];
+              store_bf16x4(out_h + r * kHeadDim + d4, Oo[i].x * inv, Oo[i].y * inv, Oo[i].z * inv,
+                           Oo[i].w * inv);
+            }
+          }
+        } else {
+          bool last = early_last;
+          if (!last) {
+            // Publish this CTA's record GPU-wide and count it.
+            float* rec = p.pieces + (int64_t)(k + h) * kPieceFloats;  // m[16] l[16] o[16][128]
+#pragma unroll
+            for (int i = 0; i < RPW; ++i) {
+              const int r = warp + kConsumerWarps * i;
+              if (r < G) {
+                *reinterpret_cast<float4*>(rec + 2 * kMaxGroup + r * kHeadDim + d4) = Oo[i];
+                if (lane == 0) {
+                  rec[r] = Mo[i];
+                  rec[kMaxGroup + r] = Lo[i];
+                }
+              }
+            }
+            __threadfence();
+            consumer_bar_sync();
+            if (tid == 0)
+              s_misc[1] = (atomic_add_acq_rel(p.piece_counters + h, 1) == k_hi - k_lo) ? 1 : 0;
+            consumer_bar_sync();
+            last = s_misc[1] != 0;
+          }
+          if (last) {
+            // Log-sum-exp merge of every CTA's part in CTA order (this CTA's from
+            // registers); the loads of the next record are in flight while the
+            // current one is merged.
+            float Mr[RPW], Lr[RPW], mA[RPW], lA[RPW], mB[RPW], lB[RPW];
+            float4 Or[RPW], oA[RPW], oB[RPW];
+#pragma unroll
+            for (int i = 0; i < RPW; ++i) {
+              Mr[i] = -INFINITY;
+              Lr[i] = 0.f;
+              Or[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            auto load = [&](float (&m)[RPW], float (&l)[RPW], float4 (&o)[RPW], int kk) {
+              const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
+#pragma unroll
+              for (int i = 0; i < RPW; ++i) {
+                const int r = warp + kConsumerWarps * i;
+                if (kk == k) {
+                  m[i] = Mo[i];
+                  l[i] = Lo[i];
+                  o[i] = Oo[i];
+                } else if (r < G) {
+                  m[i] = __ldcg(rk + r);
+                  l[i] = __ldcg(rk + kMaxGroup + r);
+                  o[i] = __ldcg(reinterpret_cast<const float4*>(rk + 2 * kMaxGroup + r * kHeadDim + d4));
+                }
+              }
+            };
+            auto merge = [&](const float (&m)[RPW], const float (&l)[RPW], const float4 (&o)[RPW]) {
+#pragma unroll
+              for (int i = 0; i < RPW; ++i) {
+                if (warp + kConsumerWarps * i < G) {
+                  const float Mn = fmaxf(Mr[i], m[i]);
+                  const float a = exp2f(Mr[i] - Mn), bw = exp2f(m[i] - Mn);
+                  Lr[i] = Lr[i] * a + l[i] * bw;
+                  Or[i].x = Or[i].x * a + o[i].x * bw;
+                  Or[i].y = Or[i].y * a + o[i].y * bw;
+                  Or[i].z = Or[i].z * a + o[i].z * bw;
+                  Or[i].w = Or[i].w * a + o[i].w * bw;
+                  Mr[i] = Mn;
+                }
+              }
+            };
+            load(mA, lA, oA, k_lo);
+            for (int kk = k_lo; kk <= k_hi; kk += 2) {
+              if (kk + 1 <= k_hi) load(mB, lB, oB, kk + 1);
+              merge(mA, lA, oA);
+              if (kk + 1 <= k_hi) {
+                if (kk + 2 <= k_hi) load(mA, lA, oA, kk + 2);
+                merge(mB, lB, oB);
+              }
+            }
+#pragma unroll
+            for (int i = 0; i < RPW; ++i) {
+              const int r = warp + kConsumerWarps * i;
+              if (r < G) {
+                const float inv = 1.f / Lr[i];
+                store_bf16x4(out_h + r * kHeadDim + d4, Or[i].x * inv, Or[i].y * inv, Or[i].z * inv,
+                             Or[i].w * inv);
+              }
+            }
+            if (tid == 0) p.piece_counters[h] = 0;
+          }
+        }
+      }
     }
     walk.advance();
   }
