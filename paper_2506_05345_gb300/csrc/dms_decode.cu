@@ -263,6 +263,30 @@ struct Split {
   }
 };
 
+// Page partition over P CTAs.  Launched behind another kernel, the CTAs with the
+// highest indices are placed last (on the SMs that kernel frees last) and start
+// streaming a few microseconds late: the last kTaperCtas CTAs share their pages at
+// kTaperPermille / 1000 of the others' weight.  Small launches split evenly.
+constexpr int kTaperCtas = 16;
+constexpr int kTaperPermille = 900;
+struct Partition {
+  Split a, b;
+  int P1, N1;  // CTAs [0, P1) own pages [0, N1) (split a); the rest split b
+  __device__ __forceinline__ void init(int N, int P) {
+    P1 = P;
+    N1 = N;
+    if (kTaperCtas > 0 && P > 4 * kTaperCtas && N >= 8 * P) {
+      P1 = P - kTaperCtas;
+      N1 = (int)((int64_t)N * P1 * 1000 / ((int64_t)P1 * 1000 + (int64_t)kTaperCtas * kTaperPermille));
+    }
+    a = Split{N1 / P1, N1 % P1};
+    const int T = P - P1, N2 = N - N1;
+    b = Split{T > 0 ? N2 / T : 0, T > 0 ? N2 % T : 0};
+  }
+  __device__ __forceinline__ int begin(int k) const { return k <= P1 ? a.begin(k) : N1 + b.begin(k - P1); }
+  __device__ __forceinline__ int cta_of(int x) const { return x < N1 ? a.cta_of(x) : P1 + b.cta_of(x - N1); }
+};
+
 // Last head h with pstart[h] <= x (x < pstart[heads]).
 __device__ __forceinline__ int head_of_page(const int32_t* pstart, int heads, int x) {
   int lo = 0, hi = heads;
@@ -460,7 +484,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
   if (P > (int)gridDim.x) P = (int)gridDim.x;
   const int k = blockIdx.x;
   if (k >= P) return;
-  const Split split{N / P, N % P};
+  Partition split;
+  split.init(N, P);
   const int pbeg = split.begin(k), pend = split.begin(k + 1);
   const int niters = pend - pbeg;
   PageWalk walk;
@@ -1035,54 +1060,52 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
           }
           if (last) {
             // Log-sum-exp merge of every CTA's part in CTA order (this CTA's from
-            // registers); the loads of the next record are in flight while the
-            // current one is merged.
-            float Mr[RPW], Lr[RPW], mA[RPW], lA[RPW], mB[RPW], lB[RPW];
-            float4 Or[RPW], oA[RPW], oB[RPW];
+            // registers), four records' loads in flight at a time.
+            float Mr[RPW], Lr[RPW];
+            float4 Or[RPW];
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
               Mr[i] = -INFINITY;
               Lr[i] = 0.f;
               Or[i] = make_float4(0.f, 0.f, 0.f, 0.f);
             }
-            auto load = [&](float (&m)[RPW], float (&l)[RPW], float4 (&o)[RPW], int kk) {
-              const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
+            constexpr int kBatch = NT == 1 ? 4 : 2;
+            for (int kk0 = k_lo; kk0 <= k_hi; kk0 += kBatch) {
+              float mb[kBatch][RPW], lb[kBatch][RPW];
+              float4 ob[kBatch][RPW];
 #pragma unroll
-              for (int i = 0; i < RPW; ++i) {
-                const int r = warp + kConsumerWarps * i;
-                if (kk == k) {
-                  m[i] = Mo[i];
-                  l[i] = Lo[i];
-                  o[i] = Oo[i];
-                } else if (r < G) {
-                  m[i] = __ldcg(rk + r);
-                  l[i] = __ldcg(rk + kMaxGroup + r);
-                  o[i] = __ldcg(reinterpret_cast<const float4*>(rk + 2 * kMaxGroup + r * kHeadDim + d4));
+              for (int u = 0; u < kBatch; ++u) {
+                const int kk = kk0 + u;
+                const float* rk = p.pieces + (int64_t)(kk + h) * kPieceFloats;
+#pragma unroll
+                for (int i = 0; i < RPW; ++i) {
+                  const int r = warp + kConsumerWarps * i;
+                  if (kk == k) {
+                    mb[u][i] = Mo[i];
+                    lb[u][i] = Lo[i];
+                    ob[u][i] = Oo[i];
+                  } else if (kk <= k_hi && r < G) {
+                    mb[u][i] = __ldcg(rk + r);
+                    lb[u][i] = __ldcg(rk + kMaxGroup + r);
+                    ob[u][i] = __ldcg(reinterpret_cast<const float4*>(rk + 2 * kMaxGroup + r * kHeadDim + d4));
+                  }
                 }
               }
-            };
-            auto merge = [&](const float (&m)[RPW], const float (&l)[RPW], const float4 (&o)[RPW]) {
 #pragma unroll
-              for (int i = 0; i < RPW; ++i) {
-                if (warp + kConsumerWarps * i < G) {
-                  const float Mn = fmaxf(Mr[i], m[i]);
-                  const float a = exp2f(Mr[i] - Mn), bw = exp2f(m[i] - Mn);
-                  Lr[i] = Lr[i] * a + l[i] * bw;
-                  Or[i].x = Or[i].x * a + o[i].x * bw;
-                  Or[i].y = Or[i].y * a + o[i].y * bw;
-                  Or[i].z = Or[i].z * a + o[i].z * bw;
-                  Or[i].w = Or[i].w * a + o[i].w * bw;
-                  Mr[i] = Mn;
+              for (int u = 0; u < kBatch; ++u) {
+#pragma unroll
+                for (int i = 0; i < RPW; ++i) {
+                  if (kk0 + u <= k_hi && warp + kConsumerWarps * i < G) {
+                    const float Mn = fmaxf(Mr[i], mb[u][i]);
+                    const float a = exp2f(Mr[i] - Mn), bw = exp2f(mb[u][i] - Mn);
+                    Lr[i] = Lr[i] * a + lb[u][i] * bw;
+                    Or[i].x = Or[i].x * a + ob[u][i].x * bw;
+                    Or[i].y = Or[i].y * a + ob[u][i].y * bw;
+                    Or[i].z = Or[i].z * a + ob[u][i].z * bw;
+                    Or[i].w = Or[i].w * a + ob[u][i].w * bw;
+                    Mr[i] = Mn;
+                  }
                 }
-              }
-            };
-            load(mA, lA, oA, k_lo);
-            for (int kk = k_lo; kk <= k_hi; kk += 2) {
-              if (kk + 1 <= k_hi) load(mB, lB, oB, kk + 1);
-              merge(mA, lA, oA);
-              if (kk + 1 <= k_hi) {
-                if (kk + 2 <= k_hi) load(mA, lA, oA, kk + 2);
-                merge(mB, lB, oB);
               }
             }
 #pragma unroll
