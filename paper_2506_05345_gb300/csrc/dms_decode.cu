@@ -1051,7 +1051,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
                 }
               }
             }
-            __threadfence();
+            // The barrier orders every consumer thread's record stores before thread
+            // 0's acquire-release atomic, whose release covers them.
             consumer_bar_sync();
             if (tid == 0)
               s_misc[1] = (atomic_add_acq_rel(p.piece_counters + h, 1) == k_hi - k_lo) ? 1 : 0;
