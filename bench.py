@@ -57,6 +57,9 @@ def parse():
     ap.add_argument("--min-pages", type=int, default=0)
     ap.add_argument("--separate", action="store_true",
                     help="append and decode as two launches instead of the fused step")
+    ap.add_argument("--borrowed", action="store_true",
+                    help="decision logits carried by element 0 of each group's first query head "
+                         "(App. B) instead of a separate tensor")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (small cases for profiling)")
     return ap.parse_args()
@@ -276,6 +279,8 @@ def run_ours(args, wl, world, rank, local, pg):
         for layer in range(L):
             k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}decode{s}", 1, dev)
             q = workloads.gen_q(wl, layer, f"{seed_tag}decode{s}", dev)
+            if args.borrowed:  # the same decisions, carried by the borrowed neuron
+                q[:, ::G, 0] = lg[:, 0]
             per.append((k, v, lg, q))
         ins.append(per)
     outs = [torch.empty((B, Hq, D), dtype=torch.bfloat16, device=dev) for _ in range(L)]
@@ -291,18 +296,26 @@ def run_ours(args, wl, world, rank, local, pg):
     lib = dms.library()
     vp = ctypes.c_void_p
     hnd, sptr = vp(cache.handle), vp(stream.cuda_stream)
+
+    def step_calls(layer, kp, vp_, lp, qp, op):
+        """One layer's decode step as a tuple of (C function, arguments)."""
+        if args.borrowed and args.separate:
+            return ((lib.dms_append_and_evict_borrowed, (hnd, layer, kp, vp_, qp, 1, G, sptr)),
+                    (lib.dms_decode_attention_borrowed, (hnd, layer, qp, op, G, 0.0, sptr)))
+        if args.borrowed:
+            return ((lib.dms_append_and_decode_borrowed,
+                     (hnd, layer, kp, vp_, qp, op, G, 0.0, sptr)),)
+        if args.separate:
+            return ((lib.dms_append_and_evict, (hnd, layer, kp, vp_, lp, 1, sptr)),
+                    (lib.dms_decode_attention, (hnd, layer, qp, op, G, 0.0, sptr)))
+        return ((lib.dms_append_and_decode, (hnd, layer, kp, vp_, lp, qp, op, G, 0.0, sptr)),)
     calls = []
     for s in range(n_dev_steps):
         per = []
         for layer in range(L):
             k, v, lg, q = ins[s][layer]
             kp, vp_, lp, qp, op = (vp(t.data_ptr()) for t in (k, v, lg, q, outs[layer]))
-            if args.separate:
-                per.append(((lib.dms_append_and_evict, (hnd, layer, kp, vp_, lp, 1, sptr)),
-                            (lib.dms_decode_attention, (hnd, layer, qp, op, G, 0.0, sptr))))
-            else:
-                per.append(((lib.dms_append_and_decode,
-                             (hnd, layer, kp, vp_, lp, qp, op, G, 0.0, sptr)),))
+            per.append(step_calls(layer, kp, vp_, lp, qp, op))
         calls.append(per)
     codes = []
 
@@ -409,6 +422,8 @@ def run_ours(args, wl, world, rank, local, pg):
             vv = np.concatenate(hist[(b, h)]["v"])
             ll = np.concatenate(hist[(b, h)]["l"])
             qq = q_last[b, h * Gs:(h + 1) * Gs]
+            if args.borrowed:  # the attention takes the borrowed element as 0 (App. B)
+                qq = oracle.borrowed(qq, Gs)[1]
             ref = oracle.decode(qq, kk, vv, ll, j, wl.window)
             errs.append(np.abs(got[b, h * Gs:(h + 1) * Gs] - ref).ravel())
             cases.append((qq, kk, vv, ll, len(oracle.retained(ll, j, wl.window))))
@@ -450,6 +465,8 @@ def run_ours(args, wl, world, rank, local, pg):
             for layer in range(L):
                 k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}e2e{s}", 1, dev)
                 q = workloads.gen_q(wl, layer, f"{seed_tag}e2e{s}", dev)
+                if args.borrowed:
+                    q[:, ::G, 0] = lg[:, 0]
                 row = host_in[s, layer]
                 for off, t in ((o_k, k), (o_v, v), (o_l, lg), (o_q, q)):
                     b = t.reshape(-1).view(torch.uint8)
@@ -469,12 +486,7 @@ def run_ours(args, wl, world, rank, local, pg):
                 lb0 = base + layer * slab
                 kp, vp_, lp, qp = (vp(lb0 + o) for o in (o_k, o_v, o_l, o_q))
                 op = vp(dev_out[i][layer].data_ptr())
-                if args.separate:
-                    per.append(((lib.dms_append_and_evict, (hnd, layer, kp, vp_, lp, 1, sptr)),
-                                (lib.dms_decode_attention, (hnd, layer, qp, op, G, 0.0, sptr))))
-                else:
-                    per.append(((lib.dms_append_and_decode,
-                                 (hnd, layer, kp, vp_, lp, qp, op, G, 0.0, sptr)),))
+                per.append(step_calls(layer, kp, vp_, lp, qp, op))
             e_calls.append(per)
         up, down = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         ev = lambda: torch.cuda.Event()  # noqa: E731
@@ -551,8 +563,10 @@ def run_ours(args, wl, world, rank, local, pg):
                          f"{units_per_launch * bytes_per_unit / 1e6:.0f} MB x {L} layers rotate, "
                          "larger than the 129 MB L2",
                    "parallelism": f"replicas x{world}"},
-        "step_mode": "separate append + decode launches" if args.separate else
-                     "fused single-token append + decode, one launch per layer",
+        "step_mode": ("separate append + decode launches" if args.separate else
+                      "fused single-token append + decode, one launch per layer") +
+                     ("; decisions from element 0 of each group's first query head (App. B)"
+                      if args.borrowed else ""),
         "decode_us_per_layer_step": dec_avg_s * 1e6,
         "isolated_launch_us": float(np.mean(dec_ms)) * 1e3,
         "append_us_per_layer_step": (float(np.mean(app_ms)) * 1e3 if args.separate else None),

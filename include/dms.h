@@ -156,6 +156,33 @@ dms_status dms_append_and_decode(dms_cache* cache, int32_t layer, const void* k,
                                  int32_t gqa_group, float sm_scale, void* stream);
 
 /*
+ * Decisions from a borrowed query neuron (App. B).  Instead of a separate logit
+ * tensor, the decision logit of (sequence b, KV head h) at each token is element 0
+ * of that group's FIRST query head, q[b, t, h * gqa_group, 0]; the decision rule
+ * is the same (alpha = 1 iff that bf16 value is > 0, Sec. 3.2).  The attention
+ * then takes that element as 0 for the first query head of every group, leaving
+ * the group's other query heads unchanged.  The caller's q is not modified.
+ *
+ * dms_append_and_evict_borrowed: as dms_append_and_evict (any n_tokens >= 1), with
+ *   q [batch, n_tokens, kv_heads * gqa_group, 128] bf16 supplying the decisions
+ *   (only element 0 of each group's first head is read).
+ * dms_decode_attention_borrowed: as dms_decode_attention, attending with element 0
+ *   of each group's first query head taken as 0.
+ * dms_append_and_decode_borrowed: one decode step, as dms_append_and_decode, with
+ *   the decisions taken from q [batch, kv_heads * gqa_group, 128] and the
+ *   attention as in dms_decode_attention_borrowed.
+ * Arguments, alignment, errors and stream semantics are those of the plain forms.
+ */
+dms_status dms_append_and_evict_borrowed(dms_cache* cache, int32_t layer, const void* k,
+                                         const void* v, const void* q, int32_t n_tokens,
+                                         int32_t gqa_group, void* stream);
+dms_status dms_decode_attention_borrowed(dms_cache* cache, int32_t layer, const void* q, void* out,
+                                         int32_t gqa_group, float sm_scale, void* stream);
+dms_status dms_append_and_decode_borrowed(dms_cache* cache, int32_t layer, const void* k,
+                                          const void* v, const void* q, void* out,
+                                          int32_t gqa_group, float sm_scale, void* stream);
+
+/*
  * Synchronise `stream`, then report totals into *out (non-NULL) and, if
  * `counts` is non-NULL, copy the per-head retained counts n_h into the HOST
  * array counts[layers * batch * kv_heads] (layer-major, then sequence, then KV

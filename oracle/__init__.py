@@ -11,6 +11,7 @@ Functions (all take bf16 data as ``numpy.uint16`` bit patterns):
   alpha(logit_bits)                      Sec. 3.2 decision, [logit > 0]
   retained(logits, j, w)                 Sec. 3.1 / Fig. 1b retained positions
   decode(q, k, v, logits, j, w, scale)   softmax attention over the retained set
+  borrowed(q, G)                         App. B decision neuron: (logits, attention q)
 """
 from __future__ import annotations
 
@@ -128,3 +129,21 @@ def decode(q, k, v, logits, j: int, w: int, scale: float = 0.0) -> np.ndarray:
                               _ptr(lg, ctypes.c_uint16), lg.strides[0] // 2, j, w,
                               float(scale), _ptr(out, ctypes.c_double))
     return out
+
+
+def borrowed(q, group: int):
+    """App. B: the decision logit of each query group is element 0 of the group's first
+    query head, and that element is set to 0 before the attention; the other query
+    heads of the group are unchanged.
+
+    q: bf16 bits (numpy.uint16) of shape [..., kv_heads * group, D].  Returns
+    (logits [..., kv_heads], q_attention) with q_attention a copy of q whose element
+    0 of heads 0, group, 2 * group, ... is +0.
+    """
+    q = _u16(q)
+    if q.shape[-2] % group:
+        raise ValueError("query heads are not a multiple of the group size")
+    logits = q[..., ::group, 0].copy()
+    q_att = q.copy()
+    q_att[..., ::group, 0] = 0
+    return logits, q_att

@@ -79,6 +79,22 @@ def dms_append_and_decode(cache, layer, k_ptr, v_ptr, logit_ptr, q_ptr, out_ptr,
                                            gqa_group, float(sm_scale), stream)
 
 
+def dms_append_and_evict_borrowed(cache, layer, k_ptr, v_ptr, q_ptr, n_tokens, gqa_group, stream):
+    return library().dms_append_and_evict_borrowed(cache, layer, k_ptr, v_ptr, q_ptr, n_tokens,
+                                                   gqa_group, stream)
+
+
+def dms_decode_attention_borrowed(cache, layer, q_ptr, out_ptr, gqa_group, sm_scale, stream):
+    return library().dms_decode_attention_borrowed(cache, layer, q_ptr, out_ptr, gqa_group,
+                                                   float(sm_scale), stream)
+
+
+def dms_append_and_decode_borrowed(cache, layer, k_ptr, v_ptr, q_ptr, out_ptr, gqa_group,
+                                   sm_scale, stream):
+    return library().dms_append_and_decode_borrowed(cache, layer, k_ptr, v_ptr, q_ptr, out_ptr,
+                                                    gqa_group, float(sm_scale), stream)
+
+
 def dms_cache_stats(cache, stats: dms_stats, counts_ptr, stream):
     return library().dms_cache_stats(cache, ctypes.byref(stats), counts_ptr, stream)
 
@@ -209,6 +225,53 @@ class DmsCache:
         op = _bf16_cuda(out, (B, H * gqa_group, D), "out")
         _check(dms_append_and_decode(self._h, layer, kp, vp, lp, qp, op, gqa_group, sm_scale,
                                      _stream_ptr(stream)), "dms_append_and_decode")
+        return out
+
+    # ---- decisions from the borrowed query neuron (App. B): element 0 of each group's
+    # first query head is the decision logit and is taken as 0 by the attention.
+
+    def append_and_evict_borrowed(self, layer: int, k, v, q, gqa_group: int, stream=None):
+        """k, v: [batch, n, kv_heads, 128]; q: [batch, n, kv_heads * gqa_group, 128] bf16."""
+        n = k.shape[1]
+        B, H, D = self.batch, self.kv_heads, self.head_dim
+        kp = _bf16_cuda(k, (B, n, H, D), "k")
+        vp = _bf16_cuda(v, (B, n, H, D), "v")
+        qp = _bf16_cuda(q, (B, n, H * gqa_group, D), "q")
+        _check(dms_append_and_evict_borrowed(self._h, layer, kp, vp, qp, n, gqa_group,
+                                             _stream_ptr(stream)), "dms_append_and_evict_borrowed")
+
+    def decode_attention_borrowed(self, layer: int, q, out=None, gqa_group: int | None = None,
+                                  sm_scale: float = 0.0, stream=None):
+        """As decode_attention, with element 0 of each group's first query head taken as 0."""
+        import torch
+        B, H, D = self.batch, self.kv_heads, self.head_dim
+        if gqa_group is None:
+            gqa_group = q.shape[1] // H
+        if out is None:
+            out = torch.empty_like(q)
+        qp = _bf16_cuda(q, (B, H * gqa_group, D), "q")
+        op = _bf16_cuda(out, (B, H * gqa_group, D), "out")
+        _check(dms_decode_attention_borrowed(self._h, layer, qp, op, gqa_group, sm_scale,
+                                             _stream_ptr(stream)), "dms_decode_attention_borrowed")
+        return out
+
+    def append_and_decode_borrowed(self, layer: int, k, v, q, out=None,
+                                   gqa_group: int | None = None, sm_scale: float = 0.0,
+                                   stream=None):
+        """One decode step with the decisions read from q (one launch when fusable)."""
+        import torch
+        B, H, D = self.batch, self.kv_heads, self.head_dim
+        if gqa_group is None:
+            gqa_group = q.shape[1] // H
+        if out is None:
+            out = torch.empty_like(q)
+        kp = _bf16_cuda(k, (B, 1, H, D), "k")
+        vp = _bf16_cuda(v, (B, 1, H, D), "v")
+        qp = _bf16_cuda(q, (B, H * gqa_group, D), "q")
+        op = _bf16_cuda(out, (B, H * gqa_group, D), "out")
+        _check(dms_append_and_decode_borrowed(self._h, layer, kp, vp, qp, op, gqa_group, sm_scale,
+                                              _stream_ptr(stream)),
+               "dms_append_and_decode_borrowed")
         return out
 
     def stats(self, stream=None, with_counts: bool = False):

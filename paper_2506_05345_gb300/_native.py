@@ -27,7 +27,8 @@ EXPORTS = (
     "dms_cache_create", "dms_cache_destroy", "dms_cache_reset", "dms_append_and_evict",
     "dms_decode_attention", "dms_cache_stats", "dms_cache_export_positions",
     "dms_cache_layer_length", "dms_status_string", "dms_decode_attention_paged_noalloc",
-    "dms_append_and_decode", "dms_selftest_bounded_wait",
+    "dms_append_and_decode", "dms_selftest_bounded_wait", "dms_append_and_evict_borrowed",
+    "dms_decode_attention_borrowed", "dms_append_and_decode_borrowed",
 )
 
 
@@ -76,6 +77,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_decode_attention": (st, [vp, i32, vp, vp, i32, f32, vp]),
         "dms_append_and_decode": (st, [vp, i32, vp, vp, vp, vp, vp, i32, f32, vp]),
         "dms_selftest_bounded_wait": (st, [i32, i64, vp]),
+        "dms_append_and_evict_borrowed": (st, [vp, i32, vp, vp, vp, i32, i32, vp]),
+        "dms_decode_attention_borrowed": (st, [vp, i32, vp, vp, i32, f32, vp]),
+        "dms_append_and_decode_borrowed": (st, [vp, i32, vp, vp, vp, vp, i32, f32, vp]),
         "dms_cache_stats": (st, [vp, ctypes.POINTER(dms_stats), vp, vp]),
         "dms_cache_export_positions": (st, [vp, i32, vp, vp]),
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),

@@ -33,6 +33,7 @@ struct AppendParams {
   const uint16_t* k;
   const uint16_t* v;
   const uint16_t* logit;
+  int64_t logit_stride;  // elements between consecutive decision logits
   int64_t t0;           // position of the first appended token
   int64_t window;
   int64_t pool_pages;
@@ -72,7 +73,7 @@ __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
   if (lane == 0) {
     const int64_t j = p.t0;
     const int64_t R = p.window + 1, RP = ring_period(p.window);
-    const uint32_t alpha = decision_from_bf16(p.logit[(int64_t)b * p.kv_heads + hk]);
+    const uint32_t alpha = decision_from_bf16(p.logit[((int64_t)b * p.kv_heads + hk) * p.logit_stride]);
     uint32_t* ring = p.ring + (int64_t)bh * p.ring_len;
     int32_t* pt = p.page_table + (int64_t)bh * p.max_pages;
     int32_t n = p.counts_cur[bh];
@@ -172,7 +173,7 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
   for (int64_t base = 0; base < n_leave_new; base += kBulkThreads) {
     int flag = 0;
     if (base + tid < n_leave_new)
-      flag = (int)decision_from_bf16(p.logit[((int64_t)b * n + base + tid) * p.kv_heads + hk]);
+      flag = (int)decision_from_bf16(p.logit[(((int64_t)b * n + base + tid) * p.kv_heads + hk) * p.logit_stride]);
     int total;
     block_scan_flags(flag, s_warp, &total);
     evicted_new += total;
@@ -210,7 +211,7 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
     const int64_t li = base + tid;
     const bool valid = li < n;
     uint32_t alpha = 0;
-    if (valid) alpha = decision_from_bf16(p.logit[((int64_t)b * n + li) * p.kv_heads + hk]);
+    if (valid) alpha = decision_from_bf16(p.logit[(((int64_t)b * n + li) * p.kv_heads + hk) * p.logit_stride]);
     const int kept = (valid && !(alpha && li < n_leave_new)) ? 1 : 0;
     int total;
     const int r = block_scan_flags(kept, s_warp, &total);
@@ -266,7 +267,7 @@ __global__ void export_positions_kernel(const int32_t* counts, const int32_t* pa
 }
 
 AppendParams make_params(const Cache& c, int32_t layer, const void* k, const void* v,
-                         const void* logit, int64_t t0, int32_t n) {
+                         const void* logit, int64_t logit_stride, int64_t t0, int32_t n) {
   AppendParams p;
   p.pool = c.pool;
   p.pos = c.pos;
@@ -279,6 +280,7 @@ AppendParams make_params(const Cache& c, int32_t layer, const void* k, const voi
   p.k = static_cast<const uint16_t*>(k);
   p.v = static_cast<const uint16_t*>(v);
   p.logit = static_cast<const uint16_t*>(logit);
+  p.logit_stride = logit_stride;
   p.t0 = t0;
   p.window = c.window;
   p.pool_pages = c.pool_pages;
@@ -293,8 +295,9 @@ AppendParams make_params(const Cache& c, int32_t layer, const void* k, const voi
 }  // namespace
 
 cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, const void* v,
-                              const void* logit, int64_t t0, cudaStream_t stream) {
-  const AppendParams p = make_params(c, layer, k, v, logit, t0, 1);
+                              const void* logit, int64_t logit_stride, int64_t t0,
+                              cudaStream_t stream) {
+  const AppendParams p = make_params(c, layer, k, v, logit, logit_stride, t0, 1);
   const int threads = 256, per_block = threads / 32;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
@@ -309,8 +312,9 @@ cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, cons
 }
 
 cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, const void* v,
-                               const void* logit, int64_t t0, int32_t n, cudaStream_t stream) {
-  const AppendParams p = make_params(c, layer, k, v, logit, t0, n);
+                               const void* logit, int64_t logit_stride, int64_t t0, int32_t n,
+                               cudaStream_t stream) {
+  const AppendParams p = make_params(c, layer, k, v, logit, logit_stride, t0, n);
   append_bulk_kernel<<<c.heads, kBulkThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }

@@ -167,28 +167,36 @@ dms_status dms_cache_reset(dms_cache* h, void* stream) {
   return DMS_OK;
 }
 
-dms_status dms_append_and_evict(dms_cache* h, int32_t layer, const void* k, const void* v,
-                                const void* decision_logit, int32_t n_tokens, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Shared bodies of the plain and the borrowed-decision entry points: the decision logit
+// of entry i sits at logit[i * logit_stride]; zero_first makes the attention take
+// element 0 of every group's first query head as 0.
+dms_status append_impl(dms_cache* h, int32_t layer, const void* k, const void* v,
+                       const void* logit, int64_t logit_stride, int32_t n_tokens, void* stream) {
   if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
   Cache& c = h->c;
   if (layer < 0 || layer >= c.layers || n_tokens < 1 || k == nullptr || v == nullptr ||
-      decision_logit == nullptr || !aligned16(k) || !aligned16(v))
+      logit == nullptr || !aligned16(k) || !aligned16(v))
     return DMS_ERR_INVALID_ARGUMENT;
-  if ((reinterpret_cast<uintptr_t>(decision_logit) & 1u) != 0) return DMS_ERR_INVALID_ARGUMENT;
+  if ((reinterpret_cast<uintptr_t>(logit) & 1u) != 0) return DMS_ERR_INVALID_ARGUMENT;
   const int64_t t0 = c.lengths[layer];
   if (t0 + n_tokens > c.capacity) return DMS_ERR_CAPACITY;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const cudaError_t e = (n_tokens == 1)
-                            ? dms::launch_append_one(c, layer, k, v, decision_logit, t0, st)
-                            : dms::launch_append_bulk(c, layer, k, v, decision_logit, t0, n_tokens, st);
+  const cudaError_t e =
+      (n_tokens == 1)
+          ? dms::launch_append_one(c, layer, k, v, logit, logit_stride, t0, st)
+          : dms::launch_append_bulk(c, layer, k, v, logit, logit_stride, t0, n_tokens, st);
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = t0 + n_tokens;
   c.last_layer = layer;
   return DMS_OK;
 }
 
-dms_status dms_decode_attention(dms_cache* h, int32_t layer, const void* q, void* out,
-                                int32_t gqa_group, float sm_scale, void* stream) {
+dms_status decode_impl(dms_cache* h, int32_t layer, const void* q, void* out, int32_t gqa_group,
+                       float sm_scale, bool zero_first, void* stream) {
   if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
   Cache& c = h->c;
   if (layer < 0 || layer >= c.layers || q == nullptr || out == nullptr || !aligned16(q) ||
@@ -198,39 +206,84 @@ dms_status dms_decode_attention(dms_cache* h, int32_t layer, const void* q, void
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e;
   if (c.decode_kernel == DMS_DECODE_SIMPLE)
-    e = dms::launch_decode_simple(c, layer, q, out, gqa_group, scale, st);
+    e = dms::launch_decode_simple(c, layer, q, out, gqa_group, scale, zero_first, st);
   else
-    e = dms::launch_decode_tiled(c, layer, q, out, gqa_group, scale * 1.4426950408889634f, st);
+    e = dms::launch_decode_tiled(c, layer, q, out, gqa_group, scale * 1.4426950408889634f,
+                                 zero_first, st);
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.last_layer = layer;
   return DMS_OK;
 }
 
-dms_status dms_append_and_decode(dms_cache* h, int32_t layer, const void* k, const void* v,
-                                 const void* decision_logit, const void* q, void* out,
-                                 int32_t gqa_group, float sm_scale, void* stream) {
+dms_status append_decode_impl(dms_cache* h, int32_t layer, const void* k, const void* v,
+                              const void* logit, int64_t logit_stride, const void* q, void* out,
+                              int32_t gqa_group, float sm_scale, bool zero_first, void* stream) {
   if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
   Cache& c = h->c;
-  if (layer < 0 || layer >= c.layers || k == nullptr || v == nullptr || decision_logit == nullptr ||
+  if (layer < 0 || layer >= c.layers || k == nullptr || v == nullptr || logit == nullptr ||
       q == nullptr || out == nullptr || !aligned16(k) || !aligned16(v) || !aligned16(q) ||
-      !aligned16(out) || (reinterpret_cast<uintptr_t>(decision_logit) & 1u) != 0 ||
+      !aligned16(out) || (reinterpret_cast<uintptr_t>(logit) & 1u) != 0 ||
       gqa_group < 1 || gqa_group > dms::kMaxGroup || !(sm_scale == sm_scale))
     return DMS_ERR_INVALID_ARGUMENT;
   const int64_t t0 = c.lengths[layer];
   if (t0 + 1 > c.capacity) return DMS_ERR_CAPACITY;
   if (!dms::append_decode_fusable(c)) {
-    const dms_status st = dms_append_and_evict(h, layer, k, v, decision_logit, 1, stream);
+    const dms_status st = append_impl(h, layer, k, v, logit, logit_stride, 1, stream);
     if (st != DMS_OK) return st;
-    return dms_decode_attention(h, layer, q, out, gqa_group, sm_scale, stream);
+    return decode_impl(h, layer, q, out, gqa_group, sm_scale, zero_first, stream);
   }
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
-  const cudaError_t e =
-      dms::launch_append_decode(c, layer, k, v, decision_logit, q, out, gqa_group,
-                                scale * 1.4426950408889634f, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = dms::launch_append_decode(
+      c, layer, k, v, logit, logit_stride, q, out, gqa_group, scale * 1.4426950408889634f,
+      zero_first, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = t0 + 1;
   c.last_layer = layer;
   return DMS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dms_status dms_append_and_evict(dms_cache* h, int32_t layer, const void* k, const void* v,
+                                const void* decision_logit, int32_t n_tokens, void* stream) {
+  return append_impl(h, layer, k, v, decision_logit, 1, n_tokens, stream);
+}
+
+dms_status dms_decode_attention(dms_cache* h, int32_t layer, const void* q, void* out,
+                                int32_t gqa_group, float sm_scale, void* stream) {
+  return decode_impl(h, layer, q, out, gqa_group, sm_scale, false, stream);
+}
+
+dms_status dms_append_and_decode(dms_cache* h, int32_t layer, const void* k, const void* v,
+                                 const void* decision_logit, const void* q, void* out,
+                                 int32_t gqa_group, float sm_scale, void* stream) {
+  return append_decode_impl(h, layer, k, v, decision_logit, 1, q, out, gqa_group, sm_scale, false,
+                            stream);
+}
+
+// App. B: the decision logit of (sequence b, KV head h) at token t is element 0 of query
+// head h * G, i.e. q + ((b * n + t) * kv_heads + h) * G * 128 for q of [B, n, kv_heads * G, 128].
+dms_status dms_append_and_evict_borrowed(dms_cache* h, int32_t layer, const void* k,
+                                         const void* v, const void* q, int32_t n_tokens,
+                                         int32_t gqa_group, void* stream) {
+  if (gqa_group < 1 || gqa_group > dms::kMaxGroup || q == nullptr || !aligned16(q))
+    return DMS_ERR_INVALID_ARGUMENT;
+  return append_impl(h, layer, k, v, q, (int64_t)gqa_group * dms::kHeadDim, n_tokens, stream);
+}
+
+dms_status dms_decode_attention_borrowed(dms_cache* h, int32_t layer, const void* q, void* out,
+                                         int32_t gqa_group, float sm_scale, void* stream) {
+  return decode_impl(h, layer, q, out, gqa_group, sm_scale, true, stream);
+}
+
+dms_status dms_append_and_decode_borrowed(dms_cache* h, int32_t layer, const void* k,
+                                          const void* v, const void* q, void* out,
+                                          int32_t gqa_group, float sm_scale, void* stream) {
+  if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
+  return append_decode_impl(h, layer, k, v, q, (int64_t)gqa_group * dms::kHeadDim, q, out,
+                            gqa_group, sm_scale, true, stream);
 }
 
 dms_status dms_cache_stats(dms_cache* h, dms_stats* out, int32_t* counts, void* stream) {

@@ -86,7 +86,8 @@ struct DecodeParams {
   // Fused single-token append (position j) in front of the decode.
   const uint16_t* k_new;      // [batch, 1, kv_heads, 128]
   const uint16_t* v_new;
-  const uint16_t* logit_new;  // [batch, 1, kv_heads]
+  const uint16_t* logit_new;  // decision logit of head h at logit_new[h * logit_stride]
+  int64_t logit_stride;
   int32_t* counts_next;       // this layer, buffer after the append
   uint32_t* ring;             // this layer: [heads][ring_len]
   int32_t* pos;
@@ -97,6 +98,9 @@ struct DecodeParams {
   // first pages are staged, before waiting for that kernel; only the inputs (q, the
   // new K/V rows, the logits), the outputs and the shared split-K scratch wait.
   int32_t state_ready;
+  // Nonzero: attend with element 0 of every group's first query head taken as 0 (that
+  // element carries the decision logit, App. B).
+  int32_t zero_first;
 };
 
 // ---------------------------------------------------------------- PTX wrappers
@@ -403,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
         if (p.j >= R)
           asm volatile("prefetch.global.L2 [%0];" ::"l"(
               p.ring + (int64_t)h * p.ring_len + (p.j - R) % ring_period(p.window)));
-        asm volatile("prefetch.global.L2 [%0];" ::"l"(p.logit_new + h));
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(p.logit_new + (int64_t)h * p.logit_stride));
       }
     }
   }
@@ -528,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
         }
         if (pg_i == s_pstart[h_i + 1] - s_pstart[h_i] - 1) {  // owner of the head's last page
           const uint32_t sl = s_slot[h_i] & 0x3fffffffu;
-          const uint32_t alpha = decision_from_bf16(p.logit_new[h_i]);
+          const uint32_t alpha = decision_from_bf16(p.logit_new[(int64_t)h_i * p.logit_stride]);
           p.counts_next[h_i] = s_cnt[h_i];
           p.ring[(int64_t)h_i * p.ring_len + p.j % ring_period(p.window)] = sl | (alpha << 31);
         }
@@ -850,6 +854,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
       }
+      // Lane 0 holds (d = 0, 1) of the group's first query head in the low / high half.
+      if (p.zero_first && lane == 0) qb[0][0][0] &= 0xffff0000u;
     }
 
     if (tb < nvalid) {
@@ -1137,7 +1143,7 @@ __global__ void __launch_bounds__(128) decode_simple_kernel(const uint8_t* pool,
                                                             const __nv_bfloat16* q,
                                                             __nv_bfloat16* out, int32_t kv_heads,
                                                             int32_t group, int32_t max_pages,
-                                                            float scale) {
+                                                            float scale, int32_t zero_first) {
   const int bh = blockIdx.x;
   const int b = bh / kv_heads, hk = bh - b * kv_heads;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1149,6 +1155,7 @@ __global__ void __launch_bounds__(128) decode_simple_kernel(const uint8_t* pool,
     float qv[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) qv[e] = __bfloat162float(q[qrow + lane * 4 + e]);
+    if (zero_first && gq == 0 && lane == 0) qv[0] = 0.f;  // the decision element (App. B)
     float m = -INFINITY, l = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
     for (int s = 0; s < n; ++s) {
       const int32_t page = pt[s / kPageTokens];
@@ -1289,8 +1296,10 @@ DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* ou
 }  // namespace
 
 cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, void* out,
-                                int32_t group, float scale_log2, cudaStream_t stream) {
-  const DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
+                                int32_t group, float scale_log2, bool zero_first,
+                                cudaStream_t stream) {
+  DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
+  p.zero_first = zero_first ? 1 : 0;
   return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false);
 }
 
@@ -1301,13 +1310,16 @@ bool append_decode_fusable(const Cache& c) {
 // Single-token append of position lengths[layer] fused with the decode (requires
 // append_decode_fusable).
 cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,
-                                 const void* logit, const void* q, void* out, int32_t group,
-                                 float scale_log2, cudaStream_t stream) {
+                                 const void* logit, int64_t logit_stride, const void* q, void* out,
+                                 int32_t group, float scale_log2, bool zero_first,
+                                 cudaStream_t stream) {
   const int64_t t0 = c.lengths[layer];
   DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
+  p.zero_first = zero_first ? 1 : 0;
   p.k_new = static_cast<const uint16_t*>(k);
   p.v_new = static_cast<const uint16_t*>(v);
   p.logit_new = static_cast<const uint16_t*>(logit);
+  p.logit_stride = logit_stride;
   p.counts_next = c.counts_at(layer, t0 + 1);
   p.ring = c.rings + (int64_t)layer * c.heads * c.ring_len;
   p.pos = c.pos;
@@ -1319,11 +1331,11 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
 }
 
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
-                                 int32_t group, float scale, cudaStream_t stream) {
+                                 int32_t group, float scale, bool zero_first, cudaStream_t stream) {
   decode_simple_kernel<<<c.heads, 128, 0, stream>>>(
       c.pool, c.page_table + (int64_t)layer * c.heads * c.max_pages,
       c.counts_at(layer, c.lengths[layer]), static_cast<const __nv_bfloat16*>(q),
-      static_cast<__nv_bfloat16*>(out), c.kv_heads, group, c.max_pages, scale);
+      static_cast<__nv_bfloat16*>(out), c.kv_heads, group, c.max_pages, scale, zero_first ? 1 : 0);
   return cudaGetLastError();
 }
 

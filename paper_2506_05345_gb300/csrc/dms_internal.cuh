@@ -106,23 +106,30 @@ __host__ __device__ __forceinline__ uint32_t swizzled_offset(uint32_t row, uint3
   return row * kRowBytes + ((chunk ^ (row & 7u)) << 4);
 }
 
-// Launchers (defined in the .cu files).
+// Launchers (defined in the .cu files).  A decision logit sits at logit[i * logit_stride]
+// for entry i = (b * n_tokens + t) * kv_heads + h: stride 1 for a separate logit tensor,
+// gqa_group * 128 for the first element of each group's first query head (App. B).
+// zero_first: attend with that element of every group's first query head taken as 0.
 cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, const void* v,
-                              const void* logit, int64_t t0, cudaStream_t stream);
+                              const void* logit, int64_t logit_stride, int64_t t0,
+                              cudaStream_t stream);
 cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, const void* v,
-                               const void* logit, int64_t t0, int32_t n, cudaStream_t stream);
+                               const void* logit, int64_t logit_stride, int64_t t0, int32_t n,
+                               cudaStream_t stream);
 cudaError_t launch_export_positions(const Cache& c, int32_t layer, int32_t* dev_out,
                                     cudaStream_t stream);
 cudaError_t prepare_decode(const Cache& c);
 cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, void* out,
-                                int32_t group, float scale_log2, cudaStream_t stream);
+                                int32_t group, float scale_log2, bool zero_first,
+                                cudaStream_t stream);
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
-                                 int32_t group, float scale, cudaStream_t stream);
+                                 int32_t group, float scale, bool zero_first, cudaStream_t stream);
 bool append_decode_fusable(const Cache& c);
 cudaError_t launch_bounded_wait_probe(int arrive, int64_t limit_ns, int32_t* dev_status,
                                       cudaStream_t stream);
 cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,
-                                 const void* logit, const void* q, void* out, int32_t group,
-                                 float scale_log2, cudaStream_t stream);
+                                 const void* logit, int64_t logit_stride, const void* q, void* out,
+                                 int32_t group, float scale_log2, bool zero_first,
+                                 cudaStream_t stream);
 
 }  // namespace dms

@@ -320,3 +320,57 @@ def test_appH_kv_read_coefficient():
     coef = workloads.kv_bytes_per_token_head() * kv_heads * n  # bytes per (B*L) per step
     digits = int(vals["printed_digits"])
     assert float(f"{coef:.{digits - 1}e}") == vals["kv_read_coefficient"]
+
+
+# --------------------------------------------------------------------------- App. B neuron
+
+
+def test_borrowed_neuron_decisions_and_attention():
+    """App. B: the decision of each token comes from the sign of element 0 of the group's
+    first query head, and the attention no longer depends on that element's value: the
+    first head equals the masked dense softmax with the element set to 0, and the group's
+    other heads equal the plain path's bit for bit."""
+    rng = np.random.default_rng(11)
+    T, G, D, w = 48, 4, 32, 5
+    q, k, v, _ = _rand_case(rng, T, G, D, 0.5)
+    q[:, 0, 0] = _bf16(rng.standard_normal(T) + _probit(0.7))  # the neuron carries the logit
+    lg, q_att = oracle.borrowed(q, G)  # one KV head: logits [T, 1]
+    lg = lg[:, 0]
+    alpha = (_f64(q[:, 0, 0]) > 0).astype(np.float64)
+    M = _training_mask(alpha, w)
+    scale = 1.0 / math.sqrt(D)
+    q0 = _f64(q)[:, 0].copy()
+    q0[:, 0] = 0.0
+    ref0 = _sdpa_masked(q0, _f64(k), _f64(v), M, scale)
+    # same signs, other magnitudes: nothing may change
+    q2 = q.copy()
+    q2[:, 0, 0] = _bf16(np.where(alpha > 0, 1.0, -1.0) * (0.5 + rng.random(T)))
+    lg2, q_att2 = oracle.borrowed(q2, G)
+    lg2 = lg2[:, 0]
+    for j in range(T):
+        want = set(i for i in range(j + 1) if alpha[i] == 0 or j - i <= w)
+        assert set(oracle.retained(lg, j, w).tolist()) == want
+        assert np.array_equal(oracle.retained(lg2, j, w), oracle.retained(lg, j, w))
+        got = oracle.decode(q_att[j], k, v, lg, j, w)
+        np.testing.assert_allclose(got[0], ref0[j], rtol=0, atol=1e-12)
+        plain = oracle.decode(q[j], k, v, lg, j, w)
+        assert np.array_equal(got[1:], plain[1:])
+        assert np.array_equal(oracle.decode(q_att2[j], k, v, lg2, j, w), got)
+
+
+def test_borrowed_neuron_multi_head_layout():
+    """[B, kv_heads * G, D] queries: the logit of KV head h is element 0 of query head h * G."""
+    rng = np.random.default_rng(12)
+    B, H, G, D = 3, 5, 3, 16
+    q = _bf16(rng.standard_normal((B, H * G, D)))
+    lg, q_att = oracle.borrowed(q, G)
+    assert lg.shape == (B, H)
+    for b in range(B):
+        for h in range(H):
+            assert lg[b, h] == q[b, h * G, 0]
+            assert q_att[b, h * G, 0] == 0
+            for g in range(G):
+                d0 = 1 if g == 0 else 0
+                assert np.array_equal(q_att[b, h * G + g, d0:], q[b, h * G + g, d0:])
+    with pytest.raises(ValueError):
+        oracle.borrowed(q[:, :-1], G)
