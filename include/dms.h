@@ -183,6 +183,49 @@ dms_status dms_append_and_decode_borrowed(dms_cache* cache, int32_t layer, const
                                           int32_t gqa_group, float sm_scale, void* stream);
 
 /*
+ * Sparse prefill attention (Sec. 3.1 mask, Fig. 1b; Sec. 3.2: the eviction sparsity is
+ * used in prefill as well).  For a prompt of n_tokens tokens, query j of every query
+ * head attends, with plain softmax, to the keys i <= j of its KV head with
+ * alpha_i = 0 or j - i <= window, alpha_i = [bf16 decision logit of token i > 0]; the
+ * result is what a decode at position j would return after appending tokens 0..j.
+ * It is stateless: no cache is read or written (dms_append_and_evict fills a cache
+ * from the same k, v and logits).
+ *
+ * Inputs (device pointers, bf16 unless stated, contiguous, 16-byte aligned):
+ *   q, out          [batch, n_tokens, kv_heads * gqa_group, 128]; query head hq uses
+ *                   KV head hq / gqa_group.
+ *   k, v            [batch, n_tokens, kv_heads, 128]
+ *   decision_logit  [batch, n_tokens, kv_heads] (2-byte aligned)
+ *   workspace       caller-owned device memory of at least
+ *                   dms_prefill_workspace_bytes(batch, n_tokens, kv_heads) bytes (about
+ *                   1 KiB per token and KV head), 16-byte aligned; it must not be used by
+ *                   other work until the call's stream work completes.
+ * sm_scale <= 0 selects 1/sqrt(128).  Limits: batch * kv_heads <= 65535,
+ * 1 <= gqa_group <= 16, ceil(n_tokens / 128) * batch * kv_heads * gqa_group < 2^31.
+ * Errors: invalid arguments -> DMS_ERR_INVALID_ARGUMENT, a workspace that is too small ->
+ * DMS_ERR_CAPACITY, both before any launch.  A bounded in-kernel wait that gives up
+ * records DMS_ERR_TIMEOUT in the workspace; dms_prefill_device_error reads it.
+ *
+ * dms_prefill_attention_borrowed takes the decision logit of (b, t, h) from element 0
+ * of query head h * gqa_group (App. B) and attends with that element taken as 0.
+ */
+dms_status dms_prefill_workspace_bytes(int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                                       size_t* out_bytes);
+dms_status dms_prefill_attention(const void* q, const void* k, const void* v,
+                                 const void* decision_logit, int32_t batch, int32_t n_tokens,
+                                 int32_t kv_heads, int32_t gqa_group, int32_t window,
+                                 float sm_scale, void* workspace, size_t workspace_bytes,
+                                 void* out, void* stream);
+dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const void* v,
+                                          int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                                          int32_t gqa_group, int32_t window, float sm_scale,
+                                          void* workspace, size_t workspace_bytes, void* out,
+                                          void* stream);
+/* Synchronise `stream` and report the sticky device error of the last prefill that used
+ * `workspace` into *out (DMS_OK when none). */
+dms_status dms_prefill_device_error(const void* workspace, void* stream, dms_status* out);
+
+/*
  * Synchronise `stream`, then report totals into *out (non-NULL) and, if
  * `counts` is non-NULL, copy the per-head retained counts n_h into the HOST
  * array counts[layers * batch * kv_heads] (layer-major, then sequence, then KV

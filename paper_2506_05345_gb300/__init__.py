@@ -95,6 +95,71 @@ def dms_append_and_decode_borrowed(cache, layer, k_ptr, v_ptr, q_ptr, out_ptr, g
                                                     gqa_group, float(sm_scale), stream)
 
 
+def dms_prefill_workspace_bytes(batch, n_tokens, kv_heads):
+    out = ctypes.c_size_t(0)
+    code = library().dms_prefill_workspace_bytes(batch, n_tokens, kv_heads, ctypes.byref(out))
+    return code, out.value
+
+
+def dms_prefill_attention(q_ptr, k_ptr, v_ptr, logit_ptr, batch, n_tokens, kv_heads, gqa_group,
+                          window, sm_scale, ws_ptr, ws_bytes, out_ptr, stream):
+    return library().dms_prefill_attention(q_ptr, k_ptr, v_ptr, logit_ptr, batch, n_tokens,
+                                           kv_heads, gqa_group, window, float(sm_scale), ws_ptr,
+                                           ws_bytes, out_ptr, stream)
+
+
+def dms_prefill_attention_borrowed(q_ptr, k_ptr, v_ptr, batch, n_tokens, kv_heads, gqa_group,
+                                   window, sm_scale, ws_ptr, ws_bytes, out_ptr, stream):
+    return library().dms_prefill_attention_borrowed(q_ptr, k_ptr, v_ptr, batch, n_tokens,
+                                                    kv_heads, gqa_group, window, float(sm_scale),
+                                                    ws_ptr, ws_bytes, out_ptr, stream)
+
+
+def dms_prefill_device_error(ws_ptr, stream):
+    out = ctypes.c_int(0)
+    code = library().dms_prefill_device_error(ws_ptr, stream, ctypes.byref(out))
+    return code, out.value
+
+
+def prefill_attention(q, k, v, decision_logit=None, window: int = 256, gqa_group=None,
+                      sm_scale: float = 0.0, workspace=None, out=None, stream=None):
+    """Sparse DMS prefill attention of a whole prompt (no cache involved).
+
+    q: [B, P, Hkv * G, 128], k, v: [B, P, Hkv, 128], decision_logit: [B, P, Hkv] bf16 CUDA
+    tensors; decision_logit=None takes the decisions from element 0 of each group's first
+    query head (App. B).  Returns out [B, P, Hkv * G, 128] bf16.  The workspace (uint8
+    CUDA tensor) is allocated when not given.
+    """
+    import torch
+    B, P, Hkv, D = k.shape
+    if gqa_group is None:
+        gqa_group = q.shape[2] // Hkv
+    code, nbytes = dms_prefill_workspace_bytes(B, P, Hkv)
+    _check(code, "dms_prefill_workspace_bytes")
+    if workspace is None:
+        workspace = torch.empty(nbytes, dtype=torch.uint8, device=q.device)
+    if out is None:
+        out = torch.empty_like(q)
+    qp = _bf16_cuda(q, (B, P, Hkv * gqa_group, D), "q")
+    kp = _bf16_cuda(k, (B, P, Hkv, D), "k")
+    vp = _bf16_cuda(v, (B, P, Hkv, D), "v")
+    op = _bf16_cuda(out, (B, P, Hkv * gqa_group, D), "out")
+    if workspace.dtype != torch.uint8 or not workspace.is_cuda:
+        raise TypeError("workspace must be a uint8 CUDA tensor")
+    wp = ctypes.c_void_p(workspace.data_ptr())
+    wb = workspace.numel()
+    if decision_logit is None:
+        code = dms_prefill_attention_borrowed(qp, kp, vp, B, P, Hkv, gqa_group, window, sm_scale,
+                                              wp, wb, op, _stream_ptr(stream))
+        _check(code, "dms_prefill_attention_borrowed")
+    else:
+        lp = _bf16_cuda(decision_logit, (B, P, Hkv), "decision_logit")
+        code = dms_prefill_attention(qp, kp, vp, lp, B, P, Hkv, gqa_group, window, sm_scale, wp,
+                                     wb, op, _stream_ptr(stream))
+        _check(code, "dms_prefill_attention")
+    return out
+
+
 def dms_cache_stats(cache, stats: dms_stats, counts_ptr, stream):
     return library().dms_cache_stats(cache, ctypes.byref(stats), counts_ptr, stream)
 

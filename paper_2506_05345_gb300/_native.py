@@ -29,6 +29,8 @@ EXPORTS = (
     "dms_cache_layer_length", "dms_status_string", "dms_decode_attention_paged_noalloc",
     "dms_append_and_decode", "dms_selftest_bounded_wait", "dms_append_and_evict_borrowed",
     "dms_decode_attention_borrowed", "dms_append_and_decode_borrowed",
+    "dms_prefill_workspace_bytes", "dms_prefill_attention", "dms_prefill_attention_borrowed",
+    "dms_prefill_device_error",
 )
 
 
@@ -80,6 +82,12 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_append_and_evict_borrowed": (st, [vp, i32, vp, vp, vp, i32, i32, vp]),
         "dms_decode_attention_borrowed": (st, [vp, i32, vp, vp, i32, f32, vp]),
         "dms_append_and_decode_borrowed": (st, [vp, i32, vp, vp, vp, vp, i32, f32, vp]),
+        "dms_prefill_workspace_bytes": (st, [i32, i32, i32, ctypes.POINTER(ctypes.c_size_t)]),
+        "dms_prefill_attention": (st, [vp, vp, vp, vp, i32, i32, i32, i32, i32, f32, vp,
+                                       ctypes.c_size_t, vp, vp]),
+        "dms_prefill_attention_borrowed": (st, [vp, vp, vp, i32, i32, i32, i32, i32, f32, vp,
+                                                ctypes.c_size_t, vp, vp]),
+        "dms_prefill_device_error": (st, [vp, vp, ctypes.POINTER(st)]),
         "dms_cache_stats": (st, [vp, ctypes.POINTER(dms_stats), vp, vp]),
         "dms_cache_export_positions": (st, [vp, i32, vp, vp]),
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),

@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libdms.so")
-SOURCES = ["dms_cache.cu", "dms_append.cu", "dms_decode.cu"]
+SOURCES = ["dms_cache.cu", "dms_append.cu", "dms_decode.cu", "dms_prefill.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -132,4 +132,13 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
                                  int32_t group, float scale_log2, bool zero_first,
                                  cudaStream_t stream);
 
+// Sparse prefill attention (dms_prefill.cu): caller-owned workspace of
+// prefill_workspace_bytes(batch * kv_heads, n_tokens) bytes whose first 64 bytes are a
+// control block (int32 [kCtrlError] holds the sticky device error).
+size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens);
+cudaError_t launch_prefill(const void* q, const void* k, const void* v, const void* logit,
+                           int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                           int32_t group, int32_t window, float scale_log2, bool zero_first,
+                           void* workspace, void* out, cudaStream_t stream);
+
 }  // namespace dms

@@ -1,0 +1,576 @@
+// Sparse DMS prefill attention (arXiv 2506.05345, Sec. 3.1 / Fig. 1b for the mask, Sec. 3.2:
+// the eviction sparsity is also used in prefill).  For a prompt of P tokens, query j of
+// every query head attends, with plain softmax, to the keys i <= j of its KV head with
+// alpha_i = 0 or j - i <= w (alpha_i = [bf16 decision logit of token i > 0]).
+//
+// The visible keys of a tile of 128 consecutive queries [j0, j0 + 128) split into two
+// disjoint sets, each a contiguous run of rows once the prompt is laid out per KV head:
+//   * retained keys: alpha_i = 0 and i < j - w.  In the per-head list of the alpha = 0
+//     tokens in position order (the compacted list), they are a prefix: the first
+//     before[jmax - w] entries, where before[x] counts the alpha = 0 tokens at positions
+//     below x and jmax is the tile's last query.  Row j masks the entries at positions
+//     >= j - w;
+//   * window keys: j - w <= i <= j, a band of dense rows [j0 - w, jmax] (start rounded
+//     down to a multiple of 8), masked per row.
+// A pre-pass (two small kernels) lays every KV head out contiguously: dense K and V rows,
+// the compacted K and V rows, the compacted rows' positions and the prefix counts, with
+// each 256-byte row's 16-byte chunks permuted (chunk ^ (row & 7)) so that 1-D bulk copies
+// land in shared memory conflict-free for ldmatrix.
+//
+// Attention kernel: one CTA per (query head, 128-query tile), heaviest tiles (latest
+// queries) first.  A producer warp streams 64-key tiles (K, V and, for retained tiles,
+// the keys' positions) into a 3-stage shared-memory ring with bulk copies on mbarriers;
+// eight consumer warps own 16 queries each: S = Q K^T and O += P V with mma.sync
+// m16n8k16 (bf16 in, fp32 accumulate), fp32 online softmax in the exp2 domain, P reused
+// from the S accumulators as the A operand.  Each warp stages its queries in shared memory
+// once and reloads their fragments with ldmatrix per tile (nine warps leave ~168
+// registers per thread; holding Q in registers would spill).
+#include <math.h>
+
+#include <atomic>
+
+#include "dms_internal.cuh"
+#include "dms_ptx.cuh"
+
+namespace dms {
+namespace {
+
+constexpr int kPfRows = 128;                                  // queries per CTA
+constexpr int kPfWarps = kPfRows / 16;                        // consumer warps
+constexpr int kPfKeys = 64;                                   // keys per tile
+constexpr int kPfStages = 3;
+constexpr int kPfThreads = (kPfWarps + 1) * 32;               // + producer warp
+constexpr int kPfTileBytes = kPfKeys * kRowBytes;             // 16 KiB
+constexpr int kPfStageBytes = 2 * kPfTileBytes + kPfKeys * 4;  // K, V, key positions
+constexpr int kPfQBytes = kPfRows * kRowBytes;                // the CTA's queries, 32 KiB
+constexpr int kPfSmemBytes = kPfStages * kPfStageBytes + kPfQBytes + 2 * kPfStages * 8 + 16;
+constexpr int kPfChunk = 1024;                                // tokens per pre-pass block
+constexpr int kPfPackThreads = 256;
+constexpr int kPfPosPad = kPfKeys;  // compacted positions padded so whole tiles copy
+
+// Row stride (int32 entries) of a head's compacted positions: whole 64-entry tiles copy
+// from any tile start, and every row starts on a 16-byte boundary (bulk-copy sources).
+__host__ __device__ __forceinline__ int64_t pc_stride(int64_t P) { return (P + kPfPosPad + 3) & ~(int64_t)3; }
+
+// Workspace regions (byte offsets, each 256-byte aligned).  H = batch * kv_heads.
+struct PfLayout {
+  size_t err, kd, vd, kc, vc, pc, before, cc, total;
+};
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+PfLayout pf_layout(int64_t H, int64_t P) {
+  PfLayout L;
+  const int64_t nch = (P + kPfChunk - 1) / kPfChunk;
+  size_t o = 0;
+  L.err = o; o = align256(o + 64);
+  L.kd = o; o = align256(o + (size_t)H * P * kRowBytes);
+  L.vd = o; o = align256(o + (size_t)H * P * kRowBytes);
+  L.kc = o; o = align256(o + (size_t)H * P * kRowBytes);
+  L.vc = o; o = align256(o + (size_t)H * P * kRowBytes);
+  L.pc = o; o = align256(o + (size_t)H * pc_stride(P) * 4);
+  L.before = o; o = align256(o + (size_t)H * (P + 1) * 4);
+  L.cc = o; o = align256(o + (size_t)H * nch * 4);
+  L.total = o;
+  return L;
+}
+
+struct PackParams {
+  const uint16_t* k;         // [B, P, Hkv, 128]
+  const uint16_t* v;
+  const uint16_t* logit;     // decision logit of (b, i, h) at logit[((b P + i) Hkv + h) stride]
+  int64_t logit_stride;
+  uint8_t* kd;               // [H][P] permuted rows
+  uint8_t* vd;
+  uint8_t* kc;               // [H][P] permuted rows of the alpha = 0 tokens, position order
+  uint8_t* vc;
+  int32_t* pc;               // [H][pc_stride(P)] positions of the compacted rows
+  int32_t* before;           // [H][P + 1] alpha = 0 tokens at positions below i
+  int32_t* cc;               // [H][nch] alpha = 0 tokens per chunk
+  int32_t P, kv_heads, nch;
+};
+
+// Byte offset of logical 16-byte chunk `chunk` inside row `row` of a permuted array (the
+// row's own offset, row * 256, is added by the caller in 64-bit arithmetic).
+__device__ __forceinline__ uint32_t chunk_in_row(int64_t row, int chunk) {
+  return (uint32_t)((chunk ^ (int)(row & 7)) << 4);
+}
+
+__device__ __forceinline__ bool keep_token(const PackParams& p, int b, int hk, int i) {
+  return decision_from_bf16(
+             p.logit[(((int64_t)b * p.P + i) * p.kv_heads + hk) * p.logit_stride]) == 0u;
+}
+
+// Alpha = 0 tokens of each (head, chunk).
+__global__ void __launch_bounds__(kPfPackThreads) prefill_count_kernel(const PackParams p) {
+  const int ch = blockIdx.x, head = blockIdx.y;
+  const int b = head / p.kv_heads, hk = head - b * p.kv_heads;
+  const int i_end = min(p.P, (ch + 1) * kPfChunk);
+  int cnt = 0;
+  for (int i = ch * kPfChunk + threadIdx.x; i < i_end; i += kPfPackThreads)
+    cnt += keep_token(p, b, hk, i) ? 1 : 0;
+  __shared__ int s_sum[kPfPackThreads / 32];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, off);
+  if ((threadIdx.x & 31) == 0) s_sum[threadIdx.x >> 5] = cnt;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int t = 0;
+    for (int w = 0; w < kPfPackThreads / 32; ++w) t += s_sum[w];
+    p.cc[(int64_t)head * p.nch + ch] = t;
+  }
+}
+
+// Lays out one (head, chunk): dense rows, compacted rows and their positions, and the
+// prefix counts.  Thread t owns tokens 4t .. 4t + 3 of the chunk for the scan; the
+// warps then move the rows, one 512-byte K + V row pair per warp step.
+__global__ void __launch_bounds__(kPfPackThreads) prefill_pack_kernel(const PackParams p) {
+  const int ch = blockIdx.x, head = blockIdx.y;
+  const int b = head / p.kv_heads, hk = head - b * p.kv_heads;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int i0 = ch * kPfChunk, n = min(kPfChunk, p.P - i0);
+  __shared__ int s_idx[kPfChunk];  // compacted index of each token, or -1 when evicted
+  __shared__ int s_warp[kPfPackThreads / 32];
+  __shared__ int s_base;
+  // alpha = 0 tokens of the earlier chunks of this head
+  int base = 0;
+  for (int c = tid; c < ch; c += kPfPackThreads) base += p.cc[(int64_t)head * p.nch + c];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) base += __shfl_xor_sync(0xffffffffu, base, off);
+  if (lane == 0) s_warp[warp] = base;
+  __syncthreads();
+  if (tid == 0) {
+    int t = 0;
+    for (int w = 0; w < kPfPackThreads / 32; ++w) t += s_warp[w];
+    s_base = t;
+  }
+  __syncthreads();
+  base = s_base;
+  // exclusive scan of the keep flags over the chunk
+  int f[4], local = 0;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int i = 4 * tid + e;
+    f[e] = (i < n && keep_token(p, b, hk, i0 + i)) ? 1 : 0;
+    local += f[e];
+  }
+  int x = local;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += y;
+  }
+  __syncthreads();  // s_warp reuse
+  if (lane == 31) s_warp[warp] = x;
+  __syncthreads();
+  int run = base + x - local;
+  for (int w = 0; w < warp; ++w) run += s_warp[w];
+  int32_t* before = p.before + (int64_t)head * (p.P + 1);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int i = 4 * tid + e;
+    if (i < n) {
+      before[i0 + i] = run;
+      s_idx[i] = f[e] ? run : -1;
+      if (i0 + i == p.P - 1) before[p.P] = run + f[e];
+    }
+    run += f[e];
+  }
+  __syncthreads();
+  // rows: lanes 0-15 move K's sixteen 16-byte chunks, lanes 16-31 V's
+  const int half = lane >> 4, chunk = lane & 15;
+  const uint16_t* src_base = half ? p.v : p.k;
+  uint8_t* dense = half ? p.vd : p.kd;
+  uint8_t* comp = half ? p.vc : p.kc;
+  const int64_t hrow = (int64_t)head * p.P;
+  for (int i = warp; i < n; i += kPfPackThreads / 32) {
+    const int pos = i0 + i;
+    const uint4 val = *reinterpret_cast<const uint4*>(
+        src_base + (((int64_t)b * p.P + pos) * p.kv_heads + hk) * kHeadDim + chunk * 8);
+    *reinterpret_cast<uint4*>(dense + (hrow + pos) * kRowBytes + chunk_in_row(pos, chunk)) = val;
+    const int c = s_idx[i];
+    if (c >= 0) {
+      *reinterpret_cast<uint4*>(comp + (hrow + c) * kRowBytes + chunk_in_row(c, chunk)) = val;
+      if (lane == 0) p.pc[(int64_t)head * pc_stride(p.P) + c] = pos;
+    }
+  }
+}
+
+struct PrefillParams {
+  const __nv_bfloat16* q;    // [B, P, Hq, 128]
+  __nv_bfloat16* out;        // [B, P, Hq, 128]
+  const uint8_t* kd;
+  const uint8_t* vd;
+  const uint8_t* kc;
+  const uint8_t* vc;
+  const int32_t* pc;
+  const int32_t* before;
+  int32_t* err;              // sticky error word (bounded waits)
+  int32_t P, kv_heads, group, window, zero_first, n_qtiles, n_qheads;
+  float scale_log2;
+};
+
+__global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const PrefillParams p) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  uint8_t* sq = smem + kPfStages * kPfStageBytes;  // [128 rows][256 B], permuted chunks
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(sq + kPfQBytes);
+  uint64_t* empty_bar = full_bar + kPfStages;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(empty_bar + kPfStages);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int Hq = p.kv_heads * p.group;
+  const int tile_rank = blockIdx.x / p.n_qheads;
+  const int qt = p.n_qtiles - 1 - tile_rank;  // latest (heaviest) query tiles first
+  const int qh = blockIdx.x - tile_rank * p.n_qheads;
+  const int b = qh / Hq, hq = qh - b * Hq, hk = hq / p.group;
+  const int64_t head = (int64_t)b * p.kv_heads + hk;
+  const int P = p.P, w = p.window;
+  const int j0 = qt * kPfRows;
+  const int jmax = min(j0 + kPfRows, P) - 1;
+  // retained keys: the first nc compacted rows; window keys: dense rows [bs, jmax]
+  const int nc = (jmax - w > 0) ? p.before[head * (P + 1) + (jmax - w)] : 0;
+  const int bs = max(0, j0 - w) & ~7;
+  const int n_ct = (nc + kPfKeys - 1) / kPfKeys;
+  const int n_tiles = n_ct + (jmax + 1 - bs + kPfKeys - 1) / kPfKeys;
+
+  if (tid == 0) {
+    *abort_flag = 0;
+    for (int s = 0; s < kPfStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], kPfWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  if (warp == kPfWarps) {
+    // ================================================================ producer warp
+    if (lane == 0) {
+      for (int t = 0; t < n_tiles; ++t) {
+        const int s = t % kPfStages, use = t / kPfStages;
+        if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.err);
+        uint8_t* st = smem + s * kPfStageBytes;
+        if (t < n_ct) {
+          const int r0 = t * kPfKeys, rows = min(kPfKeys, nc - r0);
+          const uint32_t bytes = (uint32_t)rows * kRowBytes;
+          mbar_arrive_expect_tx(&full_bar[s], 2 * bytes + kPfKeys * 4);
+          const int64_t row = head * P + r0;
+          bulk_copy_g2s(st, p.kc + row * kRowBytes, bytes, &full_bar[s]);
+          bulk_copy_g2s(st + kPfTileBytes, p.vc + row * kRowBytes, bytes, &full_bar[s]);
+          bulk_copy_g2s(st + 2 * kPfTileBytes, p.pc + head * pc_stride(P) + r0, kPfKeys * 4,
+                        &full_bar[s]);
+        } else {
+          const int r0 = bs + (t - n_ct) * kPfKeys, rows = min(kPfKeys, jmax + 1 - r0);
+          const uint32_t bytes = (uint32_t)rows * kRowBytes;
+          mbar_arrive_expect_tx(&full_bar[s], 2 * bytes);
+          const int64_t row = head * P + r0;
+          bulk_copy_g2s(st, p.kd + row * kRowBytes, bytes, &full_bar[s]);
+          bulk_copy_g2s(st + kPfTileBytes, p.vd + row * kRowBytes, bytes, &full_bar[s]);
+        }
+      }
+      // Drain: do not leave while a bulk copy may still be writing shared memory.
+      for (int s = 0; s < kPfStages && s < n_tiles; ++s) {
+        const int last_t = s + ((n_tiles - 1 - s) / kPfStages) * kPfStages;
+        mbar_wait(&full_bar[s], (last_t / kPfStages) & 1, abort_flag, p.err);
+      }
+    }
+    return;
+  }
+
+  // ================================================================ consumer warps
+  const int g = lane >> 2, c4 = lane & 3, mi = lane >> 3;
+  const int r_lo = j0 + 16 * warp + g, r_hi = r_lo + 8;  // this lane's two query rows
+  // This warp's 16 queries into shared memory (permuted chunks, read back with ldmatrix);
+  // App. B: element 0 of a group's first query head carries the decision, not attention.
+  {
+    const bool zero = p.zero_first && hq % p.group == 0;
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      const int idx = it * 32 + lane, row = idx >> 4, chunk = idx & 15;
+      const int j = j0 + 16 * warp + row;
+      uint4 val = make_uint4(0u, 0u, 0u, 0u);
+      if (j < P)
+        val = *reinterpret_cast<const uint4*>(p.q + (((int64_t)b * P + j) * Hq + hq) * kHeadDim +
+                                              chunk * 8);
+      if (zero && chunk == 0) val.x &= 0xffff0000u;
+      *reinterpret_cast<uint4*>(sq + (16 * warp + row) * kRowBytes + chunk_in_row(row, chunk)) = val;
+    }
+    __syncwarp();
+  }
+  const uint32_t qbase = smem_addr(sq + 16 * warp * kRowBytes);
+  float o[16][4];
+#pragma unroll
+  for (int nt = 0; nt < 16; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
+  float m_lo = -INFINITY, m_hi = -INFINITY, l_lo = 0.f, l_hi = 0.f;
+
+  for (int t = 0; t < n_tiles; ++t) {
+    const int s = t % kPfStages, use = t / kPfStages;
+    const bool retained = t < n_ct;
+    const int r0 = retained ? t * kPfKeys : bs + (t - n_ct) * kPfKeys;
+    const int rows = retained ? min(kPfKeys, nc - r0) : min(kPfKeys, jmax + 1 - r0);
+    const uint8_t* st = smem + s * kPfStageBytes;
+    mbar_wait(&full_bar[s], use & 1, abort_flag, p.err);
+
+    // ---- S = Q K^T (16 x 64): 8 n-tiles of 8 keys, 8 k-steps of 16 head_dim
+    float sc[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+    {
+      const uint32_t kbase = smem_addr(st);
+      const uint32_t qrow = (uint32_t)((mi & 1) * 8 + (lane & 7));
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        uint32_t qa[4];  // A-fragment: rows 0-7 / 8-15 of the warp, d 16 kk .. 16 kk + 15
+        ldsm_x4(qbase + swizzled_offset(qrow, (uint32_t)(2 * kk + (mi >> 1))), qa[0], qa[1], qa[2],
+                qa[3]);
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {
+          const uint32_t row = (uint32_t)(16 * np + (mi >> 1) * 8 + (lane & 7));
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(kbase + swizzled_offset(row, (uint32_t)(2 * kk + (mi & 1))), b0, b1, b2, b3);
+          mma_bf16_16816(sc[2 * np], qa, b0, b1);
+          mma_bf16_16816(sc[2 * np + 1], qa, b2, b3);
+        }
+      }
+    }
+    // ---- mask (retained: position < j - w; window: j - w <= position <= j), online softmax
+    const int32_t* spos = reinterpret_cast<const int32_t*>(st + 2 * kPfTileBytes);
+    float mx_lo = -INFINITY, mx_hi = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int kidx = 8 * nt + 2 * c4 + e;
+        const bool valid = kidx < rows;
+        const int pos = retained ? (valid ? spos[kidx] : 0) : r0 + kidx;
+        const bool vis_lo = valid && (retained ? pos < r_lo - w : (pos >= r_lo - w && pos <= r_lo));
+        const bool vis_hi = valid && (retained ? pos < r_hi - w : (pos >= r_hi - w && pos <= r_hi));
+        sc[nt][e] = vis_lo ? sc[nt][e] * p.scale_log2 : -INFINITY;
+        sc[nt][2 + e] = vis_hi ? sc[nt][2 + e] * p.scale_log2 : -INFINITY;
+        mx_lo = fmaxf(mx_lo, sc[nt][e]);
+        mx_hi = fmaxf(mx_hi, sc[nt][2 + e]);
+      }
+    }
+#pragma unroll
+    for (int off = 1; off < 4; off <<= 1) {
+      mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, off));
+      mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, off));
+    }
+    const float mn_lo = fmaxf(m_lo, mx_lo), mn_hi = fmaxf(m_hi, mx_hi);
+    // a row that has seen no visible key yet keeps a zero base (no -inf - -inf)
+    const float base_lo = mn_lo == -INFINITY ? 0.f : mn_lo;
+    const float base_hi = mn_hi == -INFINITY ? 0.f : mn_hi;
+    const float corr_lo = exp2f(m_lo - base_lo), corr_hi = exp2f(m_hi - base_hi);
+    m_lo = mn_lo;
+    m_hi = mn_hi;
+    float sum_lo = 0.f, sum_hi = 0.f;
+    uint32_t pa[4][4];  // P A-fragments of the four 16-key k-steps
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const float p0 = exp2f(sc[nt][0] - base_lo), p1 = exp2f(sc[nt][1] - base_lo);
+      const float p2 = exp2f(sc[nt][2] - base_hi), p3 = exp2f(sc[nt][3] - base_hi);
+      sum_lo += p0 + p1;
+      sum_hi += p2 + p3;
+      pa[nt >> 1][(nt & 1) * 2 + 0] = pack_bf16x2(p0, p1);
+      pa[nt >> 1][(nt & 1) * 2 + 1] = pack_bf16x2(p2, p3);
+    }
+    l_lo = l_lo * corr_lo + sum_lo;
+    l_hi = l_hi * corr_hi + sum_hi;
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) {
+      o[nt][0] *= corr_lo;
+      o[nt][1] *= corr_lo;
+      o[nt][2] *= corr_hi;
+      o[nt][3] *= corr_hi;
+    }
+    // ---- O += P V (16 x 128): 4 k-steps of 16 keys, 16 n-tiles of 8 head_dim
+    {
+      const uint32_t vbase = smem_addr(st + kPfTileBytes);
+#pragma unroll
+      for (int kt = 0; kt < 4; ++kt) {
+        // stale rows past the tile's valid keys must not reach the tensor cores (0 * NaN)
+        const int tk = 16 * kt + 2 * c4;
+        const uint32_t mk0 = (tk < rows ? 0x0000ffffu : 0u) | (tk + 1 < rows ? 0xffff0000u : 0u);
+        const uint32_t mk1 = (tk + 8 < rows ? 0x0000ffffu : 0u) | (tk + 9 < rows ? 0xffff0000u : 0u);
+        const uint32_t row = (uint32_t)(16 * kt + (mi & 1) * 8 + (lane & 7));
+#pragma unroll
+        for (int dp = 0; dp < 8; ++dp) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_trans(vbase + swizzled_offset(row, (uint32_t)(2 * dp + (mi >> 1))), b0, b1, b2,
+                        b3);
+          b0 &= mk0;
+          b1 &= mk1;
+          b2 &= mk0;
+          b3 &= mk1;
+          mma_bf16_16816(o[2 * dp], pa[kt], b0, b1);
+          mma_bf16_16816(o[2 * dp + 1], pa[kt], b2, b3);
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty_bar[s]);
+  }
+
+  // ---- normalise and store (rows past the prompt are not written)
+#pragma unroll
+  for (int off = 1; off < 4; off <<= 1) {
+    l_lo += __shfl_xor_sync(0xffffffffu, l_lo, off);
+    l_hi += __shfl_xor_sync(0xffffffffu, l_hi, off);
+  }
+  const float inv_lo = l_lo > 0.f ? 1.f / l_lo : 0.f, inv_hi = l_hi > 0.f ? 1.f / l_hi : 0.f;
+  __nv_bfloat16* o_lo = p.out + (((int64_t)b * P + r_lo) * Hq + hq) * kHeadDim;
+  __nv_bfloat16* o_hi = p.out + (((int64_t)b * P + r_hi) * Hq + hq) * kHeadDim;
+#pragma unroll
+  for (int nt = 0; nt < 16; ++nt) {
+    const int d = 8 * nt + 2 * c4;
+    if (r_lo < P)
+      *reinterpret_cast<uint32_t*>(o_lo + d) = pack_bf16x2(o[nt][0] * inv_lo, o[nt][1] * inv_lo);
+    if (r_hi < P)
+      *reinterpret_cast<uint32_t*>(o_hi + d) = pack_bf16x2(o[nt][2] * inv_hi, o[nt][3] * inv_hi);
+  }
+}
+
+}  // namespace
+
+size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens) {
+  return pf_layout(heads, n_tokens).total;
+}
+
+cudaError_t launch_prefill(const void* q, const void* k, const void* v, const void* logit,
+                           int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                           int32_t group, int32_t window, float scale_log2, bool zero_first,
+                           void* workspace, void* out, cudaStream_t stream) {
+  // The kernel's shared-memory limit, raised once per device.
+  static std::atomic<uint64_t> attr_set{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (1ull << dev) : 0ull;
+  if (bit == 0 || (attr_set.load() & bit) == 0) {
+    e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kPfSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set.fetch_or(bit);
+  }
+  const int64_t H = (int64_t)batch * kv_heads;
+  const PfLayout L = pf_layout(H, n_tokens);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  e = cudaMemsetAsync(ws + L.err, 0, 64, stream);
+  if (e != cudaSuccess) return e;
+  PackParams pk;
+  pk.k = static_cast<const uint16_t*>(k);
+  pk.v = static_cast<const uint16_t*>(v);
+  pk.logit = static_cast<const uint16_t*>(logit);
+  pk.logit_stride = logit_stride;
+  pk.kd = ws + L.kd;
+  pk.vd = ws + L.vd;
+  pk.kc = ws + L.kc;
+  pk.vc = ws + L.vc;
+  pk.pc = reinterpret_cast<int32_t*>(ws + L.pc);
+  pk.before = reinterpret_cast<int32_t*>(ws + L.before);
+  pk.cc = reinterpret_cast<int32_t*>(ws + L.cc);
+  pk.P = n_tokens;
+  pk.kv_heads = kv_heads;
+  pk.nch = (n_tokens + kPfChunk - 1) / kPfChunk;
+  const dim3 pgrid((unsigned)pk.nch, (unsigned)H);
+  prefill_count_kernel<<<pgrid, kPfPackThreads, 0, stream>>>(pk);
+  prefill_pack_kernel<<<pgrid, kPfPackThreads, 0, stream>>>(pk);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  PrefillParams pp;
+  pp.q = static_cast<const __nv_bfloat16*>(q);
+  pp.out = static_cast<__nv_bfloat16*>(out);
+  pp.kd = pk.kd;
+  pp.vd = pk.vd;
+  pp.kc = pk.kc;
+  pp.vc = pk.vc;
+  pp.pc = pk.pc;
+  pp.before = pk.before;
+  pp.err = reinterpret_cast<int32_t*>(ws + L.err);
+  pp.P = n_tokens;
+  pp.kv_heads = kv_heads;
+  pp.group = group;
+  pp.window = window;
+  pp.zero_first = zero_first ? 1 : 0;
+  pp.n_qtiles = (n_tokens + kPfRows - 1) / kPfRows;
+  pp.n_qheads = (int32_t)(H * group);
+  pp.scale_log2 = scale_log2;
+  const int64_t grid = (int64_t)pp.n_qtiles * pp.n_qheads;
+  prefill_attn_kernel<<<(unsigned)grid, kPfThreads, kPfSmemBytes, stream>>>(pp);
+  return cudaGetLastError();
+}
+
+}  // namespace dms
+
+// ============================================================================ C ABI
+namespace {
+
+bool pf_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+dms_status prefill_impl(const void* q, const void* k, const void* v, const void* logit,
+                        int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                        int32_t gqa_group, int32_t window, float sm_scale, void* workspace,
+                        size_t workspace_bytes, void* out, bool zero_first, void* stream) {
+  if (q == nullptr || k == nullptr || v == nullptr || logit == nullptr || out == nullptr ||
+      workspace == nullptr || !pf_aligned16(q) || !pf_aligned16(k) || !pf_aligned16(v) ||
+      !pf_aligned16(out) || !pf_aligned16(workspace) ||
+      (reinterpret_cast<uintptr_t>(logit) & 1u) != 0 || batch < 1 || n_tokens < 1 ||
+      kv_heads < 1 || gqa_group < 1 || gqa_group > dms::kMaxGroup || window < 0 ||
+      !(sm_scale == sm_scale))
+    return DMS_ERR_INVALID_ARGUMENT;
+  const int64_t H = (int64_t)batch * kv_heads;
+  const int64_t qtiles = ((int64_t)n_tokens + 127) / 128;
+  if (H > 65535 || qtiles * H * gqa_group > 0x7fffffffll || n_tokens > (1 << 30))
+    return DMS_ERR_INVALID_ARGUMENT;
+  if (workspace_bytes < dms::prefill_workspace_bytes(H, n_tokens)) return DMS_ERR_CAPACITY;
+  const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
+  const cudaError_t e = dms::launch_prefill(
+      q, k, v, logit, logit_stride, batch, n_tokens, kv_heads, gqa_group, window,
+      scale * 1.4426950408889634f, zero_first, workspace, out, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+dms_status dms_prefill_workspace_bytes(int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                                       size_t* out_bytes) {
+  if (out_bytes == nullptr || batch < 1 || n_tokens < 1 || kv_heads < 1)
+    return DMS_ERR_INVALID_ARGUMENT;
+  *out_bytes = dms::prefill_workspace_bytes((int64_t)batch * kv_heads, n_tokens);
+  return DMS_OK;
+}
+
+dms_status dms_prefill_attention(const void* q, const void* k, const void* v,
+                                 const void* decision_logit, int32_t batch, int32_t n_tokens,
+                                 int32_t kv_heads, int32_t gqa_group, int32_t window,
+                                 float sm_scale, void* workspace, size_t workspace_bytes,
+                                 void* out, void* stream) {
+  return prefill_impl(q, k, v, decision_logit, 1, batch, n_tokens, kv_heads, gqa_group, window,
+                      sm_scale, workspace, workspace_bytes, out, false, stream);
+}
+
+dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const void* v,
+                                          int32_t batch, int32_t n_tokens, int32_t kv_heads,
+                                          int32_t gqa_group, int32_t window, float sm_scale,
+                                          void* workspace, size_t workspace_bytes, void* out,
+                                          void* stream) {
+  if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
+  return prefill_impl(q, k, v, q, (int64_t)gqa_group * dms::kHeadDim, batch, n_tokens, kv_heads,
+                      gqa_group, window, sm_scale, workspace, workspace_bytes, out, true, stream);
+}
+
+dms_status dms_prefill_device_error(const void* workspace, void* stream, dms_status* out) {
+  if (workspace == nullptr || out == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  int32_t word = 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&word, static_cast<const int32_t*>(workspace) + dms::kCtrlError,
+                      sizeof(word), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return DMS_ERR_CUDA;
+  *out = static_cast<dms_status>(word);
+  return DMS_OK;
+}
+
+}  // extern "C"
