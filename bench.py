@@ -60,6 +60,9 @@ def parse():
     ap.add_argument("--borrowed", action="store_true",
                     help="decision logits carried by element 0 of each group's first query head "
                          "(App. B) instead of a separate tensor")
+    ap.add_argument("--prefill", action="store_true",
+                    help="time the sparse prefill attention of the workload's prompt instead of "
+                         "the decode step")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (small cases for profiling)")
     return ap.parse_args()
@@ -79,6 +82,15 @@ def get_workload(args):
     if args.dense:
         wl = dataclasses.replace(wl, p_evict=0.0, ragged_beta=False, name=wl.name + "-dense")
     return wl
+
+
+def measured_bf16_peak():
+    """Measured dense bf16 peak (TFLOP/s): the burst figure, for a kernel timed alone."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 def measured_peak():
@@ -654,12 +666,166 @@ def run_reference(args, wl, world, rank):
             "gpu_launches": 0}
 
 
+PREFILL_METRIC = "sparse DMS prefill attention TFLOP/s (4*128 flop per visible (query head, key) pair)"
+
+
+def prefill_pairs(lg, window):
+    """Visible (query, key) pairs per KV head, summed: sum_j |R_j| with
+    |R_j| = j + 1 - #{i <= j - w - 1 : alpha_i = 1} (alpha_i = [logit_i > 0])."""
+    import torch
+    B, P, H = lg.shape
+    alpha = (lg.float() > 0).to(torch.int64)           # NaN keeps, +inf evicts
+    cum = torch.cumsum(alpha, dim=1)                   # [B, P, H]
+    out_sum = cum[:, :max(0, P - window - 1)].sum().item()
+    return B * H * P * (P + 1) // 2 - out_sum
+
+
+def run_prefill(args, wl, world, rank, local, pg):
+    """One step = the sparse prefill attention (pack pre-pass + attention kernel) of the
+    workload's whole prompt, for every layer in the rotation."""
+    import ctypes
+
+    import torch
+
+    import paper_2506_05345_gb300 as dms
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    B, H, G, D = wl.batch, wl.kv_heads, wl.gqa_group, wl.head_dim
+    P, w, Hq = wl.prefill_tokens, wl.window, wl.kv_heads * wl.gqa_group
+    L = max(1, min(args.layers or 2, wl.layers))
+    K_, W_ = args.steps, args.warmup
+    seed_tag = replica_tag(rank)
+    ins = []
+    for layer in range(L):
+        k, v, lg = workloads.gen_kv(wl, layer, f"{seed_tag}prompt", P, dev)
+        g = torch.Generator(device=dev).manual_seed(workloads.stable_seed(wl.name, layer, seed_tag, "pq"))
+        q = torch.randn((B, P, Hq, D), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+        if args.borrowed:
+            q[:, :, ::G, 0] = lg
+        ins.append((q, k, v, lg))
+    code, ws_bytes = dms.dms_prefill_workspace_bytes(B, P, H)
+    if code != dms.DMS_OK:
+        raise RuntimeError(f"dms_prefill_workspace_bytes: {code}")
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    outs = [torch.empty((B, P, Hq, D), dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    pairs = [prefill_pairs(lg, w) for (_, _, _, lg) in ins]
+    flops_per_step = sum(pairs) * G * 4 * D
+    lib = dms.library()
+    vp = ctypes.c_void_p
+    sptr = vp(torch.cuda.current_stream().cuda_stream)
+    calls = []
+    for layer in range(L):
+        q, k, v, lg = ins[layer]
+        if args.borrowed:
+            calls.append((lib.dms_prefill_attention_borrowed,
+                          (vp(q.data_ptr()), vp(k.data_ptr()), vp(v.data_ptr()), B, P, H, G, w, 0.0,
+                           vp(ws.data_ptr()), ws_bytes, vp(outs[layer].data_ptr()), sptr)))
+        else:
+            calls.append((lib.dms_prefill_attention,
+                          (vp(q.data_ptr()), vp(k.data_ptr()), vp(v.data_ptr()), vp(lg.data_ptr()),
+                           B, P, H, G, w, 0.0, vp(ws.data_ptr()), ws_bytes,
+                           vp(outs[layer].data_ptr()), sptr)))
+    codes = []
+
+    def step():
+        for fn, a in calls:
+            codes.append(fn(*a))
+
+    for _ in range(W_):
+        step()
+    torch.cuda.synchronize()
+    clocks = Clocks(local)
+    barrier(pg, dev)
+    clocks.start()
+    a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record()
+    for _ in range(K_):
+        step()
+    z.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(pg, dev)
+    if any(codes):
+        raise RuntimeError(f"C ABI returned {sorted(set(codes))}")
+    code, err = dms.dms_prefill_device_error(ws.data_ptr(), None)
+    if code != dms.DMS_OK or err != dms.DMS_OK:
+        raise RuntimeError(f"prefill device error {err}")
+    ms = a.elapsed_time(z)
+    ms_max = max_over_ranks(pg, ms, dev)
+    t_layer = ms_max / 1e3 / (K_ * L)
+    value = sum_over_ranks(pg, flops_per_step * K_, dev) / (ms_max / 1e3) / 1e12
+    if rank != 0:
+        return None
+    # ---- parity sample (layer 0) and CPU baseline: the fp64 oracle on sampled rows
+    import oracle
+    q, k, v, lg = ins[0]
+    rng = np.random.default_rng(workloads.stable_seed(wl.name, "prefill-sample"))
+    rows = {(int(rng.integers(B)), int(rng.integers(P)), int(rng.integers(H))) for _ in range(24)}
+    rows |= {(0, P - 1, 0), (B - 1, 0, H - 1)}
+    rows = sorted(rows)
+    got = outs[0]
+    errs, cases = [], []
+    for b, j, h in rows:
+        qq = workloads.bf16_bits(q[b, j, h * G:(h + 1) * G])
+        if args.borrowed:
+            qq = oracle.borrowed(qq, G)[1]
+        kk, vv = workloads.bf16_bits(k[b, :, h]), workloads.bf16_bits(v[b, :, h])
+        ll = workloads.bf16_bits(lg[b, :, h])
+        ref = oracle.decode(qq, kk, vv, ll, j, w)
+        errs.append(np.abs(got[b, j, h * G:(h + 1) * G].float().cpu().numpy() - ref).ravel())
+        cases.append((qq, kk, vv, ll, j, len(oracle.retained(ll, j, w))))
+    e = np.concatenate(errs)
+    parity = {"sampled_rows": len(rows), "max_abs": float(e.max()), "mean_abs": float(e.mean()),
+              "ok": bool(e.max() <= 2e-2 and e.mean() <= 2e-3)}
+    flops_cpu, t0, n = 0, time.time(), 0
+    while time.time() - t0 < args.cpu_seconds or n == 0:
+        qq, kk, vv, ll, j, nr = cases[n % len(cases)]
+        oracle.decode(qq, kk, vv, ll, j, w)
+        flops_cpu += nr * G * 4 * D
+        n += 1
+    cpu_s = time.time() - t0
+    peak, peak_kind = measured_bf16_peak()
+    achieved = flops_per_step / L / t_layer / 1e12
+    dense_pairs = B * H * P * (P + 1) // 2
+    return {
+        "metric": PREFILL_METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": K_, "warmup": W_, "ms_per_step": ms_max / K_, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "impl": "ours",
+        "config": {"workload": wl.name + "-prompt", "batch_per_gpu": B, "prompt_tokens": P,
+                   "q_heads": Hq, "kv_heads": H, "head_dim": D, "window": w,
+                   "p_evict": 0.0 if args.dense else wl.p_evict, "layers": L,
+                   "decisions": "borrowed query neuron (App. B)" if args.borrowed else "logit tensor",
+                   "l2": "no flush: each layer's prompt (q, k, v, out, workspace) is several GB",
+                   "parallelism": f"replicas x{world}"},
+        "us_per_layer": t_layer * 1e6,
+        "prompt_tokens_per_s_per_layer": B * P / t_layer,
+        "visible_pairs_per_layer": pairs[0], "dense_causal_pairs_per_layer": dense_pairs,
+        "sparsity": 1.0 - pairs[0] / dense_pairs,
+        "roofline": {"kernel": "prefill_attn_kernel + pack pre-pass", "bound": "tensor",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "peak_kind": f"{peak_kind} dense bf16 (burst)",
+                     "traffic": None,
+                     "algorithmic_flops_per_layer": flops_per_step / L,
+                     "duration": "timed region elapsed / (steps * layers)"},
+        "cpu_baseline": {"value": flops_cpu / cpu_s / 1e12, "unit": "TFLOP/s", "cores": 1,
+                         "kind": "oracle",
+                         "sample": f"{n} fp64 oracle decodes of {len(cases)} sampled (sequence, "
+                                   f"query, KV head) rows of layer 0, {cpu_s:.1f} s single-threaded"},
+        "e2e": None, "gpu_launches": 3 * L * K_, "clocks": clk, "parity_sample": parity,
+    }
+
+
 def main():
     args = parse()
     wl = get_workload(args)
     world, rank, local, pg = dist_setup(args)
     if args.impl == "reference":
         res = run_reference(args, wl, world, rank)
+    elif args.prefill:
+        res = run_prefill(args, wl, world, rank, local, pg)
     else:
         res = run_ours(args, wl, world, rank, local, pg)
     if rank == 0 and res is not None:
