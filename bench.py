@@ -63,6 +63,8 @@ def parse():
     ap.add_argument("--prefill", action="store_true",
                     help="time the sparse prefill attention of the workload's prompt instead of "
                          "the decode step")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the batch (small cases for profiling)")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (small cases for profiling)")
     return ap.parse_args()
@@ -79,6 +81,8 @@ def get_workload(args):
     import dataclasses
     if args.layers > 0:
         wl = dataclasses.replace(wl, layers=args.layers)
+    if args.batch > 0:
+        wl = dataclasses.replace(wl, batch=args.batch)
     if args.dense:
         wl = dataclasses.replace(wl, p_evict=0.0, ragged_beta=False, name=wl.name + "-dense")
     return wl
