@@ -58,6 +58,15 @@ typedef enum dms_status {
   DMS_ERR_STATE = 6             /* call not valid in the cache's current state */
 } dms_status;
 
+/* Eviction policies selectable through dms_options.eviction_policy. */
+enum {
+  DMS_EVICT_DELAYED = 0,   /* default, the method (Sec. 3.1): the token leaving the window
+                              at step j is evicted iff its own decision alpha_{j-w-1} = 1 */
+  DMS_EVICT_IMMEDIATE = 1  /* the ablation of Sec. 5: it is evicted iff the decision of
+                              token j - 1 (= (j - w - 1) + w) is 1; the same as delayed
+                              when window = 0                                            */
+};
+
 /* Decode kernels selectable through dms_options.decode_kernel. */
 enum {
   DMS_DECODE_TILED = 0,  /* default: TMA-staged, tensor-core, page-balanced split-K */
@@ -74,7 +83,8 @@ typedef struct dms_options {
   int32_t decode_kernel; /* DMS_DECODE_TILED (0) or DMS_DECODE_SIMPLE (1)           */
   int32_t ctas_per_sm;   /* split-K CTAs per SM for the tiled kernel; 0 = 1         */
   int32_t min_pages_per_cta; /* lower bound on pages per split-K CTA; 0 = 2         */
-  int32_t reserved[5];   /* must be zero                                            */
+  int32_t eviction_policy;   /* DMS_EVICT_DELAYED (0) or DMS_EVICT_IMMEDIATE (1)    */
+  int32_t reserved[4];   /* must be zero                                            */
 } dms_options;
 
 typedef struct dms_stats {
@@ -221,6 +231,14 @@ dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const vo
                                           int32_t gqa_group, int32_t window, float sm_scale,
                                           void* workspace, size_t workspace_bytes, void* out,
                                           void* stream);
+/* The general form: decision_logit == NULL takes the decisions from the queries as in
+ * the borrowed form; eviction_policy DMS_EVICT_DELAYED or DMS_EVICT_IMMEDIATE (the Sec. 5
+ * ablation: key i is visible outside the window iff the decision of token i + window is 0). */
+dms_status dms_prefill_attention_ex(const void* q, const void* k, const void* v,
+                                    const void* decision_logit, int32_t batch, int32_t n_tokens,
+                                    int32_t kv_heads, int32_t gqa_group, int32_t window,
+                                    int32_t eviction_policy, float sm_scale, void* workspace,
+                                    size_t workspace_bytes, void* out, void* stream);
 /* Synchronise `stream` and report the sticky device error of the last prefill that used
  * `workspace` into *out (DMS_OK when none). */
 dms_status dms_prefill_device_error(const void* workspace, void* stream, dms_status* out);

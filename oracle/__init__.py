@@ -9,8 +9,9 @@ module compiles it with gcc on first use and wraps it with ctypes.
 
 Functions (all take bf16 data as ``numpy.uint16`` bit patterns):
   alpha(logit_bits)                      Sec. 3.2 decision, [logit > 0]
-  retained(logits, j, w)                 Sec. 3.1 / Fig. 1b retained positions
-  decode(q, k, v, logits, j, w, scale)   softmax attention over the retained set
+  retained(logits, j, w, immediate)      Sec. 3.1 / Fig. 1b retained positions (Sec. 5
+                                         immediate-eviction ablation when immediate)
+  decode(q, k, v, logits, j, w, scale, immediate)  softmax attention over the retained set
   borrowed(q, G)                         App. B decision neuron: (logits, attention q)
 """
 from __future__ import annotations
@@ -60,6 +61,14 @@ def _load():
                                               ctypes.c_int64, ctypes.c_int64, ctypes.c_double,
                                               f64p]
             lib.dms_oracle_decode.restype = None
+            lib.dms_oracle_retained_policy.argtypes = [u16p, ctypes.c_int64, ctypes.c_int64,
+                                                       ctypes.c_int64, ctypes.c_int, i32p]
+            lib.dms_oracle_retained_policy.restype = ctypes.c_int64
+            lib.dms_oracle_decode_policy.argtypes = [u16p, ctypes.c_int32, ctypes.c_int32, u16p,
+                                                     u16p, ctypes.c_int64, u16p, ctypes.c_int64,
+                                                     ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
+                                                     ctypes.c_double, f64p]
+            lib.dms_oracle_decode_policy.restype = None
             _lib = lib
     return _lib
 
@@ -84,10 +93,11 @@ def alpha(logit_bits: int) -> int:
     return int(_load().dms_oracle_alpha(int(logit_bits) & 0xFFFF))
 
 
-def retained(logits, j: int, w: int) -> np.ndarray:
+def retained(logits, j: int, w: int, immediate: bool = False) -> np.ndarray:
     """Sorted positions retained by one KV head after appending position j.
 
     ``logits`` is a 1-D uint16 array (any stride) holding positions 0..j.
+    ``immediate``: the eviction ablation of Sec. 5 (token i decided by alpha_{i+w}).
     """
     lg = _u16(logits)
     if lg.ndim != 1:
@@ -96,12 +106,13 @@ def retained(logits, j: int, w: int) -> np.ndarray:
         raise ValueError("j beyond the logits given")
     stride = lg.strides[0] // 2
     out = np.empty(max(j + 1, 1), dtype=np.int32)
-    n = _load().dms_oracle_retained(_ptr(lg, ctypes.c_uint16), stride, j, w,
-                                    _ptr(out, ctypes.c_int32))
+    n = _load().dms_oracle_retained_policy(_ptr(lg, ctypes.c_uint16), stride, j, w,
+                                           1 if immediate else 0, _ptr(out, ctypes.c_int32))
     return out[:n].copy()
 
 
-def decode(q, k, v, logits, j: int, w: int, scale: float = 0.0) -> np.ndarray:
+def decode(q, k, v, logits, j: int, w: int, scale: float = 0.0,
+           immediate: bool = False) -> np.ndarray:
     """Attention of G query heads over the retained set of their KV head at step j.
 
     q: [G, D] uint16; k, v: [T, D] uint16 (row-strided views allowed, rows 0..j);
@@ -124,10 +135,11 @@ def decode(q, k, v, logits, j: int, w: int, scale: float = 0.0) -> np.ndarray:
     if j >= k.shape[0] or j >= lg.shape[0]:
         raise ValueError("j beyond the data given")
     out = np.zeros((G, D), dtype=np.float64)
-    _load().dms_oracle_decode(_ptr(q, ctypes.c_uint16), G, D, _ptr(k, ctypes.c_uint16),
-                              _ptr(v, ctypes.c_uint16), k.strides[0] // 2,
-                              _ptr(lg, ctypes.c_uint16), lg.strides[0] // 2, j, w,
-                              float(scale), _ptr(out, ctypes.c_double))
+    _load().dms_oracle_decode_policy(_ptr(q, ctypes.c_uint16), G, D, _ptr(k, ctypes.c_uint16),
+                                     _ptr(v, ctypes.c_uint16), k.strides[0] // 2,
+                                     _ptr(lg, ctypes.c_uint16), lg.strides[0] // 2, j, w,
+                                     1 if immediate else 0, float(scale),
+                                     _ptr(out, ctypes.c_double))
     return out
 
 

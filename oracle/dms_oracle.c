@@ -21,6 +21,12 @@
  *   - Sec. 3.2 / Sec. 4 (GQA): plain softmax attention of each query head over
  *     the retained set of its KV head, scale 1/sqrt(D) unless given.
  *
+ *   - Sec. 5 (Ablations), immediate eviction: the eviction of past token t at time
+ *     t + w is decided by alpha_{t+w} instead of alpha_t.  Reading used here (the
+ *     timing kept, only the deciding variable changed): key i is visible to the
+ *     query at step j iff i <= j and (j - i <= w or alpha_{i+w} == 0).  With
+ *     w = 0 the two policies coincide.
+ *
  * The retained set R_j is built by scanning the decisions directly from the
  * definition above; there is no ring, slot or page logic here.  All arithmetic
  * is fp64 with plain sequential sums in index order.  bf16 inputs are widened
@@ -57,17 +63,27 @@ static int visible(const uint16_t* logits, int64_t logit_stride, int64_t i,
   return dms_oracle_alpha(logits[i * logit_stride]) ? 0 : 1;
 }
 
+/* Sec. 5 immediate eviction: key i is decided by the token at position i + w. */
+static int visible_immediate(const uint16_t* logits, int64_t logit_stride, int64_t i,
+                             int64_t j, int64_t w) {
+  if (i > j) return 0;                 /* causal */
+  if (j - i <= w) return 1;            /* still inside the sliding window */
+  /* j - i > w, so the deciding token i + w < j has already been seen */
+  return dms_oracle_alpha(logits[(i + w) * logit_stride]) ? 0 : 1;
+}
+
 /*
  * Retained set R_j of one (layer, sequence, KV head) after the token at
  * position j has been appended.  logits[i * logit_stride] is the bf16 decision
  * logit of position i.  Writes the sorted positions to pos_out (may be NULL)
  * and returns |R_j|.  Returns 0 for j < 0.
  */
-int64_t dms_oracle_retained(const uint16_t* logits, int64_t logit_stride,
-                            int64_t j, int64_t w, int32_t* pos_out) {
+int64_t dms_oracle_retained_policy(const uint16_t* logits, int64_t logit_stride,
+                                   int64_t j, int64_t w, int immediate, int32_t* pos_out) {
   int64_t n = 0;
   for (int64_t i = 0; i <= j; ++i) {
-    if (visible(logits, logit_stride, i, j, w)) {
+    if (immediate ? visible_immediate(logits, logit_stride, i, j, w)
+                  : visible(logits, logit_stride, i, j, w)) {
       if (pos_out) pos_out[n] = (int32_t)i;
       ++n;
     }
@@ -85,15 +101,26 @@ int64_t dms_oracle_retained(const uint16_t* logits, int64_t logit_stride,
  * Softmax over R_j of s_i = scale * <q, k_i>; out = sum_i p_i v_i.
  * An empty retained set (j < 0) yields zeros.
  */
-void dms_oracle_decode(const uint16_t* q, int32_t G, int32_t D,
-                       const uint16_t* k, const uint16_t* v, int64_t kv_stride,
-                       const uint16_t* logits, int64_t logit_stride, int64_t j,
-                       int64_t w, double scale, double* out) {
+/* Delayed eviction (Sec. 3.1), the method's policy. */
+int64_t dms_oracle_retained(const uint16_t* logits, int64_t logit_stride,
+                            int64_t j, int64_t w, int32_t* pos_out) {
+  return dms_oracle_retained_policy(logits, logit_stride, j, w, 0, pos_out);
+}
+
+/*
+ * Softmax attention at step j of the G query heads q[G][D] of one group over
+ * the retained set of their KV head (k, v rows at k + i * kv_stride), under the
+ * delayed (immediate = 0) or immediate (1) eviction policy; out[G][D].
+ */
+void dms_oracle_decode_policy(const uint16_t* q, int32_t G, int32_t D,
+                              const uint16_t* k, const uint16_t* v, int64_t kv_stride,
+                              const uint16_t* logits, int64_t logit_stride, int64_t j,
+                              int64_t w, int immediate, double scale, double* out) {
   if (scale <= 0.0) scale = 1.0 / sqrt((double)D);
   int64_t cap = j + 1 > 0 ? j + 1 : 0;
   int32_t* pos = (int32_t*)malloc(sizeof(int32_t) * (size_t)(cap > 0 ? cap : 1));
   double* s = (double*)malloc(sizeof(double) * (size_t)(cap > 0 ? cap : 1));
-  int64_t n = dms_oracle_retained(logits, logit_stride, j, w, pos);
+  int64_t n = dms_oracle_retained_policy(logits, logit_stride, j, w, immediate, pos);
   for (int32_t g = 0; g < G; ++g) {
     double* o = out + (int64_t)g * D;
     for (int32_t d = 0; d < D; ++d) o[d] = 0.0;
@@ -121,4 +148,11 @@ void dms_oracle_decode(const uint16_t* q, int32_t G, int32_t D,
   }
   free(pos);
   free(s);
+}
+
+void dms_oracle_decode(const uint16_t* q, int32_t G, int32_t D,
+                       const uint16_t* k, const uint16_t* v, int64_t kv_stride,
+                       const uint16_t* logits, int64_t logit_stride, int64_t j,
+                       int64_t w, double scale, double* out) {
+  dms_oracle_decode_policy(q, G, D, k, v, kv_stride, logits, logit_stride, j, w, 0, scale, out);
 }

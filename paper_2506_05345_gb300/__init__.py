@@ -20,7 +20,8 @@ import ctypes
 import numpy as np
 
 from . import _native
-from ._native import (DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
+from ._native import (DMS_EVICT_DELAYED, DMS_EVICT_IMMEDIATE,  # noqa: F401
+                      DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
                       DMS_ERR_INVALID_ARGUMENT, DMS_ERR_TIMEOUT, DMS_OK, DmsLibraryError,
                       dms_options, dms_stats)
 
@@ -121,8 +122,17 @@ def dms_prefill_device_error(ws_ptr, stream):
     return code, out.value
 
 
+def dms_prefill_attention_ex(q_ptr, k_ptr, v_ptr, logit_ptr, batch, n_tokens, kv_heads,
+                             gqa_group, window, eviction_policy, sm_scale, ws_ptr, ws_bytes,
+                             out_ptr, stream):
+    return library().dms_prefill_attention_ex(q_ptr, k_ptr, v_ptr, logit_ptr, batch, n_tokens,
+                                              kv_heads, gqa_group, window, eviction_policy,
+                                              float(sm_scale), ws_ptr, ws_bytes, out_ptr, stream)
+
+
 def prefill_attention(q, k, v, decision_logit=None, window: int = 256, gqa_group=None,
-                      sm_scale: float = 0.0, workspace=None, out=None, stream=None):
+                      sm_scale: float = 0.0, workspace=None, out=None, stream=None,
+                      eviction_policy: int = 0):
     """Sparse DMS prefill attention of a whole prompt (no cache involved).
 
     q: [B, P, Hkv * G, 128], k, v: [B, P, Hkv, 128], decision_logit: [B, P, Hkv] bf16 CUDA
@@ -148,7 +158,13 @@ def prefill_attention(q, k, v, decision_logit=None, window: int = 256, gqa_group
         raise TypeError("workspace must be a uint8 CUDA tensor")
     wp = ctypes.c_void_p(workspace.data_ptr())
     wb = workspace.numel()
-    if decision_logit is None:
+    if eviction_policy != 0:
+        lp = None if decision_logit is None else _bf16_cuda(decision_logit, (B, P, Hkv),
+                                                            "decision_logit")
+        code = dms_prefill_attention_ex(qp, kp, vp, lp, B, P, Hkv, gqa_group, window,
+                                        eviction_policy, sm_scale, wp, wb, op, _stream_ptr(stream))
+        _check(code, "dms_prefill_attention_ex")
+    elif decision_logit is None:
         code = dms_prefill_attention_borrowed(qp, kp, vp, B, P, Hkv, gqa_group, window, sm_scale,
                                               wp, wb, op, _stream_ptr(stream))
         _check(code, "dms_prefill_attention_borrowed")
@@ -211,7 +227,7 @@ class DmsCache:
     def __init__(self, layers: int, kv_heads: int, window: int, capacity: int, batch: int,
                  head_dim: int = HEAD_DIM, pool_tokens: int = 0,
                  decode_kernel: int = DMS_DECODE_TILED, ctas_per_sm: int = 0,
-                 min_pages_per_cta: int = 0):
+                 min_pages_per_cta: int = 0, eviction_policy: int = 0):
         self._h = None
         opt = dms_options()
         opt.batch = batch
@@ -219,6 +235,7 @@ class DmsCache:
         opt.decode_kernel = decode_kernel
         opt.ctas_per_sm = ctas_per_sm
         opt.min_pages_per_cta = min_pages_per_cta
+        opt.eviction_policy = eviction_policy
         code, h = dms_cache_create(layers, kv_heads, head_dim, window, capacity, opt)
         _check(code, "dms_cache_create")
         self._h = h

@@ -19,6 +19,8 @@ DMS_ERR_CAPACITY = 3
 DMS_ERR_CUDA = 4
 DMS_ERR_TIMEOUT = 5
 DMS_ERR_STATE = 6
+DMS_EVICT_DELAYED = 0
+DMS_EVICT_IMMEDIATE = 1
 DMS_DECODE_TILED = 0
 DMS_DECODE_SIMPLE = 1
 
@@ -30,7 +32,7 @@ EXPORTS = (
     "dms_append_and_decode", "dms_selftest_bounded_wait", "dms_append_and_evict_borrowed",
     "dms_decode_attention_borrowed", "dms_append_and_decode_borrowed",
     "dms_prefill_workspace_bytes", "dms_prefill_attention", "dms_prefill_attention_borrowed",
-    "dms_prefill_device_error",
+    "dms_prefill_device_error", "dms_prefill_attention_ex",
 )
 
 
@@ -42,7 +44,7 @@ class dms_options(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("page_tokens", ctypes.c_int32),
                 ("pool_tokens", ctypes.c_int64), ("decode_kernel", ctypes.c_int32),
                 ("ctas_per_sm", ctypes.c_int32), ("min_pages_per_cta", ctypes.c_int32),
-                ("reserved", ctypes.c_int32 * 5)]
+                ("eviction_policy", ctypes.c_int32), ("reserved", ctypes.c_int32 * 4)]
 
 
 class dms_stats(ctypes.Structure):
@@ -88,6 +90,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_prefill_attention_borrowed": (st, [vp, vp, vp, i32, i32, i32, i32, i32, f32, vp,
                                                 ctypes.c_size_t, vp, vp]),
         "dms_prefill_device_error": (st, [vp, vp, ctypes.POINTER(st)]),
+        "dms_prefill_attention_ex": (st, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, f32, vp,
+                                          ctypes.c_size_t, vp, vp]),
         "dms_cache_stats": (st, [vp, ctypes.POINTER(dms_stats), vp, vp]),
         "dms_cache_export_positions": (st, [vp, i32, vp, vp]),
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),

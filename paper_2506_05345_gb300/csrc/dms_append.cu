@@ -36,6 +36,7 @@ struct AppendParams {
   int64_t logit_stride;  // elements between consecutive decision logits
   int64_t t0;           // position of the first appended token
   int64_t window;
+  int64_t decider;       // the eviction bit of token i is the decision of token i + decider
   int64_t pool_pages;
   int32_t n;            // tokens appended by this call
   int32_t heads, kv_heads, max_pages, ring_len;
@@ -97,7 +98,10 @@ __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
     }
     p.counts_next[bh] = n;  // unchanged if the page pool ran out
     if (ok) {
-      ring[j % RP] = (uint32_t)slot | (alpha << 31);
+      // This token's decision: its own eviction bit (delayed), or that of token
+      // j - decider (immediate-eviction ablation; its entry is still in the ring).
+      ring[j % RP] = (uint32_t)slot | ((p.decider == 0 ? alpha : 0u) << 31);
+      if (p.decider > 0 && j >= p.decider) ring[(j - p.decider) % RP] |= alpha << 31;
       page = pt[slot / kPageTokens];
       p.pos[(int64_t)page * kPageTokens + (slot & (kPageTokens - 1))] = (int32_t)j;
     }
@@ -148,6 +152,23 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
   int32_t* pt = p.page_table + (int64_t)bh * p.max_pages;
   const int32_t nh = p.counts_cur[bh];
 
+  // Decision of new token li (local index), 0 past the call.
+  auto alpha_new = [&](int64_t li) -> uint32_t {
+    return li < n ? decision_from_bf16(p.logit[(((int64_t)b * n + li) * p.kv_heads + hk) * p.logit_stride])
+                  : 0u;
+  };
+  const int64_t dec = p.decider;
+  // 0. Immediate-eviction ablation: old tokens still in the window whose deciding
+  //    token (i + decider) arrives in this call receive their eviction bit now.
+  if (dec > 0) {
+    const int64_t a = t0 - dec > 0 ? t0 - dec : 0;
+    for (int64_t i = a + tid; i < t0; i += kBulkThreads) {
+      const int64_t li = i + dec - t0;
+      if (li < n) ring[i % RP] |= alpha_new(li) << 31;
+    }
+    __syncthreads();
+  }
+
   // 1. Old tokens leaving the window during this call: positions [lo, hi], all < t0.
   const int64_t lo = t0 - R > 0 ? t0 - R : 0;
   const int64_t hi = (t0 - 1) < (t0 + n - R - 1) ? (t0 - 1) : (t0 + n - R - 1);
@@ -167,13 +188,13 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
   }
 
   // 2. New tokens that also leave within this call (local index < n - R) and are
-  //    flagged are never stored.
+  //    flagged (their deciding token, li + decider < n - 1, is in the call) are never
+  //    stored.
   const int64_t n_leave_new = n - R > 0 ? n - R : 0;
   int evicted_new = 0;
   for (int64_t base = 0; base < n_leave_new; base += kBulkThreads) {
     int flag = 0;
-    if (base + tid < n_leave_new)
-      flag = (int)decision_from_bf16(p.logit[(((int64_t)b * n + base + tid) * p.kv_heads + hk) * p.logit_stride]);
+    if (base + tid < n_leave_new) flag = (int)alpha_new(base + tid + dec);
     int total;
     block_scan_flags(flag, s_warp, &total);
     evicted_new += total;
@@ -210,8 +231,8 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
   for (int64_t base = 0; base < n; base += kBulkThreads) {
     const int64_t li = base + tid;
     const bool valid = li < n;
-    uint32_t alpha = 0;
-    if (valid) alpha = decision_from_bf16(p.logit[(((int64_t)b * n + li) * p.kv_heads + hk) * p.logit_stride]);
+    // eviction bit of token li: the decision of token li + decider if it is in the call
+    const uint32_t alpha = valid ? alpha_new(li + dec) : 0u;
     const int kept = (valid && !(alpha && li < n_leave_new)) ? 1 : 0;
     int total;
     const int r = block_scan_flags(kept, s_warp, &total);
@@ -283,6 +304,7 @@ AppendParams make_params(const Cache& c, int32_t layer, const void* k, const voi
   p.logit_stride = logit_stride;
   p.t0 = t0;
   p.window = c.window;
+  p.decider = c.decider();
   p.pool_pages = c.pool_pages;
   p.n = n;
   p.heads = c.heads;

@@ -67,9 +67,10 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
     return DMS_ERR_INVALID_ARGUMENT;
   if (opt->page_tokens != 0 && opt->page_tokens != dms::kPageTokens) return DMS_ERR_INVALID_ARGUMENT;
   if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SIMPLE ||
-      opt->ctas_per_sm < 0 || opt->ctas_per_sm > dms::kMaxCtasPerSm || opt->min_pages_per_cta < 0)
+      opt->ctas_per_sm < 0 || opt->ctas_per_sm > dms::kMaxCtasPerSm || opt->min_pages_per_cta < 0 ||
+      opt->eviction_policy < DMS_EVICT_DELAYED || opt->eviction_policy > DMS_EVICT_IMMEDIATE)
     return DMS_ERR_INVALID_ARGUMENT;
-  for (int i = 0; i < 5; ++i)
+  for (int i = 0; i < 4; ++i)
     if (opt->reserved[i] != 0) return DMS_ERR_INVALID_ARGUMENT;
   const int64_t heads = (int64_t)opt->batch * kv_heads;
   if (heads > dms::kMaxHeads) return DMS_ERR_INVALID_ARGUMENT;
@@ -91,6 +92,7 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
                      ? (opt->pool_tokens + dms::kPageTokens - 1) / dms::kPageTokens
                      : (int64_t)layers * heads * c.max_pages;
   c.decode_kernel = opt->decode_kernel;
+  c.eviction_policy = opt->eviction_policy;
   c.ctas_per_sm = opt->ctas_per_sm > 0 ? opt->ctas_per_sm : 1;
   c.min_pages_per_cta = opt->min_pages_per_cta > 0 ? opt->min_pages_per_cta : 2;
   if (c.pool_pages < 1 || c.pool_pages > 0x7fffffffLL) {

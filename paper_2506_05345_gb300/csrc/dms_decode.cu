@@ -93,6 +93,7 @@ struct DecodeParams {
   uint32_t* ring;             // this layer: [heads][ring_len]
   int32_t* pos;
   int64_t j, window, pool_pages;
+  int64_t decider;  // the eviction bit of token i is the decision of token i + decider
   int32_t ring_len;
   // Nonzero when the kernel launched just before on the stream cannot have written
   // this layer's cache state (it served another layer): the state is read, and the
@@ -393,7 +394,13 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
           const uint32_t sl = s_slot[h_i] & 0x3fffffffu;
           const uint32_t alpha = decision_from_bf16(p.logit_new[(int64_t)h_i * p.logit_stride]);
           p.counts_next[h_i] = s_cnt[h_i];
-          p.ring[(int64_t)h_i * p.ring_len + p.j % ring_period(p.window)] = sl | (alpha << 31);
+          // the new token's decision: its own eviction bit (delayed), or that of token
+          // j - decider (immediate-eviction ablation; still in the ring, and not the
+          // leaving token's entry that every CTA reads)
+          uint32_t* rh = p.ring + (int64_t)h_i * p.ring_len;
+          const int64_t RP = ring_period(p.window);
+          rh[p.j % RP] = sl | ((p.decider == 0 ? alpha : 0u) << 31);
+          if (p.decider > 0 && p.j >= p.decider) rh[(p.j - p.decider) % RP] |= alpha << 31;
         }
       }
     };
@@ -1184,6 +1191,7 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
   p.pos = c.pos;
   p.j = t0;
   p.window = c.window;
+  p.decider = c.decider();
   p.pool_pages = c.pool_pages;
   p.ring_len = c.ring_len;
   return launch_tiled(p, c.num_sms, 1, stream, true, true);

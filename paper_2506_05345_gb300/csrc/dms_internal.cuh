@@ -16,7 +16,10 @@
 //               a kernel whose CTAs all read every head's count never sees a count
 //               that another CTA of the same launch has already advanced.
 //   rings       [layers][heads][ring_len] u32    decisions of recent tokens: the entry of
-//               position j sits at j % (window + 2) and holds slot | alpha << 31.  The
+//               position j sits at j % (window + 2) and holds slot | e << 31, e the bit
+//               that decides the token's eviction when it leaves the window: its own
+//               alpha_j (delayed eviction), or alpha_{j+window}, OR-ed in when token
+//               j + window arrives (immediate-eviction ablation; 0 until then).  The
 //               period is one longer than the window + 1 tokens that must be kept, so
 //               the entry read for the token leaving at step j ((j - window - 1) %
 //               (window + 2)) and the entry written for the new token (j % (window + 2))
@@ -62,6 +65,10 @@ struct Cache {
   int32_t max_pages = 0;    // ceil(capacity / 64)
   int64_t pool_pages = 0;
   int32_t decode_kernel = 0, ctas_per_sm = 1, min_pages_per_cta = 2;
+  int32_t eviction_policy = DMS_EVICT_DELAYED;
+  // Position offset of the token whose decision evicts a given token: 0 for delayed
+  // eviction (its own decision), window for the immediate-eviction ablation.
+  int64_t decider() const { return eviction_policy == DMS_EVICT_IMMEDIATE ? window : 0; }
   int32_t device = 0, num_sms = 0;
   int64_t piece_capacity = 0;
 
@@ -138,7 +145,7 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
 size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens);
 cudaError_t launch_prefill(const void* q, const void* k, const void* v, const void* logit,
                            int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
-                           int32_t group, int32_t window, float scale_log2, bool zero_first,
-                           void* workspace, void* out, cudaStream_t stream);
+                           int32_t group, int32_t window, bool immediate, float scale_log2,
+                           bool zero_first, void* workspace, void* out, cudaStream_t stream);
 
 }  // namespace dms

@@ -80,6 +80,7 @@ struct PackParams {
   const uint16_t* v;
   const uint16_t* logit;     // decision logit of (b, i, h) at logit[((b P + i) Hkv + h) stride]
   int64_t logit_stride;
+  int64_t decider;           // token i is evicted by the decision of token i + decider
   uint8_t* kd;               // [H][P] permuted rows
   uint8_t* vd;
   uint8_t* kc;               // [H][P] permuted rows of the alpha = 0 tokens, position order
@@ -96,9 +97,14 @@ __device__ __forceinline__ uint32_t chunk_in_row(int64_t row, int chunk) {
   return (uint32_t)((chunk ^ (int)(row & 7)) << 4);
 }
 
+// Token i stays visible outside the window iff the decision that evicts it is 0: its
+// own (delayed eviction) or that of token i + decider (immediate-eviction ablation).  A
+// token whose deciding token lies past the prompt is inside the window of every query
+// of the prompt, so it is never needed in the compacted list.
 __device__ __forceinline__ bool keep_token(const PackParams& p, int b, int hk, int i) {
-  return decision_from_bf16(
-             p.logit[(((int64_t)b * p.P + i) * p.kv_heads + hk) * p.logit_stride]) == 0u;
+  const int64_t d = i + p.decider;
+  return d < p.P &&
+         decision_from_bf16(p.logit[(((int64_t)b * p.P + d) * p.kv_heads + hk) * p.logit_stride]) == 0u;
 }
 
 // Alpha = 0 tokens of each (head, chunk).
@@ -438,8 +444,8 @@ size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens) {
 
 cudaError_t launch_prefill(const void* q, const void* k, const void* v, const void* logit,
                            int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
-                           int32_t group, int32_t window, float scale_log2, bool zero_first,
-                           void* workspace, void* out, cudaStream_t stream) {
+                           int32_t group, int32_t window, bool immediate, float scale_log2,
+                           bool zero_first, void* workspace, void* out, cudaStream_t stream) {
   // The kernel's shared-memory limit, raised once per device.
   static std::atomic<uint64_t> attr_set{0};
   int dev = 0;
@@ -462,6 +468,7 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
   pk.v = static_cast<const uint16_t*>(v);
   pk.logit = static_cast<const uint16_t*>(logit);
   pk.logit_stride = logit_stride;
+  pk.decider = immediate ? window : 0;
   pk.kd = ws + L.kd;
   pk.vd = ws + L.vd;
   pk.kc = ws + L.kc;
@@ -509,14 +516,15 @@ bool pf_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u)
 
 dms_status prefill_impl(const void* q, const void* k, const void* v, const void* logit,
                         int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
-                        int32_t gqa_group, int32_t window, float sm_scale, void* workspace,
-                        size_t workspace_bytes, void* out, bool zero_first, void* stream) {
+                        int32_t gqa_group, int32_t window, int32_t policy, float sm_scale,
+                        void* workspace, size_t workspace_bytes, void* out, bool zero_first,
+                        void* stream) {
   if (q == nullptr || k == nullptr || v == nullptr || logit == nullptr || out == nullptr ||
       workspace == nullptr || !pf_aligned16(q) || !pf_aligned16(k) || !pf_aligned16(v) ||
       !pf_aligned16(out) || !pf_aligned16(workspace) ||
       (reinterpret_cast<uintptr_t>(logit) & 1u) != 0 || batch < 1 || n_tokens < 1 ||
       kv_heads < 1 || gqa_group < 1 || gqa_group > dms::kMaxGroup || window < 0 ||
-      !(sm_scale == sm_scale))
+      !(sm_scale == sm_scale) || policy < DMS_EVICT_DELAYED || policy > DMS_EVICT_IMMEDIATE)
     return DMS_ERR_INVALID_ARGUMENT;
   const int64_t H = (int64_t)batch * kv_heads;
   const int64_t qtiles = ((int64_t)n_tokens + 127) / 128;
@@ -526,7 +534,8 @@ dms_status prefill_impl(const void* q, const void* k, const void* v, const void*
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
   const cudaError_t e = dms::launch_prefill(
       q, k, v, logit, logit_stride, batch, n_tokens, kv_heads, gqa_group, window,
-      scale * 1.4426950408889634f, zero_first, workspace, out, static_cast<cudaStream_t>(stream));
+      policy == DMS_EVICT_IMMEDIATE, scale * 1.4426950408889634f, zero_first, workspace, out,
+      static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
 }
 
@@ -548,7 +557,7 @@ dms_status dms_prefill_attention(const void* q, const void* k, const void* v,
                                  float sm_scale, void* workspace, size_t workspace_bytes,
                                  void* out, void* stream) {
   return prefill_impl(q, k, v, decision_logit, 1, batch, n_tokens, kv_heads, gqa_group, window,
-                      sm_scale, workspace, workspace_bytes, out, false, stream);
+                      DMS_EVICT_DELAYED, sm_scale, workspace, workspace_bytes, out, false, stream);
 }
 
 dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const void* v,
@@ -558,7 +567,21 @@ dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const vo
                                           void* stream) {
   if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
   return prefill_impl(q, k, v, q, (int64_t)gqa_group * dms::kHeadDim, batch, n_tokens, kv_heads,
-                      gqa_group, window, sm_scale, workspace, workspace_bytes, out, true, stream);
+                      gqa_group, window, DMS_EVICT_DELAYED, sm_scale, workspace, workspace_bytes,
+                      out, true, stream);
+}
+
+dms_status dms_prefill_attention_ex(const void* q, const void* k, const void* v,
+                                    const void* decision_logit, int32_t batch, int32_t n_tokens,
+                                    int32_t kv_heads, int32_t gqa_group, int32_t window,
+                                    int32_t eviction_policy, float sm_scale, void* workspace,
+                                    size_t workspace_bytes, void* out, void* stream) {
+  if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
+  const bool borrowed = decision_logit == nullptr;
+  return prefill_impl(q, k, v, borrowed ? q : decision_logit,
+                      borrowed ? (int64_t)gqa_group * dms::kHeadDim : 1, batch, n_tokens,
+                      kv_heads, gqa_group, window, eviction_policy, sm_scale, workspace,
+                      workspace_bytes, out, borrowed, stream);
 }
 
 dms_status dms_prefill_device_error(const void* workspace, void* stream, dms_status* out) {

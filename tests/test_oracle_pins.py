@@ -374,3 +374,46 @@ def test_borrowed_neuron_multi_head_layout():
                 assert np.array_equal(q_att[b, h * G + g, d0:], q[b, h * G + g, d0:])
     with pytest.raises(ValueError):
         oracle.borrowed(q[:, :-1], G)
+
+
+# --------------------------------------------------------------------------- Sec. 5 ablation
+
+
+@pytest.mark.parametrize("w", [0, 1, 3, 16])
+def test_immediate_eviction_is_delayed_on_shifted_decisions(w):
+    """Immediate eviction (token i decided by alpha_{i+w}) equals delayed eviction on the
+    decisions shifted by w; w = 0 makes the two policies identical; the count is
+    (j + 1) - #{k in [w, j - 1] : alpha_k = 1}."""
+    rng = np.random.default_rng(13 + w)
+    T = 120
+    lg = _bf16(rng.standard_normal(T) + 0.4)
+    alpha = (_f64(lg) > 0).astype(int)
+    shifted = np.concatenate([lg[w:], np.zeros(w, dtype=np.uint16)])  # +0 keeps
+    for j in range(T):
+        imm = oracle.retained(lg, j, w, immediate=True)
+        assert np.array_equal(imm, oracle.retained(shifted, j, w))
+        if w == 0:
+            assert np.array_equal(imm, oracle.retained(lg, j, w))
+        assert len(imm) == (j + 1) - int(alpha[w:j].sum()) if j > w else len(imm) == j + 1
+
+
+def test_immediate_eviction_decode_brute_force():
+    """Decode under immediate eviction equals the dense softmax with its mask."""
+    rng = np.random.default_rng(17)
+    T, G, D, w = 50, 3, 32, 4
+    q, k, v, lg = _rand_case(rng, T, G, D, 0.6)
+    alpha = (_f64(lg) > 0).astype(np.float64)
+    M = np.full((T, T), -np.inf)
+    for j in range(T):
+        for i in range(j + 1):
+            if j - i <= w or alpha[i + w] == 0:
+                M[j, i] = 0.0
+    scale = 1.0 / math.sqrt(D)
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    ref = np.stack([_sdpa_masked(qd[:, g], kd, vd, M, scale) for g in range(G)], axis=1)
+    differs = False
+    for j in range(T):
+        got = oracle.decode(q[j], k, v, lg, j, w, immediate=True)
+        np.testing.assert_allclose(got, ref[j], rtol=0, atol=1e-12)
+        differs |= not np.array_equal(got, oracle.decode(q[j], k, v, lg, j, w))
+    assert differs  # the ablation is a different policy
