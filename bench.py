@@ -63,6 +63,9 @@ def parse():
     ap.add_argument("--prefill", action="store_true",
                     help="time the sparse prefill attention of the workload's prompt instead of "
                          "the decode step")
+    ap.add_argument("--shared-prefix", action="store_true",
+                    help="append the workload's shared prompt once and share its frozen pages "
+                         "between the sequences")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the batch (small cases for profiling)")
     ap.add_argument("--layers", type=int, default=0,
@@ -268,14 +271,19 @@ def run_ours(args, wl, world, rank, local, pg):
             for c0 in range(0, n, chunk):
                 nc = min(chunk, n - c0)
                 tag = f"{seed_tag}prefill{i}" + (f"c{c0}" if n > chunk else "")
-                if shared:
+                if shared and args.shared_prefix and cache.layer_length(layer) == 0:
+                    k, v, lg = workloads.gen_kv(wl, layer, tag, nc, dev, batch=1)
+                    cache.append_shared_prefix(layer, k, v, lg)  # stored once, pages shared
+                    k, v, lg = k.expand(B, -1, -1, -1), v.expand(B, -1, -1, -1), lg.expand(B, -1, -1)
+                elif shared:
                     k, v, lg = workloads.gen_kv(wl, layer, tag, nc, dev, batch=1)
                     k = k.expand(B, -1, -1, -1).contiguous()
                     v = v.expand(B, -1, -1, -1).contiguous()
                     lg = lg.expand(B, -1, -1).contiguous()
+                    cache.append_and_evict(layer, k, v, lg)
                 else:
                     k, v, lg = workloads.gen_kv(wl, layer, tag, nc, dev)
-                cache.append_and_evict(layer, k, v, lg)
+                    cache.append_and_evict(layer, k, v, lg)
                 if layer == 0 and rank == 0:
                     for (b, h) in sample:
                         hist[(b, h)]["k"].append(workloads.bf16_bits(k[b, :, h]))
@@ -575,6 +583,7 @@ def run_ours(args, wl, world, rank, local, pg):
                    "timed_positions": [wl.prefill_tokens + W_, wl.prefill_tokens + W_ + K_ - 1],
                    "p_evict": (None if wl.ragged_beta else wl.p_evict),
                    "ragged_beta": wl.ragged_beta,
+                   "shared_prefix_pages": bool(args.shared_prefix and any(sh for _, sh in wl.prefill)),
                    "l2": "no flush: per-layer retained KV "
                          f"{units_per_launch * bytes_per_unit / 1e6:.0f} MB x {L} layers rotate, "
                          "larger than the 129 MB L2",

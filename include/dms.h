@@ -166,6 +166,22 @@ dms_status dms_append_and_decode(dms_cache* cache, int32_t layer, const void* k,
                                  int32_t gqa_group, float sm_scale, void* stream);
 
 /*
+ * Shared prompt: append n_tokens tokens that are IDENTICAL in every sequence (the same
+ * k, v and decision logits, given once: [1, n_tokens, kv_heads, 128] and
+ * [1, n_tokens, kv_heads]) to an EMPTY layer.  The result is the cache that
+ * dms_append_and_evict would leave with those inputs repeated for every sequence, but
+ * the pages that can no longer change -- those entirely below slot n_h - min(window + 1,
+ * n_tokens), whose tokens have already left the window and are kept for good -- are
+ * stored once and mapped into every sequence's page table, read-only; the rest are
+ * copied per sequence.  Later appends and decodes are unchanged (they never write those
+ * pages), and decode reads of the shared pages by the other sequences are served from L2
+ * when they are close in time.  Errors: DMS_ERR_STATE if the layer is not empty, else as
+ * dms_append_and_evict (pool exhaustion is the sticky device error).
+ */
+dms_status dms_append_shared_prefix(dms_cache* cache, int32_t layer, const void* k, const void* v,
+                                    const void* decision_logit, int32_t n_tokens, void* stream);
+
+/*
  * Decisions from a borrowed query neuron (App. B).  Instead of a separate logit
  * tensor, the decision logit of (sequence b, KV head h) at each token is element 0
  * of that group's FIRST query head, q[b, t, h * gqa_group, 0]; the decision rule

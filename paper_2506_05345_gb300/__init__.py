@@ -22,7 +22,8 @@ import numpy as np
 from . import _native
 from ._native import (DMS_EVICT_DELAYED, DMS_EVICT_IMMEDIATE,  # noqa: F401
                       DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
-                      DMS_ERR_INVALID_ARGUMENT, DMS_ERR_TIMEOUT, DMS_OK, DmsLibraryError,
+                      DMS_ERR_INVALID_ARGUMENT, DMS_ERR_STATE, DMS_ERR_TIMEOUT, DMS_OK,
+                      DmsLibraryError,
                       dms_options, dms_stats)
 
 HEAD_DIM = 128
@@ -78,6 +79,11 @@ def dms_append_and_decode(cache, layer, k_ptr, v_ptr, logit_ptr, q_ptr, out_ptr,
                           sm_scale, stream):
     return library().dms_append_and_decode(cache, layer, k_ptr, v_ptr, logit_ptr, q_ptr, out_ptr,
                                            gqa_group, float(sm_scale), stream)
+
+
+def dms_append_shared_prefix(cache, layer, k_ptr, v_ptr, logit_ptr, n_tokens, stream):
+    return library().dms_append_shared_prefix(cache, layer, k_ptr, v_ptr, logit_ptr, n_tokens,
+                                              stream)
 
 
 def dms_append_and_evict_borrowed(cache, layer, k_ptr, v_ptr, q_ptr, n_tokens, gqa_group, stream):
@@ -308,6 +314,18 @@ class DmsCache:
         _check(dms_append_and_decode(self._h, layer, kp, vp, lp, qp, op, gqa_group, sm_scale,
                                      _stream_ptr(stream)), "dms_append_and_decode")
         return out
+
+    def append_shared_prefix(self, layer: int, k, v, decision_logit, stream=None):
+        """A prompt identical in every sequence, given once: k, v [1, n, kv_heads, 128],
+        decision_logit [1, n, kv_heads] bf16; the layer must be empty.  Its frozen pages
+        are stored once and shared by all sequences."""
+        n = k.shape[1]
+        H, D = self.kv_heads, self.head_dim
+        kp = _bf16_cuda(k, (1, n, H, D), "k")
+        vp = _bf16_cuda(v, (1, n, H, D), "v")
+        lp = _bf16_cuda(decision_logit, (1, n, H), "decision_logit")
+        _check(dms_append_shared_prefix(self._h, layer, kp, vp, lp, n, _stream_ptr(stream)),
+               "dms_append_shared_prefix")
 
     # ---- decisions from the borrowed query neuron (App. B): element 0 of each group's
     # first query head is the decision logit and is taken as 0 by the attention.

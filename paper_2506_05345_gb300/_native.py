@@ -32,7 +32,7 @@ EXPORTS = (
     "dms_append_and_decode", "dms_selftest_bounded_wait", "dms_append_and_evict_borrowed",
     "dms_decode_attention_borrowed", "dms_append_and_decode_borrowed",
     "dms_prefill_workspace_bytes", "dms_prefill_attention", "dms_prefill_attention_borrowed",
-    "dms_prefill_device_error", "dms_prefill_attention_ex",
+    "dms_prefill_device_error", "dms_prefill_attention_ex", "dms_append_shared_prefix",
 )
 
 
@@ -90,6 +90,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_prefill_attention_borrowed": (st, [vp, vp, vp, i32, i32, i32, i32, i32, f32, vp,
                                                 ctypes.c_size_t, vp, vp]),
         "dms_prefill_device_error": (st, [vp, vp, ctypes.POINTER(st)]),
+        "dms_append_shared_prefix": (st, [vp, i32, vp, vp, vp, i32, vp]),
         "dms_prefill_attention_ex": (st, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, f32, vp,
                                           ctypes.c_size_t, vp, vp]),
         "dms_cache_stats": (st, [vp, ctypes.POINTER(dms_stats), vp, vp]),

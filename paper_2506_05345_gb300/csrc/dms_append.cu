@@ -273,6 +273,56 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
   if (tid == 0) p.counts_next[bh] = (int32_t)new_n;
 }
 
+// Shared prompt (a prefix identical in every sequence), after the bulk append has
+// filled sequence 0 of an empty layer: every other sequence b gets sequence 0's state.
+// Slots below s_min = n_h - min(window + 1, n) hold tokens that have already left the
+// window: they are kept for good and no later append writes them (reused slots belong to
+// tokens still in the window, fresh slots start at n_h).  The pages entirely below s_min
+// are therefore mapped read-only into every sequence's page table; the pages from
+// s_min / 64 on are copied per sequence.  One CTA per (sequence b >= 1, KV head).
+__global__ void __launch_bounds__(256) share_prefix_kernel(const AppendParams p) {
+  const int h = blockIdx.x % p.kv_heads, b = 1 + blockIdx.x / p.kv_heads;
+  const int src = h, dst = b * p.kv_heads + h;
+  const int tid = threadIdx.x;
+  __shared__ int32_t s_base, s_ok;
+  const int32_t nh = p.counts_next[src];
+  const int64_t R = p.window + 1;
+  const int64_t smin = nh - (p.n < R ? p.n : R);
+  const int32_t pages = (nh + kPageTokens - 1) / kPageTokens;
+  const int32_t shared = smin > 0 ? (int32_t)(smin / kPageTokens) : 0;
+  const int32_t own = pages - shared;
+  if (tid == 0) {
+    int32_t base = 0, ok = 1;
+    if (own > 0) {
+      base = atomicAdd(p.ctrl + kCtrlPoolNext, own);
+      if ((int64_t)base + own > p.pool_pages) {
+        set_device_error(p.ctrl, DMS_ERR_CAPACITY);
+        ok = 0;
+      }
+    }
+    s_base = base;
+    s_ok = ok;
+    p.counts_next[dst] = ok ? nh : 0;  // pool exhausted: the sequence stays empty
+  }
+  __syncthreads();
+  if (!s_ok) return;
+  const int32_t* pt_src = p.page_table + (int64_t)src * p.max_pages;
+  int32_t* pt_dst = p.page_table + (int64_t)dst * p.max_pages;
+  for (int i = tid; i < shared; i += blockDim.x) pt_dst[i] = pt_src[i];
+  for (int i = tid; i < own; i += blockDim.x) pt_dst[shared + i] = s_base + i;
+  for (int i = tid; i < p.ring_len; i += blockDim.x)
+    p.ring[(int64_t)dst * p.ring_len + i] = p.ring[(int64_t)src * p.ring_len + i];
+  // private copies of the pages that may still change (rows and positions)
+  for (int i = 0; i < own; ++i) {
+    const int32_t from = pt_src[shared + i], to = s_base + i;
+    const uint4* a = reinterpret_cast<const uint4*>(p.pool + (int64_t)from * kPageBytes);
+    uint4* c = reinterpret_cast<uint4*>(p.pool + (int64_t)to * kPageBytes);
+    for (int e = tid; e < kPageBytes / 16; e += blockDim.x) c[e] = a[e];
+    for (int e = tid; e < kPageTokens; e += blockDim.x)
+      p.pos[(int64_t)to * kPageTokens + e] = p.pos[(int64_t)from * kPageTokens + e];
+  }
+}
+
 __global__ void export_positions_kernel(const int32_t* counts, const int32_t* page_table,
                                         const int32_t* pos, int32_t max_pages, int64_t capacity,
                                         int32_t* out) {
@@ -338,6 +388,18 @@ cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, con
                                cudaStream_t stream) {
   const AppendParams p = make_params(c, layer, k, v, logit, logit_stride, t0, n);
   append_bulk_kernel<<<c.heads, kBulkThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+// Shared prompt of n tokens into an empty layer: the bulk append of sequence 0 (its
+// inputs are [1, n, kv_heads, 128]), then every other sequence shares its frozen pages.
+cudaError_t launch_append_shared_prefix(const Cache& c, int32_t layer, const void* k, const void* v,
+                                        const void* logit, int32_t n, cudaStream_t stream) {
+  AppendParams p = make_params(c, layer, k, v, logit, 1, 0, n);
+  append_bulk_kernel<<<c.kv_heads, kBulkThreads, 0, stream>>>(p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || c.batch == 1) return e;
+  share_prefix_kernel<<<(c.batch - 1) * c.kv_heads, 256, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

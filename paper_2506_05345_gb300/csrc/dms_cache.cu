@@ -265,6 +265,24 @@ dms_status dms_append_and_decode(dms_cache* h, int32_t layer, const void* k, con
                             stream);
 }
 
+dms_status dms_append_shared_prefix(dms_cache* h, int32_t layer, const void* k, const void* v,
+                                    const void* decision_logit, int32_t n_tokens, void* stream) {
+  if (h == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  if (layer < 0 || layer >= c.layers || n_tokens < 1 || k == nullptr || v == nullptr ||
+      decision_logit == nullptr || !aligned16(k) || !aligned16(v) ||
+      (reinterpret_cast<uintptr_t>(decision_logit) & 1u) != 0)
+    return DMS_ERR_INVALID_ARGUMENT;
+  if (c.lengths[layer] != 0) return DMS_ERR_STATE;  // a shared prompt starts the sequences
+  if (n_tokens > c.capacity) return DMS_ERR_CAPACITY;
+  const cudaError_t e = dms::launch_append_shared_prefix(c, layer, k, v, decision_logit, n_tokens,
+                                                         static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return DMS_ERR_CUDA;
+  c.lengths[layer] = n_tokens;
+  c.last_layer = layer;
+  return DMS_OK;
+}
+
 // App. B: the decision logit of (sequence b, KV head h) at token t is element 0 of query
 // head h * G, i.e. q + ((b * n + t) * kv_heads + h) * G * 128 for q of [B, n, kv_heads * G, 128].
 dms_status dms_append_and_evict_borrowed(dms_cache* h, int32_t layer, const void* k,

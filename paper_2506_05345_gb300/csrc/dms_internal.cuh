@@ -123,6 +123,8 @@ cudaError_t launch_append_one(const Cache& c, int32_t layer, const void* k, cons
 cudaError_t launch_append_bulk(const Cache& c, int32_t layer, const void* k, const void* v,
                                const void* logit, int64_t logit_stride, int64_t t0, int32_t n,
                                cudaStream_t stream);
+cudaError_t launch_append_shared_prefix(const Cache& c, int32_t layer, const void* k, const void* v,
+                                        const void* logit, int32_t n, cudaStream_t stream);
 cudaError_t launch_export_positions(const Cache& c, int32_t layer, int32_t* dev_out,
                                     cudaStream_t stream);
 cudaError_t prepare_decode(const Cache& c);
