@@ -66,6 +66,8 @@ def parse():
     ap.add_argument("--shared-prefix", action="store_true",
                     help="append the workload's shared prompt once and share its frozen pages "
                          "between the sequences")
+    ap.add_argument("--prefill-kernel", default="mma_sync", choices=["mma_sync", "tcgen05"],
+                    help="prefill attention kernel (with --prefill)")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the batch (small cases for profiling)")
     ap.add_argument("--layers", type=int, default=0,
@@ -727,18 +729,14 @@ def run_prefill(args, wl, world, rank, local, pg):
     lib = dms.library()
     vp = ctypes.c_void_p
     sptr = vp(torch.cuda.current_stream().cuda_stream)
+    kernel = dms.DMS_PREFILL_TCGEN05 if args.prefill_kernel == "tcgen05" else dms.DMS_PREFILL_MMA_SYNC
     calls = []
     for layer in range(L):
         q, k, v, lg = ins[layer]
-        if args.borrowed:
-            calls.append((lib.dms_prefill_attention_borrowed,
-                          (vp(q.data_ptr()), vp(k.data_ptr()), vp(v.data_ptr()), B, P, H, G, w, 0.0,
-                           vp(ws.data_ptr()), ws_bytes, vp(outs[layer].data_ptr()), sptr)))
-        else:
-            calls.append((lib.dms_prefill_attention,
-                          (vp(q.data_ptr()), vp(k.data_ptr()), vp(v.data_ptr()), vp(lg.data_ptr()),
-                           B, P, H, G, w, 0.0, vp(ws.data_ptr()), ws_bytes,
-                           vp(outs[layer].data_ptr()), sptr)))
+        calls.append((lib.dms_prefill_attention_ex,
+                      (vp(q.data_ptr()), vp(k.data_ptr()), vp(v.data_ptr()),
+                       None if args.borrowed else vp(lg.data_ptr()), B, P, H, G, w, 0, kernel,
+                       0.0, vp(ws.data_ptr()), ws_bytes, vp(outs[layer].data_ptr()), sptr)))
     codes = []
 
     def step():
@@ -817,7 +815,9 @@ def run_prefill(args, wl, world, rank, local, pg):
         "prompt_tokens_per_s_per_layer": B * P / t_layer,
         "visible_pairs_per_layer": pairs[0], "dense_causal_pairs_per_layer": dense_pairs,
         "sparsity": 1.0 - pairs[0] / dense_pairs,
-        "roofline": {"kernel": "prefill_attn_kernel + pack pre-pass", "bound": "tensor",
+        "roofline": {"kernel": ("prefill_tc_kernel (tcgen05)" if kernel == dms.DMS_PREFILL_TCGEN05
+                               else "prefill_attn_kernel (mma.sync)") + " + pack pre-pass",
+                     "bound": "tensor",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": f"{peak_kind} dense bf16 (burst)",
                      "traffic": None,

@@ -247,14 +247,21 @@ dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const vo
                                           int32_t gqa_group, int32_t window, float sm_scale,
                                           void* workspace, size_t workspace_bytes, void* out,
                                           void* stream);
+/* Prefill attention kernels (dms_prefill_attention_ex `kernel`). */
+enum {
+  DMS_PREFILL_TCGEN05 = 0,  /* 5th-generation tensor cores, accumulators in TMEM          */
+  DMS_PREFILL_MMA_SYNC = 1  /* warp-level mma.sync tiles (used by the plain entry points)  */
+};
 /* The general form: decision_logit == NULL takes the decisions from the queries as in
  * the borrowed form; eviction_policy DMS_EVICT_DELAYED or DMS_EVICT_IMMEDIATE (the Sec. 5
- * ablation: key i is visible outside the window iff the decision of token i + window is 0). */
+ * ablation: key i is visible outside the window iff the decision of token i + window is 0);
+ * kernel DMS_PREFILL_TCGEN05 or DMS_PREFILL_MMA_SYNC. */
 dms_status dms_prefill_attention_ex(const void* q, const void* k, const void* v,
                                     const void* decision_logit, int32_t batch, int32_t n_tokens,
                                     int32_t kv_heads, int32_t gqa_group, int32_t window,
-                                    int32_t eviction_policy, float sm_scale, void* workspace,
-                                    size_t workspace_bytes, void* out, void* stream);
+                                    int32_t eviction_policy, int32_t kernel, float sm_scale,
+                                    void* workspace, size_t workspace_bytes, void* out,
+                                    void* stream);
 /* Synchronise `stream` and report the sticky device error of the last prefill that used
  * `workspace` into *out (DMS_OK when none). */
 dms_status dms_prefill_device_error(const void* workspace, void* stream, dms_status* out);

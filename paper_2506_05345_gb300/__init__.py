@@ -21,6 +21,7 @@ import numpy as np
 
 from . import _native
 from ._native import (DMS_EVICT_DELAYED, DMS_EVICT_IMMEDIATE,  # noqa: F401
+                      DMS_PREFILL_MMA_SYNC, DMS_PREFILL_TCGEN05,  # noqa: F401
                       DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
                       DMS_ERR_INVALID_ARGUMENT, DMS_ERR_STATE, DMS_ERR_TIMEOUT, DMS_OK,
                       DmsLibraryError,
@@ -129,16 +130,16 @@ def dms_prefill_device_error(ws_ptr, stream):
 
 
 def dms_prefill_attention_ex(q_ptr, k_ptr, v_ptr, logit_ptr, batch, n_tokens, kv_heads,
-                             gqa_group, window, eviction_policy, sm_scale, ws_ptr, ws_bytes,
-                             out_ptr, stream):
+                             gqa_group, window, eviction_policy, kernel, sm_scale, ws_ptr,
+                             ws_bytes, out_ptr, stream):
     return library().dms_prefill_attention_ex(q_ptr, k_ptr, v_ptr, logit_ptr, batch, n_tokens,
-                                              kv_heads, gqa_group, window, eviction_policy,
+                                              kv_heads, gqa_group, window, eviction_policy, kernel,
                                               float(sm_scale), ws_ptr, ws_bytes, out_ptr, stream)
 
 
 def prefill_attention(q, k, v, decision_logit=None, window: int = 256, gqa_group=None,
                       sm_scale: float = 0.0, workspace=None, out=None, stream=None,
-                      eviction_policy: int = 0):
+                      eviction_policy: int = 0, kernel: int = -1):
     """Sparse DMS prefill attention of a whole prompt (no cache involved).
 
     q: [B, P, Hkv * G, 128], k, v: [B, P, Hkv, 128], decision_logit: [B, P, Hkv] bf16 CUDA
@@ -164,11 +165,13 @@ def prefill_attention(q, k, v, decision_logit=None, window: int = 256, gqa_group
         raise TypeError("workspace must be a uint8 CUDA tensor")
     wp = ctypes.c_void_p(workspace.data_ptr())
     wb = workspace.numel()
-    if eviction_policy != 0:
+    if eviction_policy != 0 or kernel >= 0:
         lp = None if decision_logit is None else _bf16_cuda(decision_logit, (B, P, Hkv),
                                                             "decision_logit")
         code = dms_prefill_attention_ex(qp, kp, vp, lp, B, P, Hkv, gqa_group, window,
-                                        eviction_policy, sm_scale, wp, wb, op, _stream_ptr(stream))
+                                        eviction_policy,
+                                        DMS_PREFILL_MMA_SYNC if kernel < 0 else kernel,
+                                        sm_scale, wp, wb, op, _stream_ptr(stream))
         _check(code, "dms_prefill_attention_ex")
     elif decision_logit is None:
         code = dms_prefill_attention_borrowed(qp, kp, vp, B, P, Hkv, gqa_group, window, sm_scale,

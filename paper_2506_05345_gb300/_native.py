@@ -21,6 +21,8 @@ DMS_ERR_TIMEOUT = 5
 DMS_ERR_STATE = 6
 DMS_EVICT_DELAYED = 0
 DMS_EVICT_IMMEDIATE = 1
+DMS_PREFILL_TCGEN05 = 0
+DMS_PREFILL_MMA_SYNC = 1
 DMS_DECODE_TILED = 0
 DMS_DECODE_SIMPLE = 1
 
@@ -91,8 +93,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                                 ctypes.c_size_t, vp, vp]),
         "dms_prefill_device_error": (st, [vp, vp, ctypes.POINTER(st)]),
         "dms_append_shared_prefix": (st, [vp, i32, vp, vp, vp, i32, vp]),
-        "dms_prefill_attention_ex": (st, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, f32, vp,
-                                          ctypes.c_size_t, vp, vp]),
+        "dms_prefill_attention_ex": (st, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32,
+                                          vp, ctypes.c_size_t, vp, vp]),
         "dms_cache_stats": (st, [vp, ctypes.POINTER(dms_stats), vp, vp]),
         "dms_cache_export_positions": (st, [vp, i32, vp, vp]),
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),

@@ -148,6 +148,7 @@ size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens);
 cudaError_t launch_prefill(const void* q, const void* k, const void* v, const void* logit,
                            int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
                            int32_t group, int32_t window, bool immediate, float scale_log2,
-                           bool zero_first, void* workspace, void* out, cudaStream_t stream);
+                           bool zero_first, int32_t kernel, void* workspace, void* out,
+                           cudaStream_t stream);
 
 }  // namespace dms

@@ -81,9 +81,9 @@ struct PackParams {
   const uint16_t* logit;     // decision logit of (b, i, h) at logit[((b P + i) Hkv + h) stride]
   int64_t logit_stride;
   int64_t decider;           // token i is evicted by the decision of token i + decider
-  uint8_t* kd;               // [H][P] permuted rows
+  uint8_t* kd;               // [H][2 d-halves][P][128 B] permuted half-rows
   uint8_t* vd;
-  uint8_t* kc;               // [H][P] permuted rows of the alpha = 0 tokens, position order
+  uint8_t* kc;               // [H][2][P][128 B]: the alpha = 0 tokens, position order
   uint8_t* vc;
   int32_t* pc;               // [H][pc_stride(P)] positions of the compacted rows
   int32_t* before;           // [H][P + 1] alpha = 0 tokens at positions below i
@@ -91,10 +91,16 @@ struct PackParams {
   int32_t P, kv_heads, nch;
 };
 
-// Byte offset of logical 16-byte chunk `chunk` inside row `row` of a permuted array (the
-// row's own offset, row * 256, is added by the caller in 64-bit arithmetic).
+// Byte offset of logical 16-byte chunk `chunk` (0..7) inside the 128-byte half-row `row`
+// (the row's own offset is added by the caller in 64-bit arithmetic).
 __device__ __forceinline__ uint32_t chunk_in_row(int64_t row, int chunk) {
   return (uint32_t)((chunk ^ (int)(row & 7)) << 4);
+}
+
+// Byte offset of logical chunk c (0..15, head_dim 8c .. 8c + 7) of row r inside a staged
+// 64-row tile stored as two 8 KiB d-halves [half][row][128 B].
+__device__ __forceinline__ uint32_t tile_off(uint32_t r, uint32_t c) {
+  return (c >> 3) * (kPfKeys * 128u) + r * 128u + (((c & 7u) ^ (r & 7u)) << 4);
 }
 
 // Token i stays visible outside the window iff the decision that evicts it is 0: its
@@ -183,22 +189,36 @@ __global__ void __launch_bounds__(kPfPackThreads) prefill_pack_kernel(const Pack
     run += f[e];
   }
   __syncthreads();
-  // rows: lanes 0-15 move K's sixteen 16-byte chunks, lanes 16-31 V's
-  const int half = lane >> 4, chunk = lane & 15;
-  const uint16_t* src_base = half ? p.v : p.k;
-  uint8_t* dense = half ? p.vd : p.kd;
-  uint8_t* comp = half ? p.vc : p.kc;
-  const int64_t hrow = (int64_t)head * p.P;
+  // rows: lanes 0-15 move K's sixteen 16-byte chunks, lanes 16-31 V's; chunk c goes to
+  // d-half c / 8 of the row
+  const int kv = lane >> 4, chunk = lane & 15, dh = chunk >> 3, c8 = chunk & 7;
+  const uint16_t* src_base = kv ? p.v : p.k;
+  uint8_t* dense = kv ? p.vd : p.kd;
+  uint8_t* comp = kv ? p.vc : p.kc;
+  const int64_t hrow = ((int64_t)head * 2 + dh) * p.P;  // this d-half of this head
   for (int i = warp; i < n; i += kPfPackThreads / 32) {
     const int pos = i0 + i;
     const uint4 val = *reinterpret_cast<const uint4*>(
         src_base + (((int64_t)b * p.P + pos) * p.kv_heads + hk) * kHeadDim + chunk * 8);
-    *reinterpret_cast<uint4*>(dense + (hrow + pos) * kRowBytes + chunk_in_row(pos, chunk)) = val;
+    *reinterpret_cast<uint4*>(dense + (hrow + pos) * 128 + chunk_in_row(pos, c8)) = val;
     const int c = s_idx[i];
     if (c >= 0) {
-      *reinterpret_cast<uint4*>(comp + (hrow + c) * kRowBytes + chunk_in_row(c, chunk)) = val;
+      *reinterpret_cast<uint4*>(comp + (hrow + c) * 128 + chunk_in_row(c, c8)) = val;
       if (lane == 0) p.pc[(int64_t)head * pc_stride(p.P) + c] = pos;
     }
+  }
+}
+
+// Rows [r0, r0 + rows) of one head's K and V (two d-halves each) into a stage laid out as
+// K [2][64][128 B] then V [2][64][128 B].
+__device__ __forceinline__ void stage_tile(uint8_t* st, const uint8_t* k, const uint8_t* v,
+                                           int64_t head, int P, int r0, int rows, uint64_t* bar) {
+  const uint32_t bytes = (uint32_t)rows * 128u;
+#pragma unroll
+  for (int dh = 0; dh < 2; ++dh) {
+    const int64_t row = (head * 2 + dh) * P + r0;
+    bulk_copy_g2s(st + dh * (kPfKeys * 128), k + row * 128, bytes, bar);
+    bulk_copy_g2s(st + kPfTileBytes + dh * (kPfKeys * 128), v + row * 128, bytes, bar);
   }
 }
 
@@ -258,20 +278,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
         uint8_t* st = smem + s * kPfStageBytes;
         if (t < n_ct) {
           const int r0 = t * kPfKeys, rows = min(kPfKeys, nc - r0);
-          const uint32_t bytes = (uint32_t)rows * kRowBytes;
-          mbar_arrive_expect_tx(&full_bar[s], 2 * bytes + kPfKeys * 4);
-          const int64_t row = head * P + r0;
-          bulk_copy_g2s(st, p.kc + row * kRowBytes, bytes, &full_bar[s]);
-          bulk_copy_g2s(st + kPfTileBytes, p.vc + row * kRowBytes, bytes, &full_bar[s]);
+          mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes + kPfKeys * 4);
+          stage_tile(st, p.kc, p.vc, head, P, r0, rows, &full_bar[s]);
           bulk_copy_g2s(st + 2 * kPfTileBytes, p.pc + head * pc_stride(P) + r0, kPfKeys * 4,
                         &full_bar[s]);
         } else {
           const int r0 = bs + (t - n_ct) * kPfKeys, rows = min(kPfKeys, jmax + 1 - r0);
-          const uint32_t bytes = (uint32_t)rows * kRowBytes;
-          mbar_arrive_expect_tx(&full_bar[s], 2 * bytes);
-          const int64_t row = head * P + r0;
-          bulk_copy_g2s(st, p.kd + row * kRowBytes, bytes, &full_bar[s]);
-          bulk_copy_g2s(st + kPfTileBytes, p.vd + row * kRowBytes, bytes, &full_bar[s]);
+          mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes);
+          stage_tile(st, p.kd, p.vd, head, P, r0, rows, &full_bar[s]);
         }
       }
       // Drain: do not leave while a bulk copy may still be writing shared memory.
@@ -333,7 +347,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
         for (int np = 0; np < 4; ++np) {
           const uint32_t row = (uint32_t)(16 * np + (mi >> 1) * 8 + (lane & 7));
           uint32_t b0, b1, b2, b3;
-          ldsm_x4(kbase + swizzled_offset(row, (uint32_t)(2 * kk + (mi & 1))), b0, b1, b2, b3);
+          ldsm_x4(kbase + tile_off(row, (uint32_t)(2 * kk + (mi & 1))), b0, b1, b2, b3);
           mma_bf16_16816(sc[2 * np], qa, b0, b1);
           mma_bf16_16816(sc[2 * np + 1], qa, b2, b3);
         }
@@ -402,8 +416,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 #pragma unroll
         for (int dp = 0; dp < 8; ++dp) {
           uint32_t b0, b1, b2, b3;
-          ldsm_x4_trans(vbase + swizzled_offset(row, (uint32_t)(2 * dp + (mi >> 1))), b0, b1, b2,
-                        b3);
+          ldsm_x4_trans(vbase + tile_off(row, (uint32_t)(2 * dp + (mi >> 1))), b0, b1, b2, b3);
           b0 &= mk0;
           b1 &= mk1;
           b2 &= mk0;
@@ -436,6 +449,264 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
   }
 }
 
+// ============================================================================ tcgen05 kernel
+// The same tiles on the 5th-generation tensor cores.  One CTA per (query head, 128-query
+// tile), 256 threads: warp 0 stages K / V tiles (bulk copies, 3 stages), warp 1 issues the
+// MMAs from one thread, warp 2 owns the tensor-memory allocation, warps 4-7 (one thread per
+// query row, TMEM lane = row) run the softmax and keep the output accumulator in registers.
+// Per 64-key tile: S = Q K^T (M 128, N 64, 8 MMAs of K 16) into TMEM; each softmax thread
+// loads its row of S, masks it, updates its running max / sum and writes its row of
+// P = exp2(S - m) as bf16 into shared memory; O_tile = P V (M 128, N 128, 4 MMAs) into TMEM;
+// the thread adds O_tile to its register accumulator after scaling that by the max
+// correction.  Operands sit in shared memory in the 128-byte-swizzled layout: rows of two
+// 128-byte d-halves, 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q, K and P
+// are K-major, V is MN-major (head_dim contiguous).
+constexpr int kTcThreads = 256;
+// Kernel of the plain entry points (the faster of the two as measured).
+constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_MMA_SYNC;
+constexpr int kTcStageBytes = 33 * 1024;  // K 16 KiB, V 16 KiB, key positions (1 KiB aligned)
+constexpr int kTcQBytes = kPfRows * kRowBytes;         // Q [2 d-halves][128 rows][128 B]
+constexpr int kTcPBytes = kPfRows * kPfKeys * 2;       // P [128 rows][64 keys] bf16
+constexpr int kTcOffQ = kPfStages * kTcStageBytes;
+constexpr int kTcOffP = kTcOffQ + kTcQBytes;
+constexpr int kTcOffBar = kTcOffP + kTcPBytes;
+constexpr int kTcSmemBytes = kTcOffBar + 256 + 1024;   // + barriers, + base alignment slack
+constexpr uint32_t kTcCols = 256;                      // TMEM: S at column 0, O_tile at 64
+constexpr uint32_t kTcColO = 64;
+
+__global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const PrefillParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sq = smem + kTcOffQ;
+  uint8_t* sp = smem + kTcOffP;
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kTcOffBar);
+  uint64_t* empty_bar = full_bar + kPfStages;
+  uint64_t* q_ready = empty_bar + kPfStages;  // 128 arrivals: Q staged
+  uint64_t* s_full = q_ready + 1;             // MMA commit: S in TMEM
+  uint64_t* p_full = s_full + 1;              // 128 arrivals: P in shared memory
+  uint64_t* o_full = p_full + 1;              // MMA commit: O_tile in TMEM
+  uint64_t* o_free = o_full + 1;              // 128 arrivals: S and O_tile read
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(o_free + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int Hq = p.kv_heads * p.group;
+  const int tile_rank = blockIdx.x / p.n_qheads;
+  const int qt = p.n_qtiles - 1 - tile_rank;
+  const int qh = blockIdx.x - tile_rank * p.n_qheads;
+  const int b = qh / Hq, hq = qh - b * Hq, hk = hq / p.group;
+  const int64_t head = (int64_t)b * p.kv_heads + hk;
+  const int P = p.P, w = p.window;
+  const int j0 = qt * kPfRows;
+  const int jmax = min(j0 + kPfRows, P) - 1;
+  const int nc = (jmax - w > 0) ? p.before[head * (P + 1) + (jmax - w)] : 0;
+  const int bs = max(0, j0 - w) & ~7;
+  const int n_ct = (nc + kPfKeys - 1) / kPfKeys;
+  const int n_tiles = n_ct + (jmax + 1 - bs + kPfKeys - 1) / kPfKeys;
+
+  if (tid == 0) {
+    *abort_flag = 0;
+    for (int s = 0; s < kPfStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    mbar_init(q_ready, kPfRows);
+    mbar_init(s_full, 1);
+    mbar_init(p_full, kPfRows);
+    mbar_init(o_full, 1);
+    mbar_init(o_free, kPfRows);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 2) {
+    tmem_alloc(s_tmem, kTcCols);
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *s_tmem;
+
+  if (warp == 0) {
+    // ================================================================ producer
+    if (lane == 0) {
+      for (int t = 0; t < n_tiles; ++t) {
+        const int s = t % kPfStages, use = t / kPfStages;
+        if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.err);
+        uint8_t* st = smem + s * kTcStageBytes;
+        if (t < n_ct) {
+          const int r0 = t * kPfKeys, rows = min(kPfKeys, nc - r0);
+          mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes + kPfKeys * 4);
+          stage_tile(st, p.kc, p.vc, head, P, r0, rows, &full_bar[s]);
+          bulk_copy_g2s(st + 2 * kPfTileBytes, p.pc + head * pc_stride(P) + r0, kPfKeys * 4,
+                        &full_bar[s]);
+        } else {
+          const int r0 = bs + (t - n_ct) * kPfKeys, rows = min(kPfKeys, jmax + 1 - r0);
+          mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes);
+          stage_tile(st, p.kd, p.vd, head, P, r0, rows, &full_bar[s]);
+        }
+      }
+      for (int s = 0; s < kPfStages && s < n_tiles; ++s) {
+        const int last_t = s + ((n_tiles - 1 - s) / kPfStages) * kPfStages;
+        mbar_wait(&full_bar[s], (last_t / kPfStages) & 1, abort_flag, p.err);
+      }
+    }
+  } else if (warp == 1) {
+    // ================================================================ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = f16_idesc(kPfRows, kPfKeys, 0);    // Q K^T: both K-major
+      constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
+      const uint32_t q_base = smem_addr(sq), p_base = smem_addr(sp);
+      mbar_wait(q_ready, 0, abort_flag, p.err);
+      for (int t = 0; t < n_tiles; ++t) {
+        const int s = t % kPfStages;
+        const uint32_t k_base = smem_addr(smem + s * kTcStageBytes);
+        const uint32_t v_base = k_base + kPfTileBytes;
+        mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);
+        if (t > 0) mbar_wait(o_free, (t - 1) & 1, abort_flag, p.err);
+        tc_fence_after();
+        // S = Q K^T: k-step kk covers head_dim 16 kk .. 16 kk + 15 (d-half kk / 4)
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (uint32_t)(kk & 3) * 32u;  // 16 head_dim elements = 32 B
+          const uint64_t a = sw128_desc(q_base + (uint32_t)(kk >> 2) * (kPfRows * 128u) + off, 16u, 1024u);
+          const uint64_t bk = sw128_desc(k_base + (uint32_t)(kk >> 2) * (kPfKeys * 128u) + off, 16u, 1024u);
+          tc_mma_ss(tmem, a, bk, idesc_s, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(s_full);
+        mbar_wait(p_full, t & 1, abort_flag, p.err);
+        tc_fence_after();
+        // O_tile = P V: k-step kk covers keys 16 kk .. 16 kk + 15; V atoms along head_dim
+        // are the two d-halves (leading offset 8 KiB), 8-key groups 1 KiB apart
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t a = sw128_desc(p_base + (uint32_t)kk * 32u, 16u, 1024u);
+          const uint64_t bv = sw128_desc(v_base + (uint32_t)kk * 2048u, kPfKeys * 128u, 1024u);
+          tc_mma_ss(tmem + kTcColO, a, bv, idesc_o, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(o_full);
+        tc_commit(&empty_bar[s]);  // the stage is free once both products are done
+      }
+    }
+  } else if (warp >= 4) {
+    // ================================================================ softmax warpgroup
+    const int row = tid - 128;           // query row of the tile = TMEM lane
+    const int j = j0 + row;              // its query position
+    const uint32_t lane_addr = tmem + ((uint32_t)(32 * (warp - 4)) << 16);
+    // this row of Q into the K-major swizzled layout [d-half][row][128 B]
+    {
+      const bool zero = p.zero_first && hq % p.group == 0;
+      const __nv_bfloat16* qrow = p.q + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        uint4 val = make_uint4(0u, 0u, 0u, 0u);
+        if (j < P) val = *reinterpret_cast<const uint4*>(qrow + c * 8);
+        if (zero && c == 0) val.x &= 0xffff0000u;  // App. B: the decision element
+        *reinterpret_cast<uint4*>(sq + (c >> 3) * (kPfRows * 128) + row * 128 +
+                                  chunk_in_row(row, c & 7)) = val;
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(q_ready);
+    }
+    float o[kHeadDim];
+#pragma unroll
+    for (int d = 0; d < kHeadDim; ++d) o[d] = 0.f;
+    float m = -INFINITY, l = 0.f;
+    for (int t = 0; t < n_tiles; ++t) {
+      const int s = t % kPfStages;
+      const bool retained = t < n_ct;
+      const int r0 = retained ? t * kPfKeys : bs + (t - n_ct) * kPfKeys;
+      const int rows = retained ? min(kPfKeys, nc - r0) : min(kPfKeys, jmax + 1 - r0);
+      const uint8_t* st = smem + s * kTcStageBytes;
+      mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);  // key positions
+      if (rows < kPfKeys) {
+        // V rows past the tile's keys hold stale bytes, possibly NaN patterns; P is 0
+        // there, but 0 * NaN is not: zero them before P V reads the tile (the proxy
+        // fence before the P-ready arrival orders these writes for the tensor cores).
+        uint8_t* vt = smem + s * kTcStageBytes + kPfTileBytes;
+        for (int i = row; i < (kPfKeys - rows) * 16; i += kPfRows)
+          *reinterpret_cast<uint4*>(vt + tile_off((uint32_t)(rows + i / 16), (uint32_t)(i & 15))) =
+              make_uint4(0u, 0u, 0u, 0u);
+      }
+      mbar_wait(s_full, t & 1, abort_flag, p.err);
+      tc_fence_after();
+      float sc[kPfKeys];
+#pragma unroll
+      for (int c = 0; c < kPfKeys / 16; ++c) {
+        float r[16];
+        tmem_ld16(lane_addr + (uint32_t)(16 * c), r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sc[16 * c + i] = r[i];
+      }
+      const int32_t* spos = reinterpret_cast<const int32_t*>(st + 2 * kPfTileBytes);
+      float mx = -INFINITY;
+#pragma unroll
+      for (int kidx = 0; kidx < kPfKeys; ++kidx) {
+        const bool valid = kidx < rows;
+        const int pos = retained ? (valid ? spos[kidx] : 0) : r0 + kidx;
+        const bool vis = valid && (retained ? pos < j - w : (pos >= j - w && pos <= j));
+        sc[kidx] = vis ? sc[kidx] * p.scale_log2 : -INFINITY;
+        mx = fmaxf(mx, sc[kidx]);
+      }
+      const float mn = fmaxf(m, mx);
+      const float base = mn == -INFINITY ? 0.f : mn;
+      const float corr = exp2f(m - base);
+      m = mn;
+      float sum = 0.f;
+      // P row: 64 bf16 = 8 chunks of 16 bytes, chunk c at (c ^ (row & 7))
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float p0 = exp2f(sc[8 * c + 2 * e] - base), p1 = exp2f(sc[8 * c + 2 * e + 1] - base);
+          sum += p0 + p1;
+          pk[e] = pack_bf16x2(p0, p1);
+        }
+        *reinterpret_cast<uint4*>(sp + row * 128 + chunk_in_row(row, c)) =
+            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+      l = l * corr + sum;
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(p_full);
+      mbar_wait(o_full, t & 1, abort_flag, p.err);
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < kHeadDim / 16; ++c) {
+        float r[16];
+        tmem_ld16(lane_addr + kTcColO + (uint32_t)(16 * c), r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[16 * c + i] = o[16 * c + i] * corr + r[i];
+      }
+      tc_fence_before();
+      mbar_arrive(o_free);
+    }
+    // normalise and store this row
+    if (j < P) {
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      __nv_bfloat16* orow = p.out + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        uint4 val;
+        val.x = pack_bf16x2(o[8 * c + 0] * inv, o[8 * c + 1] * inv);
+        val.y = pack_bf16x2(o[8 * c + 2] * inv, o[8 * c + 3] * inv);
+        val.z = pack_bf16x2(o[8 * c + 4] * inv, o[8 * c + 5] * inv);
+        val.w = pack_bf16x2(o[8 * c + 6] * inv, o[8 * c + 7] * inv);
+        *reinterpret_cast<uint4*>(orow + 8 * c) = val;
+      }
+    }
+  }
+  // ---- teardown: every tensor-memory access is done before the columns are released
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTcCols);
+  }
+}
+
 }  // namespace
 
 size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens) {
@@ -445,8 +716,9 @@ size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens) {
 cudaError_t launch_prefill(const void* q, const void* k, const void* v, const void* logit,
                            int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
                            int32_t group, int32_t window, bool immediate, float scale_log2,
-                           bool zero_first, void* workspace, void* out, cudaStream_t stream) {
-  // The kernel's shared-memory limit, raised once per device.
+                           bool zero_first, int32_t kernel, void* workspace, void* out,
+                           cudaStream_t stream) {
+  // The kernels' shared-memory limits, raised once per device.
   static std::atomic<uint64_t> attr_set{0};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -455,6 +727,9 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
   if (bit == 0 || (attr_set.load() & bit) == 0) {
     e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              kPfSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kTcSmemBytes);
     if (e != cudaSuccess) return e;
     attr_set.fetch_or(bit);
   }
@@ -503,7 +778,10 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
   pp.n_qheads = (int32_t)(H * group);
   pp.scale_log2 = scale_log2;
   const int64_t grid = (int64_t)pp.n_qtiles * pp.n_qheads;
-  prefill_attn_kernel<<<(unsigned)grid, kPfThreads, kPfSmemBytes, stream>>>(pp);
+  if (kernel == DMS_PREFILL_MMA_SYNC)
+    prefill_attn_kernel<<<(unsigned)grid, kPfThreads, kPfSmemBytes, stream>>>(pp);
+  else
+    prefill_tc_kernel<<<(unsigned)grid, kTcThreads, kTcSmemBytes, stream>>>(pp);
   return cudaGetLastError();
 }
 
@@ -516,15 +794,16 @@ bool pf_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u)
 
 dms_status prefill_impl(const void* q, const void* k, const void* v, const void* logit,
                         int64_t logit_stride, int32_t batch, int32_t n_tokens, int32_t kv_heads,
-                        int32_t gqa_group, int32_t window, int32_t policy, float sm_scale,
-                        void* workspace, size_t workspace_bytes, void* out, bool zero_first,
-                        void* stream) {
+                        int32_t gqa_group, int32_t window, int32_t policy, int32_t kernel,
+                        float sm_scale, void* workspace, size_t workspace_bytes, void* out,
+                        bool zero_first, void* stream) {
   if (q == nullptr || k == nullptr || v == nullptr || logit == nullptr || out == nullptr ||
       workspace == nullptr || !pf_aligned16(q) || !pf_aligned16(k) || !pf_aligned16(v) ||
       !pf_aligned16(out) || !pf_aligned16(workspace) ||
       (reinterpret_cast<uintptr_t>(logit) & 1u) != 0 || batch < 1 || n_tokens < 1 ||
       kv_heads < 1 || gqa_group < 1 || gqa_group > dms::kMaxGroup || window < 0 ||
-      !(sm_scale == sm_scale) || policy < DMS_EVICT_DELAYED || policy > DMS_EVICT_IMMEDIATE)
+      !(sm_scale == sm_scale) || policy < DMS_EVICT_DELAYED || policy > DMS_EVICT_IMMEDIATE ||
+      kernel < DMS_PREFILL_TCGEN05 || kernel > DMS_PREFILL_MMA_SYNC)
     return DMS_ERR_INVALID_ARGUMENT;
   const int64_t H = (int64_t)batch * kv_heads;
   const int64_t qtiles = ((int64_t)n_tokens + 127) / 128;
@@ -534,8 +813,8 @@ dms_status prefill_impl(const void* q, const void* k, const void* v, const void*
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
   const cudaError_t e = dms::launch_prefill(
       q, k, v, logit, logit_stride, batch, n_tokens, kv_heads, gqa_group, window,
-      policy == DMS_EVICT_IMMEDIATE, scale * 1.4426950408889634f, zero_first, workspace, out,
-      static_cast<cudaStream_t>(stream));
+      policy == DMS_EVICT_IMMEDIATE, scale * 1.4426950408889634f, zero_first, kernel, workspace,
+      out, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
 }
 
@@ -557,7 +836,8 @@ dms_status dms_prefill_attention(const void* q, const void* k, const void* v,
                                  float sm_scale, void* workspace, size_t workspace_bytes,
                                  void* out, void* stream) {
   return prefill_impl(q, k, v, decision_logit, 1, batch, n_tokens, kv_heads, gqa_group, window,
-                      DMS_EVICT_DELAYED, sm_scale, workspace, workspace_bytes, out, false, stream);
+                      DMS_EVICT_DELAYED, kPrefillDefaultKernel, sm_scale, workspace,
+                      workspace_bytes, out, false, stream);
 }
 
 dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const void* v,
@@ -567,20 +847,21 @@ dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const vo
                                           void* stream) {
   if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
   return prefill_impl(q, k, v, q, (int64_t)gqa_group * dms::kHeadDim, batch, n_tokens, kv_heads,
-                      gqa_group, window, DMS_EVICT_DELAYED, sm_scale, workspace, workspace_bytes,
-                      out, true, stream);
+                      gqa_group, window, DMS_EVICT_DELAYED, kPrefillDefaultKernel, sm_scale,
+                      workspace, workspace_bytes, out, true, stream);
 }
 
 dms_status dms_prefill_attention_ex(const void* q, const void* k, const void* v,
                                     const void* decision_logit, int32_t batch, int32_t n_tokens,
                                     int32_t kv_heads, int32_t gqa_group, int32_t window,
-                                    int32_t eviction_policy, float sm_scale, void* workspace,
-                                    size_t workspace_bytes, void* out, void* stream) {
+                                    int32_t eviction_policy, int32_t kernel, float sm_scale,
+                                    void* workspace, size_t workspace_bytes, void* out,
+                                    void* stream) {
   if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
   const bool borrowed = decision_logit == nullptr;
   return prefill_impl(q, k, v, borrowed ? q : decision_logit,
                       borrowed ? (int64_t)gqa_group * dms::kHeadDim : 1, batch, n_tokens,
-                      kv_heads, gqa_group, window, eviction_policy, sm_scale, workspace,
+                      kv_heads, gqa_group, window, eviction_policy, kernel, sm_scale, workspace,
                       workspace_bytes, out, borrowed, stream);
 }
 

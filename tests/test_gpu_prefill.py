@@ -65,6 +65,10 @@ def _check_rows(q, k, v, lg, out, w, G, rows=None, q_att=None):
     return e
 
 
+KERNELS = [dms.DMS_PREFILL_TCGEN05, dms.DMS_PREFILL_MMA_SYNC]
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("B,P,H,G,w,p", [
     (2, 300, 2, 4, 32, 0.75),     # partial last tile, retained + window keys
     (1, 1000, 1, 4, 64, 0.9),     # many retained tiles
@@ -75,16 +79,17 @@ def _check_rows(q, k, v, lg, out, w, G, rows=None, q_att=None):
     (1, 1, 1, 1, 0, 1.0),         # one token
     (1, 129, 2, 7, 3, 0.7),       # G = 7, tile boundary + 1
 ])
-def test_prefill_matches_oracle(B, P, H, G, w, p):
+def test_prefill_matches_oracle(B, P, H, G, w, p, kernel):
     q, k, v, lg = _inputs(B, P, H, G, p, seed=P + G)
     ws_bytes = dms.dms_prefill_workspace_bytes(B, P, H)[1]
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
-    out = dms.prefill_attention(q, k, v, lg, window=w, workspace=ws)
+    out = torch.full_like(q, float("nan"))  # every row must be written
+    dms.prefill_attention(q, k, v, lg, window=w, workspace=ws, out=out, kernel=kernel)
     torch.cuda.synchronize()
     assert _ws_error(ws) == dms.DMS_OK
     _check_rows(q, k, v, lg, out, w, G)
     # bitwise deterministic
-    out2 = dms.prefill_attention(q, k, v, lg, window=w, workspace=ws)
+    out2 = dms.prefill_attention(q, k, v, lg, window=w, workspace=ws, kernel=kernel)
     assert torch.equal(out, out2)
 
 
@@ -100,17 +105,18 @@ def test_prefill_special_logits():
     _check_rows(q, k, v, lg, out, w, G)
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("G", [1, 4, 16])
-def test_prefill_borrowed_equals_explicit(G):
+def test_prefill_borrowed_equals_explicit(G, kernel):
     B, P, H, w = 2, 350, 2, 40
     q, k, v, lg = _inputs(B, P, H, G, 0.8, seed=G, borrowed=True)
     q_keep = q.clone()
-    out_b = dms.prefill_attention(q, k, v, None, window=w)
+    out_b = dms.prefill_attention(q, k, v, None, window=w, kernel=kernel)
     assert torch.equal(q, q_keep), "the caller's q must not be modified"
     lg_x = q[:, :, ::G, 0].contiguous()
     qz = q.clone()
     qz[:, :, ::G, 0] = 0
-    out_x = dms.prefill_attention(qz, k, v, lg_x, window=w)
+    out_x = dms.prefill_attention(qz, k, v, lg_x, window=w, kernel=kernel)
     assert torch.equal(out_b, out_x)
     rows = [(b, j, h) for b in range(B) for j in range(0, P, 5) for h in range(H)]
     _check_rows(q, k, v, lg_x, out_b, w, G, rows=rows, q_att=qz)
@@ -131,14 +137,15 @@ def test_prefill_last_row_matches_decode_step():
     assert diff.max().item() <= 2 * MAX_ABS
 
 
-def test_prefill_full_prompt_sampled():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_prefill_full_prompt_sampled(kernel):
     """Qwen-R1-7B attention shape (28 / 4 heads), 7936-token prompt, P(evict) 0.75: >= 256
     sampled (sequence, query, KV head) rows, always including the first and last query."""
     B, P, H, G, w = 4, 7936, 4, 7, 256
     q, k, v, lg = _inputs(B, P, H, G, 0.75, seed=77)
     ws = torch.empty(dms.dms_prefill_workspace_bytes(B, P, H)[1], dtype=torch.uint8,
                      device="cuda")
-    out = dms.prefill_attention(q, k, v, lg, window=w, workspace=ws)
+    out = dms.prefill_attention(q, k, v, lg, window=w, workspace=ws, kernel=kernel)
     torch.cuda.synchronize()
     assert _ws_error(ws) == dms.DMS_OK
     rng = np.random.default_rng(5)
@@ -167,3 +174,12 @@ def test_prefill_rejects_bad_arguments():
     assert call(args(G=17)) == dms.DMS_ERR_INVALID_ARGUMENT
     assert call(args(w=-1)) == dms.DMS_ERR_INVALID_ARGUMENT
     torch.cuda.synchronize()
+
+
+def test_prefill_kernels_agree():
+    """The tcgen05 and the mma.sync kernels compute the same tiles: equal within rounding."""
+    B, P, H, G, w = 2, 1500, 2, 7, 256
+    q, k, v, lg = _inputs(B, P, H, G, 0.8, seed=31)
+    a = dms.prefill_attention(q, k, v, lg, window=w, kernel=dms.DMS_PREFILL_TCGEN05)
+    b = dms.prefill_attention(q, k, v, lg, window=w, kernel=dms.DMS_PREFILL_MMA_SYNC)
+    assert (a.float() - b.float()).abs().max().item() <= 2e-2

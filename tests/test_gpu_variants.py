@@ -136,13 +136,14 @@ def test_bulk_equals_token_by_token(policy):
     assert sets[0] == sets[1]
 
 
+@pytest.mark.parametrize("kernel", [dms.DMS_PREFILL_TCGEN05, dms.DMS_PREFILL_MMA_SYNC])
 @pytest.mark.parametrize("w,policy", [(16, 0), (512, 0), (16, IMM), (64, IMM)])
-def test_prefill_variants(w, policy):
+def test_prefill_variants(w, policy, kernel):
     B, P, H, G = 2, 700, 2, 4
     g = torch.Generator(device="cuda").manual_seed(w + policy)
     q = torch.randn((B, P, H * G, D), generator=g, device="cuda").to(torch.bfloat16)
     k, v, lg = _kvl(B, P, H, 0.7, 7 + w)
-    out = dms.prefill_attention(q, k, v, lg, window=w, eviction_policy=policy)
+    out = dms.prefill_attention(q, k, v, lg, window=w, eviction_policy=policy, kernel=kernel)
     Q, K, V, L = (workloads.bf16_bits(t) for t in (q, k, v, lg))
     got = out.float().cpu().numpy()
     errs = []
