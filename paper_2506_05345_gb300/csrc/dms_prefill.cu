@@ -836,7 +836,7 @@ dms_status dms_prefill_attention(const void* q, const void* k, const void* v,
                                  float sm_scale, void* workspace, size_t workspace_bytes,
                                  void* out, void* stream) {
   return prefill_impl(q, k, v, decision_logit, 1, batch, n_tokens, kv_heads, gqa_group, window,
-                      DMS_EVICT_DELAYED, kPrefillDefaultKernel, sm_scale, workspace,
+                      DMS_EVICT_DELAYED, dms::kPrefillDefaultKernel, sm_scale, workspace,
                       workspace_bytes, out, false, stream);
 }
 
@@ -847,7 +847,7 @@ dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const vo
                                           void* stream) {
   if (gqa_group < 1 || gqa_group > dms::kMaxGroup) return DMS_ERR_INVALID_ARGUMENT;
   return prefill_impl(q, k, v, q, (int64_t)gqa_group * dms::kHeadDim, batch, n_tokens, kv_heads,
-                      gqa_group, window, DMS_EVICT_DELAYED, kPrefillDefaultKernel, sm_scale,
+                      gqa_group, window, DMS_EVICT_DELAYED, dms::kPrefillDefaultKernel, sm_scale,
                       workspace, workspace_bytes, out, true, stream);
 }
 
