@@ -66,7 +66,7 @@ def parse():
     ap.add_argument("--shared-prefix", action="store_true",
                     help="append the workload's shared prompt once and share its frozen pages "
                          "between the sequences")
-    ap.add_argument("--prefill-kernel", default="mma_sync", choices=["mma_sync", "tcgen05"],
+    ap.add_argument("--prefill-kernel", default="tcgen05", choices=["tcgen05", "mma_sync"],
                     help="prefill attention kernel (with --prefill)")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the batch (small cases for profiling)")

@@ -249,8 +249,8 @@ dms_status dms_prefill_attention_borrowed(const void* q, const void* k, const vo
                                           void* stream);
 /* Prefill attention kernels (dms_prefill_attention_ex `kernel`). */
 enum {
-  DMS_PREFILL_TCGEN05 = 0,  /* 5th-generation tensor cores, accumulators in TMEM          */
-  DMS_PREFILL_MMA_SYNC = 1  /* warp-level mma.sync tiles (used by the plain entry points)  */
+  DMS_PREFILL_TCGEN05 = 0,  /* default: 5th-generation tensor cores, accumulators in TMEM */
+  DMS_PREFILL_MMA_SYNC = 1  /* warp-level mma.sync tiles; a cross-check path              */
 };
 /* The general form: decision_logit == NULL takes the decisions from the queries as in
  * the borrowed form; eviction_policy DMS_EVICT_DELAYED or DMS_EVICT_IMMEDIATE (the Sec. 5

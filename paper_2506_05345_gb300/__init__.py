@@ -170,7 +170,7 @@ def prefill_attention(q, k, v, decision_logit=None, window: int = 256, gqa_group
                                                             "decision_logit")
         code = dms_prefill_attention_ex(qp, kp, vp, lp, B, P, Hkv, gqa_group, window,
                                         eviction_policy,
-                                        DMS_PREFILL_MMA_SYNC if kernel < 0 else kernel,
+                                        DMS_PREFILL_TCGEN05 if kernel < 0 else kernel,
                                         sm_scale, wp, wb, op, _stream_ptr(stream))
         _check(code, "dms_prefill_attention_ex")
     elif decision_logit is None:

@@ -450,53 +450,69 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 }
 
 // ============================================================================ tcgen05 kernel
-// The same tiles on the 5th-generation tensor cores.  One CTA per (query head, 128-query
-// tile), 256 threads: warp 0 stages K / V tiles (bulk copies, 3 stages), warp 1 issues the
-// MMAs from one thread, warp 2 owns the tensor-memory allocation, warps 4-7 (one thread per
-// query row, TMEM lane = row) run the softmax and keep the output accumulator in registers.
-// Per 64-key tile: S = Q K^T (M 128, N 64, 8 MMAs of K 16) into TMEM; each softmax thread
-// loads its row of S, masks it, updates its running max / sum and writes its row of
-// P = exp2(S - m) as bf16 into shared memory; O_tile = P V (M 128, N 128, 4 MMAs) into TMEM;
-// the thread adds O_tile to its register accumulator after scaling that by the max
-// correction.  Operands sit in shared memory in the 128-byte-swizzled layout: rows of two
-// 128-byte d-halves, 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q, K and P
-// are K-major, V is MN-major (head_dim contiguous).
-constexpr int kTcThreads = 256;
+// The same tiles on the 5th-generation tensor cores.  One CTA per (KV head, 128-query tile,
+// pair of query heads of the group): both heads attend to the same keys, so every staged
+// K / V tile serves two 128 x 64 score tiles.  384 threads: warp 0 stages K / V tiles (bulk
+// copies, 3 stages), warp 1 issues the MMAs from one thread, warp 2 owns the tensor memory
+// (all 512 columns), warps 4-7 and 8-11 are the softmax warpgroups of the two heads (one
+// thread per query row, TMEM lane = row).
+// Tensor memory per head h: O (128 columns, fp32, accumulated by the MMAs) at 256 h and two
+// S buffers (64 columns each) at 256 h + 128 + 64 i.
+// Per 64-key tile t: S_h(t) = Q_h K^T (8 MMAs of K 16) into S buffer t % 2, issued before
+// the MMA thread waits for P(t - 1), so the tensor cores compute the next scores while the
+// softmax runs; each softmax thread loads its row of S, masks it (tiles visible to every
+// row of the CTA skip the mask), and writes its row of P = exp2(S - m) as bf16 into shared
+// memory; O_h += P_h V (4 MMAs).  The reference max m of a row moves only when the row max
+// exceeds it by more than 2^8 (then the row's O in tensor memory is rescaled first); the
+// same stale m is used for P and for the running sum l, so O / l is exact up to rounding.
+// Operands sit in shared memory in the 128-byte-swizzled layout: rows of two 128-byte
+// d-halves, 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q, K and P are
+// K-major, V is MN-major (head_dim contiguous).
+constexpr int kTcHeads = 2;                              // query heads per CTA
+constexpr int kTcThreads = (4 + 4 * kTcHeads) * 32;      // 384
 // Kernel of the plain entry points (the faster of the two as measured).
-constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_MMA_SYNC;
+constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_TCGEN05;
 constexpr int kTcStageBytes = 33 * 1024;  // K 16 KiB, V 16 KiB, key positions (1 KiB aligned)
 constexpr int kTcQBytes = kPfRows * kRowBytes;         // Q [2 d-halves][128 rows][128 B]
 constexpr int kTcPBytes = kPfRows * kPfKeys * 2;       // P [128 rows][64 keys] bf16
 constexpr int kTcOffQ = kPfStages * kTcStageBytes;
-constexpr int kTcOffP = kTcOffQ + kTcQBytes;
-constexpr int kTcOffBar = kTcOffP + kTcPBytes;
-constexpr int kTcSmemBytes = kTcOffBar + 256 + 1024;   // + barriers, + base alignment slack
-constexpr uint32_t kTcCols = 256;                      // TMEM: S at column 0, O_tile at 64
-constexpr uint32_t kTcColO = 64;
+constexpr int kTcOffP = kTcOffQ + kTcHeads * kTcQBytes;
+constexpr int kTcOffBar = kTcOffP + kTcHeads * kTcPBytes;
+constexpr int kTcSmemBytes = kTcOffBar + 512 + 1024;   // + barriers, + base alignment slack
+constexpr uint32_t kTcCols = 512;
+constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
+
+// Barriers of one head's pipeline.
+struct TcHeadBars {
+  uint64_t s_full[2];  // MMA commit: S buffer i holds the scores
+  uint64_t s_free[2];  // 128 arrivals: S buffer i read
+  uint64_t p_full;     // 128 arrivals: P in shared memory (and O rescaled)
+  uint64_t pv_done;    // MMA commit: O += P V done (P buffer free, O stable)
+};
 
 __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const PrefillParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* sq = smem + kTcOffQ;
-  uint8_t* sp = smem + kTcOffP;
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kTcOffBar);
   uint64_t* empty_bar = full_bar + kPfStages;
-  uint64_t* q_ready = empty_bar + kPfStages;  // 128 arrivals: Q staged
-  uint64_t* s_full = q_ready + 1;             // MMA commit: S in TMEM
-  uint64_t* p_full = s_full + 1;              // 128 arrivals: P in shared memory
-  uint64_t* o_full = p_full + 1;              // MMA commit: O_tile in TMEM
-  uint64_t* o_free = o_full + 1;              // 128 arrivals: S and O_tile read
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(o_free + 1);
+  uint64_t* q_ready = empty_bar + kPfStages;
+  TcHeadBars* hb = reinterpret_cast<TcHeadBars*>(q_ready + 1);
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(hb + kTcHeads);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int Hq = p.kv_heads * p.group;
-  const int tile_rank = blockIdx.x / p.n_qheads;
-  const int qt = p.n_qtiles - 1 - tile_rank;
-  const int qh = blockIdx.x - tile_rank * p.n_qheads;
-  const int b = qh / Hq, hq = qh - b * Hq, hk = hq / p.group;
-  const int64_t head = (int64_t)b * p.kv_heads + hk;
+  const int G = p.group, Hq = p.kv_heads * G;
+  const int pairs = (G + kTcHeads - 1) / kTcHeads;
+  const int n_units = p.n_qheads / G * pairs;  // (sequence, KV head, head pair)
+  const int tile_rank = blockIdx.x / n_units;
+  const int qt = p.n_qtiles - 1 - tile_rank;  // latest (heaviest) query tiles first
+  const int unit = blockIdx.x - tile_rank * n_units;
+  const int pair = unit % pairs, bh = unit / pairs;
+  const int b = bh / p.kv_heads, hk = bh - b * p.kv_heads;
+  const int hq0 = hk * G + kTcHeads * pair;
+  const int nh = min(kTcHeads, G - kTcHeads * pair);  // query heads of this CTA
+  const int64_t head = (int64_t)bh;
   const int P = p.P, w = p.window;
   const int j0 = qt * kPfRows;
   const int jmax = min(j0 + kPfRows, P) - 1;
@@ -511,11 +527,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
-    mbar_init(q_ready, kPfRows);
-    mbar_init(s_full, 1);
-    mbar_init(p_full, kPfRows);
-    mbar_init(o_full, 1);
-    mbar_init(o_free, kPfRows);
+    mbar_init(q_ready, kPfRows * nh);
+    for (int h = 0; h < kTcHeads; ++h) {
+      mbar_init(&hb[h].s_full[0], 1);
+      mbar_init(&hb[h].s_full[1], 1);
+      mbar_init(&hb[h].s_free[0], kPfRows);
+      mbar_init(&hb[h].s_free[1], kPfRows);
+      mbar_init(&hb[h].p_full, kPfRows);
+      mbar_init(&hb[h].pv_done, 1);
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 2) {
@@ -555,46 +575,66 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     if (lane == 0) {
       constexpr uint32_t idesc_s = f16_idesc(kPfRows, kPfKeys, 0);    // Q K^T: both K-major
       constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
-      const uint32_t q_base = smem_addr(sq), p_base = smem_addr(sp);
+      const uint32_t q_base = smem_addr(smem + kTcOffQ), p_base = smem_addr(smem + kTcOffP);
       mbar_wait(q_ready, 0, abort_flag, p.err);
-      for (int t = 0; t < n_tiles; ++t) {
-        const int s = t % kPfStages;
+      auto issue_scores = [&](int t) {
+        const int s = t % kPfStages, i = t & 1;
         const uint32_t k_base = smem_addr(smem + s * kTcStageBytes);
-        const uint32_t v_base = k_base + kPfTileBytes;
         mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);
-        if (t > 0) mbar_wait(o_free, (t - 1) & 1, abort_flag, p.err);
+        for (int h = 0; h < nh; ++h)
+          if (t >= 2) mbar_wait(&hb[h].s_free[i], ((t - 2) >> 1) & 1, abort_flag, p.err);
         tc_fence_after();
-        // S = Q K^T: k-step kk covers head_dim 16 kk .. 16 kk + 15 (d-half kk / 4)
+        for (int h = 0; h < nh; ++h) {
+          const uint32_t qh_base = q_base + (uint32_t)h * kTcQBytes;
+          const uint32_t d_s = tmem + (uint32_t)(256 * h + 128 + 64 * i);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (uint32_t)(kk & 3) * 32u;  // 16 head_dim elements = 32 B
-          const uint64_t a = sw128_desc(q_base + (uint32_t)(kk >> 2) * (kPfRows * 128u) + off, 16u, 1024u);
-          const uint64_t bk = sw128_desc(k_base + (uint32_t)(kk >> 2) * (kPfKeys * 128u) + off, 16u, 1024u);
-          tc_mma_ss(tmem, a, bk, idesc_s, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (uint32_t)(kk & 3) * 32u;  // 16 head_dim elements = 32 B
+            const uint64_t a = sw128_desc(qh_base + (uint32_t)(kk >> 2) * (kPfRows * 128u) + off,
+                                          16u, 1024u);
+            const uint64_t bk = sw128_desc(k_base + (uint32_t)(kk >> 2) * (kPfKeys * 128u) + off,
+                                           16u, 1024u);
+            tc_mma_ss(d_s, a, bk, idesc_s, kk > 0 ? 1u : 0u);
+          }
+          tc_commit(&hb[h].s_full[i]);
         }
-        tc_commit(s_full);
-        mbar_wait(p_full, t & 1, abort_flag, p.err);
-        tc_fence_after();
-        // O_tile = P V: k-step kk covers keys 16 kk .. 16 kk + 15; V atoms along head_dim
-        // are the two d-halves (leading offset 8 KiB), 8-key groups 1 KiB apart
+      };
+      if (n_tiles > 0) issue_scores(0);
+      for (int t = 0; t < n_tiles; ++t) {
+        if (t + 1 < n_tiles) issue_scores(t + 1);
+        const int s = t % kPfStages;
+        const uint32_t v_base = smem_addr(smem + s * kTcStageBytes) + kPfTileBytes;
+        for (int h = 0; h < nh; ++h) {
+          mbar_wait(&hb[h].p_full, t & 1, abort_flag, p.err);
+          tc_fence_after();
+          const uint32_t ph_base = p_base + (uint32_t)h * kTcPBytes;
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const uint64_t a = sw128_desc(p_base + (uint32_t)kk * 32u, 16u, 1024u);
-          const uint64_t bv = sw128_desc(v_base + (uint32_t)kk * 2048u, kPfKeys * 128u, 1024u);
-          tc_mma_ss(tmem + kTcColO, a, bv, idesc_o, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < 4; ++kk) {
+            // keys 16 kk .. 16 kk + 15; V atoms along head_dim are the two d-halves
+            // (leading offset 8 KiB), 8-key groups 1 KiB apart
+            const uint64_t a = sw128_desc(ph_base + (uint32_t)kk * 32u, 16u, 1024u);
+            const uint64_t bv = sw128_desc(v_base + (uint32_t)kk * 2048u, kPfKeys * 128u, 1024u);
+            tc_mma_ss(tmem + (uint32_t)(256 * h), a, bv, idesc_o, (t > 0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(&hb[h].pv_done);
         }
-        tc_commit(o_full);
-        tc_commit(&empty_bar[s]);  // the stage is free once both products are done
+        tc_commit(&empty_bar[s]);  // the stage is free once every product on it is done
       }
     }
-  } else if (warp >= 4) {
-    // ================================================================ softmax warpgroup
-    const int row = tid - 128;           // query row of the tile = TMEM lane
-    const int j = j0 + row;              // its query position
-    const uint32_t lane_addr = tmem + ((uint32_t)(32 * (warp - 4)) << 16);
+  } else if (warp >= 4 && (warp - 4) / 4 < nh) {
+    // ================================================================ softmax warpgroups
+    const int h = (warp - 4) / 4;
+    const int row = tid - 128 * (1 + h);  // query row of the tile = TMEM lane
+    const int j = j0 + row;
+    const int hq = hq0 + h;
+    const uint32_t lane_addr = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
+    const uint32_t o_col = (uint32_t)(256 * h);
+    TcHeadBars& bar = hb[h];
+    uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;
+    uint8_t* sp = smem + kTcOffP + h * kTcPBytes;
     // this row of Q into the K-major swizzled layout [d-half][row][128 B]
     {
-      const bool zero = p.zero_first && hq % p.group == 0;
+      const bool zero = p.zero_first && hq % G == 0;
       const __nv_bfloat16* qrow = p.q + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
 #pragma unroll
       for (int c = 0; c < 16; ++c) {
@@ -607,51 +647,82 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
       fence_proxy_async_smem();
       mbar_arrive(q_ready);
     }
-    float o[kHeadDim];
-#pragma unroll
-    for (int d = 0; d < kHeadDim; ++d) o[d] = 0.f;
-    float m = -INFINITY, l = 0.f;
+    float m = -INFINITY, l = 0.f;  // reference max and running sum of this row
     for (int t = 0; t < n_tiles; ++t) {
-      const int s = t % kPfStages;
+      const int s = t % kPfStages, i = t & 1;
       const bool retained = t < n_ct;
       const int r0 = retained ? t * kPfKeys : bs + (t - n_ct) * kPfKeys;
       const int rows = retained ? min(kPfKeys, nc - r0) : min(kPfKeys, jmax + 1 - r0);
       const uint8_t* st = smem + s * kTcStageBytes;
-      mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);  // key positions
-      if (rows < kPfKeys) {
+      mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);
+      if (rows < kPfKeys && h == 0) {
         // V rows past the tile's keys hold stale bytes, possibly NaN patterns; P is 0
-        // there, but 0 * NaN is not: zero them before P V reads the tile (the proxy
-        // fence before the P-ready arrival orders these writes for the tensor cores).
+        // there, but 0 * NaN is not: zero them before any P V reads the tile (ordered for
+        // the tensor cores by the proxy fence before the P-ready arrival).
         uint8_t* vt = smem + s * kTcStageBytes + kPfTileBytes;
-        for (int i = row; i < (kPfKeys - rows) * 16; i += kPfRows)
-          *reinterpret_cast<uint4*>(vt + tile_off((uint32_t)(rows + i / 16), (uint32_t)(i & 15))) =
+        for (int e = row; e < (kPfKeys - rows) * 16; e += kPfRows)
+          *reinterpret_cast<uint4*>(vt + tile_off((uint32_t)(rows + e / 16), (uint32_t)(e & 15))) =
               make_uint4(0u, 0u, 0u, 0u);
       }
-      mbar_wait(s_full, t & 1, abort_flag, p.err);
+      mbar_wait(&bar.s_full[i], (t >> 1) & 1, abort_flag, p.err);
       tc_fence_after();
       float sc[kPfKeys];
 #pragma unroll
       for (int c = 0; c < kPfKeys / 16; ++c) {
         float r[16];
-        tmem_ld16(lane_addr + (uint32_t)(16 * c), r);
+        tmem_ld16(lane_addr + (uint32_t)(256 * h + 128 + 64 * i + 16 * c), r);
         tmem_wait_ld();
 #pragma unroll
-        for (int i = 0; i < 16; ++i) sc[16 * c + i] = r[i];
+        for (int e = 0; e < 16; ++e) sc[16 * c + e] = r[e];
       }
+      tc_fence_before();
+      mbar_arrive(&bar.s_free[i]);
+      // mask: skipped when every key of the tile is visible to every query of the CTA
       const int32_t* spos = reinterpret_cast<const int32_t*>(st + 2 * kPfTileBytes);
+      const bool all_visible =
+          rows == kPfKeys && (retained ? spos[kPfKeys - 1] < j0 - w
+                                       : (r0 >= jmax - w && r0 + kPfKeys - 1 <= j0));
       float mx = -INFINITY;
+      if (all_visible) {
 #pragma unroll
-      for (int kidx = 0; kidx < kPfKeys; ++kidx) {
-        const bool valid = kidx < rows;
-        const int pos = retained ? (valid ? spos[kidx] : 0) : r0 + kidx;
-        const bool vis = valid && (retained ? pos < j - w : (pos >= j - w && pos <= j));
-        sc[kidx] = vis ? sc[kidx] * p.scale_log2 : -INFINITY;
-        mx = fmaxf(mx, sc[kidx]);
+        for (int k = 0; k < kPfKeys; ++k) {
+          sc[k] *= p.scale_log2;
+          mx = fmaxf(mx, sc[k]);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < kPfKeys; ++k) {
+          const bool valid = k < rows;
+          const int pos = retained ? (valid ? spos[k] : 0) : r0 + k;
+          const bool vis = valid && (retained ? pos < j - w : (pos >= j - w && pos <= j));
+          sc[k] = vis ? sc[k] * p.scale_log2 : -INFINITY;
+          mx = fmaxf(mx, sc[k]);
+        }
       }
-      const float mn = fmaxf(m, mx);
-      const float base = mn == -INFINITY ? 0.f : mn;
-      const float corr = exp2f(m - base);
-      m = mn;
+      // P buffer and O are in use until the previous product is done
+      if (t > 0) {
+        mbar_wait(&bar.pv_done, (t - 1) & 1, abort_flag, p.err);
+        tc_fence_after();
+      }
+      float corr = 1.f;
+      if (mx > m + kTcRescale || (m == -INFINITY && mx > -INFINITY)) {
+        const float mn = mx;
+        corr = exp2f(m - mn);  // 0 when m = -inf
+        m = mn;
+      }
+      if (t > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
+#pragma unroll
+        for (int c = 0; c < kHeadDim / 16; ++c) {
+          float r[16];
+          tmem_ld16(lane_addr + o_col + (uint32_t)(16 * c), r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) r[e] *= corr;
+          tmem_st16(lane_addr + o_col + (uint32_t)(16 * c), r);
+        }
+        tmem_wait_st();
+      }
+      const float base = m == -INFINITY ? 0.f : m;
       float sum = 0.f;
       // P row: 64 bf16 = 8 chunks of 16 bytes, chunk c at (c ^ (row & 7))
 #pragma unroll
@@ -669,32 +740,32 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
       l = l * corr + sum;
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(p_full);
-      mbar_wait(o_full, t & 1, abort_flag, p.err);
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < kHeadDim / 16; ++c) {
-        float r[16];
-        tmem_ld16(lane_addr + kTcColO + (uint32_t)(16 * c), r);
-        tmem_wait_ld();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) o[16 * c + i] = o[16 * c + i] * corr + r[i];
-      }
-      tc_fence_before();
-      mbar_arrive(o_free);
+      mbar_arrive(&bar.p_full);
     }
     // normalise and store this row
-    if (j < P) {
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-      __nv_bfloat16* orow = p.out + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
+    if (n_tiles > 0) {
+      mbar_wait(&bar.pv_done, (n_tiles - 1) & 1, abort_flag, p.err);
+      tc_fence_after();
+    }
+    const float inv = l > 0.f ? 1.f / l : 0.f;
+    __nv_bfloat16* orow = p.out + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        uint4 val;
-        val.x = pack_bf16x2(o[8 * c + 0] * inv, o[8 * c + 1] * inv);
-        val.y = pack_bf16x2(o[8 * c + 2] * inv, o[8 * c + 3] * inv);
-        val.z = pack_bf16x2(o[8 * c + 4] * inv, o[8 * c + 5] * inv);
-        val.w = pack_bf16x2(o[8 * c + 6] * inv, o[8 * c + 7] * inv);
-        *reinterpret_cast<uint4*>(orow + 8 * c) = val;
+    for (int c = 0; c < kHeadDim / 16; ++c) {
+      float r[16];
+      tmem_ld16(lane_addr + o_col + (uint32_t)(16 * c), r);
+      tmem_wait_ld();
+      if (j < P) {
+        uint4 v0, v1;
+        v0.x = pack_bf16x2(r[0] * inv, r[1] * inv);
+        v0.y = pack_bf16x2(r[2] * inv, r[3] * inv);
+        v0.z = pack_bf16x2(r[4] * inv, r[5] * inv);
+        v0.w = pack_bf16x2(r[6] * inv, r[7] * inv);
+        v1.x = pack_bf16x2(r[8] * inv, r[9] * inv);
+        v1.y = pack_bf16x2(r[10] * inv, r[11] * inv);
+        v1.z = pack_bf16x2(r[12] * inv, r[13] * inv);
+        v1.w = pack_bf16x2(r[14] * inv, r[15] * inv);
+        *reinterpret_cast<uint4*>(orow + 16 * c) = v0;
+        *reinterpret_cast<uint4*>(orow + 16 * c + 8) = v1;
       }
     }
   }
@@ -778,10 +849,12 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
   pp.n_qheads = (int32_t)(H * group);
   pp.scale_log2 = scale_log2;
   const int64_t grid = (int64_t)pp.n_qtiles * pp.n_qheads;
-  if (kernel == DMS_PREFILL_MMA_SYNC)
+  if (kernel == DMS_PREFILL_MMA_SYNC) {
     prefill_attn_kernel<<<(unsigned)grid, kPfThreads, kPfSmemBytes, stream>>>(pp);
-  else
-    prefill_tc_kernel<<<(unsigned)grid, kTcThreads, kTcSmemBytes, stream>>>(pp);
+  } else {
+    const int64_t units = H * ((group + kTcHeads - 1) / kTcHeads);
+    prefill_tc_kernel<<<(unsigned)(pp.n_qtiles * units), kTcThreads, kTcSmemBytes, stream>>>(pp);
+  }
   return cudaGetLastError();
 }
 
