@@ -462,7 +462,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // the MMA thread waits for P(t - 1), so the tensor cores compute the next scores while the
 // softmax runs; each softmax thread loads its row of S, masks it (tiles visible to every
 // row of the CTA skip the mask), and writes its row of P = exp2(S - m) as bf16 into shared
-// memory; O_h += P_h V (4 MMAs).  The reference max m of a row moves only when the row max
+// memory buffer t % 2, so the next softmax overlaps O_h += P_h V (4 MMAs).  The reference max m of a row moves only when the row max
 // exceeds it by more than 2^8 (then the row's O in tensor memory is rescaled first); the
 // same stale m is used for P and for the running sum l, so O / l is exact up to rounding.
 // Operands sit in shared memory in the 128-byte-swizzled layout: rows of two 128-byte
@@ -472,22 +472,34 @@ constexpr int kTcHeads = 2;                              // query heads per CTA
 constexpr int kTcThreads = (4 + 4 * kTcHeads) * 32;      // 384
 // Kernel of the plain entry points (the faster of the two as measured).
 constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_TCGEN05;
-constexpr int kTcStageBytes = 33 * 1024;  // K 16 KiB, V 16 KiB, key positions (1 KiB aligned)
+#ifndef DMS_TC_STAGES
+#define DMS_TC_STAGES 4
+#endif
+#ifndef DMS_TC_PBUFS
+#define DMS_TC_PBUFS 1
+#endif
+constexpr int kTcStages = DMS_TC_STAGES;  // K / V stages
+constexpr int kTcPBufs = DMS_TC_PBUFS;    // P buffers per head
+constexpr int kTcStageBytes = 2 * kPfTileBytes;        // K 16 KiB, V 16 KiB (1 KiB aligned)
 constexpr int kTcQBytes = kPfRows * kRowBytes;         // Q [2 d-halves][128 rows][128 B]
 constexpr int kTcPBytes = kPfRows * kPfKeys * 2;       // P [128 rows][64 keys] bf16
-constexpr int kTcOffQ = kPfStages * kTcStageBytes;
-constexpr int kTcOffP = kTcOffQ + kTcHeads * kTcQBytes;
-constexpr int kTcOffBar = kTcOffP + kTcHeads * kTcPBytes;
+constexpr int kTcOffQ = kTcStages * kTcStageBytes;
+constexpr int kTcOffP = kTcOffQ + kTcHeads * kTcQBytes;  // P [head][buffer]
+constexpr int kTcOffPos = kTcOffP + kTcHeads * kTcPBufs * kTcPBytes;  // key positions [stage][64]
+constexpr int kTcOffBar = kTcOffPos + kTcStages * kPfKeys * 4;
 constexpr int kTcSmemBytes = kTcOffBar + 512 + 1024;   // + barriers, + base alignment slack
+static_assert(kTcSmemBytes <= 227 * 1024, "tcgen05 prefill shared memory");
 constexpr uint32_t kTcCols = 512;
 constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
 
-// Barriers of one head's pipeline.
+// Barriers of one head's pipeline.  S buffer i serves the tiles with t % 2 = i, P buffer
+// u the tiles with t % kTcPBufs = u, so each barrier completes once per use of its buffer
+// and no wait is ever two phases behind (a buffer is reused only after its waiter moved on).
 struct TcHeadBars {
-  uint64_t s_full[2];  // MMA commit: S buffer i holds the scores
-  uint64_t s_free[2];  // 128 arrivals: S buffer i read
-  uint64_t p_full;     // 128 arrivals: P in shared memory (and O rescaled)
-  uint64_t pv_done;    // MMA commit: O += P V done (P buffer free, O stable)
+  uint64_t s_full[2];          // MMA commit: S buffer i holds the scores
+  uint64_t s_free[2];          // 128 arrivals: S buffer i read
+  uint64_t p_full[kTcPBufs];   // 128 arrivals: P buffer u written (and O rescaled)
+  uint64_t pv_done[kTcPBufs];  // MMA commit: O += P_u V done (buffer free; O stable then)
 };
 
 __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const PrefillParams p) {
@@ -495,8 +507,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kTcOffBar);
-  uint64_t* empty_bar = full_bar + kPfStages;
-  uint64_t* q_ready = empty_bar + kPfStages;
+  uint64_t* empty_bar = full_bar + kTcStages;
+  uint64_t* q_ready = empty_bar + kTcStages;
   TcHeadBars* hb = reinterpret_cast<TcHeadBars*>(q_ready + 1);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(hb + kTcHeads);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(s_tmem + 1);
@@ -523,18 +535,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
 
   if (tid == 0) {
     *abort_flag = 0;
-    for (int s = 0; s < kPfStages; ++s) {
+    for (int s = 0; s < kTcStages; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
     mbar_init(q_ready, kPfRows * nh);
     for (int h = 0; h < kTcHeads; ++h) {
-      mbar_init(&hb[h].s_full[0], 1);
-      mbar_init(&hb[h].s_full[1], 1);
-      mbar_init(&hb[h].s_free[0], kPfRows);
-      mbar_init(&hb[h].s_free[1], kPfRows);
-      mbar_init(&hb[h].p_full, kPfRows);
-      mbar_init(&hb[h].pv_done, 1);
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&hb[h].s_full[i], 1);
+        mbar_init(&hb[h].s_free[i], kPfRows);
+      }
+      for (int u = 0; u < kTcPBufs; ++u) {
+        mbar_init(&hb[h].p_full[u], kPfRows);
+        mbar_init(&hb[h].pv_done[u], 1);
+      }
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -550,24 +564,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     // ================================================================ producer
     if (lane == 0) {
       for (int t = 0; t < n_tiles; ++t) {
-        const int s = t % kPfStages, use = t / kPfStages;
+        const int s = t % kTcStages, use = t / kTcStages;
         if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.err);
         uint8_t* st = smem + s * kTcStageBytes;
         if (t < n_ct) {
           const int r0 = t * kPfKeys, rows = min(kPfKeys, nc - r0);
           mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes + kPfKeys * 4);
           stage_tile(st, p.kc, p.vc, head, P, r0, rows, &full_bar[s]);
-          bulk_copy_g2s(st + 2 * kPfTileBytes, p.pc + head * pc_stride(P) + r0, kPfKeys * 4,
-                        &full_bar[s]);
+          bulk_copy_g2s(smem + kTcOffPos + s * kPfKeys * 4, p.pc + head * pc_stride(P) + r0,
+                        kPfKeys * 4, &full_bar[s]);
         } else {
           const int r0 = bs + (t - n_ct) * kPfKeys, rows = min(kPfKeys, jmax + 1 - r0);
           mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes);
           stage_tile(st, p.kd, p.vd, head, P, r0, rows, &full_bar[s]);
         }
       }
-      for (int s = 0; s < kPfStages && s < n_tiles; ++s) {
-        const int last_t = s + ((n_tiles - 1 - s) / kPfStages) * kPfStages;
-        mbar_wait(&full_bar[s], (last_t / kPfStages) & 1, abort_flag, p.err);
+      for (int s = 0; s < kTcStages && s < n_tiles; ++s) {
+        const int last_t = s + ((n_tiles - 1 - s) / kTcStages) * kTcStages;
+        mbar_wait(&full_bar[s], (last_t / kTcStages) & 1, abort_flag, p.err);
       }
     }
   } else if (warp == 1) {
@@ -575,48 +589,58 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     if (lane == 0) {
       constexpr uint32_t idesc_s = f16_idesc(kPfRows, kPfKeys, 0);    // Q K^T: both K-major
       constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
-      const uint32_t q_base = smem_addr(smem + kTcOffQ), p_base = smem_addr(smem + kTcOffP);
+      // Descriptors are built once; the start address (16-byte units, low bits) is stepped:
+      // +2 per 16 head_dim elements of Q / K inside a d-half, + half size at kk = 4;
+      // +2 per 16 keys of P; +128 (2 KiB) per 16 keys of V.
+      const uint64_t dq0 = sw128_desc(smem_addr(smem + kTcOffQ), 16u, 1024u);
+      const uint64_t dp0 = sw128_desc(smem_addr(smem + kTcOffP), 16u, 1024u);
+      const uint64_t dk0 = sw128_desc(smem_addr(smem), 16u, 1024u);
+      const uint64_t dv0 = sw128_desc(smem_addr(smem) + kPfTileBytes, kPfKeys * 128u, 1024u);
+      constexpr uint64_t kQHead = kTcQBytes >> 4, kQHalf = (kPfRows * 128) >> 4;
+      constexpr uint64_t kKHalf = (kPfKeys * 128) >> 4, kStage = kTcStageBytes >> 4;
+      constexpr uint64_t kPBuf = kTcPBytes >> 4;
       mbar_wait(q_ready, 0, abort_flag, p.err);
       auto issue_scores = [&](int t) {
-        const int s = t % kPfStages, i = t & 1;
-        const uint32_t k_base = smem_addr(smem + s * kTcStageBytes);
-        mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);
+        const int s = t % kTcStages, i = t & 1;
+        mbar_wait(&full_bar[s], (t / kTcStages) & 1, abort_flag, p.err);
         for (int h = 0; h < nh; ++h)
           if (t >= 2) mbar_wait(&hb[h].s_free[i], ((t - 2) >> 1) & 1, abort_flag, p.err);
         tc_fence_after();
+        const uint64_t dk = dk0 + (uint64_t)s * kStage;
         for (int h = 0; h < nh; ++h) {
-          const uint32_t qh_base = q_base + (uint32_t)h * kTcQBytes;
+          const uint64_t dq = dq0 + (uint64_t)h * kQHead;
           const uint32_t d_s = tmem + (uint32_t)(256 * h + 128 + 64 * i);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (uint32_t)(kk & 3) * 32u;  // 16 head_dim elements = 32 B
-            const uint64_t a = sw128_desc(qh_base + (uint32_t)(kk >> 2) * (kPfRows * 128u) + off,
-                                          16u, 1024u);
-            const uint64_t bk = sw128_desc(k_base + (uint32_t)(kk >> 2) * (kPfKeys * 128u) + off,
-                                           16u, 1024u);
-            tc_mma_ss(d_s, a, bk, idesc_s, kk > 0 ? 1u : 0u);
-          }
+          tc_mma_ss_k<false>(d_s, dq, dk, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + 2, dk + 2, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + 4, dk + 4, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + 6, dk + 6, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf, dk + kKHalf, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf + 2, dk + kKHalf + 2, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf + 4, dk + kKHalf + 4, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
           tc_commit(&hb[h].s_full[i]);
         }
       };
       if (n_tiles > 0) issue_scores(0);
       for (int t = 0; t < n_tiles; ++t) {
         if (t + 1 < n_tiles) issue_scores(t + 1);
-        const int s = t % kPfStages;
-        const uint32_t v_base = smem_addr(smem + s * kTcStageBytes) + kPfTileBytes;
+        const int s = t % kTcStages, u = t % kTcPBufs;
+        const uint64_t dv = dv0 + (uint64_t)s * kStage;
         for (int h = 0; h < nh; ++h) {
-          mbar_wait(&hb[h].p_full, t & 1, abort_flag, p.err);
+          mbar_wait(&hb[h].p_full[u], (t / kTcPBufs) & 1, abort_flag, p.err);
           tc_fence_after();
-          const uint32_t ph_base = p_base + (uint32_t)h * kTcPBytes;
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {
-            // keys 16 kk .. 16 kk + 15; V atoms along head_dim are the two d-halves
-            // (leading offset 8 KiB), 8-key groups 1 KiB apart
-            const uint64_t a = sw128_desc(ph_base + (uint32_t)kk * 32u, 16u, 1024u);
-            const uint64_t bv = sw128_desc(v_base + (uint32_t)kk * 2048u, kPfKeys * 128u, 1024u);
-            tc_mma_ss(tmem + (uint32_t)(256 * h), a, bv, idesc_o, (t > 0 || kk > 0) ? 1u : 0u);
-          }
-          tc_commit(&hb[h].pv_done);
+          // keys 16 kk .. 16 kk + 15; V atoms along head_dim are the two d-halves (leading
+          // offset 8 KiB), 8-key groups 1 KiB apart
+          const uint64_t dp = dp0 + (uint64_t)(kTcPBufs * h + u) * kPBuf;
+          const uint32_t d_o = tmem + (uint32_t)(256 * h);
+          if (t == 0)
+            tc_mma_ss_k<false>(d_o, dp, dv, idesc_o);
+          else
+            tc_mma_ss_k<true>(d_o, dp, dv, idesc_o);
+          tc_mma_ss_k<true>(d_o, dp + 2, dv + 128, idesc_o);
+          tc_mma_ss_k<true>(d_o, dp + 4, dv + 256, idesc_o);
+          tc_mma_ss_k<true>(d_o, dp + 6, dv + 384, idesc_o);
+          tc_commit(&hb[h].pv_done[u]);
         }
         tc_commit(&empty_bar[s]);  // the stage is free once every product on it is done
       }
@@ -631,7 +655,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     const uint32_t o_col = (uint32_t)(256 * h);
     TcHeadBars& bar = hb[h];
     uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;
-    uint8_t* sp = smem + kTcOffP + h * kTcPBytes;
     // this row of Q into the K-major swizzled layout [d-half][row][128 B]
     {
       const bool zero = p.zero_first && hq % G == 0;
@@ -649,12 +672,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     }
     float m = -INFINITY, l = 0.f;  // reference max and running sum of this row
     for (int t = 0; t < n_tiles; ++t) {
-      const int s = t % kPfStages, i = t & 1;
+      const int s = t % kTcStages, i = t & 1;
       const bool retained = t < n_ct;
       const int r0 = retained ? t * kPfKeys : bs + (t - n_ct) * kPfKeys;
       const int rows = retained ? min(kPfKeys, nc - r0) : min(kPfKeys, jmax + 1 - r0);
-      const uint8_t* st = smem + s * kTcStageBytes;
-      mbar_wait(&full_bar[s], (t / kPfStages) & 1, abort_flag, p.err);
+      const int u = t % kTcPBufs;
+      uint8_t* sp = smem + kTcOffP + (kTcPBufs * h + u) * kTcPBytes;
+      mbar_wait(&full_bar[s], (t / kTcStages) & 1, abort_flag, p.err);
       if (rows < kPfKeys && h == 0) {
         // V rows past the tile's keys hold stale bytes, possibly NaN patterns; P is 0
         // there, but 0 * NaN is not: zero them before any P V reads the tile (ordered for
@@ -666,29 +690,26 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
       }
       mbar_wait(&bar.s_full[i], (t >> 1) & 1, abort_flag, p.err);
       tc_fence_after();
+      // the row of S: four loads in flight, one wait
       float sc[kPfKeys];
-#pragma unroll
-      for (int c = 0; c < kPfKeys / 16; ++c) {
-        float r[16];
-        tmem_ld16(lane_addr + (uint32_t)(256 * h + 128 + 64 * i + 16 * c), r);
+      {
+        const uint32_t sa = lane_addr + (uint32_t)(256 * h + 128 + 64 * i);
+        tmem_ld16_at(sa, sc);
+        tmem_ld16_at(sa + 16, sc + 16);
+        tmem_ld16_at(sa + 32, sc + 32);
+        tmem_ld16_at(sa + 48, sc + 48);
         tmem_wait_ld();
-#pragma unroll
-        for (int e = 0; e < 16; ++e) sc[16 * c + e] = r[e];
       }
       tc_fence_before();
       mbar_arrive(&bar.s_free[i]);
       // mask: skipped when every key of the tile is visible to every query of the CTA
-      const int32_t* spos = reinterpret_cast<const int32_t*>(st + 2 * kPfTileBytes);
+      const int32_t* spos = reinterpret_cast<const int32_t*>(smem + kTcOffPos + s * kPfKeys * 4);
       const bool all_visible =
           rows == kPfKeys && (retained ? spos[kPfKeys - 1] < j0 - w
                                        : (r0 >= jmax - w && r0 + kPfKeys - 1 <= j0));
-      float mx = -INFINITY;
       if (all_visible) {
 #pragma unroll
-        for (int k = 0; k < kPfKeys; ++k) {
-          sc[k] *= p.scale_log2;
-          mx = fmaxf(mx, sc[k]);
-        }
+        for (int k = 0; k < kPfKeys; ++k) sc[k] *= p.scale_log2;
       } else {
 #pragma unroll
         for (int k = 0; k < kPfKeys; ++k) {
@@ -696,12 +717,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
           const int pos = retained ? (valid ? spos[k] : 0) : r0 + k;
           const bool vis = valid && (retained ? pos < j - w : (pos >= j - w && pos <= j));
           sc[k] = vis ? sc[k] * p.scale_log2 : -INFINITY;
-          mx = fmaxf(mx, sc[k]);
         }
       }
-      // P buffer and O are in use until the previous product is done
-      if (t > 0) {
-        mbar_wait(&bar.pv_done, (t - 1) & 1, abort_flag, p.err);
+      // row max over eight independent chains
+      float mx8[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx8[e] = sc[e];
+#pragma unroll
+      for (int k = 8; k < kPfKeys; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], sc[k]);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      // P buffer u is in use until the product of tile t - kTcPBufs is done
+      if (t >= kTcPBufs) {
+        mbar_wait(&bar.pv_done[u], ((t - kTcPBufs) / kTcPBufs) & 1, abort_flag, p.err);
         tc_fence_after();
       }
       float corr = 1.f;
@@ -710,8 +738,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
         corr = exp2f(m - mn);  // 0 when m = -inf
         m = mn;
       }
-      if (t > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
-#pragma unroll
+      const bool rescale = t > 0 && __any_sync(0xffffffffu, corr != 1.f);
+      if (rescale && kTcPBufs > 1) {
+        // O must hold every earlier product first: wait for the one of tile t - 1
+        mbar_wait(&bar.pv_done[(t - 1) % kTcPBufs], ((t - 1) / kTcPBufs) & 1, abort_flag, p.err);
+        tc_fence_after();
+      }
+      if (rescale) {
+        // (rare: only when a row's max grew past the threshold; 16 columns at a time, the
+        // scores of the tile stay in registers meanwhile)
+#pragma unroll 1
         for (int c = 0; c < kHeadDim / 16; ++c) {
           float r[16];
           tmem_ld16(lane_addr + o_col + (uint32_t)(16 * c), r);
@@ -723,28 +759,33 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
         tmem_wait_st();
       }
       const float base = m == -INFINITY ? 0.f : m;
-      float sum = 0.f;
+      float sum8[8];  // eight independent partial sums (chunk c)
       // P row: 64 bf16 = 8 chunks of 16 bytes, chunk c at (c ^ (row & 7))
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         uint32_t pk[4];
+        float sc_sum = 0.f;
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float p0 = exp2f(sc[8 * c + 2 * e] - base), p1 = exp2f(sc[8 * c + 2 * e + 1] - base);
-          sum += p0 + p1;
+          sc_sum += p0 + p1;
           pk[e] = pack_bf16x2(p0, p1);
         }
+        sum8[c] = sc_sum;
         *reinterpret_cast<uint4*>(sp + row * 128 + chunk_in_row(row, c)) =
             make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
+      const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) +
+                        ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
       l = l * corr + sum;
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&bar.p_full);
+      mbar_arrive(&bar.p_full[u]);
     }
-    // normalise and store this row
+    // normalise and store this row (the last product completes after all earlier ones)
     if (n_tiles > 0) {
-      mbar_wait(&bar.pv_done, (n_tiles - 1) & 1, abort_flag, p.err);
+      mbar_wait(&bar.pv_done[(n_tiles - 1) % kTcPBufs], ((n_tiles - 1) / kTcPBufs) & 1, abort_flag,
+                p.err);
       tc_fence_after();
     }
     const float inv = l > 0.f ? 1.f / l : 0.f;
