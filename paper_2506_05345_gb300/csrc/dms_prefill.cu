@@ -450,68 +450,96 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 }
 
 // ============================================================================ tcgen05 kernel
-// The same tiles on the 5th-generation tensor cores.  One CTA per (KV head, 128-query tile,
-// pair of query heads of the group): both heads attend to the same keys, so every staged
-// K / V tile serves two 128 x 64 score tiles.  384 threads: warp 0 stages K / V tiles (bulk
-// copies, 3 stages), warp 1 issues the MMAs from one thread, warp 2 owns the tensor memory
-// (all 512 columns), warps 4-7 and 8-11 are the softmax warpgroups of the two heads (one
-// thread per query row, TMEM lane = row).
-// Tensor memory per head h: O (128 columns, fp32, accumulated by the MMAs) at 256 h and two
-// S buffers (64 columns each) at 256 h + 128 + 64 i.
-// Per 64-key tile t: S_h(t) = Q_h K^T (8 MMAs of K 16) into S buffer t % 2, issued before
-// the MMA thread waits for P(t - 1), so the tensor cores compute the next scores while the
-// softmax runs; each softmax thread loads its row of S, masks it (tiles visible to every
-// row of the CTA skip the mask), and writes its row of P = exp2(S - m) as bf16 into shared
-// memory buffer t % 2, so the next softmax overlaps O_h += P_h V (4 MMAs).  The reference max m of a row moves only when the row max
-// exceeds it by more than 2^8 (then the row's O in tensor memory is rescaled first); the
-// same stale m is used for P and for the running sum l, so O / l is exact up to rounding.
-// Operands sit in shared memory in the 128-byte-swizzled layout: rows of two 128-byte
-// d-halves, 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q, K and P are
-// K-major, V is MN-major (head_dim contiguous).
+// The same attention on the 5th-generation tensor cores.  One CTA per (KV head, 128-query
+// tile, pair of query heads of the group): both heads attend to the same keys, so every
+// staged K / V tile serves two score tiles.  Key tiles hold 128 keys, so every MMA is
+// M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the time of an N 128
+// one for half its work).  384 threads: warp 0 stages K tiles (3-slot ring) and V tiles
+// (2-slot ring) with bulk copies, warp 1 issues the MMAs from one thread, warp 2 owns the
+// tensor memory (all 512 columns), warps 4-7 and 8-11 are the softmax warpgroups of the two
+// heads (one thread per query row, TMEM lane = row).
+// Tensor memory per head h: O (128 fp32 columns) at 256 h and S (128 fp32 columns) at
+// 256 h + 128.  P overwrites S in place as packed bf16 pairs (keys 2c, 2c + 1 in column c)
+// and is the A operand of O += P V straight from tensor memory.  S_h(t + 1) is issued after
+// O_h += P_h(t) V(t) and one thread's MMAs run in issue order, so new scores never
+// overwrite P before it is read.
+// Each softmax thread takes its row of S in two 64-key halves: mask (skipped for halves the
+// whole warp sees), row max, P = 2^(S scale - m) into tensor memory; the half's O += P V
+// (4 MMAs) starts while the thread works on the next half, and one head's softmax overlaps
+// the other head's MMAs.  The reference max m of a row moves only when a half's max exceeds
+// it by more than 2^8 (then O is rescaled first); P and the running sum l use the same m,
+// so O / l is exact up to rounding.
+// Visibility: the retained keys query j sees are the first before[j - w] compacted rows, so
+// one count masks a retained tile; window keys are a contiguous run of the band.  Stale rows
+// of a partial V tile are zeroed before its copy (P is 0 there, but 0 * NaN is not).
+// Shared-memory operands use the 128-byte-swizzled layout: rows of two 128-byte d-halves,
+// 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q and K are K-major, V is
+// MN-major (head_dim contiguous).
 constexpr int kTcHeads = 2;                              // query heads per CTA
 constexpr int kTcThreads = (4 + 4 * kTcHeads) * 32;      // 384
 // Kernel of the plain entry points (the faster of the two as measured).
 constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_TCGEN05;
-#ifndef DMS_TC_STAGES
-#define DMS_TC_STAGES 4
-#endif
-#ifndef DMS_TC_PBUFS
-#define DMS_TC_PBUFS 1
-#endif
-constexpr int kTcStages = DMS_TC_STAGES;  // K / V stages
-constexpr int kTcPBufs = DMS_TC_PBUFS;    // P buffers per head
-constexpr int kTcStageBytes = 2 * kPfTileBytes;        // K 16 KiB, V 16 KiB (1 KiB aligned)
-constexpr int kTcQBytes = kPfRows * kRowBytes;         // Q [2 d-halves][128 rows][128 B]
-constexpr int kTcPBytes = kPfRows * kPfKeys * 2;       // P [128 rows][64 keys] bf16
-constexpr int kTcOffQ = kTcStages * kTcStageBytes;
-constexpr int kTcOffP = kTcOffQ + kTcHeads * kTcQBytes;  // P [head][buffer]
-constexpr int kTcOffPos = kTcOffP + kTcHeads * kTcPBufs * kTcPBytes;  // key positions [stage][64]
-constexpr int kTcOffBar = kTcOffPos + kTcStages * kPfKeys * 4;
-constexpr int kTcSmemBytes = kTcOffBar + 512 + 1024;   // + barriers, + base alignment slack
+constexpr int kTcKeys = 128;                             // keys per tile
+constexpr int kTcKSlots = 3;                             // K ring
+constexpr int kTcVSlots = 2;                             // V ring
+constexpr int kTcHalfBytes = kTcKeys * 128;              // one d-half of a tile, 16 KiB
+constexpr int kTcTileBytes = 2 * kTcHalfBytes;           // [2 d-halves][128 rows][128 B]
+constexpr int kTcQBytes = kPfRows * kRowBytes;           // Q, same layout
+constexpr int kTcOffV = kTcKSlots * kTcTileBytes;
+constexpr int kTcOffQ = kTcOffV + kTcVSlots * kTcTileBytes;
+constexpr int kTcOffBar = kTcOffQ + kTcHeads * kTcQBytes;
+constexpr int kTcSmemBytes = kTcOffBar + 256 + 1024;    // + barriers, + base alignment slack
 static_assert(kTcSmemBytes <= 227 * 1024, "tcgen05 prefill shared memory");
 constexpr uint32_t kTcCols = 512;
 constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
 
-// Barriers of one head's pipeline.  S buffer i serves the tiles with t % 2 = i, P buffer
-// u the tiles with t % kTcPBufs = u, so each barrier completes once per use of its buffer
-// and no wait is ever two phases behind (a buffer is reused only after its waiter moved on).
+// Barriers of one head: s_full completes once per tile (scores ready), p_full[x] and
+// pv_done[x] once per tile for key half x (P written; its O += P V done).  Parity waits
+// need the waiter at most one phase behind; each wait below states why it is.
 struct TcHeadBars {
-  uint64_t s_full[2];          // MMA commit: S buffer i holds the scores
-  uint64_t s_free[2];          // 128 arrivals: S buffer i read
-  uint64_t p_full[kTcPBufs];   // 128 arrivals: P buffer u written (and O rescaled)
-  uint64_t pv_done[kTcPBufs];  // MMA commit: O += P_u V done (buffer free; O stable then)
+  uint64_t s_full;
+  uint64_t p_full[2];
+  uint64_t pv_done[2];
 };
+struct TcBars {
+  uint64_t k_full[kTcKSlots], k_empty[kTcKSlots];
+  uint64_t v_full[kTcVSlots], v_empty[kTcVSlots];
+  uint64_t q_ready;
+  TcHeadBars h[kTcHeads];
+  uint32_t tmem;
+  int abort;
+};
+static_assert(sizeof(TcBars) <= 256, "tcgen05 prefill barrier block");
+
+// Key tile t of a CTA: the first n_ct tiles cover the nc retained rows, the rest the band
+// [bs, jmax] of dense rows.
+struct TcTile {
+  bool retained;
+  int r0, rows;
+};
+__device__ __forceinline__ TcTile tc_tile(int t, int n_ct, int nc, int bs, int jmax) {
+  TcTile x;
+  x.retained = t < n_ct;
+  x.r0 = x.retained ? t * kTcKeys : bs + (t - n_ct) * kTcKeys;
+  x.rows = min(kTcKeys, (x.retained ? nc : jmax + 1) - x.r0);
+  return x;
+}
+
+// Rows [r0, r0 + rows) of one head's packed K or V (two d-halves) into a 128-row tile.
+__device__ __forceinline__ void tc_stage_rows(uint8_t* dst, const uint8_t* src, int64_t head,
+                                              int P, int r0, int rows, uint64_t* bar) {
+  const uint32_t bytes = (uint32_t)rows * 128u;
+#pragma unroll
+  for (int dh = 0; dh < 2; ++dh)
+    bulk_copy_g2s(dst + dh * kTcHalfBytes, src + ((head * 2 + dh) * P + r0) * 128, bytes, bar);
+}
 
 __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const PrefillParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kTcOffBar);
-  uint64_t* empty_bar = full_bar + kTcStages;
-  uint64_t* q_ready = empty_bar + kTcStages;
-  TcHeadBars* hb = reinterpret_cast<TcHeadBars*>(q_ready + 1);
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(hb + kTcHeads);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(s_tmem + 1);
+  TcBars& bars = *reinterpret_cast<TcBars*>(smem + kTcOffBar);
+  volatile int* abort_flag = &bars.abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = p.group, Hq = p.kv_heads * G;
@@ -530,119 +558,146 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
   const int jmax = min(j0 + kPfRows, P) - 1;
   const int nc = (jmax - w > 0) ? p.before[head * (P + 1) + (jmax - w)] : 0;
   const int bs = max(0, j0 - w) & ~7;
-  const int n_ct = (nc + kPfKeys - 1) / kPfKeys;
-  const int n_tiles = n_ct + (jmax + 1 - bs + kPfKeys - 1) / kPfKeys;
+  const int n_ct = (nc + kTcKeys - 1) / kTcKeys;
+  const int n_tiles = n_ct + (jmax + 1 - bs + kTcKeys - 1) / kTcKeys;
 
   if (tid == 0) {
     *abort_flag = 0;
-    for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(&full_bar[s], 1);
-      mbar_init(&empty_bar[s], 1);
+    for (int s = 0; s < kTcKSlots; ++s) {
+      mbar_init(&bars.k_full[s], 1);
+      mbar_init(&bars.k_empty[s], 1);
     }
-    mbar_init(q_ready, kPfRows * nh);
+    for (int s = 0; s < kTcVSlots; ++s) {
+      mbar_init(&bars.v_full[s], 1);
+      mbar_init(&bars.v_empty[s], 1);
+    }
+    mbar_init(&bars.q_ready, kPfRows * nh);
     for (int h = 0; h < kTcHeads; ++h) {
-      for (int i = 0; i < 2; ++i) {
-        mbar_init(&hb[h].s_full[i], 1);
-        mbar_init(&hb[h].s_free[i], kPfRows);
-      }
-      for (int u = 0; u < kTcPBufs; ++u) {
-        mbar_init(&hb[h].p_full[u], kPfRows);
-        mbar_init(&hb[h].pv_done[u], 1);
+      mbar_init(&bars.h[h].s_full, 1);
+      for (int x = 0; x < 2; ++x) {
+        mbar_init(&bars.h[h].p_full[x], kPfRows);
+        mbar_init(&bars.h[h].pv_done[x], 1);
       }
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 2) {
-    tmem_alloc(s_tmem, kTcCols);
+    tmem_alloc(&bars.tmem, kTcCols);
     tc_fence_before();
   }
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *s_tmem;
+  const uint32_t tmem = bars.tmem;
 
   if (warp == 0) {
     // ================================================================ producer
-    if (lane == 0) {
-      for (int t = 0; t < n_tiles; ++t) {
-        const int s = t % kTcStages, use = t / kTcStages;
-        if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.err);
-        uint8_t* st = smem + s * kTcStageBytes;
-        if (t < n_ct) {
-          const int r0 = t * kPfKeys, rows = min(kPfKeys, nc - r0);
-          mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes + kPfKeys * 4);
-          stage_tile(st, p.kc, p.vc, head, P, r0, rows, &full_bar[s]);
-          bulk_copy_g2s(smem + kTcOffPos + s * kPfKeys * 4, p.pc + head * pc_stride(P) + r0,
-                        kPfKeys * 4, &full_bar[s]);
-        } else {
-          const int r0 = bs + (t - n_ct) * kPfKeys, rows = min(kPfKeys, jmax + 1 - r0);
-          mbar_arrive_expect_tx(&full_bar[s], 2 * (uint32_t)rows * kRowBytes);
-          stage_tile(st, p.kd, p.vd, head, P, r0, rows, &full_bar[s]);
-        }
+    // The whole warp waits and zeroes stale V rows; lane 0 issues the copies.  A slot is
+    // refilled only after the MMAs that read its previous tile are done (empty barriers).
+    for (int t = 0; t < n_tiles; ++t) {
+      const TcTile x = tc_tile(t, n_ct, nc, bs, jmax);
+      const int ks = t % kTcKSlots, vs = t % kTcVSlots;
+      if (t >= kTcKSlots) mbar_wait(&bars.k_empty[ks], (t / kTcKSlots - 1) & 1, abort_flag, p.err);
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars.k_full[ks], 2u * (uint32_t)x.rows * 128u);
+        tc_stage_rows(smem + ks * kTcTileBytes, x.retained ? p.kc : p.kd, head, P, x.r0, x.rows,
+                      &bars.k_full[ks]);
       }
-      for (int s = 0; s < kTcStages && s < n_tiles; ++s) {
-        const int last_t = s + ((n_tiles - 1 - s) / kTcStages) * kTcStages;
-        mbar_wait(&full_bar[s], (last_t / kTcStages) & 1, abort_flag, p.err);
+      if (t >= kTcVSlots) mbar_wait(&bars.v_empty[vs], (t / kTcVSlots - 1) & 1, abort_flag, p.err);
+      uint8_t* vt = smem + kTcOffV + vs * kTcTileBytes;
+      if (x.rows < kTcKeys) {
+        const int n16 = (kTcKeys - x.rows) * 8;  // 16-byte words past the rows, per d-half
+        for (int e = lane; e < 2 * n16; e += 32) {
+          const int dh = e >= n16 ? 1 : 0;
+          *reinterpret_cast<uint4*>(vt + dh * kTcHalfBytes + x.rows * 128 + (e - dh * n16) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();  // visible to the tensor cores via the full barrier
+        __syncwarp();
+      }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars.v_full[vs], 2u * (uint32_t)x.rows * 128u);
+        tc_stage_rows(vt, x.retained ? p.vc : p.vd, head, P, x.r0, x.rows, &bars.v_full[vs]);
+      }
+    }
+    // no copy may still be in flight when the CTA exits (matters only after a timeout)
+    if (lane == 0) {
+      for (int s = 0; s < kTcKSlots && s < n_tiles; ++s) {
+        const int last = s + ((n_tiles - 1 - s) / kTcKSlots) * kTcKSlots;
+        mbar_wait(&bars.k_full[s], (last / kTcKSlots) & 1, abort_flag, p.err);
+      }
+      for (int s = 0; s < kTcVSlots && s < n_tiles; ++s) {
+        const int last = s + ((n_tiles - 1 - s) / kTcVSlots) * kTcVSlots;
+        mbar_wait(&bars.v_full[s], (last / kTcVSlots) & 1, abort_flag, p.err);
       }
     }
   } else if (warp == 1) {
     // ================================================================ MMA issuer
+    // Order per tile t: for each head h, O_h += P_h(t) V(t) by halves, then S_h(t + 1).
+    // The thread is the only waiter on k_full / v_full / p_full and consumes them in order.
     if (lane == 0) {
-      constexpr uint32_t idesc_s = f16_idesc(kPfRows, kPfKeys, 0);    // Q K^T: both K-major
+      constexpr uint32_t idesc_s = f16_idesc(kPfRows, kTcKeys, 0);    // Q K^T: both K-major
       constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
-      // Descriptors are built once; the start address (16-byte units, low bits) is stepped:
-      // +2 per 16 head_dim elements of Q / K inside a d-half, + half size at kk = 4;
-      // +2 per 16 keys of P; +128 (2 KiB) per 16 keys of V.
+      // Descriptors are built once and their start address (16-byte units) stepped: +2 per
+      // 16 head_dim elements of Q / K inside a d-half, + the d-half size at k-step 4; +128
+      // (2 KiB) per 16 keys of V, whose two d-halves are the leading-offset atoms.
       const uint64_t dq0 = sw128_desc(smem_addr(smem + kTcOffQ), 16u, 1024u);
-      const uint64_t dp0 = sw128_desc(smem_addr(smem + kTcOffP), 16u, 1024u);
       const uint64_t dk0 = sw128_desc(smem_addr(smem), 16u, 1024u);
-      const uint64_t dv0 = sw128_desc(smem_addr(smem) + kPfTileBytes, kPfKeys * 128u, 1024u);
+      const uint64_t dv0 = sw128_desc(smem_addr(smem + kTcOffV), (uint32_t)kTcHalfBytes, 1024u);
       constexpr uint64_t kQHead = kTcQBytes >> 4, kQHalf = (kPfRows * 128) >> 4;
-      constexpr uint64_t kKHalf = (kPfKeys * 128) >> 4, kStage = kTcStageBytes >> 4;
-      constexpr uint64_t kPBuf = kTcPBytes >> 4;
-      mbar_wait(q_ready, 0, abort_flag, p.err);
-      auto issue_scores = [&](int t) {
-        const int s = t % kTcStages, i = t & 1;
-        mbar_wait(&full_bar[s], (t / kTcStages) & 1, abort_flag, p.err);
-        for (int h = 0; h < nh; ++h)
-          if (t >= 2) mbar_wait(&hb[h].s_free[i], ((t - 2) >> 1) & 1, abort_flag, p.err);
-        tc_fence_after();
-        const uint64_t dk = dk0 + (uint64_t)s * kStage;
-        for (int h = 0; h < nh; ++h) {
-          const uint64_t dq = dq0 + (uint64_t)h * kQHead;
-          const uint32_t d_s = tmem + (uint32_t)(256 * h + 128 + 64 * i);
-          tc_mma_ss_k<false>(d_s, dq, dk, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + 2, dk + 2, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + 4, dk + 4, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + 6, dk + 6, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + kQHalf, dk + kKHalf, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + kQHalf + 2, dk + kKHalf + 2, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + kQHalf + 4, dk + kKHalf + 4, idesc_s);
-          tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
-          tc_commit(&hb[h].s_full[i]);
-        }
+      constexpr uint64_t kKHalf = kTcHalfBytes >> 4, kSlot = kTcTileBytes >> 4;
+      auto issue_scores = [&](int h, int t) {
+        const uint64_t dq = dq0 + (uint64_t)h * kQHead;
+        const uint64_t dk = dk0 + (uint64_t)(t % kTcKSlots) * kSlot;
+        const uint32_t d_s = tmem + (uint32_t)(256 * h + 128);
+        tc_mma_ss_k<false>(d_s, dq, dk, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + 2, dk + 2, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + 4, dk + 4, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + 6, dk + 6, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + kQHalf, dk + kKHalf, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + kQHalf + 2, dk + kKHalf + 2, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + kQHalf + 4, dk + kKHalf + 4, idesc_s);
+        tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
+        tc_commit(&bars.h[h].s_full);
       };
-      if (n_tiles > 0) issue_scores(0);
+      mbar_wait(&bars.q_ready, 0, abort_flag, p.err);
+      mbar_wait(&bars.k_full[0], 0, abort_flag, p.err);
+      tc_fence_after();
+      for (int h = 0; h < nh; ++h) issue_scores(h, 0);
+      tc_commit(&bars.k_empty[0]);
       for (int t = 0; t < n_tiles; ++t) {
-        if (t + 1 < n_tiles) issue_scores(t + 1);
-        const int s = t % kTcStages, u = t % kTcPBufs;
-        const uint64_t dv = dv0 + (uint64_t)s * kStage;
+        const int vs = t % kTcVSlots;
+        const bool more = t + 1 < n_tiles;
+        mbar_wait(&bars.v_full[vs], (t / kTcVSlots) & 1, abort_flag, p.err);
+        const uint64_t dv = dv0 + (uint64_t)vs * kSlot;
         for (int h = 0; h < nh; ++h) {
-          mbar_wait(&hb[h].p_full[u], (t / kTcPBufs) & 1, abort_flag, p.err);
-          tc_fence_after();
-          // keys 16 kk .. 16 kk + 15; V atoms along head_dim are the two d-halves (leading
-          // offset 8 KiB), 8-key groups 1 KiB apart
-          const uint64_t dp = dp0 + (uint64_t)(kTcPBufs * h + u) * kPBuf;
+          TcHeadBars& hb = bars.h[h];
           const uint32_t d_o = tmem + (uint32_t)(256 * h);
-          if (t == 0)
-            tc_mma_ss_k<false>(d_o, dp, dv, idesc_o);
-          else
-            tc_mma_ss_k<true>(d_o, dp, dv, idesc_o);
-          tc_mma_ss_k<true>(d_o, dp + 2, dv + 128, idesc_o);
-          tc_mma_ss_k<true>(d_o, dp + 4, dv + 256, idesc_o);
-          tc_mma_ss_k<true>(d_o, dp + 6, dv + 384, idesc_o);
-          tc_commit(&hb[h].pv_done[u]);
+          for (int x = 0; x < 2; ++x) {
+            // P_h(t) half x (keys 64 x ..): packed columns 32 x .., V rows 64 x ..
+            mbar_wait(&hb.p_full[x], t & 1, abort_flag, p.err);
+            tc_fence_after();
+            const uint32_t a = tmem + (uint32_t)(256 * h + 128 + 32 * x);
+            const uint64_t bv = dv + (uint64_t)(512 * x);
+            if (t == 0 && x == 0)
+              tc_mma_ts_k<false>(d_o, a, bv, idesc_o);
+            else
+              tc_mma_ts_k<true>(d_o, a, bv, idesc_o);
+            tc_mma_ts_k<true>(d_o, a + 8, bv + 128, idesc_o);
+            tc_mma_ts_k<true>(d_o, a + 16, bv + 256, idesc_o);
+            tc_mma_ts_k<true>(d_o, a + 24, bv + 384, idesc_o);
+            tc_commit(&hb.pv_done[x]);
+          }
+          if (more) {
+            if (h == 0) {
+              mbar_wait(&bars.k_full[(t + 1) % kTcKSlots], ((t + 1) / kTcKSlots) & 1, abort_flag,
+                        p.err);
+              tc_fence_after();
+            }
+            issue_scores(h, t + 1);
+          }
         }
-        tc_commit(&empty_bar[s]);  // the stage is free once every product on it is done
+        tc_commit(&bars.v_empty[vs]);  // a slot is free once every product on it is done
+        if (more) tc_commit(&bars.k_empty[(t + 1) % kTcKSlots]);
       }
     }
   } else if (warp >= 4 && (warp - 4) / 4 < nh) {
@@ -651,9 +706,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     const int row = tid - 128 * (1 + h);  // query row of the tile = TMEM lane
     const int j = j0 + row;
     const int hq = hq0 + h;
-    const uint32_t lane_addr = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
-    const uint32_t o_col = (uint32_t)(256 * h);
-    TcHeadBars& bar = hb[h];
+    const uint32_t o_addr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(256 * h);
+    const uint32_t s_addr = o_addr + 128u;
+    TcHeadBars& hb = bars.h[h];
     uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;
     // this row of Q into the K-major swizzled layout [d-half][row][128 B]
     {
@@ -668,132 +723,103 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
                                   chunk_in_row(row, c & 7)) = val;
       }
       fence_proxy_async_smem();
-      mbar_arrive(q_ready);
+      mbar_arrive(&bars.q_ready);
     }
-    float m = -INFINITY, l = 0.f;  // reference max and running sum of this row
+    // the retained keys of this row: the first bj compacted rows
+    const int bj = j - w > 0 ? p.before[head * (P + 1) + min(j - w, P)] : 0;
+    const float scale = p.scale_log2;
+    float m = -INFINITY, l = 0.f;  // reference max (log2 domain) and running sum of the row
     for (int t = 0; t < n_tiles; ++t) {
-      const int s = t % kTcStages, i = t & 1;
-      const bool retained = t < n_ct;
-      const int r0 = retained ? t * kPfKeys : bs + (t - n_ct) * kPfKeys;
-      const int rows = retained ? min(kPfKeys, nc - r0) : min(kPfKeys, jmax + 1 - r0);
-      const int u = t % kTcPBufs;
-      uint8_t* sp = smem + kTcOffP + (kTcPBufs * h + u) * kTcPBytes;
-      mbar_wait(&full_bar[s], (t / kTcStages) & 1, abort_flag, p.err);
-      if (rows < kPfKeys && h == 0) {
-        // V rows past the tile's keys hold stale bytes, possibly NaN patterns; P is 0
-        // there, but 0 * NaN is not: zero them before any P V reads the tile (ordered for
-        // the tensor cores by the proxy fence before the P-ready arrival).
-        uint8_t* vt = smem + s * kTcStageBytes + kPfTileBytes;
-        for (int e = row; e < (kPfKeys - rows) * 16; e += kPfRows)
-          *reinterpret_cast<uint4*>(vt + tile_off((uint32_t)(rows + e / 16), (uint32_t)(e & 15))) =
-              make_uint4(0u, 0u, 0u, 0u);
+      const TcTile x = tc_tile(t, n_ct, nc, bs, jmax);
+      int lo, nvis;  // visible keys of the tile: lo .. lo + nvis - 1
+      if (x.retained) {
+        lo = 0;
+        nvis = min(max(bj - x.r0, 0), x.rows);
+      } else {
+        lo = max(j - w - x.r0, 0);
+        nvis = max(min(j - x.r0, x.rows - 1) - lo + 1, 0);
       }
-      mbar_wait(&bar.s_full[i], (t >> 1) & 1, abort_flag, p.err);
+      // S(t) is issued after P(t - 1) is read, so this wait is at most one phase behind;
+      // its commit also covers every earlier product, so P(t - 1) is free to overwrite
+      mbar_wait(&hb.s_full, t & 1, abort_flag, p.err);
       tc_fence_after();
-      // the row of S: four loads in flight, one wait
-      float sc[kPfKeys];
-      {
-        const uint32_t sa = lane_addr + (uint32_t)(256 * h + 128 + 64 * i);
+#pragma unroll 1
+      for (int half = 0; half < 2; ++half) {
+        float sc[64];
+        const uint32_t sa = s_addr + (uint32_t)(64 * half);
         tmem_ld16_at(sa, sc);
         tmem_ld16_at(sa + 16, sc + 16);
         tmem_ld16_at(sa + 32, sc + 32);
         tmem_ld16_at(sa + 48, sc + 48);
         tmem_wait_ld();
-      }
-      tc_fence_before();
-      mbar_arrive(&bar.s_free[i]);
-      // mask: skipped when every key of the tile is visible to every query of the CTA
-      const int32_t* spos = reinterpret_cast<const int32_t*>(smem + kTcOffPos + s * kPfKeys * 4);
-      const bool all_visible =
-          rows == kPfKeys && (retained ? spos[kPfKeys - 1] < j0 - w
-                                       : (r0 >= jmax - w && r0 + kPfKeys - 1 <= j0));
-      if (all_visible) {
+        const int key0 = 64 * half;
+        if (!__all_sync(0xffffffffu, lo <= key0 && key0 + 64 <= lo + nvis)) {
 #pragma unroll
-        for (int k = 0; k < kPfKeys; ++k) sc[k] *= p.scale_log2;
-      } else {
-#pragma unroll
-        for (int k = 0; k < kPfKeys; ++k) {
-          const bool valid = k < rows;
-          const int pos = retained ? (valid ? spos[k] : 0) : r0 + k;
-          const bool vis = valid && (retained ? pos < j - w : (pos >= j - w && pos <= j));
-          sc[k] = vis ? sc[k] * p.scale_log2 : -INFINITY;
+          for (int k = 0; k < 64; ++k)
+            if ((unsigned)(key0 + k - lo) >= (unsigned)nvis) sc[k] = -INFINITY;
         }
-      }
-      // row max over eight independent chains
-      float mx8[8];
+        float mx8[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) mx8[e] = sc[e];
+        for (int e = 0; e < 8; ++e) mx8[e] = sc[e];
 #pragma unroll
-      for (int k = 8; k < kPfKeys; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], sc[k]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-      // P buffer u is in use until the product of tile t - kTcPBufs is done
-      if (t >= kTcPBufs) {
-        mbar_wait(&bar.pv_done[u], ((t - kTcPBufs) / kTcPBufs) & 1, abort_flag, p.err);
-        tc_fence_after();
-      }
-      float corr = 1.f;
-      if (mx > m + kTcRescale || (m == -INFINITY && mx > -INFINITY)) {
-        const float mn = mx;
-        corr = exp2f(m - mn);  // 0 when m = -inf
-        m = mn;
-      }
-      const bool rescale = t > 0 && __any_sync(0xffffffffu, corr != 1.f);
-      if (rescale && kTcPBufs > 1) {
-        // O must hold every earlier product first: wait for the one of tile t - 1
-        mbar_wait(&bar.pv_done[(t - 1) % kTcPBufs], ((t - 1) / kTcPBufs) & 1, abort_flag, p.err);
-        tc_fence_after();
-      }
-      if (rescale) {
-        // (rare: only when a row's max grew past the threshold; 16 columns at a time, the
-        // scores of the tile stay in registers meanwhile)
+        for (int k = 8; k < 64; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], sc[k]);
+        const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        const float mx_s = mx * scale;
+        // O += P V of this half of tile t - 1: done already (the S(t) commit covers it);
+        // waiting keeps pv_done[half] at most one phase ahead of this thread
+        if (t > 0) mbar_wait(&hb.pv_done[half], (t - 1) & 1, abort_flag, p.err);
+        float corr = 1.f;
+        if (mx_s > m + kTcRescale) {
+          corr = ex2_approx(m - mx_s);  // 0 when m = -inf
+          m = mx_s;
+        }
+        if ((t > 0 || half > 0) && __any_sync(0xffffffffu, corr != 1.f)) {
+          // (rare) O must hold the previous half's product: that of (t, 0) or (t - 1, 1)
+          mbar_wait(&hb.pv_done[half ^ 1], (half ? t : t - 1) & 1, abort_flag, p.err);
+          tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < kHeadDim / 16; ++c) {
-          float r[16];
-          tmem_ld16(lane_addr + o_col + (uint32_t)(16 * c), r);
-          tmem_wait_ld();
+          for (int c = 0; c < kHeadDim / 16; ++c) {
+            float r[16];
+            tmem_ld16(o_addr + (uint32_t)(16 * c), r);
+            tmem_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 16; ++e) r[e] *= corr;
-          tmem_st16(lane_addr + o_col + (uint32_t)(16 * c), r);
+            for (int e = 0; e < 16; ++e) r[e] *= corr;
+            tmem_st16(o_addr + (uint32_t)(16 * c), r);
+          }
+          tmem_wait_st();
         }
+        const float nb = m == -INFINITY ? 0.f : -m;
+        uint32_t pk[32];
+        float s8[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) s8[e] = 0.f;
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const float p0 = ex2_approx(fmaf(sc[2 * c], scale, nb));
+          const float p1 = ex2_approx(fmaf(sc[2 * c + 1], scale, nb));
+          s8[c & 7] += p0 + p1;
+          pk[c] = pack_bf16x2(p0, p1);
+        }
+        tmem_st16_u32(s_addr + (uint32_t)(32 * half), pk);
+        tmem_st16_u32(s_addr + (uint32_t)(32 * half + 16), pk + 16);
         tmem_wait_st();
+        l = l * corr + (((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7])));
+        tc_fence_before();
+        mbar_arrive(&hb.p_full[half]);
       }
-      const float base = m == -INFINITY ? 0.f : m;
-      float sum8[8];  // eight independent partial sums (chunk c)
-      // P row: 64 bf16 = 8 chunks of 16 bytes, chunk c at (c ^ (row & 7))
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint32_t pk[4];
-        float sc_sum = 0.f;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float p0 = exp2f(sc[8 * c + 2 * e] - base), p1 = exp2f(sc[8 * c + 2 * e + 1] - base);
-          sc_sum += p0 + p1;
-          pk[e] = pack_bf16x2(p0, p1);
-        }
-        sum8[c] = sc_sum;
-        *reinterpret_cast<uint4*>(sp + row * 128 + chunk_in_row(row, c)) =
-            make_uint4(pk[0], pk[1], pk[2], pk[3]);
-      }
-      const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) +
-                        ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
-      l = l * corr + sum;
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(&bar.p_full[u]);
     }
-    // normalise and store this row (the last product completes after all earlier ones)
-    if (n_tiles > 0) {
-      mbar_wait(&bar.pv_done[(n_tiles - 1) % kTcPBufs], ((n_tiles - 1) / kTcPBufs) & 1, abort_flag,
-                p.err);
-      tc_fence_after();
-    }
+    // normalise and store this row once both halves of the last product are done (each wait
+    // is at most one phase behind: the products of tile n - 2 were awaited above)
+    mbar_wait(&hb.pv_done[0], (n_tiles - 1) & 1, abort_flag, p.err);
+    mbar_wait(&hb.pv_done[1], (n_tiles - 1) & 1, abort_flag, p.err);
+    tc_fence_after();
     const float inv = l > 0.f ? 1.f / l : 0.f;
     __nv_bfloat16* orow = p.out + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
 #pragma unroll
     for (int c = 0; c < kHeadDim / 16; ++c) {
       float r[16];
-      tmem_ld16(lane_addr + o_col + (uint32_t)(16 * c), r);
+      tmem_ld16(o_addr + (uint32_t)(16 * c), r);
       tmem_wait_ld();
       if (j < P) {
         uint4 v0, v1;
