@@ -25,9 +25,11 @@
 // from the S accumulators as the A operand.  Each warp stages its queries in shared memory
 // once and reloads their fragments with ldmatrix per tile (nine warps leave ~168
 // registers per thread; holding Q in registers would spill).
+#include <cuda.h>  // tensor-map types only; the encoder is reached through the runtime
 #include <math.h>
 
 #include <atomic>
+#include <mutex>
 
 #include "dms_internal.cuh"
 #include "dms_ptx.cuh"
@@ -452,7 +454,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // ============================================================================ tcgen05 kernel
 // The same attention on the 5th-generation tensor cores.  One CTA per (KV head, 128-query
 // tile, pair of query heads of the group): both heads attend to the same keys, so every
-// staged K / V tile serves two score tiles.  Key tiles hold 128 keys, so every MMA is
+// staged K / V tile serves two score tiles.  Q arrives and O leaves by tensor-map copies
+// (TMA, 128-byte swizzle: the tile lands in the MMA operand layout; O is staged in its
+// head's Q buffer, free once the last product is done).  Key tiles hold 128 keys, so every MMA is
 // M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the time of an N 128
 // one for half its work).  384 threads: warp 0 stages K tiles (3-slot ring) and V tiles
 // (2-slot ring) with bulk copies, warp 1 issues the MMAs from one thread, warp 2 owns the
@@ -504,12 +508,19 @@ struct TcHeadBars {
 struct TcBars {
   uint64_t k_full[kTcKSlots], k_empty[kTcKSlots];
   uint64_t v_full[kTcVSlots], v_empty[kTcVSlots];
-  uint64_t q_ready;
+  uint64_t q_full;   // the CTA's Q tiles landed
+  uint64_t q_ready;  // ... and patched (borrowed decisions only)
   TcHeadBars h[kTcHeads];
   uint32_t tmem;
   int abort;
 };
 static_assert(sizeof(TcBars) <= 256, "tcgen05 prefill barrier block");
+
+// Tensor maps of q and out, both [B][P][Hq * 128] bf16 (innermost first: Hq * 128, P, B),
+// box 64 x 128 x 1 (one d-half of 128 query rows of one head), 128-byte swizzle.
+struct TcMaps {
+  CUtensorMap q, out;
+};
 
 // Key tile t of a CTA: the first n_ct tiles cover the nc retained rows, the rest the band
 // [bs, jmax] of dense rows.
@@ -534,7 +545,8 @@ __device__ __forceinline__ void tc_stage_rows(uint8_t* dst, const uint8_t* src, 
     bulk_copy_g2s(dst + dh * kTcHalfBytes, src + ((head * 2 + dh) * P + r0) * 128, bytes, bar);
 }
 
-__global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const PrefillParams p) {
+__global__ void __launch_bounds__(kTcThreads, 1)
+    prefill_tc_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ TcMaps maps) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -542,7 +554,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
   volatile int* abort_flag = &bars.abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int G = p.group, Hq = p.kv_heads * G;
+  const int G = p.group;
   const int pairs = (G + kTcHeads - 1) / kTcHeads;
   const int n_units = p.n_qheads / G * pairs;  // (sequence, KV head, head pair)
   const int tile_rank = blockIdx.x / n_units;
@@ -571,6 +583,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
       mbar_init(&bars.v_full[s], 1);
       mbar_init(&bars.v_empty[s], 1);
     }
+    mbar_init(&bars.q_full, 1);
     mbar_init(&bars.q_ready, kPfRows * nh);
     for (int h = 0; h < kTcHeads; ++h) {
       mbar_init(&bars.h[h].s_full, 1);
@@ -593,6 +606,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     // ================================================================ producer
     // The whole warp waits and zeroes stale V rows; lane 0 issues the copies.  A slot is
     // refilled only after the MMAs that read its previous tile are done (empty barriers).
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&bars.q_full, (uint32_t)(nh * kTcQBytes));
+      for (int h = 0; h < nh; ++h)
+        for (int dh = 0; dh < 2; ++dh)
+          tma_load_3d(smem + kTcOffQ + h * kTcQBytes + dh * (kPfRows * 128), &maps.q,
+                      (hq0 + h) * kHeadDim + 64 * dh, j0, b, &bars.q_full);
+    }
     for (int t = 0; t < n_tiles; ++t) {
       const TcTile x = tc_tile(t, n_ct, nc, bs, jmax);
       const int ks = t % kTcKSlots, vs = t % kTcVSlots;
@@ -621,6 +641,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     }
     // no copy may still be in flight when the CTA exits (matters only after a timeout)
     if (lane == 0) {
+      mbar_wait(&bars.q_full, 0, abort_flag, p.err);
       for (int s = 0; s < kTcKSlots && s < n_tiles; ++s) {
         const int last = s + ((n_tiles - 1 - s) / kTcKSlots) * kTcKSlots;
         mbar_wait(&bars.k_full[s], (last / kTcKSlots) & 1, abort_flag, p.err);
@@ -659,7 +680,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
         tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
         tc_commit(&bars.h[h].s_full);
       };
-      mbar_wait(&bars.q_ready, 0, abort_flag, p.err);
+      mbar_wait(p.zero_first ? &bars.q_ready : &bars.q_full, 0, abort_flag, p.err);
       mbar_wait(&bars.k_full[0], 0, abort_flag, p.err);
       tc_fence_after();
       for (int h = 0; h < nh; ++h) issue_scores(h, 0);
@@ -709,19 +730,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
     const uint32_t o_addr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(256 * h);
     const uint32_t s_addr = o_addr + 128u;
     TcHeadBars& hb = bars.h[h];
-    uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;
-    // this row of Q into the K-major swizzled layout [d-half][row][128 B]
-    {
-      const bool zero = p.zero_first && hq % G == 0;
-      const __nv_bfloat16* qrow = p.q + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        uint4 val = make_uint4(0u, 0u, 0u, 0u);
-        if (j < P) val = *reinterpret_cast<const uint4*>(qrow + c * 8);
-        if (zero && c == 0) val.x &= 0xffff0000u;  // App. B: the decision element
-        *reinterpret_cast<uint4*>(sq + (c >> 3) * (kPfRows * 128) + row * 128 +
-                                  chunk_in_row(row, c & 7)) = val;
-      }
+    uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;  // [d-half][row][128 B], swizzled
+    if (p.zero_first) {
+      // App. B: the decision element (head_dim 0 of the group's first head) is not a query
+      // feature; zero it in the landed tile before any score reads it
+      mbar_wait(&bars.q_full, 0, abort_flag, p.err);
+      if (hq % G == 0) *reinterpret_cast<uint16_t*>(sq + row * 128 + chunk_in_row(row, 0)) = 0;
       fence_proxy_async_smem();
       mbar_arrive(&bars.q_ready);
     }
@@ -809,31 +823,43 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
         mbar_arrive(&hb.p_full[half]);
       }
     }
-    // normalise and store this row once both halves of the last product are done (each wait
-    // is at most one phase behind: the products of tile n - 2 were awaited above)
+    // normalise this row once both halves of the last product are done (each wait is at
+    // most one phase behind: the products of tile n - 2 were awaited above); every MMA of
+    // this head is then done, so its Q buffer takes the bf16 row of O for the store
     mbar_wait(&hb.pv_done[0], (n_tiles - 1) & 1, abort_flag, p.err);
     mbar_wait(&hb.pv_done[1], (n_tiles - 1) & 1, abort_flag, p.err);
     tc_fence_after();
     const float inv = l > 0.f ? 1.f / l : 0.f;
-    __nv_bfloat16* orow = p.out + (((int64_t)b * P + j) * Hq + hq) * kHeadDim;
 #pragma unroll
     for (int c = 0; c < kHeadDim / 16; ++c) {
       float r[16];
       tmem_ld16(o_addr + (uint32_t)(16 * c), r);
       tmem_wait_ld();
-      if (j < P) {
-        uint4 v0, v1;
-        v0.x = pack_bf16x2(r[0] * inv, r[1] * inv);
-        v0.y = pack_bf16x2(r[2] * inv, r[3] * inv);
-        v0.z = pack_bf16x2(r[4] * inv, r[5] * inv);
-        v0.w = pack_bf16x2(r[6] * inv, r[7] * inv);
-        v1.x = pack_bf16x2(r[8] * inv, r[9] * inv);
-        v1.y = pack_bf16x2(r[10] * inv, r[11] * inv);
-        v1.z = pack_bf16x2(r[12] * inv, r[13] * inv);
-        v1.w = pack_bf16x2(r[14] * inv, r[15] * inv);
-        *reinterpret_cast<uint4*>(orow + 16 * c) = v0;
-        *reinterpret_cast<uint4*>(orow + 16 * c + 8) = v1;
-      }
+      uint4 v0, v1;
+      v0.x = pack_bf16x2(r[0] * inv, r[1] * inv);
+      v0.y = pack_bf16x2(r[2] * inv, r[3] * inv);
+      v0.z = pack_bf16x2(r[4] * inv, r[5] * inv);
+      v0.w = pack_bf16x2(r[6] * inv, r[7] * inv);
+      v1.x = pack_bf16x2(r[8] * inv, r[9] * inv);
+      v1.y = pack_bf16x2(r[10] * inv, r[11] * inv);
+      v1.z = pack_bf16x2(r[12] * inv, r[13] * inv);
+      v1.w = pack_bf16x2(r[14] * inv, r[15] * inv);
+      // logical chunks 2c, 2c + 1 (head_dim 16c .. 16c + 15) of d-half c / 4
+      uint8_t* half_row = sq + (c >> 2) * (kPfRows * 128) + row * 128;
+      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, (2 * c) & 7)) = v0;
+      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, (2 * c + 1) & 7)) = v1;
+    }
+    fence_proxy_async_smem();
+    if (h == 0)
+      named_barrier_sync<1>(kPfRows);
+    else
+      named_barrier_sync<2>(kPfRows);
+    if (row == 0) {
+      // rows past the prompt fall outside the tensor map and are not written
+      tma_store_3d(&maps.out, hq * kHeadDim, j0, b, sq);
+      tma_store_3d(&maps.out, hq * kHeadDim + 64, j0, b, sq + kPfRows * 128);
+      bulk_commit_group();
+      bulk_wait_group_read0();
     }
   }
   // ---- teardown: every tensor-memory access is done before the columns are released
@@ -846,6 +872,38 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kernel(const Prefill
 }
 
 }  // namespace
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link to the driver).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+  });
+  return fn;
+}
+
+// [B][P][Hq * 128] bf16 tensor map with a box of one d-half of 128 rows of one head.
+bool encode_qo_map(CUtensorMap* map, const void* base, int64_t batch, int64_t P, int64_t hq) {
+  const EncodeTiledFn fn = encode_tiled_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)(hq * kHeadDim), (cuuint64_t)P, (cuuint64_t)batch};
+  const cuuint64_t strides[2] = {(cuuint64_t)(hq * kRowBytes), (cuuint64_t)(P * hq * kRowBytes)};
+  const cuuint32_t box[3] = {64u, (cuuint32_t)kPfRows, 1u};
+  const cuuint32_t estr[3] = {1u, 1u, 1u};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3u, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 size_t prefill_workspace_bytes(int64_t heads, int64_t n_tokens) {
   return pf_layout(heads, n_tokens).total;
@@ -919,8 +977,13 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
   if (kernel == DMS_PREFILL_MMA_SYNC) {
     prefill_attn_kernel<<<(unsigned)grid, kPfThreads, kPfSmemBytes, stream>>>(pp);
   } else {
+    TcMaps maps;
+    if (!encode_qo_map(&maps.q, q, batch, n_tokens, pp.n_qheads / batch) ||
+        !encode_qo_map(&maps.out, out, batch, n_tokens, pp.n_qheads / batch))
+      return cudaErrorInvalidValue;
     const int64_t units = H * ((group + kTcHeads - 1) / kTcHeads);
-    prefill_tc_kernel<<<(unsigned)(pp.n_qtiles * units), kTcThreads, kTcSmemBytes, stream>>>(pp);
+    prefill_tc_kernel<<<(unsigned)(pp.n_qtiles * units), kTcThreads, kTcSmemBytes, stream>>>(pp,
+                                                                                              maps);
   }
   return cudaGetLastError();
 }
