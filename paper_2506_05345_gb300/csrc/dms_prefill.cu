@@ -456,23 +456,25 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // tile, pair of query heads of the group): both heads attend to the same keys, so every
 // staged K / V tile serves two score tiles.  Q arrives and O leaves by tensor-map copies
 // (TMA, 128-byte swizzle: the tile lands in the MMA operand layout; O is staged in its
-// head's Q buffer, free once the last product is done).  Key tiles hold 128 keys, so every MMA is
-// M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the time of an N 128
-// one for half its work).  384 threads: warp 0 stages K tiles (3-slot ring) and V tiles
-// (2-slot ring) with bulk copies, warp 1 issues the MMAs from one thread, warp 2 owns the
-// tensor memory (all 512 columns), warps 4-7 and 8-11 are the softmax warpgroups of the two
-// heads (one thread per query row, TMEM lane = row).
+// head's Q buffer, free once the head's last product is done).  Key tiles hold 128 keys,
+// so every MMA is M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the
+// time of an N 128 one for half its work).
+// 576 threads: warp 0 stages K tiles (3-slot ring) and V tiles (2-slot ring) with bulk
+// copies; warp 1 owns the tensor memory (all 512 columns) and issues the MMAs from one
+// thread; warps 2-17 run the softmax, two warps per (head, 32-row quarter): one takes keys
+// 0-63 of each row, the other keys 64-127 (a warp reaches only TMEM lanes 32 (warp % 4) ..,
+// so warps 2 + 4i .. 5 + 4i cover the four quarters for i = 2 h + half).
 // Tensor memory per head h: O (128 fp32 columns) at 256 h and S (128 fp32 columns) at
-// 256 h + 128.  P overwrites S in place as packed bf16 pairs (keys 2c, 2c + 1 in column c)
-// and is the A operand of O += P V straight from tensor memory.  S_h(t + 1) is issued after
-// O_h += P_h(t) V(t) and one thread's MMAs run in issue order, so new scores never
-// overwrite P before it is read.
-// Each softmax thread takes its row of S in two 64-key halves: mask (skipped for halves the
-// whole warp sees), row max, P = 2^(S scale - m) into tensor memory; the half's O += P V
-// (4 MMAs) starts while the thread works on the next half, and one head's softmax overlaps
-// the other head's MMAs.  The reference max m of a row moves only when a half's max exceeds
-// it by more than 2^8 (then O is rescaled first); P and the running sum l use the same m,
-// so O / l is exact up to rounding.
+// 256 h + 128.  Each softmax warp overwrites its half of S in place with P = 2^(S scale - m)
+// as packed bf16 pairs (keys 2c, 2c + 1 in column c of the half), the A operand of
+// O += P V straight from tensor memory.  S_h(t + 1) is issued after O_h += P_h(t) V(t) and
+// one thread's MMAs run in issue order, so new scores never overwrite P before it is read.
+// The two warps of a row exchange their halves' maxima through shared memory at a named
+// barrier, so both scale P by the same reference max m; m moves only when the tile max
+// exceeds it by more than 2^8 (each warp then rescales its half of O before its P-ready
+// arrival; the tile's scores commit covers every earlier product, so O is stable).  P and the running sums use
+// the same m, so O / l is exact up to rounding.  One head's softmax overlaps the other
+// head's MMAs.
 // Visibility: the retained keys query j sees are the first before[j - w] compacted rows, so
 // one count masks a retained tile; window keys are a contiguous run of the band.  Stale rows
 // of a partial V tile are zeroed before its copy (P is 0 there, but 0 * NaN is not).
@@ -480,7 +482,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q and K are K-major, V is
 // MN-major (head_dim contiguous).
 constexpr int kTcHeads = 2;                              // query heads per CTA
-constexpr int kTcThreads = (4 + 4 * kTcHeads) * 32;      // 384
+constexpr int kTcSoftmaxWarps = 8 * kTcHeads;            // 2 per (head, row quarter)
+constexpr int kTcThreads = (2 + kTcSoftmaxWarps) * 32;   // 576
 // Kernel of the plain entry points (the faster of the two as measured).
 constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_TCGEN05;
 constexpr int kTcKeys = 128;                             // keys per tile
@@ -491,19 +494,21 @@ constexpr int kTcTileBytes = 2 * kTcHalfBytes;           // [2 d-halves][128 row
 constexpr int kTcQBytes = kPfRows * kRowBytes;           // Q, same layout
 constexpr int kTcOffV = kTcKSlots * kTcTileBytes;
 constexpr int kTcOffQ = kTcOffV + kTcVSlots * kTcTileBytes;
-constexpr int kTcOffBar = kTcOffQ + kTcHeads * kTcQBytes;
-constexpr int kTcSmemBytes = kTcOffBar + 256 + 1024;    // + barriers, + base alignment slack
+constexpr int kTcOffBar = kTcOffQ + kTcHeads * kTcQBytes;          // barrier block
+constexpr int kTcOffX = kTcOffBar + 256;                           // row-max exchange
+constexpr int kTcSmemBytes = kTcOffX + kTcHeads * 2 * kPfRows * 4;
+// The dynamic shared memory base is 1 KiB aligned (no static shared memory precedes it);
+// the kernel checks this and reports DMS_ERR_CUDA otherwise.
 static_assert(kTcSmemBytes <= 227 * 1024, "tcgen05 prefill shared memory");
 constexpr uint32_t kTcCols = 512;
 constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
 
-// Barriers of one head: s_full completes once per tile (scores ready), p_full[x] and
-// pv_done[x] once per tile for key half x (P written; its O += P V done).  Parity waits
-// need the waiter at most one phase behind; each wait below states why it is.
+// Barriers of one head: s_full completes once per tile (scores ready), p_full once per tile
+// (256 arrivals: P written by both halves), o_final once (every product done).
 struct TcHeadBars {
   uint64_t s_full;
-  uint64_t p_full[2];
-  uint64_t pv_done[2];
+  uint64_t p_full;
+  uint64_t o_final;
 };
 struct TcBars {
   uint64_t k_full[kTcKSlots], k_empty[kTcKSlots];
@@ -547,10 +552,14 @@ __device__ __forceinline__ void tc_stage_rows(uint8_t* dst, const uint8_t* src, 
 
 __global__ void __launch_bounds__(kTcThreads, 1)
     prefill_tc_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ TcMaps maps) {
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  extern __shared__ __align__(1024) uint8_t smem_tc[];
+  uint8_t* smem = smem_tc;
+  if (smem_addr(smem) & 1023u) {  // uniform over the CTA: nothing has started yet
+    if (threadIdx.x == 0) set_device_error(p.err, DMS_ERR_CUDA);
+    return;
+  }
   TcBars& bars = *reinterpret_cast<TcBars*>(smem + kTcOffBar);
+  float* xch = reinterpret_cast<float*>(smem + kTcOffX);  // [head][half][row]
   volatile int* abort_flag = &bars.abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -587,14 +596,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     mbar_init(&bars.q_ready, kPfRows * nh);
     for (int h = 0; h < kTcHeads; ++h) {
       mbar_init(&bars.h[h].s_full, 1);
-      for (int x = 0; x < 2; ++x) {
-        mbar_init(&bars.h[h].p_full[x], kPfRows);
-        mbar_init(&bars.h[h].pv_done[x], 1);
-      }
+      mbar_init(&bars.h[h].p_full, 2 * kPfRows);
+      mbar_init(&bars.h[h].o_final, 1);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 2) {
+  if (warp == 1) {
     tmem_alloc(&bars.tmem, kTcCols);
     tc_fence_before();
   }
@@ -653,8 +660,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
   } else if (warp == 1) {
     // ================================================================ MMA issuer
-    // Order per tile t: for each head h, O_h += P_h(t) V(t) by halves, then S_h(t + 1).
-    // The thread is the only waiter on k_full / v_full / p_full and consumes them in order.
+    // Order per tile t: for each head h, O_h += P_h(t) V(t), then S_h(t + 1) (or, after the
+    // last tile, the commit that releases O_h).  The thread is the only waiter on k_full /
+    // v_full / p_full and consumes them in order.
     if (lane == 0) {
       constexpr uint32_t idesc_s = f16_idesc(kPfRows, kTcKeys, 0);    // Q K^T: both K-major
       constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
@@ -692,22 +700,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const uint64_t dv = dv0 + (uint64_t)vs * kSlot;
         for (int h = 0; h < nh; ++h) {
           TcHeadBars& hb = bars.h[h];
+          mbar_wait(&hb.p_full, t & 1, abort_flag, p.err);
+          tc_fence_after();
+          // keys 16 kk .. 16 kk + 15: P columns 8 kk of the first half, 64 + 8 (kk - 4) of
+          // the second; V rows 16 kk .. (2 KiB per 16 rows)
           const uint32_t d_o = tmem + (uint32_t)(256 * h);
-          for (int x = 0; x < 2; ++x) {
-            // P_h(t) half x (keys 64 x ..): packed columns 32 x .., V rows 64 x ..
-            mbar_wait(&hb.p_full[x], t & 1, abort_flag, p.err);
-            tc_fence_after();
-            const uint32_t a = tmem + (uint32_t)(256 * h + 128 + 32 * x);
-            const uint64_t bv = dv + (uint64_t)(512 * x);
-            if (t == 0 && x == 0)
-              tc_mma_ts_k<false>(d_o, a, bv, idesc_o);
-            else
-              tc_mma_ts_k<true>(d_o, a, bv, idesc_o);
-            tc_mma_ts_k<true>(d_o, a + 8, bv + 128, idesc_o);
-            tc_mma_ts_k<true>(d_o, a + 16, bv + 256, idesc_o);
-            tc_mma_ts_k<true>(d_o, a + 24, bv + 384, idesc_o);
-            tc_commit(&hb.pv_done[x]);
-          }
+          const uint32_t a = tmem + (uint32_t)(256 * h + 128);
+          if (t == 0)
+            tc_mma_ts_k<false>(d_o, a, dv, idesc_o);
+          else
+            tc_mma_ts_k<true>(d_o, a, dv, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 8, dv + 128, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 16, dv + 256, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 24, dv + 384, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 64, dv + 512, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 72, dv + 640, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 80, dv + 768, idesc_o);
+          tc_mma_ts_k<true>(d_o, a + 88, dv + 896, idesc_o);
           if (more) {
             if (h == 0) {
               mbar_wait(&bars.k_full[(t + 1) % kTcKSlots], ((t + 1) / kTcKSlots) & 1, abort_flag,
@@ -715,23 +724,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               tc_fence_after();
             }
             issue_scores(h, t + 1);
+          } else {
+            tc_commit(&hb.o_final);
           }
         }
         tc_commit(&bars.v_empty[vs]);  // a slot is free once every product on it is done
         if (more) tc_commit(&bars.k_empty[(t + 1) % kTcKSlots]);
       }
     }
-  } else if (warp >= 4 && (warp - 4) / 4 < nh) {
-    // ================================================================ softmax warpgroups
-    const int h = (warp - 4) / 4;
-    const int row = tid - 128 * (1 + h);  // query row of the tile = TMEM lane
+  } else if ((warp - 2) / 8 < nh) {
+    // ================================================================ softmax
+    const int idx = (warp - 2) >> 2;            // 2 h + half
+    const int h = idx >> 1, half = idx & 1;     // head of the CTA, key half of the tile
+    const int row = 32 * (warp & 3) + lane;     // query row of the tile = TMEM lane
     const int j = j0 + row;
     const int hq = hq0 + h;
     const uint32_t o_addr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(256 * h);
-    const uint32_t s_addr = o_addr + 128u;
+    const uint32_t s_addr = o_addr + 128u + (uint32_t)(64 * half);  // this half of S / P
+    const int bar_id = 1 + 4 * h + (warp & 3);  // the two warps of this (head, quarter)
     TcHeadBars& hb = bars.h[h];
     uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;  // [d-half][row][128 B], swizzled
-    if (p.zero_first) {
+    float* x_mine = xch + (2 * h + half) * kPfRows + row;
+    const float* x_other = xch + (2 * h + (half ^ 1)) * kPfRows + row;
+    if (p.zero_first && half == 0) {
       // App. B: the decision element (head_dim 0 of the group's first head) is not a query
       // feature; zero it in the landed tile before any score reads it
       mbar_wait(&bars.q_full, 0, abort_flag, p.err);
@@ -741,8 +756,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     // the retained keys of this row: the first bj compacted rows
     const int bj = j - w > 0 ? p.before[head * (P + 1) + min(j - w, P)] : 0;
-    const float scale = p.scale_log2;
-    float m = -INFINITY, l = 0.f;  // reference max (log2 domain) and running sum of the row
+    const float2 scale2 = make_float2(p.scale_log2, p.scale_log2);
+    const int key0 = 64 * half;
+    float m = -INFINITY;  // reference max of the row (log2 domain), the same in both warps
+    float l = 0.f;        // running sum over this warp's half of the keys
     for (int t = 0; t < n_tiles; ++t) {
       const TcTile x = tc_tile(t, n_ct, nc, bs, jmax);
       int lo, nvis;  // visible keys of the tile: lo .. lo + nvis - 1
@@ -753,87 +770,89 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         lo = max(j - w - x.r0, 0);
         nvis = max(min(j - x.r0, x.rows - 1) - lo + 1, 0);
       }
-      // S(t) is issued after P(t - 1) is read, so this wait is at most one phase behind;
-      // its commit also covers every earlier product, so P(t - 1) is free to overwrite
+      // S(t) is issued after P(t - 1) is read, so this wait is at most one phase behind; its
+      // commit also covers every earlier product (O is stable, P(t - 1) is free)
       mbar_wait(&hb.s_full, t & 1, abort_flag, p.err);
       tc_fence_after();
-#pragma unroll 1
-      for (int half = 0; half < 2; ++half) {
-        float sc[64];
-        const uint32_t sa = s_addr + (uint32_t)(64 * half);
-        tmem_ld16_at(sa, sc);
-        tmem_ld16_at(sa + 16, sc + 16);
-        tmem_ld16_at(sa + 32, sc + 32);
-        tmem_ld16_at(sa + 48, sc + 48);
-        tmem_wait_ld();
-        const int key0 = 64 * half;
-        if (!__all_sync(0xffffffffu, lo <= key0 && key0 + 64 <= lo + nvis)) {
+      float sc[64];
+      tmem_ld16_at(s_addr, sc);
+      tmem_ld16_at(s_addr + 16, sc + 16);
+      tmem_ld16_at(s_addr + 32, sc + 32);
+      tmem_ld16_at(s_addr + 48, sc + 48);
+      tmem_wait_ld();
+      if (!__all_sync(0xffffffffu, lo <= key0 && key0 + 64 <= lo + nvis)) {
 #pragma unroll
-          for (int k = 0; k < 64; ++k)
-            if ((unsigned)(key0 + k - lo) >= (unsigned)nvis) sc[k] = -INFINITY;
-        }
-        float mx8[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) mx8[e] = sc[e];
-#pragma unroll
-        for (int k = 8; k < 64; ++k) mx8[k & 7] = fmaxf(mx8[k & 7], sc[k]);
-        const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-        const float mx_s = mx * scale;
-        // O += P V of this half of tile t - 1: done already (the S(t) commit covers it);
-        // waiting keeps pv_done[half] at most one phase ahead of this thread
-        if (t > 0) mbar_wait(&hb.pv_done[half], (t - 1) & 1, abort_flag, p.err);
-        float corr = 1.f;
-        if (mx_s > m + kTcRescale) {
-          corr = ex2_approx(m - mx_s);  // 0 when m = -inf
-          m = mx_s;
-        }
-        if ((t > 0 || half > 0) && __any_sync(0xffffffffu, corr != 1.f)) {
-          // (rare) O must hold the previous half's product: that of (t, 0) or (t - 1, 1)
-          mbar_wait(&hb.pv_done[half ^ 1], (half ? t : t - 1) & 1, abort_flag, p.err);
-          tc_fence_after();
-#pragma unroll 1
-          for (int c = 0; c < kHeadDim / 16; ++c) {
-            float r[16];
-            tmem_ld16(o_addr + (uint32_t)(16 * c), r);
-            tmem_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 16; ++e) r[e] *= corr;
-            tmem_st16(o_addr + (uint32_t)(16 * c), r);
-          }
-          tmem_wait_st();
-        }
-        const float nb = m == -INFINITY ? 0.f : -m;
-        uint32_t pk[32];
-        float s8[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) s8[e] = 0.f;
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const float p0 = ex2_approx(fmaf(sc[2 * c], scale, nb));
-          const float p1 = ex2_approx(fmaf(sc[2 * c + 1], scale, nb));
-          s8[c & 7] += p0 + p1;
-          pk[c] = pack_bf16x2(p0, p1);
-        }
-        tmem_st16_u32(s_addr + (uint32_t)(32 * half), pk);
-        tmem_st16_u32(s_addr + (uint32_t)(32 * half + 16), pk + 16);
-        tmem_wait_st();
-        l = l * corr + (((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7])));
-        tc_fence_before();
-        mbar_arrive(&hb.p_full[half]);
+        for (int k = 0; k < 64; ++k)
+          if ((unsigned)(key0 + k - lo) >= (unsigned)nvis) sc[k] = -INFINITY;
       }
-    }
-    // normalise this row once both halves of the last product are done (each wait is at
-    // most one phase behind: the products of tile n - 2 were awaited above); every MMA of
-    // this head is then done, so its Q buffer takes the bf16 row of O for the store
-    mbar_wait(&hb.pv_done[0], (n_tiles - 1) & 1, abort_flag, p.err);
-    mbar_wait(&hb.pv_done[1], (n_tiles - 1) & 1, abort_flag, p.err);
-    tc_fence_after();
-    const float inv = l > 0.f ? 1.f / l : 0.f;
+      float mx8[8];
 #pragma unroll
-    for (int c = 0; c < kHeadDim / 16; ++c) {
+      for (int e = 0; e < 8; ++e) mx8[e] = max3f(sc[e], sc[8 + e], sc[16 + e]);
+#pragma unroll
+      for (int k = 24; k < 64; k += 16)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx8[e] = max3f(mx8[e], sc[k + e], sc[k + 8 + e]);
+      const float mh = max3f(max3f(mx8[0], mx8[1], mx8[2]), max3f(mx8[3], mx8[4], mx8[5]),
+                             fmaxf(mx8[6], mx8[7]));
+      // the other half's max of this row (its previous value was read before it could be
+      // rewritten: the next tile's scores need both halves' P of this one)
+      *x_mine = mh;
+      named_barrier_sync_id(bar_id, 64);
+      const float mt = fmaxf(mh, *x_other) * p.scale_log2;
+      float corr = 1.f;
+      if (mt > m + kTcRescale) {
+        corr = ex2_approx(m - mt);  // 0 when m = -inf
+        m = mt;
+      }
+      const float nb = m == -INFINITY ? 0.f : -m;
+      const float2 nb2 = make_float2(nb, nb);
+      float2 s2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {  // 16 keys -> 8 packed columns, stored at once
+        uint32_t pk[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int k = 16 * g + 2 * c;
+          const float2 y = fma_f32x2(make_float2(sc[k], sc[k + 1]), scale2, nb2);
+          const float2 pp = make_float2(ex2_approx(y.x), ex2_approx(y.y));
+          s2[c & 1] = add_f32x2(s2[c & 1], pp);
+          pk[c] = pack_bf16x2(pp.x, pp.y);
+        }
+        tmem_st8_u32(s_addr + (uint32_t)(8 * g), pk);
+      }
+      const float2 ss = add_f32x2(s2[0], s2[1]);
+      l = l * corr + (ss.x + ss.y);
+      if (t > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
+        // (rare) this warp's half of the row of O, 16 columns at a time; O(t) += P V is
+        // issued only after this thread's P-ready arrival below
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float r[16];
+          const uint32_t oa = o_addr + (uint32_t)(64 * half + 16 * c);
+          tmem_ld16(oa, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) r[e] *= corr;
+          tmem_st16(oa, r);
+        }
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&hb.p_full);
+    }
+    // every product of this head is done: normalise this warp's half of the row and stage
+    // it as bf16 in the head's Q buffer (d-half = key half), then one thread stores the tile
+    mbar_wait(&hb.o_final, 0, abort_flag, p.err);
+    tc_fence_after();
+    *x_mine = l;  // both warps passed their last exchange before o_final could complete
+    named_barrier_sync_id(bar_id, 64);
+    const float lt = l + *x_other;
+    const float inv = lt > 0.f ? 1.f / lt : 0.f;
+    uint8_t* half_row = sq + half * (kPfRows * 128) + row * 128;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
       float r[16];
-      tmem_ld16(o_addr + (uint32_t)(16 * c), r);
+      tmem_ld16(o_addr + (uint32_t)(64 * half + 16 * c), r);
       tmem_wait_ld();
       uint4 v0, v1;
       v0.x = pack_bf16x2(r[0] * inv, r[1] * inv);
@@ -844,17 +863,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       v1.y = pack_bf16x2(r[10] * inv, r[11] * inv);
       v1.z = pack_bf16x2(r[12] * inv, r[13] * inv);
       v1.w = pack_bf16x2(r[14] * inv, r[15] * inv);
-      // logical chunks 2c, 2c + 1 (head_dim 16c .. 16c + 15) of d-half c / 4
-      uint8_t* half_row = sq + (c >> 2) * (kPfRows * 128) + row * 128;
-      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, (2 * c) & 7)) = v0;
-      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, (2 * c + 1) & 7)) = v1;
+      // head_dim 64 half + 16c .. + 15: logical chunks 2c, 2c + 1 of the d-half
+      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, 2 * c)) = v0;
+      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, 2 * c + 1)) = v1;
     }
     fence_proxy_async_smem();
-    if (h == 0)
-      named_barrier_sync<1>(kPfRows);
-    else
-      named_barrier_sync<2>(kPfRows);
-    if (row == 0) {
+    named_barrier_sync_id(9 + h, 2 * kPfRows);
+    if (half == 0 && row == 0) {
       // rows past the prompt fall outside the tensor map and are not written
       tma_store_3d(&maps.out, hq * kHeadDim, j0, b, sq);
       tma_store_3d(&maps.out, hq * kHeadDim + 64, j0, b, sq + kPfRows * 128);
@@ -865,7 +880,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   // ---- teardown: every tensor-memory access is done before the columns are released
   tc_fence_before();
   __syncthreads();
-  if (warp == 2) {
+  if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTcCols);
   }
