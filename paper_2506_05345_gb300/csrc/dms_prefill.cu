@@ -504,7 +504,8 @@ constexpr uint32_t kTcCols = 512;
 constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
 
 // Barriers of one head: s_full completes once per tile (scores ready), p_full once per tile
-// (256 arrivals: P written by both halves), o_final once (every product done).
+// (8 arrivals, one per softmax warp once the warp's P is written), o_final once (every
+// product done).
 struct TcHeadBars {
   uint64_t s_full;
   uint64_t p_full;
@@ -593,10 +594,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&bars.v_empty[s], 1);
     }
     mbar_init(&bars.q_full, 1);
-    mbar_init(&bars.q_ready, kPfRows * nh);
+    mbar_init(&bars.q_ready, 4 * nh);
     for (int h = 0; h < kTcHeads; ++h) {
       mbar_init(&bars.h[h].s_full, 1);
-      mbar_init(&bars.h[h].p_full, 2 * kPfRows);
+      mbar_init(&bars.h[h].p_full, 8);
       mbar_init(&bars.h[h].o_final, 1);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -752,7 +753,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_wait(&bars.q_full, 0, abort_flag, p.err);
       if (hq % G == 0) *reinterpret_cast<uint16_t*>(sq + row * 128 + chunk_in_row(row, 0)) = 0;
       fence_proxy_async_smem();
-      mbar_arrive(&bars.q_ready);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars.q_ready);
     }
     // the retained keys of this row: the first bj compacted rows
     const int bj = j - w > 0 ? p.before[head * (P + 1) + min(j - w, P)] : 0;
@@ -838,7 +840,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&hb.p_full);
+      __syncwarp();  // the warp's stores are ordered before its one arrival
+      if (lane == 0) mbar_arrive(&hb.p_full);
     }
     // every product of this head is done: normalise this warp's half of the row and stage
     // it as bf16 in the head's Q buffer (d-half = key half), then one thread stores the tile
