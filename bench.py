@@ -39,7 +39,8 @@ METRIC = "retained KV tokens read/s and decode-attn µs/layer-step; % of GB300 H
 UNIT = "tokens/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-DECODE_SRC = os.path.join(ROOT, "paper_2506_05345_gb300", "csrc", "dms_decode.cu")
+DECODE_SRCS = [os.path.join(ROOT, "paper_2506_05345_gb300", "csrc", f)
+               for f in ("dms_decode.cu", "dms_ptx.cuh", "dms_internal.cuh")]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
 
 
@@ -113,8 +114,12 @@ def measured_peak():
 
 
 def decode_source_sha():
-    with open(DECODE_SRC, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """Hash of every source the decode kernel is compiled from."""
+    h = hashlib.sha256()
+    for path in DECODE_SRCS:
+        with open(path, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def traffic_per_launch(units_per_launch):
