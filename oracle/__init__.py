@@ -13,6 +13,10 @@ Functions (all take bf16 data as ``numpy.uint16`` bit patterns):
                                          immediate-eviction ablation when immediate)
   decode(q, k, v, logits, j, w, scale, immediate)  softmax attention over the retained set
   borrowed(q, G)                         App. B decision neuron: (logits, attention q)
+  e4m3_to_double(code), e4m3_from_float(x)   fp8 E4M3FN value of a code / nearest code
+  quantize_rows_e4m3(rows)               per-row fp32 scale and E4M3 codes of bf16 rows
+  decode_fp8(q, kc, ks, vc, vs, logits, j, w, scale, immediate)
+                                         the attention over the dequantised rows
 """
 from __future__ import annotations
 
@@ -69,6 +73,19 @@ def _load():
                                                      ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
                                                      ctypes.c_double, f64p]
             lib.dms_oracle_decode_policy.restype = None
+            u8p = ctypes.POINTER(ctypes.c_uint8)
+            f32p = ctypes.POINTER(ctypes.c_float)
+            lib.dms_oracle_e4m3_to_double.argtypes = [ctypes.c_uint8]
+            lib.dms_oracle_e4m3_to_double.restype = ctypes.c_double
+            lib.dms_oracle_e4m3_from_float.argtypes = [ctypes.c_float]
+            lib.dms_oracle_e4m3_from_float.restype = ctypes.c_uint8
+            lib.dms_oracle_quantize_row_e4m3.argtypes = [u16p, ctypes.c_int32, u8p, f32p]
+            lib.dms_oracle_quantize_row_e4m3.restype = None
+            lib.dms_oracle_decode_kv64.argtypes = [u16p, ctypes.c_int32, ctypes.c_int32, f64p,
+                                                   f64p, ctypes.c_int64, u16p, ctypes.c_int64,
+                                                   ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
+                                                   ctypes.c_double, f64p]
+            lib.dms_oracle_decode_kv64.restype = None
             _lib = lib
     return _lib
 
@@ -159,3 +176,71 @@ def borrowed(q, group: int):
     q_att = q.copy()
     q_att[..., ::group, 0] = 0
     return logits, q_att
+
+
+def e4m3_to_double(code: int) -> float:
+    """Value of an fp8 E4M3FN code (NaN for S.1111.111)."""
+    return _load().dms_oracle_e4m3_to_double(int(code) & 0xFF)
+
+
+def e4m3_from_float(x: float) -> int:
+    """Nearest E4M3FN code of the float32 value x: ties to even, magnitudes above 448
+    saturated, NaN -> 0x7f."""
+    return int(_load().dms_oracle_e4m3_from_float(float(np.float32(x))))
+
+
+def quantize_rows_e4m3(rows):
+    """Per-row quantisation of bf16 rows [..., D] (uint16 bits): returns (codes uint8
+    [..., D], scales float32 [...]) with scale = fl32(amax / 448) and code =
+    E4M3(fl32(x / scale)); zero rows get scale 0 and zero codes."""
+    r = np.ascontiguousarray(_u16(rows))
+    D = r.shape[-1]
+    flat = r.reshape(-1, D)
+    codes = np.zeros(flat.shape, dtype=np.uint8)
+    scales = np.zeros(flat.shape[0], dtype=np.float32)
+    lib = _load()
+    for i in range(flat.shape[0]):
+        row = np.ascontiguousarray(flat[i])
+        sc = ctypes.c_float(0.0)
+        lib.dms_oracle_quantize_row_e4m3(_ptr(row, ctypes.c_uint16), D,
+                                         codes[i].ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)),
+                                         ctypes.byref(sc))
+        scales[i] = sc.value
+    return codes.reshape(r.shape), scales.reshape(r.shape[:-1])
+
+
+_E4M3 = None
+
+
+def _e4m3_table() -> np.ndarray:
+    global _E4M3
+    if _E4M3 is None:
+        _E4M3 = np.array([e4m3_to_double(c) for c in range(256)], dtype=np.float64)
+    return _E4M3
+
+
+def dequantize_e4m3(codes, scales) -> np.ndarray:
+    """codes [..., D] uint8, scales [...] -> fp64 rows code value * scale (exact)."""
+    c = np.asarray(codes, dtype=np.uint8)
+    return _e4m3_table()[c] * np.asarray(scales, dtype=np.float64)[..., None]
+
+
+def decode_fp8(q, k_codes, k_scales, v_codes, v_scales, logits, j: int, w: int,
+               scale: float = 0.0, immediate: bool = False) -> np.ndarray:
+    """Attention of G query heads (q [G, D] bf16 bits) over the retained set at step j
+    of a cache whose rows are E4M3 codes [T, D] with per-row scales [T]."""
+    q = np.ascontiguousarray(_u16(q))
+    lg = _u16(logits)
+    kd = np.ascontiguousarray(dequantize_e4m3(k_codes, k_scales))
+    vd = np.ascontiguousarray(dequantize_e4m3(v_codes, v_scales))
+    G, D = q.shape
+    if kd.shape != vd.shape or kd.shape[1] != D:
+        raise ValueError("shape mismatch")
+    if j >= kd.shape[0] or j >= lg.shape[0]:
+        raise ValueError("j beyond the data given")
+    out = np.zeros((G, D), dtype=np.float64)
+    _load().dms_oracle_decode_kv64(_ptr(q, ctypes.c_uint16), G, D, _ptr(kd, ctypes.c_double),
+                                   _ptr(vd, ctypes.c_double), D, _ptr(lg, ctypes.c_uint16),
+                                   lg.strides[0] // 2, j, w, 1 if immediate else 0, float(scale),
+                                   _ptr(out, ctypes.c_double))
+    return out

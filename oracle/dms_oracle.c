@@ -32,9 +32,21 @@
  * is fp64 with plain sequential sums in index order.  bf16 inputs are widened
  * exactly (a bf16 value is the upper half of an IEEE binary32).
  *
+ *   - Related work (KV cache reduction): quantisation of the cache is orthogonal to
+ *     DMS and can be combined with it.  The quantised page format checked here is
+ *     fp8 E4M3 (the OCP "E4M3FN" encoding: 1 sign, 4 exponent bits with bias 7,
+ *     3 mantissa bits, no infinities, S.1111.111 = NaN, largest finite 448, smallest
+ *     normal 2^-6, subnormals m * 2^-9) with one fp32 scale per row: scale =
+ *     fl32(amax / 448), code = e4m3(fl32(x / scale)) rounded to nearest even and
+ *     saturated to +-448; a row of zeros has scale 0 and zero codes.  These roundings
+ *     decide integer codes, so both sides take them in fp32.  The attention then runs
+ *     in fp64 over the dequantised rows code * scale.
+ *
  * Parity pins (tests, no GPU): Fig. 1b pattern, brute-force dense masked
  * softmax with the training mask M_alpha of Sec. 3.1, dense causal attention
- * when nothing is evicted, w = 0 with all-evict, the closed-form retained count.
+ * when nothing is evicted, w = 0 with all-evict, the closed-form retained count;
+ * for fp8: every code against PyTorch's float8_e4m3fn, round-to-nearest-even at
+ * midpoints, exact rows (values already on the e4m3 grid times a power of two).
  */
 #include <math.h>
 #include <stdint.h>
@@ -155,4 +167,100 @@ void dms_oracle_decode(const uint16_t* q, int32_t G, int32_t D,
                        const uint16_t* logits, int64_t logit_stride, int64_t j,
                        int64_t w, double scale, double* out) {
   dms_oracle_decode_policy(q, G, D, k, v, kv_stride, logits, logit_stride, j, w, 0, scale, out);
+}
+
+/* ------------------------------------------------------------------ fp8 E4M3 page format */
+
+/* Value of an E4M3FN code (exact in double); NaN for S.1111.111. */
+double dms_oracle_e4m3_to_double(uint8_t code) {
+  const int sign = code >> 7, e = (code >> 3) & 15, m = code & 7;
+  if (e == 15 && m == 7) return NAN;
+  double mag = e == 0 ? ldexp((double)m, -9) : ldexp((double)(8 + m), e - 10);
+  return sign ? -mag : mag;
+}
+
+/*
+ * Nearest E4M3FN code of x, ties to even, magnitudes above 448 saturated to 448,
+ * NaN -> 0x7f.  The non-negative codes are ordered like their values: code
+ * 8 (e - 1) + k holds k * 2^(e - 10) for e >= 1 and k = 8..15 (k = 16 rolls over to
+ * the next binade), code k holds k * 2^-9 for k = 0..8.
+ */
+uint8_t dms_oracle_e4m3_from_float(float x) {
+  if (x != x) return 0x7f;
+  const uint8_t sign = signbit(x) ? 0x80 : 0x00;
+  const double a = fabs((double)x);
+  if (a >= 448.0) return sign | 0x7e;
+  int code;
+  if (a < ldexp(1.0, -6)) {
+    code = (int)rint(a / ldexp(1.0, -9)); /* 0 .. 8, exact quotient */
+  } else {
+    int e2;
+    frexp(a, &e2);                          /* a in [2^(e2-1), 2^e2) */
+    const int e = e2 + 6;                   /* binade exponent field, 1 .. 15 */
+    const int k = (int)rint(a / ldexp(1.0, e - 10)); /* 8 .. 16 */
+    code = 8 * (e - 1) + k;
+  }
+  if (code > 0x7e) code = 0x7e;
+  return sign | (uint8_t)code;
+}
+
+/* One row of D bf16 values to E4M3 codes and its fp32 scale (see the header). */
+void dms_oracle_quantize_row_e4m3(const uint16_t* x, int32_t D, uint8_t* codes, float* scale) {
+  float amax = 0.0f;
+  for (int32_t d = 0; d < D; ++d) {
+    const float a = fabsf((float)dms_oracle_bf16_to_double(x[d]));
+    if (a > amax) amax = a;
+  }
+  if (amax == 0.0f) {
+    *scale = 0.0f;
+    for (int32_t d = 0; d < D; ++d) codes[d] = 0;
+    return;
+  }
+  const float s = amax / 448.0f;
+  *scale = s;
+  for (int32_t d = 0; d < D; ++d) {
+    const float q = (float)dms_oracle_bf16_to_double(x[d]) / s;
+    codes[d] = dms_oracle_e4m3_from_float(q);
+  }
+}
+
+/*
+ * Decode attention as dms_oracle_decode_policy, over fp64 key / value rows (row i at
+ * k + i * kv_stride): the dequantised rows of a quantised cache.
+ */
+void dms_oracle_decode_kv64(const uint16_t* q, int32_t G, int32_t D, const double* k,
+                            const double* v, int64_t kv_stride, const uint16_t* logits,
+                            int64_t logit_stride, int64_t j, int64_t w, int immediate,
+                            double scale, double* out) {
+  if (scale <= 0.0) scale = 1.0 / sqrt((double)D);
+  int64_t cap = j + 1 > 0 ? j + 1 : 0;
+  int32_t* pos = (int32_t*)malloc(sizeof(int32_t) * (size_t)(cap > 0 ? cap : 1));
+  double* s = (double*)malloc(sizeof(double) * (size_t)(cap > 0 ? cap : 1));
+  int64_t n = dms_oracle_retained_policy(logits, logit_stride, j, w, immediate, pos);
+  for (int32_t g = 0; g < G; ++g) {
+    double* o = out + (int64_t)g * D;
+    for (int32_t d = 0; d < D; ++d) o[d] = 0.0;
+    if (n == 0) continue;
+    const uint16_t* qg = q + (int64_t)g * D;
+    double m = -INFINITY;
+    for (int64_t r = 0; r < n; ++r) {
+      const double* kr = k + (int64_t)pos[r] * kv_stride;
+      double dot = 0.0;
+      for (int32_t d = 0; d < D; ++d) dot += dms_oracle_bf16_to_double(qg[d]) * kr[d];
+      s[r] = scale * dot;
+      if (s[r] > m) m = s[r];
+    }
+    double den = 0.0;
+    for (int64_t r = 0; r < n; ++r) {
+      s[r] = exp(s[r] - m);
+      den += s[r];
+    }
+    for (int64_t r = 0; r < n; ++r) {
+      const double* vr = v + (int64_t)pos[r] * kv_stride;
+      double p = s[r] / den;
+      for (int32_t d = 0; d < D; ++d) o[d] += p * vr[d];
+    }
+  }
+  free(pos);
+  free(s);
 }

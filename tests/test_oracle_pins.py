@@ -417,3 +417,93 @@ def test_immediate_eviction_decode_brute_force():
         np.testing.assert_allclose(got, ref[j], rtol=0, atol=1e-12)
         differs |= not np.array_equal(got, oracle.decode(q[j], k, v, lg, j, w))
     assert differs  # the ablation is a different policy
+
+
+# --------------------------------------------------------------------------- fp8 KV page format
+
+
+def _torch_e4m3_codes(x: np.ndarray) -> np.ndarray:
+    return torch.from_numpy(np.asarray(x, dtype=np.float32)).to(torch.float8_e4m3fn) \
+        .view(torch.uint8).numpy()
+
+
+def test_e4m3_values_match_torch():
+    """Every code's value equals PyTorch's float8_e4m3fn (an independent implementation of
+    the OCP E4M3FN definition), NaN codes included."""
+    ref = torch.arange(256, dtype=torch.uint8).view(torch.float8_e4m3fn).double().numpy()
+    mine = np.array([oracle.e4m3_to_double(c) for c in range(256)])
+    assert np.array_equal(np.isnan(ref), np.isnan(mine))
+    ok = ~np.isnan(ref)
+    assert np.array_equal(ref[ok], mine[ok])
+    assert mine[0x7E] == 448.0 and mine[0x08] == 2.0 ** -6 and mine[0x01] == 2.0 ** -9
+    assert mine[0x38] == 1.0 and np.isnan(mine[0x7F]) and np.isnan(mine[0xFF])
+
+
+def test_e4m3_encoding_matches_torch_and_ties_to_even():
+    """Round to nearest, ties to even, on every value, every midpoint between neighbours
+    and random floats in [-448, 448]; saturation above 448."""
+    vals = np.array([oracle.e4m3_to_double(c) for c in range(0x7F)])  # 0 .. 448, increasing
+    assert np.all(np.diff(vals) > 0)
+    mids = (vals[:-1] + vals[1:]) / 2  # exact in float32 (at most 5 significant bits)
+    rng = np.random.default_rng(5)
+    xs = np.concatenate([vals, mids, -vals, -mids, rng.uniform(-448, 448, 4000),
+                         rng.standard_normal(4000) * 0.01]).astype(np.float32)
+    mine = np.array([oracle.e4m3_from_float(x) for x in xs], dtype=np.uint8)
+    assert np.array_equal(mine, _torch_e4m3_codes(xs))
+    for m_lo, m_hi in zip(range(0, 0x7E), range(1, 0x7F)):
+        got = oracle.e4m3_from_float((vals[m_lo] + vals[m_hi]) / 2)
+        assert got == (m_lo if m_lo % 2 == 0 else m_hi)
+    for x, code in [(449.0, 0x7E), (464.0, 0x7E), (1e30, 0x7E), (-1e30, 0xFE), (-0.0, 0x80)]:
+        assert oracle.e4m3_from_float(x) == code
+    assert oracle.e4m3_from_float(float("nan")) == 0x7F
+
+
+def test_quantize_rows_bounds_and_scale():
+    """scale = fl32(amax / 448); the largest element maps to +-448 (code 0x7E / 0xFE); every
+    dequantised element is within half a step of its value; zero rows stay zero."""
+    rng = np.random.default_rng(6)
+    rows = _bf16(rng.standard_normal((64, 128)) * rng.uniform(1e-3, 50, (64, 1)))
+    rows[3] = 0
+    rows[5, 7] = _bf16([-300.0])[0]  # a negative outlier sets amax
+    codes, scales = oracle.quantize_rows_e4m3(rows)
+    x = _f64(rows)
+    amax = np.abs(x).max(axis=1).astype(np.float32)
+    assert np.array_equal(scales, (amax / np.float32(448)).astype(np.float32))
+    assert scales[3] == 0 and np.all(codes[3] == 0)
+    deq = oracle.dequantize_e4m3(codes, scales)
+    for i in range(64):
+        if scales[i] == 0:
+            continue
+        top = np.argmax(np.abs(x[i]))
+        assert codes[i, top] & 0x7F == 0x7E
+        y = x[i] / scales[i]
+        step = np.where(np.abs(y) >= 2.0 ** -6, 2.0 ** (np.floor(np.log2(np.maximum(np.abs(y), 2.0 ** -6))) - 3),
+                        2.0 ** -9)
+        assert np.all(np.abs(deq[i] - x[i]) <= 0.5 * step * scales[i] * (1 + 1e-6))
+    assert codes[5, 7] == 0xFE
+
+
+def test_fp8_decode_exact_rows_equal_bf16_decode():
+    """Rows already on the E4M3 grid times 2^k with amax = 448 * 2^k quantise exactly, so the
+    quantised-cache attention equals the bf16 attention on the same rows."""
+    rng = np.random.default_rng(7)
+    T, G, D, w = 40, 3, 128, 6
+    grid = np.array([oracle.e4m3_to_double(c) for c in range(0x7F)])
+    def exact_rows(n):
+        r = rng.choice(np.concatenate([grid, -grid]), (n, D))
+        r[:, 0] = 448.0
+        return r * 2.0 ** rng.integers(-12, -4, (n, 1))
+    kf, vf = exact_rows(T), exact_rows(T)
+    k, v = _bf16(kf), _bf16(vf)
+    assert np.array_equal(_f64(k), kf) and np.array_equal(_f64(v), vf)
+    q = _bf16(rng.standard_normal((G, D)))
+    lg = _bf16(rng.standard_normal(T) + 0.5)
+    kc, ks = oracle.quantize_rows_e4m3(k)
+    vc, vs = oracle.quantize_rows_e4m3(v)
+    assert np.array_equal(oracle.dequantize_e4m3(kc, ks), kf)
+    for j in (0, 17, T - 1):
+        np.testing.assert_allclose(oracle.decode_fp8(q, kc, ks, vc, vs, lg, j, w),
+                                   oracle.decode(q, k, v, lg, j, w), rtol=0, atol=1e-12)
+    # a plausible mistake (the value scales applied to the keys) is caught
+    bad = oracle.decode_fp8(q, kc, vs, vc, ks, lg, T - 1, w)
+    assert not np.allclose(bad, oracle.decode(q, k, v, lg, T - 1, w), atol=1e-6)
