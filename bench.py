@@ -54,6 +54,8 @@ def parse():
     ap.add_argument("--dense", action="store_true", help="no evictions (CR 1) with the same shape")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--kv-fp8", action="store_true",
+                    help="fp8 E4M3 page format (per-row scales); append and decode as two launches")
     ap.add_argument("--ctas-per-sm", type=int, default=0)
     ap.add_argument("--min-pages", type=int, default=0)
     ap.add_argument("--separate", action="store_true",
@@ -258,8 +260,11 @@ def run_ours(args, wl, world, rank, local, pg):
     decode_needed = max(wl.decode_steps, W_ + K_ + K2 + E_W + E_K)
     capacity = wl.prefill_tokens + decode_needed
     seed_tag = replica_tag(rank)
+    if args.kv_fp8:
+        args.separate = True  # the fp8 format has no fused append + decode kernel
     cache = dms.DmsCache(layers=L, kv_heads=H, window=wl.window, capacity=capacity, batch=B,
-                         ctas_per_sm=args.ctas_per_sm, min_pages_per_cta=args.min_pages)
+                         ctas_per_sm=args.ctas_per_sm, min_pages_per_cta=args.min_pages,
+                         kv_format=dms.DMS_KV_FP8_E4M3 if args.kv_fp8 else dms.DMS_KV_BF16)
     stream = torch.cuda.current_stream()
 
     # ---- sampled heads for the parity check and the CPU baseline (layer 0)
@@ -415,7 +420,8 @@ def run_ours(args, wl, world, rank, local, pg):
               for i in range(K2) for layer in range(L)]
     app_ms = ([ev_app[i][layer][0].elapsed_time(ev_app[i][layer][1])
                for i in range(K2) for layer in range(L)] if args.separate else [0.0])
-    bytes_per_unit = workloads.kv_bytes_per_token_head(D)
+    # bf16: K and V rows, 2 * 2 * D bytes; fp8: 2 * D codes and two fp32 scales
+    bytes_per_unit = 2 * D + 8 if args.kv_fp8 else workloads.kv_bytes_per_token_head(D)
     if args.separate:
         # two kernels per layer-step: the decode launches' own event-bracketed durations
         units_per_launch = 0.5 * (tok_last + st_k2["total_retained"]) / L
@@ -455,7 +461,12 @@ def run_ours(args, wl, world, rank, local, pg):
             qq = q_last[b, h * Gs:(h + 1) * Gs]
             if args.borrowed:  # the attention takes the borrowed element as 0 (App. B)
                 qq = oracle.borrowed(qq, Gs)[1]
-            ref = oracle.decode(qq, kk, vv, ll, j, wl.window)
+            if args.kv_fp8:  # the oracle quantises the history itself
+                kk = oracle.quantize_rows_e4m3(kk)
+                vv = oracle.quantize_rows_e4m3(vv)
+                ref = oracle.decode_fp8(qq, *kk, *vv, ll, j, wl.window)
+            else:
+                ref = oracle.decode(qq, kk, vv, ll, j, wl.window)
             errs.append(np.abs(got[b, h * Gs:(h + 1) * Gs] - ref).ravel())
             cases.append((qq, kk, vv, ll, len(oracle.retained(ll, j, wl.window))))
         e = np.concatenate(errs)
@@ -467,7 +478,10 @@ def run_ours(args, wl, world, rank, local, pg):
         t0 = time.perf_counter()
         while True:
             for (qq, kk, vv, ll, n) in cases:
-                oracle.decode(qq, kk, vv, ll, j, wl.window)
+                if args.kv_fp8:
+                    oracle.decode_fp8(qq, *kk, *vv, ll, j, wl.window)
+                else:
+                    oracle.decode(qq, kk, vv, ll, j, wl.window)
                 tok += n
                 calls += 1
             if time.perf_counter() - t0 >= args.cpu_seconds:
@@ -579,13 +593,16 @@ def run_ours(args, wl, world, rank, local, pg):
 
     peak, peak_kind = measured_peak()
     achieved_gbs = units_per_launch * bytes_per_unit / dec_avg_s / 1e9
-    traffic = traffic_per_launch(units_per_launch)
+    traffic = None if args.kv_fp8 else traffic_per_launch(units_per_launch)
     res = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K_,
         "warmup": W_, "ms_per_step": elapsed_max_ms / K_, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "fp8 E4M3 K/V codes, f16 MMA, fp32 accumulate" if args.kv_fp8 else "bf16",
+        "data": "synthetic",
         "impl": "ours",
         "config": {"workload": wl.name, "batch_per_gpu": B, "layers": L, "q_heads": Hq,
+                   "kv_format": "fp8_e4m3 (per-row fp32 scales)" if args.kv_fp8 else "bf16",
                    "kv_heads": H, "head_dim": D, "window": wl.window, "prefill": wl.prefill_tokens,
                    "timed_positions": [wl.prefill_tokens + W_, wl.prefill_tokens + W_ + K_ - 1],
                    "p_evict": (None if wl.ragged_beta else wl.p_evict),
@@ -605,7 +622,8 @@ def run_ours(args, wl, world, rank, local, pg):
         "retained_tokens_per_layer_step": units_per_launch,
         "compression": (wl.prefill_tokens + n_dev_steps) * B * H / units_per_launch,
         "hbm_frac_of_nominal_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
-        "roofline": {"kernel": "decode_tiled_kernel" + ("" if args.separate else " (append fused)"),
+        "roofline": {"kernel": "decode_tiled_kernel" + (" (fp8 pages)" if args.kv_fp8 else "") +
+                               ("" if args.separate else " (append fused)"),
                      "bound": "hbm", "achieved": achieved_gbs,
                      "peak": peak, "unit": "GB/s", "frac": achieved_gbs / peak,
                      "peak_kind": f"{peak_kind} copy bandwidth",

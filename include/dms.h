@@ -73,6 +73,24 @@ enum {
   DMS_DECODE_SIMPLE = 1  /* one CTA per KV head, CUDA cores; a cross-check path     */
 };
 
+/*
+ * Page formats selectable through dms_options.kv_format.  The paper treats KV
+ * quantisation as orthogonal to DMS and combinable with it (related-work section:
+ * quantisation, e.g. per-channel keys and per-token values, is a separate axis of
+ * KV-cache reduction).
+ */
+enum {
+  DMS_KV_BF16 = 0,     /* default: K and V rows of 128 bf16; pages of 32 KiB          */
+  DMS_KV_FP8_E4M3 = 1  /* K and V rows of 128 fp8 E4M3 codes (OCP E4M3FN: bias 7,
+                          no infinities, largest finite 448) with one fp32 scale per
+                          row and tensor: scale = amax(|row|) / 448 (fp32 division),
+                          code = E4M3(row / scale) rounded to nearest even and
+                          saturated; a row of zeros has scale 0.  Pages of 16 KiB
+                          (+ 512 bytes of scales).  Rows must be finite.  Taken only
+                          by the tiled decode kernel; single-token append + decode
+                          runs as two launches.                                      */
+};
+
 typedef struct dms_options {
   int32_t batch;         /* sequences per layer (required, >= 1)                    */
   int32_t page_tokens;   /* tokens per page; 0 = 64 (only 64 is accepted)           */
@@ -84,7 +102,9 @@ typedef struct dms_options {
   int32_t ctas_per_sm;   /* split-K CTAs per SM for the tiled kernel; 0 = 1         */
   int32_t min_pages_per_cta; /* lower bound on pages per split-K CTA; 0 = 2         */
   int32_t eviction_policy;   /* DMS_EVICT_DELAYED (0) or DMS_EVICT_IMMEDIATE (1)    */
-  int32_t reserved[4];   /* must be zero                                            */
+  int32_t kv_format;     /* DMS_KV_BF16 (0) or DMS_KV_FP8_E4M3 (1); fp8 requires the
+                            tiled decode kernel                                     */
+  int32_t reserved[3];   /* must be zero                                            */
 } dms_options;
 
 typedef struct dms_stats {
@@ -283,6 +303,20 @@ dms_status dms_cache_stats(dms_cache* cache, dms_stats* out, int32_t* counts, vo
 dms_status dms_cache_export_positions(dms_cache* cache, int32_t layer, int32_t* host_pos,
                                       void* stream);
 
+/*
+ * Test/inspection helper.  Synchronise `stream` and write, for every
+ * (sequence b, KV head h) of `layer` and every slot s < n_h, the stored key and
+ * value rows in head_dim order into the HOST arrays
+ *   host_k[((b * kv_heads + h) * capacity + s) * 128 + d]   (and host_v likewise),
+ * elements of the cache's format: bf16 bit patterns (uint16) for DMS_KV_BF16,
+ * E4M3 codes (uint8) for DMS_KV_FP8_E4M3; and, for fp8 caches, the row scales
+ * into host_scales[((b * kv_heads + h) * capacity + s) * 2 + {0: key, 1: value}]
+ * (host_scales is ignored, and may be NULL, for bf16 caches).  Entries of slots
+ * >= n_h are zero.  Copies page by page (a few calls per page); meant for tests.
+ */
+dms_status dms_cache_export_kv(dms_cache* cache, int32_t layer, void* host_k, void* host_v,
+                               float* host_scales, void* stream);
+
 /* Current length (tokens appended per sequence) of `layer`, into *out. */
 dms_status dms_cache_layer_length(const dms_cache* cache, int32_t layer, int64_t* out);
 
@@ -299,7 +333,7 @@ dms_status dms_cache_layer_length(const dms_cache* cache, int32_t layer, int64_t
  * file-scope device array of about 8.5 MB that every GPU loading the library
  * holds until the process exits.
  *
- * Inputs (device pointers, 16-byte aligned where they hold bf16 rows):
+ * Inputs (device pointers, 16-byte aligned where they hold bf16 rows; bf16 pages only):
  *   pool        pages of 32 KiB: page p holds 64 K rows then 64 V rows, each row
  *               128 bf16 (256 bytes) whose sixteen 16-byte chunks are stored
  *               permuted -- logical chunk c of row r at physical chunk

@@ -23,6 +23,7 @@ from . import _native
 from ._native import (DMS_EVICT_DELAYED, DMS_EVICT_IMMEDIATE,  # noqa: F401
                       DMS_PREFILL_MMA_SYNC, DMS_PREFILL_TCGEN05,  # noqa: F401
                       DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
+                      DMS_KV_BF16, DMS_KV_FP8_E4M3,  # noqa: F401
                       DMS_ERR_INVALID_ARGUMENT, DMS_ERR_STATE, DMS_ERR_TIMEOUT, DMS_OK,
                       DmsLibraryError,
                       dms_options, dms_stats)
@@ -193,6 +194,11 @@ def dms_cache_export_positions(cache, layer, host_pos_ptr, stream):
     return library().dms_cache_export_positions(cache, layer, host_pos_ptr, stream)
 
 
+def dms_cache_export_kv(cache, layer, host_k_ptr, host_v_ptr, host_scales_ptr, stream):
+    return library().dms_cache_export_kv(cache, layer, host_k_ptr, host_v_ptr, host_scales_ptr,
+                                         stream)
+
+
 def dms_cache_layer_length(cache, layer):
     out = ctypes.c_int64()
     code = library().dms_cache_layer_length(cache, layer, ctypes.byref(out))
@@ -236,9 +242,11 @@ class DmsCache:
     def __init__(self, layers: int, kv_heads: int, window: int, capacity: int, batch: int,
                  head_dim: int = HEAD_DIM, pool_tokens: int = 0,
                  decode_kernel: int = DMS_DECODE_TILED, ctas_per_sm: int = 0,
-                 min_pages_per_cta: int = 0, eviction_policy: int = 0):
+                 min_pages_per_cta: int = 0, eviction_policy: int = 0,
+                 kv_format: int = DMS_KV_BF16):
         self._h = None
         opt = dms_options()
+        opt.kv_format = kv_format
         opt.batch = batch
         opt.pool_tokens = pool_tokens
         opt.decode_kernel = decode_kernel
@@ -250,6 +258,7 @@ class DmsCache:
         self._h = h
         self.layers, self.kv_heads, self.window = layers, kv_heads, window
         self.capacity, self.batch, self.head_dim = capacity, batch, head_dim
+        self.kv_format = kv_format
 
     def close(self):
         if self._h is not None:
@@ -398,6 +407,22 @@ class DmsCache:
         _check(dms_cache_export_positions(self._h, layer, ctypes.c_void_p(out.ctypes.data),
                                           _stream_ptr(stream)), "dms_cache_export_positions")
         return out
+
+    def export_kv(self, layer: int, stream=None):
+        """Stored rows of `layer` in head_dim order: (k, v, scales) with k, v of shape
+        [batch, kv_heads, capacity, 128] (uint16 bf16 bits, or uint8 E4M3 codes for an
+        fp8 cache) and scales [batch, kv_heads, capacity, 2] float32 (key, value) for fp8
+        caches, None otherwise; zero past each head's n_h."""
+        shape = (self.batch, self.kv_heads, self.capacity, self.head_dim)
+        fp8 = self.kv_format == DMS_KV_FP8_E4M3
+        dt = np.uint8 if fp8 else np.uint16
+        k, v = np.empty(shape, dtype=dt), np.empty(shape, dtype=dt)
+        sc = np.empty(shape[:3] + (2,), dtype=np.float32) if fp8 else None
+        _check(dms_cache_export_kv(self._h, layer, ctypes.c_void_p(k.ctypes.data),
+                                   ctypes.c_void_p(v.ctypes.data),
+                                   ctypes.c_void_p(sc.ctypes.data) if fp8 else None,
+                                   _stream_ptr(stream)), "dms_cache_export_kv")
+        return k, v, sc
 
     def layer_length(self, layer: int) -> int:
         code, n = dms_cache_layer_length(self._h, layer)

@@ -25,6 +25,8 @@ DMS_PREFILL_TCGEN05 = 0
 DMS_PREFILL_MMA_SYNC = 1
 DMS_DECODE_TILED = 0
 DMS_DECODE_SIMPLE = 1
+DMS_KV_BF16 = 0
+DMS_KV_FP8_E4M3 = 1
 
 # Every symbol the header declares (checked by the CPU test suite).
 EXPORTS = (
@@ -35,6 +37,7 @@ EXPORTS = (
     "dms_decode_attention_borrowed", "dms_append_and_decode_borrowed",
     "dms_prefill_workspace_bytes", "dms_prefill_attention", "dms_prefill_attention_borrowed",
     "dms_prefill_device_error", "dms_prefill_attention_ex", "dms_append_shared_prefix",
+    "dms_cache_export_kv",
 )
 
 
@@ -46,7 +49,8 @@ class dms_options(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("page_tokens", ctypes.c_int32),
                 ("pool_tokens", ctypes.c_int64), ("decode_kernel", ctypes.c_int32),
                 ("ctas_per_sm", ctypes.c_int32), ("min_pages_per_cta", ctypes.c_int32),
-                ("eviction_policy", ctypes.c_int32), ("reserved", ctypes.c_int32 * 4)]
+                ("eviction_policy", ctypes.c_int32), ("kv_format", ctypes.c_int32),
+                ("reserved", ctypes.c_int32 * 3)]
 
 
 class dms_stats(ctypes.Structure):
@@ -97,6 +101,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                           vp, ctypes.c_size_t, vp, vp]),
         "dms_cache_stats": (st, [vp, ctypes.POINTER(dms_stats), vp, vp]),
         "dms_cache_export_positions": (st, [vp, i32, vp, vp]),
+        "dms_cache_export_kv": (st, [vp, i32, vp, vp, vp, vp]),
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),
         "dms_status_string": (ctypes.c_char_p, [st]),
         "dms_decode_attention_paged_noalloc": (st, [vp, vp, vp, i32, i32, i32, vp, vp, i32, f32,

@@ -23,6 +23,8 @@ __device__ __forceinline__ void pdl_wait_prerequisites() {
 
 struct AppendParams {
   uint8_t* pool;
+  float* scales;        // fp8 format: [pool_pages][2][64]
+  int32_t fp8;          // the cache's pages hold fp8 E4M3 rows
   int32_t* pos;
   int32_t* page_table;  // this layer: [heads][max_pages]
   const int32_t* counts_cur;  // this layer, current buffer: [heads]
@@ -50,6 +52,55 @@ __device__ __forceinline__ void store_row(uint8_t* pool, int32_t page, uint32_t 
   uint8_t* dst = pool + (int64_t)page * kPageBytes + (lane >= 16 ? kHalfPageBytes : 0) +
                  swizzled_offset(row, chunk);
   *reinterpret_cast<uint4*>(dst) = val;
+}
+
+// fp8 E4M3 page format: the warp's K row (lanes 0-15, elements 8 l .. 8 l + 7 of
+// chunk l = lane & 15) and V row (lanes 16-31) are quantised with one scale per row,
+// scale = amax / 448 (IEEE fp32 division), code = E4M3(x / scale), round to nearest
+// even, saturated; a row of zeros gets scale 0 and zero codes.  K codes go to the
+// K rows of the page, V codes to the slot's column of V^T (k8_offset / vt8_offset).
+__device__ __forceinline__ void store_row_fp8(uint8_t* pool, float* scales, int32_t page,
+                                              uint32_t row, int lane, uint4 val) {
+  const uint32_t w[4] = {val.x, val.y, val.z, val.w};
+  float x[8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    x[2 * i] = __uint_as_float(w[i] << 16);
+    x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+  }
+  float a = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) a = fmaxf(a, fabsf(x[i]));
+#pragma unroll
+  for (int off = 1; off < 16; off <<= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, off));
+  const float scale = a == 0.f ? 0.f : __fdiv_rn(a, 448.f);
+  uint8_t* pg = pool + (int64_t)page * kPageBytesFp8;
+  const uint32_t d0 = 8u * (uint32_t)(lane & 15);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float lo = scale == 0.f ? 0.f : __fdiv_rn(x[2 * e], scale);
+    const float hi = scale == 0.f ? 0.f : __fdiv_rn(x[2 * e + 1], scale);
+    uint16_t pair;  // code of lo in the low byte, of hi in the high byte
+    asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(pair) : "f"(hi), "f"(lo));
+    const uint32_t d = d0 + 2u * (uint32_t)e;
+    if (lane < 16) {
+      // d even: the pair (d, d + 1) is 2 consecutive bytes of the thread's word
+      *reinterpret_cast<uint16_t*>(pg + k8_offset(row, d)) = pair;
+    } else {
+      pg[vt8_offset(row, d)] = (uint8_t)(pair & 0xffu);
+      pg[vt8_offset(row, d + 1)] = (uint8_t)(pair >> 8);
+    }
+  }
+  if ((lane & 15) == 0) scales[(int64_t)page * 2 * kPageTokens + (lane >= 16 ? kPageTokens : 0) + row] = scale;
+}
+
+// One K and V row into `row` of `page` in the cache's format (the whole warp calls it).
+__device__ __forceinline__ void store_kv_row(const AppendParams& p, int32_t page, uint32_t row,
+                                             int lane, uint4 val) {
+  if (p.fp8)
+    store_row_fp8(p.pool, p.scales, page, row, lane, val);
+  else
+    store_row(p.pool, page, row, lane, val);
 }
 
 __device__ __forceinline__ uint4 load_row_chunk(const uint16_t* k, const uint16_t* v,
@@ -110,7 +161,7 @@ __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
   if (!ok) return;
   slot = __shfl_sync(0xffffffffu, slot, 0);
   page = __shfl_sync(0xffffffffu, page, 0);
-  store_row(p.pool, page, (uint32_t)(slot & (kPageTokens - 1)), lane, val);
+  store_kv_row(p, page, (uint32_t)(slot & (kPageTokens - 1)), lane, val);
 }
 
 constexpr int kBulkThreads = 512;
@@ -263,7 +314,7 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
         if (sl[u] >= 0) {
           const int32_t page = pt[sl[u] / kPageTokens];
           const uint32_t row = (uint32_t)(sl[u] & (kPageTokens - 1));
-          store_row(p.pool, page, row, lane, val[u]);
+          store_kv_row(p, page, row, lane, val[u]);
           if (lane == 0) p.pos[(int64_t)page * kPageTokens + row] = (int32_t)(t0 + base + t + u);
         }
       }
@@ -312,12 +363,16 @@ __global__ void __launch_bounds__(256) share_prefix_kernel(const AppendParams p)
   for (int i = tid; i < own; i += blockDim.x) pt_dst[shared + i] = s_base + i;
   for (int i = tid; i < p.ring_len; i += blockDim.x)
     p.ring[(int64_t)dst * p.ring_len + i] = p.ring[(int64_t)src * p.ring_len + i];
-  // private copies of the pages that may still change (rows and positions)
+  // private copies of the pages that may still change (rows, scales and positions)
+  const int64_t page_bytes = p.fp8 ? kPageBytesFp8 : kPageBytes;
   for (int i = 0; i < own; ++i) {
     const int32_t from = pt_src[shared + i], to = s_base + i;
-    const uint4* a = reinterpret_cast<const uint4*>(p.pool + (int64_t)from * kPageBytes);
-    uint4* c = reinterpret_cast<uint4*>(p.pool + (int64_t)to * kPageBytes);
-    for (int e = tid; e < kPageBytes / 16; e += blockDim.x) c[e] = a[e];
+    const uint4* a = reinterpret_cast<const uint4*>(p.pool + (int64_t)from * page_bytes);
+    uint4* c = reinterpret_cast<uint4*>(p.pool + (int64_t)to * page_bytes);
+    for (int e = tid; e < page_bytes / 16; e += blockDim.x) c[e] = a[e];
+    if (p.fp8)
+      for (int e = tid; e < 2 * kPageTokens; e += blockDim.x)
+        p.scales[(int64_t)to * 2 * kPageTokens + e] = p.scales[(int64_t)from * 2 * kPageTokens + e];
     for (int e = tid; e < kPageTokens; e += blockDim.x)
       p.pos[(int64_t)to * kPageTokens + e] = p.pos[(int64_t)from * kPageTokens + e];
   }
@@ -341,6 +396,8 @@ AppendParams make_params(const Cache& c, int32_t layer, const void* k, const voi
                          const void* logit, int64_t logit_stride, int64_t t0, int32_t n) {
   AppendParams p;
   p.pool = c.pool;
+  p.scales = c.scales;
+  p.fp8 = c.fp8() ? 1 : 0;
   p.pos = c.pos;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
   p.counts_cur = c.counts_at(layer, t0);

@@ -22,6 +22,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 void free_device(Cache& c) {
   cudaFree(c.pool);
+  cudaFree(c.scales);
+  c.scales = nullptr;
   cudaFree(c.pos);
   cudaFree(c.page_table);
   cudaFree(c.counts);
@@ -68,9 +70,12 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   if (opt->page_tokens != 0 && opt->page_tokens != dms::kPageTokens) return DMS_ERR_INVALID_ARGUMENT;
   if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SIMPLE ||
       opt->ctas_per_sm < 0 || opt->ctas_per_sm > dms::kMaxCtasPerSm || opt->min_pages_per_cta < 0 ||
-      opt->eviction_policy < DMS_EVICT_DELAYED || opt->eviction_policy > DMS_EVICT_IMMEDIATE)
+      opt->eviction_policy < DMS_EVICT_DELAYED || opt->eviction_policy > DMS_EVICT_IMMEDIATE ||
+      opt->kv_format < DMS_KV_BF16 || opt->kv_format > DMS_KV_FP8_E4M3)
     return DMS_ERR_INVALID_ARGUMENT;
-  for (int i = 0; i < 4; ++i)
+  if (opt->kv_format == DMS_KV_FP8_E4M3 && opt->decode_kernel != DMS_DECODE_TILED)
+    return DMS_ERR_INVALID_ARGUMENT;  // only the tiled kernel reads fp8 pages
+  for (int i = 0; i < 3; ++i)
     if (opt->reserved[i] != 0) return DMS_ERR_INVALID_ARGUMENT;
   const int64_t heads = (int64_t)opt->batch * kv_heads;
   if (heads > dms::kMaxHeads) return DMS_ERR_INVALID_ARGUMENT;
@@ -93,6 +98,7 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
                      : (int64_t)layers * heads * c.max_pages;
   c.decode_kernel = opt->decode_kernel;
   c.eviction_policy = opt->eviction_policy;
+  c.kv_format = opt->kv_format;
   c.ctas_per_sm = opt->ctas_per_sm > 0 ? opt->ctas_per_sm : 1;
   c.min_pages_per_cta = opt->min_pages_per_cta > 0 ? opt->min_pages_per_cta : 2;
   if (c.pool_pages < 1 || c.pool_pages > 0x7fffffffLL) {
@@ -113,7 +119,9 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   }
 
   cudaError_t e = cudaSuccess;
-  if (e == cudaSuccess) e = alloc(&c.pool, (size_t)c.pool_pages * dms::kPageBytes);
+  if (e == cudaSuccess) e = alloc(&c.pool, (size_t)c.pool_pages * (size_t)c.page_bytes());
+  if (e == cudaSuccess && c.fp8())
+    e = alloc(&c.scales, (size_t)c.pool_pages * 2 * dms::kPageTokens);
   if (e == cudaSuccess) e = alloc(&c.pos, (size_t)c.pool_pages * dms::kPageTokens);
   if (e == cudaSuccess) e = alloc(&c.page_table, (size_t)layers * heads * c.max_pages);
   if (e == cudaSuccess) e = alloc(&c.counts, (size_t)layers * 2 * heads);
@@ -363,6 +371,64 @@ dms_status dms_cache_export_positions(dms_cache* h, int32_t layer, int32_t* host
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   cudaFree(dev);
   return e == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+}
+
+dms_status dms_cache_export_kv(dms_cache* h, int32_t layer, void* host_k, void* host_v,
+                               float* host_scales, void* stream) {
+  if (h == nullptr || host_k == nullptr || host_v == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  if (layer < 0 || layer >= c.layers || (c.fp8() && host_scales == nullptr))
+    return DMS_ERR_INVALID_ARGUMENT;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int64_t heads = c.heads, cap = c.capacity, D = dms::kHeadDim;
+  std::vector<int32_t> cnt((size_t)heads), pt((size_t)heads * c.max_pages);
+  if (cudaMemcpyAsync(cnt.data(), c.counts_at(layer, c.lengths[layer]), heads * sizeof(int32_t),
+                      cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaMemcpyAsync(pt.data(), c.page_table + (int64_t)layer * heads * c.max_pages,
+                      pt.size() * sizeof(int32_t), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return DMS_ERR_CUDA;
+  const size_t esize = c.fp8() ? 1 : 2;
+  memset(host_k, 0, (size_t)heads * cap * D * esize);
+  memset(host_v, 0, (size_t)heads * cap * D * esize);
+  if (c.fp8()) memset(host_scales, 0, (size_t)heads * cap * 2 * sizeof(float));
+  std::vector<uint8_t> page((size_t)c.page_bytes());
+  float sc[2 * dms::kPageTokens];
+  for (int64_t bh = 0; bh < heads; ++bh) {
+    const int32_t n = cnt[(size_t)bh];
+    if (n < 0 || n > cap) return DMS_ERR_STATE;
+    for (int32_t pg = 0; pg * dms::kPageTokens < n; ++pg) {
+      const int32_t id = pt[(size_t)bh * c.max_pages + pg];
+      if (id < 0 || id >= c.pool_pages) return DMS_ERR_STATE;
+      if (cudaMemcpy(page.data(), c.pool + (int64_t)id * c.page_bytes(), page.size(),
+                     cudaMemcpyDeviceToHost) != cudaSuccess ||
+          (c.fp8() && cudaMemcpy(sc, c.scales + (int64_t)id * 2 * dms::kPageTokens, sizeof(sc),
+                                 cudaMemcpyDeviceToHost) != cudaSuccess))
+        return DMS_ERR_CUDA;
+      for (int32_t r = 0; r < dms::kPageTokens && pg * dms::kPageTokens + r < n; ++r) {
+        const int64_t slot = (int64_t)pg * dms::kPageTokens + r;
+        const size_t row = ((size_t)bh * cap + slot) * D;
+        if (c.fp8()) {
+          uint8_t* ko = static_cast<uint8_t*>(host_k) + row;
+          uint8_t* vo = static_cast<uint8_t*>(host_v) + row;
+          for (uint32_t d = 0; d < (uint32_t)D; ++d) {
+            ko[d] = page[dms::k8_offset((uint32_t)r, d)];
+            vo[d] = page[dms::vt8_offset((uint32_t)r, d)];
+          }
+          host_scales[((size_t)bh * cap + slot) * 2] = sc[r];
+          host_scales[((size_t)bh * cap + slot) * 2 + 1] = sc[dms::kPageTokens + r];
+        } else {
+          uint16_t* ko = static_cast<uint16_t*>(host_k) + row;
+          uint16_t* vo = static_cast<uint16_t*>(host_v) + row;
+          for (uint32_t ch = 0; ch < 16; ++ch) {
+            memcpy(ko + 8 * ch, page.data() + dms::swizzled_offset((uint32_t)r, ch), 16);
+            memcpy(vo + 8 * ch, page.data() + dms::kHalfPageBytes + dms::swizzled_offset((uint32_t)r, ch), 16);
+          }
+        }
+      }
+    }
+  }
+  return DMS_OK;
 }
 
 dms_status dms_selftest_bounded_wait(int32_t arrive, int64_t limit_ns, void* stream) {

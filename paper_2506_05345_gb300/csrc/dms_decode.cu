@@ -51,8 +51,14 @@ constexpr int kQBytes = kMaxGroup * kRowBytes;                 // 4096
 constexpr int kPatchBytes = 2 * kRowBytes;                     // new K and V row (fused append)
 constexpr int kStageBytesPlain = 2 * kHalfPageBytes + kQBytes;  // 36864
 constexpr int kStageBytesFused = kStageBytesPlain + kPatchBytes;  // 37376
-__host__ __device__ constexpr int stage_bytes(bool fused) {
-  return fused ? kStageBytesFused : kStageBytesPlain;
+// fp8 E4M3 pages: K rows (8 KiB), V^T (8 KiB), the queries, the page's scales.
+constexpr int kStageBytesFp8 = 2 * kHalfPageBytesFp8 + kQBytes + kScaleBytes;  // 20992
+__host__ __device__ constexpr int stage_bytes(bool fused, bool fp8 = false) {
+  return fp8 ? kStageBytesFp8 : (fused ? kStageBytesFused : kStageBytesPlain);
+}
+// Bytes of one staged half (K rows, or V rows / V^T) of a page.
+__host__ __device__ constexpr int kv_half_bytes(bool fp8) {
+  return fp8 ? kHalfPageBytesFp8 : kHalfPageBytes;
 }
 // Largest batch * kv_heads the fused append + decode kernel takes (its per-head
 // slot table must fit next to the stages); larger caches use the two kernels.
@@ -60,9 +66,11 @@ constexpr int kMaxHeadsFused = 4000;
 // Merge rows (one per query head, 128 floats of head_dim) are padded to 132
 // floats: the stores of an O^T accumulator fragment then hit 32 distinct banks.
 constexpr int kMergeRow = kHeadDim + 4;
-// Pipeline depth per CTA: 4 stages with one CTA per SM, 2 stages with two.
+// Pipeline depth per CTA: 4 stages with one CTA per SM, 2 stages with two; fp8 pages
+// are half the size, so 7 stages keep about as many bytes in flight.
 constexpr int kStagesOneCta = 4;
 constexpr int kStagesTwoCta = 2;
+constexpr int kStagesFp8 = 7;
 
 // Shared-memory plan that depends on the number of 8-head n-tiles (NT).
 template <int NT>
@@ -75,6 +83,7 @@ struct Plan {
 
 struct DecodeParams {
   uint8_t* pool;
+  const float* scales;        // fp8 pages: [pool_pages][2][64] key / value row scales
   int32_t* page_table;        // this layer
   const int32_t* counts;      // this layer, current buffer
   const __nv_bfloat16* q;
@@ -161,10 +170,10 @@ __device__ __forceinline__ int head_of_page(const int32_t* pstart, int heads, in
   return lo - 1;
 }
 
-template <int NT, bool kFused>
+template <int NT, bool kFused, bool kFp8 = false>
 size_t tiled_smem_bytes(int heads, int stages) {
   using PL = Plan<NT>;
-  return (size_t)stages * stage_bytes(kFused) +
+  return (size_t)stages * stage_bytes(kFused, kFp8) +
          (size_t)PL::kSlots * (PL::kSlotOFloats + PL::kSlotMLFloats) * 4 +
          (size_t)(2 * stages + 2 * PL::kSlots) * sizeof(uint64_t) + 64 +
          (size_t)((kFused ? 3 : 2) * heads + 1) * sizeof(int32_t);
@@ -205,12 +214,16 @@ struct PageWalk {
   }
 };
 
-template <int kStages, int NT, bool kFused>
-__global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
+template <int kStages, int NT, bool kFused, bool kFp8 = false>
+__global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
     decode_tiled_kernel(const DecodeParams p) {
+  static_assert(!(kFused && kFp8), "the fused append writes bf16 pages only");
   using PL = Plan<NT>;
   constexpr int HP = PL::kHeadsPad;
-  constexpr int kStageBytes = stage_bytes(kFused);
+  constexpr int kStageBytes = stage_bytes(kFused, kFp8);
+  constexpr int kKvHalf = kv_half_bytes(kFp8);     // offset of the V half in a stage
+  constexpr int kOffQ = 2 * kKvHalf;                // the group's queries
+  constexpr int kOffScales = kOffQ + kQBytes;       // fp8: key scales [64], value scales [64]
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
   float* merge_o = reinterpret_cast<float*>(smem + kStages * kStageBytes);  // [slots][4][HP][132]
@@ -381,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
       if (seg_start) {
         const int b = h_i / p.kv_heads, hk = h_i - b * p.kv_heads;
         const __nv_bfloat16* qsrc = p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
-        bulk_copy_g2s(st + 2 * kHalfPageBytes, qsrc, (uint32_t)G * kRowBytes, &full_bar[s]);
+        bulk_copy_g2s(st + kOffQ, qsrc, (uint32_t)G * kRowBytes, &full_bar[s]);
       }
       if constexpr (kFused) {
         if (patch) {  // the new token's K and V rows, as given (unpermuted)
@@ -453,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
             mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.ctrl);
           }
           const bool seg_start = (itg == 0) || (pg_i == 0);
-          const uint32_t kv_bytes = (uint32_t)nv_i * kRowBytes;
+          const uint32_t kv_bytes = (uint32_t)nv_i * (kFp8 ? 128u : (uint32_t)kRowBytes);
           const uint32_t q_bytes = seg_start ? (uint32_t)G * kRowBytes : 0u;
           uint8_t* st = stages + s * kStageBytes;
           bool patch = false;
@@ -461,10 +474,23 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
             patch = (int32_t)(s_slot[h_i] & 0x3fffffffu) / kPageTokens == pg_i;
             s_misc[8 + s] = page_i;
           }
-          mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + q_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
-          const uint8_t* src = p.pool + (int64_t)(page_i < 0 ? 0 : page_i) * kPageBytes;
-          bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
-          bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+          const int64_t page0 = page_i < 0 ? 0 : page_i;
+          if constexpr (kFp8) {
+            // valid K rows; all of V^T (its rows interleave the slots) and the scales
+            mbar_arrive_expect_tx(&full_bar[s], kv_bytes + (uint32_t)kHalfPageBytesFp8 +
+                                                    (uint32_t)kScaleBytes + q_bytes);
+            const uint8_t* src = p.pool + page0 * kPageBytesFp8;
+            bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
+            bulk_copy_g2s(st + kKvHalf, src + kHalfPageBytesFp8, kHalfPageBytesFp8, &full_bar[s]);
+            bulk_copy_g2s(st + kOffScales, p.scales + page0 * 2 * kPageTokens, kScaleBytes,
+                          &full_bar[s]);
+          } else {
+            mbar_arrive_expect_tx(&full_bar[s],
+                                  2 * kv_bytes + q_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
+            const uint8_t* src = p.pool + page0 * kPageBytes;
+            bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
+            bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+          }
           if (waited) {
             issue_inputs(s, h_i, pg_i, seg_start, patch);
           } else {
@@ -700,7 +726,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
     }
 
     if (seg_start) {
-      const uint32_t qbase = smem_addr(st + 2 * kHalfPageBytes);
+      const uint32_t qbase = smem_addr(st + kOffQ);
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
         const int row = 8 * nt + (lane & 7);
@@ -720,6 +746,15 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
       }
+      if constexpr (kFp8) {  // the fp8 path multiplies in f16
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            qb[kk][nt][0] = bf16x2_to_f16x2(qb[kk][nt][0]);
+            qb[kk][nt][1] = bf16x2_to_f16x2(qb[kk][nt][1]);
+          }
+      }
       // Lane 0 holds (d = 0, 1) of the group's first query head in the low / high half.
       if (p.zero_first && lane == 0) qb[0][0][0] &= 0xffff0000u;
     }
@@ -731,8 +766,33 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int e = 0; e < 4; ++e) sa[nt][e] = sb[nt][e] = 0.f;
-      const uint32_t kbase = smem_addr(st);
-      {
+      if constexpr (kFp8) {
+        // rows tb + g and tb + g + 8; the 16-byte chunk of k-steps 4 kg .. 4 kg + 3 holds
+        // this thread's codes (d = 16 kk + {2c, 2c+1, 2c+8, 2c+9}) in word kk % 4
+#pragma unroll
+        for (int kg = 0; kg < 2; ++kg) {
+          const uint4 w0 = *reinterpret_cast<const uint4*>(
+              st + (tb + g) * 128 + (((4 * kg + c4) ^ g) << 4));
+          const uint4 w1 = *reinterpret_cast<const uint4*>(
+              st + (tb + g + 8) * 128 + (((4 * kg + c4) ^ g) << 4));
+          const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int kk = 4 * kg + i;
+            uint32_t a[4];
+            a[0] = e4m3x2_to_f16x2(x0[i]);
+            a[1] = e4m3x2_to_f16x2(x1[i]);
+            a[2] = e4m3x2_to_f16x2(x0[i] >> 16);
+            a[3] = e4m3x2_to_f16x2(x1[i] >> 16);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              if (kk & 1) mma_f16_16816(sb[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
+              else mma_f16_16816(sa[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
+            }
+          }
+        }
+      } else {
+        const uint32_t kbase = smem_addr(st);
         const uint32_t row = (uint32_t)(tb + (mi & 1) * 8 + (lane & 7));
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
@@ -747,15 +807,22 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
       }
       // ---- mask tokens past n_valid, online softmax per head (column), P^T fragments
       const bool v0 = tb + g < nvalid, v1 = tb + g + 8 < nvalid;
+      // score scale of tokens tb + g and tb + g + 8 (fp8: times the keys' row scales)
+      float sl0 = p.scale_log2, sl1 = p.scale_log2;
+      if constexpr (kFp8) {
+        const float* ksc = reinterpret_cast<const float*>(st + kOffScales);
+        sl0 *= ksc[tb + g];
+        sl1 *= ksc[tb + g + 8];
+      }
       bool rescale = false;
       float ce[NT], co[NT];
       uint32_t pb[NT][2];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        const float s0 = v0 ? (sa[nt][0] + sb[nt][0]) * p.scale_log2 : -INFINITY;
-        const float s1 = v0 ? (sa[nt][1] + sb[nt][1]) * p.scale_log2 : -INFINITY;
-        const float s2 = v1 ? (sa[nt][2] + sb[nt][2]) * p.scale_log2 : -INFINITY;
-        const float s3 = v1 ? (sa[nt][3] + sb[nt][3]) * p.scale_log2 : -INFINITY;
+        const float s0 = v0 ? (sa[nt][0] + sb[nt][0]) * sl0 : -INFINITY;
+        const float s1 = v0 ? (sa[nt][1] + sb[nt][1]) * sl0 : -INFINITY;
+        const float s2 = v1 ? (sa[nt][2] + sb[nt][2]) * sl1 : -INFINITY;
+        const float s3 = v1 ? (sa[nt][3] + sb[nt][3]) * sl1 : -INFINITY;
         float xe = fmaxf(s0, s2), xo = fmaxf(s1, s3);
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
@@ -773,8 +840,13 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
         lo[nt] = lo[nt] * co[nt] + (p1 + p3);
         rescale |= (ce[nt] != 1.f) || (co[nt] != 1.f);
         // (token g, heads 2c..) -> transpose -> (head g, tokens 2c..): the B operand
-        pb[nt][0] = movmatrix_trans(pack_bf16x2(p0, p1));
-        pb[nt][1] = movmatrix_trans(pack_bf16x2(p2, p3));
+        if constexpr (kFp8) {
+          pb[nt][0] = movmatrix_trans(pack_f16x2(p0, p1));
+          pb[nt][1] = movmatrix_trans(pack_f16x2(p2, p3));
+        } else {
+          pb[nt][0] = movmatrix_trans(pack_bf16x2(p0, p1));
+          pb[nt][1] = movmatrix_trans(pack_bf16x2(p2, p3));
+        }
       }
       if (__any_sync(0xffffffffu, rescale)) {
 #pragma unroll
@@ -788,14 +860,36 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesOneCta ? 1 : 2)
           }
       }
       // ---- O^T += V^T P^T over head_dim (8 m-tiles of 16)
-      const uint32_t vbase = smem_addr(st + kHalfPageBytes);
       uint32_t mk_lo = 0xffffffffu, mk_hi = 0xffffffffu;
       if (tb + 16 > nvalid) {  // stale rows past n_valid must not reach the tensor cores
         const int t = tb + 2 * c4;
         mk_lo = (t < nvalid ? 0x0000ffffu : 0u) | (t + 1 < nvalid ? 0xffff0000u : 0u);
         mk_hi = (t + 8 < nvalid ? 0x0000ffffu : 0u) | (t + 9 < nvalid ? 0xffff0000u : 0u);
       }
-      {
+      if constexpr (kFp8) {
+        // V^T rows d = 16 mt + g and + 8: one word holds the codes of tokens tb + {2c, 2c+1,
+        // 2c+8, 2c+9}; each value times its token's scale (f16), stale tokens masked after
+        const float* vsc = reinterpret_cast<const float*>(st + kOffScales) + kPageTokens;
+        const uint32_t sv01 = pack_f16x2(vsc[tb + 2 * c4], vsc[tb + 2 * c4 + 1]);
+        const uint32_t sv89 = pack_f16x2(vsc[tb + 2 * c4 + 8], vsc[tb + 2 * c4 + 9]);
+        const int blk = tb >> 4;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          const int d0 = 16 * mt + g, d1 = d0 + 8;
+          const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
+              st + kKvHalf + d0 * 64 + ((blk ^ ((d0 >> 1) & 3)) << 4) + 4 * c4);
+          const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
+              st + kKvHalf + d1 * 64 + ((blk ^ ((d1 >> 1) & 3)) << 4) + 4 * c4);
+          uint32_t a[4];
+          a[0] = hmul2_u32(e4m3x2_to_f16x2(w0), sv01) & mk_lo;
+          a[1] = hmul2_u32(e4m3x2_to_f16x2(w1), sv01) & mk_lo;
+          a[2] = hmul2_u32(e4m3x2_to_f16x2(w0 >> 16), sv89) & mk_hi;
+          a[3] = hmul2_u32(e4m3x2_to_f16x2(w1 >> 16), sv89) & mk_hi;
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) mma_f16_16816(o[mt][nt], a, pb[nt][0], pb[nt][1]);
+        }
+      } else {
+        const uint32_t vbase = smem_addr(st + kHalfPageBytes);
         const uint32_t row = (uint32_t)(tb + (mi >> 1) * 8 + (lane & 7));
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) {
@@ -1099,6 +1193,10 @@ cudaError_t prepare_decode(const Cache& c) {
       tiled_smem_bytes<1, true>(kMaxHeadsFused, kStagesOneCta));
   set(decode_tiled_kernel<kStagesOneCta, 2, true>,
       tiled_smem_bytes<2, true>(kMaxHeadsFused, kStagesOneCta));
+  set(decode_tiled_kernel<kStagesFp8, 1, false, true>,
+      tiled_smem_bytes<1, false, true>(kMaxHeads, kStagesFp8));
+  set(decode_tiled_kernel<kStagesFp8, 2, false, true>,
+      tiled_smem_bytes<2, false, true>(kMaxHeads, kStagesFp8));
   return e;
 }
 
@@ -1108,7 +1206,7 @@ namespace {
 // prerequisites itself); the variant is picked by CTAs per SM, group size and
 // whether the single-token append is fused in.
 cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cudaStream_t stream,
-                         bool programmatic, bool fused) {
+                         bool programmatic, bool fused, bool fp8 = false) {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1117,6 +1215,15 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = programmatic ? 1 : 0;
+  if (fp8) {  // one CTA per SM, never fused
+    cfg.gridDim = dim3(num_sms);
+    if (p.group <= 8) {
+      cfg.dynamicSmemBytes = tiled_smem_bytes<1, false, true>(p.heads, kStagesFp8);
+      return cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesFp8, 1, false, true>, p);
+    }
+    cfg.dynamicSmemBytes = tiled_smem_bytes<2, false, true>(p.heads, kStagesFp8);
+    return cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesFp8, 2, false, true>, p);
+  }
   const bool two = !fused && ctas_per_sm >= 2;
   const int stages = two ? kStagesTwoCta : kStagesOneCta;
   cfg.gridDim = dim3(num_sms * (two ? ctas_per_sm : 1));
@@ -1143,6 +1250,7 @@ DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* ou
   DecodeParams p = {};
   p.state_ready = (c.last_layer != layer) ? 1 : 0;
   p.pool = c.pool;
+  p.scales = c.scales;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
   p.counts = c.counts_at(layer, c.lengths[layer]);
   p.q = static_cast<const __nv_bfloat16*>(q);
@@ -1166,11 +1274,12 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
                                 cudaStream_t stream) {
   DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
   p.zero_first = zero_first ? 1 : 0;
-  return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false);
+  return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false, c.fp8());
 }
 
 bool append_decode_fusable(const Cache& c) {
-  return c.decode_kernel == DMS_DECODE_TILED && c.heads <= kMaxHeadsFused && c.ctas_per_sm < 2;
+  return c.decode_kernel == DMS_DECODE_TILED && !c.fp8() && c.heads <= kMaxHeadsFused &&
+         c.ctas_per_sm < 2;
 }
 
 // Single-token append of position lengths[layer] fused with the decode (requires

@@ -7,6 +7,17 @@
 //               copy of whole rows therefore lands in shared memory already in a
 //               bank-conflict-free order for ldmatrix (8 consecutive rows hit 8 distinct
 //               16-byte bank groups).
+//   (fp8 E4M3 format, DMS_KV_FP8_E4M3: pages of 16 KiB)
+//   pool        [pool_pages][16384] bytes: 64 K rows of 128 codes, then V transposed,
+//               128 rows (one per head_dim index d) of 64 codes (one per slot).  Both
+//               are laid out for the tiled decode kernel's m16n8k16 A fragments: in a
+//               K row, the 16-code block of k-step kk sits in the 16-byte chunk group
+//               kk / 4 and the four codes one thread needs (d = 16 kk + {2c, 2c+1,
+//               2c+8, 2c+9}) are 4 consecutive bytes; in a V^T row the four codes of
+//               tokens {2c, 2c+1, 2c+8, 2c+9} of a 16-slot block likewise.  16-byte
+//               chunks are XOR-permuted by the row (K: row & 7; V^T: (d >> 1) & 3) so
+//               a warp's loads hit distinct banks.  k8_offset / vt8_offset below.
+//   scales      [pool_pages][2][64] fp32         per-slot key and value scales.
 //   pos         [pool_pages][64] int32          position held by each slot (inspection only;
 //                                               decode never reads it).
 //   page_table  [layers][heads][max_pages] int32 page of slot s is page_table[.][s / 64].
@@ -44,6 +55,9 @@ constexpr int kPageTokens = 64;
 constexpr int kRowBytes = kHeadDim * 2;                       // 256
 constexpr int kHalfPageBytes = kPageTokens * kRowBytes;       // 16384
 constexpr int kPageBytes = 2 * kHalfPageBytes;                // 32768
+constexpr int kPageBytesFp8 = 16384;                          // fp8 page: K 8 KiB, V^T 8 KiB
+constexpr int kHalfPageBytesFp8 = 8192;
+constexpr int kScaleBytes = 2 * kPageTokens * 4;              // per page: key, value scales
 constexpr int kMaxGroup = 16;                                 // query heads per KV head
 constexpr int kMaxHeads = 4096;                               // batch * kv_heads
 constexpr int kMaxCtasPerSm = 4;
@@ -66,6 +80,9 @@ struct Cache {
   int64_t pool_pages = 0;
   int32_t decode_kernel = 0, ctas_per_sm = 1, min_pages_per_cta = 2;
   int32_t eviction_policy = DMS_EVICT_DELAYED;
+  int32_t kv_format = DMS_KV_BF16;
+  bool fp8() const { return kv_format == DMS_KV_FP8_E4M3; }
+  int64_t page_bytes() const { return fp8() ? kPageBytesFp8 : kPageBytes; }
   // Position offset of the token whose decision evicts a given token: 0 for delayed
   // eviction (its own decision), window for the immediate-eviction ablation.
   int64_t decider() const { return eviction_policy == DMS_EVICT_IMMEDIATE ? window : 0; }
@@ -73,6 +90,7 @@ struct Cache {
   int64_t piece_capacity = 0;
 
   uint8_t* pool = nullptr;
+  float* scales = nullptr;  // fp8 format only
   int32_t* pos = nullptr;
   int32_t* page_table = nullptr;
   int32_t* counts = nullptr;
@@ -111,6 +129,28 @@ __device__ __forceinline__ uint32_t decision_from_bf16(uint16_t bits) {
 // Byte offset of logical 16-byte chunk `chunk` of row `row` inside a half page.
 __host__ __device__ __forceinline__ uint32_t swizzled_offset(uint32_t row, uint32_t chunk) {
   return row * kRowBytes + ((chunk ^ (row & 7u)) << 4);
+}
+
+// fp8 page format.  Position of logical element d (0..127) of key row `row` (0..63)
+// inside the page: k-step kk = d / 16, j = d % 16; thread c = (j & 7) / 2 of an
+// m16n8k16 fragment needs j = 2c, 2c + 1, 2c + 8, 2c + 9, stored at bytes 0..3 of word
+// kk % 4 of chunk 4 (kk / 4) + c, the chunk XOR-ed with row & 7.
+__host__ __device__ __forceinline__ uint32_t fp8_pair_index(uint32_t j) {
+  return (j & 1u) | ((j >> 3) << 1);
+}
+__host__ __device__ __forceinline__ uint32_t k8_offset(uint32_t row, uint32_t d) {
+  const uint32_t kk = d >> 4, j = d & 15u;
+  const uint32_t chunk = (4u * (kk >> 2) + ((j & 7u) >> 1)) ^ (row & 7u);
+  return row * 128u + (chunk << 4) + 4u * (kk & 3u) + fp8_pair_index(j);
+}
+// Position of the value of slot `slot` (0..63) at head_dim index d in the V^T half:
+// row d of 64 bytes, 16-slot block slot / 16 in chunk (slot / 16) ^ ((d >> 1) & 3), the
+// slot's code at byte 4 c + pair index inside it (c, pair index of j = slot % 16 as for K).
+__host__ __device__ __forceinline__ uint32_t vt8_offset(uint32_t slot, uint32_t d) {
+  const uint32_t j = slot & 15u;
+  const uint32_t chunk = (slot >> 4) ^ ((d >> 1) & 3u);
+  return (uint32_t)kHalfPageBytesFp8 + d * 64u + (chunk << 4) + 4u * ((j & 7u) >> 1) +
+         fp8_pair_index(j);
 }
 
 // Launchers (defined in the .cu files).  A decision logit sits at logit[i * logit_stride]

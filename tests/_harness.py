@@ -3,7 +3,9 @@
 The full appended history (K, V, logits) of the layer under test is kept on the
 device so that any (sequence, KV head) can be handed to the oracle at any step.
 Tolerances: retained sets bit-exact; attention outputs max-abs <= 2e-2 and
-mean-abs <= 2e-3 against the fp64 oracle on the same bf16 inputs.
+mean-abs <= 2e-3 against the fp64 oracle on the same bf16 inputs.  An fp8 cache
+(kv_format=DMS_KV_FP8_E4M3) is checked against the oracle's attention over its own
+quantisation of the history; its stored codes and scales bit-exact.
 """
 from __future__ import annotations
 
@@ -23,6 +25,7 @@ class Run:
                  capacity: int | None = None, fused: bool = False, **cache_kw):
         self.wl, self.layer, self.dev = wl, layer, torch.device(device)
         self.fused = fused  # decode steps through dms_append_and_decode
+        self.fp8 = cache_kw.get("kv_format", dms.DMS_KV_BF16) == dms.DMS_KV_FP8_E4M3
         self.T = capacity or wl.context
         B, H, D = wl.batch, wl.kv_heads, wl.head_dim
         self.cache = dms.DmsCache(layers=1, kv_heads=H, window=wl.window, capacity=self.T,
@@ -109,7 +112,13 @@ class Run:
             k = workloads.bf16_bits(self.K[b, :j + 1, h])
             v = workloads.bf16_bits(self.V[b, :j + 1, h])
             lg = workloads.bf16_bits(self.L[b, :j + 1, h])
-            ref = oracle.decode(Q[b, h * G:(h + 1) * G], k, v, lg, j, self.wl.window)
+            if self.fp8:
+                kc, ks = oracle.quantize_rows_e4m3(k)
+                vc, vs = oracle.quantize_rows_e4m3(v)
+                ref = oracle.decode_fp8(Q[b, h * G:(h + 1) * G], kc, ks, vc, vs, lg, j,
+                                        self.wl.window)
+            else:
+                ref = oracle.decode(Q[b, h * G:(h + 1) * G], k, v, lg, j, self.wl.window)
             errs.append(np.abs(got[b, h * G:(h + 1) * G].astype(np.float64) - ref).ravel())
         e = np.concatenate(errs)
         assert np.all(np.isfinite(got)), "non-finite output"
@@ -117,6 +126,29 @@ class Run:
             self.errs.append(e)
         assert e.max() <= MAX_ABS, e.max()
         return e
+
+    def check_codes(self, heads=None):
+        """Stored rows of every retained slot equal the input row at the slot's position:
+        bf16 bits, or (fp8) the oracle's E4M3 codes and fp32 scales, bit for bit."""
+        k_st, v_st, sc = self.cache.export_kv(0)
+        pos = self.cache.export_positions(0)
+        counts = self.cache.stats(with_counts=True)["counts"][0]
+        B, H = self.wl.batch, self.wl.kv_heads
+        heads = heads if heads is not None else [(b, h) for b in range(B) for h in range(H)]
+        for b, h in heads:
+            n = int(counts[b, h])
+            p = pos[b, h, :n]
+            k = workloads.bf16_bits(self.K[b, :, h])[p]
+            v = workloads.bf16_bits(self.V[b, :, h])[p]
+            if self.fp8:
+                kc, ks = oracle.quantize_rows_e4m3(k)
+                vc, vs = oracle.quantize_rows_e4m3(v)
+                assert np.array_equal(k_st[b, h, :n], kc), (b, h)
+                assert np.array_equal(v_st[b, h, :n], vc), (b, h)
+                assert np.array_equal(sc[b, h, :n, 0], ks) and np.array_equal(sc[b, h, :n, 1], vs)
+            else:
+                assert np.array_equal(k_st[b, h, :n], k) and np.array_equal(v_st[b, h, :n], v)
+            assert not k_st[b, h, n:].any() and not v_st[b, h, n:].any()
 
     def summary(self):
         e = np.concatenate(self.errs) if self.errs else np.zeros(1)

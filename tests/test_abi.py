@@ -73,3 +73,23 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert code == _native.DMS_ERR_INVALID_ARGUMENT
     assert lib.dms_append_and_evict(None, 0, None, None, None, 1, None) == 1
     assert lib.dms_decode_attention(None, 0, None, None, 4, 0.0, None) == 1
+
+
+def test_kv_format_options_checked_on_host(lib):
+    """The fp8 page format is taken only by the tiled decode kernel; unknown formats and
+    nonzero reserved fields are rejected before any device call."""
+    opt = _native.dms_options()
+    opt.batch = 1
+    opt.kv_format = _native.DMS_KV_FP8_E4M3
+    opt.decode_kernel = _native.DMS_DECODE_SIMPLE
+    code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
+    assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None
+    opt.decode_kernel = _native.DMS_DECODE_TILED
+    opt.kv_format = 2
+    code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
+    assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None
+    opt.kv_format = 0
+    opt.reserved[2] = 1
+    code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
+    assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None
+    assert lib.dms_cache_export_kv(None, 0, None, None, None, None) == 1
