@@ -42,6 +42,7 @@ FALLBACK_HBM_GBS = 6800.0
 DECODE_SRCS = [os.path.join(ROOT, "paper_2506_05345_gb300", "csrc", f)
                for f in ("dms_decode.cu", "dms_ptx.cuh", "dms_internal.cuh")]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
+TRAFFIC_FILE_FP8 = os.path.join(ROOT, "profiles", "decode_traffic_fp8.json")
 
 
 def parse():
@@ -124,11 +125,11 @@ def decode_source_sha():
     return h.hexdigest()[:16]
 
 
-def traffic_per_launch(units_per_launch):
+def traffic_per_launch(units_per_launch, fp8=False):
     """DRAM bytes per decode launch from the committed ncu summary, scaled to this
     launch's units; None if there is none or the kernel changed since."""
     try:
-        with open(TRAFFIC_FILE) as f:
+        with open(TRAFFIC_FILE_FP8 if fp8 else TRAFFIC_FILE) as f:
             t = json.load(f)
     except Exception:
         return None
@@ -593,7 +594,7 @@ def run_ours(args, wl, world, rank, local, pg):
 
     peak, peak_kind = measured_peak()
     achieved_gbs = units_per_launch * bytes_per_unit / dec_avg_s / 1e9
-    traffic = None if args.kv_fp8 else traffic_per_launch(units_per_launch)
+    traffic = traffic_per_launch(units_per_launch, fp8=args.kv_fp8)
     res = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K_,
         "warmup": W_, "ms_per_step": elapsed_max_ms / K_, "higher_is_better": True,
