@@ -56,7 +56,7 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--kv-fp8", action="store_true",
-                    help="fp8 E4M3 page format (per-row scales); append and decode as two launches")
+                    help="fp8 E4M3 page format (per-row fp32 scales)")
     ap.add_argument("--ctas-per-sm", type=int, default=0)
     ap.add_argument("--min-pages", type=int, default=0)
     ap.add_argument("--separate", action="store_true",
@@ -261,8 +261,6 @@ def run_ours(args, wl, world, rank, local, pg):
     decode_needed = max(wl.decode_steps, W_ + K_ + K2 + E_W + E_K)
     capacity = wl.prefill_tokens + decode_needed
     seed_tag = replica_tag(rank)
-    if args.kv_fp8:
-        args.separate = True  # the fp8 format has no fused append + decode kernel
     cache = dms.DmsCache(layers=L, kv_heads=H, window=wl.window, capacity=capacity, batch=B,
                          ctas_per_sm=args.ctas_per_sm, min_pages_per_cta=args.min_pages,
                          kv_format=dms.DMS_KV_FP8_E4M3 if args.kv_fp8 else dms.DMS_KV_BF16)

@@ -51,10 +51,12 @@ constexpr int kQBytes = kMaxGroup * kRowBytes;                 // 4096
 constexpr int kPatchBytes = 2 * kRowBytes;                     // new K and V row (fused append)
 constexpr int kStageBytesPlain = 2 * kHalfPageBytes + kQBytes;  // 36864
 constexpr int kStageBytesFused = kStageBytesPlain + kPatchBytes;  // 37376
-// fp8 E4M3 pages: K rows (8 KiB), V^T (8 KiB), the queries, the page's scales.
+// fp8 E4M3 pages: K rows (8 KiB), V^T (8 KiB), the queries, the page's scales (and, fused,
+// the new token's bf16 K and V rows).
 constexpr int kStageBytesFp8 = 2 * kHalfPageBytesFp8 + kQBytes + kScaleBytes;  // 20992
 __host__ __device__ constexpr int stage_bytes(bool fused, bool fp8 = false) {
-  return fp8 ? kStageBytesFp8 : (fused ? kStageBytesFused : kStageBytesPlain);
+  return fp8 ? kStageBytesFp8 + (fused ? kPatchBytes : 0)
+             : (fused ? kStageBytesFused : kStageBytesPlain);
 }
 // Bytes of one staged half (K rows, or V rows / V^T) of a page.
 __host__ __device__ constexpr int kv_half_bytes(bool fp8) {
@@ -71,6 +73,7 @@ constexpr int kMergeRow = kHeadDim + 4;
 constexpr int kStagesOneCta = 4;
 constexpr int kStagesTwoCta = 2;
 constexpr int kStagesFp8 = 7;
+constexpr int kStagesFp8Fused = 6;  // room for the fused variant's per-head slot table
 
 // Shared-memory plan that depends on the number of 8-head n-tiles (NT).
 template <int NT>
@@ -83,7 +86,7 @@ struct Plan {
 
 struct DecodeParams {
   uint8_t* pool;
-  const float* scales;        // fp8 pages: [pool_pages][2][64] key / value row scales
+  float* scales;              // fp8 pages: [pool_pages][2][64] key / value row scales
   int32_t* page_table;        // this layer
   const int32_t* counts;      // this layer, current buffer
   const __nv_bfloat16* q;
@@ -217,13 +220,13 @@ struct PageWalk {
 template <int kStages, int NT, bool kFused, bool kFp8 = false>
 __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
     decode_tiled_kernel(const DecodeParams p) {
-  static_assert(!(kFused && kFp8), "the fused append writes bf16 pages only");
   using PL = Plan<NT>;
   constexpr int HP = PL::kHeadsPad;
   constexpr int kStageBytes = stage_bytes(kFused, kFp8);
   constexpr int kKvHalf = kv_half_bytes(kFp8);     // offset of the V half in a stage
   constexpr int kOffQ = 2 * kKvHalf;                // the group's queries
   constexpr int kOffScales = kOffQ + kQBytes;       // fp8: key scales [64], value scales [64]
+  constexpr int kOffPatch = kFp8 ? kStageBytesFp8 : kStageBytesPlain;  // fused: new K, V rows
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
   float* merge_o = reinterpret_cast<float*>(smem + kStages * kStageBytes);  // [slots][4][HP][132]
@@ -398,9 +401,9 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       }
       if constexpr (kFused) {
         if (patch) {  // the new token's K and V rows, as given (unpermuted)
-          bulk_copy_g2s(st + kStageBytesPlain, p.k_new + (int64_t)h_i * kHeadDim, kRowBytes,
+          bulk_copy_g2s(st + kOffPatch, p.k_new + (int64_t)h_i * kHeadDim, kRowBytes,
                         &full_bar[s]);
-          bulk_copy_g2s(st + kStageBytesPlain + kRowBytes, p.v_new + (int64_t)h_i * kHeadDim,
+          bulk_copy_g2s(st + kOffPatch + kRowBytes, p.v_new + (int64_t)h_i * kHeadDim,
                         kRowBytes, &full_bar[s]);
         }
         if (pg_i == s_pstart[h_i + 1] - s_pstart[h_i] - 1) {  // owner of the head's last page
@@ -478,7 +481,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
           if constexpr (kFp8) {
             // valid K rows; all of V^T (its rows interleave the slots) and the scales
             mbar_arrive_expect_tx(&full_bar[s], kv_bytes + (uint32_t)kHalfPageBytesFp8 +
-                                                    (uint32_t)kScaleBytes + q_bytes);
+                                                    (uint32_t)kScaleBytes + q_bytes +
+                                                    (patch ? (uint32_t)kPatchBytes : 0u));
             const uint8_t* src = p.pool + page0 * kPageBytesFp8;
             bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
             bulk_copy_g2s(st + kKvHalf, src + kHalfPageBytesFp8, kHalfPageBytesFp8, &full_bar[s]);
@@ -706,12 +710,63 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       const uint32_t sl = s_slot[walk.h];
       const int32_t slot = (int32_t)(sl & 0x3fffffffu);
       const uint32_t r = (uint32_t)(slot % kPageTokens);
-      if (slot / kPageTokens == walk.pg && (int)(r >> 4) == warp) {
+      if (kFp8 && slot / kPageTokens == walk.pg && (int)(r >> 4) == warp) {
+        // fp8 pages: the warp whose 16 rows hold the new token quantises its K and V rows
+        // (scale = amax / 448, code = E4M3(x / scale), as the append kernels do) into the
+        // staged page and the pool; lane l takes head_dim 4 l .. 4 l + 3 of both rows.
+        const int page = s_misc[8 + s];
+        const uint2 kw = *reinterpret_cast<const uint2*>(st + kOffPatch + lane * 8);
+        const uint2 vw = *reinterpret_cast<const uint2*>(st + kOffPatch + kRowBytes + lane * 8);
+        const uint32_t in[2][2] = {{kw.x, kw.y}, {vw.x, vw.y}};
+#pragma unroll
+        for (int kv = 0; kv < 2; ++kv) {
+          float x[4];
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            x[2 * i] = __uint_as_float(in[kv][i] << 16);
+            x[2 * i + 1] = __uint_as_float(in[kv][i] & 0xffff0000u);
+          }
+          float a = fmaxf(fmaxf(fabsf(x[0]), fabsf(x[1])), fmaxf(fabsf(x[2]), fabsf(x[3])));
+#pragma unroll
+          for (int off = 1; off < 32; off <<= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, off));
+          const float scale = a == 0.f ? 0.f : __fdiv_rn(a, 448.f);
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const float lo = scale == 0.f ? 0.f : __fdiv_rn(x[2 * e], scale);
+            const float hi = scale == 0.f ? 0.f : __fdiv_rn(x[2 * e + 1], scale);
+            uint16_t pair;
+            asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(pair) : "f"(hi), "f"(lo));
+            const uint32_t d = 4u * (uint32_t)lane + 2u * (uint32_t)e;
+            if (kv == 0) {
+              const uint32_t off = k8_offset(r, d);
+              *reinterpret_cast<uint16_t*>(st + off) = pair;
+              if (page >= 0) *reinterpret_cast<uint16_t*>(p.pool + (int64_t)page * kPageBytesFp8 + off) = pair;
+            } else {
+              const uint32_t o0 = vt8_offset(r, d), o1 = vt8_offset(r, d + 1);
+              st[o0] = (uint8_t)(pair & 0xffu);
+              st[o1] = (uint8_t)(pair >> 8);
+              if (page >= 0) {
+                p.pool[(int64_t)page * kPageBytesFp8 + o0] = (uint8_t)(pair & 0xffu);
+                p.pool[(int64_t)page * kPageBytesFp8 + o1] = (uint8_t)(pair >> 8);
+              }
+            }
+          }
+          if (lane == 0) {
+            reinterpret_cast<float*>(st + kOffScales)[kv * kPageTokens + r] = scale;
+            if (page >= 0)
+              p.scales[(int64_t)page * 2 * kPageTokens + kv * kPageTokens + r] = scale;
+          }
+        }
+        if (page >= 0 && lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
+        // These generic writes precede the next bulk copy into this stage.
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+      } else if (!kFp8 && slot / kPageTokens == walk.pg && (int)(r >> 4) == warp) {
         // The warp whose 16 rows hold the new token moves its K and V row from the
         // patch buffer into the staged page (permuted layout) and into the pool.
         const int half = lane >> 4, chunk = lane & 15;
         const uint4 val =
-            *reinterpret_cast<const uint4*>(st + kStageBytesPlain + half * kRowBytes + chunk * 16);
+            *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
         const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
         *reinterpret_cast<uint4*>(st + off) = val;
         const int page = s_misc[8 + s];
@@ -1197,6 +1252,10 @@ cudaError_t prepare_decode(const Cache& c) {
       tiled_smem_bytes<1, false, true>(kMaxHeads, kStagesFp8));
   set(decode_tiled_kernel<kStagesFp8, 2, false, true>,
       tiled_smem_bytes<2, false, true>(kMaxHeads, kStagesFp8));
+  set(decode_tiled_kernel<kStagesFp8Fused, 1, true, true>,
+      tiled_smem_bytes<1, true, true>(kMaxHeadsFused, kStagesFp8Fused));
+  set(decode_tiled_kernel<kStagesFp8Fused, 2, true, true>,
+      tiled_smem_bytes<2, true, true>(kMaxHeadsFused, kStagesFp8Fused));
   return e;
 }
 
@@ -1215,7 +1274,16 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = programmatic ? 1 : 0;
-  if (fp8) {  // one CTA per SM, never fused
+  if (fp8 && fused) {  // one CTA per SM
+    cfg.gridDim = dim3(num_sms);
+    if (p.group <= 8) {
+      cfg.dynamicSmemBytes = tiled_smem_bytes<1, true, true>(p.heads, kStagesFp8Fused);
+      return cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesFp8Fused, 1, true, true>, p);
+    }
+    cfg.dynamicSmemBytes = tiled_smem_bytes<2, true, true>(p.heads, kStagesFp8Fused);
+    return cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesFp8Fused, 2, true, true>, p);
+  }
+  if (fp8) {  // one CTA per SM
     cfg.gridDim = dim3(num_sms);
     if (p.group <= 8) {
       cfg.dynamicSmemBytes = tiled_smem_bytes<1, false, true>(p.heads, kStagesFp8);
@@ -1278,8 +1346,7 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
 }
 
 bool append_decode_fusable(const Cache& c) {
-  return c.decode_kernel == DMS_DECODE_TILED && !c.fp8() && c.heads <= kMaxHeadsFused &&
-         c.ctas_per_sm < 2;
+  return c.decode_kernel == DMS_DECODE_TILED && c.heads <= kMaxHeadsFused && c.ctas_per_sm < 2;
 }
 
 // Single-token append of position lengths[layer] fused with the decode (requires
@@ -1303,7 +1370,7 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
   p.decider = c.decider();
   p.pool_pages = c.pool_pages;
   p.ring_len = c.ring_len;
-  return launch_tiled(p, c.num_sms, 1, stream, true, true);
+  return launch_tiled(p, c.num_sms, 1, stream, true, true, c.fp8());
 }
 
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
