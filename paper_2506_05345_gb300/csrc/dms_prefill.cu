@@ -234,7 +234,7 @@ struct PrefillParams {
   const int32_t* pc;
   const int32_t* before;
   int32_t* err;              // sticky error word (bounded waits)
-  int32_t P, kv_heads, group, window, zero_first, n_qtiles, n_qheads;
+  int32_t P, kv_heads, group, window, zero_first, n_qtiles, n_qheads, batch;
   float scale_log2;
 };
 
@@ -452,38 +452,46 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 }
 
 // ============================================================================ tcgen05 kernel
-// The same attention on the 5th-generation tensor cores.  One CTA per (KV head, 128-query
-// tile, pair of query heads of the group): both heads attend to the same keys, so every
-// staged K / V tile serves two score tiles.  Q arrives and O leaves by tensor-map copies
-// (TMA, 128-byte swizzle: the tile lands in the MMA operand layout; O is staged in its
-// head's Q buffer, free once the head's last product is done).  Key tiles hold 128 keys,
-// so every MMA is M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the
-// time of an N 128 one for half its work).
-// 576 threads: warp 0 stages K tiles (3-slot ring) and V tiles (2-slot ring) with bulk
-// copies; warp 1 owns the tensor memory (all 512 columns) and issues the MMAs from one
-// thread; warps 2-17 run the softmax, two warps per (head, 32-row quarter): one takes keys
-// 0-63 of each row, the other keys 64-127 (a warp reaches only TMEM lanes 32 (warp % 4) ..,
-// so warps 2 + 4i .. 5 + 4i cover the four quarters for i = 2 h + half).
-// Tensor memory per head h: O (128 fp32 columns) at 256 h and S (128 fp32 columns) at
-// 256 h + 128.  Each softmax warp overwrites its half of S in place with P = 2^(S scale - m)
-// as packed bf16 pairs (keys 2c, 2c + 1 in column c of the half), the A operand of
-// O += P V straight from tensor memory.  S_h(t + 1) is issued after O_h += P_h(t) V(t) and
-// one thread's MMAs run in issue order, so new scores never overwrite P before it is read.
-// The two warps of a row exchange their halves' maxima through shared memory at a named
-// barrier, so both scale P by the same reference max m; m moves only when the tile max
-// exceeds it by more than 2^8 (each warp then rescales its half of O before its P-ready
-// arrival; the tile's scores commit covers every earlier product, so O is stable).  P and the running sums use
-// the same m, so O / l is exact up to rounding.  One head's softmax overlaps the other
-// head's MMAs.
+// The same attention on the 5th-generation tensor cores: a persistent kernel, one CTA per SM,
+// each walking work units (one query head x one 128-query tile; heaviest tiles first, and
+// consecutive units are the query heads of one KV head, so their K / V tiles are read from L2
+// close together in time) with a static stride.  Key tiles hold 128 keys, so every MMA is
+// M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the time of an N 128 one
+// for half its work).
+// 352 threads: warp 0 stages the K tiles (3-slot ring) and V tiles (2-slot ring) of the units
+// with bulk copies; warp 1 owns the tensor memory and issues the MMAs from one thread; warp 2
+// moves Q in and O out (tensor-map copies, 128-byte swizzle: a Q tile lands in the MMA operand
+// layout; two Q buffers, each also staging its unit's O); warps 3-10 run the softmax as two
+// sets of four warps, one thread per query row in each (a warp reaches only TMEM lanes
+// 32 (warp % 4) ..).  Set s takes the key tiles of one parity: tile tau of the CTA goes to set
+// tau % 2, so two tiles are in the softmax at once while a row's max and sum stay in a thread.
+// Tensor memory (512 columns): per set an O accumulator (128 fp32 columns, at 128 s) and an S
+// buffer (at 256 + 128 s); the scores of a tile are computed while the other set works on the
+// previous one.  A set overwrites its S in place with P = 2^(S scale - m) as packed bf16 pairs
+// (keys 2c, 2c + 1 in column c), the A operand of O_s += P V straight from tensor memory;
+// S(tau + 2) reuses the buffer after O += P(tau) V(tau), in issue order.  The reference max m
+// of a row in a set moves only when its tile max exceeds m by more than 2^8; the thread then
+// rescales its row of O_s before its P-ready arrival (the previous product into O_s completed
+// before S(tau), which was issued after it).
+// A unit ends with both sets: each publishes its row's (m, l), combines the two accumulators
+// for one d-half, O = (O_0 2^(m_0 - M) + O_1 2^(m_1 - M)) / (l_0 2^(m_0 - M) + l_1 2^(m_1 - M)),
+// M = max(m_0, m_1), and stages it as bf16 in the unit's Q buffer (every score of the unit is
+// done); warp 2 stores the tile (rows past the prompt fall outside the tensor map) and then
+// loads the Q two units on into the buffer.  The set that did not take the unit's last tile
+// first writes the P of its next tile, so the tensor cores wait only for the accumulators to
+// be read out before the next unit's products.
 // Visibility: the retained keys query j sees are the first before[j - w] compacted rows, so
 // one count masks a retained tile; window keys are a contiguous run of the band.  Stale rows
-// of a partial V tile are zeroed before its copy (P is 0 there, but 0 * NaN is not).
+// of a partial V tile are zeroed before its copy (P is 0 there, but 0 * NaN is not).  Each
+// role loads the counts of its next unit one unit ahead.
 // Shared-memory operands use the 128-byte-swizzled layout: rows of two 128-byte d-halves,
 // 16-byte chunks permuted by (row & 7), 1 KiB-aligned bases; Q and K are K-major, V is
 // MN-major (head_dim contiguous).
-constexpr int kTcHeads = 2;                              // query heads per CTA
-constexpr int kTcSoftmaxWarps = 8 * kTcHeads;            // 2 per (head, row quarter)
-constexpr int kTcThreads = (2 + kTcSoftmaxWarps) * 32;   // 576
+constexpr int kTcSets = 2;                               // softmax sets (tile parities)
+constexpr int kTcSoftmaxWarps = 4 * kTcSets;             // one thread per query row per set
+constexpr int kTcThreads = (3 + kTcSoftmaxWarps) * 32;   // 352
+constexpr int kTcQWarp = 2;
+constexpr int kTcSoftmax0 = 3;                           // first softmax warp
 // Kernel of the plain entry points (the faster of the two as measured).
 constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_TCGEN05;
 constexpr int kTcKeys = 128;                             // keys per tile
@@ -491,32 +499,35 @@ constexpr int kTcKSlots = 3;                             // K ring
 constexpr int kTcVSlots = 2;                             // V ring
 constexpr int kTcHalfBytes = kTcKeys * 128;              // one d-half of a tile, 16 KiB
 constexpr int kTcTileBytes = 2 * kTcHalfBytes;           // [2 d-halves][128 rows][128 B]
-constexpr int kTcQBytes = kPfRows * kRowBytes;           // Q, same layout
+constexpr int kTcQBytes = kPfRows * kRowBytes;           // Q (then O), same layout
 constexpr int kTcOffV = kTcKSlots * kTcTileBytes;
-constexpr int kTcOffQ = kTcOffV + kTcVSlots * kTcTileBytes;
-constexpr int kTcOffBar = kTcOffQ + kTcHeads * kTcQBytes;          // barrier block
-constexpr int kTcOffX = kTcOffBar + 256;                           // row-max exchange
-constexpr int kTcSmemBytes = kTcOffX + kTcHeads * 2 * kPfRows * 4;
+constexpr int kTcOffQ = kTcOffV + kTcVSlots * kTcTileBytes;        // two Q buffers
+constexpr int kTcOffBar = kTcOffQ + 2 * kTcQBytes;                 // barrier block
+constexpr int kTcOffX = kTcOffBar + 256;                           // (m, l) exchange
+constexpr int kTcSmemBytes = kTcOffX + kTcSets * kPfRows * 8;      // [set][row] float2
 // The dynamic shared memory base is 1 KiB aligned (no static shared memory precedes it);
 // the kernel checks this and reports DMS_ERR_CUDA otherwise.
 static_assert(kTcSmemBytes <= 227 * 1024, "tcgen05 prefill shared memory");
 constexpr uint32_t kTcCols = 512;
+constexpr uint32_t kTcColS = 256;  // S buffers at 256, 384; O accumulators at 0, 128
 constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
 
-// Barriers of one head: s_full completes once per tile (scores ready), p_full once per tile
-// (8 arrivals, one per softmax warp once the warp's P is written), o_final once (every
-// product done).
-struct TcHeadBars {
-  uint64_t s_full;
-  uint64_t p_full;
-  uint64_t o_final;
-};
+// Barriers.  Tiles are counted globally over the CTA's units (tau), units by their ordinal
+// (un).  s_full[i] and p_full[i] serve the tiles with tau % 2 = i; q_full[i], q_ready[i] and
+// o_staged[i] the units with un % 2 = i (Q buffer i); o_full and o_free complete once per
+// unit.  Every waiter is at most one phase behind the barrier it waits on (parity waits need
+// that); the waits say why.
 struct TcBars {
   uint64_t k_full[kTcKSlots], k_empty[kTcKSlots];
   uint64_t v_full[kTcVSlots], v_empty[kTcVSlots];
-  uint64_t q_full;   // the CTA's Q tiles landed
-  uint64_t q_ready;  // ... and patched (borrowed decisions only)
-  TcHeadBars h[kTcHeads];
+  uint64_t q_full[2];    // Q landed
+  uint64_t q_ready[2];   // Q patched (borrowed decisions only)
+  uint64_t o_staged[2];  // one arrival per softmax warp: the unit's O staged in its Q buffer
+  uint64_t s_full[2];    // MMA commit: scores ready
+  uint64_t p_full[2];    // one arrival per warp of the set: P written (and O rescaled)
+  uint64_t o_full;       // MMA commit: every product of the unit done
+  uint64_t o_free;       // one arrival per softmax warp: both accumulators read out
+  uint64_t mma_done;     // MMA commit at exit
   uint32_t tmem;
   int abort;
 };
@@ -528,7 +539,7 @@ struct TcMaps {
   CUtensorMap q, out;
 };
 
-// Key tile t of a CTA: the first n_ct tiles cover the nc retained rows, the rest the band
+// Key tile t of a unit: the first n_ct tiles cover the nc retained rows, the rest the band
 // [bs, jmax] of dense rows.
 struct TcTile {
   bool retained;
@@ -542,6 +553,66 @@ __device__ __forceinline__ TcTile tc_tile(int t, int n_ct, int nc, int bs, int j
   return x;
 }
 
+// Work unit u = ((rank B + b) H + hk) G + g: query head hq = hk G + g of sequence b on query
+// tile n_qtiles - 1 - rank (latest, heaviest tiles first).  A CTA visits u, u + stride, ...;
+// its roles step these digits by the stride's digits with carries (no divisions per unit).
+struct TcIter {
+  int g, hk, b, rank;
+};
+__device__ __forceinline__ TcIter tc_iter(const PrefillParams& p, int u) {
+  TcIter it;
+  const int B = p.batch;
+  it.g = u % p.group;
+  u /= p.group;
+  it.hk = u % p.kv_heads;
+  u /= p.kv_heads;
+  it.b = u % B;
+  it.rank = u / B;
+  return it;
+}
+__device__ __forceinline__ void tc_advance(const PrefillParams& p, TcIter& it, const TcIter& st) {
+  const int B = p.batch;
+  it.g += st.g;
+  int c = it.g >= p.group;
+  if (c) it.g -= p.group;
+  it.hk += st.hk + c;
+  c = it.hk >= p.kv_heads;
+  if (c) it.hk -= p.kv_heads;
+  it.b += st.b + c;
+  c = it.b >= B;
+  if (c) it.b -= B;
+  it.rank += st.rank + c;
+}
+__device__ __forceinline__ bool tc_valid(const PrefillParams& p, const TcIter& it) {
+  return it.rank < p.n_qtiles;
+}
+// The unit's fields; the retained count nc (a load) is fetched separately, one unit ahead,
+// by tc_unit_nc.
+struct TcUnit {
+  int b, hq, j0, jmax, nc, bs, n_ct, n_tiles;
+  int64_t head;  // b * kv_heads + hk: the packed K / V rows
+};
+__device__ __forceinline__ TcUnit tc_unit(const PrefillParams& p, const TcIter& it, int nc) {
+  TcUnit x;
+  x.b = it.b;
+  x.hq = it.hk * p.group + it.g;
+  x.head = (int64_t)it.b * p.kv_heads + it.hk;
+  x.j0 = (p.n_qtiles - 1 - it.rank) * kPfRows;
+  x.jmax = min(x.j0 + kPfRows, p.P) - 1;
+  x.nc = nc;
+  x.bs = max(0, x.j0 - p.window) & ~7;
+  x.n_ct = (nc + kTcKeys - 1) / kTcKeys;
+  x.n_tiles = x.n_ct + (x.jmax + 1 - x.bs + kTcKeys - 1) / kTcKeys;
+  return x;
+}
+// Retained keys visible to the unit's last query (0 past the last unit).
+__device__ __forceinline__ int tc_unit_nc(const PrefillParams& p, const TcIter& it) {
+  if (!tc_valid(p, it)) return 0;
+  const int64_t head = (int64_t)it.b * p.kv_heads + it.hk;
+  const int jmax = min((p.n_qtiles - it.rank) * kPfRows, p.P) - 1;
+  return jmax - p.window > 0 ? p.before[head * (p.P + 1) + (jmax - p.window)] : 0;
+}
+
 // Rows [r0, r0 + rows) of one head's packed K or V (two d-halves) into a 128-row tile.
 __device__ __forceinline__ void tc_stage_rows(uint8_t* dst, const uint8_t* src, int64_t head,
                                               int P, int r0, int rows, uint64_t* bar) {
@@ -550,6 +621,7 @@ __device__ __forceinline__ void tc_stage_rows(uint8_t* dst, const uint8_t* src, 
   for (int dh = 0; dh < 2; ++dh)
     bulk_copy_g2s(dst + dh * kTcHalfBytes, src + ((head * 2 + dh) * P + r0) * 128, bytes, bar);
 }
+
 
 __global__ void __launch_bounds__(kTcThreads, 1)
     prefill_tc_kernel(const __grid_constant__ PrefillParams p, const __grid_constant__ TcMaps maps) {
@@ -560,28 +632,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     return;
   }
   TcBars& bars = *reinterpret_cast<TcBars*>(smem + kTcOffBar);
-  float* xch = reinterpret_cast<float*>(smem + kTcOffX);  // [head][half][row]
   volatile int* abort_flag = &bars.abort;
-
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int G = p.group;
-  const int pairs = (G + kTcHeads - 1) / kTcHeads;
-  const int n_units = p.n_qheads / G * pairs;  // (sequence, KV head, head pair)
-  const int tile_rank = blockIdx.x / n_units;
-  const int qt = p.n_qtiles - 1 - tile_rank;  // latest (heaviest) query tiles first
-  const int unit = blockIdx.x - tile_rank * n_units;
-  const int pair = unit % pairs, bh = unit / pairs;
-  const int b = bh / p.kv_heads, hk = bh - b * p.kv_heads;
-  const int hq0 = hk * G + kTcHeads * pair;
-  const int nh = min(kTcHeads, G - kTcHeads * pair);  // query heads of this CTA
-  const int64_t head = (int64_t)bh;
-  const int P = p.P, w = p.window;
-  const int j0 = qt * kPfRows;
-  const int jmax = min(j0 + kPfRows, P) - 1;
-  const int nc = (jmax - w > 0) ? p.before[head * (P + 1) + (jmax - w)] : 0;
-  const int bs = max(0, j0 - w) & ~7;
-  const int n_ct = (nc + kTcKeys - 1) / kTcKeys;
-  const int n_tiles = n_ct + (jmax + 1 - bs + kTcKeys - 1) / kTcKeys;
+  const int P = p.P, w = p.window, G = p.group;
+  const TcIter first = tc_iter(p, blockIdx.x), step = tc_iter(p, gridDim.x);
 
   if (tid == 0) {
     *abort_flag = 0;
@@ -593,13 +647,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&bars.v_full[s], 1);
       mbar_init(&bars.v_empty[s], 1);
     }
-    mbar_init(&bars.q_full, 1);
-    mbar_init(&bars.q_ready, 4 * nh);
-    for (int h = 0; h < kTcHeads; ++h) {
-      mbar_init(&bars.h[h].s_full, 1);
-      mbar_init(&bars.h[h].p_full, 8);
-      mbar_init(&bars.h[h].o_final, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars.q_full[i], 1);
+      mbar_init(&bars.q_ready[i], 1);
+      mbar_init(&bars.o_staged[i], kTcSoftmaxWarps);
+      mbar_init(&bars.s_full[i], 1);
+      mbar_init(&bars.p_full[i], 4);
     }
+    mbar_init(&bars.o_full, 1);
+    mbar_init(&bars.o_free, kTcSoftmaxWarps);
+    mbar_init(&bars.mma_done, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -611,60 +668,118 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t tmem = bars.tmem;
 
   if (warp == 0) {
-    // ================================================================ producer
+    // ================================================================ K / V producer
     // The whole warp waits and zeroes stale V rows; lane 0 issues the copies.  A slot is
-    // refilled only after the MMAs that read its previous tile are done (empty barriers).
-    if (lane == 0) {
-      mbar_arrive_expect_tx(&bars.q_full, (uint32_t)(nh * kTcQBytes));
-      for (int h = 0; h < nh; ++h)
-        for (int dh = 0; dh < 2; ++dh)
-          tma_load_3d(smem + kTcOffQ + h * kTcQBytes + dh * (kPfRows * 128), &maps.q,
-                      (hq0 + h) * kHeadDim + 64 * dh, j0, b, &bars.q_full);
-    }
-    for (int t = 0; t < n_tiles; ++t) {
-      const TcTile x = tc_tile(t, n_ct, nc, bs, jmax);
-      const int ks = t % kTcKSlots, vs = t % kTcVSlots;
-      if (t >= kTcKSlots) mbar_wait(&bars.k_empty[ks], (t / kTcKSlots - 1) & 1, abort_flag, p.err);
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&bars.k_full[ks], 2u * (uint32_t)x.rows * 128u);
-        tc_stage_rows(smem + ks * kTcTileBytes, x.retained ? p.kc : p.kd, head, P, x.r0, x.rows,
-                      &bars.k_full[ks]);
-      }
-      if (t >= kTcVSlots) mbar_wait(&bars.v_empty[vs], (t / kTcVSlots - 1) & 1, abort_flag, p.err);
-      uint8_t* vt = smem + kTcOffV + vs * kTcTileBytes;
-      if (x.rows < kTcKeys) {
-        const int n16 = (kTcKeys - x.rows) * 8;  // 16-byte words past the rows, per d-half
-        for (int e = lane; e < 2 * n16; e += 32) {
-          const int dh = e >= n16 ? 1 : 0;
-          *reinterpret_cast<uint4*>(vt + dh * kTcHalfBytes + x.rows * 128 + (e - dh * n16) * 16) =
-              make_uint4(0u, 0u, 0u, 0u);
+    // refilled only after the MMAs that read its previous tile are done.
+    int gk = 0;  // tiles staged so far
+    TcIter it = first, nx = first;
+    tc_advance(p, nx, step);
+    int nc = tc_unit_nc(p, it);
+    for (; tc_valid(p, it); it = nx, tc_advance(p, nx, step)) {
+      const int nc_next = tc_unit_nc(p, nx);  // used one unit later
+      const TcUnit x = tc_unit(p, it, nc);
+      for (int t = 0; t < x.n_tiles; ++t, ++gk) {
+        const TcTile tl = tc_tile(t, x.n_ct, x.nc, x.bs, x.jmax);
+        const int ks = gk % kTcKSlots, vs = gk % kTcVSlots;
+        if (gk >= kTcKSlots)
+          mbar_wait(&bars.k_empty[ks], (gk / kTcKSlots - 1) & 1, abort_flag, p.err);
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&bars.k_full[ks], 2u * (uint32_t)tl.rows * 128u);
+          tc_stage_rows(smem + ks * kTcTileBytes, tl.retained ? p.kc : p.kd, x.head, P, tl.r0,
+                        tl.rows, &bars.k_full[ks]);
         }
-        fence_proxy_async_smem();  // visible to the tensor cores via the full barrier
-        __syncwarp();
+        if (gk >= kTcVSlots)
+          mbar_wait(&bars.v_empty[vs], (gk / kTcVSlots - 1) & 1, abort_flag, p.err);
+        uint8_t* vt = smem + kTcOffV + vs * kTcTileBytes;
+        if (tl.rows < kTcKeys) {
+          const int n16 = (kTcKeys - tl.rows) * 8;  // 16-byte words past the rows, per d-half
+          for (int e = lane; e < 2 * n16; e += 32) {
+            const int dh = e >= n16 ? 1 : 0;
+            *reinterpret_cast<uint4*>(vt + dh * kTcHalfBytes + tl.rows * 128 + (e - dh * n16) * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+          }
+          fence_proxy_async_smem();  // visible to the tensor cores via the full barrier
+          __syncwarp();
+        }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&bars.v_full[vs], 2u * (uint32_t)tl.rows * 128u);
+          tc_stage_rows(vt, tl.retained ? p.vc : p.vd, x.head, P, tl.r0, tl.rows, &bars.v_full[vs]);
+        }
       }
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&bars.v_full[vs], 2u * (uint32_t)x.rows * 128u);
-        tc_stage_rows(vt, x.retained ? p.vc : p.vd, head, P, x.r0, x.rows, &bars.v_full[vs]);
-      }
+      nc = nc_next;
     }
     // no copy may still be in flight when the CTA exits (matters only after a timeout)
     if (lane == 0) {
-      mbar_wait(&bars.q_full, 0, abort_flag, p.err);
-      for (int s = 0; s < kTcKSlots && s < n_tiles; ++s) {
-        const int last = s + ((n_tiles - 1 - s) / kTcKSlots) * kTcKSlots;
-        mbar_wait(&bars.k_full[s], (last / kTcKSlots) & 1, abort_flag, p.err);
+      for (int s = 0; s < kTcKSlots && s < gk; ++s) {
+        const int last = s + ((gk - 1 - s) / kTcKSlots) * kTcKSlots;
+        mbar_drain(&bars.k_full[s], (last / kTcKSlots) & 1);
       }
-      for (int s = 0; s < kTcVSlots && s < n_tiles; ++s) {
-        const int last = s + ((n_tiles - 1 - s) / kTcVSlots) * kTcVSlots;
-        mbar_wait(&bars.v_full[s], (last / kTcVSlots) & 1, abort_flag, p.err);
+      for (int s = 0; s < kTcVSlots && s < gk; ++s) {
+        const int last = s + ((gk - 1 - s) / kTcVSlots) * kTcVSlots;
+        mbar_drain(&bars.v_full[s], (last / kTcVSlots) & 1);
       }
     }
+  } else if (warp == kTcQWarp) {
+    // ================================================================ Q in, O out
+    // Before the Q of unit un goes into buffer un % 2, the O of unit un - 2 staged there is
+    // stored and read out (its scores are done by then).
+    int un = 0;
+    TcUnit x1, x2;  // the units one and two before
+    auto store_o = [&](int v, const TcUnit& y) {
+      // o_staged[v % 2] is one phase ahead at most: unit v + 2 needs the Q loaded after this
+      mbar_wait(&bars.o_staged[v & 1], (v >> 1) & 1, abort_flag, p.err);
+      if (lane == 0) {
+        const uint8_t* so = smem + kTcOffQ + (v & 1) * kTcQBytes;
+        tma_store_3d(&maps.out, y.hq * kHeadDim, y.j0, y.b, so);
+        tma_store_3d(&maps.out, y.hq * kHeadDim + 64, y.j0, y.b, so + kPfRows * 128);
+        bulk_commit_group();
+        bulk_wait_group_read0();
+      }
+      __syncwarp();
+    };
+    for (TcIter it = first; tc_valid(p, it); tc_advance(p, it, step), ++un) {
+      const TcUnit x = tc_unit(p, it, 0);  // position fields only
+      const int qi = un & 1;
+      uint8_t* sq = smem + kTcOffQ + qi * kTcQBytes;  // [d-half][row][128 B], swizzled
+      if (un >= 2) store_o(un - 2, x2);
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars.q_full[qi], (uint32_t)kTcQBytes);
+        for (int dh = 0; dh < 2; ++dh)
+          tma_load_3d(sq + dh * (kPfRows * 128), &maps.q, x.hq * kHeadDim + 64 * dh, x.j0, x.b,
+                      &bars.q_full[qi]);
+      }
+      if (p.zero_first) {
+        // App. B: the decision element (head_dim 0 of the group's first head) is not a query
+        // feature; zero it in the landed tile before any score reads it (q_full[qi] is one
+        // phase ahead at most: the next Q for this buffer is loaded by this warp)
+        mbar_wait(&bars.q_full[qi], (un >> 1) & 1, abort_flag, p.err);
+        if (x.hq % G == 0)
+          for (int r = lane; r < kPfRows; r += 32)
+            *reinterpret_cast<uint16_t*>(sq + r * 128 + chunk_in_row(r, 0)) = 0;
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars.q_ready[qi]);
+      }
+      x2 = x1;
+      x1 = x;
+    }
+    if (un >= 2) store_o(un - 2, x2);
+    if (un >= 1) store_o(un - 1, x1);
+    if (lane == 0)  // no copy may still be in flight when the CTA exits
+      for (int i = 0; i < 2 && i < un; ++i) {
+        const int last = i + ((un - 1 - i) / 2) * 2;
+        mbar_drain(&bars.q_full[i], (last >> 1) & 1);
+      }
   } else if (warp == 1) {
     // ================================================================ MMA issuer
-    // Order per tile t: for each head h, O_h += P_h(t) V(t), then S_h(t + 1) (or, after the
-    // last tile, the commit that releases O_h).  The thread is the only waiter on k_full /
-    // v_full / p_full and consumes them in order.
-    if (lane == 0) {
+    // Order: S(0), S(1), then per tile tau: O_(tau % 2) += P(tau) V(tau), S(tau + 2).
+    // S(tau + 2) goes into the buffer of P(tau) after the product that reads it, in issue
+    // order.  The warp runs the loop (its values stay warp-uniform) and one elected lane, the
+    // same throughout, issues each group of MMAs with its commits: issued from a divergent
+    // single thread the MMAs of a tile took up to 1.5x the tensor cores' time.  The warp is
+    // the only waiter on q_full / q_ready / k_full / v_full / p_full / o_free and takes each
+    // phase in order.
+    {
       constexpr uint32_t idesc_s = f16_idesc(kPfRows, kTcKeys, 0);    // Q K^T: both K-major
       constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
       // Descriptors are built once and their start address (16-byte units) stepped: +2 per
@@ -673,212 +788,267 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint64_t dq0 = sw128_desc(smem_addr(smem + kTcOffQ), 16u, 1024u);
       const uint64_t dk0 = sw128_desc(smem_addr(smem), 16u, 1024u);
       const uint64_t dv0 = sw128_desc(smem_addr(smem + kTcOffV), (uint32_t)kTcHalfBytes, 1024u);
-      constexpr uint64_t kQHead = kTcQBytes >> 4, kQHalf = (kPfRows * 128) >> 4;
+      constexpr uint64_t kQBuf = kTcQBytes >> 4, kQHalf = (kPfRows * 128) >> 4;
       constexpr uint64_t kKHalf = kTcHalfBytes >> 4, kSlot = kTcTileBytes >> 4;
-      auto issue_scores = [&](int h, int t) {
-        const uint64_t dq = dq0 + (uint64_t)h * kQHead;
-        const uint64_t dk = dk0 + (uint64_t)(t % kTcKSlots) * kSlot;
-        const uint32_t d_s = tmem + (uint32_t)(256 * h + 128);
-        tc_mma_ss_k<false>(d_s, dq, dk, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + 2, dk + 2, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + 4, dk + 4, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + 6, dk + 6, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + kQHalf, dk + kKHalf, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + kQHalf + 2, dk + kKHalf + 2, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + kQHalf + 4, dk + kKHalf + 4, idesc_s);
-        tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
-        tc_commit(&bars.h[h].s_full);
+      // Cursors over the CTA's tiles: the unit and the next one, unit ordinal, tile in unit,
+      // tiles of unit, and the retained count of the next unit (loaded one unit ahead).
+      struct Cur {
+        TcIter it, nx;
+        int un, t, n, nc_next;
       };
-      mbar_wait(p.zero_first ? &bars.q_ready : &bars.q_full, 0, abort_flag, p.err);
-      mbar_wait(&bars.k_full[0], 0, abort_flag, p.err);
-      tc_fence_after();
-      for (int h = 0; h < nh; ++h) issue_scores(h, 0);
-      tc_commit(&bars.k_empty[0]);
-      for (int t = 0; t < n_tiles; ++t) {
-        const int vs = t % kTcVSlots;
-        const bool more = t + 1 < n_tiles;
-        mbar_wait(&bars.v_full[vs], (t / kTcVSlots) & 1, abort_flag, p.err);
-        const uint64_t dv = dv0 + (uint64_t)vs * kSlot;
-        for (int h = 0; h < nh; ++h) {
-          TcHeadBars& hb = bars.h[h];
-          mbar_wait(&hb.p_full, t & 1, abort_flag, p.err);
-          tc_fence_after();
-          // keys 16 kk .. 16 kk + 15: P columns 8 kk of the first half, 64 + 8 (kk - 4) of
-          // the second; V rows 16 kk .. (2 KiB per 16 rows)
-          const uint32_t d_o = tmem + (uint32_t)(256 * h);
-          const uint32_t a = tmem + (uint32_t)(256 * h + 128);
-          if (t == 0)
+      auto start = [&](Cur& c) {
+        c.it = c.nx = first;
+        tc_advance(p, c.nx, step);
+        c.un = c.t = 0;
+        c.n = tc_valid(p, c.it) ? tc_unit(p, c.it, tc_unit_nc(p, c.it)).n_tiles : 0;
+        c.nc_next = tc_unit_nc(p, c.nx);
+      };
+      auto next = [&](Cur& c) {
+        if (++c.t == c.n) {
+          c.t = 0;
+          c.it = c.nx;
+          tc_advance(p, c.nx, step);
+          ++c.un;
+          c.n = tc_valid(p, c.it) ? tc_unit(p, c.it, c.nc_next).n_tiles : 0;
+          c.nc_next = tc_unit_nc(p, c.nx);
+        }
+      };
+      Cur sc, pc;
+      start(sc);
+      start(pc);
+      auto issue_scores = [&](int tau) {
+        const int qi = sc.un & 1;
+        if (sc.t == 0)  // the unit's Q has landed (and, borrowed decisions, is patched)
+          mbar_wait(p.zero_first ? &bars.q_ready[qi] : &bars.q_full[qi], (sc.un >> 1) & 1,
+                    abort_flag, p.err);
+        mbar_wait(&bars.k_full[tau % kTcKSlots], (tau / kTcKSlots) & 1, abort_flag, p.err);
+        tc_fence_after();
+        const uint64_t dq = dq0 + (uint64_t)qi * kQBuf;
+        const uint64_t dk = dk0 + (uint64_t)(tau % kTcKSlots) * kSlot;
+        const uint32_t d_s = tmem + kTcColS + (uint32_t)(128 * (tau & 1));
+        if (elect_one()) {
+          tc_mma_ss_k<false>(d_s, dq, dk, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + 2, dk + 2, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + 4, dk + 4, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + 6, dk + 6, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf, dk + kKHalf, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf + 2, dk + kKHalf + 2, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf + 4, dk + kKHalf + 4, idesc_s);
+          tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
+          tc_commit(&bars.s_full[tau & 1]);
+          tc_commit(&bars.k_empty[tau % kTcKSlots]);  // the K slot is free once these are done
+        }
+        __syncwarp();
+        next(sc);
+      };
+      int s_tau = 0;
+      if (sc.n > 0) issue_scores(s_tau++);
+      if (sc.n > 0) issue_scores(s_tau++);
+      for (int tau = 0; pc.n > 0; ++tau) {
+        // S(tau) was issued after O += P(tau - 2) V: p_full[tau & 1] is one phase ahead at most
+        mbar_wait(&bars.p_full[tau & 1], (tau >> 1) & 1, abort_flag, p.err);
+        // a unit's first product overwrites an accumulator: the previous unit's are read out
+        // (o_free completes once per unit, after o_full, which needs this unit's products)
+        if (pc.t == 0 && pc.un > 0) mbar_wait(&bars.o_free, (pc.un - 1) & 1, abort_flag, p.err);
+        mbar_wait(&bars.v_full[tau % kTcVSlots], (tau / kTcVSlots) & 1, abort_flag, p.err);
+        tc_fence_after();
+        // keys 16 kk .. 16 kk + 15: P columns 8 kk .. of the buffer; V rows 16 kk .. (2 KiB
+        // per 16 rows).  The set's first tile of the unit starts its accumulator.
+        const uint64_t dv = dv0 + (uint64_t)(tau % kTcVSlots) * kSlot;
+        const uint32_t a = tmem + kTcColS + (uint32_t)(128 * (tau & 1));
+        const uint32_t d_o = tmem + (uint32_t)(128 * (tau & 1));
+        const bool first_of_set = pc.t < kTcSets, last_of_unit = pc.t == pc.n - 1;
+        if (elect_one()) {
+          if (first_of_set)
             tc_mma_ts_k<false>(d_o, a, dv, idesc_o);
           else
             tc_mma_ts_k<true>(d_o, a, dv, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 8, dv + 128, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 16, dv + 256, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 24, dv + 384, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 64, dv + 512, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 72, dv + 640, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 80, dv + 768, idesc_o);
-          tc_mma_ts_k<true>(d_o, a + 88, dv + 896, idesc_o);
-          if (more) {
-            if (h == 0) {
-              mbar_wait(&bars.k_full[(t + 1) % kTcKSlots], ((t + 1) / kTcKSlots) & 1, abort_flag,
-                        p.err);
-              tc_fence_after();
-            }
-            issue_scores(h, t + 1);
-          } else {
-            tc_commit(&hb.o_final);
+#pragma unroll
+          for (int kk = 1; kk < kTcKeys / 16; ++kk)
+            tc_mma_ts_k<true>(d_o, a + 8 * kk, dv + 128 * kk, idesc_o);
+          tc_commit(&bars.v_empty[tau % kTcVSlots]);
+          if (last_of_unit) tc_commit(&bars.o_full);  // the unit's O is complete
+        }
+        __syncwarp();
+        next(pc);
+        if (sc.n > 0) issue_scores(s_tau++);
+      }
+      // the tensor memory is released only after every product has landed
+      if (elect_one()) tc_commit(&bars.mma_done);
+      __syncwarp();
+      mbar_drain(&bars.mma_done, 0);
+    }
+  } else {
+    // ================================================================ softmax
+    const int set = (warp - kTcSoftmax0) >> 2;  // takes the tiles with tau % 2 = set
+    const int quarter = warp & 3;
+    const int row = 32 * quarter + lane;        // query row of the tile = TMEM lane
+    const uint32_t lane_addr = tmem + ((uint32_t)(32 * quarter) << 16);
+    const uint32_t o_own = lane_addr + (uint32_t)(128 * set);
+    const uint32_t o_other = lane_addr + (uint32_t)(128 * (set ^ 1));
+    const uint32_t s_own = lane_addr + kTcColS + (uint32_t)(128 * set);
+    float2* xml = reinterpret_cast<float2*>(smem + kTcOffX);  // [set][row]: (m, l)
+    const float scale = p.scale_log2;
+    const float2 scale2 = make_float2(scale, scale);
+    // the row's count of visible retained keys, before[j - w] (0 for j <= w), one unit ahead
+    auto row_before = [&](const TcIter& it) {
+      if (!tc_valid(p, it)) return 0;
+      const TcUnit y = tc_unit(p, it, 0);
+      const int j = y.j0 + row;
+      return j - w > 0 ? p.before[y.head * (P + 1) + min(j - w, P)] : 0;
+    };
+    // End of unit v (both sets): publish this set's (m, l) of the row, combine the two
+    // accumulators for d-half `set` and stage it as bf16 in the unit's Q buffer.  o_full is
+    // one phase ahead at most: the next unit's products need this call's o_free arrival.
+    auto finish_unit = [&](int v, float mv, float lv) {
+      mbar_wait(&bars.o_full, v & 1, abort_flag, p.err);
+      tc_fence_after();
+      xml[set * kPfRows + row] = make_float2(mv, lv);
+      named_barrier_sync_id(1 + quarter, 64);  // the two sets' warps of this quarter
+      const float2 ot = xml[(set ^ 1) * kPfRows + row];
+      named_barrier_sync_id(1 + quarter, 64);  // read before either writes the next unit's
+      // weights 2^(m_s - M); a set without visible keys (m = -inf) contributes nothing
+      const float M = fmaxf(mv, ot.x);
+      const bool own = mv != -INFINITY, oth = ot.x != -INFINITY;
+      const float a0 = own ? ex2_approx(mv - M) : 0.f, a1 = oth ? ex2_approx(ot.x - M) : 0.f;
+      const float lt = (own ? lv * a0 : 0.f) + (oth ? ot.y * a1 : 0.f);
+      const float inv = lt > 0.f ? 1.f / lt : 0.f;
+      const float c0 = a0 * inv, c1 = a1 * inv;
+      uint8_t* half_row = smem + kTcOffQ + (v & 1) * kTcQBytes + set * (kPfRows * 128) + row * 128;
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {  // head_dim 64 set + 32 hh .. + 31
+        float r0[32], r1[32];
+#pragma unroll
+        for (int c = 0; c < 32; c += 16) {
+          tmem_ld16_at(o_own + (uint32_t)(64 * set + 32 * hh + c), r0 + c);
+          tmem_ld16_at(o_other + (uint32_t)(64 * set + 32 * hh + c), r1 + c);
+        }
+        tmem_wait_ld();
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {  // logical chunk 4 hh + c of the d-half
+          float o[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            o[e] = (own ? r0[8 * c + e] * c0 : 0.f) + (oth ? r1[8 * c + e] * c1 : 0.f);
+          uint4 q4;
+          q4.x = pack_bf16x2(o[0], o[1]);
+          q4.y = pack_bf16x2(o[2], o[3]);
+          q4.z = pack_bf16x2(o[4], o[5]);
+          q4.w = pack_bf16x2(o[6], o[7]);
+          *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, 4 * hh + c)) = q4;
+        }
+      }
+      tc_fence_before();  // the reads precede the next unit's products (via o_free)
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars.o_free);
+      fence_proxy_async_smem();  // visible to the tensor-map store
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars.o_staged[v & 1]);
+    };
+    int tau = 0, un = 0;
+    TcIter it = first, nx = first;
+    tc_advance(p, nx, step);
+    int nc = tc_unit_nc(p, it), bj_next = row_before(it);
+    // an unfinished unit: its ordinal (or -1) and this set's (m, l) of the row
+    int pend = -1;
+    float m_pend = -INFINITY, l_pend = 0.f;
+    for (; tc_valid(p, it); it = nx, tc_advance(p, nx, step), ++un) {
+      const TcUnit x = tc_unit(p, it, nc);
+      const int bj = bj_next;  // the first bj compacted rows are this row's retained keys
+      nc = tc_unit_nc(p, nx);  // both used one unit later
+      bj_next = row_before(nx);
+      const int j = x.j0 + row;
+      float m = -INFINITY;  // reference max of the row in this set (log2 domain)
+      float l = 0.f;        // running sum of the row in this set
+      bool started = false; // this set has taken a tile of the unit
+      for (int t = 0; t < x.n_tiles; ++t, ++tau) {
+        if ((tau & 1) != set) continue;
+        const TcTile tl = tc_tile(t, x.n_ct, x.nc, x.bs, x.jmax);
+        int lo, nvis;  // visible keys of the tile: lo .. lo + nvis - 1
+        if (tl.retained) {
+          lo = 0;
+          nvis = min(max(bj - tl.r0, 0), tl.rows);
+        } else {
+          lo = max(j - w - tl.r0, 0);
+          nvis = max(min(j - tl.r0, tl.rows - 1) - lo + 1, 0);
+        }
+        // S(tau + 2) into this buffer follows this tile's P-ready arrival: one phase at most
+        mbar_wait(&bars.s_full[set], (tau >> 1) & 1, abort_flag, p.err);
+        tc_fence_after();
+        float sc[kTcKeys];
+#pragma unroll
+        for (int c = 0; c < kTcKeys; c += 16) tmem_ld16_at(s_own + c, sc + c);
+        tmem_wait_ld();
+        if (!__all_sync(0xffffffffu, lo == 0 && nvis == kTcKeys)) {
+#pragma unroll
+          for (int k = 0; k < kTcKeys; ++k)
+            if ((unsigned)(k - lo) >= (unsigned)nvis) sc[k] = -INFINITY;
+        }
+        float mx8[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mx8[e] = fmaxf(sc[e], sc[8 + e]);
+#pragma unroll
+        for (int k = 16; k < kTcKeys; k += 16)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mx8[e] = max3f(mx8[e], sc[k + e], sc[k + 8 + e]);
+        const float mt = max3f(max3f(mx8[0], mx8[1], mx8[2]), max3f(mx8[3], mx8[4], mx8[5]),
+                               fmaxf(mx8[6], mx8[7])) * scale;
+        float corr = 1.f;
+        if (mt > m + kTcRescale) {
+          corr = ex2_approx(m - mt);  // 0 when m = -inf
+          m = mt;
+        }
+        const float nb = m == -INFINITY ? 0.f : -m;
+        const float2 nb2 = make_float2(nb, nb);
+        float2 s2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+        for (int g = 0; g < kTcKeys / 16; ++g) {  // 16 keys -> 8 packed columns, stored at once
+          uint32_t pk[8];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const int k = 16 * g + 2 * c;
+            const float2 y = fma_f32x2(make_float2(sc[k], sc[k + 1]), scale2, nb2);
+            const float2 pp = make_float2(ex2_approx(y.x), ex2_approx(y.y));
+            s2[c & 1] = add_f32x2(s2[c & 1], pp);
+            pk[c] = pack_bf16x2(pp.x, pp.y);
+          }
+          tmem_st8_u32(s_own + (uint32_t)(8 * g), pk);
+        }
+        const float2 ss = add_f32x2(s2[0], s2[1]);
+        l = l * corr + (ss.x + ss.y);
+        if (started && __any_sync(0xffffffffu, corr != 1.f)) {
+          // (rare) the row of O_s: the product of this set's previous tile completed before
+          // S(tau) (issued after it); O += P(tau) V waits for the arrival below
+#pragma unroll 1
+          for (int c = 0; c < kHeadDim; c += 16) {
+            float r[16];
+            tmem_ld16(o_own + (uint32_t)c, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) r[e] *= corr;
+            tmem_st16(o_own + (uint32_t)c, r);
           }
         }
-        tc_commit(&bars.v_empty[vs]);  // a slot is free once every product on it is done
-        if (more) tc_commit(&bars.k_empty[(t + 1) % kTcKSlots]);
-      }
-    }
-  } else if ((warp - 2) / 8 < nh) {
-    // ================================================================ softmax
-    const int idx = (warp - 2) >> 2;            // 2 h + half
-    const int h = idx >> 1, half = idx & 1;     // head of the CTA, key half of the tile
-    const int row = 32 * (warp & 3) + lane;     // query row of the tile = TMEM lane
-    const int j = j0 + row;
-    const int hq = hq0 + h;
-    const uint32_t o_addr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(256 * h);
-    const uint32_t s_addr = o_addr + 128u + (uint32_t)(64 * half);  // this half of S / P
-    const int bar_id = 1 + 4 * h + (warp & 3);  // the two warps of this (head, quarter)
-    TcHeadBars& hb = bars.h[h];
-    uint8_t* sq = smem + kTcOffQ + h * kTcQBytes;  // [d-half][row][128 B], swizzled
-    float* x_mine = xch + (2 * h + half) * kPfRows + row;
-    const float* x_other = xch + (2 * h + (half ^ 1)) * kPfRows + row;
-    if (p.zero_first && half == 0) {
-      // App. B: the decision element (head_dim 0 of the group's first head) is not a query
-      // feature; zero it in the landed tile before any score reads it
-      mbar_wait(&bars.q_full, 0, abort_flag, p.err);
-      if (hq % G == 0) *reinterpret_cast<uint16_t*>(sq + row * 128 + chunk_in_row(row, 0)) = 0;
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars.q_ready);
-    }
-    // the retained keys of this row: the first bj compacted rows
-    const int bj = j - w > 0 ? p.before[head * (P + 1) + min(j - w, P)] : 0;
-    const float2 scale2 = make_float2(p.scale_log2, p.scale_log2);
-    const int key0 = 64 * half;
-    float m = -INFINITY;  // reference max of the row (log2 domain), the same in both warps
-    float l = 0.f;        // running sum over this warp's half of the keys
-    for (int t = 0; t < n_tiles; ++t) {
-      const TcTile x = tc_tile(t, n_ct, nc, bs, jmax);
-      int lo, nvis;  // visible keys of the tile: lo .. lo + nvis - 1
-      if (x.retained) {
-        lo = 0;
-        nvis = min(max(bj - x.r0, 0), x.rows);
-      } else {
-        lo = max(j - w - x.r0, 0);
-        nvis = max(min(j - x.r0, x.rows - 1) - lo + 1, 0);
-      }
-      // S(t) is issued after P(t - 1) is read, so this wait is at most one phase behind; its
-      // commit also covers every earlier product (O is stable, P(t - 1) is free)
-      mbar_wait(&hb.s_full, t & 1, abort_flag, p.err);
-      tc_fence_after();
-      float sc[64];
-      tmem_ld16_at(s_addr, sc);
-      tmem_ld16_at(s_addr + 16, sc + 16);
-      tmem_ld16_at(s_addr + 32, sc + 32);
-      tmem_ld16_at(s_addr + 48, sc + 48);
-      tmem_wait_ld();
-      if (!__all_sync(0xffffffffu, lo <= key0 && key0 + 64 <= lo + nvis)) {
-#pragma unroll
-        for (int k = 0; k < 64; ++k)
-          if ((unsigned)(key0 + k - lo) >= (unsigned)nvis) sc[k] = -INFINITY;
-      }
-      float mx8[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) mx8[e] = max3f(sc[e], sc[8 + e], sc[16 + e]);
-#pragma unroll
-      for (int k = 24; k < 64; k += 16)
-#pragma unroll
-        for (int e = 0; e < 8; ++e) mx8[e] = max3f(mx8[e], sc[k + e], sc[k + 8 + e]);
-      const float mh = max3f(max3f(mx8[0], mx8[1], mx8[2]), max3f(mx8[3], mx8[4], mx8[5]),
-                             fmaxf(mx8[6], mx8[7]));
-      // the other half's max of this row (its previous value was read before it could be
-      // rewritten: the next tile's scores need both halves' P of this one)
-      *x_mine = mh;
-      named_barrier_sync_id(bar_id, 64);
-      const float mt = fmaxf(mh, *x_other) * p.scale_log2;
-      float corr = 1.f;
-      if (mt > m + kTcRescale) {
-        corr = ex2_approx(m - mt);  // 0 when m = -inf
-        m = mt;
-      }
-      const float nb = m == -INFINITY ? 0.f : -m;
-      const float2 nb2 = make_float2(nb, nb);
-      float2 s2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-#pragma unroll
-      for (int g = 0; g < 4; ++g) {  // 16 keys -> 8 packed columns, stored at once
-        uint32_t pk[8];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int k = 16 * g + 2 * c;
-          const float2 y = fma_f32x2(make_float2(sc[k], sc[k + 1]), scale2, nb2);
-          const float2 pp = make_float2(ex2_approx(y.x), ex2_approx(y.y));
-          s2[c & 1] = add_f32x2(s2[c & 1], pp);
-          pk[c] = pack_bf16x2(pp.x, pp.y);
+        started = true;
+        tmem_wait_st();
+        tc_fence_before();
+        // the previous unit, when this set did not take its last tile: its accumulators are
+        // read out before this tile's product may start the next one
+        if (pend >= 0) {
+          finish_unit(pend, m_pend, l_pend);
+          pend = -1;
         }
-        tmem_st8_u32(s_addr + (uint32_t)(8 * g), pk);
+        __syncwarp();  // the warp's stores are ordered before its one arrival
+        if (lane == 0) mbar_arrive(&bars.p_full[set]);
+        if (t == x.n_tiles - 1) finish_unit(un, m, l);  // this set took the unit's last tile
       }
-      const float2 ss = add_f32x2(s2[0], s2[1]);
-      l = l * corr + (ss.x + ss.y);
-      if (t > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
-        // (rare) this warp's half of the row of O, 16 columns at a time; O(t) += P V is
-        // issued only after this thread's P-ready arrival below
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float r[16];
-          const uint32_t oa = o_addr + (uint32_t)(64 * half + 16 * c);
-          tmem_ld16(oa, r);
-          tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 16; ++e) r[e] *= corr;
-          tmem_st16(oa, r);
-        }
+      if (((tau - 1) & 1) != set) {  // the other set took the last tile: finish with the next
+        pend = un;
+        m_pend = m;
+        l_pend = l;
       }
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();  // the warp's stores are ordered before its one arrival
-      if (lane == 0) mbar_arrive(&hb.p_full);
     }
-    // every product of this head is done: normalise this warp's half of the row and stage
-    // it as bf16 in the head's Q buffer (d-half = key half), then one thread stores the tile
-    mbar_wait(&hb.o_final, 0, abort_flag, p.err);
-    tc_fence_after();
-    *x_mine = l;  // both warps passed their last exchange before o_final could complete
-    named_barrier_sync_id(bar_id, 64);
-    const float lt = l + *x_other;
-    const float inv = lt > 0.f ? 1.f / lt : 0.f;
-    uint8_t* half_row = sq + half * (kPfRows * 128) + row * 128;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      float r[16];
-      tmem_ld16(o_addr + (uint32_t)(64 * half + 16 * c), r);
-      tmem_wait_ld();
-      uint4 v0, v1;
-      v0.x = pack_bf16x2(r[0] * inv, r[1] * inv);
-      v0.y = pack_bf16x2(r[2] * inv, r[3] * inv);
-      v0.z = pack_bf16x2(r[4] * inv, r[5] * inv);
-      v0.w = pack_bf16x2(r[6] * inv, r[7] * inv);
-      v1.x = pack_bf16x2(r[8] * inv, r[9] * inv);
-      v1.y = pack_bf16x2(r[10] * inv, r[11] * inv);
-      v1.z = pack_bf16x2(r[12] * inv, r[13] * inv);
-      v1.w = pack_bf16x2(r[14] * inv, r[15] * inv);
-      // head_dim 64 half + 16c .. + 15: logical chunks 2c, 2c + 1 of the d-half
-      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, 2 * c)) = v0;
-      *reinterpret_cast<uint4*>(half_row + chunk_in_row(row, 2 * c + 1)) = v1;
-    }
-    fence_proxy_async_smem();
-    named_barrier_sync_id(9 + h, 2 * kPfRows);
-    if (half == 0 && row == 0) {
-      // rows past the prompt fall outside the tensor map and are not written
-      tma_store_3d(&maps.out, hq * kHeadDim, j0, b, sq);
-      tma_store_3d(&maps.out, hq * kHeadDim + 64, j0, b, sq + kPfRows * 128);
-      bulk_commit_group();
-      bulk_wait_group_read0();
-    }
+    if (pend >= 0) finish_unit(pend, m_pend, l_pend);
   }
   // ---- teardown: every tensor-memory access is done before the columns are released
   tc_fence_before();
@@ -990,6 +1160,7 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
   pp.zero_first = zero_first ? 1 : 0;
   pp.n_qtiles = (n_tokens + kPfRows - 1) / kPfRows;
   pp.n_qheads = (int32_t)(H * group);
+  pp.batch = batch;
   pp.scale_log2 = scale_log2;
   const int64_t grid = (int64_t)pp.n_qtiles * pp.n_qheads;
   if (kernel == DMS_PREFILL_MMA_SYNC) {
@@ -999,9 +1170,13 @@ cudaError_t launch_prefill(const void* q, const void* k, const void* v, const vo
     if (!encode_qo_map(&maps.q, q, batch, n_tokens, pp.n_qheads / batch) ||
         !encode_qo_map(&maps.out, out, batch, n_tokens, pp.n_qheads / batch))
       return cudaErrorInvalidValue;
-    const int64_t units = H * ((group + kTcHeads - 1) / kTcHeads);
-    prefill_tc_kernel<<<(unsigned)(pp.n_qtiles * units), kTcThreads, kTcSmemBytes, stream>>>(pp,
-                                                                                              maps);
+    // persistent: one CTA per SM (fewer when there are fewer work units)
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int64_t units = (int64_t)pp.n_qtiles * pp.n_qheads;
+    const unsigned ctas = (unsigned)(units < sms ? units : sms);
+    prefill_tc_kernel<<<ctas, kTcThreads, kTcSmemBytes, stream>>>(pp, maps);
   }
   return cudaGetLastError();
 }

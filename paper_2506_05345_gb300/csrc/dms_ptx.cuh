@@ -75,6 +75,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   return mbar_wait_slow(bar, parity, abort, ctrl);
 }
 
+// Wait at kernel exit for a bulk copy or tensor-core operation this thread issued: bounded by
+// its own limit and independent of the abort flag, so that after a timeout elsewhere nothing
+// issued by the CTA still writes its shared or tensor memory when the CTA leaves.
+constexpr unsigned long long kDrainLimitNs = 20ull * 1000 * 1000;
+__device__ __noinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const unsigned long long t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (global_timer_ns() - t0 > kDrainLimitNs) return;
+}
+
 // atomicAdd with acquire-release semantics at GPU scope; returns the old value.
 __device__ __forceinline__ int atomic_add_acq_rel(int32_t* addr, int v) {
   int old;
@@ -300,6 +310,16 @@ __device__ __forceinline__ void tc_mma_ts_k(uint32_t d_tmem, uint32_t a_tmem, ui
                  : "memory");
 }
 
+// One lane of the (fully active) warp: the lowest, the same on every call.  Issuing the MMAs of
+// a warp-uniform loop under it keeps their operands in uniform registers.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred = 0;
+  asm volatile(
+      "{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.b32 %0, 1, 0, P;\n\t}"
+      : "=r"(pred));
+  return pred != 0;
+}
+
 // Arrive once on `bar` when every tcgen05 operation issued so far by this thread is done.
 __device__ __forceinline__ void tc_commit(uint64_t* bar) {
   asm volatile(
@@ -365,6 +385,32 @@ __device__ __forceinline__ void tmem_st16_u32(uint32_t taddr, const uint32_t* r)
       "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
       "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
       : "memory");
+}
+// One 32-bit word into one column of this thread's lane.
+__device__ __forceinline__ void tmem_st1_f32(uint32_t taddr, float v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr),
+               "r"(__float_as_uint(v))
+               : "memory");
+}
+// Four consecutive columns of this thread's lane (complete after tmem_wait_ld).
+__device__ __forceinline__ void tmem_ld4(uint32_t taddr, float (&r)[4]) {
+  uint32_t a, b, c, d;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
+               : "r"(taddr)
+               : "memory");
+  r[0] = __uint_as_float(a);
+  r[1] = __uint_as_float(b);
+  r[2] = __uint_as_float(c);
+  r[3] = __uint_as_float(d);
+}
+// Order-preserving map of a float (not NaN) to an int and back: integer max = float max.
+__device__ __forceinline__ int ordered_key(float f) {
+  const int i = __float_as_int(f);
+  return i >= 0 ? i : i ^ 0x7fffffff;
+}
+__device__ __forceinline__ float from_ordered_key(int k) {
+  return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff);
 }
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
