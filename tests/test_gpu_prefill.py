@@ -78,6 +78,8 @@ KERNELS = [dms.DMS_PREFILL_TCGEN05, dms.DMS_PREFILL_MMA_SYNC]
     (2, 257, 1, 4, 128, 0.0),     # nothing evicted: dense causal
     (1, 1, 1, 1, 0, 1.0),         # one token
     (1, 129, 2, 7, 3, 0.7),       # G = 7, tile boundary + 1
+    (2, 1200, 2, 8, 64, 0.75),    # 320 (head, tile) units: > 2 per CTA of the persistent kernel
+    (2, 1100, 3, 7, 16, 0.5),     # 378 units, G = 7; each CTA ends on one-tile units
 ])
 def test_prefill_matches_oracle(B, P, H, G, w, p, kernel):
     q, k, v, lg = _inputs(B, P, H, G, p, seed=P + G)
