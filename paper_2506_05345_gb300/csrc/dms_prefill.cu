@@ -458,13 +458,15 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // close together in time) with a static stride.  Key tiles hold 128 keys, so every MMA is
 // M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the time of an N 128 one
 // for half its work).
-// 352 threads: warp 0 stages the K tiles (3-slot ring) and V tiles (2-slot ring) of the units
-// with bulk copies; warp 1 owns the tensor memory and issues the MMAs from one thread; warp 2
-// moves Q in and O out (tensor-map copies, 128-byte swizzle: a Q tile lands in the MMA operand
-// layout; two Q buffers, each also staging its unit's O); warps 3-10 run the softmax as two
-// sets of four warps, one thread per query row in each (a warp reaches only TMEM lanes
-// 32 (warp % 4) ..).  Set s takes the key tiles of one parity: tile tau of the CTA goes to set
-// tau % 2, so two tiles are in the softmax at once while a row's max and sum stay in a thread.
+// 384 threads: warp 0 stages the K tiles (3-slot ring) and V tiles (2-slot ring) of the units
+// with bulk copies; warp 2 moves Q in and O out (tensor-map copies, 128-byte swizzle: a Q tile
+// lands in the MMA operand layout; two Q buffers, each also staging its unit's O); warps 4-11
+// run the softmax as two sets of four warps, one thread per query row in each (a warp reaches
+// only TMEM lanes 32 (warp % 4) ..).  Set s takes the key tiles of one parity: tile tau of the
+// CTA goes to set tau % 2, so two tiles are in the softmax at once while a row's max and sum
+// stay in a thread.  Warps 1 and 3 issue the MMAs of sets 0 and 1: the two streams share no
+// tensor memory, so the tensor cores interleave them and one set's waits do not stall the
+// other's products (warp 1 also owns the tensor memory).
 // Tensor memory (512 columns): per set an O accumulator (128 fp32 columns, at 128 s) and an S
 // buffer (at 256 + 128 s); the scores of a tile are computed while the other set works on the
 // previous one.  A set overwrites its S in place with P = 2^(S scale - m) as packed bf16 pairs
@@ -489,9 +491,10 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // MN-major (head_dim contiguous).
 constexpr int kTcSets = 2;                               // softmax sets (tile parities)
 constexpr int kTcSoftmaxWarps = 4 * kTcSets;             // one thread per query row per set
-constexpr int kTcThreads = (3 + kTcSoftmaxWarps) * 32;   // 352
+constexpr int kTcThreads = (4 + kTcSoftmaxWarps) * 32;   // 384
 constexpr int kTcQWarp = 2;
-constexpr int kTcSoftmax0 = 3;                           // first softmax warp
+constexpr int kTcMmaWarp1 = 3;                           // MMAs of set 1 (set 0: warp 1)
+constexpr int kTcSoftmax0 = 4;                           // first softmax warp
 // Kernel of the plain entry points (the faster of the two as measured).
 constexpr int32_t kPrefillDefaultKernel = DMS_PREFILL_TCGEN05;
 constexpr int kTcKeys = 128;                             // keys per tile
@@ -513,9 +516,9 @@ constexpr uint32_t kTcColS = 256;  // S buffers at 256, 384; O accumulators at 0
 constexpr float kTcRescale = 8.f;  // log2 of the largest growth of P before O is rescaled
 
 // Barriers.  Tiles are counted globally over the CTA's units (tau), units by their ordinal
-// (un).  s_full[i] and p_full[i] serve the tiles with tau % 2 = i; q_full[i], q_ready[i] and
-// o_staged[i] the units with un % 2 = i (Q buffer i); o_full and o_free complete once per
-// unit.  Every waiter is at most one phase behind the barrier it waits on (parity waits need
+// (un).  s_full[i], p_full[i] and o_full[i] serve set i (the tiles with tau % 2 = i);
+// q_full[i], q_ready[i] and o_staged[i] the units with un % 2 = i (Q buffer i); o_full[i] and
+// o_free complete once per unit.  Every waiter is at most one phase behind the barrier it waits on (parity waits need
 // that); the waits say why.
 struct TcBars {
   uint64_t k_full[kTcKSlots], k_empty[kTcKSlots];
@@ -525,9 +528,9 @@ struct TcBars {
   uint64_t o_staged[2];  // one arrival per softmax warp: the unit's O staged in its Q buffer
   uint64_t s_full[2];    // MMA commit: scores ready
   uint64_t p_full[2];    // one arrival per warp of the set: P written (and O rescaled)
-  uint64_t o_full;       // MMA commit: every product of the unit done
+  uint64_t o_full[2];    // MMA commit: every product of the unit into O_i done
   uint64_t o_free;       // one arrival per softmax warp: both accumulators read out
-  uint64_t mma_done;     // MMA commit at exit
+  uint64_t mma_done[2];  // MMA commit at exit
   uint32_t tmem;
   int abort;
 };
@@ -654,9 +657,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&bars.s_full[i], 1);
       mbar_init(&bars.p_full[i], 4);
     }
-    mbar_init(&bars.o_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars.o_full[i], 1);
+      mbar_init(&bars.mma_done[i], 1);
+    }
     mbar_init(&bars.o_free, kTcSoftmaxWarps);
-    mbar_init(&bars.mma_done, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -770,15 +775,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int last = i + ((un - 1 - i) / 2) * 2;
         mbar_drain(&bars.q_full[i], (last >> 1) & 1);
       }
-  } else if (warp == 1) {
-    // ================================================================ MMA issuer
-    // Order: S(0), S(1), then per tile tau: O_(tau % 2) += P(tau) V(tau), S(tau + 2).
-    // S(tau + 2) goes into the buffer of P(tau) after the product that reads it, in issue
-    // order.  The warp runs the loop (its values stay warp-uniform) and one elected lane, the
-    // same throughout, issues each group of MMAs with its commits: issued from a divergent
-    // single thread the MMAs of a tile took up to 1.5x the tensor cores' time.  The warp is
-    // the only waiter on q_full / q_ready / k_full / v_full / p_full / o_free and takes each
-    // phase in order.
+  } else if (warp == 1 || warp == kTcMmaWarp1) {
+    // ================================================================ MMA issuers
+    // Warp 1 issues set 0's products, warp 3 set 1's: per set, S of its first tile, then per
+    // tile tau of the set O_s += P(tau) V(tau), S of the set's next tile (into the same buffer,
+    // after the product that reads it, in issue order).  The warp runs the loop (its values
+    // stay warp-uniform) and one elected lane, the same throughout, issues each group of MMAs
+    // with its commits: issued from a divergent single thread the MMAs of a tile took up to
+    // 1.5x the tensor cores' time.  Each unit of the CTA passes both warps: at its start
+    // after both accumulators of the unit before are read out (o_free), at its end with an
+    // o_full commit, also for a unit without a tile of the set.
+    const int ms = warp == 1 ? 0 : 1;
     {
       constexpr uint32_t idesc_s = f16_idesc(kPfRows, kTcKeys, 0);    // Q K^T: both K-major
       constexpr uint32_t idesc_o = f16_idesc(kPfRows, kHeadDim, 1);   // P V: V MN-major
@@ -790,42 +797,46 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint64_t dv0 = sw128_desc(smem_addr(smem + kTcOffV), (uint32_t)kTcHalfBytes, 1024u);
       constexpr uint64_t kQBuf = kTcQBytes >> 4, kQHalf = (kPfRows * 128) >> 4;
       constexpr uint64_t kKHalf = kTcHalfBytes >> 4, kSlot = kTcTileBytes >> 4;
-      // Cursors over the CTA's tiles: the unit and the next one, unit ordinal, tile in unit,
-      // tiles of unit, and the retained count of the next unit (loaded one unit ahead).
+      const uint32_t d_s = tmem + kTcColS + (uint32_t)(128 * ms);  // this set's S buffer
+      const uint32_t d_o = tmem + (uint32_t)(128 * ms);            // and accumulator
+      // Cursor over the set's tiles for the scores: unit and next unit, unit ordinal, tile in
+      // unit, tiles of unit, global tile index, next unit's retained count (one unit ahead).
       struct Cur {
         TcIter it, nx;
-        int un, t, n, nc_next;
+        int un, t, n, tau, nc_next;
       };
-      auto start = [&](Cur& c) {
-        c.it = c.nx = first;
-        tc_advance(p, c.nx, step);
-        c.un = c.t = 0;
-        c.n = tc_valid(p, c.it) ? tc_unit(p, c.it, tc_unit_nc(p, c.it)).n_tiles : 0;
-        c.nc_next = tc_unit_nc(p, c.nx);
-      };
-      auto next = [&](Cur& c) {
-        if (++c.t == c.n) {
-          c.t = 0;
-          c.it = c.nx;
-          tc_advance(p, c.nx, step);
-          ++c.un;
-          c.n = tc_valid(p, c.it) ? tc_unit(p, c.it, c.nc_next).n_tiles : 0;
-          c.nc_next = tc_unit_nc(p, c.nx);
+      Cur sc;
+      sc.it = sc.nx = first;
+      tc_advance(p, sc.nx, step);
+      sc.un = sc.t = sc.tau = 0;
+      sc.n = tc_valid(p, sc.it) ? tc_unit(p, sc.it, tc_unit_nc(p, sc.it)).n_tiles : 0;
+      sc.nc_next = tc_unit_nc(p, sc.nx);
+      auto step_tile = [&]() {
+        ++sc.tau;
+        if (++sc.t == sc.n) {
+          sc.t = 0;
+          sc.it = sc.nx;
+          tc_advance(p, sc.nx, step);
+          ++sc.un;
+          sc.n = tc_valid(p, sc.it) ? tc_unit(p, sc.it, sc.nc_next).n_tiles : 0;
+          sc.nc_next = tc_unit_nc(p, sc.nx);
         }
       };
-      Cur sc, pc;
-      start(sc);
-      start(pc);
-      auto issue_scores = [&](int tau) {
-        const int qi = sc.un & 1;
-        if (sc.t == 0)  // the unit's Q has landed (and, borrowed decisions, is patched)
+      auto seek = [&]() {  // to the set's next tile (n = 0: none left)
+        while (sc.n > 0 && (sc.tau & 1) != ms) step_tile();
+      };
+      auto issue_scores = [&]() {
+        const int tau = sc.tau, qi = sc.un & 1;
+        // the set's first tile of a unit: the unit's Q has landed (and, borrowed decisions,
+        // is patched); q_full is one phase ahead at most, since Q two units on needs this
+        // unit's O staged
+        if (sc.t < kTcSets)
           mbar_wait(p.zero_first ? &bars.q_ready[qi] : &bars.q_full[qi], (sc.un >> 1) & 1,
                     abort_flag, p.err);
         mbar_wait(&bars.k_full[tau % kTcKSlots], (tau / kTcKSlots) & 1, abort_flag, p.err);
         tc_fence_after();
         const uint64_t dq = dq0 + (uint64_t)qi * kQBuf;
         const uint64_t dk = dk0 + (uint64_t)(tau % kTcKSlots) * kSlot;
-        const uint32_t d_s = tmem + kTcColS + (uint32_t)(128 * (tau & 1));
         if (elect_one()) {
           tc_mma_ss_k<false>(d_s, dq, dk, idesc_s);
           tc_mma_ss_k<true>(d_s, dq + 2, dk + 2, idesc_s);
@@ -835,48 +846,61 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           tc_mma_ss_k<true>(d_s, dq + kQHalf + 2, dk + kKHalf + 2, idesc_s);
           tc_mma_ss_k<true>(d_s, dq + kQHalf + 4, dk + kKHalf + 4, idesc_s);
           tc_mma_ss_k<true>(d_s, dq + kQHalf + 6, dk + kKHalf + 6, idesc_s);
-          tc_commit(&bars.s_full[tau & 1]);
+          tc_commit(&bars.s_full[ms]);
           tc_commit(&bars.k_empty[tau % kTcKSlots]);  // the K slot is free once these are done
         }
         __syncwarp();
-        next(sc);
+        step_tile();
+        seek();
       };
-      int s_tau = 0;
-      if (sc.n > 0) issue_scores(s_tau++);
-      if (sc.n > 0) issue_scores(s_tau++);
-      for (int tau = 0; pc.n > 0; ++tau) {
-        // S(tau) was issued after O += P(tau - 2) V: p_full[tau & 1] is one phase ahead at most
-        mbar_wait(&bars.p_full[tau & 1], (tau >> 1) & 1, abort_flag, p.err);
-        // a unit's first product overwrites an accumulator: the previous unit's are read out
-        // (o_free completes once per unit, after o_full, which needs this unit's products)
-        if (pc.t == 0 && pc.un > 0) mbar_wait(&bars.o_free, (pc.un - 1) & 1, abort_flag, p.err);
-        mbar_wait(&bars.v_full[tau % kTcVSlots], (tau / kTcVSlots) & 1, abort_flag, p.err);
-        tc_fence_after();
-        // keys 16 kk .. 16 kk + 15: P columns 8 kk .. of the buffer; V rows 16 kk .. (2 KiB
-        // per 16 rows).  The set's first tile of the unit starts its accumulator.
-        const uint64_t dv = dv0 + (uint64_t)(tau % kTcVSlots) * kSlot;
-        const uint32_t a = tmem + kTcColS + (uint32_t)(128 * (tau & 1));
-        const uint32_t d_o = tmem + (uint32_t)(128 * (tau & 1));
-        const bool first_of_set = pc.t < kTcSets, last_of_unit = pc.t == pc.n - 1;
-        if (elect_one()) {
-          if (first_of_set)
-            tc_mma_ts_k<false>(d_o, a, dv, idesc_o);
-          else
-            tc_mma_ts_k<true>(d_o, a, dv, idesc_o);
-#pragma unroll
-          for (int kk = 1; kk < kTcKeys / 16; ++kk)
-            tc_mma_ts_k<true>(d_o, a + 8 * kk, dv + 128 * kk, idesc_o);
-          tc_commit(&bars.v_empty[tau % kTcVSlots]);
-          if (last_of_unit) tc_commit(&bars.o_full);  // the unit's O is complete
-        }
+      seek();
+      if (sc.n > 0) issue_scores();
+      // products, unit by unit
+      TcIter it = first, nx = first;
+      tc_advance(p, nx, step);
+      int nc = tc_unit_nc(p, it), tau0 = 0, un = 0;
+      for (; tc_valid(p, it); it = nx, tc_advance(p, nx, step), ++un) {
+        const int nc_next = tc_unit_nc(p, nx);  // used one unit later
+        const int n = tc_unit(p, it, nc).n_tiles;
+        // a unit's products overwrite the accumulators: the previous unit's are read out
+        // (o_free completes once per unit, after both o_full of that unit, which need this
+        // warp's commit below)
+        if (un > 0) mbar_wait(&bars.o_free, (un - 1) & 1, abort_flag, p.err);
+        int t = (tau0 & 1) == ms ? 0 : 1;
+        if (t >= n && elect_one()) tc_commit(&bars.o_full[ms]);  // no tile of this set
         __syncwarp();
-        next(pc);
-        if (sc.n > 0) issue_scores(s_tau++);
+        for (; t < n; t += kTcSets) {
+          const int tau = tau0 + t;
+          // S(tau) was issued after the set's previous product: p_full[ms] is one phase
+          // ahead at most
+          mbar_wait(&bars.p_full[ms], (tau >> 1) & 1, abort_flag, p.err);
+          mbar_wait(&bars.v_full[tau % kTcVSlots], (tau / kTcVSlots) & 1, abort_flag, p.err);
+          tc_fence_after();
+          // keys 16 kk .. 16 kk + 15: P columns 8 kk .. of the buffer; V rows 16 kk ..
+          // (2 KiB per 16 rows).  The set's first tile of the unit starts its accumulator.
+          const uint64_t dv = dv0 + (uint64_t)(tau % kTcVSlots) * kSlot;
+          const bool first_of_set = t < kTcSets, last_of_set = t + kTcSets >= n;
+          if (elect_one()) {
+            if (first_of_set)
+              tc_mma_ts_k<false>(d_o, d_s, dv, idesc_o);
+            else
+              tc_mma_ts_k<true>(d_o, d_s, dv, idesc_o);
+#pragma unroll
+            for (int kk = 1; kk < kTcKeys / 16; ++kk)
+              tc_mma_ts_k<true>(d_o, d_s + 8 * kk, dv + 128 * kk, idesc_o);
+            tc_commit(&bars.v_empty[tau % kTcVSlots]);
+            if (last_of_set) tc_commit(&bars.o_full[ms]);  // the set's part of the unit's O
+          }
+          __syncwarp();
+          if (sc.n > 0) issue_scores();
+        }
+        tau0 += n;
+        nc = nc_next;
       }
       // the tensor memory is released only after every product has landed
-      if (elect_one()) tc_commit(&bars.mma_done);
+      if (elect_one()) tc_commit(&bars.mma_done[ms]);
       __syncwarp();
-      mbar_drain(&bars.mma_done, 0);
+      mbar_drain(&bars.mma_done[ms], 0);
     }
   } else {
     // ================================================================ softmax
@@ -901,7 +925,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // accumulators for d-half `set` and stage it as bf16 in the unit's Q buffer.  o_full is
     // one phase ahead at most: the next unit's products need this call's o_free arrival.
     auto finish_unit = [&](int v, float mv, float lv) {
-      mbar_wait(&bars.o_full, v & 1, abort_flag, p.err);
+      mbar_wait(&bars.o_full[0], v & 1, abort_flag, p.err);
+      mbar_wait(&bars.o_full[1], v & 1, abort_flag, p.err);
       tc_fence_after();
       xml[set * kPfRows + row] = make_float2(mv, lv);
       named_barrier_sync_id(1 + quarter, 64);  // the two sets' warps of this quarter
