@@ -675,43 +675,78 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (warp == 0) {
     // ================================================================ K / V producer
     // The whole warp waits and zeroes stale V rows; lane 0 issues the copies.  A slot is
-    // refilled only after the MMAs that read its previous tile are done.
-    int gk = 0;  // tiles staged so far
-    TcIter it = first, nx = first;
-    tc_advance(p, nx, step);
-    int nc = tc_unit_nc(p, it);
-    for (; tc_valid(p, it); it = nx, tc_advance(p, nx, step)) {
-      const int nc_next = tc_unit_nc(p, nx);  // used one unit later
-      const TcUnit x = tc_unit(p, it, nc);
-      for (int t = 0; t < x.n_tiles; ++t, ++gk) {
-        const TcTile tl = tc_tile(t, x.n_ct, x.nc, x.bs, x.jmax);
-        const int ks = gk % kTcKSlots, vs = gk % kTcVSlots;
-        if (gk >= kTcKSlots)
-          mbar_wait(&bars.k_empty[ks], (gk / kTcKSlots - 1) & 1, abort_flag, p.err);
-        if (lane == 0) {
-          mbar_arrive_expect_tx(&bars.k_full[ks], 2u * (uint32_t)tl.rows * 128u);
-          tc_stage_rows(smem + ks * kTcTileBytes, tl.retained ? p.kc : p.kd, x.head, P, tl.r0,
-                        tl.rows, &bars.k_full[ks]);
-        }
-        if (gk >= kTcVSlots)
-          mbar_wait(&bars.v_empty[vs], (gk / kTcVSlots - 1) & 1, abort_flag, p.err);
-        uint8_t* vt = smem + kTcOffV + vs * kTcTileBytes;
-        if (tl.rows < kTcKeys) {
-          const int n16 = (kTcKeys - tl.rows) * 8;  // 16-byte words past the rows, per d-half
-          for (int e = lane; e < 2 * n16; e += 32) {
-            const int dh = e >= n16 ? 1 : 0;
-            *reinterpret_cast<uint4*>(vt + dh * kTcHalfBytes + tl.rows * 128 + (e - dh * n16) * 16) =
-                make_uint4(0u, 0u, 0u, 0u);
-          }
-          fence_proxy_async_smem();  // visible to the tensor cores via the full barrier
-          __syncwarp();
-        }
-        if (lane == 0) {
-          mbar_arrive_expect_tx(&bars.v_full[vs], 2u * (uint32_t)tl.rows * 128u);
-          tc_stage_rows(vt, tl.retained ? p.vc : p.vd, x.head, P, tl.r0, tl.rows, &bars.v_full[vs]);
-        }
+    // refilled only after the MMAs that read its previous tile are done.  K runs two tiles
+    // ahead of V in this warp's order (K(g + 2) before V(g)): a V slot is freed by the
+    // product two tiles back, which must not hold up the keys the next scores need.
+    struct PCur {  // a tile of the CTA: unit, next unit, its fields, tile in unit
+      TcIter it, nx;
+      TcUnit x;
+      int nc_next, t;
+      bool valid;
+    };
+    auto pstart = [&](PCur& c) {
+      c.it = c.nx = first;
+      tc_advance(p, c.nx, step);
+      c.valid = tc_valid(p, c.it);
+      c.x = tc_unit(p, c.it, tc_unit_nc(p, c.it));
+      c.nc_next = tc_unit_nc(p, c.nx);  // used one unit later
+      c.t = 0;
+    };
+    auto pnext = [&](PCur& c) {
+      if (++c.t == c.x.n_tiles) {
+        c.t = 0;
+        c.it = c.nx;
+        tc_advance(p, c.nx, step);
+        c.valid = tc_valid(p, c.it);
+        c.x = tc_unit(p, c.it, c.nc_next);
+        c.nc_next = tc_unit_nc(p, c.nx);
       }
-      nc = nc_next;
+    };
+    PCur kc, vc;
+    pstart(kc);
+    pstart(vc);
+    int gk = 0, gv = 0;  // K and V tiles staged so far
+    auto load_k = [&]() {
+      const TcTile tl = tc_tile(kc.t, kc.x.n_ct, kc.x.nc, kc.x.bs, kc.x.jmax);
+      const int ks = gk % kTcKSlots;
+      if (gk >= kTcKSlots)
+        mbar_wait(&bars.k_empty[ks], (gk / kTcKSlots - 1) & 1, abort_flag, p.err);
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars.k_full[ks], 2u * (uint32_t)tl.rows * 128u);
+        tc_stage_rows(smem + ks * kTcTileBytes, tl.retained ? p.kc : p.kd, kc.x.head, P, tl.r0,
+                      tl.rows, &bars.k_full[ks]);
+      }
+      ++gk;
+      pnext(kc);
+    };
+    auto load_v = [&]() {
+      const TcTile tl = tc_tile(vc.t, vc.x.n_ct, vc.x.nc, vc.x.bs, vc.x.jmax);
+      const int vs = gv % kTcVSlots;
+      if (gv >= kTcVSlots)
+        mbar_wait(&bars.v_empty[vs], (gv / kTcVSlots - 1) & 1, abort_flag, p.err);
+      uint8_t* vt = smem + kTcOffV + vs * kTcTileBytes;
+      if (tl.rows < kTcKeys) {
+        const int n16 = (kTcKeys - tl.rows) * 8;  // 16-byte words past the rows, per d-half
+        for (int e = lane; e < 2 * n16; e += 32) {
+          const int dh = e >= n16 ? 1 : 0;
+          *reinterpret_cast<uint4*>(vt + dh * kTcHalfBytes + tl.rows * 128 + (e - dh * n16) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();  // visible to the tensor cores via the full barrier
+        __syncwarp();
+      }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars.v_full[vs], 2u * (uint32_t)tl.rows * 128u);
+        tc_stage_rows(vt, tl.retained ? p.vc : p.vd, vc.x.head, P, tl.r0, tl.rows, &bars.v_full[vs]);
+      }
+      ++gv;
+      pnext(vc);
+    };
+    // K(g + 2) needs only the scores of tile g - 1, whose V was staged before: no cycle
+    for (int i = 0; i < 2 && kc.valid; ++i) load_k();
+    while (vc.valid) {
+      if (kc.valid) load_k();
+      load_v();
     }
     // no copy may still be in flight when the CTA exits (matters only after a timeout)
     if (lane == 0) {
@@ -719,8 +754,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int last = s + ((gk - 1 - s) / kTcKSlots) * kTcKSlots;
         mbar_drain(&bars.k_full[s], (last / kTcKSlots) & 1);
       }
-      for (int s = 0; s < kTcVSlots && s < gk; ++s) {
-        const int last = s + ((gk - 1 - s) / kTcVSlots) * kTcVSlots;
+      for (int s = 0; s < kTcVSlots && s < gv; ++s) {
+        const int last = s + ((gv - 1 - s) / kTcVSlots) * kTcVSlots;
         mbar_drain(&bars.v_full[s], (last / kTcVSlots) & 1);
       }
     }
