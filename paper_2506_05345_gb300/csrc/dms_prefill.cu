@@ -459,7 +459,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_attn_kernel(const Prefi
 // M 128 x N 128 x K 16 (on this tensor core an N 64 MMA costs 3/4 of the time of an N 128 one
 // for half its work).
 // 384 threads: warp 0 stages the K tiles (3-slot ring) and V tiles (2-slot ring) of the units
-// with bulk copies; warp 2 moves Q in and O out (tensor-map copies, 128-byte swizzle: a Q tile
+// with bulk copies, K two tiles ahead of V; warp 2 moves Q in and O out (tensor-map copies, 128-byte swizzle: a Q tile
 // lands in the MMA operand layout; two Q buffers, each also staging its unit's O); warps 4-11
 // run the softmax as two sets of four warps, one thread per query row in each (a warp reaches
 // only TMEM lanes 32 (warp % 4) ..).  Set s takes the key tiles of one parity: tile tau of the
