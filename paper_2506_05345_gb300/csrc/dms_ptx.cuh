@@ -129,11 +129,6 @@ __device__ __forceinline__ void bulk_commit_group() {
 __device__ __forceinline__ void bulk_wait_group_read0() {
   asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
-// Barrier kId (1..15) over `count` threads (a multiple of 32) of the CTA.
-template <int kId>
-__device__ __forceinline__ void named_barrier_sync(int count) {
-  asm volatile("bar.sync %0, %1;" ::"n"(kId), "r"(count) : "memory");
-}
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
                                         uint32_t& r3) {
@@ -270,18 +265,8 @@ __host__ __device__ constexpr uint32_t f16_idesc(int m, int n, int b_mn_major) {
          ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
-// D[tmem] (+)= A[smem] * B[smem]; issued by one thread.
-__device__ __forceinline__ void tc_mma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                          uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// As tc_mma_ss with the accumulate flag fixed at compile time (no predicate setup).
+// D[tmem] (+)= A[smem] * B[smem], the accumulate flag fixed at compile time; issued by one
+// thread.
 template <bool kAccumulate>
 __device__ __forceinline__ void tc_mma_ss_k(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                             uint32_t idesc) {
@@ -376,41 +361,6 @@ __device__ __forceinline__ void tmem_st8_u32(uint32_t taddr, const uint32_t* r) 
                "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
                "r"(r[7])
                : "memory");
-}
-// 16 32-bit words into 16 consecutive columns of this thread's lane.
-__device__ __forceinline__ void tmem_st16_u32(uint32_t taddr, const uint32_t* r) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
-      : "memory");
-}
-// One 32-bit word into one column of this thread's lane.
-__device__ __forceinline__ void tmem_st1_f32(uint32_t taddr, float v) {
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr),
-               "r"(__float_as_uint(v))
-               : "memory");
-}
-// Four consecutive columns of this thread's lane (complete after tmem_wait_ld).
-__device__ __forceinline__ void tmem_ld4(uint32_t taddr, float (&r)[4]) {
-  uint32_t a, b, c, d;
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
-               : "r"(taddr)
-               : "memory");
-  r[0] = __uint_as_float(a);
-  r[1] = __uint_as_float(b);
-  r[2] = __uint_as_float(c);
-  r[3] = __uint_as_float(d);
-}
-// Order-preserving map of a float (not NaN) to an int and back: integer max = float max.
-__device__ __forceinline__ int ordered_key(float f) {
-  const int i = __float_as_int(f);
-  return i >= 0 ? i : i ^ 0x7fffffff;
-}
-__device__ __forceinline__ float from_ordered_key(int k) {
-  return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff);
 }
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
