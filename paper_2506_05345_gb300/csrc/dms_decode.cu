@@ -872,6 +872,14 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       bool rescale = false;
       float ce[NT], co[NT];
       uint32_t pb[NT][2];
+      // fp8: each value's row scale is folded into P (O^T += V^T (s P^T)), per token instead
+      // of per value; stale tokens take 0 (their P is 0 and their scale word is not theirs)
+      float vs0 = 1.f, vs1 = 1.f;
+      if constexpr (kFp8) {
+        const float* vsc = reinterpret_cast<const float*>(st + kOffScales) + kPageTokens;
+        vs0 = v0 ? vsc[tb + g] : 0.f;
+        vs1 = v1 ? vsc[tb + g + 8] : 0.f;
+      }
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
         const float s0 = v0 ? (sa[nt][0] + sb[nt][0]) * sl0 : -INFINITY;
@@ -896,8 +904,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
         rescale |= (ce[nt] != 1.f) || (co[nt] != 1.f);
         // (token g, heads 2c..) -> transpose -> (head g, tokens 2c..): the B operand
         if constexpr (kFp8) {
-          pb[nt][0] = movmatrix_trans(pack_f16x2(p0, p1));
-          pb[nt][1] = movmatrix_trans(pack_f16x2(p2, p3));
+          pb[nt][0] = movmatrix_trans(pack_f16x2(p0 * vs0, p1 * vs0));
+          pb[nt][1] = movmatrix_trans(pack_f16x2(p2 * vs1, p3 * vs1));
         } else {
           pb[nt][0] = movmatrix_trans(pack_bf16x2(p0, p1));
           pb[nt][1] = movmatrix_trans(pack_bf16x2(p2, p3));
@@ -923,10 +931,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       }
       if constexpr (kFp8) {
         // V^T rows d = 16 mt + g and + 8: one word holds the codes of tokens tb + {2c, 2c+1,
-        // 2c+8, 2c+9}; each value times its token's scale (f16), stale tokens masked after
-        const float* vsc = reinterpret_cast<const float*>(st + kOffScales) + kPageTokens;
-        const uint32_t sv01 = pack_f16x2(vsc[tb + 2 * c4], vsc[tb + 2 * c4 + 1]);
-        const uint32_t sv89 = pack_f16x2(vsc[tb + 2 * c4 + 8], vsc[tb + 2 * c4 + 9]);
+        // 2c+8, 2c+9} (the row scales are in P); stale tokens masked
         const int blk = tb >> 4;
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) {
@@ -936,10 +941,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
           const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
               st + kKvHalf + d1 * 64 + ((blk ^ ((d1 >> 1) & 3)) << 4) + 4 * c4);
           uint32_t a[4];
-          a[0] = hmul2_u32(e4m3x2_to_f16x2(w0), sv01) & mk_lo;
-          a[1] = hmul2_u32(e4m3x2_to_f16x2(w1), sv01) & mk_lo;
-          a[2] = hmul2_u32(e4m3x2_to_f16x2(w0 >> 16), sv89) & mk_hi;
-          a[3] = hmul2_u32(e4m3x2_to_f16x2(w1 >> 16), sv89) & mk_hi;
+          a[0] = e4m3x2_to_f16x2(w0) & mk_lo;
+          a[1] = e4m3x2_to_f16x2(w1) & mk_lo;
+          a[2] = e4m3x2_to_f16x2(w0 >> 16) & mk_hi;
+          a[3] = e4m3x2_to_f16x2(w1 >> 16) & mk_hi;
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) mma_f16_16816(o[mt][nt], a, pb[nt][0], pb[nt][1]);
         }
