@@ -353,14 +353,39 @@ dms_status dms_cache_layer_length(const dms_cache* cache, int32_t layer, int64_t
  * capture.  Every call clears the scratch counters it needs with an asynchronous
  * memset on `stream` and then launches; all calls share the one array, so calls
  * whose work overlaps on the GPU (other streams, other host threads) race and
- * must be serialised by the caller.  A bounded in-kernel wait that gives up is
- * recorded only in the scratch array, not reported.
+ * must be serialised by the caller.  A bounded in-kernel wait that gives up
+ * (DMS_ERR_TIMEOUT) does not change the return code, which reports only what the
+ * host saw; it is kept in the scratch array's error word until the next call
+ * clears it, and dms_decode_noalloc_device_error reads it.
+ * page_table and counts must be 4-byte aligned.
  */
 dms_status dms_decode_attention_paged_noalloc(const void* pool, const int32_t* page_table,
                                               const int32_t* counts, int32_t batch,
                                               int32_t kv_heads, int32_t max_pages,
                                               const void* q, void* out, int32_t gqa_group,
                                               float sm_scale, void* stream);
+
+/*
+ * Device-side status of the last dms_decode_attention_paged_noalloc call on the
+ * current device (no counterpart in the paper: failure detection of the
+ * implementation).  Synchronises `stream`, then writes into *out the error word
+ * that call's kernel left in the static scratch array: DMS_OK, or DMS_ERR_TIMEOUT
+ * when one of its bounded shared-memory barrier waits gave up (its outputs are
+ * then not valid).  Allocates nothing: the word is copied into host stack memory.
+ * Returns DMS_ERR_CUDA if the copy or the synchronisation fails.
+ */
+dms_status dms_decode_noalloc_device_error(void* stream, dms_status* out);
+
+/*
+ * Self-test of that report (no counterpart in the paper).  Clears the static
+ * scratch array's error word, then runs on `stream` a small kernel whose bounded
+ * barrier wait can never complete, with the limit `limit_ns` (1 us .. 10 s): the
+ * wait gives up, records DMS_ERR_TIMEOUT in the error word exactly as a decode
+ * kernel would, and the kernel exits normally, so the CUDA context stays usable.
+ * dms_decode_noalloc_device_error then reports DMS_ERR_TIMEOUT until the next
+ * allocation-free decode clears the word.  Synchronises `stream`; allocates nothing.
+ */
+dms_status dms_selftest_noalloc_timeout(int64_t limit_ns, void* stream);
 
 /*
  * Self-test of the bounded wait every kernel of this library uses on its

@@ -213,6 +213,17 @@ def dms_decode_attention_paged_noalloc(pool_ptr, page_table_ptr, counts_ptr, bat
         gqa_group, float(sm_scale), stream)
 
 
+def dms_decode_noalloc_device_error(stream):
+    """(status of the call, device-side status of the last allocation-free decode)."""
+    out = ctypes.c_int(0)
+    code = library().dms_decode_noalloc_device_error(stream, ctypes.byref(out))
+    return code, out.value
+
+
+def dms_selftest_noalloc_timeout(limit_ns, stream):
+    return library().dms_selftest_noalloc_timeout(int(limit_ns), stream)
+
+
 def dms_selftest_bounded_wait(arrive, limit_ns, stream):
     return library().dms_selftest_bounded_wait(int(arrive), int(limit_ns), stream)
 

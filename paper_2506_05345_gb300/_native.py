@@ -37,7 +37,7 @@ EXPORTS = (
     "dms_decode_attention_borrowed", "dms_append_and_decode_borrowed",
     "dms_prefill_workspace_bytes", "dms_prefill_attention", "dms_prefill_attention_borrowed",
     "dms_prefill_device_error", "dms_prefill_attention_ex", "dms_append_shared_prefix",
-    "dms_cache_export_kv",
+    "dms_cache_export_kv", "dms_decode_noalloc_device_error", "dms_selftest_noalloc_timeout",
 )
 
 
@@ -106,6 +106,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_status_string": (ctypes.c_char_p, [st]),
         "dms_decode_attention_paged_noalloc": (st, [vp, vp, vp, i32, i32, i32, vp, vp, i32, f32,
                                                     vp]),
+        "dms_decode_noalloc_device_error": (st, [vp, ctypes.POINTER(st)]),
+        "dms_selftest_noalloc_timeout": (st, [i64, vp]),
     }
     for name, (res, args) in proto.items():
         fn = getattr(lib, name)

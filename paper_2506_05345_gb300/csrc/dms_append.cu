@@ -154,7 +154,8 @@ __global__ void __launch_bounds__(256) append_one_kernel(const AppendParams p) {
       ring[j % RP] = (uint32_t)slot | ((p.decider == 0 ? alpha : 0u) << 31);
       if (p.decider > 0 && j >= p.decider) ring[(j - p.decider) % RP] |= alpha << 31;
       page = pt[slot / kPageTokens];
-      p.pos[(int64_t)page * kPageTokens + (slot & (kPageTokens - 1))] = (int32_t)j;
+      if (page < 0) ok = 0;  // a fused step could not open this slot's page
+      else p.pos[(int64_t)page * kPageTokens + (slot & (kPageTokens - 1))] = (int32_t)j;
     }
   }
   ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -314,8 +315,10 @@ __global__ void __launch_bounds__(kBulkThreads) append_bulk_kernel(const AppendP
         if (sl[u] >= 0) {
           const int32_t page = pt[sl[u] / kPageTokens];
           const uint32_t row = (uint32_t)(sl[u] & (kPageTokens - 1));
-          store_kv_row(p, page, row, lane, val[u]);
-          if (lane == 0) p.pos[(int64_t)page * kPageTokens + row] = (int32_t)(t0 + base + t + u);
+          if (page >= 0) {  // -1: a fused step could not open this slot's page
+            store_kv_row(p, page, row, lane, val[u]);
+            if (lane == 0) p.pos[(int64_t)page * kPageTokens + row] = (int32_t)(t0 + base + t + u);
+          }
         }
       }
     }
@@ -387,7 +390,10 @@ __global__ void export_positions_kernel(const int32_t* counts, const int32_t* pa
   int32_t* o = out + (int64_t)bh * capacity;
   for (int64_t s = threadIdx.x; s < capacity; s += blockDim.x) {
     int32_t val = -1;
-    if (s < n) val = pos[(int64_t)pt[s / kPageTokens] * kPageTokens + (s & (kPageTokens - 1))];
+    if (s < n) {
+      const int32_t page = pt[s / kPageTokens];  // -1: a page the pool could not give
+      val = page < 0 ? -1 : pos[(int64_t)page * kPageTokens + (s & (kPageTokens - 1))];
+    }
     o[s] = val;
   }
 }

@@ -38,6 +38,11 @@ void free_device(Cache& c) {
   c.pieces = nullptr;
 }
 
+void free_host(Cache& c) {
+  free(c.lengths);
+  c.lengths = nullptr;
+}
+
 template <typename T>
 cudaError_t alloc(T** p, size_t count) {
   return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) > 0 ? count * sizeof(T) : 16);
@@ -139,7 +144,7 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
     const bool oom = (e == cudaErrorMemoryAllocation);
     cudaGetLastError();
     free_device(c);
-    free(c.lengths);
+    free_host(c);
     delete h;
     return oom ? DMS_ERR_OUT_OF_MEMORY : DMS_ERR_CUDA;
   }
@@ -151,7 +156,7 @@ dms_status dms_cache_destroy(dms_cache* h) {
   if (h == nullptr) return DMS_OK;
   cudaDeviceSynchronize();
   free_device(h->c);
-  free(h->c.lengths);
+  free_host(h->c);
   delete h;
   return DMS_OK;
 }
@@ -174,6 +179,7 @@ dms_status dms_cache_reset(dms_cache* h, void* stream) {
     return DMS_ERR_CUDA;
   for (int l = 0; l < c.layers; ++l) c.lengths[l] = 0;
   c.last_layer = -1;
+  c.last_full_tiled = false;
   return DMS_OK;
 }
 
@@ -202,6 +208,7 @@ dms_status append_impl(dms_cache* h, int32_t layer, const void* k, const void* v
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = t0 + n_tokens;
   c.last_layer = layer;
+  c.last_full_tiled = false;
   return DMS_OK;
 }
 
@@ -222,6 +229,7 @@ dms_status decode_impl(dms_cache* h, int32_t layer, const void* q, void* out, in
                                  zero_first, st);
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.last_layer = layer;
+  c.last_full_tiled = c.decode_kernel == DMS_DECODE_TILED && dms::tiled_one_cta_per_sm(c);
   return DMS_OK;
 }
 
@@ -249,6 +257,7 @@ dms_status append_decode_impl(dms_cache* h, int32_t layer, const void* k, const 
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = t0 + 1;
   c.last_layer = layer;
+  c.last_full_tiled = true;
   return DMS_OK;
 }
 
@@ -288,6 +297,7 @@ dms_status dms_append_shared_prefix(dms_cache* h, int32_t layer, const void* k, 
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.lengths[layer] = n_tokens;
   c.last_layer = layer;
+  c.last_full_tiled = false;
   return DMS_OK;
 }
 

@@ -107,10 +107,16 @@ struct DecodeParams {
   int64_t j, window, pool_pages;
   int64_t decider;  // the eviction bit of token i is the decision of token i + decider
   int32_t ring_len;
-  // Nonzero when the kernel launched just before on the stream cannot have written
-  // this layer's cache state (it served another layer): the state is read, and the
-  // first pages are staged, before waiting for that kernel; only the inputs (q, the
-  // new K/V rows, the logits), the outputs and the shared split-K scratch wait.
+  // Nonzero when the launch just before on the stream was a tiled decode of another layer
+  // with one CTA per SM: the state is then read, and the first pages are staged, before
+  // waiting for that kernel; only the inputs (q, the new K/V rows, the logits), the
+  // outputs and the shared split-K scratch wait.  Why that is safe: this launch's CTAs
+  // start only after the launch before has started all its CTAs (programmatic launch).
+  // Those CTAs need more than half an SM's shared memory each, one per SM, and every one
+  // of them -- also one without pages -- waits for ITS predecessor before it exits.  So
+  // while the launch two back runs, the launch before fills every SM and no CTA of this
+  // launch can be resident: whatever last wrote this layer (two or more launches back) has
+  // completed.
   int32_t state_ready;
   // Nonzero: attend with element 0 of every group's first query head taken as 0 (that
   // element carries the decision logit, App. B).
@@ -178,7 +184,7 @@ size_t tiled_smem_bytes(int heads, int stages) {
   using PL = Plan<NT>;
   return (size_t)stages * stage_bytes(kFused, kFp8) +
          (size_t)PL::kSlots * (PL::kSlotOFloats + PL::kSlotMLFloats) * 4 +
-         (size_t)(2 * stages + 2 * PL::kSlots) * sizeof(uint64_t) + 64 +
+         (size_t)(2 * stages + 2 * PL::kSlots + 1) * sizeof(uint64_t) + 64 +
          (size_t)((kFused ? 3 : 2) * heads + 1) * sizeof(int32_t);
 }
 
@@ -236,7 +242,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   uint64_t* mfull_bar = empty_bar + kStages;
   uint64_t* mempty_bar = mfull_bar + PL::kSlots;
   // s_misc: [0] abort, [2..7] warp sums, [8..8+kStages) page id staged in each stage
-  int* s_misc = reinterpret_cast<int*>(mempty_bar + PL::kSlots);
+  uint64_t* rec_bar = mempty_bar + PL::kSlots;  // records of the CTA's last head (prefetch)
+  int* s_misc = reinterpret_cast<int*>(rec_bar + 1);
   int32_t* s_cnt = s_misc + 16;                                   // [heads] n_h (after the append)
   int32_t* s_pstart = s_cnt + p.heads;                            // [heads + 1]
   // fused: new token's slot | fresh << 30 per head
@@ -258,6 +265,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       mbar_init(&mfull_bar[s], kConsumerWarps);
       mbar_init(&mempty_bar[s], 1);
     }
+    mbar_init(rec_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   // While the previous kernel finishes, warm L2 with the small tables the prologue
@@ -265,16 +273,20 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   // entries and decision logits).  L2 is coherent with the previous kernel's
   // writes, so a prefetch can never make a later load stale.
   {
-    const size_t pt_bytes = (size_t)heads * p.max_pages * sizeof(int32_t);
-    const size_t slice = ((pt_bytes + gridDim.x - 1) / gridDim.x + 15) & ~(size_t)15;
+    // The bulk prefetch wants a 16-byte aligned start and length: it covers the
+    // 16-byte aligned span inside the layer's page table (whose base need not be
+    // aligned), split into per-CTA slices of whole 16-byte units.
+    const uintptr_t pt_lo = (reinterpret_cast<uintptr_t>(p.page_table) + 15) & ~(uintptr_t)15;
+    const uintptr_t pt_hi = (reinterpret_cast<uintptr_t>(p.page_table) +
+                             (size_t)heads * p.max_pages * sizeof(int32_t)) & ~(uintptr_t)15;
+    const size_t span = pt_hi > pt_lo ? (size_t)(pt_hi - pt_lo) : 0;
+    const size_t slice = ((span + gridDim.x - 1) / gridDim.x + 15) & ~(size_t)15;
     const size_t beg = slice * blockIdx.x;
-    if (tid == 0 && beg < pt_bytes) {
-      const size_t len = (beg + slice <= pt_bytes ? slice : pt_bytes - beg) & ~(size_t)15;
-      if (len > 0)
-        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(
-                         reinterpret_cast<const uint8_t*>(p.page_table) + beg),
-                     "r"((uint32_t)len)
-                     : "memory");
+    if (tid == 0 && beg < span) {
+      const size_t len = beg + slice <= span ? slice : span - beg;  // a multiple of 16
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(pt_lo + beg),
+                   "r"((uint32_t)len)
+                   : "memory");
     }
     for (int h = blockIdx.x * kThreads + tid; h < heads; h += gridDim.x * kThreads) {
       asm volatile("prefetch.global.L2 [%0];" ::"l"(p.counts + h));
@@ -303,9 +315,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
 #pragma unroll
       for (int i = 0; i < kPer; ++i) {
         const int h = base + tid + i * kThreads;
-        if (h < heads) {
-          nn[i] = p.counts[h];
-          if constexpr (kFused) ee[i] = p.j >= R ? p.ring[(int64_t)h * p.ring_len + (p.j - R) % RP] : 0u;
+        if (h < heads) {  // L2 reads (the state may come from a kernel that ran on this SM)
+          nn[i] = __ldcg(p.counts + h);
+          if constexpr (kFused)
+            ee[i] = p.j >= R ? __ldcg(p.ring + (int64_t)h * p.ring_len + (p.j - R) % RP) : 0u;
         }
       }
 #pragma unroll
@@ -363,7 +376,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   if (P < 1) P = 1;
   if (P > (int)gridDim.x) P = (int)gridDim.x;
   const int k = blockIdx.x;
-  if (k >= P) return;
+  if (k >= P) {  // no pages: still wait for the previous kernel before leaving (see state_ready)
+    if (p.state_ready) pdl_wait_prerequisites();
+    return;
+  }
   Partition split;
   split.init(N, P);
   const int pbeg = split.begin(k), pend = split.begin(k + 1);
@@ -444,14 +460,13 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
         }
         if (new_page) {  // fused: the new token opens a page
           page = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
-          if ((int64_t)page >= p.pool_pages) {
+          if ((int64_t)page >= p.pool_pages) {  // entered as -1: nothing is written there
             set_device_error(p.ctrl, DMS_ERR_CAPACITY);
             page = -1;
-          } else {
-            p.page_table[(int64_t)hh * p.max_pages + pg] = page;
           }
+          p.page_table[(int64_t)hh * p.max_pages + pg] = page;
         } else {
-          page = __ldg(p.page_table + (int64_t)hh * p.max_pages + pg);
+          page = __ldcg(p.page_table + (int64_t)hh * p.max_pages + pg);
         }
       }
       const int nb = min(32, niters - it0);
@@ -692,6 +707,11 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   // every other CTA of a split head has already arrived, this CTA merges their
   // records directly, without publishing its own.
   int arrivals_seen = -1;
+  // Thread 0, when every other CTA of the last segment's split head has arrived by its
+  // last page: their records are copied (bulk) into the idle merge slot while that page
+  // is computed, so the merge that ends the CTA waits for no round trip.
+  int pre_rec = 0;
+  const uint32_t rec_bytes = (uint32_t)(2 * kMaxGroup + G * kHeadDim) * 4u;  // m, l, G rows of O
 
   for (int it = 0; it < niters; ++it) {
     walk.enter(it);
@@ -702,8 +722,31 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
     const bool seg_end = walk.seg_end(it, niters);
     uint8_t* st = stages + s * kStageBytes;
     if (it == niters - 1 && tid == 0 &&
-        split.cta_of(s_pstart[walk.h]) != split.cta_of(s_pstart[walk.h + 1] - 1))
+        split.cta_of(s_pstart[walk.h]) != split.cta_of(s_pstart[walk.h + 1] - 1)) {
       arrivals_seen = ld_relaxed_gpu(p.piece_counters + walk.h);
+      if constexpr (PL::kSlots == 2) {
+        const int k_lo = split.cta_of(s_pstart[walk.h]), k_hi = split.cta_of(s_pstart[walk.h + 1] - 1);
+        const int others = k_hi - k_lo;
+        if (arrivals_seen == others && (uint32_t)others * rec_bytes <= (uint32_t)PL::kSlotOFloats * 4u) {
+          asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
+          // the other merge slot is idle once the epilogue has finished the previous segment
+          const int other = (q + 1) % PL::kSlots;
+          if (q >= 1) mbar_wait(&mempty_bar[other], ((q - 1) / PL::kSlots) & 1, abort_flag, p.ctrl);
+          fence_proxy_async_shared();
+          fence_proxy_async_global();
+          uint8_t* dst = reinterpret_cast<uint8_t*>(merge_o + other * PL::kSlotOFloats);
+          mbar_arrive_expect_tx(rec_bar, (uint32_t)others * rec_bytes);
+          int u = 0;
+          for (int kk = k_lo; kk <= k_hi; ++kk) {
+            if (kk == k) continue;
+            bulk_copy_g2s(dst + (size_t)u * rec_bytes,
+                          p.pieces + (int64_t)(kk + walk.h) * kPieceFloats, rec_bytes, rec_bar);
+            ++u;
+          }
+          pre_rec = 1;
+        }
+      }
+    }
     mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
 
     if constexpr (kFused) {
@@ -815,12 +858,14 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
     }
 
     if (tb < nvalid) {
-      // ---- S^T = K Q^T for tokens tb .. tb+15: two independent chains over k
-      float sa[NT][4], sb[NT][4];
+      // ---- S^T = K Q^T for tokens tb .. tb+15: four independent chains over k
+      float sacc[4][NT][4];
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
+      for (int c = 0; c < 4; ++c)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) sa[nt][e] = sb[nt][e] = 0.f;
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) sacc[c][nt][e] = 0.f;
       if constexpr (kFp8) {
         // rows tb + g and tb + g + 8; the 16-byte chunk of k-steps 4 kg .. 4 kg + 3 holds
         // this thread's codes (d = 16 kk + {2c, 2c+1, 2c+8, 2c+9}) in word kk % 4
@@ -840,10 +885,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
             a[2] = e4m3x2_to_f16x2(x0[i] >> 16);
             a[3] = e4m3x2_to_f16x2(x1[i] >> 16);
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              if (kk & 1) mma_f16_16816(sb[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
-              else mma_f16_16816(sa[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
-            }
+            for (int nt = 0; nt < NT; ++nt) mma_f16_16816(sacc[kk & 3][nt], a, qb[kk][nt][0], qb[kk][nt][1]);
           }
         }
       } else {
@@ -854,10 +896,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
           uint32_t a[4];
           ldsm_x4(kbase + swizzled_offset(row, (uint32_t)(2 * kk + (mi >> 1))), a[0], a[1], a[2], a[3]);
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (kk & 1) mma_bf16_16816(sb[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
-            else mma_bf16_16816(sa[nt], a, qb[kk][nt][0], qb[kk][nt][1]);
-          }
+          for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(sacc[kk & 3][nt], a, qb[kk][nt][0], qb[kk][nt][1]);
         }
       }
       // ---- mask tokens past n_valid, online softmax per head (column), P^T fragments
@@ -882,10 +921,14 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       }
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        const float s0 = v0 ? (sa[nt][0] + sb[nt][0]) * sl0 : -INFINITY;
-        const float s1 = v0 ? (sa[nt][1] + sb[nt][1]) * sl0 : -INFINITY;
-        const float s2 = v1 ? (sa[nt][2] + sb[nt][2]) * sl1 : -INFINITY;
-        const float s3 = v1 ? (sa[nt][3] + sb[nt][3]) * sl1 : -INFINITY;
+        float sc[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          sc[e] = (sacc[0][nt][e] + sacc[1][nt][e]) + (sacc[2][nt][e] + sacc[3][nt][e]);
+        const float s0 = v0 ? sc[0] * sl0 : -INFINITY;
+        const float s1 = v0 ? sc[1] * sl0 : -INFINITY;
+        const float s2 = v1 ? sc[2] * sl1 : -INFINITY;
+        const float s3 = v1 ? sc[3] * sl1 : -INFINITY;
         float xe = fmaxf(s0, s2), xo = fmaxf(s1, s3);
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
@@ -893,12 +936,12 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
           xo = fmaxf(xo, __shfl_xor_sync(0xffffffffu, xo, off));
         }
         const float ne = fmaxf(me[nt], xe), no = fmaxf(mo[nt], xo);
-        ce[nt] = exp2f(me[nt] - ne);
-        co[nt] = exp2f(mo[nt] - no);
+        ce[nt] = ex2_approx(me[nt] - ne);  // 0 while the running max is -inf
+        co[nt] = ex2_approx(mo[nt] - no);
         me[nt] = ne;
         mo[nt] = no;
-        const float p0 = exp2f(s0 - ne), p1 = exp2f(s1 - no);
-        const float p2 = exp2f(s2 - ne), p3 = exp2f(s3 - no);
+        const float p0 = ex2_approx(s0 - ne), p1 = ex2_approx(s1 - no);
+        const float p2 = ex2_approx(s2 - ne), p3 = ex2_approx(s3 - no);
         le[nt] = le[nt] * ce[nt] + (p0 + p2);
         lo[nt] = lo[nt] * co[nt] + (p1 + p3);
         rescale |= (ce[nt] != 1.f) || (co[nt] != 1.f);
@@ -1012,13 +1055,14 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
         if (tid == 0) {
           int early = 0;
           if (!single && arrivals_seen == k_hi - k_lo) {
-            asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
+            if (!pre_rec) asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
             early = 1;
           }
-          s_misc[1] = early;
+          s_misc[1] = early | (pre_rec << 1);
         }
         consumer_bar_sync();
-        const bool early_last = s_misc[1] != 0;
+        const bool early_last = (s_misc[1] & 1) != 0;
+        const bool prefetched = (s_misc[1] & 2) != 0;
         constexpr int RPW = HP / kConsumerWarps;  // rows per warp
         const int d4 = 4 * lane;
         __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
@@ -1097,6 +1141,11 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
               Or[i] = make_float4(0.f, 0.f, 0.f, 0.f);
             }
             constexpr int kBatch = NT == 1 ? 4 : 2;
+            // prefetched records: in the idle merge slot, CTA order without this CTA's
+            const float* rec_smem = merge_o + ((q + 1) % PL::kSlots) * PL::kSlotOFloats;
+            if (prefetched) {
+              if (!mbar_wait(rec_bar, 0, abort_flag, p.ctrl)) mbar_drain(rec_bar, 0);
+            }
             for (int kk0 = k_lo; kk0 <= k_hi; kk0 += kBatch) {
               float mb[kBatch][RPW], lb[kBatch][RPW];
               float4 ob[kBatch][RPW];
@@ -1111,6 +1160,11 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
                     mb[u][i] = Mo[i];
                     lb[u][i] = Lo[i];
                     ob[u][i] = Oo[i];
+                  } else if (kk <= k_hi && r < G && prefetched) {
+                    const float* rs = rec_smem + (size_t)(kk - k_lo - (kk > k ? 1 : 0)) * (rec_bytes / 4u);
+                    mb[u][i] = rs[r];
+                    lb[u][i] = rs[kMaxGroup + r];
+                    ob[u][i] = *reinterpret_cast<const float4*>(rs + 2 * kMaxGroup + r * kHeadDim + d4);
                   } else if (kk <= k_hi && r < G) {
                     mb[u][i] = __ldcg(rk + r);
                     lb[u][i] = __ldcg(rk + kMaxGroup + r);
@@ -1179,6 +1233,7 @@ __global__ void __launch_bounds__(128) decode_simple_kernel(const uint8_t* pool,
     float m = -INFINITY, l = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
     for (int s = 0; s < n; ++s) {
       const int32_t page = pt[s / kPageTokens];
+      if (page < 0) continue;  // the page pool ran out when this slot's page was to open
       const uint32_t row = (uint32_t)(s & (kPageTokens - 1));
       const uint8_t* kp = pool + (int64_t)page * kPageBytes;
       // elements 4*lane .. 4*lane+3 live in logical chunk lane/2, half lane&1
@@ -1321,7 +1376,7 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
 DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* out, int32_t group,
                           float scale_log2) {
   DecodeParams p = {};
-  p.state_ready = (c.last_layer != layer) ? 1 : 0;
+  p.state_ready = (c.last_full_tiled && c.last_layer != layer) ? 1 : 0;
   p.pool = c.pool;
   p.scales = c.scales;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
@@ -1353,6 +1408,8 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
 bool append_decode_fusable(const Cache& c) {
   return c.decode_kernel == DMS_DECODE_TILED && c.heads <= kMaxHeadsFused && c.ctas_per_sm < 2;
 }
+
+bool tiled_one_cta_per_sm(const Cache& c) { return c.ctas_per_sm < 2; }
 
 // Single-token append of position lengths[layer] fused with the decode (requires
 // append_decode_fusable).
@@ -1427,52 +1484,67 @@ StaticDeviceState g_static_state[kMaxDevices];
 // 32-bit words: [records][kPieceFloats] floats, then counters, then the error word.
 static __device__ __align__(256) float g_decode_scratch[kStaticScratchWords];
 
+namespace {
+
+// One-time set-up per device, with that device current: the device address of the
+// scratch array (the host-side name is only a stand-in), the kernel's shared-memory
+// limit and the SM count.  Returns false on a CUDA error.
+bool static_device_state(StaticDeviceState* out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    cudaGetLastError();
+    return false;
+  }
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  StaticDeviceState& s = g_static_state[dev];
+  if (!s.ready) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_decode_scratch) != cudaSuccess) {
+      cudaGetLastError();
+      return false;
+    }
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        dms::prepare_decode(dms::Cache()) != cudaSuccess) {
+      cudaGetLastError();
+      return false;
+    }
+    s.scratch = static_cast<float*>(ptr);
+    s.num_sms = sms;
+    s.ready = true;
+  }
+  *out = s;
+  return true;
+}
+
+int32_t* static_counters(const StaticDeviceState& st) {
+  return reinterpret_cast<int32_t*>(st.scratch + (size_t)kStaticRecords * dms::kPieceFloats);
+}
+int32_t* static_ctrl(const StaticDeviceState& st) { return static_counters(st) + kStaticCounters; }
+
+}  // namespace
+
 extern "C" dms_status dms_decode_attention_paged_noalloc(
     const void* pool, const int32_t* page_table, const int32_t* counts, int32_t batch,
     int32_t kv_heads, int32_t max_pages, const void* q, void* out, int32_t gqa_group,
     float sm_scale, void* stream) {
   using namespace dms;
-  auto misaligned = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; };
+  auto misaligned = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; };
   if (pool == nullptr || page_table == nullptr || counts == nullptr || q == nullptr ||
-      out == nullptr || misaligned(pool) || misaligned(q) || misaligned(out) || batch < 1 ||
-      kv_heads < 1 || max_pages < 1 || gqa_group < 1 || gqa_group > kMaxGroup ||
-      !(sm_scale == sm_scale))
+      out == nullptr || misaligned(pool, 16) || misaligned(q, 16) || misaligned(out, 16) ||
+      misaligned(page_table, 4) || misaligned(counts, 4) || batch < 1 || kv_heads < 1 ||
+      max_pages < 1 || gqa_group < 1 || gqa_group > kMaxGroup || !(sm_scale == sm_scale))
     return DMS_ERR_INVALID_ARGUMENT;
   const int64_t heads = (int64_t)batch * kv_heads;
   if (heads > kMaxHeads) return DMS_ERR_INVALID_ARGUMENT;
 
-  // One-time set-up per device, with that device current: the device address of
-  // the scratch array (the host-side name is only a stand-in), the kernel's
-  // shared-memory limit and the SM count.
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return DMS_ERR_CUDA;
   StaticDeviceState st;
-  {
-    std::lock_guard<std::mutex> lock(g_static_mu);
-    StaticDeviceState& s = g_static_state[dev];
-    if (!s.ready) {
-      void* ptr = nullptr;
-      if (cudaGetSymbolAddress(&ptr, g_decode_scratch) != cudaSuccess) {
-        cudaGetLastError();
-        return DMS_ERR_CUDA;
-      }
-      int sms = 0;
-      if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-          prepare_decode(Cache()) != cudaSuccess) {
-        cudaGetLastError();
-        return DMS_ERR_CUDA;
-      }
-      s.scratch = static_cast<float*>(ptr);
-      s.num_sms = sms;
-      s.ready = true;
-    }
-    st = s;
-  }
+  if (!static_device_state(&st)) return DMS_ERR_CUDA;
   const int grid = st.num_sms;
   if (grid + heads > kStaticRecords) return DMS_ERR_CAPACITY;  // scratch too small for this batch
 
-  int32_t* counters = reinterpret_cast<int32_t*>(st.scratch + (size_t)kStaticRecords * kPieceFloats);
-  int32_t* ctrl = counters + kStaticCounters;
+  int32_t* counters = static_counters(st);
+  int32_t* ctrl = static_ctrl(st);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // The array keeps whatever the previous call left: the arrival counters and the
   // error word must start at zero.
@@ -1497,4 +1569,37 @@ extern "C" dms_status dms_decode_attention_paged_noalloc(
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)kHeadDim);
   p.scale_log2 = scale * 1.4426950408889634f;
   return launch_tiled(p, grid, 1, s, false, false) == cudaSuccess ? DMS_OK : DMS_ERR_CUDA;
+}
+
+extern "C" dms_status dms_decode_noalloc_device_error(void* stream, dms_status* out) {
+  if (out == nullptr) return DMS_ERR_INVALID_ARGUMENT;
+  StaticDeviceState st;
+  if (!static_device_state(&st)) return DMS_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t word = 0;  // the error word, read into host (stack) memory: nothing is allocated
+  if (cudaMemcpyAsync(&word, static_ctrl(st) + dms::kCtrlError, sizeof(word),
+                      cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return DMS_ERR_CUDA;
+  }
+  *out = static_cast<dms_status>(word);
+  return DMS_OK;
+}
+
+extern "C" dms_status dms_selftest_noalloc_timeout(int64_t limit_ns, void* stream) {
+  if (limit_ns < 1000 || limit_ns > 10000000000LL) return DMS_ERR_INVALID_ARGUMENT;
+  StaticDeviceState st;
+  if (!static_device_state(&st)) return DMS_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t* ctrl = static_ctrl(st);
+  // A barrier that nothing completes: the bounded wait gives up after limit_ns and
+  // records DMS_ERR_TIMEOUT in the error word the allocation-free decode uses.
+  if (cudaMemsetAsync(ctrl, 0, sizeof(int32_t) * (size_t)kStaticCtrl, s) != cudaSuccess ||
+      dms::launch_bounded_wait_probe(0, limit_ns, ctrl, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    return DMS_ERR_CUDA;
+  }
+  return DMS_OK;
 }

@@ -103,8 +103,11 @@ struct Cache {
   int64_t* lengths = nullptr;  // host: tokens appended per layer
   int64_t peak_pages = 0;      // host: largest pages_in_use observed
   // host: layer of the last kernel launched on this cache (-1: none since creation or
-  // reset).  A launch for another layer cannot depend on that kernel's cache writes.
+  // reset), and whether it was a tiled decode with one CTA per SM.  After such a launch
+  // for another layer, a tiled decode may read its layer's state before its dependency
+  // wait (DecodeParams::state_ready in dms_decode.cu).
   int32_t last_layer = -1;
+  bool last_full_tiled = false;
 
   // Count buffer of `layer` for a layer length of parity `parity`.
   int32_t* counts_at(int32_t layer, int64_t parity) const {
@@ -174,6 +177,7 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
 cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, void* out,
                                  int32_t group, float scale, bool zero_first, cudaStream_t stream);
 bool append_decode_fusable(const Cache& c);
+bool tiled_one_cta_per_sm(const Cache& c);  // tiled decode launches use one CTA per SM
 cudaError_t launch_bounded_wait_probe(int arrive, int64_t limit_ns, int32_t* dev_status,
                                       cudaStream_t stream);
 cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,

@@ -30,6 +30,12 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
+// `count` arrivals at once (one thread standing in for `count` expected arrivals).
+__device__ __forceinline__ void mbar_arrive_cnt(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+               : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t done;
   asm volatile(
@@ -186,12 +192,6 @@ __device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t x) {
   return pack_f16x2(__uint_as_float(x << 16), __uint_as_float(x & 0xffff0000u));
 }
 
-__device__ __forceinline__ uint32_t hmul2_u32(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-
 // Transpose of an 8x8 b16 matrix held one 32-bit fragment per thread.
 __device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
   uint32_t y;
@@ -207,6 +207,35 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // Four consecutive bf16 outputs (round to nearest even) with one 8-byte store.
 __device__ __forceinline__ void store_bf16x4(__nv_bfloat16* dst, float a, float b, float c, float d) {
   *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(a, b), pack_bf16x2(c, d));
+}
+
+// Acquire / release accesses of a 32-bit flag at GPU scope.
+__device__ __forceinline__ uint32_t ld_acquire_gpu_u32(const uint32_t* addr) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_gpu_u32(uint32_t* addr, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(addr), "r"(v) : "memory");
+}
+
+// Order this thread's generic-proxy accesses of global (resp. shared) memory with its
+// later async-proxy (bulk copy) accesses of it.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Named barriers (0 is __syncthreads): wait for `count` threads, or only count this one.
+template <int kId>
+__device__ __forceinline__ void named_bar_sync(int count) {
+  asm volatile("bar.sync %0, %1;" ::"n"(kId), "r"(count) : "memory");
+}
+template <int kId>
+__device__ __forceinline__ void named_bar_arrive(int count) {
+  asm volatile("bar.arrive %0, %1;" ::"n"(kId), "r"(count) : "memory");
 }
 
 // Relaxed GPU-scope load (no ordering); paired with fence.acq_rel.gpu once its
