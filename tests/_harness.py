@@ -1,7 +1,7 @@
 """Drives the CUDA path through the C ABI and checks it against the fp64 oracle.
 
-The full appended history (K, V, logits) of the layer under test is kept on the
-device so that any (sequence, KV head) can be handed to the oracle at any step.
+The full appended history (K, V, logits) of every layer under test is kept on the
+device so that any (layer, sequence, KV head) can be handed to the oracle at any step.
 Tolerances: retained sets bit-exact; attention outputs max-abs <= 2e-2 and
 mean-abs <= 2e-3 against the fp64 oracle on the same bf16 inputs.  An fp8 cache
 (kv_format=DMS_KV_FP8_E4M3) is checked against the oracle's attention over its own
@@ -21,97 +21,135 @@ MEAN_ABS = 2e-3
 
 
 class Run:
+    """A cache of `layers` layers driven through the C ABI, with every layer's appended history
+    (K, V, decision logits) kept on the device; layer l draws the inputs of workload layer
+    `layer + l`.  Steps append the new token and decode every layer in order, as the bench does."""
+
+    # Largest K or V tensor generated at once (elements); bigger prompts are appended in chunks.
+    CHUNK_ELEMS = 1 << 28
+
     def __init__(self, wl: workloads.Workload, device="cuda", layer: int = 0,
-                 capacity: int | None = None, fused: bool = False, **cache_kw):
+                 capacity: int | None = None, fused: bool = False, layers: int = 1, **cache_kw):
         self.wl, self.layer, self.dev = wl, layer, torch.device(device)
         self.fused = fused  # decode steps through dms_append_and_decode
         self.fp8 = cache_kw.get("kv_format", dms.DMS_KV_BF16) == dms.DMS_KV_FP8_E4M3
         self.T = capacity or wl.context
+        self.n_layers = layers
         B, H, D = wl.batch, wl.kv_heads, wl.head_dim
-        self.cache = dms.DmsCache(layers=1, kv_heads=H, window=wl.window, capacity=self.T,
+        self.cache = dms.DmsCache(layers=layers, kv_heads=H, window=wl.window, capacity=self.T,
                                   batch=B, **cache_kw)
-        self.K = torch.zeros((B, self.T, H, D), dtype=torch.bfloat16, device=self.dev)
-        self.V = torch.zeros_like(self.K)
-        self.L = torch.zeros((B, self.T, H), dtype=torch.bfloat16, device=self.dev)
-        self.t = 0
+        self.Ks = [torch.zeros((B, self.T, H, D), dtype=torch.bfloat16, device=self.dev)
+                   for _ in range(layers)]
+        self.Vs = [torch.zeros_like(k) for k in self.Ks]
+        self.Ls = [torch.zeros((B, self.T, H), dtype=torch.bfloat16, device=self.dev)
+                   for _ in range(layers)]
+        self.ts = [0] * layers
         self.errs = []
+
+    # layer 0's history (the single-layer view most tests use)
+    K = property(lambda self: self.Ks[0])
+    V = property(lambda self: self.Vs[0])
+    L = property(lambda self: self.Ls[0])
+
+    @property
+    def t(self):
+        return self.ts[0]
+
+    @t.setter
+    def t(self, value):
+        self.ts[0] = value
 
     def close(self):
         self.cache.close()
 
-    def append(self, k, v, lg):
-        n = k.shape[1]
-        self.cache.append_and_evict(0, k, v, lg)
-        self.K[:, self.t:self.t + n] = k
-        self.V[:, self.t:self.t + n] = v
-        self.L[:, self.t:self.t + n] = lg
-        self.t += n
+    def record(self, k, v, lg, layer=0):
+        n, t = k.shape[1], self.ts[layer]
+        self.Ks[layer][:, t:t + n] = k
+        self.Vs[layer][:, t:t + n] = v
+        self.Ls[layer][:, t:t + n] = lg
+        self.ts[layer] = t + n
+
+    def append(self, k, v, lg, layer=0):
+        self.cache.append_and_evict(layer, k, v, lg)
+        self.record(k, v, lg, layer)
 
     def prefill(self):
-        for i, (n, shared) in enumerate(self.wl.prefill):
-            if shared:
-                k, v, lg = workloads.gen_kv(self.wl, self.layer, f"prefill{i}", n, self.dev, batch=1)
-                B = self.wl.batch
-                k, v = k.expand(B, -1, -1, -1).contiguous(), v.expand(B, -1, -1, -1).contiguous()
-                lg = lg.expand(B, -1, -1).contiguous()
-            else:
-                k, v, lg = workloads.gen_kv(self.wl, self.layer, f"prefill{i}", n, self.dev)
-            self.append(k, v, lg)
+        wl = self.wl
+        per_token = wl.batch * wl.kv_heads * wl.head_dim
+        chunk = max(64, self.CHUNK_ELEMS // per_token)
+        for layer in range(self.n_layers):
+            for i, (n, shared) in enumerate(wl.prefill):
+                for c0 in range(0, n, chunk):
+                    nc = min(chunk, n - c0)
+                    tag = f"prefill{i}" + (f"c{c0}" if n > chunk else "")
+                    if shared:
+                        k, v, lg = workloads.gen_kv(wl, self.layer + layer, tag, nc, self.dev,
+                                                    batch=1)
+                        B = wl.batch
+                        k = k.expand(B, -1, -1, -1).contiguous()
+                        v = v.expand(B, -1, -1, -1).contiguous()
+                        lg = lg.expand(B, -1, -1).contiguous()
+                    else:
+                        k, v, lg = workloads.gen_kv(wl, self.layer + layer, tag, nc, self.dev)
+                    self.append(k, v, lg, layer)
+                    del k, v, lg
 
-    def record(self, k, v, lg):
-        n = k.shape[1]
-        self.K[:, self.t:self.t + n] = k
-        self.V[:, self.t:self.t + n] = v
-        self.L[:, self.t:self.t + n] = lg
-        self.t += n
+    def step_layer(self, s: int, layer: int = 0, p_override=None):
+        k, v, lg = workloads.gen_kv(self.wl, self.layer + layer, f"decode{s}", 1, self.dev,
+                                    p_override=p_override)
+        q = workloads.gen_q(self.wl, self.layer + layer, f"decode{s}", self.dev)
+        if self.fused:
+            out = self.cache.append_and_decode(layer, k, v, lg, q, gqa_group=self.wl.gqa_group)
+            self.record(k, v, lg, layer)
+        else:
+            self.append(k, v, lg, layer)
+            out = self.cache.decode_attention(layer, q, gqa_group=self.wl.gqa_group)
+        return q, out
 
     def step(self, s: int, p_override=None):
-        k, v, lg = workloads.gen_kv(self.wl, self.layer, f"decode{s}", 1, self.dev,
-                                    p_override=p_override)
-        q = workloads.gen_q(self.wl, self.layer, f"decode{s}", self.dev)
-        if self.fused:
-            out = self.cache.append_and_decode(0, k, v, lg, q, gqa_group=self.wl.gqa_group)
-            self.record(k, v, lg)
-        else:
-            self.append(k, v, lg)
-            out = self.cache.decode_attention(0, q, gqa_group=self.wl.gqa_group)
-        return q, out
+        """Decode step s of layer 0 (single-layer runs)."""
+        return self.step_layer(s, 0, p_override)
+
+    def step_all(self, s: int):
+        """Decode step s of every layer, in layer order; [(q, out)] per layer."""
+        return [self.step_layer(s, layer) for layer in range(self.n_layers)]
 
     # ---- checks
 
-    def logits_host(self) -> np.ndarray:
-        return workloads.bf16_bits(self.L[:, :self.t])
+    def logits_host(self, layer=0) -> np.ndarray:
+        return workloads.bf16_bits(self.Ls[layer][:, :self.ts[layer]])
 
-    def check_retained(self, heads=None):
-        """Retained positions of every (b, h) equal the oracle's R_j, bit for bit."""
-        j = self.t - 1
-        pos = self.cache.export_positions(0)
-        L = self.logits_host()
+    def check_retained(self, heads=None, layer=0):
+        """Retained positions of every (b, h) of `layer` equal the oracle's R_j, bit for bit."""
+        j = self.ts[layer] - 1
+        pos = self.cache.export_positions(layer)
+        L = self.logits_host(layer)
         B, H = self.wl.batch, self.wl.kv_heads
         heads = heads if heads is not None else [(b, h) for b in range(B) for h in range(H)]
         st = self.cache.stats(with_counts=True)
         assert st["device_error"] == 0, st
         for b, h in heads:
             row = pos[b, h]
-            n = int(st["counts"][0, b, h])
+            n = int(st["counts"][layer, b, h])
             assert np.all(row[:n] >= 0) and np.all(row[n:] == -1), (b, h)
             have = np.sort(row[:n])
             want = oracle.retained(L[b, :, h], j, self.wl.window)
-            assert np.array_equal(have, want), (b, h, len(have), len(want))
+            assert np.array_equal(have, want), (layer, b, h, len(have), len(want))
         return st
 
-    def check_outputs(self, q, out, pairs=None, record=True):
-        """Outputs of the given (b, h) KV heads (all G query heads each) vs the oracle."""
-        j = self.t - 1
+    def check_outputs(self, q, out, pairs=None, record=True, layer=0):
+        """Outputs of the given (b, h) KV heads (all G query heads each) of `layer` vs the
+        oracle."""
+        j = self.ts[layer] - 1
         G, B, H = self.wl.gqa_group, self.wl.batch, self.wl.kv_heads
         pairs = pairs if pairs is not None else [(b, h) for b in range(B) for h in range(H)]
         Q = workloads.bf16_bits(q)
         got = out.float().cpu().numpy()
         errs = []
         for b, h in pairs:
-            k = workloads.bf16_bits(self.K[b, :j + 1, h])
-            v = workloads.bf16_bits(self.V[b, :j + 1, h])
-            lg = workloads.bf16_bits(self.L[b, :j + 1, h])
+            k = workloads.bf16_bits(self.Ks[layer][b, :j + 1, h])
+            v = workloads.bf16_bits(self.Vs[layer][b, :j + 1, h])
+            lg = workloads.bf16_bits(self.Ls[layer][b, :j + 1, h])
             if self.fp8:
                 kc, ks = oracle.quantize_rows_e4m3(k)
                 vc, vs = oracle.quantize_rows_e4m3(v)

@@ -58,3 +58,23 @@ def test_two_gloo_ranks():
     assert v0 == v1 == pytest.approx(4000.0 / 10e-3)  # all units / slowest time
     assert tag0 != tag1                         # independent replicas
     assert ref1 is None                         # the reference arm runs on rank 0 only
+
+
+def test_gpus_flag_must_match_the_launched_ranks():
+    """--gpus N without N launched ranks is an error, not a silent one-GPU run."""
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    import bench
+    bench.check_world(1, 1)
+    bench.check_world(2, 2)
+    with pytest.raises(SystemExit):
+        bench.check_world(8, 1)
+    env = {k: v for k, v in os.environ.items() if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK")}
+    run = subprocess.run([sys.executable, "bench.py", "--gpus", "2", "--impl", "reference",
+                          "--steps", "1", "--warmup", "1"], cwd=root, env=env,
+                         capture_output=True, text=True, timeout=300)
+    assert run.returncode != 0
+    assert "--gpus 2 but 1 rank(s)" in run.stderr
+    assert not [ln for ln in run.stdout.splitlines() if ln.startswith("{")]
