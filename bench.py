@@ -3,8 +3,10 @@
 One step = one decode step of the whole model: for every layer, the fused
 append + delayed eviction of the new token (all sequences, all KV heads) and the
 split-K decode attention over the retained sets (GQA).  The default workload is
-the Qwen-R1-7B shape: 28 layers, 28 query / 4 KV heads, head_dim 128, batch 64,
-context 8192 (prefill 7936, then decode), window 256, P(evict) = 0.75.
+the 8x-compressed Qwen-R1-32B shape: 64 layers, 40 query / 8 KV heads, head_dim
+128, batch 8, context 32768 (prefill 32512, then decode), window 256,
+P(evict) = 0.875, 1 % of the key channels scaled x8.  The Qwen-R1-7B shape (4x)
+and the others are selected with --workload.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
@@ -50,7 +52,7 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default=workloads.QWEN7B_B64_8K.name)
+    ap.add_argument("--workload", default=workloads.QWEN32B_B8_32K.name)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--dense", action="store_true", help="no evictions (CR 1) with the same shape")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
@@ -190,11 +192,22 @@ class Clocks:
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
 
 
+def check_world(gpus, world):
+    """--gpus N must equal the number of ranks the launcher started (torchrun's WORLD_SIZE,
+    1 without a launcher): the bench never spreads itself over GPUs it was not given."""
+    if gpus != world:
+        raise SystemExit(
+            f"bench.py: --gpus {gpus} but {world} rank(s) were launched (WORLD_SIZE); for N > 1 "
+            f"run: python -m torch.distributed.run --nnodes=1 --nproc-per-node {gpus} "
+            f"--master-addr 127.0.0.1 --master-port <port> bench.py --gpus {gpus} ...")
+
+
 def dist_setup(args):
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    check_world(getattr(args, "gpus", world), world)
     pg = None
     if world > 1:
         import torch.distributed as dist
@@ -244,6 +257,39 @@ def replica_tag(rank):
 
 
 # ============================================================================ ours
+
+
+def expected_retained_per_layer(wl):
+    """Retained tokens of one layer at the start of decoding, in expectation:
+    B * sum_h (T - p_h (T - w - 1)) (Sec. 3.1 delayed eviction; layer 0's p_h)."""
+    T = wl.prefill_tokens
+    p = workloads.head_evict_prob(wl, 0)
+    evictable = max(0, T - wl.window - 1)
+    return float(wl.batch * np.sum(T - p * evictable))
+
+
+def decode_config(args, wl, world, warmup, steps):
+    """The `config` object of a decode line; the GPU arm and the reference arm print the same."""
+    D = wl.head_dim
+    bytes_per_unit = 2 * D + 8 if args.kv_fp8 else workloads.kv_bytes_per_token_head(D)
+    per_layer_mb = expected_retained_per_layer(wl) * bytes_per_unit / 1e6
+    if per_layer_mb * wl.layers > 2 * 129.0:
+        l2 = (f"no flush: ~{per_layer_mb:.0f} MB of retained KV per layer x {wl.layers} layers "
+              "rotate, larger than the 129 MB L2")
+    else:
+        l2 = (f"not flushed: ~{per_layer_mb:.1f} MB of retained KV per layer x {wl.layers} "
+              "layer(s) stays in the 129 MB L2 (a latency-bound shape)")
+    return {"workload": wl.name, "batch_per_gpu": wl.batch, "layers": wl.layers,
+            "q_heads": wl.q_heads,
+            "kv_format": "fp8_e4m3 (per-row fp32 scales)" if args.kv_fp8 else "bf16",
+            "kv_heads": wl.kv_heads, "head_dim": D, "window": wl.window,
+            "prefill": wl.prefill_tokens,
+            "timed_positions": [wl.prefill_tokens + warmup, wl.prefill_tokens + warmup + steps - 1],
+            "p_evict": (None if wl.ragged_beta else wl.p_evict),
+            "ragged_beta": wl.ragged_beta,
+            "shared_prefix_pages": bool(getattr(args, "shared_prefix", False) and
+                                        any(sh for _, sh in wl.prefill)),
+            "l2": l2, "parallelism": f"replicas x{world}"}
 
 
 def run_ours(args, wl, world, rank, local, pg):
@@ -600,17 +646,7 @@ def run_ours(args, wl, world, rank, local, pg):
         "dtype": "fp8 E4M3 K/V codes, f16 MMA, fp32 accumulate" if args.kv_fp8 else "bf16",
         "data": "synthetic",
         "impl": "ours",
-        "config": {"workload": wl.name, "batch_per_gpu": B, "layers": L, "q_heads": Hq,
-                   "kv_format": "fp8_e4m3 (per-row fp32 scales)" if args.kv_fp8 else "bf16",
-                   "kv_heads": H, "head_dim": D, "window": wl.window, "prefill": wl.prefill_tokens,
-                   "timed_positions": [wl.prefill_tokens + W_, wl.prefill_tokens + W_ + K_ - 1],
-                   "p_evict": (None if wl.ragged_beta else wl.p_evict),
-                   "ragged_beta": wl.ragged_beta,
-                   "shared_prefix_pages": bool(args.shared_prefix and any(sh for _, sh in wl.prefill)),
-                   "l2": "no flush: per-layer retained KV "
-                         f"{units_per_launch * bytes_per_unit / 1e6:.0f} MB x {L} layers rotate, "
-                         "larger than the 129 MB L2",
-                   "parallelism": f"replicas x{world}"},
+        "config": decode_config(args, wl, world, W_, K_),
         "step_mode": ("separate append + decode launches" if args.separate else
                       "fused single-token append + decode, one launch per layer") +
                      ("; decisions from element 0 of each group's first query head (App. B)"
@@ -625,7 +661,9 @@ def run_ours(args, wl, world, rank, local, pg):
                                ("" if args.separate else " (append fused)"),
                      "bound": "hbm", "achieved": achieved_gbs,
                      "peak": peak, "unit": "GB/s", "frac": achieved_gbs / peak,
-                     "peak_kind": f"{peak_kind} copy bandwidth",
+                     "peak_kind": f"{peak_kind} copy bandwidth (read + write; the kernel only "
+                                  "reads, so a fraction a little above 1 is possible)",
+                     "frac_of_nominal_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
                      "traffic": traffic,
                      "algorithmic_bytes_per_launch": units_per_launch * bytes_per_unit,
                      "duration": duration_source},
@@ -682,7 +720,11 @@ def run_reference(args, wl, world, rank):
             j = len(ll) - 1
             qq = workloads.bf16_bits(q[0, h * G:(h + 1) * G])
             t1 = time.perf_counter()
-            oracle.decode(qq, kk, vv, ll, j, wl.window)
+            if getattr(args, "kv_fp8", False):  # the oracle quantises the history itself
+                oracle.decode_fp8(qq, *oracle.quantize_rows_e4m3(kk),
+                                  *oracle.quantize_rows_e4m3(vv), ll, j, wl.window)
+            else:
+                oracle.decode(qq, kk, vv, ll, j, wl.window)
             per_step_s.append(time.perf_counter() - t1)
             tok += len(oracle.retained(ll, j, wl.window))
         per_step_tok.append(tok)
@@ -693,8 +735,7 @@ def run_reference(args, wl, world, rank):
             "warmup": args.warmup, "ms_per_step": 1e3 * timed_s / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.name, "batch_per_gpu": B, "layers": wl.layers,
-                       "q_heads": wl.q_heads, "kv_heads": H, "head_dim": D, "window": wl.window},
+            "config": decode_config(args, wl, world, args.warmup, args.steps),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"{n_sample} sampled (layer 0, seq, KV head) groups per step, "
                                        f"{G} query heads each, fp64 single-threaded"},
