@@ -69,8 +69,16 @@ enum {
 
 /* Decode kernels selectable through dms_options.decode_kernel. */
 enum {
-  DMS_DECODE_TILED = 0,  /* default: TMA-staged, tensor-core, page-balanced split-K */
-  DMS_DECODE_SIMPLE = 1  /* one CTA per KV head, CUDA cores; a cross-check path     */
+  DMS_DECODE_TILED = 0,  /* default: TMA-staged tensor-core kernels.  When every
+                            (sequence, KV head) can have a resident thread-block
+                            cluster of 16 (else 8) CTAs at once (few heads: a batch
+                            of one or two), bf16 pages, G <= 8 and the default
+                            ctas_per_sm / min_pages_per_cta, each head's pages are
+                            split over its own cluster and merged in distributed
+                            shared memory; otherwise as DMS_DECODE_SPLIT           */
+  DMS_DECODE_SIMPLE = 1, /* one CTA per KV head, CUDA cores; a cross-check path     */
+  DMS_DECODE_SPLIT = 2   /* the tiled kernel with the flat, page-balanced split-K of
+                            all heads' pages over all SMs, for every batch          */
 };
 
 /*
@@ -98,12 +106,12 @@ typedef struct dms_options {
                             shared by all layers and heads; 0 = the dense worst
                             case, layers * batch * kv_heads * ceil(capacity / 64)
                             pages                                                  */
-  int32_t decode_kernel; /* DMS_DECODE_TILED (0) or DMS_DECODE_SIMPLE (1)           */
+  int32_t decode_kernel; /* DMS_DECODE_TILED (0), _SIMPLE (1) or _SPLIT (2)          */
   int32_t ctas_per_sm;   /* split-K CTAs per SM for the tiled kernel; 0 = 1         */
   int32_t min_pages_per_cta; /* lower bound on pages per split-K CTA; 0 = 2         */
   int32_t eviction_policy;   /* DMS_EVICT_DELAYED (0) or DMS_EVICT_IMMEDIATE (1)    */
-  int32_t kv_format;     /* DMS_KV_BF16 (0) or DMS_KV_FP8_E4M3 (1); fp8 requires the
-                            tiled decode kernel                                     */
+  int32_t kv_format;     /* DMS_KV_BF16 (0) or DMS_KV_FP8_E4M3 (1); fp8 requires a
+                            tiled decode kernel (TILED or SPLIT)                    */
   int32_t reserved[3];   /* must be zero                                            */
 } dms_options;
 

@@ -22,7 +22,8 @@ import numpy as np
 from . import _native
 from ._native import (DMS_EVICT_DELAYED, DMS_EVICT_IMMEDIATE,  # noqa: F401
                       DMS_PREFILL_MMA_SYNC, DMS_PREFILL_TCGEN05,  # noqa: F401
-                      DMS_DECODE_SIMPLE, DMS_DECODE_TILED, DMS_ERR_CAPACITY,  # noqa: F401
+                      DMS_DECODE_SIMPLE, DMS_DECODE_SPLIT, DMS_DECODE_TILED,  # noqa: F401
+                      DMS_ERR_CAPACITY,  # noqa: F401
                       DMS_KV_BF16, DMS_KV_FP8_E4M3,  # noqa: F401
                       DMS_ERR_INVALID_ARGUMENT, DMS_ERR_STATE, DMS_ERR_TIMEOUT, DMS_OK,
                       DmsLibraryError,

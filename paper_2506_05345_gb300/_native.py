@@ -25,6 +25,7 @@ DMS_PREFILL_TCGEN05 = 0
 DMS_PREFILL_MMA_SYNC = 1
 DMS_DECODE_TILED = 0
 DMS_DECODE_SIMPLE = 1
+DMS_DECODE_SPLIT = 2
 DMS_KV_BF16 = 0
 DMS_KV_FP8_E4M3 = 1
 

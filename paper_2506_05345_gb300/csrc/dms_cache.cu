@@ -32,6 +32,8 @@ void free_device(Cache& c) {
   cudaFree(c.freed);
   cudaFree(c.pieces);
   cudaFree(c.piece_counters);
+  cudaFree(c.head_flags);
+  c.head_flags = nullptr;
   c.pool = nullptr;
   c.pos = c.page_table = c.counts = c.ctrl = c.freed = c.piece_counters = nullptr;
   c.rings = nullptr;
@@ -41,6 +43,10 @@ void free_device(Cache& c) {
 void free_host(Cache& c) {
   free(c.lengths);
   c.lengths = nullptr;
+  free(c.flag_seq);
+  c.flag_seq = nullptr;
+  free(c.flag_valid);
+  c.flag_valid = nullptr;
 }
 
 template <typename T>
@@ -73,12 +79,12 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
       capacity < 1 || capacity > dms::kMaxCapacity || opt->batch < 1)
     return DMS_ERR_INVALID_ARGUMENT;
   if (opt->page_tokens != 0 && opt->page_tokens != dms::kPageTokens) return DMS_ERR_INVALID_ARGUMENT;
-  if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SIMPLE ||
+  if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SPLIT ||
       opt->ctas_per_sm < 0 || opt->ctas_per_sm > dms::kMaxCtasPerSm || opt->min_pages_per_cta < 0 ||
       opt->eviction_policy < DMS_EVICT_DELAYED || opt->eviction_policy > DMS_EVICT_IMMEDIATE ||
       opt->kv_format < DMS_KV_BF16 || opt->kv_format > DMS_KV_FP8_E4M3)
     return DMS_ERR_INVALID_ARGUMENT;
-  if (opt->kv_format == DMS_KV_FP8_E4M3 && opt->decode_kernel != DMS_DECODE_TILED)
+  if (opt->kv_format == DMS_KV_FP8_E4M3 && opt->decode_kernel == DMS_DECODE_SIMPLE)
     return DMS_ERR_INVALID_ARGUMENT;  // only the tiled kernel reads fp8 pages
   for (int i = 0; i < 3; ++i)
     if (opt->reserved[i] != 0) return DMS_ERR_INVALID_ARGUMENT;
@@ -118,7 +124,10 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   }
   c.piece_capacity = (int64_t)c.num_sms * dms::kMaxCtasPerSm + heads;
   c.lengths = static_cast<int64_t*>(calloc((size_t)layers, sizeof(int64_t)));
-  if (c.lengths == nullptr) {
+  c.flag_seq = static_cast<uint32_t*>(calloc((size_t)layers, sizeof(uint32_t)));
+  c.flag_valid = static_cast<uint8_t*>(calloc((size_t)layers, sizeof(uint8_t)));
+  if (c.lengths == nullptr || c.flag_seq == nullptr || c.flag_valid == nullptr) {
+    free_host(c);
     delete h;
     return DMS_ERR_OUT_OF_MEMORY;
   }
@@ -135,10 +144,13 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
   if (e == cudaSuccess) e = alloc(&c.freed, (size_t)heads * c.ring_len);
   if (e == cudaSuccess) e = alloc(&c.pieces, (size_t)c.piece_capacity * dms::kPieceFloats);
   if (e == cudaSuccess) e = alloc(&c.piece_counters, (size_t)heads);
+  if (e == cudaSuccess) e = alloc(&c.head_flags, (size_t)layers * heads);
+  if (e == cudaSuccess) e = cudaMemset(c.head_flags, 0, sizeof(uint32_t) * (size_t)layers * heads);
   if (e == cudaSuccess) e = cudaMemset(c.counts, 0, sizeof(int32_t) * (size_t)layers * 2 * heads);
   if (e == cudaSuccess) e = cudaMemset(c.ctrl, 0, sizeof(int32_t) * dms::kCtrlWords);
   if (e == cudaSuccess) e = cudaMemset(c.piece_counters, 0, sizeof(int32_t) * (size_t)heads);
   if (e == cudaSuccess) e = dms::prepare_decode(c);
+  if (e == cudaSuccess) e = dms::prepare_cluster_decode(c);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
     const bool oom = (e == cudaErrorMemoryAllocation);
@@ -177,7 +189,10 @@ dms_status dms_cache_reset(dms_cache* h, void* stream) {
       cudaMemsetAsync(c.ctrl, 0, sizeof(int32_t) * dms::kCtrlWords, st) != cudaSuccess ||
       cudaMemsetAsync(c.piece_counters, 0, sizeof(int32_t) * (size_t)c.heads, st) != cudaSuccess)
     return DMS_ERR_CUDA;
-  for (int l = 0; l < c.layers; ++l) c.lengths[l] = 0;
+  for (int l = 0; l < c.layers; ++l) {
+    c.lengths[l] = 0;
+    c.flag_valid[l] = 0;
+  }
   c.last_layer = -1;
   c.last_full_tiled = false;
   return DMS_OK;
@@ -201,6 +216,7 @@ dms_status append_impl(dms_cache* h, int32_t layer, const void* k, const void* v
   const int64_t t0 = c.lengths[layer];
   if (t0 + n_tokens > c.capacity) return DMS_ERR_CAPACITY;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  c.flag_valid[layer] = 0;  // this append publishes no completion flags
   const cudaError_t e =
       (n_tokens == 1)
           ? dms::launch_append_one(c, layer, k, v, logit, logit_stride, t0, st)
@@ -229,7 +245,8 @@ dms_status decode_impl(dms_cache* h, int32_t layer, const void* q, void* out, in
                                  zero_first, st);
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.last_layer = layer;
-  c.last_full_tiled = c.decode_kernel == DMS_DECODE_TILED && dms::tiled_one_cta_per_sm(c);
+  c.last_full_tiled = c.decode_kernel != DMS_DECODE_SIMPLE && dms::tiled_one_cta_per_sm(c) &&
+                      dms::decode_cluster_size(c, gqa_group) == 0;
   return DMS_OK;
 }
 
@@ -251,13 +268,17 @@ dms_status append_decode_impl(dms_cache* h, int32_t layer, const void* k, const 
     return decode_impl(h, layer, q, out, gqa_group, sm_scale, zero_first, stream);
   }
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
+  const bool cluster = dms::decode_cluster_size(c, gqa_group) > 0;
   const cudaError_t e = dms::launch_append_decode(
       c, layer, k, v, logit, logit_stride, q, out, gqa_group, scale * 1.4426950408889634f,
       zero_first, static_cast<cudaStream_t>(stream));
+  // A cluster launch publishes the next sequence number in the layer's completion flags.
+  c.flag_valid[layer] = (e == cudaSuccess && cluster) ? 1 : 0;
   if (e != cudaSuccess) return DMS_ERR_CUDA;
+  if (cluster) c.flag_seq[layer] = dms::next_flag_seq(c.flag_seq[layer]);
   c.lengths[layer] = t0 + 1;
   c.last_layer = layer;
-  c.last_full_tiled = true;
+  c.last_full_tiled = !cluster;
   return DMS_OK;
 }
 
@@ -292,6 +313,7 @@ dms_status dms_append_shared_prefix(dms_cache* h, int32_t layer, const void* k, 
     return DMS_ERR_INVALID_ARGUMENT;
   if (c.lengths[layer] != 0) return DMS_ERR_STATE;  // a shared prompt starts the sequences
   if (n_tokens > c.capacity) return DMS_ERR_CAPACITY;
+  c.flag_valid[layer] = 0;
   const cudaError_t e = dms::launch_append_shared_prefix(c, layer, k, v, decision_logit, n_tokens,
                                                          static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return DMS_ERR_CUDA;

@@ -118,6 +118,11 @@ struct DecodeParams {
   // launch can be resident: whatever last wrote this layer (two or more launches back) has
   // completed.
   int32_t state_ready;
+  // Cluster kernel: this layer's per-head completion flags, the number the launch that
+  // last wrote the layer's state published (0: none; wait for the dependency first) and
+  // the number this launch publishes (fused; 0: none).
+  uint32_t* head_flags;
+  uint32_t flag_expect, flag_publish;
   // Nonzero: attend with element 0 of every group's first query head taken as 0 (that
   // element carries the decision logit, App. B).
   int32_t zero_first;
@@ -184,7 +189,7 @@ size_t tiled_smem_bytes(int heads, int stages) {
   using PL = Plan<NT>;
   return (size_t)stages * stage_bytes(kFused, kFp8) +
          (size_t)PL::kSlots * (PL::kSlotOFloats + PL::kSlotMLFloats) * 4 +
-         (size_t)(2 * stages + 2 * PL::kSlots + 1) * sizeof(uint64_t) + 64 +
+         (size_t)(2 * stages + 2 * PL::kSlots) * sizeof(uint64_t) + 64 +
          (size_t)((kFused ? 3 : 2) * heads + 1) * sizeof(int32_t);
 }
 
@@ -242,8 +247,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   uint64_t* mfull_bar = empty_bar + kStages;
   uint64_t* mempty_bar = mfull_bar + PL::kSlots;
   // s_misc: [0] abort, [2..7] warp sums, [8..8+kStages) page id staged in each stage
-  uint64_t* rec_bar = mempty_bar + PL::kSlots;  // records of the CTA's last head (prefetch)
-  int* s_misc = reinterpret_cast<int*>(rec_bar + 1);
+  int* s_misc = reinterpret_cast<int*>(mempty_bar + PL::kSlots);
   int32_t* s_cnt = s_misc + 16;                                   // [heads] n_h (after the append)
   int32_t* s_pstart = s_cnt + p.heads;                            // [heads + 1]
   // fused: new token's slot | fresh << 30 per head
@@ -265,7 +269,6 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       mbar_init(&mfull_bar[s], kConsumerWarps);
       mbar_init(&mempty_bar[s], 1);
     }
-    mbar_init(rec_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   // While the previous kernel finishes, warm L2 with the small tables the prologue
@@ -707,11 +710,6 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   // every other CTA of a split head has already arrived, this CTA merges their
   // records directly, without publishing its own.
   int arrivals_seen = -1;
-  // Thread 0, when every other CTA of the last segment's split head has arrived by its
-  // last page: their records are copied (bulk) into the idle merge slot while that page
-  // is computed, so the merge that ends the CTA waits for no round trip.
-  int pre_rec = 0;
-  const uint32_t rec_bytes = (uint32_t)(2 * kMaxGroup + G * kHeadDim) * 4u;  // m, l, G rows of O
 
   for (int it = 0; it < niters; ++it) {
     walk.enter(it);
@@ -722,31 +720,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
     const bool seg_end = walk.seg_end(it, niters);
     uint8_t* st = stages + s * kStageBytes;
     if (it == niters - 1 && tid == 0 &&
-        split.cta_of(s_pstart[walk.h]) != split.cta_of(s_pstart[walk.h + 1] - 1)) {
+        split.cta_of(s_pstart[walk.h]) != split.cta_of(s_pstart[walk.h + 1] - 1))
       arrivals_seen = ld_relaxed_gpu(p.piece_counters + walk.h);
-      if constexpr (PL::kSlots == 2) {
-        const int k_lo = split.cta_of(s_pstart[walk.h]), k_hi = split.cta_of(s_pstart[walk.h + 1] - 1);
-        const int others = k_hi - k_lo;
-        if (arrivals_seen == others && (uint32_t)others * rec_bytes <= (uint32_t)PL::kSlotOFloats * 4u) {
-          asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
-          // the other merge slot is idle once the epilogue has finished the previous segment
-          const int other = (q + 1) % PL::kSlots;
-          if (q >= 1) mbar_wait(&mempty_bar[other], ((q - 1) / PL::kSlots) & 1, abort_flag, p.ctrl);
-          fence_proxy_async_shared();
-          fence_proxy_async_global();
-          uint8_t* dst = reinterpret_cast<uint8_t*>(merge_o + other * PL::kSlotOFloats);
-          mbar_arrive_expect_tx(rec_bar, (uint32_t)others * rec_bytes);
-          int u = 0;
-          for (int kk = k_lo; kk <= k_hi; ++kk) {
-            if (kk == k) continue;
-            bulk_copy_g2s(dst + (size_t)u * rec_bytes,
-                          p.pieces + (int64_t)(kk + walk.h) * kPieceFloats, rec_bytes, rec_bar);
-            ++u;
-          }
-          pre_rec = 1;
-        }
-      }
-    }
     mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
 
     if constexpr (kFused) {
@@ -1055,14 +1030,13 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
         if (tid == 0) {
           int early = 0;
           if (!single && arrivals_seen == k_hi - k_lo) {
-            if (!pre_rec) asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
+            asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the others' records
             early = 1;
           }
-          s_misc[1] = early | (pre_rec << 1);
+          s_misc[1] = early;
         }
         consumer_bar_sync();
-        const bool early_last = (s_misc[1] & 1) != 0;
-        const bool prefetched = (s_misc[1] & 2) != 0;
+        const bool early_last = s_misc[1] != 0;
         constexpr int RPW = HP / kConsumerWarps;  // rows per warp
         const int d4 = 4 * lane;
         __nv_bfloat16* out_h = p.out + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
@@ -1141,11 +1115,6 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
               Or[i] = make_float4(0.f, 0.f, 0.f, 0.f);
             }
             constexpr int kBatch = NT == 1 ? 4 : 2;
-            // prefetched records: in the idle merge slot, CTA order without this CTA's
-            const float* rec_smem = merge_o + ((q + 1) % PL::kSlots) * PL::kSlotOFloats;
-            if (prefetched) {
-              if (!mbar_wait(rec_bar, 0, abort_flag, p.ctrl)) mbar_drain(rec_bar, 0);
-            }
             for (int kk0 = k_lo; kk0 <= k_hi; kk0 += kBatch) {
               float mb[kBatch][RPW], lb[kBatch][RPW];
               float4 ob[kBatch][RPW];
@@ -1160,11 +1129,6 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
                     mb[u][i] = Mo[i];
                     lb[u][i] = Lo[i];
                     ob[u][i] = Oo[i];
-                  } else if (kk <= k_hi && r < G && prefetched) {
-                    const float* rs = rec_smem + (size_t)(kk - k_lo - (kk > k ? 1 : 0)) * (rec_bytes / 4u);
-                    mb[u][i] = rs[r];
-                    lb[u][i] = rs[kMaxGroup + r];
-                    ob[u][i] = *reinterpret_cast<const float4*>(rs + 2 * kMaxGroup + r * kHeadDim + d4);
                   } else if (kk <= k_hi && r < G) {
                     mb[u][i] = __ldcg(rk + r);
                     lb[u][i] = __ldcg(rk + kMaxGroup + r);
@@ -1207,7 +1171,455 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   }
 }
 
-// ---------------------------------------------------------------- simple kernel
+// ---------------------------------------------------------------- cluster kernel
+//
+// Few heads (a batch of one or two sequences): one flat split of their pages over all
+// SMs would split every head over many CTAs, and the merge of a head's records then
+// costs global round trips (an arrival atomic, then the records).  Instead a
+// thread-block cluster of C CTAs takes each head: CTA r of the cluster streams the
+// head's pages r, r + C, r + 2C, ... exactly as a tiled CTA streams one segment, leaves
+// its partial (m, l, O) in its shared memory, and after a cluster barrier CTA r merges
+// query-head row r over all C partials, read from the cluster's distributed shared
+// memory in rank order (deterministic), and writes it.
+//
+// Early start.  The layer's state (count, ring, page table, pages) changes only in
+// launches that append to this layer.  A fused cluster launch publishes, per head, a
+// sequence number once its cluster is done with that head's state (after every read of
+// its pages and every write: count, ring entry, opened page, new row); the host knows
+// the number the last such launch published (flag_expect, 0 if the state was last
+// written otherwise).  A launch with flag_expect != 0 waits only for its head's flag,
+// then reads the state and stages its first pages before the dependency wait, which
+// then guards only the inputs (q, the new K/V rows and logits) and the output.  A flag
+// that does not arrive within the wait limit records DMS_ERR_TIMEOUT and the launch
+// falls back to the dependency wait, which orders everything before it.
+constexpr int kClusterConsumerWarps = 4;
+constexpr int kClusterThreads = (kClusterConsumerWarps + 1) * 32;  // + a producer warp
+constexpr int kClusterStages = 4;
+constexpr int kClusterMaxSize = 16;
+constexpr int kClusterQBytes = 8 * kRowBytes;  // up to 8 query heads
+
+__host__ __device__ constexpr int cluster_stage_bytes(bool fused) {
+  return 2 * kHalfPageBytes + (fused ? kPatchBytes : 0);
+}
+
+template <bool kFused>
+size_t cluster_smem_bytes() {
+  return (size_t)kClusterStages * cluster_stage_bytes(kFused) + kClusterQBytes +
+         (size_t)(2 * kClusterStages + 1) * sizeof(uint64_t) + 16 * sizeof(int);
+}
+
+// The per-warp and per-CTA partials overlay the stages once every page is consumed.
+static_assert((kConsumerWarps * 8 * (kMergeRow + 2) + 8 * 2 + 8 * kHeadDim) * 4 <=
+                  kClusterStages * cluster_stage_bytes(false),
+              "merge buffers must fit in the stages");
+static_assert(8 + kClusterStages <= 16, "page ids per stage live in s_misc[8..16)");
+
+template <bool kFused>
+__global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(const DecodeParams p) {
+  constexpr int HP = 8;
+  constexpr int kStageBytes = cluster_stage_bytes(kFused);
+  constexpr int kOffPatch = 2 * kHalfPageBytes;
+  extern __shared__ __align__(128) uint8_t smem[];
+  uint8_t* stages = smem;
+  uint8_t* q_buf = smem + kClusterStages * kStageBytes;
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(q_buf + kClusterQBytes);
+  uint64_t* empty_bar = full_bar + kClusterStages;
+  uint64_t* q_bar = empty_bar + kClusterStages;
+  // [0] abort, [1] count after the append, [2] new slot | fresh << 30, [8..) page per stage
+  int* s_misc = reinterpret_cast<int*>(q_bar + 1);
+  float* merge_o = reinterpret_cast<float*>(smem);             // [4][HP][132]
+  float* merge_ml = merge_o + kConsumerWarps * HP * kMergeRow;  // [4][HP][2]
+  float* cta_ml = merge_ml + kConsumerWarps * HP * 2;           // [HP][2]
+  float* cta_o = cta_ml + HP * 2;                               // [HP][128]
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int G = p.group, Hq = p.kv_heads * p.group;
+  volatile int* abort_flag = s_misc;
+  const int C = (int)(gridDim.x / (unsigned)p.heads);  // cluster size (one cluster per head)
+  const int rank = (int)cluster_ctarank();
+  const int h = (int)blockIdx.x / C;
+  const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
+  const int32_t* pt = p.page_table + (int64_t)h * p.max_pages;
+
+  pdl_launch_dependents();
+  if (tid == 0) {
+    s_misc[0] = 0;
+    for (int s = 0; s < kClusterStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], kClusterConsumerWarps);
+    }
+    mbar_init(q_bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  bool waited = false;  // producer warp: the dependency wait is behind it
+  int32_t spec_page = -1;
+  if (warp == kClusterConsumerWarps) {
+    bool early = p.flag_expect != 0u;
+    if (early) {
+      int ok = 1;
+      if (lane == 0) {
+        const unsigned long long t0 = global_timer_ns();
+        for (uint32_t spin = 1;; ++spin) {
+          if (ld_acquire_gpu_u32(p.head_flags + h) == p.flag_expect) break;
+          __nanosleep(32);
+          if ((spin & 31u) == 0u && global_timer_ns() - t0 > kWaitLimitNs) {
+            ok = 0;
+            break;
+          }
+        }
+        if (!ok) set_device_error(p.ctrl, DMS_ERR_TIMEOUT);
+        fence_proxy_async_global();  // the pages were written through the generic proxy
+      }
+      early = __shfl_sync(0xffffffffu, ok, 0) != 0;
+    }
+    if (!early) {
+      pdl_wait_prerequisites();
+      waited = true;
+    }
+    // The head's count, (fused) the ring entry of the token leaving the window, and the
+    // page-table entry of this CTA's first pages (one per lane), all in flight at once.
+    // Fused: delayed eviction for position j (Sec. 3.1-3.2): the token j - window - 1
+    // leaves the window; if it was flagged, the new token takes its slot, otherwise the
+    // fresh slot n_h.
+    const int32_t n = __ldcg(p.counts + h);
+    uint32_t e = 0u;
+    if (kFused && lane == 0 && p.j >= p.window + 1)
+      e = __ldcg(p.ring + (int64_t)h * p.ring_len + (p.j - p.window - 1) % ring_period(p.window));
+    const int spec_pg = rank + C * lane;
+    if (spec_pg < p.max_pages) spec_page = __ldcg(pt + spec_pg);
+    if (lane == 0) {
+      int32_t cnt = n;
+      uint32_t slot_info = 0u;
+      if constexpr (kFused) {
+        const bool reuse = (e & kAlphaBit) != 0u;
+        const uint32_t slot = reuse ? (e & kSlotMask) : (uint32_t)n;
+        cnt = n + (reuse ? 0 : 1);
+        slot_info = slot | ((reuse ? 0u : 1u) << 30);
+      }
+      s_misc[1] = cnt;
+      s_misc[2] = (int)slot_info;
+    }
+  }
+  __syncthreads();
+  const int cnt = s_misc[1];
+  const uint32_t slot_info = (uint32_t)s_misc[2];
+  const int32_t new_slot = (int32_t)(slot_info & 0x3fffffffu);
+  const bool fresh = ((slot_info >> 30) & 1u) != 0u;
+  const int pg_new = kFused ? new_slot / kPageTokens : -1;  // the page the new token lands in
+  const bool opens = kFused && fresh && new_slot % kPageTokens == 0;
+  const int pages = (cnt + kPageTokens - 1) / kPageTokens;
+  const int niters = rank < pages ? (pages - 1 - rank) / C + 1 : 0;
+
+  if (warp == kClusterConsumerWarps) {
+    // ================================================================ producer warp
+    int patch_stage = -1;  // a stage staged before the wait whose patch is still to come
+    // After the dependency wait: the query rows, a pending patch and (rank 0, fused) the
+    // head's new count and ring entry.
+    auto after_wait = [&]() {
+      if (lane == 0) {
+        if (niters > 0) {
+          mbar_arrive_expect_tx(q_bar, (uint32_t)G * kRowBytes);
+          bulk_copy_g2s(q_buf, p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim,
+                        (uint32_t)G * kRowBytes, q_bar);
+        }
+        if (kFused && patch_stage >= 0) {
+          uint8_t* st = stages + patch_stage * kStageBytes;
+          bulk_copy_g2s(st + kOffPatch, p.k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[patch_stage]);
+          bulk_copy_g2s(st + kOffPatch + kRowBytes, p.v_new + (int64_t)h * kHeadDim, kRowBytes,
+                        &full_bar[patch_stage]);
+        }
+        if (kFused && rank == 0) {
+          const uint32_t alpha = decision_from_bf16(p.logit_new[(int64_t)h * p.logit_stride]);
+          p.counts_next[h] = cnt;
+          uint32_t* rh = p.ring + (int64_t)h * p.ring_len;
+          const int64_t RP = ring_period(p.window);
+          rh[p.j % RP] = (uint32_t)new_slot | ((p.decider == 0 ? alpha : 0u) << 31);
+          if (p.decider > 0 && p.j >= p.decider) rh[(p.j - p.decider) % RP] |= alpha << 31;
+        }
+      }
+      __syncwarp();
+    };
+    if (waited) after_wait();
+    const int first = niters < kClusterStages ? niters : kClusterStages;  // staged before the wait
+    for (int it0 = 0; it0 < niters; it0 += 32) {
+      const int it = it0 + lane;
+      int nv = 0, page = 0;
+      if (it < niters) {
+        const int pg = rank + C * it;
+        nv = min(kPageTokens, cnt - pg * kPageTokens);
+        if (opens && pg == pg_new) {  // the new token opens a page
+          page = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
+          if ((int64_t)page >= p.pool_pages) {  // entered as -1: nothing is written there
+            set_device_error(p.ctrl, DMS_ERR_CAPACITY);
+            page = -1;
+          }
+          p.page_table[(int64_t)h * p.max_pages + pg] = page;
+        } else {
+          page = it0 == 0 ? spec_page : __ldcg(pt + pg);
+        }
+      }
+      const int nb = min(32, niters - it0);
+      for (int i = 0; i < nb; ++i) {
+        const int nv_i = __shfl_sync(0xffffffffu, nv, i);
+        const int page_i = __shfl_sync(0xffffffffu, page, i);
+        const int itg = it0 + i;
+        if (lane == 0) {
+          const int s = itg % kClusterStages;
+          const int use = itg / kClusterStages;
+          if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.ctrl);
+          const bool patch = kFused && rank + C * itg == pg_new;
+          const uint32_t kv_bytes = (uint32_t)nv_i * (uint32_t)kRowBytes;
+          uint8_t* st = stages + s * kStageBytes;
+          if constexpr (kFused) s_misc[8 + s] = page_i;
+          mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
+          const uint8_t* src = p.pool + (int64_t)(page_i < 0 ? 0 : page_i) * kPageBytes;
+          bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
+          bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+          if (patch) {  // the new token's K and V rows, as given (unpermuted)
+            if (waited) {
+              bulk_copy_g2s(st + kOffPatch, p.k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[s]);
+              bulk_copy_g2s(st + kOffPatch + kRowBytes, p.v_new + (int64_t)h * kHeadDim, kRowBytes,
+                            &full_bar[s]);
+            } else {
+              patch_stage = s;
+            }
+          }
+        }
+        if (!waited && itg + 1 == first) {  // the first stages are in flight: now the inputs
+          pdl_wait_prerequisites();
+          waited = true;
+          patch_stage = __shfl_sync(0xffffffffu, patch_stage, 0);
+          after_wait();
+        }
+      }
+    }
+    if (!waited) {  // a CTA without pages
+      pdl_wait_prerequisites();
+      waited = true;
+      after_wait();
+    }
+    // Drain: do not leave while a bulk copy may still be writing shared memory.
+    if (lane == 0) {
+      for (int s = 0; s < kClusterStages && s < niters; ++s) {
+        const int last_it = s + ((niters - 1 - s) / kClusterStages) * kClusterStages;
+        mbar_wait(&full_bar[s], (last_it / kClusterStages) & 1, abort_flag, p.ctrl);
+      }
+      if (niters > 0) mbar_wait(q_bar, 0, abort_flag, p.ctrl);
+    }
+    __syncwarp();
+  } else {
+    // ================================================================ consumer warps
+    const int g = lane >> 2, c4 = lane & 3;
+    const int tb = warp * 16;  // this warp's first token within a page
+    const int mi = lane >> 3;
+    uint32_t qb[8][2];
+    float o[8][4];
+    float me = -INFINITY, mo = -INFINITY, le = 0.f, lo = 0.f;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+    if (niters > 0) {
+      mbar_wait(q_bar, 0, abort_flag, p.ctrl);
+      const uint32_t qbase = smem_addr(q_buf);
+      const int row = lane & 7;
+#pragma unroll
+      for (int k2 = 0; k2 < 4; ++k2) {
+        const int kk = 2 * k2 + (mi >> 1);
+        uint32_t r0, r1, r2, r3;
+        ldsm_x4(qbase + row * kRowBytes + (2 * kk + (mi & 1)) * 16, r0, r1, r2, r3);
+        const bool live = g < G;
+        qb[2 * k2][0] = live ? r0 : 0u;
+        qb[2 * k2][1] = live ? r1 : 0u;
+        qb[2 * k2 + 1][0] = live ? r2 : 0u;
+        qb[2 * k2 + 1][1] = live ? r3 : 0u;
+      }
+      if (p.zero_first && lane == 0) qb[0][0] &= 0xffff0000u;
+    }
+    for (int it = 0; it < niters; ++it) {
+      const int s = it % kClusterStages;
+      const int use = it / kClusterStages;
+      const int pg = rank + C * it;
+      const int nvalid = min(kPageTokens, cnt - pg * kPageTokens);
+      uint8_t* st = stages + s * kStageBytes;
+      mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
+      if constexpr (kFused) {
+        const uint32_t r = (uint32_t)(new_slot % kPageTokens);
+        if (pg == pg_new && (int)(r >> 4) == warp) {
+          // the warp whose 16 rows hold the new token moves its K and V row from the
+          // patch buffer into the staged page (permuted layout) and into the pool
+          const int half = lane >> 4, chunk = lane & 15;
+          const uint4 val =
+              *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
+          const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
+          *reinterpret_cast<uint4*>(st + off) = val;
+          const int page = s_misc[8 + s];
+          if (page >= 0) {
+            *reinterpret_cast<uint4*>(p.pool + (int64_t)page * kPageBytes + off) = val;
+            if (lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
+            fence_proxy_async_global();  // a later launch reads this row with a bulk copy
+          }
+          fence_proxy_async_shared();
+          __syncwarp();
+        }
+      }
+      if (tb < nvalid) {
+        float sacc[4][4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) sacc[c][e] = 0.f;
+        const uint32_t kbase = smem_addr(st);
+        const uint32_t krow = (uint32_t)(tb + (mi & 1) * 8 + (lane & 7));
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          uint32_t a[4];
+          ldsm_x4(kbase + swizzled_offset(krow, (uint32_t)(2 * kk + (mi >> 1))), a[0], a[1], a[2], a[3]);
+          mma_bf16_16816(sacc[kk & 3], a, qb[kk][0], qb[kk][1]);
+        }
+        const bool v0 = tb + g < nvalid, v1 = tb + g + 8 < nvalid;
+        const float sl = p.scale_log2;
+        float sc[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sc[e] = (sacc[0][e] + sacc[1][e]) + (sacc[2][e] + sacc[3][e]);
+        const float s0 = v0 ? sc[0] * sl : -INFINITY, s1 = v0 ? sc[1] * sl : -INFINITY;
+        const float s2 = v1 ? sc[2] * sl : -INFINITY, s3 = v1 ? sc[3] * sl : -INFINITY;
+        float xe = fmaxf(s0, s2), xo = fmaxf(s1, s3);
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+          xe = fmaxf(xe, __shfl_xor_sync(0xffffffffu, xe, off));
+          xo = fmaxf(xo, __shfl_xor_sync(0xffffffffu, xo, off));
+        }
+        const float ne = fmaxf(me, xe), no = fmaxf(mo, xo);
+        const float ce = ex2_approx(me - ne), co = ex2_approx(mo - no);
+        me = ne;
+        mo = no;
+        const float p0 = ex2_approx(s0 - ne), p1 = ex2_approx(s1 - no);
+        const float p2 = ex2_approx(s2 - ne), p3 = ex2_approx(s3 - no);
+        le = le * ce + (p0 + p2);
+        lo = lo * co + (p1 + p3);
+        const uint32_t pb0 = movmatrix_trans(pack_bf16x2(p0, p1));
+        const uint32_t pb1 = movmatrix_trans(pack_bf16x2(p2, p3));
+        if (__any_sync(0xffffffffu, (ce != 1.f) || (co != 1.f))) {
+#pragma unroll
+          for (int mt = 0; mt < 8; ++mt) {
+            o[mt][0] *= ce;
+            o[mt][1] *= co;
+            o[mt][2] *= ce;
+            o[mt][3] *= co;
+          }
+        }
+        uint32_t mk_lo = 0xffffffffu, mk_hi = 0xffffffffu;
+        if (tb + 16 > nvalid) {  // stale rows past n_valid must not reach the tensor cores
+          const int t = tb + 2 * c4;
+          mk_lo = (t < nvalid ? 0x0000ffffu : 0u) | (t + 1 < nvalid ? 0xffff0000u : 0u);
+          mk_hi = (t + 8 < nvalid ? 0x0000ffffu : 0u) | (t + 9 < nvalid ? 0xffff0000u : 0u);
+        }
+        const uint32_t vbase = smem_addr(st + kHalfPageBytes);
+        const uint32_t vrow = (uint32_t)(tb + (mi >> 1) * 8 + (lane & 7));
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          uint32_t a[4];
+          ldsm_x4_trans(vbase + swizzled_offset(vrow, (uint32_t)(2 * mt + (mi & 1))), a[0], a[1], a[2], a[3]);
+          a[0] &= mk_lo;
+          a[1] &= mk_lo;
+          a[2] &= mk_hi;
+          a[3] &= mk_hi;
+          mma_bf16_16816(o[mt], a, pb0, pb1);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[s]);
+    }
+    // ---- every consumer warp is done with the stages (and every copy into them has
+    // landed): the partials overlay them.  This warp's partial, then the CTA's (warp w
+    // merges query-head rows w, w + 4).
+    consumer_bar_sync();
+    {
+      float te = le, to = lo;
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+        te += __shfl_xor_sync(0xffffffffu, te, off);
+        to += __shfl_xor_sync(0xffffffffu, to, off);
+      }
+      float* so = merge_o + warp * HP * kMergeRow;
+      float* sml = merge_ml + warp * HP * 2;
+      const int he = 2 * c4, ho = he + 1;
+      if (g == 0) {
+        sml[he * 2] = me;
+        sml[he * 2 + 1] = te;
+        sml[ho * 2] = mo;
+        sml[ho * 2 + 1] = to;
+      }
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        so[he * kMergeRow + 16 * mt + g] = o[mt][0];
+        so[ho * kMergeRow + 16 * mt + g] = o[mt][1];
+        so[he * kMergeRow + 16 * mt + g + 8] = o[mt][2];
+        so[ho * kMergeRow + 16 * mt + g + 8] = o[mt][3];
+      }
+    }
+    consumer_bar_sync();
+    const int d4 = 4 * lane;
+#pragma unroll
+    for (int i = 0; i < HP / kConsumerWarps; ++i) {
+      const int r = warp + kConsumerWarps * i;
+      float M = -INFINITY, L = 0.f;
+      float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (r < G) {
+        float mw[kConsumerWarps];
+#pragma unroll
+        for (int w = 0; w < kConsumerWarps; ++w) {
+          mw[w] = merge_ml[(w * HP + r) * 2];
+          M = fmaxf(M, mw[w]);
+        }
+#pragma unroll
+        for (int w = 0; w < kConsumerWarps; ++w) {
+          const float a = mw[w] == -INFINITY ? 0.f : exp2f(mw[w] - M);
+          const float4 x = *reinterpret_cast<const float4*>(merge_o + (w * HP + r) * kMergeRow + d4);
+          L += a * merge_ml[(w * HP + r) * 2 + 1];
+          O.x += a * x.x;
+          O.y += a * x.y;
+          O.z += a * x.z;
+          O.w += a * x.w;
+        }
+      }
+      if (lane == 0) {
+        cta_ml[r * 2] = M;
+        cta_ml[r * 2 + 1] = L;
+      }
+      *reinterpret_cast<float4*>(cta_o + r * kHeadDim + d4) = O;
+    }
+  }
+  // ---- every CTA's partial is in place, and the cluster is done with the head's state
+  cluster_sync();
+  if (kFused && rank == 0 && tid == 0 && p.flag_publish != 0u)
+    st_release_gpu_u32(p.head_flags + h, p.flag_publish);
+  // CTA `rank` merges row `rank` over the cluster, in rank order
+  if (warp == 0 && rank < G) {
+    const int r = rank, d4 = 4 * lane;
+    const uint32_t ml_addr = smem_addr(cta_ml + r * 2);
+    const uint32_t o_addr = smem_addr(cta_o + r * kHeadDim + d4);
+    float M = -INFINITY, L = 0.f;
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j = 0; j < C; ++j) {
+      const float mj = ld_shared_cluster_f32(mapa_shared(ml_addr, (uint32_t)j));
+      const float lj = ld_shared_cluster_f32(mapa_shared(ml_addr + 4u, (uint32_t)j));
+      const float4 oj = ld_shared_cluster_v4(mapa_shared(o_addr, (uint32_t)j));
+      if (mj == -INFINITY) continue;  // a CTA without pages (or tokens) adds nothing
+      const float Mn = fmaxf(M, mj);
+      const float a = exp2f(M - Mn), w = exp2f(mj - Mn);
+      L = L * a + lj * w;
+      O.x = O.x * a + oj.x * w;
+      O.y = O.y * a + oj.y * w;
+      O.z = O.z * a + oj.z * w;
+      O.w = O.w * a + oj.w * w;
+      M = Mn;
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;  // an empty head gives zeros
+    store_bf16x4(p.out + ((int64_t)b * Hq + (int64_t)hk * G + r) * kHeadDim + d4, O.x * inv,
+                 O.y * inv, O.z * inv, O.w * inv);
+  }
+  cluster_sync();  // no CTA leaves while another still reads its shared memory
+}
 
 // ---------------------------------------------------------------- simple kernel
 
@@ -1316,7 +1728,62 @@ cudaError_t prepare_decode(const Cache& c) {
       tiled_smem_bytes<1, true, true>(kMaxHeadsFused, kStagesFp8Fused));
   set(decode_tiled_kernel<kStagesFp8Fused, 2, true, true>,
       tiled_smem_bytes<2, true, true>(kMaxHeadsFused, kStagesFp8Fused));
+  set(decode_cluster_kernel<false>, cluster_smem_bytes<false>());
+  set(decode_cluster_kernel<true>, cluster_smem_bytes<true>());
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(decode_cluster_kernel<false>,
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(decode_cluster_kernel<true>,
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   return e;
+}
+
+// Clusters of C CTAs of the cluster kernel that fit on the device at once (0 if none):
+// one head per cluster, so a launch takes the cluster kernel only when every head's
+// cluster is resident at the same time.
+int max_active_clusters(int cluster_size, bool fused) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)cluster_size;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3((unsigned)cluster_size * 16u);
+  cfg.blockDim = dim3(kClusterThreads);
+  cfg.dynamicSmemBytes = fused ? cluster_smem_bytes<true>() : cluster_smem_bytes<false>();
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  const cudaError_t e = fused
+      ? cudaOccupancyMaxActiveClusters(&n, decode_cluster_kernel<true>, &cfg)
+      : cudaOccupancyMaxActiveClusters(&n, decode_cluster_kernel<false>, &cfg);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+cudaError_t prepare_cluster_decode(Cache& c) {
+  c.clusters16 = max_active_clusters(16, true);
+  c.clusters8 = max_active_clusters(8, true);
+  const int u16 = max_active_clusters(16, false), u8 = max_active_clusters(8, false);
+  c.clusters16 = c.clusters16 < u16 ? c.clusters16 : u16;
+  c.clusters8 = c.clusters8 < u8 ? c.clusters8 : u8;
+  return cudaSuccess;
+}
+
+// Cluster size for a decode of `group` query heads per KV head on cache `c`, or 0 for the
+// tiled kernel: bf16 pages, up to 8 query heads, the default split options, and few
+// enough heads that every head gets a resident cluster of 16 (else 8) CTAs.
+int decode_cluster_size(const Cache& c, int group) {
+  if (c.fp8() || group > 8 || c.decode_kernel != DMS_DECODE_TILED || c.ctas_per_sm >= 2 ||
+      c.min_pages_per_cta != 2)
+    return 0;
+  if (c.heads <= c.clusters16) return kClusterMaxSize;
+  if (c.heads <= c.clusters8) return 8;
+  return 0;
 }
 
 namespace {
@@ -1373,6 +1840,28 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
              : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 2, false>, p);
 }
 
+cudaError_t launch_cluster(const DecodeParams& p, int cluster_size, cudaStream_t stream, bool fused) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)cluster_size;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3((unsigned)(p.heads * cluster_size));
+  cfg.blockDim = dim3(kClusterThreads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (fused) {
+    cfg.dynamicSmemBytes = cluster_smem_bytes<true>();
+    return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<true>, p);
+  }
+  cfg.dynamicSmemBytes = cluster_smem_bytes<false>();
+  return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<false>, p);
+}
+
 DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* out, int32_t group,
                           float scale_log2) {
   DecodeParams p = {};
@@ -1402,11 +1891,18 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
                                 cudaStream_t stream) {
   DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
   p.zero_first = zero_first ? 1 : 0;
+  const int cs = decode_cluster_size(c, group);
+  if (cs > 0) {
+    p.state_ready = 0;
+    p.head_flags = c.head_flags + (int64_t)layer * c.heads;
+    p.flag_expect = c.flag_valid[layer] ? c.flag_seq[layer] : 0u;
+    return launch_cluster(p, cs, stream, false);
+  }
   return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false, c.fp8());
 }
 
 bool append_decode_fusable(const Cache& c) {
-  return c.decode_kernel == DMS_DECODE_TILED && c.heads <= kMaxHeadsFused && c.ctas_per_sm < 2;
+  return c.decode_kernel != DMS_DECODE_SIMPLE && c.heads <= kMaxHeadsFused && c.ctas_per_sm < 2;
 }
 
 bool tiled_one_cta_per_sm(const Cache& c) { return c.ctas_per_sm < 2; }
@@ -1432,6 +1928,14 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
   p.decider = c.decider();
   p.pool_pages = c.pool_pages;
   p.ring_len = c.ring_len;
+  const int cs = decode_cluster_size(c, group);
+  if (cs > 0) {
+    p.state_ready = 0;
+    p.head_flags = c.head_flags + (int64_t)layer * c.heads;
+    p.flag_expect = c.flag_valid[layer] ? c.flag_seq[layer] : 0u;
+    p.flag_publish = next_flag_seq(c.flag_seq[layer]);
+    return launch_cluster(p, cs, stream, true);
+  }
   return launch_tiled(p, c.num_sms, 1, stream, true, true, c.fp8());
 }
 

@@ -39,6 +39,7 @@
 //   freed       [heads][ring_len] int32          bulk-append scratch (slots freed this call).
 //   pieces      [piece_capacity][kPieceFloats]   split-K partial records of the decode.
 //   piece_counters [heads] int32                 arrivals per head for the last-CTA combine.
+//   head_flags  [layers][heads] u32              completion flags of the cluster kernel.
 // heads = batch * kv_heads, indexed b * kv_heads + h.
 #pragma once
 
@@ -108,12 +109,25 @@ struct Cache {
   // wait (DecodeParams::state_ready in dms_decode.cu).
   int32_t last_layer = -1;
   bool last_full_tiled = false;
+  // Clusters of 16 and of 8 CTAs of the cluster decode kernel resident at once.
+  int32_t clusters16 = 0, clusters8 = 0;
+  // Per-head completion flags of the cluster kernel's fused append + decode: the launch
+  // for length t of layer l stores its sequence number into head_flags[l][h] once head
+  // h's cluster has finished every read and write of the layer's state.  Host: the last
+  // number published per layer, and whether the layer's state was last written by such
+  // a launch (cleared by any other append, a shared prompt or a reset).
+  uint32_t* head_flags = nullptr;  // device [layers][heads]
+  uint32_t* flag_seq = nullptr;    // host [layers]
+  uint8_t* flag_valid = nullptr;   // host [layers]
 
   // Count buffer of `layer` for a layer length of parity `parity`.
   int32_t* counts_at(int32_t layer, int64_t parity) const {
     return counts + ((int64_t)layer * 2 + (parity & 1)) * heads;
   }
 };
+
+// Sequence numbers of the completion flags: nonzero (0 marks "no flag to wait for").
+inline uint32_t next_flag_seq(uint32_t seq) { return seq + 1u == 0u ? 1u : seq + 1u; }
 
 // Ring period (entries per head cycle) for a sliding window w.
 __host__ __device__ __forceinline__ int64_t ring_period(int64_t window) { return window + 2; }
@@ -178,6 +192,9 @@ cudaError_t launch_decode_simple(const Cache& c, int32_t layer, const void* q, v
                                  int32_t group, float scale, bool zero_first, cudaStream_t stream);
 bool append_decode_fusable(const Cache& c);
 bool tiled_one_cta_per_sm(const Cache& c);  // tiled decode launches use one CTA per SM
+cudaError_t prepare_cluster_decode(Cache& c);
+// Cluster size of the decode of `group` query heads per KV head (0: the tiled kernel).
+int decode_cluster_size(const Cache& c, int group);
 cudaError_t launch_bounded_wait_probe(int arrive, int64_t limit_ns, int32_t* dev_status,
                                       cudaStream_t stream);
 cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,

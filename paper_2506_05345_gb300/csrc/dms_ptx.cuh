@@ -238,6 +238,37 @@ __device__ __forceinline__ void named_bar_arrive(int count) {
   asm volatile("bar.arrive %0, %1;" ::"n"(kId), "r"(count) : "memory");
 }
 
+// Thread-block clusters: this CTA's rank, a barrier of every thread of every CTA of the
+// cluster (release / acquire at cluster scope), and loads from another CTA's shared
+// memory (the address of the same variable in CTA `rank`, then a cluster-scope load).
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_shared_cluster_f32(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld_shared_cluster_v4(uint32_t caddr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(caddr)
+               : "memory");
+  return v;
+}
+
 // Relaxed GPU-scope load (no ordering); paired with fence.acq_rel.gpu once its
 // value is acted on, it forms an acquire.
 __device__ __forceinline__ int ld_relaxed_gpu(const int32_t* addr) {

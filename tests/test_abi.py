@@ -84,6 +84,10 @@ def test_kv_format_options_checked_on_host(lib):
     opt.decode_kernel = _native.DMS_DECODE_SIMPLE
     code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
     assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None
+    opt.decode_kernel = 3  # no such decode kernel
+    opt.kv_format = 0
+    code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
+    assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None
     opt.decode_kernel = _native.DMS_DECODE_TILED
     opt.kv_format = 2
     code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)

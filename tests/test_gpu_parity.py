@@ -49,10 +49,12 @@ def _run_all_steps(wl, check_every=1, retained_every=4, **cache_kw):
 
 
 @pytest.mark.parametrize("kernel,fused", [(dms.DMS_DECODE_TILED, False), (dms.DMS_DECODE_TILED, True),
+                                          (dms.DMS_DECODE_SPLIT, False), (dms.DMS_DECODE_SPLIT, True),
                                           (dms.DMS_DECODE_SIMPLE, False)])
 def test_llama_b1_ctx4352_every_step(kernel, fused):
     """Batch 1, 32 q / 8 kv heads, prefill 4096 + 256 decode steps, w = 256, P(evict) 0.875:
-    every step, every query head; retained sets every 16 steps."""
+    every step, every query head; retained sets every 16 steps.  The default kernel runs the
+    8 heads as per-head clusters; DMS_DECODE_SPLIT as the flat split over all SMs."""
     wl = workloads.LLAMA_B1_4K
     mx, mean = _run_all_steps(wl, check_every=1, retained_every=16, decode_kernel=kernel,
                               fused=fused)
@@ -62,30 +64,54 @@ def test_llama_b1_ctx4352_every_step(kernel, fused):
 # ---------------------------------------------------------------- edge cases
 
 
+# The small shapes below have few heads, so the default kernel runs them as per-head clusters;
+# each also runs with DMS_DECODE_SPLIT, the flat split over all SMs.
+TILED_KERNELS = pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_SPLIT],
+                                        ids=["tiled", "split"])
+
+
+@TILED_KERNELS
 @pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("w", [0, 1, 15, 63, 64, 255, 256])
-def test_windows(w, fused):
-    _run_all_steps(small(window=w, prefill=((333, False),), decode_steps=6), fused=fused)
+def test_windows(w, fused, kernel):
+    _run_all_steps(small(window=w, prefill=((333, False),), decode_steps=6), fused=fused,
+                   decode_kernel=kernel)
 
 
+@TILED_KERNELS
 @pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("G", [1, 3, 4, 5, 7, 8, 9, 16])
-def test_gqa_groups(G, fused):
-    _run_all_steps(small(q_heads=2 * G, kv_heads=2, decode_steps=4), fused=fused)
+def test_gqa_groups(G, fused, kernel):
+    _run_all_steps(small(q_heads=2 * G, kv_heads=2, decode_steps=4), fused=fused,
+                   decode_kernel=kernel)
+
+
+@TILED_KERNELS
+@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("prefill", [1, 2, 63, 64, 65, 127, 128, 129, 1000])
+def test_page_boundaries(prefill, fused, kernel):
+    _run_all_steps(small(prefill=((prefill, False),), decode_steps=5, window=20, p_evict=0.5),
+                   fused=fused, decode_kernel=kernel)
+
+
+@TILED_KERNELS
+@pytest.mark.parametrize("w", [0, 3, 40])
+def test_fused_decode_from_empty_cache(w, kernel):
+    """The fused step appends and attends from the very first token (pages opened in-kernel)."""
+    wl = small(window=w, prefill=(), decode_steps=150, p_evict=0.6)
+    _run_all_steps(wl, check_every=7, retained_every=10, fused=True, decode_kernel=kernel)
 
 
 @pytest.mark.parametrize("fused", [False, True])
-@pytest.mark.parametrize("prefill", [1, 2, 63, 64, 65, 127, 128, 129, 1000])
-def test_page_boundaries(prefill, fused):
-    _run_all_steps(small(prefill=((prefill, False),), decode_steps=5, window=20, p_evict=0.5),
-                   fused=fused)
-
-
-@pytest.mark.parametrize("w", [0, 3, 40])
-def test_fused_decode_from_empty_cache(w):
-    """The fused step appends and attends from the very first token (pages opened in-kernel)."""
-    wl = small(window=w, prefill=(), decode_steps=150, p_evict=0.6)
-    _run_all_steps(wl, check_every=7, retained_every=10, fused=True)
+@pytest.mark.parametrize("batch,kv_heads,prefill", [(1, 1, 5000), (1, 8, 20000), (2, 8, 3000),
+                                                    (1, 16, 700), (3, 6, 1500)])
+def test_cluster_shapes(batch, kv_heads, prefill, fused):
+    """Head counts around the cluster sizes' limits (1 to 18 heads), with heads of many pages
+    (5000 and 20000 tokens at P(evict) 0.2: up to 250 pages over 16 CTAs) and of few (a head of
+    700 tokens at 0.2 leaves most of its cluster's CTAs without pages)."""
+    wl = small(batch=batch, kv_heads=kv_heads, q_heads=kv_heads * 5, window=100,
+               prefill=((prefill, False),), decode_steps=3, p_evict=0.2)
+    _run_all_steps(wl, fused=fused)
 
 
 def test_fused_matches_separate_bitwise():
@@ -236,9 +262,10 @@ def test_empty_cache_gives_zeros():
         r.close()
 
 
-def test_deterministic_outputs():
+@pytest.mark.parametrize("kw", [{}, {"min_pages_per_cta": 1}], ids=["cluster", "split1"])
+def test_deterministic_outputs(kw):
     wl = small(prefill=((3000, False),), decode_steps=1, window=64)
-    r = Run(wl, min_pages_per_cta=1)
+    r = Run(wl, **kw)
     try:
         r.prefill()
         q, out = r.step(0)
@@ -303,8 +330,9 @@ def test_reset_and_reuse():
         r.close()
 
 
+@pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_SPLIT], ids=["tiled", "split"])
 @pytest.mark.parametrize("fused", [True, False])
-def test_multilayer_interleaved_steps(fused):
+def test_multilayer_interleaved_steps(fused, kernel):
     """Three layers advanced together, as a model decodes: each step visits layer 0, 1, 2.
     Consecutive launches serve different layers, so the fused kernel reads the layer's state
     and stages its first pages before waiting for the previous launch."""
@@ -313,7 +341,8 @@ def test_multilayer_interleaved_steps(fused):
     L, B, Hkv, G, w, P, steps = 3, 2, 2, 4, 24, 500, 12
     wl = small(batch=B, kv_heads=Hkv, q_heads=Hkv * G, window=w)
     dev = torch.device("cuda")
-    cache = dms.DmsCache(layers=L, kv_heads=Hkv, window=w, capacity=P + steps, batch=B)
+    cache = dms.DmsCache(layers=L, kv_heads=Hkv, window=w, capacity=P + steps, batch=B,
+                         decode_kernel=kernel)
     hist = []
     try:
         for l in range(L):
@@ -355,3 +384,43 @@ def test_multilayer_interleaved_steps(fused):
         assert cache.stats()["device_error"] == 0
     finally:
         cache.close()
+
+
+def test_cluster_early_start_across_mixed_calls():
+    """The per-head completion flags of the cluster kernel: fused steps (which publish),
+    plain decodes in between (which read the state early and publish nothing), single and
+    bulk appends and a reset (after which the next launch waits for its dependency
+    first), on one layer of 1 x 4 heads; outputs and retained sets against the oracle
+    after every call, and no device error."""
+    wl = small(batch=1, kv_heads=4, q_heads=20, window=30, prefill=((700, False),),
+               decode_steps=20, p_evict=0.6)  # capacity 720: 12 tokens appended per round
+    r = Run(wl)
+    try:
+        r.prefill()
+        plan = ["fused", "fused", "decode", "fused", "append1", "decode", "fused", "bulk",
+                "fused", "fused", "decode", "decode", "fused"]
+        for round_ in range(2):
+            for i, what in enumerate(plan):
+                tag = f"r{round_}s{i}"
+                if what in ("fused", "append1", "bulk"):
+                    n = 5 if what == "bulk" else 1
+                    k, v, lg = workloads.gen_kv(wl, 0, tag, n, r.dev)
+                    q = workloads.gen_q(wl, 0, tag, r.dev)
+                    if what == "fused":
+                        out = r.cache.append_and_decode(0, k, v, lg, q, gqa_group=wl.gqa_group)
+                        r.record(k, v, lg)
+                        r.check_outputs(q, out)
+                    else:
+                        r.append(k, v, lg)
+                else:
+                    q = workloads.gen_q(wl, 0, tag, r.dev)
+                    out = r.cache.decode_attention(0, q, gqa_group=wl.gqa_group)
+                    r.check_outputs(q, out)
+                r.check_retained()
+            if round_ == 0:  # start again from an empty layer
+                r.cache.reset()
+                r.t = 0
+                r.prefill()
+        r.summary()
+    finally:
+        r.close()
