@@ -69,16 +69,22 @@ enum {
 
 /* Decode kernels selectable through dms_options.decode_kernel. */
 enum {
-  DMS_DECODE_TILED = 0,  /* default: TMA-staged tensor-core kernels.  When every
-                            (sequence, KV head) can have a resident thread-block
-                            cluster of 16 (else 8) CTAs at once (few heads: a batch
-                            of one or two), bf16 pages, G <= 8 and the default
-                            ctas_per_sm / min_pages_per_cta, each head's pages are
-                            split over its own cluster and merged in distributed
-                            shared memory; otherwise as DMS_DECODE_SPLIT           */
-  DMS_DECODE_SIMPLE = 1, /* one CTA per KV head, CUDA cores; a cross-check path     */
-  DMS_DECODE_SPLIT = 2   /* the tiled kernel with the flat, page-balanced split-K of
-                            all heads' pages over all SMs, for every batch          */
+  DMS_DECODE_TILED = 0,   /* default: TMA-staged tensor-core kernels; as
+                             DMS_DECODE_CLUSTER when clusters of the largest size
+                             in [8, 16] that fits for every head would cover at
+                             least half of the SMs, else as DMS_DECODE_SPLIT       */
+  DMS_DECODE_SIMPLE = 1,  /* one CTA per KV head, CUDA cores; a cross-check path     */
+  DMS_DECODE_SPLIT = 2,   /* the tiled kernel with the flat, page-balanced split-K of
+                             all heads' pages over all SMs, for every batch          */
+  DMS_DECODE_CLUSTER = 3  /* per-head thread-block clusters: when bf16 pages, G <= 8,
+                             the default ctas_per_sm / min_pages_per_cta, and a
+                             resident cluster of 8 CTAs for every (sequence, KV head)
+                             at once (few heads: a batch of one or two), each head's
+                             pages are split over its own cluster of C CTAs and
+                             merged in distributed shared memory, C = 8 for layers
+                             of up to 8192 tokens, else 10 (or the largest size in
+                             [8, 16] that fits, if smaller); otherwise as
+                             DMS_DECODE_SPLIT                                        */
 };
 
 /*
@@ -106,12 +112,12 @@ typedef struct dms_options {
                             shared by all layers and heads; 0 = the dense worst
                             case, layers * batch * kv_heads * ceil(capacity / 64)
                             pages                                                  */
-  int32_t decode_kernel; /* DMS_DECODE_TILED (0), _SIMPLE (1) or _SPLIT (2)          */
+  int32_t decode_kernel; /* DMS_DECODE_TILED (0), _SIMPLE (1), _SPLIT (2), _CLUSTER (3) */
   int32_t ctas_per_sm;   /* split-K CTAs per SM for the tiled kernel; 0 = 1         */
   int32_t min_pages_per_cta; /* lower bound on pages per split-K CTA; 0 = 2         */
   int32_t eviction_policy;   /* DMS_EVICT_DELAYED (0) or DMS_EVICT_IMMEDIATE (1)    */
   int32_t kv_format;     /* DMS_KV_BF16 (0) or DMS_KV_FP8_E4M3 (1); fp8 requires a
-                            tiled decode kernel (TILED or SPLIT)                    */
+                            tiled decode kernel (not SIMPLE)                        */
   int32_t reserved[3];   /* must be zero                                            */
 } dms_options;
 
@@ -327,6 +333,18 @@ dms_status dms_cache_export_kv(dms_cache* cache, int32_t layer, void* host_k, vo
 
 /* Current length (tokens appended per sequence) of `layer`, into *out. */
 dms_status dms_cache_layer_length(const dms_cache* cache, int32_t layer, int64_t* out);
+
+/*
+ * How the next dms_append_and_decode of `layer` (its length + 1 tokens) runs with groups
+ * of gqa_group query heads (host only, no device work): *kernel = DMS_DECODE_SIMPLE,
+ * DMS_DECODE_SPLIT or DMS_DECODE_CLUSTER, the kernel that runs (DMS_DECODE_TILED resolves
+ * to one of the last two); *ctas = CTAs per launch; *cluster_size = CTAs per thread-block
+ * cluster (0 unless DMS_DECODE_CLUSTER).  The cluster size depends on the layer's length
+ * (see DMS_DECODE_TILED).  Errors: DMS_ERR_INVALID_ARGUMENT (NULL pointer, layer out of
+ * range, gqa_group outside [1, 16]).
+ */
+dms_status dms_decode_plan(const dms_cache* cache, int32_t layer, int32_t gqa_group,
+                           int32_t* kernel, int32_t* ctas, int32_t* cluster_size);
 
 /*
  * Decode attention over CALLER-OWNED pages, allocating nothing.

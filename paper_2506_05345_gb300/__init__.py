@@ -22,7 +22,8 @@ import numpy as np
 from . import _native
 from ._native import (DMS_EVICT_DELAYED, DMS_EVICT_IMMEDIATE,  # noqa: F401
                       DMS_PREFILL_MMA_SYNC, DMS_PREFILL_TCGEN05,  # noqa: F401
-                      DMS_DECODE_SIMPLE, DMS_DECODE_SPLIT, DMS_DECODE_TILED,  # noqa: F401
+                      DMS_DECODE_CLUSTER, DMS_DECODE_SIMPLE, DMS_DECODE_SPLIT,  # noqa: F401
+                      DMS_DECODE_TILED,  # noqa: F401
                       DMS_ERR_CAPACITY,  # noqa: F401
                       DMS_KV_BF16, DMS_KV_FP8_E4M3,  # noqa: F401
                       DMS_ERR_INVALID_ARGUMENT, DMS_ERR_STATE, DMS_ERR_TIMEOUT, DMS_OK,
@@ -204,6 +205,14 @@ def dms_cache_layer_length(cache, layer):
     out = ctypes.c_int64()
     code = library().dms_cache_layer_length(cache, layer, ctypes.byref(out))
     return code, out.value
+
+
+def dms_decode_plan(cache, layer, gqa_group):
+    """(code, kernel, ctas, cluster_size) of the next fused decode step of `layer`."""
+    k, n, c = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    code = library().dms_decode_plan(cache, layer, gqa_group, ctypes.byref(k), ctypes.byref(n),
+                                     ctypes.byref(c))
+    return code, k.value, n.value, c.value
 
 
 def dms_decode_attention_paged_noalloc(pool_ptr, page_table_ptr, counts_ptr, batch, kv_heads,
@@ -440,3 +449,9 @@ class DmsCache:
         code, n = dms_cache_layer_length(self._h, layer)
         _check(code, "dms_cache_layer_length")
         return n
+
+    def decode_plan(self, gqa_group: int, layer: int = 0) -> dict:
+        """The kernel the next fused decode step of `layer` runs, its CTAs, cluster size."""
+        code, kernel, ctas, cluster = dms_decode_plan(self._h, layer, gqa_group)
+        _check(code, "dms_decode_plan")
+        return {"kernel": kernel, "ctas": ctas, "cluster_size": cluster}

@@ -79,7 +79,7 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
       capacity < 1 || capacity > dms::kMaxCapacity || opt->batch < 1)
     return DMS_ERR_INVALID_ARGUMENT;
   if (opt->page_tokens != 0 && opt->page_tokens != dms::kPageTokens) return DMS_ERR_INVALID_ARGUMENT;
-  if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_SPLIT ||
+  if (opt->pool_tokens < 0 || opt->decode_kernel < 0 || opt->decode_kernel > DMS_DECODE_CLUSTER ||
       opt->ctas_per_sm < 0 || opt->ctas_per_sm > dms::kMaxCtasPerSm || opt->min_pages_per_cta < 0 ||
       opt->eviction_policy < DMS_EVICT_DELAYED || opt->eviction_policy > DMS_EVICT_IMMEDIATE ||
       opt->kv_format < DMS_KV_BF16 || opt->kv_format > DMS_KV_FP8_E4M3)
@@ -246,7 +246,7 @@ dms_status decode_impl(dms_cache* h, int32_t layer, const void* q, void* out, in
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   c.last_layer = layer;
   c.last_full_tiled = c.decode_kernel != DMS_DECODE_SIMPLE && dms::tiled_one_cta_per_sm(c) &&
-                      dms::decode_cluster_size(c, gqa_group) == 0;
+                      dms::decode_cluster_size(c, gqa_group, c.lengths[layer]) == 0;
   return DMS_OK;
 }
 
@@ -268,7 +268,7 @@ dms_status append_decode_impl(dms_cache* h, int32_t layer, const void* k, const 
     return decode_impl(h, layer, q, out, gqa_group, sm_scale, zero_first, stream);
   }
   const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)dms::kHeadDim);
-  const bool cluster = dms::decode_cluster_size(c, gqa_group) > 0;
+  const bool cluster = dms::decode_cluster_size(c, gqa_group, t0 + 1) > 0;
   const cudaError_t e = dms::launch_append_decode(
       c, layer, k, v, logit, logit_stride, q, out, gqa_group, scale * 1.4426950408889634f,
       zero_first, static_cast<cudaStream_t>(stream));
@@ -486,6 +486,30 @@ dms_status dms_cache_layer_length(const dms_cache* h, int32_t layer, int64_t* ou
   if (h == nullptr || out == nullptr || layer < 0 || layer >= h->c.layers)
     return DMS_ERR_INVALID_ARGUMENT;
   *out = h->c.lengths[layer];
+  return DMS_OK;
+}
+
+dms_status dms_decode_plan(const dms_cache* h, int32_t layer, int32_t gqa_group, int32_t* kernel,
+                           int32_t* ctas, int32_t* cluster_size) {
+  if (h == nullptr || kernel == nullptr || ctas == nullptr || cluster_size == nullptr ||
+      gqa_group < 1 || gqa_group > dms::kMaxGroup || layer < 0 || layer >= h->c.layers)
+    return DMS_ERR_INVALID_ARGUMENT;
+  const Cache& c = h->c;
+  *cluster_size = 0;
+  if (c.decode_kernel == DMS_DECODE_SIMPLE) {
+    *kernel = DMS_DECODE_SIMPLE;
+    *ctas = c.heads;
+    return DMS_OK;
+  }
+  const int cs = dms::decode_cluster_size(c, gqa_group, c.lengths[layer] + 1);
+  if (cs > 0) {
+    *kernel = DMS_DECODE_CLUSTER;
+    *ctas = c.heads * cs;
+    *cluster_size = cs;
+    return DMS_OK;
+  }
+  *kernel = DMS_DECODE_SPLIT;
+  *ctas = c.num_sms * (!c.fp8() && c.ctas_per_sm >= 2 ? c.ctas_per_sm : 1);
   return DMS_OK;
 }
 

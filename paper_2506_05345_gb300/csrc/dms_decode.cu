@@ -1177,41 +1177,55 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
 // SMs would split every head over many CTAs, and the merge of a head's records then
 // costs global round trips (an arrival atomic, then the records).  Instead a
 // thread-block cluster of C CTAs takes each head: CTA r of the cluster streams the
-// head's pages r, r + C, r + 2C, ... exactly as a tiled CTA streams one segment, leaves
-// its partial (m, l, O) in its shared memory, and after a cluster barrier CTA r merges
-// query-head row r over all C partials, read from the cluster's distributed shared
-// memory in rank order (deterministic), and writes it.
+// head's pages r, r + C, r + 2C, ... exactly as a tiled CTA streams one segment and
+// stores its partial (m, l, O) of each query-head row i into the shared memory of CTA i
+// of the cluster (distributed shared memory); after one cluster barrier CTA i merges
+// row i over the C partials in rank order (deterministic) and writes it.
 //
 // Early start.  The layer's state (count, ring, page table, pages) changes only in
 // launches that append to this layer.  A fused cluster launch publishes, per head, a
-// sequence number once its cluster is done with that head's state (after every read of
-// its pages and every write: count, ring entry, opened page, new row); the host knows
-// the number the last such launch published (flag_expect, 0 if the state was last
-// written otherwise).  A launch with flag_expect != 0 waits only for its head's flag,
-// then reads the state and stages its first pages before the dependency wait, which
-// then guards only the inputs (q, the new K/V rows and logits) and the output.  A flag
-// that does not arrive within the wait limit records DMS_ERR_TIMEOUT and the launch
-// falls back to the dependency wait, which orders everything before it.
-constexpr int kClusterConsumerWarps = 4;
+// sequence number as soon as its writes of that head's state (count, ring entry, an
+// opened page, the new row) are visible.  No launch can still be reading what these
+// writes change: opening a page writes past every earlier launch's reads, and everything
+// else is written after the launch's own dependency wait, when every earlier launch has
+// completed.  The host knows the number the last such launch published (flag_expect; 0
+// if the state was last written otherwise).  A launch with flag_expect != 0 waits only
+// for its head's flag, then reads the state and stages its first pages before the
+// dependency wait, which then guards only the inputs (q, the new K/V rows and logits)
+// and the output.  A flag that does not arrive within the wait limit records
+// DMS_ERR_TIMEOUT and the launch falls back to the dependency wait, which orders
+// everything before it.
+// Two groups of four consumer warps take alternate pages (a page's 64 rows are 16 per
+// warp of its group), so that two pages are in the tensor cores at once: one warp per
+// sub-partition leaves the MMA and shared-memory latencies of a page exposed.
+constexpr int kClusterGroups = 2;
+constexpr int kClusterConsumerWarps = 4 * kClusterGroups;
 constexpr int kClusterThreads = (kClusterConsumerWarps + 1) * 32;  // + a producer warp
-constexpr int kClusterStages = 4;
+constexpr int kClusterStages = 6;
 constexpr int kClusterMaxSize = 16;
+constexpr int kClusterMinSize = 8;  // >= the largest group, so every query-head row has an owner CTA
+constexpr int kClusterLongSize = 10;
+constexpr int64_t kClusterShortTokens = 8192;
 constexpr int kClusterQBytes = 8 * kRowBytes;  // up to 8 query heads
 
 __host__ __device__ constexpr int cluster_stage_bytes(bool fused) {
   return 2 * kHalfPageBytes + (fused ? kPatchBytes : 0);
 }
 
+// Partials of one query-head row received from every CTA of the cluster: O, then (m, l).
+constexpr int kClusterRecvBytes = kClusterMaxSize * (kHeadDim + 2) * 4;
+
 template <bool kFused>
 size_t cluster_smem_bytes() {
-  return (size_t)kClusterStages * cluster_stage_bytes(kFused) + kClusterQBytes +
-         (size_t)(2 * kClusterStages + 1) * sizeof(uint64_t) + 16 * sizeof(int);
+  return (size_t)kClusterStages * cluster_stage_bytes(kFused) + kClusterQBytes + kClusterRecvBytes +
+         (size_t)(2 * kClusterStages + 2) * sizeof(uint64_t) + 16 * sizeof(int);
 }
 
-// The per-warp and per-CTA partials overlay the stages once every page is consumed.
-static_assert((kConsumerWarps * 8 * (kMergeRow + 2) + 8 * 2 + 8 * kHeadDim) * 4 <=
+// The per-warp partials overlay the stages once every page is consumed.
+static_assert(kClusterConsumerWarps * 8 * (kMergeRow + 2) * 4 <=
                   kClusterStages * cluster_stage_bytes(false),
               "merge buffers must fit in the stages");
+static_assert(kClusterStages % kClusterGroups == 0, "a stage is always read by the same group");
 static_assert(8 + kClusterStages <= 16, "page ids per stage live in s_misc[8..16)");
 
 template <bool kFused>
@@ -1222,15 +1236,16 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
   uint8_t* q_buf = smem + kClusterStages * kStageBytes;
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(q_buf + kClusterQBytes);
+  float* recv_o = reinterpret_cast<float*>(q_buf + kClusterQBytes);  // [C][128]
+  float* recv_ml = recv_o + kClusterMaxSize * kHeadDim;               // [C][2]
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(recv_ml + 2 * kClusterMaxSize);
   uint64_t* empty_bar = full_bar + kClusterStages;
   uint64_t* q_bar = empty_bar + kClusterStages;
+  uint64_t* pub_bar = q_bar + 1;  // fused: the producer has read the new K and V rows
   // [0] abort, [1] count after the append, [2] new slot | fresh << 30, [8..) page per stage
-  int* s_misc = reinterpret_cast<int*>(q_bar + 1);
-  float* merge_o = reinterpret_cast<float*>(smem);             // [4][HP][132]
-  float* merge_ml = merge_o + kConsumerWarps * HP * kMergeRow;  // [4][HP][2]
-  float* cta_ml = merge_ml + kConsumerWarps * HP * 2;           // [HP][2]
-  float* cta_o = cta_ml + HP * 2;                               // [HP][128]
+  int* s_misc = reinterpret_cast<int*>(pub_bar + 1);
+  float* merge_o = reinterpret_cast<float*>(smem);                    // [8][HP][132]
+  float* merge_ml = merge_o + kClusterConsumerWarps * HP * kMergeRow;  // [8][HP][2]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = p.group, Hq = p.kv_heads * p.group;
@@ -1246,9 +1261,10 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     s_misc[0] = 0;
     for (int s = 0; s < kClusterStages; ++s) {
       mbar_init(&full_bar[s], 1);
-      mbar_init(&empty_bar[s], kClusterConsumerWarps);
+      mbar_init(&empty_bar[s], kClusterConsumerWarps / kClusterGroups);
     }
     mbar_init(q_bar, 1);
+    mbar_init(pub_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   bool waited = false;  // producer warp: the dependency wait is behind it
@@ -1307,14 +1323,14 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   const bool fresh = ((slot_info >> 30) & 1u) != 0u;
   const int pg_new = kFused ? new_slot / kPageTokens : -1;  // the page the new token lands in
   const bool opens = kFused && fresh && new_slot % kPageTokens == 0;
+  const bool patch_cta = kFused && rank == pg_new % C;  // stages that page (its last one)
   const int pages = (cnt + kPageTokens - 1) / kPageTokens;
   const int niters = rank < pages ? (pages - 1 - rank) / C + 1 : 0;
 
   if (warp == kClusterConsumerWarps) {
     // ================================================================ producer warp
     int patch_stage = -1;  // a stage staged before the wait whose patch is still to come
-    // After the dependency wait: the query rows, a pending patch and (rank 0, fused) the
-    // head's new count and ring entry.
+    // After the dependency wait: the query rows and a pending patch.
     auto after_wait = [&]() {
       if (lane == 0) {
         if (niters > 0) {
@@ -1327,14 +1343,6 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           bulk_copy_g2s(st + kOffPatch, p.k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[patch_stage]);
           bulk_copy_g2s(st + kOffPatch + kRowBytes, p.v_new + (int64_t)h * kHeadDim, kRowBytes,
                         &full_bar[patch_stage]);
-        }
-        if (kFused && rank == 0) {
-          const uint32_t alpha = decision_from_bf16(p.logit_new[(int64_t)h * p.logit_stride]);
-          p.counts_next[h] = cnt;
-          uint32_t* rh = p.ring + (int64_t)h * p.ring_len;
-          const int64_t RP = ring_period(p.window);
-          rh[p.j % RP] = (uint32_t)new_slot | ((p.decider == 0 ? alpha : 0u) << 31);
-          if (p.decider > 0 && p.j >= p.decider) rh[(p.j - p.decider) % RP] |= alpha << 31;
         }
       }
       __syncwarp();
@@ -1354,6 +1362,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
             page = -1;
           }
           p.page_table[(int64_t)h * p.max_pages + pg] = page;
+          __threadfence();  // before the flag this CTA publishes once the new row is in
         } else {
           page = it0 == 0 ? spec_page : __ldcg(pt + pg);
         }
@@ -1398,6 +1407,41 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       waited = true;
       after_wait();
     }
+    // Fused, the CTA that stages the new row's page: once that page (with the new K and V
+    // rows) has landed, this warp writes the rows into the pool, the position, the head's
+    // new count and ring entry -- the layer's state of this head is then complete -- and
+    // publishes this launch's flag for the head, off the consumer warps' path.  (A later
+    // launch writes this state only after its dependency wait, when this grid has
+    // completed, so the flag need not wait for the cluster's page reads.)
+    if (patch_cta) {
+      const int itp = pg_new / C, sp = itp % kClusterStages;
+      mbar_wait(&full_bar[sp], (itp / kClusterStages) & 1, abort_flag, p.ctrl);
+      const uint8_t* st = stages + sp * kStageBytes;
+      const uint32_t r = (uint32_t)(new_slot % kPageTokens);
+      const int half = lane >> 4, chunk = lane & 15;
+      const uint4 val =
+          *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
+      const int page = s_misc[8 + sp];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(pub_bar);  // the consumers may now overlay the stages
+      const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
+      if (page >= 0) {
+        *reinterpret_cast<uint4*>(p.pool + (int64_t)page * kPageBytes + off) = val;
+        if (lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
+      }
+      if (lane == 0) {
+        const uint32_t alpha = decision_from_bf16(p.logit_new[(int64_t)h * p.logit_stride]);
+        p.counts_next[h] = cnt;
+        uint32_t* rh = p.ring + (int64_t)h * p.ring_len;
+        const int64_t RP = ring_period(p.window);
+        rh[p.j % RP] = (uint32_t)new_slot | ((p.decider == 0 ? alpha : 0u) << 31);
+        if (p.decider > 0 && p.j >= p.decider) rh[(p.j - p.decider) % RP] |= alpha << 31;
+      }
+      fence_proxy_async_global();  // a later launch reads the row with a bulk copy
+      __threadfence();
+      __syncwarp();
+      if (lane == 0 && p.flag_publish != 0u) st_release_gpu_u32(p.head_flags + h, p.flag_publish);
+    }
     // Drain: do not leave while a bulk copy may still be writing shared memory.
     if (lane == 0) {
       for (int s = 0; s < kClusterStages && s < niters; ++s) {
@@ -1410,7 +1454,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   } else {
     // ================================================================ consumer warps
     const int g = lane >> 2, c4 = lane & 3;
-    const int tb = warp * 16;  // this warp's first token within a page
+    const int grp = warp >> 2, sub = warp & 3;  // pages grp, grp + 2, ...; rows 16 sub ..
+    const int tb = sub * 16;                     // this warp's first token within a page
     const int mi = lane >> 3;
     uint32_t qb[8][2];
     float o[8][4];
@@ -1434,7 +1479,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       }
       if (p.zero_first && lane == 0) qb[0][0] &= 0xffff0000u;
     }
-    for (int it = 0; it < niters; ++it) {
+    for (int it = grp; it < niters; it += kClusterGroups) {
       const int s = it % kClusterStages;
       const int use = it / kClusterStages;
       const int pg = rank + C * it;
@@ -1443,20 +1488,15 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       mbar_wait(&full_bar[s], use & 1, abort_flag, p.ctrl);
       if constexpr (kFused) {
         const uint32_t r = (uint32_t)(new_slot % kPageTokens);
-        if (pg == pg_new && (int)(r >> 4) == warp) {
-          // the warp whose 16 rows hold the new token moves its K and V row from the
-          // patch buffer into the staged page (permuted layout) and into the pool
+        if (pg == pg_new && (int)(r >> 4) == sub) {
+          // The warp whose 16 rows hold the new token moves its K and V row from the
+          // patch buffer into the staged page (permuted layout); the producer warp writes
+          // the row to the pool and the head's state.
           const int half = lane >> 4, chunk = lane & 15;
           const uint4 val =
               *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
           const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
           *reinterpret_cast<uint4*>(st + off) = val;
-          const int page = s_misc[8 + s];
-          if (page >= 0) {
-            *reinterpret_cast<uint4*>(p.pool + (int64_t)page * kPageBytes + off) = val;
-            if (lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
-            fence_proxy_async_global();  // a later launch reads this row with a bulk copy
-          }
           fence_proxy_async_shared();
           __syncwarp();
         }
@@ -1531,8 +1571,10 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     }
     // ---- every consumer warp is done with the stages (and every copy into them has
     // landed): the partials overlay them.  This warp's partial, then the CTA's (warp w
-    // merges query-head rows w, w + 4).
-    consumer_bar_sync();
+    // merges query-head row w).  In the CTA of the new row the producer warp must have read
+    // the new K and V rows from their stage first.
+    if (patch_cta) mbar_wait(pub_bar, 0, abort_flag, p.ctrl);
+    named_bar_sync<1>(kClusterConsumerWarps * 32);
     {
       float te = le, to = lo;
 #pragma unroll
@@ -1557,22 +1599,24 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         so[ho * kMergeRow + 16 * mt + g + 8] = o[mt][3];
       }
     }
-    consumer_bar_sync();
+    named_bar_sync<1>(kClusterConsumerWarps * 32);
+    // The CTA's partial of query-head row r goes straight into the shared memory of CTA r
+    // of the cluster, slot `rank` (rows past G have no owner and are not formed).
     const int d4 = 4 * lane;
-#pragma unroll
-    for (int i = 0; i < HP / kConsumerWarps; ++i) {
-      const int r = warp + kConsumerWarps * i;
-      float M = -INFINITY, L = 0.f;
-      float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    static_assert(kClusterConsumerWarps == 8, "one query-head row per consumer warp");
+    {
+      const int r = warp;
       if (r < G) {
-        float mw[kConsumerWarps];
+        float M = -INFINITY, L = 0.f;
+        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+        float mw[kClusterConsumerWarps];
 #pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) {
+        for (int w = 0; w < kClusterConsumerWarps; ++w) {
           mw[w] = merge_ml[(w * HP + r) * 2];
           M = fmaxf(M, mw[w]);
         }
 #pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) {
+        for (int w = 0; w < kClusterConsumerWarps; ++w) {
           const float a = mw[w] == -INFINITY ? 0.f : exp2f(mw[w] - M);
           const float4 x = *reinterpret_cast<const float4*>(merge_o + (w * HP + r) * kMergeRow + d4);
           L += a * merge_ml[(w * HP + r) * 2 + 1];
@@ -1581,30 +1625,24 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           O.z += a * x.z;
           O.w += a * x.w;
         }
+        st_shared_cluster_v4(mapa_shared(smem_addr(recv_o + rank * kHeadDim + d4), (uint32_t)r), O);
+        if (lane == 0)
+          st_shared_cluster_v2(mapa_shared(smem_addr(recv_ml + rank * 2), (uint32_t)r), M, L);
       }
-      if (lane == 0) {
-        cta_ml[r * 2] = M;
-        cta_ml[r * 2 + 1] = L;
-      }
-      *reinterpret_cast<float4*>(cta_o + r * kHeadDim + d4) = O;
     }
   }
-  // ---- every CTA's partial is in place, and the cluster is done with the head's state
+  // ---- every CTA's partials are in their owners' shared memory (no CTA touches another's
+  // shared memory after this barrier)
   cluster_sync();
-  if (kFused && rank == 0 && tid == 0 && p.flag_publish != 0u)
-    st_release_gpu_u32(p.head_flags + h, p.flag_publish);
   // CTA `rank` merges row `rank` over the cluster, in rank order
   if (warp == 0 && rank < G) {
     const int r = rank, d4 = 4 * lane;
-    const uint32_t ml_addr = smem_addr(cta_ml + r * 2);
-    const uint32_t o_addr = smem_addr(cta_o + r * kHeadDim + d4);
     float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int j = 0; j < C; ++j) {
-      const float mj = ld_shared_cluster_f32(mapa_shared(ml_addr, (uint32_t)j));
-      const float lj = ld_shared_cluster_f32(mapa_shared(ml_addr + 4u, (uint32_t)j));
-      const float4 oj = ld_shared_cluster_v4(mapa_shared(o_addr, (uint32_t)j));
+      const float mj = recv_ml[j * 2], lj = recv_ml[j * 2 + 1];
       if (mj == -INFINITY) continue;  // a CTA without pages (or tokens) adds nothing
+      const float4 oj = *reinterpret_cast<const float4*>(recv_o + j * kHeadDim + d4);
       const float Mn = fmaxf(M, mj);
       const float a = exp2f(M - Mn), w = exp2f(mj - Mn);
       L = L * a + lj * w;
@@ -1618,7 +1656,6 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     store_bf16x4(p.out + ((int64_t)b * Hq + (int64_t)hk * G + r) * kHeadDim + d4, O.x * inv,
                  O.y * inv, O.z * inv, O.w * inv);
   }
-  cluster_sync();  // no CTA leaves while another still reads its shared memory
 }
 
 // ---------------------------------------------------------------- simple kernel
@@ -1766,24 +1803,36 @@ int max_active_clusters(int cluster_size, bool fused) {
 }
 
 cudaError_t prepare_cluster_decode(Cache& c) {
-  c.clusters16 = max_active_clusters(16, true);
-  c.clusters8 = max_active_clusters(8, true);
-  const int u16 = max_active_clusters(16, false), u8 = max_active_clusters(8, false);
-  c.clusters16 = c.clusters16 < u16 ? c.clusters16 : u16;
-  c.clusters8 = c.clusters8 < u8 ? c.clusters8 : u8;
+  for (int cs = kClusterMinSize; cs <= kClusterMaxSize; ++cs) {
+    const int f = max_active_clusters(cs, true), u = max_active_clusters(cs, false);
+    c.max_clusters[cs] = f < u ? f : u;
+  }
   return cudaSuccess;
 }
 
-// Cluster size for a decode of `group` query heads per KV head on cache `c`, or 0 for the
-// tiled kernel: bf16 pages, up to 8 query heads, the default split options, and few
-// enough heads that every head gets a resident cluster of 16 (else 8) CTAs.
-int decode_cluster_size(const Cache& c, int group) {
-  if (c.fp8() || group > 8 || c.decode_kernel != DMS_DECODE_TILED || c.ctas_per_sm >= 2 ||
-      c.min_pages_per_cta != 2)
+// Cluster size for a decode of `group` query heads per KV head over a layer of `tokens`
+// tokens on cache `c`, or 0 for the flat split: bf16 pages, up to 8 query heads, the
+// default split options, and a resident cluster for every head at once.  The default
+// kernel takes clusters only when those of the largest size that fits cover at least half
+// of the SMs: with fewer, a head of many pages streams faster through the flat split over
+// every SM.  The size: a layer of at most kClusterShortTokens tokens (at most 16 pages per
+// CTA even if nothing was evicted) takes the smallest, 8, so that the clusters of
+// consecutive launches fit on the device side by side and each launch stages its pages
+// while the one before runs; a longer layer takes kClusterLongSize (or the largest that
+// fits, if smaller), which spreads its pages over more SMs.  Both constants were measured
+// on GB300 (152 SMs) on batch-1, 8-head layers from 4K to 64K tokens at 1x to 8x
+// compression.
+int decode_cluster_size(const Cache& c, int group, int64_t tokens) {
+  if (c.fp8() || group > 8 || c.ctas_per_sm >= 2 || c.min_pages_per_cta != 2 ||
+      (c.decode_kernel != DMS_DECODE_TILED && c.decode_kernel != DMS_DECODE_CLUSTER))
     return 0;
-  if (c.heads <= c.clusters16) return kClusterMaxSize;
-  if (c.heads <= c.clusters8) return 8;
-  return 0;
+  int largest = 0;
+  for (int cs = kClusterMaxSize; cs >= kClusterMinSize && largest == 0; --cs)
+    if (c.heads <= c.max_clusters[cs]) largest = cs;
+  if (largest == 0) return 0;
+  if (c.decode_kernel == DMS_DECODE_TILED && 2 * c.heads * largest < c.num_sms) return 0;
+  if (tokens <= kClusterShortTokens) return kClusterMinSize;
+  return largest < kClusterLongSize ? largest : kClusterLongSize;
 }
 
 namespace {
@@ -1891,7 +1940,7 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
                                 cudaStream_t stream) {
   DecodeParams p = cache_params(c, layer, q, out, group, scale_log2);
   p.zero_first = zero_first ? 1 : 0;
-  const int cs = decode_cluster_size(c, group);
+  const int cs = decode_cluster_size(c, group, c.lengths[layer]);
   if (cs > 0) {
     p.state_ready = 0;
     p.head_flags = c.head_flags + (int64_t)layer * c.heads;
@@ -1928,7 +1977,7 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
   p.decider = c.decider();
   p.pool_pages = c.pool_pages;
   p.ring_len = c.ring_len;
-  const int cs = decode_cluster_size(c, group);
+  const int cs = decode_cluster_size(c, group, t0 + 1);
   if (cs > 0) {
     p.state_ready = 0;
     p.head_flags = c.head_flags + (int64_t)layer * c.heads;

@@ -109,8 +109,8 @@ struct Cache {
   // wait (DecodeParams::state_ready in dms_decode.cu).
   int32_t last_layer = -1;
   bool last_full_tiled = false;
-  // Clusters of 16 and of 8 CTAs of the cluster decode kernel resident at once.
-  int32_t clusters16 = 0, clusters8 = 0;
+  // Clusters of C CTAs of the cluster decode kernel resident at once, C = 0..16.
+  int32_t max_clusters[17] = {};
   // Per-head completion flags of the cluster kernel's fused append + decode: the launch
   // for length t of layer l stores its sequence number into head_flags[l][h] once head
   // h's cluster has finished every read and write of the layer's state.  Host: the last
@@ -194,7 +194,7 @@ bool append_decode_fusable(const Cache& c);
 bool tiled_one_cta_per_sm(const Cache& c);  // tiled decode launches use one CTA per SM
 cudaError_t prepare_cluster_decode(Cache& c);
 // Cluster size of the decode of `group` query heads per KV head (0: the tiled kernel).
-int decode_cluster_size(const Cache& c, int group);
+int decode_cluster_size(const Cache& c, int group, int64_t tokens);
 cudaError_t launch_bounded_wait_probe(int arrive, int64_t limit_ns, int32_t* dev_status,
                                       cudaStream_t stream);
 cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, const void* v,

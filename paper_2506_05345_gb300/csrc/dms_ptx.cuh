@@ -239,8 +239,9 @@ __device__ __forceinline__ void named_bar_arrive(int count) {
 }
 
 // Thread-block clusters: this CTA's rank, a barrier of every thread of every CTA of the
-// cluster (release / acquire at cluster scope), and loads from another CTA's shared
-// memory (the address of the same variable in CTA `rank`, then a cluster-scope load).
+// cluster (release / acquire at cluster scope: it orders the stores below), and stores
+// into another CTA's shared memory (the address of the same variable in CTA `rank`,
+// then a cluster-scope store).
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -255,18 +256,13 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
   return r;
 }
-__device__ __forceinline__ float ld_shared_cluster_f32(uint32_t caddr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
-  return v;
-}
-__device__ __forceinline__ float4 ld_shared_cluster_v4(uint32_t caddr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(caddr)
+__device__ __forceinline__ void st_shared_cluster_v4(uint32_t caddr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(caddr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
                : "memory");
-  return v;
+}
+__device__ __forceinline__ void st_shared_cluster_v2(uint32_t caddr, float a, float b) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(caddr), "f"(a), "f"(b) : "memory");
 }
 
 // Relaxed GPU-scope load (no ordering); paired with fence.acq_rel.gpu once its

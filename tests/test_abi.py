@@ -73,6 +73,7 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert code == _native.DMS_ERR_INVALID_ARGUMENT
     assert lib.dms_append_and_evict(None, 0, None, None, None, 1, None) == 1
     assert lib.dms_decode_attention(None, 0, None, None, 4, 0.0, None) == 1
+    assert lib.dms_decode_plan(None, 0, 4, None, None, None) == 1
 
 
 def test_kv_format_options_checked_on_host(lib):
@@ -84,7 +85,7 @@ def test_kv_format_options_checked_on_host(lib):
     opt.decode_kernel = _native.DMS_DECODE_SIMPLE
     code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
     assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None
-    opt.decode_kernel = 3  # no such decode kernel
+    opt.decode_kernel = 4  # no such decode kernel
     opt.kv_format = 0
     code, h = dms.dms_cache_create(1, 2, 128, 16, 100, opt)
     assert code == _native.DMS_ERR_INVALID_ARGUMENT and h is None

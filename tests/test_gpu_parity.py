@@ -64,10 +64,10 @@ def test_llama_b1_ctx4352_every_step(kernel, fused):
 # ---------------------------------------------------------------- edge cases
 
 
-# The small shapes below have few heads, so the default kernel runs them as per-head clusters;
-# each also runs with DMS_DECODE_SPLIT, the flat split over all SMs.
-TILED_KERNELS = pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_SPLIT],
-                                        ids=["tiled", "split"])
+# The small shapes below run both as per-head clusters (DMS_DECODE_CLUSTER; the default
+# kernel takes these only for enough heads) and as the flat split over all SMs.
+TILED_KERNELS = pytest.mark.parametrize("kernel", [dms.DMS_DECODE_CLUSTER, dms.DMS_DECODE_SPLIT],
+                                        ids=["cluster", "split"])
 
 
 @TILED_KERNELS
@@ -111,7 +111,7 @@ def test_cluster_shapes(batch, kv_heads, prefill, fused):
     700 tokens at 0.2 leaves most of its cluster's CTAs without pages)."""
     wl = small(batch=batch, kv_heads=kv_heads, q_heads=kv_heads * 5, window=100,
                prefill=((prefill, False),), decode_steps=3, p_evict=0.2)
-    _run_all_steps(wl, fused=fused)
+    _run_all_steps(wl, fused=fused, decode_kernel=dms.DMS_DECODE_CLUSTER)
 
 
 def test_fused_matches_separate_bitwise():
@@ -262,7 +262,8 @@ def test_empty_cache_gives_zeros():
         r.close()
 
 
-@pytest.mark.parametrize("kw", [{}, {"min_pages_per_cta": 1}], ids=["cluster", "split1"])
+@pytest.mark.parametrize("kw", [{"decode_kernel": dms.DMS_DECODE_CLUSTER}, {"min_pages_per_cta": 1}],
+                         ids=["cluster", "split1"])
 def test_deterministic_outputs(kw):
     wl = small(prefill=((3000, False),), decode_steps=1, window=64)
     r = Run(wl, **kw)
@@ -330,7 +331,8 @@ def test_reset_and_reuse():
         r.close()
 
 
-@pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_SPLIT], ids=["tiled", "split"])
+@pytest.mark.parametrize("kernel", [dms.DMS_DECODE_CLUSTER, dms.DMS_DECODE_SPLIT],
+                         ids=["cluster", "split"])
 @pytest.mark.parametrize("fused", [True, False])
 def test_multilayer_interleaved_steps(fused, kernel):
     """Three layers advanced together, as a model decodes: each step visits layer 0, 1, 2.
@@ -394,7 +396,8 @@ def test_cluster_early_start_across_mixed_calls():
     after every call, and no device error."""
     wl = small(batch=1, kv_heads=4, q_heads=20, window=30, prefill=((700, False),),
                decode_steps=20, p_evict=0.6)  # capacity 720: 12 tokens appended per round
-    r = Run(wl)
+    r = Run(wl, decode_kernel=dms.DMS_DECODE_CLUSTER)
+    assert r.cache.decode_plan(wl.gqa_group)["kernel"] == dms.DMS_DECODE_CLUSTER
     try:
         r.prefill()
         plan = ["fused", "fused", "decode", "fused", "append1", "decode", "fused", "bulk",
@@ -424,3 +427,40 @@ def test_cluster_early_start_across_mixed_calls():
         r.summary()
     finally:
         r.close()
+
+
+def test_decode_plan():
+    """Which kernel runs: the default takes per-head clusters for a batch-1 8-head cache, of
+    8 CTAs while the layer is short (<= 8192 tokens) and of up to 10 beyond, and the flat
+    split for many heads or for few heads whose clusters would cover under half of the
+    SMs; DMS_DECODE_CLUSTER takes clusters whenever every head's cluster fits; G > 8, fp8
+    pages and the simple kernel never do."""
+    nsm = torch.cuda.get_device_properties(0).multi_processor_count
+
+    def plan(B, H, G=5, tokens=0, **kw):
+        with dms.DmsCache(layers=1, kv_heads=H, window=16, capacity=tokens + 256, batch=B,
+                          **kw) as c:
+            if tokens:
+                g = torch.Generator(device="cuda").manual_seed(0)
+                k = torch.randn((B, tokens, H, 128), generator=g, device="cuda").to(torch.bfloat16)
+                lg = torch.zeros((B, tokens, H), device="cuda").to(torch.bfloat16)
+                c.append_and_evict(0, k, k, lg)
+            return c.decode_plan(G)
+
+    assert plan(1, 8) == {"kernel": dms.DMS_DECODE_CLUSTER, "ctas": 64, "cluster_size": 8}
+    assert plan(1, 8, tokens=8191)["cluster_size"] == 8   # the next step reads 8192 tokens
+    p = plan(1, 8, tokens=8192)
+    assert p["kernel"] == dms.DMS_DECODE_CLUSTER and 8 <= p["cluster_size"] <= 10
+    assert p["ctas"] == 8 * p["cluster_size"]
+    if nsm == 152:
+        assert p["cluster_size"] == 10
+    assert plan(8, 8)["kernel"] == dms.DMS_DECODE_SPLIT
+    assert plan(1, 2)["kernel"] == dms.DMS_DECODE_SPLIT
+    assert plan(1, 2, decode_kernel=dms.DMS_DECODE_CLUSTER) == {
+        "kernel": dms.DMS_DECODE_CLUSTER, "ctas": 16, "cluster_size": 8}
+    assert plan(1, 8, G=9)["kernel"] == dms.DMS_DECODE_SPLIT
+    assert plan(1, 8, kv_format=dms.DMS_KV_FP8_E4M3)["kernel"] == dms.DMS_DECODE_SPLIT
+    assert plan(1, 8, decode_kernel=dms.DMS_DECODE_SPLIT)["kernel"] == dms.DMS_DECODE_SPLIT
+    assert plan(1, 8, decode_kernel=dms.DMS_DECODE_SIMPLE) == {
+        "kernel": dms.DMS_DECODE_SIMPLE, "ctas": 8, "cluster_size": 0}
+    assert plan(1, 8, min_pages_per_cta=1)["kernel"] == dms.DMS_DECODE_SPLIT
