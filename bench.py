@@ -45,6 +45,8 @@ DECODE_SRCS = [os.path.join(ROOT, "paper_2506_05345_gb300", "csrc", f)
                for f in ("dms_decode.cu", "dms_ptx.cuh", "dms_internal.cuh")]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
 TRAFFIC_FILE_FP8 = os.path.join(ROOT, "profiles", "decode_traffic_fp8.json")
+# dms_options.decode_kernel values (include/dms.h)
+DECODE_KERNELS = {"tiled": 0, "simple": 1, "split": 2, "cluster": 3}
 
 
 def parse():
@@ -59,6 +61,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--kv-fp8", action="store_true",
                     help="fp8 E4M3 page format (per-row fp32 scales)")
+    ap.add_argument("--decode-kernel", default="tiled", choices=list(DECODE_KERNELS),
+                    help="tiled (default: per-head clusters or the flat split), split, cluster, "
+                         "simple")
     ap.add_argument("--ctas-per-sm", type=int, default=0)
     ap.add_argument("--min-pages", type=int, default=0)
     ap.add_argument("--separate", action="store_true",
@@ -309,7 +314,8 @@ def run_ours(args, wl, world, rank, local, pg):
     seed_tag = replica_tag(rank)
     cache = dms.DmsCache(layers=L, kv_heads=H, window=wl.window, capacity=capacity, batch=B,
                          ctas_per_sm=args.ctas_per_sm, min_pages_per_cta=args.min_pages,
-                         kv_format=dms.DMS_KV_FP8_E4M3 if args.kv_fp8 else dms.DMS_KV_BF16)
+                         kv_format=dms.DMS_KV_FP8_E4M3 if args.kv_fp8 else dms.DMS_KV_BF16,
+                         decode_kernel=DECODE_KERNELS[args.decode_kernel])
     stream = torch.cuda.current_stream()
 
     # ---- sampled heads for the parity check and the CPU baseline (layer 0)
@@ -351,6 +357,11 @@ def run_ours(args, wl, world, rank, local, pg):
     st0 = cache.stats()
     if st0["device_error"]:
         raise RuntimeError(f"device error after prefill: {st0}")
+    # the kernel the fused steps launch (per-head clusters or the flat split)
+    plan = cache.decode_plan(G, 0)
+    plan["kernel"] = {v: k for k, v in DECODE_KERNELS.items()}[plan["kernel"]]
+    kernel_name = {"cluster": "decode_cluster_kernel", "simple": "decode_simple_kernel"}.get(
+        plan["kernel"], "decode_tiled_kernel")
 
     # ---- step inputs, resident in HBM before the timed region
     n_dev_steps = W_ + K_ + K2
@@ -657,8 +668,9 @@ def run_ours(args, wl, world, rank, local, pg):
         "retained_tokens_per_layer_step": units_per_launch,
         "compression": (wl.prefill_tokens + n_dev_steps) * B * H / units_per_launch,
         "hbm_frac_of_nominal_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
-        "roofline": {"kernel": "decode_tiled_kernel" + (" (fp8 pages)" if args.kv_fp8 else "") +
+        "roofline": {"kernel": kernel_name + (" (fp8 pages)" if args.kv_fp8 else "") +
                                ("" if args.separate else " (append fused)"),
+                     "launch": plan,
                      "bound": "hbm", "achieved": achieved_gbs,
                      "peak": peak, "unit": "GB/s", "frac": achieved_gbs / peak,
                      "peak_kind": f"{peak_kind} copy bandwidth (read + write; the kernel only "

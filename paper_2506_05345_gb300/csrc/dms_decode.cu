@@ -1203,7 +1203,8 @@ constexpr int kClusterConsumerWarps = 4 * kClusterGroups;
 constexpr int kClusterThreads = (kClusterConsumerWarps + 1) * 32;  // + a producer warp
 constexpr int kClusterStages = 6;
 constexpr int kClusterMaxSize = 16;
-constexpr int kClusterMinSize = 8;  // >= the largest group, so every query-head row has an owner CTA
+constexpr int kClusterMinSize = 2;
+constexpr int kClusterShortSize = 8;
 constexpr int kClusterLongSize = 10;
 constexpr int64_t kClusterShortTokens = 8192;
 constexpr int kClusterQBytes = 8 * kRowBytes;  // up to 8 query heads
@@ -1212,8 +1213,11 @@ __host__ __device__ constexpr int cluster_stage_bytes(bool fused) {
   return 2 * kHalfPageBytes + (fused ? kPatchBytes : 0);
 }
 
-// Partials of one query-head row received from every CTA of the cluster: O, then (m, l).
-constexpr int kClusterRecvBytes = kClusterMaxSize * (kHeadDim + 2) * 4;
+// Partials received from every CTA of the cluster for the query-head rows this CTA owns
+// (rows r with r % C == rank: at most ceil(8 / C) rows, ceil(8 / C) C <= 16 partials for
+// every C in [2, 16]): O, then (m, l).
+constexpr int kClusterRecvSlots = 16;
+constexpr int kClusterRecvBytes = kClusterRecvSlots * (kHeadDim + 2) * 4;
 
 template <bool kFused>
 size_t cluster_smem_bytes() {
@@ -1237,8 +1241,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   uint8_t* stages = smem;
   uint8_t* q_buf = smem + kClusterStages * kStageBytes;
   float* recv_o = reinterpret_cast<float*>(q_buf + kClusterQBytes);  // [C][128]
-  float* recv_ml = recv_o + kClusterMaxSize * kHeadDim;               // [C][2]
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(recv_ml + 2 * kClusterMaxSize);
+  float* recv_ml = recv_o + kClusterRecvSlots * kHeadDim;             // [C][2]
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(recv_ml + 2 * kClusterRecvSlots);
   uint64_t* empty_bar = full_bar + kClusterStages;
   uint64_t* q_bar = empty_bar + kClusterStages;
   uint64_t* pub_bar = q_bar + 1;  // fused: the producer has read the new K and V rows
@@ -1255,6 +1259,18 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   const int h = (int)blockIdx.x / C;
   const int b = h / p.kv_heads, hk = h - b * p.kv_heads;
   const int32_t* pt = p.page_table + (int64_t)h * p.max_pages;
+  // Parameters used after the dependency wait, read before it (see pin_u32).
+  const float scale_log2 = pin_f32(p.scale_log2);
+  const uint32_t zero_first = pin_u32((uint32_t)p.zero_first);
+  __nv_bfloat16* const out = pin_ptr(p.out);
+  const __nv_bfloat16* const q_src = pin_ptr(p.q);
+  const uint16_t* const k_new = pin_ptr(p.k_new);
+  const uint16_t* const v_new = pin_ptr(p.v_new);
+  const uint16_t* const logit_new = pin_ptr(p.logit_new);
+  const int64_t logit_stride = pin_i64(p.logit_stride);
+  int32_t* const counts_next = pin_ptr(p.counts_next);
+  int32_t* const pos_out = pin_ptr(p.pos);
+  const uint32_t flag_publish = pin_u32(p.flag_publish);
 
   pdl_launch_dependents();
   if (tid == 0) {
@@ -1335,13 +1351,13 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       if (lane == 0) {
         if (niters > 0) {
           mbar_arrive_expect_tx(q_bar, (uint32_t)G * kRowBytes);
-          bulk_copy_g2s(q_buf, p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim,
+          bulk_copy_g2s(q_buf, q_src + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim,
                         (uint32_t)G * kRowBytes, q_bar);
         }
         if (kFused && patch_stage >= 0) {
           uint8_t* st = stages + patch_stage * kStageBytes;
-          bulk_copy_g2s(st + kOffPatch, p.k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[patch_stage]);
-          bulk_copy_g2s(st + kOffPatch + kRowBytes, p.v_new + (int64_t)h * kHeadDim, kRowBytes,
+          bulk_copy_g2s(st + kOffPatch, k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[patch_stage]);
+          bulk_copy_g2s(st + kOffPatch + kRowBytes, v_new + (int64_t)h * kHeadDim, kRowBytes,
                         &full_bar[patch_stage]);
         }
       }
@@ -1386,8 +1402,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
           if (patch) {  // the new token's K and V rows, as given (unpermuted)
             if (waited) {
-              bulk_copy_g2s(st + kOffPatch, p.k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[s]);
-              bulk_copy_g2s(st + kOffPatch + kRowBytes, p.v_new + (int64_t)h * kHeadDim, kRowBytes,
+              bulk_copy_g2s(st + kOffPatch, k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[s]);
+              bulk_copy_g2s(st + kOffPatch + kRowBytes, v_new + (int64_t)h * kHeadDim, kRowBytes,
                             &full_bar[s]);
             } else {
               patch_stage = s;
@@ -1427,11 +1443,11 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
       if (page >= 0) {
         *reinterpret_cast<uint4*>(p.pool + (int64_t)page * kPageBytes + off) = val;
-        if (lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
+        if (lane == 0) pos_out[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
       }
       if (lane == 0) {
-        const uint32_t alpha = decision_from_bf16(p.logit_new[(int64_t)h * p.logit_stride]);
-        p.counts_next[h] = cnt;
+        const uint32_t alpha = decision_from_bf16(logit_new[(int64_t)h * logit_stride]);
+        counts_next[h] = cnt;
         uint32_t* rh = p.ring + (int64_t)h * p.ring_len;
         const int64_t RP = ring_period(p.window);
         rh[p.j % RP] = (uint32_t)new_slot | ((p.decider == 0 ? alpha : 0u) << 31);
@@ -1440,7 +1456,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       fence_proxy_async_global();  // a later launch reads the row with a bulk copy
       __threadfence();
       __syncwarp();
-      if (lane == 0 && p.flag_publish != 0u) st_release_gpu_u32(p.head_flags + h, p.flag_publish);
+      if (lane == 0 && flag_publish != 0u) st_release_gpu_u32(p.head_flags + h, flag_publish);
     }
     // Drain: do not leave while a bulk copy may still be writing shared memory.
     if (lane == 0) {
@@ -1477,7 +1493,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         qb[2 * k2 + 1][0] = live ? r2 : 0u;
         qb[2 * k2 + 1][1] = live ? r3 : 0u;
       }
-      if (p.zero_first && lane == 0) qb[0][0] &= 0xffff0000u;
+      if (zero_first && lane == 0) qb[0][0] &= 0xffff0000u;
     }
     for (int it = grp; it < niters; it += kClusterGroups) {
       const int s = it % kClusterStages;
@@ -1516,7 +1532,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           mma_bf16_16816(sacc[kk & 3], a, qb[kk][0], qb[kk][1]);
         }
         const bool v0 = tb + g < nvalid, v1 = tb + g + 8 < nvalid;
-        const float sl = p.scale_log2;
+        const float sl = scale_log2;
         float sc[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) sc[e] = (sacc[0][e] + sacc[1][e]) + (sacc[2][e] + sacc[3][e]);
@@ -1600,8 +1616,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       }
     }
     named_bar_sync<1>(kClusterConsumerWarps * 32);
-    // The CTA's partial of query-head row r goes straight into the shared memory of CTA r
-    // of the cluster, slot `rank` (rows past G have no owner and are not formed).
+    // The CTA's partial of query-head row r goes straight into the shared memory of its
+    // owner, CTA r % C of the cluster, slot (r / C) C + rank (rows past G are not formed).
     const int d4 = 4 * lane;
     static_assert(kClusterConsumerWarps == 8, "one query-head row per consumer warp");
     {
@@ -1625,24 +1641,27 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           O.z += a * x.z;
           O.w += a * x.w;
         }
-        st_shared_cluster_v4(mapa_shared(smem_addr(recv_o + rank * kHeadDim + d4), (uint32_t)r), O);
-        if (lane == 0)
-          st_shared_cluster_v2(mapa_shared(smem_addr(recv_ml + rank * 2), (uint32_t)r), M, L);
+        const int slot = (r / C) * C + rank;
+        const uint32_t owner = (uint32_t)(r % C);
+        st_shared_cluster_v4(mapa_shared(smem_addr(recv_o + slot * kHeadDim + d4), owner), O);
+        if (lane == 0) st_shared_cluster_v2(mapa_shared(smem_addr(recv_ml + slot * 2), owner), M, L);
       }
     }
   }
   // ---- every CTA's partials are in their owners' shared memory (no CTA touches another's
   // shared memory after this barrier)
   cluster_sync();
-  // CTA `rank` merges row `rank` over the cluster, in rank order
-  if (warp == 0 && rank < G) {
-    const int r = rank, d4 = 4 * lane;
+  // CTA `rank` merges its rows r = li C + rank (warp li) over the cluster, in rank order
+  if (warp * C + rank < G) {
+    const int li = warp, r = li * C + rank, d4 = 4 * lane;
+    const float* rml = recv_ml + li * C * 2;
+    const float* ro = recv_o + li * C * kHeadDim;
     float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int j = 0; j < C; ++j) {
-      const float mj = recv_ml[j * 2], lj = recv_ml[j * 2 + 1];
+      const float mj = rml[j * 2], lj = rml[j * 2 + 1];
       if (mj == -INFINITY) continue;  // a CTA without pages (or tokens) adds nothing
-      const float4 oj = *reinterpret_cast<const float4*>(recv_o + j * kHeadDim + d4);
+      const float4 oj = *reinterpret_cast<const float4*>(ro + j * kHeadDim + d4);
       const float Mn = fmaxf(M, mj);
       const float a = exp2f(M - Mn), w = exp2f(mj - Mn);
       L = L * a + lj * w;
@@ -1653,7 +1672,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       M = Mn;
     }
     const float inv = L > 0.f ? 1.f / L : 0.f;  // an empty head gives zeros
-    store_bf16x4(p.out + ((int64_t)b * Hq + (int64_t)hk * G + r) * kHeadDim + d4, O.x * inv,
+    store_bf16x4(out + ((int64_t)b * Hq + (int64_t)hk * G + r) * kHeadDim + d4, O.x * inv,
                  O.y * inv, O.z * inv, O.w * inv);
   }
 }
@@ -1816,12 +1835,12 @@ cudaError_t prepare_cluster_decode(Cache& c) {
 // kernel takes clusters only when those of the largest size that fits cover at least half
 // of the SMs: with fewer, a head of many pages streams faster through the flat split over
 // every SM.  The size: a layer of at most kClusterShortTokens tokens (at most 16 pages per
-// CTA even if nothing was evicted) takes the smallest, 8, so that the clusters of
-// consecutive launches fit on the device side by side and each launch stages its pages
-// while the one before runs; a longer layer takes kClusterLongSize (or the largest that
-// fits, if smaller), which spreads its pages over more SMs.  Both constants were measured
-// on GB300 (152 SMs) on batch-1, 8-head layers from 4K to 64K tokens at 1x to 8x
-// compression.
+// CTA at size 8 even if nothing was evicted) takes kClusterShortSize, small enough that
+// the clusters of consecutive launches fit on the device side by side, so that each
+// launch stages its pages while the one before runs; a longer layer takes
+// kClusterLongSize, which spreads its pages over more SMs; either is capped by the largest
+// size that fits.  The constants were measured on GB300 (152 SMs) on batch-1, 8-head
+// layers from 4K to 64K tokens at 1x to 8x compression.
 int decode_cluster_size(const Cache& c, int group, int64_t tokens) {
   if (c.fp8() || group > 8 || c.ctas_per_sm >= 2 || c.min_pages_per_cta != 2 ||
       (c.decode_kernel != DMS_DECODE_TILED && c.decode_kernel != DMS_DECODE_CLUSTER))
@@ -1831,8 +1850,8 @@ int decode_cluster_size(const Cache& c, int group, int64_t tokens) {
     if (c.heads <= c.max_clusters[cs]) largest = cs;
   if (largest == 0) return 0;
   if (c.decode_kernel == DMS_DECODE_TILED && 2 * c.heads * largest < c.num_sms) return 0;
-  if (tokens <= kClusterShortTokens) return kClusterMinSize;
-  return largest < kClusterLongSize ? largest : kClusterLongSize;
+  const int want = tokens <= kClusterShortTokens ? kClusterShortSize : kClusterLongSize;
+  return largest < want ? largest : want;
 }
 
 namespace {

@@ -273,6 +273,28 @@ __device__ __forceinline__ int ld_relaxed_gpu(const int32_t* addr) {
   return v;
 }
 
+// Read a kernel parameter into a register here (a volatile move cannot sink past the
+// dependency wait): the first read of a launch's parameters misses the constant cache,
+// and done after the wait that miss lands on the critical path.
+__device__ __forceinline__ uint32_t pin_u32(uint32_t v) {
+  asm volatile("mov.b32 %0, %0;" : "+r"(v));
+  return v;
+}
+__device__ __forceinline__ float pin_f32(float v) {
+  asm volatile("mov.b32 %0, %0;" : "+f"(v));
+  return v;
+}
+__device__ __forceinline__ int64_t pin_i64(int64_t v) {
+  asm volatile("mov.b64 %0, %0;" : "+l"(v));
+  return v;
+}
+template <class T>
+__device__ __forceinline__ T* pin_ptr(T* v) {
+  uint64_t x = reinterpret_cast<uint64_t>(v);
+  asm volatile("mov.b64 %0, %0;" : "+l"(x));
+  return reinterpret_cast<T*>(x);
+}
+
 // Programmatic dependent launch: let the next kernel of the stream start its
 // prologue now; wait until the previous kernel's results are visible.  Both are
 // no-ops when the launches carry no programmatic dependency.

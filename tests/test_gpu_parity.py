@@ -103,14 +103,21 @@ def test_fused_decode_from_empty_cache(w, kernel):
 
 
 @pytest.mark.parametrize("fused", [False, True])
-@pytest.mark.parametrize("batch,kv_heads,prefill", [(1, 1, 5000), (1, 8, 20000), (2, 8, 3000),
-                                                    (1, 16, 700), (3, 6, 1500)])
-def test_cluster_shapes(batch, kv_heads, prefill, fused):
-    """Head counts around the cluster sizes' limits (1 to 18 heads), with heads of many pages
-    (5000 and 20000 tokens at P(evict) 0.2: up to 250 pages over 16 CTAs) and of few (a head of
-    700 tokens at 0.2 leaves most of its cluster's CTAs without pages)."""
-    wl = small(batch=batch, kv_heads=kv_heads, q_heads=kv_heads * 5, window=100,
+@pytest.mark.parametrize("batch,kv_heads,G,prefill", [
+    (1, 1, 5, 5000), (1, 8, 5, 20000), (2, 8, 5, 3000), (1, 16, 5, 700), (3, 6, 5, 1500),
+    (5, 8, 5, 1200), (8, 8, 8, 900), (8, 8, 3, 9000)])
+def test_cluster_shapes(batch, kv_heads, G, prefill, fused):
+    """Head counts over the cluster sizes' range (1 to 64 heads: clusters of 16 CTAs down to 2),
+    with heads of many pages (5000 and 20000 tokens at P(evict) 0.2: up to 250 pages over a
+    cluster) and of few (a head of 700 tokens leaves most of its cluster's CTAs without
+    pages), and clusters smaller than the group (40 heads of G = 5 and 64 heads of G = 8,
+    whose query-head rows are shared out over the cluster's CTAs)."""
+    wl = small(batch=batch, kv_heads=kv_heads, q_heads=kv_heads * G, window=100,
                prefill=((prefill, False),), decode_steps=3, p_evict=0.2)
+    r = Run(wl, decode_kernel=dms.DMS_DECODE_CLUSTER)
+    plan = r.cache.decode_plan(G)
+    r.close()
+    assert plan["kernel"] == dms.DMS_DECODE_CLUSTER, plan
     _run_all_steps(wl, fused=fused, decode_kernel=dms.DMS_DECODE_CLUSTER)
 
 
@@ -431,10 +438,11 @@ def test_cluster_early_start_across_mixed_calls():
 
 def test_decode_plan():
     """Which kernel runs: the default takes per-head clusters for a batch-1 8-head cache, of
-    8 CTAs while the layer is short (<= 8192 tokens) and of up to 10 beyond, and the flat
-    split for many heads or for few heads whose clusters would cover under half of the
-    SMs; DMS_DECODE_CLUSTER takes clusters whenever every head's cluster fits; G > 8, fp8
-    pages and the simple kernel never do."""
+    8 CTAs while the layer is short (<= 8192 tokens) and of up to 10 beyond, and for 64
+    heads (clusters of 2 on GB300); the flat split for more heads than clusters fit, or for
+    few heads whose clusters would cover under half of the SMs; DMS_DECODE_CLUSTER takes
+    clusters whenever every head's cluster fits; G > 8, fp8 pages and the simple kernel
+    never do."""
     nsm = torch.cuda.get_device_properties(0).multi_processor_count
 
     def plan(B, H, G=5, tokens=0, **kw):
@@ -454,7 +462,11 @@ def test_decode_plan():
     assert p["ctas"] == 8 * p["cluster_size"]
     if nsm == 152:
         assert p["cluster_size"] == 10
-    assert plan(8, 8)["kernel"] == dms.DMS_DECODE_SPLIT
+    p = plan(8, 8)  # 64 heads: the largest size that fits is small
+    assert p["kernel"] == dms.DMS_DECODE_CLUSTER and p["cluster_size"] >= 2
+    if nsm == 152:
+        assert p == {"kernel": dms.DMS_DECODE_CLUSTER, "ctas": 128, "cluster_size": 2}
+    assert plan(16, 8)["kernel"] == dms.DMS_DECODE_SPLIT  # 128 heads: no cluster fits each
     assert plan(1, 2)["kernel"] == dms.DMS_DECODE_SPLIT
     assert plan(1, 2, decode_kernel=dms.DMS_DECODE_CLUSTER) == {
         "kernel": dms.DMS_DECODE_CLUSTER, "ctas": 16, "cluster_size": 8}
