@@ -1222,7 +1222,7 @@ constexpr int kClusterRecvBytes = kClusterRecvSlots * (kHeadDim + 2) * 4;
 template <bool kFused>
 size_t cluster_smem_bytes() {
   return (size_t)kClusterStages * cluster_stage_bytes(kFused) + kClusterQBytes + kClusterRecvBytes +
-         (size_t)(2 * kClusterStages + 2) * sizeof(uint64_t) + 16 * sizeof(int);
+         (size_t)(2 * kClusterStages + 1) * sizeof(uint64_t) + 16 * sizeof(int);
 }
 
 // The per-warp partials overlay the stages once every page is consumed.
@@ -1230,7 +1230,6 @@ static_assert(kClusterConsumerWarps * 8 * (kMergeRow + 2) * 4 <=
                   kClusterStages * cluster_stage_bytes(false),
               "merge buffers must fit in the stages");
 static_assert(kClusterStages % kClusterGroups == 0, "a stage is always read by the same group");
-static_assert(8 + kClusterStages <= 16, "page ids per stage live in s_misc[8..16)");
 
 template <bool kFused>
 __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(const DecodeParams p) {
@@ -1245,9 +1244,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(recv_ml + 2 * kClusterRecvSlots);
   uint64_t* empty_bar = full_bar + kClusterStages;
   uint64_t* q_bar = empty_bar + kClusterStages;
-  uint64_t* pub_bar = q_bar + 1;  // fused: the producer has read the new K and V rows
-  // [0] abort, [1] count after the append, [2] new slot | fresh << 30, [8..) page per stage
-  int* s_misc = reinterpret_cast<int*>(pub_bar + 1);
+  // [0] abort, [1] count after the append, [2] new slot | fresh << 30
+  int* s_misc = reinterpret_cast<int*>(q_bar + 1);
   float* merge_o = reinterpret_cast<float*>(smem);                    // [8][HP][132]
   float* merge_ml = merge_o + kClusterConsumerWarps * HP * kMergeRow;  // [8][HP][2]
 
@@ -1280,9 +1278,9 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       mbar_init(&empty_bar[s], kClusterConsumerWarps / kClusterGroups);
     }
     mbar_init(q_bar, 1);
-    mbar_init(pub_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  cluster_arrive_relaxed();  // waited for before the first store into another CTA
   bool waited = false;  // producer warp: the dependency wait is behind it
   int32_t spec_page = -1;
   if (warp == kClusterConsumerWarps) {
@@ -1303,6 +1301,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         fence_proxy_async_global();  // the pages were written through the generic proxy
       }
       early = __shfl_sync(0xffffffffu, ok, 0) != 0;
+      // every lane reads the state: each acquires the (already published) flag itself
+      if (early) (void)ld_acquire_gpu_u32(p.head_flags + h);
     }
     if (!early) {
       pdl_wait_prerequisites();
@@ -1339,15 +1339,62 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   const bool fresh = ((slot_info >> 30) & 1u) != 0u;
   const int pg_new = kFused ? new_slot / kPageTokens : -1;  // the page the new token lands in
   const bool opens = kFused && fresh && new_slot % kPageTokens == 0;
-  const bool patch_cta = kFused && rank == pg_new % C;  // stages that page (its last one)
+  const bool patch_cta = kFused && rank == pg_new % C;  // the CTA of the new row's page
   const int pages = (cnt + kPageTokens - 1) / kPageTokens;
   const int niters = rank < pages ? (pages - 1 - rank) / C + 1 : 0;
 
   if (warp == kClusterConsumerWarps) {
     // ================================================================ producer warp
     int patch_stage = -1;  // a stage staged before the wait whose patch is still to come
-    // After the dependency wait: the query rows and a pending patch.
+    // Fused, the CTA whose pages include the new row's page (pg_new): that page's id,
+    // opened here if the new token starts it.
+    int patch_page = -1;
+    if (patch_cta) {
+      if (lane == 0) {
+        if (opens) {
+          patch_page = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
+          if ((int64_t)patch_page >= p.pool_pages) {  // entered as -1: nothing is written there
+            set_device_error(p.ctrl, DMS_ERR_CAPACITY);
+            patch_page = -1;
+          }
+          p.page_table[(int64_t)h * p.max_pages + pg_new] = patch_page;
+        } else {
+          patch_page = __ldcg(pt + pg_new);
+        }
+      }
+      patch_page = __shfl_sync(0xffffffffu, patch_page, 0);
+    }
+    // After the dependency wait: the query rows and a pending patch; and (fused, the CTA of
+    // the new row's page) the new K and V rows into the pool (from the inputs), the
+    // position, the head's new count and ring entry.  The layer's state of this head is
+    // then complete and this launch's flag for the head is published.  (A later launch
+    // writes this state only after its dependency wait, when this grid has completed, so
+    // the flag need not wait for this launch's page reads; and this launch's consumer warps
+    // take the new row from their own copy of it, whatever the bulk copy of the page read.)
     auto after_wait = [&]() {
+      if (kFused && patch_cta) {
+        const uint32_t r = (uint32_t)(new_slot % kPageTokens);
+        const int half = lane >> 4, chunk = lane & 15;
+        const uint4 val = __ldg(reinterpret_cast<const uint4*>((half ? v_new : k_new) +
+                                                               (int64_t)h * kHeadDim) + chunk);
+        if (patch_page >= 0) {
+          const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
+          *reinterpret_cast<uint4*>(p.pool + (int64_t)patch_page * kPageBytes + off) = val;
+          if (lane == 0) pos_out[(int64_t)patch_page * kPageTokens + r] = (int32_t)p.j;
+        }
+        if (lane == 0) {
+          const uint32_t alpha = decision_from_bf16(logit_new[(int64_t)h * logit_stride]);
+          counts_next[h] = cnt;
+          uint32_t* rh = p.ring + (int64_t)h * p.ring_len;
+          const int64_t RP = ring_period(p.window);
+          rh[p.j % RP] = (uint32_t)new_slot | ((p.decider == 0 ? alpha : 0u) << 31);
+          if (p.decider > 0 && p.j >= p.decider) rh[(p.j - p.decider) % RP] |= alpha << 31;
+        }
+        fence_proxy_async_global();  // a later launch reads the row with a bulk copy
+        __threadfence();
+        __syncwarp();
+        if (lane == 0 && flag_publish != 0u) st_release_gpu_u32(p.head_flags + h, flag_publish);
+      }
       if (lane == 0) {
         if (niters > 0) {
           mbar_arrive_expect_tx(q_bar, (uint32_t)G * kRowBytes);
@@ -1371,14 +1418,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       if (it < niters) {
         const int pg = rank + C * it;
         nv = min(kPageTokens, cnt - pg * kPageTokens);
-        if (opens && pg == pg_new) {  // the new token opens a page
-          page = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
-          if ((int64_t)page >= p.pool_pages) {  // entered as -1: nothing is written there
-            set_device_error(p.ctrl, DMS_ERR_CAPACITY);
-            page = -1;
-          }
-          p.page_table[(int64_t)h * p.max_pages + pg] = page;
-          __threadfence();  // before the flag this CTA publishes once the new row is in
+        if (kFused && pg == pg_new) {
+          page = patch_page;
         } else {
           page = it0 == 0 ? spec_page : __ldcg(pt + pg);
         }
@@ -1395,7 +1436,6 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           const bool patch = kFused && rank + C * itg == pg_new;
           const uint32_t kv_bytes = (uint32_t)nv_i * (uint32_t)kRowBytes;
           uint8_t* st = stages + s * kStageBytes;
-          if constexpr (kFused) s_misc[8 + s] = page_i;
           mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
           const uint8_t* src = p.pool + (int64_t)(page_i < 0 ? 0 : page_i) * kPageBytes;
           bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
@@ -1423,41 +1463,6 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       waited = true;
       after_wait();
     }
-    // Fused, the CTA that stages the new row's page: once that page (with the new K and V
-    // rows) has landed, this warp writes the rows into the pool, the position, the head's
-    // new count and ring entry -- the layer's state of this head is then complete -- and
-    // publishes this launch's flag for the head, off the consumer warps' path.  (A later
-    // launch writes this state only after its dependency wait, when this grid has
-    // completed, so the flag need not wait for the cluster's page reads.)
-    if (patch_cta) {
-      const int itp = pg_new / C, sp = itp % kClusterStages;
-      mbar_wait(&full_bar[sp], (itp / kClusterStages) & 1, abort_flag, p.ctrl);
-      const uint8_t* st = stages + sp * kStageBytes;
-      const uint32_t r = (uint32_t)(new_slot % kPageTokens);
-      const int half = lane >> 4, chunk = lane & 15;
-      const uint4 val =
-          *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
-      const int page = s_misc[8 + sp];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(pub_bar);  // the consumers may now overlay the stages
-      const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
-      if (page >= 0) {
-        *reinterpret_cast<uint4*>(p.pool + (int64_t)page * kPageBytes + off) = val;
-        if (lane == 0) pos_out[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
-      }
-      if (lane == 0) {
-        const uint32_t alpha = decision_from_bf16(logit_new[(int64_t)h * logit_stride]);
-        counts_next[h] = cnt;
-        uint32_t* rh = p.ring + (int64_t)h * p.ring_len;
-        const int64_t RP = ring_period(p.window);
-        rh[p.j % RP] = (uint32_t)new_slot | ((p.decider == 0 ? alpha : 0u) << 31);
-        if (p.decider > 0 && p.j >= p.decider) rh[(p.j - p.decider) % RP] |= alpha << 31;
-      }
-      fence_proxy_async_global();  // a later launch reads the row with a bulk copy
-      __threadfence();
-      __syncwarp();
-      if (lane == 0 && flag_publish != 0u) st_release_gpu_u32(p.head_flags + h, flag_publish);
-    }
     // Drain: do not leave while a bulk copy may still be writing shared memory.
     if (lane == 0) {
       for (int s = 0; s < kClusterStages && s < niters; ++s) {
@@ -1467,6 +1472,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       if (niters > 0) mbar_wait(q_bar, 0, abort_flag, p.ctrl);
     }
     __syncwarp();
+    cluster_wait();
   } else {
     // ================================================================ consumer warps
     const int g = lane >> 2, c4 = lane & 3;
@@ -1587,9 +1593,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     }
     // ---- every consumer warp is done with the stages (and every copy into them has
     // landed): the partials overlay them.  This warp's partial, then the CTA's (warp w
-    // merges query-head row w).  In the CTA of the new row the producer warp must have read
-    // the new K and V rows from their stage first.
-    if (patch_cta) mbar_wait(pub_bar, 0, abort_flag, p.ctrl);
+    // merges query-head row w).
     named_bar_sync<1>(kClusterConsumerWarps * 32);
     {
       float te = le, to = lo;
@@ -1620,6 +1624,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     // owner, CTA r % C of the cluster, slot (r / C) C + rank (rows past G are not formed).
     const int d4 = 4 * lane;
     static_assert(kClusterConsumerWarps == 8, "one query-head row per consumer warp");
+    cluster_wait();  // every CTA of the cluster runs
     {
       const int r = warp;
       if (r < G) {

@@ -476,3 +476,31 @@ def test_decode_plan():
     assert plan(1, 8, decode_kernel=dms.DMS_DECODE_SIMPLE) == {
         "kernel": dms.DMS_DECODE_SIMPLE, "ctas": 8, "cluster_size": 0}
     assert plan(1, 8, min_pages_per_cta=1)["kernel"] == dms.DMS_DECODE_SPLIT
+
+
+@pytest.mark.parametrize("batch,kv_heads", [(1, 1), (1, 2)])
+def test_cluster_stored_rows_after_fused_steps(batch, kv_heads):
+    """Fused steps on per-head clusters whose CTAs stream more pages than they have stages,
+    with a window of 4000 tokens at P(evict) 0.9: the slots the window's tokens hold are
+    spread over the whole head, so the new token usually takes a slot in a page its CTA
+    staged early and has reused since.  Every stored K/V row stays bit-exact (the row at
+    each retained slot is its position's input), and outputs and retained sets match the
+    oracle."""
+    wl = small(batch=batch, kv_heads=kv_heads, q_heads=kv_heads * 5, window=4000,
+               prefill=((8000, False),), decode_steps=40, p_evict=0.9)
+    r = Run(wl, fused=True, decode_kernel=dms.DMS_DECODE_CLUSTER)
+    try:
+        plan = r.cache.decode_plan(wl.gqa_group)
+        assert plan["kernel"] == dms.DMS_DECODE_CLUSTER
+        r.prefill()
+        pages = int(r.cache.stats(with_counts=True)["counts"].max() + 63) // 64
+        assert pages > 6 * plan["cluster_size"]  # more pages per CTA than stages
+        for s in range(wl.decode_steps):
+            q, out = r.step(s)
+            if s % 10 == 9:
+                r.check_outputs(q, out)
+                r.check_retained()
+        r.check_codes()
+        r.summary()
+    finally:
+        r.close()
