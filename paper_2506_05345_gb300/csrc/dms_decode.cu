@@ -48,6 +48,14 @@ constexpr int kProducerWarp = 4;
 constexpr int kEpilogueWarp = 5;
 constexpr int kThreads = 6 * 32;
 constexpr int kQBytes = kMaxGroup * kRowBytes;                 // 4096
+// Staged query rows are read by ldmatrix, eight rows at a time at the same column: at a
+// 256-byte row stride those eight 16-byte reads fall on the same four banks.  Groups of
+// up to 8 query heads are staged one row per bulk copy at a 272-byte stride instead, which
+// puts the eight rows on distinct banks (16 rows at that stride would not fit the area).
+constexpr int kQRowPadded = kRowBytes + 16;
+static_assert(8 * kQRowPadded <= kQBytes, "padded rows of one n-tile fit the query area");
+template <int NT>
+__host__ __device__ constexpr int q_row_stride() { return NT == 1 ? kQRowPadded : kRowBytes; }
 constexpr int kPatchBytes = 2 * kRowBytes;                     // new K and V row (fused append)
 constexpr int kStageBytesPlain = 2 * kHalfPageBytes + kQBytes;  // 36864
 constexpr int kStageBytesFused = kStageBytesPlain + kPatchBytes;  // 37376
@@ -416,7 +424,13 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
       if (seg_start) {
         const int b = h_i / p.kv_heads, hk = h_i - b * p.kv_heads;
         const __nv_bfloat16* qsrc = p.q + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
-        bulk_copy_g2s(st + kOffQ, qsrc, (uint32_t)G * kRowBytes, &full_bar[s]);
+        if constexpr (NT == 1) {
+          for (int i = 0; i < G; ++i)
+            bulk_copy_g2s(st + kOffQ + i * kQRowPadded, qsrc + (int64_t)i * kHeadDim, kRowBytes,
+                          &full_bar[s]);
+        } else {
+          bulk_copy_g2s(st + kOffQ, qsrc, (uint32_t)G * kRowBytes, &full_bar[s]);
+        }
       }
       if constexpr (kFused) {
         if (patch) {  // the new token's K and V rows, as given (unpermuted)
@@ -807,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
         for (int k2 = 0; k2 < 4; ++k2) {
           const int kk = 2 * k2 + (mi >> 1);
           uint32_t r0, r1, r2, r3;
-          ldsm_x4(qbase + row * kRowBytes + (2 * kk + (mi & 1)) * 16, r0, r1, r2, r3);
+          ldsm_x4(qbase + row * q_row_stride<NT>() + (2 * kk + (mi & 1)) * 16, r0, r1, r2, r3);
           const bool live = 8 * nt + g < G;
           qb[2 * k2][nt][0] = live ? r0 : 0u;
           qb[2 * k2][nt][1] = live ? r1 : 0u;
@@ -1207,7 +1221,7 @@ constexpr int kClusterMinSize = 2;
 constexpr int kClusterShortSize = 8;
 constexpr int kClusterLongSize = 10;
 constexpr int64_t kClusterShortTokens = 8192;
-constexpr int kClusterQBytes = 8 * kRowBytes;  // up to 8 query heads
+constexpr int kClusterQBytes = 8 * kQRowPadded;  // up to 8 query heads, padded rows
 
 __host__ __device__ constexpr int cluster_stage_bytes(bool fused) {
   return 2 * kHalfPageBytes + (fused ? kPatchBytes : 0);
@@ -1398,8 +1412,9 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       if (lane == 0) {
         if (niters > 0) {
           mbar_arrive_expect_tx(q_bar, (uint32_t)G * kRowBytes);
-          bulk_copy_g2s(q_buf, q_src + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim,
-                        (uint32_t)G * kRowBytes, q_bar);
+          const __nv_bfloat16* qs = q_src + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+          for (int i = 0; i < G; ++i)
+            bulk_copy_g2s(q_buf + i * kQRowPadded, qs + (int64_t)i * kHeadDim, kRowBytes, q_bar);
         }
         if (kFused && patch_stage >= 0) {
           uint8_t* st = stages + patch_stage * kStageBytes;
@@ -1492,7 +1507,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       for (int k2 = 0; k2 < 4; ++k2) {
         const int kk = 2 * k2 + (mi >> 1);
         uint32_t r0, r1, r2, r3;
-        ldsm_x4(qbase + row * kRowBytes + (2 * kk + (mi & 1)) * 16, r0, r1, r2, r3);
+        ldsm_x4(qbase + row * kQRowPadded + (2 * kk + (mi & 1)) * 16, r0, r1, r2, r3);
         const bool live = g < G;
         qb[2 * k2][0] = live ? r0 : 0u;
         qb[2 * k2][1] = live ? r1 : 0u;
