@@ -100,9 +100,10 @@ enum {
                           row and tensor: scale = amax(|row|) / 448 (fp32 division),
                           code = E4M3(row / scale) rounded to nearest even and
                           saturated; a row of zeros has scale 0.  Pages of 16 KiB
-                          (+ 512 bytes of scales).  Rows must be finite.  Taken only
-                          by the tiled decode kernel; single-token append + decode
-                          runs as two launches.                                      */
+                          (+ 512 bytes of scales).  Rows must be finite.  Read by
+                          the tiled kernels (the flat split and the per-head
+                          clusters), not by DMS_DECODE_SIMPLE; the single-token
+                          append + decode runs in one launch.                        */
 };
 
 typedef struct dms_options {

@@ -1215,7 +1215,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
 constexpr int kClusterGroups = 2;
 constexpr int kClusterConsumerWarps = 4 * kClusterGroups;
 constexpr int kClusterThreads = (kClusterConsumerWarps + 1) * 32;  // + a producer warp
-constexpr int kClusterStages = 6;
+// Stages of the page ring: six 32 KiB bf16 pages, or twelve 16.5 KiB fp8 pages (K codes,
+// V^T codes, the 128 row scales), in about the same 210 KB.
+template <bool kFp8>
+__host__ __device__ constexpr int cluster_stages() { return kFp8 ? 12 : 6; }
 constexpr int kClusterMaxSize = 16;
 constexpr int kClusterMinSize = 2;
 constexpr int kClusterShortSize = 8;
@@ -1223,8 +1226,8 @@ constexpr int kClusterLongSize = 10;
 constexpr int64_t kClusterShortTokens = 8192;
 constexpr int kClusterQBytes = 8 * kQRowPadded;  // up to 8 query heads, padded rows
 
-__host__ __device__ constexpr int cluster_stage_bytes(bool fused) {
-  return 2 * kHalfPageBytes + (fused ? kPatchBytes : 0);
+__host__ __device__ constexpr int cluster_stage_bytes(bool fused, bool fp8) {
+  return (fp8 ? 2 * kHalfPageBytesFp8 + kScaleBytes : 2 * kHalfPageBytes) + (fused ? kPatchBytes : 0);
 }
 
 // Partials received from every CTA of the cluster for the query-head rows this CTA owns
@@ -1233,23 +1236,54 @@ __host__ __device__ constexpr int cluster_stage_bytes(bool fused) {
 constexpr int kClusterRecvSlots = 16;
 constexpr int kClusterRecvBytes = kClusterRecvSlots * (kHeadDim + 2) * 4;
 
-template <bool kFused>
+template <bool kFused, bool kFp8>
 size_t cluster_smem_bytes() {
-  return (size_t)kClusterStages * cluster_stage_bytes(kFused) + kClusterQBytes + kClusterRecvBytes +
-         (size_t)(2 * kClusterStages + 1) * sizeof(uint64_t) + 16 * sizeof(int);
+  return (size_t)cluster_stages<kFp8>() * cluster_stage_bytes(kFused, kFp8) + kClusterQBytes +
+         kClusterRecvBytes + (size_t)(2 * cluster_stages<kFp8>() + 1) * sizeof(uint64_t) +
+         16 * sizeof(int);
 }
 
 // The per-warp partials overlay the stages once every page is consumed.
 static_assert(kClusterConsumerWarps * 8 * (kMergeRow + 2) * 4 <=
-                  kClusterStages * cluster_stage_bytes(false),
+                  cluster_stages<false>() * cluster_stage_bytes(false, false) &&
+              kClusterConsumerWarps * 8 * (kMergeRow + 2) * 4 <=
+                  cluster_stages<true>() * cluster_stage_bytes(false, true),
               "merge buffers must fit in the stages");
-static_assert(kClusterStages % kClusterGroups == 0, "a stage is always read by the same group");
+static_assert(cluster_stages<false>() % kClusterGroups == 0 &&
+              cluster_stages<true>() % kClusterGroups == 0, "a stage is always read by the same group");
 
-template <bool kFused>
+// E4M3 codes of head_dim 4 lane .. 4 lane + 3 of a bf16 row (two words per lane, the whole
+// warp holding the row) and the row's scale, as the append kernels quantise: scale =
+// amax(|row|) / 448 (fp32 division), code = E4M3(x / scale) rounded to nearest even and
+// saturated; a row of zeros has scale 0 and codes 0.  pair[e] holds dims 4 lane + 2e (low
+// byte) and 4 lane + 2e + 1.
+__device__ __forceinline__ float quantize_row_e4m3(uint2 w, uint16_t (&pair)[2]) {
+  float x[4];
+  x[0] = __uint_as_float(w.x << 16);
+  x[1] = __uint_as_float(w.x & 0xffff0000u);
+  x[2] = __uint_as_float(w.y << 16);
+  x[3] = __uint_as_float(w.y & 0xffff0000u);
+  float a = fmaxf(fmaxf(fabsf(x[0]), fabsf(x[1])), fmaxf(fabsf(x[2]), fabsf(x[3])));
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, off));
+  const float scale = a == 0.f ? 0.f : __fdiv_rn(a, 448.f);
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const float lo = scale == 0.f ? 0.f : __fdiv_rn(x[2 * e], scale);
+    const float hi = scale == 0.f ? 0.f : __fdiv_rn(x[2 * e + 1], scale);
+    asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(pair[e]) : "f"(hi), "f"(lo));
+  }
+  return scale;
+}
+
+template <bool kFused, bool kFp8>
 __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(const DecodeParams p) {
   constexpr int HP = 8;
-  constexpr int kStageBytes = cluster_stage_bytes(kFused);
-  constexpr int kOffPatch = 2 * kHalfPageBytes;
+  constexpr int kClusterStages = cluster_stages<kFp8>();
+  constexpr int kStageBytes = cluster_stage_bytes(kFused, kFp8);
+  constexpr int kKvHalf = kFp8 ? kHalfPageBytesFp8 : kHalfPageBytes;  // the V half of a stage
+  constexpr int kOffScales = 2 * kHalfPageBytesFp8;                   // fp8: K, V row scales
+  constexpr int kOffPatch = kFp8 ? kOffScales + kScaleBytes : 2 * kHalfPageBytes;
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
   uint8_t* q_buf = smem + kClusterStages * kStageBytes;
@@ -1388,13 +1422,40 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     auto after_wait = [&]() {
       if (kFused && patch_cta) {
         const uint32_t r = (uint32_t)(new_slot % kPageTokens);
-        const int half = lane >> 4, chunk = lane & 15;
-        const uint4 val = __ldg(reinterpret_cast<const uint4*>((half ? v_new : k_new) +
-                                                               (int64_t)h * kHeadDim) + chunk);
-        if (patch_page >= 0) {
-          const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
-          *reinterpret_cast<uint4*>(p.pool + (int64_t)patch_page * kPageBytes + off) = val;
-          if (lane == 0) pos_out[(int64_t)patch_page * kPageTokens + r] = (int32_t)p.j;
+        if constexpr (kFp8) {  // quantise both rows (lane: head_dim 4 lane .. 4 lane + 3)
+          uint8_t* pg8 = p.pool + (int64_t)(patch_page < 0 ? 0 : patch_page) * kPageBytesFp8;
+#pragma unroll
+          for (int kv = 0; kv < 2; ++kv) {
+            const uint2 w = __ldg(reinterpret_cast<const uint2*>((kv ? v_new : k_new) +
+                                                                 (int64_t)h * kHeadDim) + lane);
+            uint16_t pair[2];
+            const float scale = quantize_row_e4m3(w, pair);
+            if (patch_page >= 0) {
+#pragma unroll
+              for (int e = 0; e < 2; ++e) {
+                const uint32_t d = 4u * (uint32_t)lane + 2u * (uint32_t)e;
+                if (kv == 0) {
+                  *reinterpret_cast<uint16_t*>(pg8 + k8_offset(r, d)) = pair[e];
+                } else {
+                  pg8[vt8_offset(r, d)] = (uint8_t)(pair[e] & 0xffu);
+                  pg8[vt8_offset(r, d + 1)] = (uint8_t)(pair[e] >> 8);
+                }
+              }
+              if (lane == 0)
+                p.scales[(int64_t)patch_page * 2 * kPageTokens + kv * kPageTokens + r] = scale;
+            }
+          }
+          if (patch_page >= 0 && lane == 0)
+            pos_out[(int64_t)patch_page * kPageTokens + r] = (int32_t)p.j;
+        } else {
+          const int half = lane >> 4, chunk = lane & 15;
+          const uint4 val = __ldg(reinterpret_cast<const uint4*>((half ? v_new : k_new) +
+                                                                 (int64_t)h * kHeadDim) + chunk);
+          if (patch_page >= 0) {
+            const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
+            *reinterpret_cast<uint4*>(p.pool + (int64_t)patch_page * kPageBytes + off) = val;
+            if (lane == 0) pos_out[(int64_t)patch_page * kPageTokens + r] = (int32_t)p.j;
+          }
         }
         if (lane == 0) {
           const uint32_t alpha = decision_from_bf16(logit_new[(int64_t)h * logit_stride]);
@@ -1449,12 +1510,26 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           const int use = itg / kClusterStages;
           if (use > 0) mbar_wait(&empty_bar[s], (use - 1) & 1, abort_flag, p.ctrl);
           const bool patch = kFused && rank + C * itg == pg_new;
-          const uint32_t kv_bytes = (uint32_t)nv_i * (uint32_t)kRowBytes;
           uint8_t* st = stages + s * kStageBytes;
-          mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
-          const uint8_t* src = p.pool + (int64_t)(page_i < 0 ? 0 : page_i) * kPageBytes;
-          bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
-          bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+          const int64_t page0 = page_i < 0 ? 0 : page_i;
+          if constexpr (kFp8) {
+            // the valid K rows; all of V^T (its rows interleave the slots) and the scales
+            const uint32_t k_bytes = (uint32_t)nv_i * 128u;
+            mbar_arrive_expect_tx(&full_bar[s], k_bytes + (uint32_t)kHalfPageBytesFp8 +
+                                                    (uint32_t)kScaleBytes +
+                                                    (patch ? (uint32_t)kPatchBytes : 0u));
+            const uint8_t* src = p.pool + page0 * kPageBytesFp8;
+            bulk_copy_g2s(st, src, k_bytes, &full_bar[s]);
+            bulk_copy_g2s(st + kKvHalf, src + kHalfPageBytesFp8, kHalfPageBytesFp8, &full_bar[s]);
+            bulk_copy_g2s(st + kOffScales, p.scales + page0 * 2 * kPageTokens, kScaleBytes,
+                          &full_bar[s]);
+          } else {
+            const uint32_t kv_bytes = (uint32_t)nv_i * (uint32_t)kRowBytes;
+            mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
+            const uint8_t* src = p.pool + page0 * kPageBytes;
+            bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
+            bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+          }
           if (patch) {  // the new token's K and V rows, as given (unpermuted)
             if (waited) {
               bulk_copy_g2s(st + kOffPatch, k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[s]);
@@ -1514,6 +1589,13 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         qb[2 * k2 + 1][0] = live ? r2 : 0u;
         qb[2 * k2 + 1][1] = live ? r3 : 0u;
       }
+      if constexpr (kFp8) {  // the fp8 path multiplies in f16
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          qb[kk][0] = bf16x2_to_f16x2(qb[kk][0]);
+          qb[kk][1] = bf16x2_to_f16x2(qb[kk][1]);
+        }
+      }
       if (zero_first && lane == 0) qb[0][0] &= 0xffff0000u;
     }
     for (int it = grp; it < niters; it += kClusterGroups) {
@@ -1527,13 +1609,34 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         const uint32_t r = (uint32_t)(new_slot % kPageTokens);
         if (pg == pg_new && (int)(r >> 4) == sub) {
           // The warp whose 16 rows hold the new token moves its K and V row from the
-          // patch buffer into the staged page (permuted layout); the producer warp writes
-          // the row to the pool and the head's state.
-          const int half = lane >> 4, chunk = lane & 15;
-          const uint4 val =
-              *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
-          const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
-          *reinterpret_cast<uint4*>(st + off) = val;
+          // patch buffer into the staged page (permuted layout; fp8: quantised, with the
+          // row scales, exactly as the producer warp writes them to the pool); the producer
+          // warp writes the row to the pool and the head's state.
+          if constexpr (kFp8) {
+#pragma unroll
+            for (int kv = 0; kv < 2; ++kv) {
+              const uint2 w = *reinterpret_cast<const uint2*>(st + kOffPatch + kv * kRowBytes + lane * 8);
+              uint16_t pair[2];
+              const float scale = quantize_row_e4m3(w, pair);
+#pragma unroll
+              for (int e = 0; e < 2; ++e) {
+                const uint32_t d = 4u * (uint32_t)lane + 2u * (uint32_t)e;
+                if (kv == 0) {
+                  *reinterpret_cast<uint16_t*>(st + k8_offset(r, d)) = pair[e];
+                } else {
+                  st[vt8_offset(r, d)] = (uint8_t)(pair[e] & 0xffu);
+                  st[vt8_offset(r, d + 1)] = (uint8_t)(pair[e] >> 8);
+                }
+              }
+              if (lane == 0) reinterpret_cast<float*>(st + kOffScales)[kv * kPageTokens + r] = scale;
+            }
+          } else {
+            const int half = lane >> 4, chunk = lane & 15;
+            const uint4 val =
+                *reinterpret_cast<const uint4*>(st + kOffPatch + half * kRowBytes + chunk * 16);
+            const uint32_t off = (uint32_t)half * kHalfPageBytes + swizzled_offset(r, (uint32_t)chunk);
+            *reinterpret_cast<uint4*>(st + off) = val;
+          }
           fence_proxy_async_shared();
           __syncwarp();
         }
@@ -1544,21 +1647,52 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         for (int c = 0; c < 4; ++c)
 #pragma unroll
           for (int e = 0; e < 4; ++e) sacc[c][e] = 0.f;
-        const uint32_t kbase = smem_addr(st);
-        const uint32_t krow = (uint32_t)(tb + (mi & 1) * 8 + (lane & 7));
+        if constexpr (kFp8) {
+          // rows tb + g and tb + g + 8; the 16-byte chunk of k-steps 4 kg .. 4 kg + 3 holds
+          // this thread's codes (d = 16 kk + {2c, 2c+1, 2c+8, 2c+9}) in word kk % 4
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          uint32_t a[4];
-          ldsm_x4(kbase + swizzled_offset(krow, (uint32_t)(2 * kk + (mi >> 1))), a[0], a[1], a[2], a[3]);
-          mma_bf16_16816(sacc[kk & 3], a, qb[kk][0], qb[kk][1]);
+          for (int kg = 0; kg < 2; ++kg) {
+            const uint4 w0 = *reinterpret_cast<const uint4*>(st + (tb + g) * 128 + (((4 * kg + c4) ^ g) << 4));
+            const uint4 w1 =
+                *reinterpret_cast<const uint4*>(st + (tb + g + 8) * 128 + (((4 * kg + c4) ^ g) << 4));
+            const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int kk = 4 * kg + i;
+              uint32_t a[4];
+              a[0] = e4m3x2_to_f16x2(x0[i]);
+              a[1] = e4m3x2_to_f16x2(x1[i]);
+              a[2] = e4m3x2_to_f16x2(x0[i] >> 16);
+              a[3] = e4m3x2_to_f16x2(x1[i] >> 16);
+              mma_f16_16816(sacc[kk & 3], a, qb[kk][0], qb[kk][1]);
+            }
+          }
+        } else {
+          const uint32_t kbase = smem_addr(st);
+          const uint32_t krow = (uint32_t)(tb + (mi & 1) * 8 + (lane & 7));
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            uint32_t a[4];
+            ldsm_x4(kbase + swizzled_offset(krow, (uint32_t)(2 * kk + (mi >> 1))), a[0], a[1], a[2], a[3]);
+            mma_bf16_16816(sacc[kk & 3], a, qb[kk][0], qb[kk][1]);
+          }
         }
         const bool v0 = tb + g < nvalid, v1 = tb + g + 8 < nvalid;
-        const float sl = scale_log2;
+        // score scale of tokens tb + g and tb + g + 8 (fp8: times the keys' row scales); fp8
+        // also folds each value's row scale into P, per token (stale tokens take 0)
+        float sl0 = scale_log2, sl1 = scale_log2, vs0 = 1.f, vs1 = 1.f;
+        if constexpr (kFp8) {
+          const float* ksc = reinterpret_cast<const float*>(st + kOffScales);
+          sl0 *= ksc[tb + g];
+          sl1 *= ksc[tb + g + 8];
+          vs0 = v0 ? ksc[kPageTokens + tb + g] : 0.f;
+          vs1 = v1 ? ksc[kPageTokens + tb + g + 8] : 0.f;
+        }
         float sc[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) sc[e] = (sacc[0][e] + sacc[1][e]) + (sacc[2][e] + sacc[3][e]);
-        const float s0 = v0 ? sc[0] * sl : -INFINITY, s1 = v0 ? sc[1] * sl : -INFINITY;
-        const float s2 = v1 ? sc[2] * sl : -INFINITY, s3 = v1 ? sc[3] * sl : -INFINITY;
+        const float s0 = v0 ? sc[0] * sl0 : -INFINITY, s1 = v0 ? sc[1] * sl0 : -INFINITY;
+        const float s2 = v1 ? sc[2] * sl1 : -INFINITY, s3 = v1 ? sc[3] * sl1 : -INFINITY;
         float xe = fmaxf(s0, s2), xo = fmaxf(s1, s3);
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
@@ -1573,8 +1707,10 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         const float p2 = ex2_approx(s2 - ne), p3 = ex2_approx(s3 - no);
         le = le * ce + (p0 + p2);
         lo = lo * co + (p1 + p3);
-        const uint32_t pb0 = movmatrix_trans(pack_bf16x2(p0, p1));
-        const uint32_t pb1 = movmatrix_trans(pack_bf16x2(p2, p3));
+        const uint32_t pb0 = kFp8 ? movmatrix_trans(pack_f16x2(p0 * vs0, p1 * vs0))
+                                  : movmatrix_trans(pack_bf16x2(p0, p1));
+        const uint32_t pb1 = kFp8 ? movmatrix_trans(pack_f16x2(p2 * vs1, p3 * vs1))
+                                  : movmatrix_trans(pack_bf16x2(p2, p3));
         if (__any_sync(0xffffffffu, (ce != 1.f) || (co != 1.f))) {
 #pragma unroll
           for (int mt = 0; mt < 8; ++mt) {
@@ -1590,17 +1726,37 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           mk_lo = (t < nvalid ? 0x0000ffffu : 0u) | (t + 1 < nvalid ? 0xffff0000u : 0u);
           mk_hi = (t + 8 < nvalid ? 0x0000ffffu : 0u) | (t + 9 < nvalid ? 0xffff0000u : 0u);
         }
-        const uint32_t vbase = smem_addr(st + kHalfPageBytes);
-        const uint32_t vrow = (uint32_t)(tb + (mi >> 1) * 8 + (lane & 7));
+        if constexpr (kFp8) {
+          // V^T rows d = 16 mt + g and + 8: one word holds the codes of tokens tb + {2c, 2c+1,
+          // 2c+8, 2c+9} (the row scales are in P); stale tokens masked
+          const int blk = tb >> 4;
 #pragma unroll
-        for (int mt = 0; mt < 8; ++mt) {
-          uint32_t a[4];
-          ldsm_x4_trans(vbase + swizzled_offset(vrow, (uint32_t)(2 * mt + (mi & 1))), a[0], a[1], a[2], a[3]);
-          a[0] &= mk_lo;
-          a[1] &= mk_lo;
-          a[2] &= mk_hi;
-          a[3] &= mk_hi;
-          mma_bf16_16816(o[mt], a, pb0, pb1);
+          for (int mt = 0; mt < 8; ++mt) {
+            const int d0 = 16 * mt + g, d1 = d0 + 8;
+            const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
+                st + kKvHalf + d0 * 64 + ((blk ^ ((d0 >> 1) & 3)) << 4) + 4 * c4);
+            const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
+                st + kKvHalf + d1 * 64 + ((blk ^ ((d1 >> 1) & 3)) << 4) + 4 * c4);
+            uint32_t a[4];
+            a[0] = e4m3x2_to_f16x2(w0) & mk_lo;
+            a[1] = e4m3x2_to_f16x2(w1) & mk_lo;
+            a[2] = e4m3x2_to_f16x2(w0 >> 16) & mk_hi;
+            a[3] = e4m3x2_to_f16x2(w1 >> 16) & mk_hi;
+            mma_f16_16816(o[mt], a, pb0, pb1);
+          }
+        } else {
+          const uint32_t vbase = smem_addr(st + kHalfPageBytes);
+          const uint32_t vrow = (uint32_t)(tb + (mi >> 1) * 8 + (lane & 7));
+#pragma unroll
+          for (int mt = 0; mt < 8; ++mt) {
+            uint32_t a[4];
+            ldsm_x4_trans(vbase + swizzled_offset(vrow, (uint32_t)(2 * mt + (mi & 1))), a[0], a[1], a[2], a[3]);
+            a[0] &= mk_lo;
+            a[1] &= mk_lo;
+            a[2] &= mk_hi;
+            a[3] &= mk_hi;
+            mma_bf16_16816(o[mt], a, pb0, pb1);
+          }
         }
       }
       __syncwarp();
@@ -1804,21 +1960,23 @@ cudaError_t prepare_decode(const Cache& c) {
       tiled_smem_bytes<1, true, true>(kMaxHeadsFused, kStagesFp8Fused));
   set(decode_tiled_kernel<kStagesFp8Fused, 2, true, true>,
       tiled_smem_bytes<2, true, true>(kMaxHeadsFused, kStagesFp8Fused));
-  set(decode_cluster_kernel<false>, cluster_smem_bytes<false>());
-  set(decode_cluster_kernel<true>, cluster_smem_bytes<true>());
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(decode_cluster_kernel<false>,
-                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(decode_cluster_kernel<true>,
-                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  auto set_cluster = [&](auto kernel, size_t bytes) {
+    set(kernel, bytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  };
+  set_cluster(decode_cluster_kernel<false, false>, cluster_smem_bytes<false, false>());
+  set_cluster(decode_cluster_kernel<true, false>, cluster_smem_bytes<true, false>());
+  set_cluster(decode_cluster_kernel<false, true>, cluster_smem_bytes<false, true>());
+  set_cluster(decode_cluster_kernel<true, true>, cluster_smem_bytes<true, true>());
   return e;
 }
 
 // Clusters of C CTAs of the cluster kernel that fit on the device at once (0 if none):
 // one head per cluster, so a launch takes the cluster kernel only when every head's
 // cluster is resident at the same time.
-int max_active_clusters(int cluster_size, bool fused) {
+template <bool kFused, bool kFp8>
+int max_active_clusters(int cluster_size) {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1827,13 +1985,12 @@ int max_active_clusters(int cluster_size, bool fused) {
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3((unsigned)cluster_size * 16u);
   cfg.blockDim = dim3(kClusterThreads);
-  cfg.dynamicSmemBytes = fused ? cluster_smem_bytes<true>() : cluster_smem_bytes<false>();
+  cfg.dynamicSmemBytes = cluster_smem_bytes<kFused, kFp8>();
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  const cudaError_t e = fused
-      ? cudaOccupancyMaxActiveClusters(&n, decode_cluster_kernel<true>, &cfg)
-      : cudaOccupancyMaxActiveClusters(&n, decode_cluster_kernel<false>, &cfg);
+  const cudaError_t e =
+      cudaOccupancyMaxActiveClusters(&n, decode_cluster_kernel<kFused, kFp8>, &cfg);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return 0;
@@ -1843,15 +2000,18 @@ int max_active_clusters(int cluster_size, bool fused) {
 
 cudaError_t prepare_cluster_decode(Cache& c) {
   for (int cs = kClusterMinSize; cs <= kClusterMaxSize; ++cs) {
-    const int f = max_active_clusters(cs, true), u = max_active_clusters(cs, false);
-    c.max_clusters[cs] = f < u ? f : u;
+    const int n[4] = {max_active_clusters<false, false>(cs), max_active_clusters<true, false>(cs),
+                      max_active_clusters<false, true>(cs), max_active_clusters<true, true>(cs)};
+    int m = n[0];
+    for (int i = 1; i < 4; ++i) m = n[i] < m ? n[i] : m;
+    c.max_clusters[cs] = m;
   }
   return cudaSuccess;
 }
 
 // Cluster size for a decode of `group` query heads per KV head over a layer of `tokens`
-// tokens on cache `c`, or 0 for the flat split: bf16 pages, up to 8 query heads, the
-// default split options, and a resident cluster for every head at once.  The default
+// tokens on cache `c`, or 0 for the flat split: up to 8 query heads, the default split
+// options, and a resident cluster for every head at once.  The default
 // kernel takes clusters only when those of the largest size that fits cover at least half
 // of the SMs: with fewer, a head of many pages streams faster through the flat split over
 // every SM.  The size: a layer of at most kClusterShortTokens tokens (at most 16 pages per
@@ -1862,7 +2022,7 @@ cudaError_t prepare_cluster_decode(Cache& c) {
 // size that fits.  The constants were measured on GB300 (152 SMs) on batch-1, 8-head
 // layers from 4K to 64K tokens at 1x to 8x compression.
 int decode_cluster_size(const Cache& c, int group, int64_t tokens) {
-  if (c.fp8() || group > 8 || c.ctas_per_sm >= 2 || c.min_pages_per_cta != 2 ||
+  if (group > 8 || c.ctas_per_sm >= 2 || c.min_pages_per_cta != 2 ||
       (c.decode_kernel != DMS_DECODE_TILED && c.decode_kernel != DMS_DECODE_CLUSTER))
     return 0;
   int largest = 0;
@@ -1928,7 +2088,8 @@ cudaError_t launch_tiled(const DecodeParams& p, int num_sms, int ctas_per_sm, cu
              : cudaLaunchKernelEx(&cfg, decode_tiled_kernel<kStagesOneCta, 2, false>, p);
 }
 
-cudaError_t launch_cluster(const DecodeParams& p, int cluster_size, cudaStream_t stream, bool fused) {
+cudaError_t launch_cluster(const DecodeParams& p, int cluster_size, cudaStream_t stream, bool fused,
+                           bool fp8) {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1942,12 +2103,20 @@ cudaError_t launch_cluster(const DecodeParams& p, int cluster_size, cudaStream_t
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (fused) {
-    cfg.dynamicSmemBytes = cluster_smem_bytes<true>();
-    return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<true>, p);
+  if (fp8) {
+    if (fused) {
+      cfg.dynamicSmemBytes = cluster_smem_bytes<true, true>();
+      return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<true, true>, p);
+    }
+    cfg.dynamicSmemBytes = cluster_smem_bytes<false, true>();
+    return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<false, true>, p);
   }
-  cfg.dynamicSmemBytes = cluster_smem_bytes<false>();
-  return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<false>, p);
+  if (fused) {
+    cfg.dynamicSmemBytes = cluster_smem_bytes<true, false>();
+    return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<true, false>, p);
+  }
+  cfg.dynamicSmemBytes = cluster_smem_bytes<false, false>();
+  return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<false, false>, p);
 }
 
 DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* out, int32_t group,
@@ -1984,7 +2153,7 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
     p.state_ready = 0;
     p.head_flags = c.head_flags + (int64_t)layer * c.heads;
     p.flag_expect = c.flag_valid[layer] ? c.flag_seq[layer] : 0u;
-    return launch_cluster(p, cs, stream, false);
+    return launch_cluster(p, cs, stream, false, c.fp8());
   }
   return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false, c.fp8());
 }
@@ -2022,7 +2191,7 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
     p.head_flags = c.head_flags + (int64_t)layer * c.heads;
     p.flag_expect = c.flag_valid[layer] ? c.flag_seq[layer] : 0u;
     p.flag_publish = next_flag_seq(c.flag_seq[layer]);
-    return launch_cluster(p, cs, stream, true);
+    return launch_cluster(p, cs, stream, true, c.fp8());
   }
   return launch_tiled(p, c.num_sms, 1, stream, true, true, c.fp8());
 }

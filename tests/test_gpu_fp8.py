@@ -51,19 +51,29 @@ def _run(wl, fused=False, codes_every=3, **kw):
         r.close()
 
 
+# fp8 pages are read both by the flat split (the default for these few-head shapes) and by
+# the per-head clusters (DMS_DECODE_CLUSTER; G <= 8)
+KERNELS = pytest.mark.parametrize("kernel", [dms.DMS_DECODE_TILED, dms.DMS_DECODE_CLUSTER],
+                                  ids=["split", "cluster"])
+
+
+@KERNELS
 @pytest.mark.parametrize("w", [0, 1, 16, 63, 64, 256])
-def test_fp8_windows(w):
-    _run(small(window=w, prefill=((333, False),)))
+def test_fp8_windows(w, kernel):
+    _run(small(window=w, prefill=((333, False),)), decode_kernel=kernel)
 
 
+@KERNELS
 @pytest.mark.parametrize("G", [1, 4, 7, 8, 9, 16])
-def test_fp8_gqa_groups(G):
-    _run(small(q_heads=2 * G, decode_steps=4))
+def test_fp8_gqa_groups(G, kernel):
+    _run(small(q_heads=2 * G, decode_steps=4), decode_kernel=kernel)
 
 
+@KERNELS
 @pytest.mark.parametrize("prefill", [1, 15, 16, 17, 63, 64, 65, 129, 1000])
-def test_fp8_page_boundaries(prefill):
-    _run(small(prefill=((prefill, False),), window=20, p_evict=0.5, decode_steps=5))
+def test_fp8_page_boundaries(prefill, kernel):
+    _run(small(prefill=((prefill, False),), window=20, p_evict=0.5, decode_steps=5),
+         decode_kernel=kernel)
 
 
 @pytest.mark.parametrize("p", [0.0, 1.0])
@@ -71,9 +81,34 @@ def test_fp8_no_and_total_eviction(p):
     _run(small(p_evict=p, prefill=((200, False),), window=8))
 
 
-def test_fp8_fused_entry_point():
-    """dms_append_and_decode on an fp8 cache runs the append and the decode as two launches."""
-    _run(small(), fused=True)
+@KERNELS
+def test_fp8_fused_entry_point(kernel):
+    """dms_append_and_decode on an fp8 cache: the single-token append (quantising the new
+    rows) fused into the decode launch."""
+    _run(small(), fused=True, decode_kernel=kernel)
+
+
+@pytest.mark.parametrize("batch,kv_heads,fused", [(1, 1, True), (1, 2, False), (8, 8, True)])
+def test_fp8_cluster_stored_codes(batch, kv_heads, fused):
+    """fp8 pages on per-head clusters (down to 2 CTAs per head for 64 heads) with more pages
+    per CTA than stages and a 2000-token window at P(evict) 0.9, so that new tokens take slots
+    in pages staged early: stored codes and scales bit-exact after the steps, outputs and
+    retained sets against the oracle."""
+    wl = small(batch=batch, kv_heads=kv_heads, q_heads=kv_heads * 5, window=2000,
+               prefill=((4000 if batch > 1 else 8000, False),), decode_steps=30, p_evict=0.9)
+    r = Run(wl, kv_format=FP8, fused=fused, decode_kernel=dms.DMS_DECODE_CLUSTER)
+    try:
+        assert r.cache.decode_plan(wl.gqa_group)["kernel"] == dms.DMS_DECODE_CLUSTER
+        r.prefill()
+        for s in range(wl.decode_steps):
+            q, out = r.step(s)
+            if s % 10 == 9:
+                r.check_outputs(q, out)
+                r.check_retained()
+        r.check_codes()
+        r.summary()
+    finally:
+        r.close()
 
 
 def test_fp8_llama_shape_long():

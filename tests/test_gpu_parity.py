@@ -441,8 +441,8 @@ def test_decode_plan():
     8 CTAs while the layer is short (<= 8192 tokens) and of up to 10 beyond, and for 64
     heads (clusters of 2 on GB300); the flat split for more heads than clusters fit, or for
     few heads whose clusters would cover under half of the SMs; DMS_DECODE_CLUSTER takes
-    clusters whenever every head's cluster fits; G > 8, fp8 pages and the simple kernel
-    never do."""
+    clusters whenever every head's cluster fits (bf16 or fp8 pages); G > 8 and the simple
+    kernel never do."""
     nsm = torch.cuda.get_device_properties(0).multi_processor_count
 
     def plan(B, H, G=5, tokens=0, **kw):
@@ -471,7 +471,7 @@ def test_decode_plan():
     assert plan(1, 2, decode_kernel=dms.DMS_DECODE_CLUSTER) == {
         "kernel": dms.DMS_DECODE_CLUSTER, "ctas": 16, "cluster_size": 8}
     assert plan(1, 8, G=9)["kernel"] == dms.DMS_DECODE_SPLIT
-    assert plan(1, 8, kv_format=dms.DMS_KV_FP8_E4M3)["kernel"] == dms.DMS_DECODE_SPLIT
+    assert plan(1, 8, kv_format=dms.DMS_KV_FP8_E4M3)["kernel"] == dms.DMS_DECODE_CLUSTER
     assert plan(1, 8, decode_kernel=dms.DMS_DECODE_SPLIT)["kernel"] == dms.DMS_DECODE_SPLIT
     assert plan(1, 8, decode_kernel=dms.DMS_DECODE_SIMPLE) == {
         "kernel": dms.DMS_DECODE_SIMPLE, "ctas": 8, "cluster_size": 0}
