@@ -861,9 +861,9 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
 #pragma unroll
         for (int kg = 0; kg < 2; ++kg) {
           const uint4 w0 = *reinterpret_cast<const uint4*>(
-              st + (tb + g) * 128 + (((4 * kg + c4) ^ g) << 4));
+              st + (tb + g) * 128 + (((4 * kg + c4) ^ k8_swizzle(g)) << 4));
           const uint4 w1 = *reinterpret_cast<const uint4*>(
-              st + (tb + g + 8) * 128 + (((4 * kg + c4) ^ g) << 4));
+              st + (tb + g + 8) * 128 + (((4 * kg + c4) ^ k8_swizzle(g)) << 4));
           const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
@@ -1652,9 +1652,9 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           // this thread's codes (d = 16 kk + {2c, 2c+1, 2c+8, 2c+9}) in word kk % 4
 #pragma unroll
           for (int kg = 0; kg < 2; ++kg) {
-            const uint4 w0 = *reinterpret_cast<const uint4*>(st + (tb + g) * 128 + (((4 * kg + c4) ^ g) << 4));
+            const uint4 w0 = *reinterpret_cast<const uint4*>(st + (tb + g) * 128 + (((4 * kg + c4) ^ k8_swizzle(g)) << 4));
             const uint4 w1 =
-                *reinterpret_cast<const uint4*>(st + (tb + g + 8) * 128 + (((4 * kg + c4) ^ g) << 4));
+                *reinterpret_cast<const uint4*>(st + (tb + g + 8) * 128 + (((4 * kg + c4) ^ k8_swizzle(g)) << 4));
             const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
             for (int i = 0; i < 4; ++i) {

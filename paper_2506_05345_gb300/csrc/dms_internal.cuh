@@ -15,7 +15,7 @@
 //               kk / 4 and the four codes one thread needs (d = 16 kk + {2c, 2c+1,
 //               2c+8, 2c+9}) are 4 consecutive bytes; in a V^T row the four codes of
 //               tokens {2c, 2c+1, 2c+8, 2c+9} of a 16-slot block likewise.  16-byte
-//               chunks are XOR-permuted by the row (K: row & 7; V^T: (d >> 1) & 3) so
+//               chunks are XOR-permuted by the row (K: k8_swizzle(row); V^T: (d >> 1) & 3) so
 //               a warp's loads hit distinct banks.  k8_offset / vt8_offset below.
 //   scales      [pool_pages][2][64] fp32         per-slot key and value scales.
 //   pos         [pool_pages][64] int32          position held by each slot (inspection only;
@@ -151,13 +151,19 @@ __host__ __device__ __forceinline__ uint32_t swizzled_offset(uint32_t row, uint3
 // fp8 page format.  Position of logical element d (0..127) of key row `row` (0..63)
 // inside the page: k-step kk = d / 16, j = d % 16; thread c = (j & 7) / 2 of an
 // m16n8k16 fragment needs j = 2c, 2c + 1, 2c + 8, 2c + 9, stored at bytes 0..3 of word
-// kk % 4 of chunk 4 (kk / 4) + c, the chunk XOR-ed with row & 7.
+// kk % 4 of chunk 4 (kk / 4) + c, the chunk XOR-ed with k8_swizzle(row).  A quarter warp
+// of the decode loads chunks 4 kg + c (c = 0..3) of two adjacent rows with 16-byte loads;
+// the swizzle sends those two rows to different halves of the row's 8 chunks (the second
+// term), so the eight loads hit eight different bank groups.
 __host__ __device__ __forceinline__ uint32_t fp8_pair_index(uint32_t j) {
   return (j & 1u) | ((j >> 3) << 1);
 }
+__host__ __device__ __forceinline__ uint32_t k8_swizzle(uint32_t row) {
+  return (row & 7u) ^ ((row & 1u) << 2);
+}
 __host__ __device__ __forceinline__ uint32_t k8_offset(uint32_t row, uint32_t d) {
   const uint32_t kk = d >> 4, j = d & 15u;
-  const uint32_t chunk = (4u * (kk >> 2) + ((j & 7u) >> 1)) ^ (row & 7u);
+  const uint32_t chunk = (4u * (kk >> 2) + ((j & 7u) >> 1)) ^ k8_swizzle(row);
   return row * 128u + (chunk << 4) + 4u * (kk & 3u) + fp8_pair_index(j);
 }
 // Position of the value of slot `slot` (0..63) at head_dim index d in the V^T half:
