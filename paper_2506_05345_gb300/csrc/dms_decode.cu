@@ -1249,6 +1249,10 @@ static_assert(kClusterConsumerWarps * 8 * (kMergeRow + 2) * 4 <=
               kClusterConsumerWarps * 8 * (kMergeRow + 2) * 4 <=
                   cluster_stages<true>() * cluster_stage_bytes(false, true),
               "merge buffers must fit in the stages");
+// The consumers wait on a stage's full barrier by phase parity, which only tells the last
+// completed phase from the one before: a group must never wait for use u + 1 of a stage
+// before use u has completed.  That holds when every use of a stage is read by the same
+// group (in order), i.e. when the stage count is a multiple of the group count.
 static_assert(cluster_stages<false>() % kClusterGroups == 0 &&
               cluster_stages<true>() % kClusterGroups == 0, "a stage is always read by the same group");
 
