@@ -415,6 +415,17 @@ dms_status dms_decode_noalloc_device_error(void* stream, dms_status* out);
 dms_status dms_selftest_noalloc_timeout(int64_t limit_ns, void* stream);
 
 /*
+ * Self-test of the per-head completion flags of the cluster decode kernel (no counterpart
+ * in the paper).  Makes the next cluster launch of `layer` wait, with the limit `limit_ns`
+ * (1 us .. 10 s), for a flag value no launch ever published: each head's wait gives up,
+ * records DMS_ERR_TIMEOUT (sticky, read with dms_cache_stats; cleared by dms_cache_reset)
+ * and falls back to the dependency wait, so that launch still reads the completed state and
+ * computes the right result.  Host only (nothing is launched here).  Errors:
+ * DMS_ERR_INVALID_ARGUMENT (NULL cache, layer out of range, limit out of range).
+ */
+dms_status dms_selftest_stale_flag(dms_cache* cache, int32_t layer, int64_t limit_ns);
+
+/*
  * Self-test of the bounded wait every kernel of this library uses on its
  * shared-memory barriers (the paper has no counterpart: this is failure
  * detection of the implementation).  Launches one small kernel in which a thread

@@ -40,7 +40,7 @@ EXPORTS = (
     "dms_prefill_workspace_bytes", "dms_prefill_attention", "dms_prefill_attention_borrowed",
     "dms_prefill_device_error", "dms_prefill_attention_ex", "dms_append_shared_prefix",
     "dms_cache_export_kv", "dms_decode_noalloc_device_error", "dms_selftest_noalloc_timeout",
-    "dms_decode_plan",
+    "dms_decode_plan", "dms_selftest_stale_flag",
 )
 
 
@@ -108,6 +108,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "dms_cache_layer_length": (st, [vp, i32, ctypes.POINTER(i64)]),
         "dms_decode_plan": (st, [vp, i32, i32, ctypes.POINTER(i32), ctypes.POINTER(i32),
                                  ctypes.POINTER(i32)]),
+        "dms_selftest_stale_flag": (st, [vp, i32, i64]),
         "dms_status_string": (ctypes.c_char_p, [st]),
         "dms_decode_attention_paged_noalloc": (st, [vp, vp, vp, i32, i32, i32, vp, vp, i32, f32,
                                                     vp]),

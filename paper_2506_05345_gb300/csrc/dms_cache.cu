@@ -244,9 +244,12 @@ dms_status decode_impl(dms_cache* h, int32_t layer, const void* q, void* out, in
     e = dms::launch_decode_tiled(c, layer, q, out, gqa_group, scale * 1.4426950408889634f,
                                  zero_first, st);
   if (e != cudaSuccess) return DMS_ERR_CUDA;
+  const bool cluster = c.decode_kernel != DMS_DECODE_SIMPLE &&
+                       dms::decode_cluster_size(c, gqa_group, c.lengths[layer]) > 0;
+  if (cluster && c.flag_test_layer == layer) c.flag_test_layer = -1;  // the self-test ran
   c.last_layer = layer;
   c.last_full_tiled = c.decode_kernel != DMS_DECODE_SIMPLE && dms::tiled_one_cta_per_sm(c) &&
-                      dms::decode_cluster_size(c, gqa_group, c.lengths[layer]) == 0;
+                      !cluster;
   return DMS_OK;
 }
 
@@ -276,6 +279,7 @@ dms_status append_decode_impl(dms_cache* h, int32_t layer, const void* k, const 
   c.flag_valid[layer] = (e == cudaSuccess && cluster) ? 1 : 0;
   if (e != cudaSuccess) return DMS_ERR_CUDA;
   if (cluster) c.flag_seq[layer] = dms::next_flag_seq(c.flag_seq[layer]);
+  if (cluster && c.flag_test_layer == layer) c.flag_test_layer = -1;  // the self-test ran
   c.lengths[layer] = t0 + 1;
   c.last_layer = layer;
   c.last_full_tiled = !cluster;
@@ -486,6 +490,19 @@ dms_status dms_cache_layer_length(const dms_cache* h, int32_t layer, int64_t* ou
   if (h == nullptr || out == nullptr || layer < 0 || layer >= h->c.layers)
     return DMS_ERR_INVALID_ARGUMENT;
   *out = h->c.lengths[layer];
+  return DMS_OK;
+}
+
+dms_status dms_selftest_stale_flag(dms_cache* h, int32_t layer, int64_t limit_ns) {
+  if (h == nullptr || layer < 0 || layer >= h->c.layers || limit_ns < 1000 ||
+      limit_ns > 10000000000LL)
+    return DMS_ERR_INVALID_ARGUMENT;
+  Cache& c = h->c;
+  // a value above every number published so far (they only grow): no launch stores it
+  c.flag_seq[layer] = dms::next_flag_seq(c.flag_seq[layer] + 1000u);
+  c.flag_valid[layer] = 1;
+  c.flag_test_layer = layer;
+  c.flag_test_wait_ns = limit_ns;
   return DMS_OK;
 }
 

@@ -131,6 +131,7 @@ struct DecodeParams {
   // the number this launch publishes (fused; 0: none).
   uint32_t* head_flags;
   uint32_t flag_expect, flag_publish;
+  int64_t flag_wait_ns;  // limit of the wait for a head's flag; 0: kWaitLimitNs
   // Nonzero: attend with element 0 of every group's first query head taken as 0 (that
   // element carries the decision logit, App. B).
   int32_t zero_first;
@@ -1341,10 +1342,12 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       int ok = 1;
       if (lane == 0) {
         const unsigned long long t0 = global_timer_ns();
+        const unsigned long long limit =
+            p.flag_wait_ns > 0 ? (unsigned long long)p.flag_wait_ns : kWaitLimitNs;
         for (uint32_t spin = 1;; ++spin) {
           if (ld_acquire_gpu_u32(p.head_flags + h) == p.flag_expect) break;
           __nanosleep(32);
-          if ((spin & 31u) == 0u && global_timer_ns() - t0 > kWaitLimitNs) {
+          if ((spin & 31u) == 0u && global_timer_ns() - t0 > limit) {
             ok = 0;
             break;
           }
@@ -2157,6 +2160,7 @@ cudaError_t launch_decode_tiled(const Cache& c, int32_t layer, const void* q, vo
     p.state_ready = 0;
     p.head_flags = c.head_flags + (int64_t)layer * c.heads;
     p.flag_expect = c.flag_valid[layer] ? c.flag_seq[layer] : 0u;
+    p.flag_wait_ns = c.flag_test_layer == layer ? c.flag_test_wait_ns : 0;
     return launch_cluster(p, cs, stream, false, c.fp8());
   }
   return launch_tiled(p, c.num_sms, c.ctas_per_sm, stream, true, false, c.fp8());
@@ -2195,6 +2199,7 @@ cudaError_t launch_append_decode(const Cache& c, int32_t layer, const void* k, c
     p.head_flags = c.head_flags + (int64_t)layer * c.heads;
     p.flag_expect = c.flag_valid[layer] ? c.flag_seq[layer] : 0u;
     p.flag_publish = next_flag_seq(c.flag_seq[layer]);
+    p.flag_wait_ns = c.flag_test_layer == layer ? c.flag_test_wait_ns : 0;
     return launch_cluster(p, cs, stream, true, c.fp8());
   }
   return launch_tiled(p, c.num_sms, 1, stream, true, true, c.fp8());

@@ -119,6 +119,9 @@ struct Cache {
   uint32_t* head_flags = nullptr;  // device [layers][heads]
   uint32_t* flag_seq = nullptr;    // host [layers]
   uint8_t* flag_valid = nullptr;   // host [layers]
+  // Self-test: the wait limit (ns) of the next cluster launch of layer flag_test_layer (0: none).
+  int64_t flag_test_wait_ns = 0;
+  int32_t flag_test_layer = -1;
 
   // Count buffer of `layer` for a layer length of parity `parity`.
   int32_t* counts_at(int32_t layer, int64_t parity) const {

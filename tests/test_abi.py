@@ -74,6 +74,7 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert lib.dms_append_and_evict(None, 0, None, None, None, 1, None) == 1
     assert lib.dms_decode_attention(None, 0, None, None, 4, 0.0, None) == 1
     assert lib.dms_decode_plan(None, 0, 4, None, None, None) == 1
+    assert lib.dms_selftest_stale_flag(None, 0, 2000000) == 1
 
 
 def test_kv_format_options_checked_on_host(lib):

@@ -55,3 +55,34 @@ def test_bounded_wait_times_out_and_context_survives():
 
 def test_selftest_rejects_bad_limits():
     assert dms.dms_selftest_bounded_wait(0, 10, _stream()) == dms.DMS_ERR_INVALID_ARGUMENT
+
+
+def test_cluster_flag_wait_times_out_and_falls_back():
+    """A cluster launch whose head flags never arrive (the self-test makes it wait for a value
+    no launch publishes, 2 ms limit): every head's wait gives up, DMS_ERR_TIMEOUT is recorded,
+    the launch falls back to the dependency wait and still computes the oracle's result; the
+    next launches run normally, and a reset clears the sticky error."""
+    import _harness
+    import workloads
+    wl = workloads.Workload(name="stale-flag", batch=1, layers=1, q_heads=20, kv_heads=4,
+                            window=32, prefill=((600, False),), decode_steps=8, p_evict=0.6)
+    r = _harness.Run(wl, fused=True, decode_kernel=dms.DMS_DECODE_CLUSTER)
+    try:
+        assert r.cache.decode_plan(wl.gqa_group)["kernel"] == dms.DMS_DECODE_CLUSTER
+        r.prefill()
+        for s in range(2):  # the layer's state is now last written by flag-publishing launches
+            q, out = r.step(s)
+            r.check_outputs(q, out)
+        assert r.cache.stats()["device_error"] == 0
+        code = dms.library().dms_selftest_stale_flag(ctypes.c_void_p(r.cache.handle), 0, 2_000_000)
+        assert code == dms.DMS_OK
+        q, out = r.step(2)
+        r.check_outputs(q, out)  # the fallback read the completed state
+        assert r.cache.stats()["device_error"] == dms.DMS_ERR_TIMEOUT
+        for s in range(3, 6):
+            q, out = r.step(s)
+            r.check_outputs(q, out)
+        r.cache.reset()
+        assert r.cache.stats()["device_error"] == 0
+    finally:
+        r.close()
