@@ -71,20 +71,20 @@ enum {
 enum {
   DMS_DECODE_TILED = 0,   /* default: TMA-staged tensor-core kernels; as
                              DMS_DECODE_CLUSTER when clusters of the largest size
-                             in [2, 16] that fits for every head would cover at
+                             in [1, 16] that fits for every head would cover at
                              least half of the SMs, else as DMS_DECODE_SPLIT       */
   DMS_DECODE_SIMPLE = 1,  /* one CTA per KV head, CUDA cores; a cross-check path     */
   DMS_DECODE_SPLIT = 2,   /* the tiled kernel with the flat, page-balanced split-K of
                              all heads' pages over all SMs, for every batch          */
   DMS_DECODE_CLUSTER = 3  /* per-head thread-block clusters: when bf16 pages, G <= 8,
                              the default ctas_per_sm / min_pages_per_cta, and a
-                             resident cluster of at least 2 CTAs for every (sequence,
-                             KV head) at once (up to a few dozen heads), each head's
-                             pages are split over its own cluster of C CTAs and
-                             merged in distributed shared memory, C = 8 for layers
-                             of up to 8192 tokens, else 10, or the largest size in
-                             [2, 16] that fits if smaller; otherwise as
-                             DMS_DECODE_SPLIT                                        */
+                             resident cluster for every (sequence, KV head) at once
+                             (up to one head per SM), each head's pages are split
+                             over its own cluster of C CTAs and merged in
+                             distributed shared memory, C = 8 for layers of up to
+                             8192 tokens, else 10, or the largest size in [1, 16]
+                             that fits if smaller (1: one CTA takes the whole head);
+                             otherwise as DMS_DECODE_SPLIT                           */
 };
 
 /*

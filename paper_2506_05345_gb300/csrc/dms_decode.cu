@@ -1221,7 +1221,7 @@ constexpr int kClusterThreads = (kClusterConsumerWarps + 1) * 32;  // + a produc
 template <bool kFp8>
 __host__ __device__ constexpr int cluster_stages() { return kFp8 ? 12 : 6; }
 constexpr int kClusterMaxSize = 16;
-constexpr int kClusterMinSize = 2;
+constexpr int kClusterMinSize = 1;  // a cluster of one CTA: the head's pages, no merge
 constexpr int kClusterShortSize = 8;
 constexpr int kClusterLongSize = 10;
 constexpr int64_t kClusterShortTokens = 8192;
@@ -1233,7 +1233,7 @@ __host__ __device__ constexpr int cluster_stage_bytes(bool fused, bool fp8) {
 
 // Partials received from every CTA of the cluster for the query-head rows this CTA owns
 // (rows r with r % C == rank: at most ceil(8 / C) rows, ceil(8 / C) C <= 16 partials for
-// every C in [2, 16]): O, then (m, l).
+// every C in [1, 16]): O, then (m, l).
 constexpr int kClusterRecvSlots = 16;
 constexpr int kClusterRecvBytes = kClusterRecvSlots * (kHeadDim + 2) * 4;
 

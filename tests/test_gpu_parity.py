@@ -105,9 +105,9 @@ def test_fused_decode_from_empty_cache(w, kernel):
 @pytest.mark.parametrize("fused", [False, True])
 @pytest.mark.parametrize("batch,kv_heads,G,prefill", [
     (1, 1, 5, 5000), (1, 8, 5, 20000), (2, 8, 5, 3000), (1, 16, 5, 700), (3, 6, 5, 1500),
-    (5, 8, 5, 1200), (8, 8, 8, 900), (8, 8, 3, 9000)])
+    (5, 8, 5, 1200), (8, 8, 8, 900), (8, 8, 3, 9000), (16, 8, 5, 700), (12, 8, 8, 2500)])
 def test_cluster_shapes(batch, kv_heads, G, prefill, fused):
-    """Head counts over the cluster sizes' range (1 to 64 heads: clusters of 16 CTAs down to 2),
+    """Head counts over the cluster sizes' range (1 to 128 heads: clusters of 16 CTAs down to 1),
     with heads of many pages (5000 and 20000 tokens at P(evict) 0.2: up to 250 pages over a
     cluster) and of few (a head of 700 tokens leaves most of its cluster's CTAs without
     pages), and clusters smaller than the group (40 heads of G = 5 and 64 heads of G = 8,
@@ -437,12 +437,12 @@ def test_cluster_early_start_across_mixed_calls():
 
 
 def test_decode_plan():
-    """Which kernel runs: the default takes per-head clusters for a batch-1 8-head cache, of
-    8 CTAs while the layer is short (<= 8192 tokens) and of up to 10 beyond, and for 64
-    heads (clusters of 2 on GB300); the flat split for more heads than clusters fit, or for
-    few heads whose clusters would cover under half of the SMs; DMS_DECODE_CLUSTER takes
-    clusters whenever every head's cluster fits (bf16 or fp8 pages); G > 8 and the simple
-    kernel never do."""
+    """Which kernel runs: the default takes per-head clusters for a batch-1 8-head cache (8
+    CTAs each while the layer is short, <= 8192 tokens, up to 10 beyond), for 64 heads
+    (clusters of 2 on GB300) and for 128 (one CTA per head); the flat split for more heads
+    than SMs, or for few heads whose clusters would cover under half of the SMs.
+    DMS_DECODE_CLUSTER takes clusters whenever every head's cluster fits (bf16 or fp8
+    pages); G > 8 and the simple kernel never do."""
     nsm = torch.cuda.get_device_properties(0).multi_processor_count
 
     def plan(B, H, G=5, tokens=0, **kw):
@@ -466,7 +466,11 @@ def test_decode_plan():
     assert p["kernel"] == dms.DMS_DECODE_CLUSTER and p["cluster_size"] >= 2
     if nsm == 152:
         assert p == {"kernel": dms.DMS_DECODE_CLUSTER, "ctas": 128, "cluster_size": 2}
-    assert plan(16, 8)["kernel"] == dms.DMS_DECODE_SPLIT  # 128 heads: no cluster fits each
+    p = plan(16, 8)  # 128 heads: one CTA per head
+    assert p["kernel"] == dms.DMS_DECODE_CLUSTER and p["ctas"] == 128 * p["cluster_size"]
+    if nsm == 152:
+        assert p["cluster_size"] == 1
+    assert plan(32, 8)["kernel"] == dms.DMS_DECODE_SPLIT  # 256 heads: more than SMs
     assert plan(1, 2)["kernel"] == dms.DMS_DECODE_SPLIT
     assert plan(1, 2, decode_kernel=dms.DMS_DECODE_CLUSTER) == {
         "kernel": dms.DMS_DECODE_CLUSTER, "ctas": 16, "cluster_size": 8}
