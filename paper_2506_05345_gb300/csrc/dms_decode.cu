@@ -1419,14 +1419,35 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       }
       patch_page = __shfl_sync(0xffffffffu, patch_page, 0);
     }
-    // After the dependency wait: the query rows and a pending patch; and (fused, the CTA of
-    // the new row's page) the new K and V rows into the pool (from the inputs), the
-    // position, the head's new count and ring entry.  The layer's state of this head is
-    // then complete and this launch's flag for the head is published.  (A later launch
-    // writes this state only after its dependency wait, when this grid has completed, so
-    // the flag need not wait for this launch's page reads; and this launch's consumer warps
-    // take the new row from their own copy of it, whatever the bulk copy of the page read.)
+    // After the dependency wait: the query rows and a pending patch.  Then (fused, the CTA
+    // of the new row's page, write_new_row) the new K and V rows into the pool (from the
+    // inputs), the position, the head's new count and ring entry: the layer's state of this
+    // head is then complete and this launch's flag for the head is published.  (A later
+    // launch writes this state only after its dependency wait, when this grid has
+    // completed, so the flag need not wait for this launch's page reads; and this launch's
+    // consumer warps take the new row from their own copy of it, whatever the bulk copy of
+    // the page read.)
     auto after_wait = [&]() {
+      if (lane == 0) {
+        if (niters > 0) {
+          mbar_arrive_expect_tx(q_bar, (uint32_t)G * kRowBytes);
+          const __nv_bfloat16* qs = q_src + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
+          for (int i = 0; i < G; ++i)
+            bulk_copy_g2s(q_buf + i * kQRowPadded, qs + (int64_t)i * kHeadDim, kRowBytes, q_bar);
+        }
+        if (kFused && patch_stage >= 0) {
+          uint8_t* st = stages + patch_stage * kStageBytes;
+          bulk_copy_g2s(st + kOffPatch, k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[patch_stage]);
+          bulk_copy_g2s(st + kOffPatch + kRowBytes, v_new + (int64_t)h * kHeadDim, kRowBytes,
+                        &full_bar[patch_stage]);
+        }
+      }
+      __syncwarp();
+    };
+    // Fused, the CTA of the new row's page, once the dependency wait is behind it and its
+    // first pages are in flight: the new row and the head's state, then the flag.
+    bool row_done = !(kFused && patch_cta);
+    auto write_new_row = [&]() {
       if (kFused && patch_cta) {
         const uint32_t r = (uint32_t)(new_slot % kPageTokens);
         if constexpr (kFp8) {  // quantise both rows (lane: head_dim 4 lane .. 4 lane + 3)
@@ -1477,21 +1498,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         __syncwarp();
         if (lane == 0 && flag_publish != 0u) st_release_gpu_u32(p.head_flags + h, flag_publish);
       }
-      if (lane == 0) {
-        if (niters > 0) {
-          mbar_arrive_expect_tx(q_bar, (uint32_t)G * kRowBytes);
-          const __nv_bfloat16* qs = q_src + ((int64_t)b * Hq + (int64_t)hk * G) * kHeadDim;
-          for (int i = 0; i < G; ++i)
-            bulk_copy_g2s(q_buf + i * kQRowPadded, qs + (int64_t)i * kHeadDim, kRowBytes, q_bar);
-        }
-        if (kFused && patch_stage >= 0) {
-          uint8_t* st = stages + patch_stage * kStageBytes;
-          bulk_copy_g2s(st + kOffPatch, k_new + (int64_t)h * kHeadDim, kRowBytes, &full_bar[patch_stage]);
-          bulk_copy_g2s(st + kOffPatch + kRowBytes, v_new + (int64_t)h * kHeadDim, kRowBytes,
-                        &full_bar[patch_stage]);
-        }
-      }
-      __syncwarp();
+      row_done = true;
     };
     if (waited) after_wait();
     const int first = niters < kClusterStages ? niters : kClusterStages;  // staged before the wait
@@ -1553,6 +1560,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           patch_stage = __shfl_sync(0xffffffffu, patch_stage, 0);
           after_wait();
         }
+        if (!row_done && itg + 1 >= first) write_new_row();
       }
     }
     if (!waited) {  // a CTA without pages
@@ -1560,6 +1568,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       waited = true;
       after_wait();
     }
+    if (!row_done) write_new_row();
     // Drain: do not leave while a bulk copy may still be writing shared memory.
     if (lane == 0) {
       for (int s = 0; s < kClusterStages && s < niters; ++s) {
