@@ -81,7 +81,7 @@ enum {
                              resident cluster for every (sequence, KV head) at once
                              (up to one head per SM), each head's pages are split
                              over its own cluster of C CTAs and merged in
-                             distributed shared memory, C = 8 for layers of up to
+                             distributed shared memory, C = 6 for layers of up to
                              8192 tokens, else 10, or the largest size in [1, 16]
                              that fits if smaller (1: one CTA takes the whole head);
                              otherwise as DMS_DECODE_SPLIT                           */

@@ -1193,9 +1193,10 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
 // costs global round trips (an arrival atomic, then the records).  Instead a
 // thread-block cluster of C CTAs takes each head: CTA r of the cluster streams the
 // head's pages r, r + C, r + 2C, ... exactly as a tiled CTA streams one segment and
-// stores its partial (m, l, O) of each query-head row i into the shared memory of CTA i
-// of the cluster (distributed shared memory); after one cluster barrier CTA i merges
-// row i over the C partials in rank order (deterministic) and writes it.
+// stores its partial (m, l, O) of each query-head row i into the shared memory of CTA
+// i mod C of the cluster (asynchronous distributed-shared-memory stores counted on that
+// CTA's mbarrier); once its rows' partials have landed, that CTA merges each row over the
+// C partials in rank order (deterministic) and writes it.
 //
 // Early start.  The layer's state (count, ring, page table, pages) changes only in
 // launches that append to this layer.  A fused cluster launch publishes, per head, a
@@ -1222,7 +1223,7 @@ template <bool kFp8>
 __host__ __device__ constexpr int cluster_stages() { return kFp8 ? 12 : 6; }
 constexpr int kClusterMaxSize = 16;
 constexpr int kClusterMinSize = 1;  // a cluster of one CTA: the head's pages, no merge
-constexpr int kClusterShortSize = 8;
+constexpr int kClusterShortSize = 6;
 constexpr int kClusterLongSize = 10;
 constexpr int64_t kClusterShortTokens = 8192;
 constexpr int kClusterQBytes = 8 * kQRowPadded;  // up to 8 query heads, padded rows
@@ -1240,7 +1241,7 @@ constexpr int kClusterRecvBytes = kClusterRecvSlots * (kHeadDim + 2) * 4;
 template <bool kFused, bool kFp8>
 size_t cluster_smem_bytes() {
   return (size_t)cluster_stages<kFp8>() * cluster_stage_bytes(kFused, kFp8) + kClusterQBytes +
-         kClusterRecvBytes + (size_t)(2 * cluster_stages<kFp8>() + 1) * sizeof(uint64_t) +
+         kClusterRecvBytes + (size_t)(2 * cluster_stages<kFp8>() + 2) * sizeof(uint64_t) +
          16 * sizeof(int);
 }
 
@@ -1298,7 +1299,8 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   uint64_t* empty_bar = full_bar + kClusterStages;
   uint64_t* q_bar = empty_bar + kClusterStages;
   // [0] abort, [1] count after the append, [2] new slot | fresh << 30
-  int* s_misc = reinterpret_cast<int*>(q_bar + 1);
+  uint64_t* recv_bar = q_bar + 1;  // the partials of this CTA's rows have landed
+  int* s_misc = reinterpret_cast<int*>(recv_bar + 1);
   float* merge_o = reinterpret_cast<float*>(smem);                    // [8][HP][132]
   float* merge_ml = merge_o + kClusterConsumerWarps * HP * kMergeRow;  // [8][HP][2]
 
@@ -1331,9 +1333,16 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       mbar_init(&empty_bar[s], kClusterConsumerWarps / kClusterGroups);
     }
     mbar_init(q_bar, 1);
+    mbar_init(recv_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    // Query-head rows r = rank, rank + C, ... (< G) are this CTA's: C partials of 520 bytes
+    // each arrive for every one of them.
+    const int own = G > rank ? (G - 1 - rank) / C + 1 : 0;
+    if (own > 0 && C > 1) mbar_arrive_expect_tx(recv_bar, (uint32_t)(own * C * (kHeadDim + 2) * 4));
   }
-  cluster_arrive_relaxed();  // waited for before the first store into another CTA
+  // Waited for before the first store into another CTA: that CTA runs, and its receive
+  // barrier is initialised and expects its bytes (release / acquire).
+  cluster_arrive_release();
   bool waited = false;  // producer warp: the dependency wait is behind it
   int32_t spec_page = -1;
   if (warp == kClusterConsumerWarps) {
@@ -1833,18 +1842,26 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           O.z += a * x.z;
           O.w += a * x.w;
         }
-        const int slot = (r / C) * C + rank;
-        const uint32_t owner = (uint32_t)(r % C);
-        st_shared_cluster_v4(mapa_shared(smem_addr(recv_o + slot * kHeadDim + d4), owner), O);
-        if (lane == 0) st_shared_cluster_v2(mapa_shared(smem_addr(recv_ml + slot * 2), owner), M, L);
+        if (C == 1) {  // the CTA holds the whole head: its partial is the result
+          const float inv = L > 0.f ? 1.f / L : 0.f;  // an empty head gives zeros
+          store_bf16x4(out + ((int64_t)b * Hq + (int64_t)hk * G + r) * kHeadDim + d4, O.x * inv,
+                       O.y * inv, O.z * inv, O.w * inv);
+        } else {
+          const int slot = (r / C) * C + rank;
+          const uint32_t owner = (uint32_t)(r % C);
+          const uint32_t rbar = mapa_shared(smem_addr(recv_bar), owner);
+          st_async_cluster_v4(mapa_shared(smem_addr(recv_o + slot * kHeadDim + d4), owner), O, rbar);
+          if (lane == 0)
+            st_async_cluster_v2(mapa_shared(smem_addr(recv_ml + slot * 2), owner), M, L, rbar);
+        }
       }
     }
   }
-  // ---- every CTA's partials are in their owners' shared memory (no CTA touches another's
-  // shared memory after this barrier)
-  cluster_sync();
-  // CTA `rank` merges its rows r = li C + rank (warp li) over the cluster, in rank order
-  if (warp * C + rank < G) {
+  // ---- CTA `rank` merges its rows r = li C + rank (warp li) over the cluster, in rank
+  // order, once every CTA's partials of them have landed (no barrier across the cluster: a
+  // CTA without rows leaves, and no CTA's shared memory is written after its rows are in)
+  if (C > 1 && warp * C + rank < G) {
+    mbar_wait(recv_bar, 0, abort_flag, p.ctrl);
     const int li = warp, r = li * C + rank, d4 = 4 * lane;
     const float* rml = recv_ml + li * C * 2;
     const float* ro = recv_o + li * C * kHeadDim;
@@ -2030,8 +2047,8 @@ cudaError_t prepare_cluster_decode(Cache& c) {
 // options, and a resident cluster for every head at once.  The default
 // kernel takes clusters only when those of the largest size that fits cover at least half
 // of the SMs: with fewer, a head of many pages streams faster through the flat split over
-// every SM.  The size: a layer of at most kClusterShortTokens tokens (at most 16 pages per
-// CTA at size 8 even if nothing was evicted) takes kClusterShortSize, small enough that
+// every SM.  The size: a layer of at most kClusterShortTokens tokens (at most 22 pages per
+// CTA at size 6 even if nothing was evicted) takes kClusterShortSize, small enough that
 // the clusters of consecutive launches fit on the device side by side, so that each
 // launch stages its pages while the one before runs; a longer layer takes
 // kClusterLongSize, which spreads its pages over more SMs; either is capped by the largest

@@ -437,7 +437,7 @@ def test_cluster_early_start_across_mixed_calls():
 
 
 def test_decode_plan():
-    """Which kernel runs: the default takes per-head clusters for a batch-1 8-head cache (8
+    """Which kernel runs: the default takes per-head clusters for a batch-1 8-head cache (6
     CTAs each while the layer is short, <= 8192 tokens, up to 10 beyond), for 64 heads
     (clusters of 2 on GB300) and for 128 (one CTA per head); the flat split for more heads
     than SMs, or for few heads whose clusters would cover under half of the SMs.
@@ -455,10 +455,10 @@ def test_decode_plan():
                 c.append_and_evict(0, k, k, lg)
             return c.decode_plan(G)
 
-    assert plan(1, 8) == {"kernel": dms.DMS_DECODE_CLUSTER, "ctas": 64, "cluster_size": 8}
-    assert plan(1, 8, tokens=8191)["cluster_size"] == 8   # the next step reads 8192 tokens
+    assert plan(1, 8) == {"kernel": dms.DMS_DECODE_CLUSTER, "ctas": 48, "cluster_size": 6}
+    assert plan(1, 8, tokens=8191)["cluster_size"] == 6   # the next step reads 8192 tokens
     p = plan(1, 8, tokens=8192)
-    assert p["kernel"] == dms.DMS_DECODE_CLUSTER and 8 <= p["cluster_size"] <= 10
+    assert p["kernel"] == dms.DMS_DECODE_CLUSTER and 6 <= p["cluster_size"] <= 10
     assert p["ctas"] == 8 * p["cluster_size"]
     if nsm == 152:
         assert p["cluster_size"] == 10
@@ -473,7 +473,7 @@ def test_decode_plan():
     assert plan(32, 8)["kernel"] == dms.DMS_DECODE_SPLIT  # 256 heads: more than SMs
     assert plan(1, 2)["kernel"] == dms.DMS_DECODE_SPLIT
     assert plan(1, 2, decode_kernel=dms.DMS_DECODE_CLUSTER) == {
-        "kernel": dms.DMS_DECODE_CLUSTER, "ctas": 16, "cluster_size": 8}
+        "kernel": dms.DMS_DECODE_CLUSTER, "ctas": 12, "cluster_size": 6}
     assert plan(1, 8, G=9)["kernel"] == dms.DMS_DECODE_SPLIT
     assert plan(1, 8, kv_format=dms.DMS_KV_FP8_E4M3)["kernel"] == dms.DMS_DECODE_CLUSTER
     assert plan(1, 8, decode_kernel=dms.DMS_DECODE_SPLIT)["kernel"] == dms.DMS_DECODE_SPLIT
