@@ -99,8 +99,9 @@ enum {
                           no infinities, largest finite 448) with one fp32 scale per
                           row and tensor: scale = amax(|row|) / 448 (fp32 division),
                           code = E4M3(row / scale) rounded to nearest even and
-                          saturated; a row of zeros has scale 0.  Pages of 16 KiB
-                          (+ 512 bytes of scales).  Rows must be finite.  Read by
+                          saturated; a row of zeros has scale 0.  Pages of 16.5
+                          KiB: K codes, V^T codes, then the 128 row scales (one
+                          bulk copy each).  Rows must be finite.  Read by
                           the tiled kernels (the flat split and the per-head
                           clusters), not by DMS_DECODE_SIMPLE; the single-token
                           append + decode runs in one launch.                        */

@@ -23,7 +23,6 @@ __device__ __forceinline__ void pdl_wait_prerequisites() {
 
 struct AppendParams {
   uint8_t* pool;
-  float* scales;        // fp8 format: [pool_pages][2][64]
   int32_t fp8;          // the cache's pages hold fp8 E4M3 rows
   int32_t* pos;
   int32_t* page_table;  // this layer: [heads][max_pages]
@@ -58,9 +57,10 @@ __device__ __forceinline__ void store_row(uint8_t* pool, int32_t page, uint32_t 
 // chunk l = lane & 15) and V row (lanes 16-31) are quantised with one scale per row,
 // scale = amax / 448 (IEEE fp32 division), code = E4M3(x / scale), round to nearest
 // even, saturated; a row of zeros gets scale 0 and zero codes.  K codes go to the
-// K rows of the page, V codes to the slot's column of V^T (k8_offset / vt8_offset).
-__device__ __forceinline__ void store_row_fp8(uint8_t* pool, float* scales, int32_t page,
-                                              uint32_t row, int lane, uint4 val) {
+// K rows of the page, V codes to the slot's column of V^T (k8_offset / vt8_offset),
+// the two scales to the page's scale words (page_scales_fp8).
+__device__ __forceinline__ void store_row_fp8(uint8_t* pool, int32_t page, uint32_t row, int lane,
+                                              uint4 val) {
   const uint32_t w[4] = {val.x, val.y, val.z, val.w};
   float x[8];
 #pragma unroll
@@ -91,14 +91,14 @@ __device__ __forceinline__ void store_row_fp8(uint8_t* pool, float* scales, int3
       pg[vt8_offset(row, d + 1)] = (uint8_t)(pair >> 8);
     }
   }
-  if ((lane & 15) == 0) scales[(int64_t)page * 2 * kPageTokens + (lane >= 16 ? kPageTokens : 0) + row] = scale;
+  if ((lane & 15) == 0) page_scales_fp8(pool, page)[(lane >= 16 ? kPageTokens : 0) + row] = scale;
 }
 
 // One K and V row into `row` of `page` in the cache's format (the whole warp calls it).
 __device__ __forceinline__ void store_kv_row(const AppendParams& p, int32_t page, uint32_t row,
                                              int lane, uint4 val) {
   if (p.fp8)
-    store_row_fp8(p.pool, p.scales, page, row, lane, val);
+    store_row_fp8(p.pool, page, row, lane, val);
   else
     store_row(p.pool, page, row, lane, val);
 }
@@ -373,9 +373,6 @@ __global__ void __launch_bounds__(256) share_prefix_kernel(const AppendParams p)
     const uint4* a = reinterpret_cast<const uint4*>(p.pool + (int64_t)from * page_bytes);
     uint4* c = reinterpret_cast<uint4*>(p.pool + (int64_t)to * page_bytes);
     for (int e = tid; e < page_bytes / 16; e += blockDim.x) c[e] = a[e];
-    if (p.fp8)
-      for (int e = tid; e < 2 * kPageTokens; e += blockDim.x)
-        p.scales[(int64_t)to * 2 * kPageTokens + e] = p.scales[(int64_t)from * 2 * kPageTokens + e];
     for (int e = tid; e < kPageTokens; e += blockDim.x)
       p.pos[(int64_t)to * kPageTokens + e] = p.pos[(int64_t)from * kPageTokens + e];
   }
@@ -402,7 +399,6 @@ AppendParams make_params(const Cache& c, int32_t layer, const void* k, const voi
                          const void* logit, int64_t logit_stride, int64_t t0, int32_t n) {
   AppendParams p;
   p.pool = c.pool;
-  p.scales = c.scales;
   p.fp8 = c.fp8() ? 1 : 0;
   p.pos = c.pos;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;

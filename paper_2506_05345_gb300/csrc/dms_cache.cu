@@ -22,8 +22,6 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 void free_device(Cache& c) {
   cudaFree(c.pool);
-  cudaFree(c.scales);
-  c.scales = nullptr;
   cudaFree(c.pos);
   cudaFree(c.page_table);
   cudaFree(c.counts);
@@ -134,8 +132,6 @@ dms_status dms_cache_create(int32_t layers, int32_t kv_heads, int32_t head_dim, 
 
   cudaError_t e = cudaSuccess;
   if (e == cudaSuccess) e = alloc(&c.pool, (size_t)c.pool_pages * (size_t)c.page_bytes());
-  if (e == cudaSuccess && c.fp8())
-    e = alloc(&c.scales, (size_t)c.pool_pages * 2 * dms::kPageTokens);
   if (e == cudaSuccess) e = alloc(&c.pos, (size_t)c.pool_pages * dms::kPageTokens);
   if (e == cudaSuccess) e = alloc(&c.page_table, (size_t)layers * heads * c.max_pages);
   if (e == cudaSuccess) e = alloc(&c.counts, (size_t)layers * 2 * heads);
@@ -429,7 +425,6 @@ dms_status dms_cache_export_kv(dms_cache* h, int32_t layer, void* host_k, void* 
   memset(host_v, 0, (size_t)heads * cap * D * esize);
   if (c.fp8()) memset(host_scales, 0, (size_t)heads * cap * 2 * sizeof(float));
   std::vector<uint8_t> page((size_t)c.page_bytes());
-  float sc[2 * dms::kPageTokens];
   for (int64_t bh = 0; bh < heads; ++bh) {
     const int32_t n = cnt[(size_t)bh];
     if (n < 0 || n > cap) return DMS_ERR_STATE;
@@ -437,10 +432,10 @@ dms_status dms_cache_export_kv(dms_cache* h, int32_t layer, void* host_k, void* 
       const int32_t id = pt[(size_t)bh * c.max_pages + pg];
       if (id < 0 || id >= c.pool_pages) return DMS_ERR_STATE;
       if (cudaMemcpy(page.data(), c.pool + (int64_t)id * c.page_bytes(), page.size(),
-                     cudaMemcpyDeviceToHost) != cudaSuccess ||
-          (c.fp8() && cudaMemcpy(sc, c.scales + (int64_t)id * 2 * dms::kPageTokens, sizeof(sc),
-                                 cudaMemcpyDeviceToHost) != cudaSuccess))
+                     cudaMemcpyDeviceToHost) != cudaSuccess)
         return DMS_ERR_CUDA;
+      float sc[2 * dms::kPageTokens];  // fp8: the page's key and value row scales
+      if (c.fp8()) memcpy(sc, page.data() + dms::kPageCodesBytesFp8, sizeof(sc));
       for (int32_t r = 0; r < dms::kPageTokens && pg * dms::kPageTokens + r < n; ++r) {
         const int64_t slot = (int64_t)pg * dms::kPageTokens + r;
         const size_t row = ((size_t)bh * cap + slot) * D;

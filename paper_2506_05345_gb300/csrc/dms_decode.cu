@@ -94,7 +94,6 @@ struct Plan {
 
 struct DecodeParams {
   uint8_t* pool;
-  float* scales;              // fp8 pages: [pool_pages][2][64] key / value row scales
   int32_t* page_table;        // this layer
   const int32_t* counts;      // this layer, current buffer
   const __nv_bfloat16* q;
@@ -244,8 +243,8 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
   constexpr int HP = PL::kHeadsPad;
   constexpr int kStageBytes = stage_bytes(kFused, kFp8);
   constexpr int kKvHalf = kv_half_bytes(kFp8);     // offset of the V half in a stage
-  constexpr int kOffQ = 2 * kKvHalf;                // the group's queries
-  constexpr int kOffScales = kOffQ + kQBytes;       // fp8: key scales [64], value scales [64]
+  constexpr int kOffScales = 2 * kKvHalf;           // fp8: key scales [64], value scales [64]
+  constexpr int kOffQ = kOffScales + (kFp8 ? kScaleBytes : 0);  // the group's queries
   constexpr int kOffPatch = kFp8 ? kStageBytesFp8 : kStageBytesPlain;  // fused: new K, V rows
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* stages = smem;
@@ -512,15 +511,14 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
           }
           const int64_t page0 = page_i < 0 ? 0 : page_i;
           if constexpr (kFp8) {
-            // valid K rows; all of V^T (its rows interleave the slots) and the scales
-            mbar_arrive_expect_tx(&full_bar[s], kv_bytes + (uint32_t)kHalfPageBytesFp8 +
-                                                    (uint32_t)kScaleBytes + q_bytes +
+            // the whole page (K codes, V^T codes, row scales) in one copy: K rows past n_valid
+            // are masked like stale ones, and all of V^T is needed (its rows interleave the
+            // slots)
+            static_assert(kKvHalf == kHalfPageBytesFp8 && kOffScales == kPageCodesBytesFp8,
+                          "a stage holds the page as laid out in the pool");
+            mbar_arrive_expect_tx(&full_bar[s], (uint32_t)kPageBytesFp8 + q_bytes +
                                                     (patch ? (uint32_t)kPatchBytes : 0u));
-            const uint8_t* src = p.pool + page0 * kPageBytesFp8;
-            bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
-            bulk_copy_g2s(st + kKvHalf, src + kHalfPageBytesFp8, kHalfPageBytesFp8, &full_bar[s]);
-            bulk_copy_g2s(st + kOffScales, p.scales + page0 * 2 * kPageTokens, kScaleBytes,
-                          &full_bar[s]);
+            bulk_copy_g2s(st, p.pool + page0 * kPageBytesFp8, kPageBytesFp8, &full_bar[s]);
           } else {
             mbar_arrive_expect_tx(&full_bar[s],
                                   2 * kv_bytes + q_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
@@ -787,7 +785,7 @@ __global__ void __launch_bounds__(kThreads, kStages == kStagesTwoCta ? 2 : 1)
           if (lane == 0) {
             reinterpret_cast<float*>(st + kOffScales)[kv * kPageTokens + r] = scale;
             if (page >= 0)
-              p.scales[(int64_t)page * 2 * kPageTokens + kv * kPageTokens + r] = scale;
+              page_scales_fp8(p.pool, page)[kv * kPageTokens + r] = scale;
           }
         }
         if (page >= 0 && lane == 0) p.pos[(int64_t)page * kPageTokens + r] = (int32_t)p.j;
@@ -1344,36 +1342,38 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
   // barrier is initialised and expects its bytes (release / acquire).
   cluster_arrive_release();
   bool waited = false;  // producer warp: the dependency wait is behind it
-  int32_t spec_page = -1;
+  int32_t spec_page = -1, spec_page2 = -1;  // producer: page ids of its pages lane, lane + 32
   if (warp == kClusterConsumerWarps) {
     bool early = p.flag_expect != 0u;
     if (early) {
       int ok = 1;
-      if (lane == 0) {
+      if (lane == 0 && ld_acquire_gpu_u32(p.head_flags + h) != p.flag_expect) {
+        // Not yet published (the timer is read only here: it costs a round trip).
         const unsigned long long t0 = global_timer_ns();
         const unsigned long long limit =
             p.flag_wait_ns > 0 ? (unsigned long long)p.flag_wait_ns : kWaitLimitNs;
         for (uint32_t spin = 1;; ++spin) {
-          if (ld_acquire_gpu_u32(p.head_flags + h) == p.flag_expect) break;
           __nanosleep(32);
+          if (ld_acquire_gpu_u32(p.head_flags + h) == p.flag_expect) break;
           if ((spin & 31u) == 0u && global_timer_ns() - t0 > limit) {
             ok = 0;
             break;
           }
         }
         if (!ok) set_device_error(p.ctrl, DMS_ERR_TIMEOUT);
-        fence_proxy_async_global();  // the pages were written through the generic proxy
       }
+      if (lane == 0) fence_proxy_async_global();  // the pages were written through the generic proxy
       early = __shfl_sync(0xffffffffu, ok, 0) != 0;
-      // every lane reads the state: each acquires the (already published) flag itself
-      if (early) (void)ld_acquire_gpu_u32(p.head_flags + h);
+      // Lane 0's acquire, then a warp barrier (which orders memory among its threads): every
+      // lane's state reads below come after the flag.
+      __syncwarp();
     }
     if (!early) {
       pdl_wait_prerequisites();
       waited = true;
     }
     // The head's count, (fused) the ring entry of the token leaving the window, and the
-    // page-table entry of this CTA's first pages (one per lane), all in flight at once.
+    // page-table entries of this CTA's first 64 pages (two per lane), all in flight at once.
     // Fused: delayed eviction for position j (Sec. 3.1-3.2): the token j - window - 1
     // leaves the window; if it was flagged, the new token takes its slot, otherwise the
     // fresh slot n_h.
@@ -1383,6 +1383,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
       e = __ldcg(p.ring + (int64_t)h * p.ring_len + (p.j - p.window - 1) % ring_period(p.window));
     const int spec_pg = rank + C * lane;
     if (spec_pg < p.max_pages) spec_page = __ldcg(pt + spec_pg);
+    if (spec_pg + 32 * C < p.max_pages) spec_page2 = __ldcg(pt + spec_pg + 32 * C);
     if (lane == 0) {
       int32_t cnt = n;
       uint32_t slot_info = 0u;
@@ -1414,6 +1415,9 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
     // opened here if the new token starts it.
     int patch_page = -1;
     if (patch_cta) {
+      // An existing page among this CTA's first 64 has its id in a lane already.
+      const int li = (pg_new - rank) / C;  // pg_new's place among this CTA's pages
+      const int known = __shfl_sync(0xffffffffu, li < 32 ? spec_page : spec_page2, li & 31);
       if (lane == 0) {
         if (opens) {
           patch_page = atomicAdd(p.ctrl + kCtrlPoolNext, 1);
@@ -1423,7 +1427,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           }
           p.page_table[(int64_t)h * p.max_pages + pg_new] = patch_page;
         } else {
-          patch_page = __ldcg(pt + pg_new);
+          patch_page = li < 64 ? known : __ldcg(pt + pg_new);
         }
       }
       patch_page = __shfl_sync(0xffffffffu, patch_page, 0);
@@ -1479,7 +1483,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
                 }
               }
               if (lane == 0)
-                p.scales[(int64_t)patch_page * 2 * kPageTokens + kv * kPageTokens + r] = scale;
+                page_scales_fp8(p.pool, patch_page)[kv * kPageTokens + r] = scale;
             }
           }
           if (patch_page >= 0 && lane == 0)
@@ -1520,7 +1524,7 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
         if (kFused && pg == pg_new) {
           page = patch_page;
         } else {
-          page = it0 == 0 ? spec_page : __ldcg(pt + pg);
+          page = it0 == 0 ? spec_page : it0 == 32 ? spec_page2 : __ldcg(pt + pg);
         }
       }
       const int nb = min(32, niters - it0);
@@ -1536,22 +1540,24 @@ __global__ void __launch_bounds__(kClusterThreads, 1) decode_cluster_kernel(cons
           uint8_t* st = stages + s * kStageBytes;
           const int64_t page0 = page_i < 0 ? 0 : page_i;
           if constexpr (kFp8) {
-            // the valid K rows; all of V^T (its rows interleave the slots) and the scales
-            const uint32_t k_bytes = (uint32_t)nv_i * 128u;
-            mbar_arrive_expect_tx(&full_bar[s], k_bytes + (uint32_t)kHalfPageBytesFp8 +
-                                                    (uint32_t)kScaleBytes +
+            // the whole page (K codes, V^T codes, row scales) in one copy, as each bulk copy
+            // has a fixed issue cost: K rows past n_valid are masked like stale ones, and all
+            // of V^T is needed (its rows interleave the slots)
+            static_assert(kKvHalf == kHalfPageBytesFp8 && kOffScales == kPageCodesBytesFp8,
+                          "a stage holds the page as laid out in the pool");
+            mbar_arrive_expect_tx(&full_bar[s], (uint32_t)kPageBytesFp8 +
                                                     (patch ? (uint32_t)kPatchBytes : 0u));
-            const uint8_t* src = p.pool + page0 * kPageBytesFp8;
-            bulk_copy_g2s(st, src, k_bytes, &full_bar[s]);
-            bulk_copy_g2s(st + kKvHalf, src + kHalfPageBytesFp8, kHalfPageBytesFp8, &full_bar[s]);
-            bulk_copy_g2s(st + kOffScales, p.scales + page0 * 2 * kPageTokens, kScaleBytes,
-                          &full_bar[s]);
+            bulk_copy_g2s(st, p.pool + page0 * kPageBytesFp8, kPageBytesFp8, &full_bar[s]);
           } else {
             const uint32_t kv_bytes = (uint32_t)nv_i * (uint32_t)kRowBytes;
             mbar_arrive_expect_tx(&full_bar[s], 2 * kv_bytes + (patch ? (uint32_t)kPatchBytes : 0u));
             const uint8_t* src = p.pool + page0 * kPageBytes;
-            bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
-            bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+            if (nv_i == kPageTokens) {  // a full page: K and V halves in one copy
+              bulk_copy_g2s(st, src, 2 * kHalfPageBytes, &full_bar[s]);
+            } else {  // the valid rows of each half
+              bulk_copy_g2s(st, src, kv_bytes, &full_bar[s]);
+              bulk_copy_g2s(st + kHalfPageBytes, src + kHalfPageBytes, kv_bytes, &full_bar[s]);
+            }
           }
           if (patch) {  // the new token's K and V rows, as given (unpermuted)
             if (waited) {
@@ -2157,7 +2163,6 @@ DecodeParams cache_params(const Cache& c, int32_t layer, const void* q, void* ou
   DecodeParams p = {};
   p.state_ready = (c.last_full_tiled && c.last_layer != layer) ? 1 : 0;
   p.pool = c.pool;
-  p.scales = c.scales;
   p.page_table = c.page_table + (int64_t)layer * c.heads * c.max_pages;
   p.counts = c.counts_at(layer, c.lengths[layer]);
   p.q = static_cast<const __nv_bfloat16*>(q);

@@ -56,9 +56,10 @@ constexpr int kPageTokens = 64;
 constexpr int kRowBytes = kHeadDim * 2;                       // 256
 constexpr int kHalfPageBytes = kPageTokens * kRowBytes;       // 16384
 constexpr int kPageBytes = 2 * kHalfPageBytes;                // 32768
-constexpr int kPageBytesFp8 = 16384;                          // fp8 page: K 8 KiB, V^T 8 KiB
-constexpr int kHalfPageBytesFp8 = 8192;
-constexpr int kScaleBytes = 2 * kPageTokens * 4;              // per page: key, value scales
+constexpr int kHalfPageBytesFp8 = 8192;                       // fp8 page: K codes 8 KiB, V^T 8 KiB,
+constexpr int kScaleBytes = 2 * kPageTokens * 4;              // then the key and value row scales
+constexpr int kPageCodesBytesFp8 = 2 * kHalfPageBytesFp8;     // 16384
+constexpr int kPageBytesFp8 = kPageCodesBytesFp8 + kScaleBytes;  // 16896: one bulk copy per page
 constexpr int kMaxGroup = 16;                                 // query heads per KV head
 constexpr int kMaxHeads = 4096;                               // batch * kv_heads
 constexpr int kMaxCtasPerSm = 4;
@@ -71,6 +72,11 @@ constexpr int kCtrlPoolNext = 0;
 constexpr int kCtrlError = 1;
 // A bounded wait gives up after this many nanoseconds of %globaltimer.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+// The row scales of fp8 page `page` of the pool: [0, 64) the keys', [64, 128) the values'.
+__host__ __device__ inline float* page_scales_fp8(uint8_t* pool, int64_t page) {
+  return reinterpret_cast<float*>(pool + page * kPageBytesFp8 + kPageCodesBytesFp8);
+}
 
 struct Cache {
   int32_t layers = 0, kv_heads = 0, head_dim = 0, window = 0, batch = 0;
@@ -91,7 +97,6 @@ struct Cache {
   int64_t piece_capacity = 0;
 
   uint8_t* pool = nullptr;
-  float* scales = nullptr;  // fp8 format only
   int32_t* pos = nullptr;
   int32_t* page_table = nullptr;
   int32_t* counts = nullptr;
