@@ -341,13 +341,16 @@ def test_reset_and_reuse():
 @pytest.mark.parametrize("kernel", [dms.DMS_DECODE_CLUSTER, dms.DMS_DECODE_SPLIT],
                          ids=["cluster", "split"])
 @pytest.mark.parametrize("fused", [True, False])
-def test_multilayer_interleaved_steps(fused, kernel):
+@pytest.mark.parametrize("B,Hkv,P", [(2, 2, 500), (1, 3, 560)], ids=["aligned", "odd-table"])
+def test_multilayer_interleaved_steps(fused, kernel, B, Hkv, P):
     """Three layers advanced together, as a model decodes: each step visits layer 0, 1, 2.
     Consecutive launches serve different layers, so the fused kernel reads the layer's state
-    and stages its first pages before waiting for the previous launch."""
+    and stages its first pages before waiting for the previous launch.  In the second shape a
+    layer's page table holds 3 heads x 9 pages = 27 entries, so the tables of layers 1 and 2
+    start off a 16-byte boundary (the L2 prefetch of the table must stay aligned)."""
     import oracle
     from _harness import MAX_ABS, MEAN_ABS
-    L, B, Hkv, G, w, P, steps = 3, 2, 2, 4, 24, 500, 12
+    L, G, w, steps = 3, 4, 24, 12
     wl = small(batch=B, kv_heads=Hkv, q_heads=Hkv * G, window=w)
     dev = torch.device("cuda")
     cache = dms.DmsCache(layers=L, kv_heads=Hkv, window=w, capacity=P + steps, batch=B,
