@@ -7,9 +7,11 @@
 //               copy of whole rows therefore lands in shared memory already in a
 //               bank-conflict-free order for ldmatrix (8 consecutive rows hit 8 distinct
 //               16-byte bank groups).
-//   (fp8 E4M3 format, DMS_KV_FP8_E4M3: pages of 16 KiB)
-//   pool        [pool_pages][16384] bytes: 64 K rows of 128 codes, then V transposed,
-//               128 rows (one per head_dim index d) of 64 codes (one per slot).  Both
+//   (fp8 E4M3 format, DMS_KV_FP8_E4M3: pages of 16.5 KiB)
+//   pool        [pool_pages][16896] bytes: 64 K rows of 128 codes, then V transposed,
+//               128 rows (one per head_dim index d) of 64 codes (one per slot), then
+//               the 64 key and 64 value row scales (fp32, page_scales_fp8), so that one
+//               bulk copy fetches a page.  Both code halves
 //               are laid out for the tiled decode kernel's m16n8k16 A fragments: in a
 //               K row, the 16-code block of k-step kk sits in the 16-byte chunk group
 //               kk / 4 and the four codes one thread needs (d = 16 kk + {2c, 2c+1,
@@ -17,7 +19,6 @@
 //               tokens {2c, 2c+1, 2c+8, 2c+9} of a 16-slot block likewise.  16-byte
 //               chunks are XOR-permuted by the row (K: k8_swizzle(row); V^T: (d >> 1) & 3) so
 //               a warp's loads hit distinct banks.  k8_offset / vt8_offset below.
-//   scales      [pool_pages][2][64] fp32         per-slot key and value scales.
 //   pos         [pool_pages][64] int32          position held by each slot (inspection only;
 //                                               decode never reads it).
 //   page_table  [layers][heads][max_pages] int32 page of slot s is page_table[.][s / 64].
